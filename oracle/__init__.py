@@ -1,0 +1,182 @@
+"""CPU oracle for the ASP linear layer (Q-WAM, Sec. 3.2 Eq. (asp); Sec. 2 Eq. (quant); App. B.1).
+
+TEST INFRASTRUCTURE ONLY.  The tests, the smoke check and the CPU-baseline leg of the benchmark
+load this module; the library under ``paper_2609_33269_gb300`` never imports it and shares no
+code with it.  The arithmetic lives in ``qwam_oracle.c`` (float64 / int64, OpenMP over rows);
+this file only compiles it with gcc and marshals numpy arrays through ctypes.
+
+Every function returns semantic arrays in the paper's row-major notation:
+X [M,K] tokens, W [K,N], U [K,r] (the paper's V), codes as int8 in [-7, 7], activation scales
+float32 [M, K/G], weight scales float16 [K/G, N], branch factors float16.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "qwam_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libqwam_oracle.so")
+_lib = None
+_lock = threading.Lock()
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (-O2 -fopenmp -ffp-contract=off); returns the .so path."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-ffp-contract=off", "-fno-fast-math",
+           "-fPIC", "-shared", _SRC, "-o", tmp, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            I = ctypes.c_int
+            lib.qo_pack.argtypes = [P, P, I, I, I, I, P, P, P, P, P]
+            lib.qo_quantize_act.argtypes = [P, P, I, I, I, I, P, P, P, P, P]
+            lib.qo_quantize_residual_f32.argtypes = [P, I, I, I, P, P]
+            lib.qo_linear.argtypes = [P, P, P, P, P, P, I, I, I, I, I, P]
+            lib.qo_linear_split_exact.argtypes = [P, P, P, P, I, I, I, I, P]
+            lib.qo_f16_bits_rn.argtypes = [ctypes.c_double]
+            lib.qo_f16_bits_rn.restype = ctypes.c_uint16
+            lib.qo_f16_value.argtypes = [ctypes.c_uint16]
+            lib.qo_f16_value.restype = ctypes.c_double
+            lib.qo_nearest_code.argtypes = [ctypes.c_double, ctypes.c_double]
+            lib.qo_nearest_code.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def _check(rc, what):
+    if rc != 0:
+        raise OracleError(f"{what}: oracle status {rc} ({'range' if rc == -2 else 'invalid argument'})")
+
+
+def pack(W_bf16_bits, U, G, want_float64=False):
+    """Offline packing (Sec. 3.2 Eq. (asp) and the W_perp derivation; Eq. (quant) on weights).
+
+    W_bf16_bits: uint16 [K,N]; U: float32 [K,r] (r may be 0).
+    Returns dict(qw int8 [N,K], sw uint16 fp16-bits [K/G,N], Bh uint16 fp16-bits [r,N],
+    and Bf / Wperp float64 when want_float64)."""
+    W = _c(W_bf16_bits, np.uint16)
+    K, N = W.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qw = np.empty((N, K), np.int8)
+    sw = np.empty((K // G, N), np.uint16)
+    Bh = np.empty((r, N), np.uint16)
+    Bf = np.empty((r, N), np.float64) if want_float64 else None
+    Wp = np.empty((K, N), np.float64) if want_float64 else None
+    _check(_load().qo_pack(_ptr(W), _ptr(U), K, N, r, G, _ptr(qw), _ptr(sw), _ptr(Bh), _ptr(Bf), _ptr(Wp)),
+           "pack")
+    out = dict(qw=qw, sw=sw, Bh=Bh)
+    if want_float64:
+        out.update(Bf=Bf, Wperp=Wp)
+    return out
+
+
+def quantize_act(X_bf16_bits, U, G, want_float64=False):
+    """Run-time activation path (Eq. (xsplit), then Eq. (quant) per token and group).
+
+    Returns dict(qx int8 [M,K], sx float32 [M,K/G], ph uint16 fp16-bits [M,r],
+    and p / Xperp float64 when want_float64)."""
+    X = _c(X_bf16_bits, np.uint16)
+    M, K = X.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qx = np.empty((M, K), np.int8)
+    sx = np.empty((M, K // G), np.float32)
+    ph = np.empty((M, r), np.uint16)
+    p = np.empty((M, r), np.float64) if want_float64 else None
+    Xp = np.empty((M, K), np.float64) if want_float64 else None
+    _check(_load().qo_quantize_act(_ptr(X), _ptr(U), M, K, r, G, _ptr(qx), _ptr(sx), _ptr(ph), _ptr(p), _ptr(Xp)),
+           "quantize_act")
+    out = dict(qx=qx, sx=sx, ph=ph)
+    if want_float64:
+        out.update(p=p, Xperp=Xp)
+    return out
+
+
+def quantize_residual(R_f32, G):
+    """The quantizer alone on a float32 remainder R [M,K] -> (codes int8 [M,K], scales f32 [M,K/G])."""
+    R = _c(R_f32, np.float32)
+    M, K = R.shape
+    q = np.empty((M, K), np.int8)
+    s = np.empty((M, K // G), np.float32)
+    _check(_load().qo_quantize_residual_f32(_ptr(R), M, K, G, _ptr(q), _ptr(s)), "quantize_residual")
+    return q, s
+
+
+def linear(act, wts, G):
+    """Layer output of Eq. (asp) from codes and scales -> float64 Y [M,N]."""
+    qx = _c(act["qx"], np.int8)
+    M, K = qx.shape
+    qw = _c(wts["qw"], np.int8)
+    N = qw.shape[0]
+    r = wts["Bh"].shape[0]
+    Y = np.empty((M, N), np.float64)
+    _check(_load().qo_linear(_ptr(qx), _ptr(_c(act["sx"], np.float32)), _ptr(_c(act["ph"], np.uint16)),
+                             _ptr(qw), _ptr(_c(wts["sw"], np.uint16)), _ptr(_c(wts["Bh"], np.uint16)),
+                             M, K, N, r, G, _ptr(Y)), "linear")
+    return Y
+
+
+def linear_split_exact(p, Xperp, Bf, Wperp):
+    """Eq. (asp) with Q replaced by the identity: p B_f + X_perp W_perp (float64)."""
+    p = _c(p, np.float64)
+    Xp = _c(Xperp, np.float64)
+    Bf = _c(Bf, np.float64)
+    Wp = _c(Wperp, np.float64)
+    M, K = Xp.shape
+    N = Wp.shape[1]
+    r = p.shape[1]
+    Y = np.empty((M, N), np.float64)
+    _check(_load().qo_linear_split_exact(_ptr(p), _ptr(Xp), _ptr(Bf), _ptr(Wp), M, K, N, r, _ptr(Y)),
+           "linear_split_exact")
+    return Y
+
+
+def forward(X_bf16_bits, W_bf16_bits, U, G):
+    """Whole layer: pack, quantize the activations, output.  Returns (Y, act, wts)."""
+    wts = pack(W_bf16_bits, U, G)
+    act = quantize_act(X_bf16_bits, U, G)
+    return linear(act, wts, G), act, wts
+
+
+def f16_bits(x: float) -> int:
+    return int(_load().qo_f16_bits_rn(float(x)))
+
+
+def f16_value(h: int) -> float:
+    return float(_load().qo_f16_value(int(h)))
+
+
+def nearest_code(x: float, s: float) -> int:
+    return int(_load().qo_nearest_code(float(x), float(s)))

@@ -1,0 +1,327 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix (no GPU).
+
+Each pin is independent of the oracle's own code:
+  * exact rational arithmetic (fractions.Fraction) of the whole layer on tiny shapes,
+  * brute-force argmin over the code grid for the quantizer (Eq. (quant)),
+  * hand-derived closed-form group cases (tests/golden/quant_cases.txt),
+  * library conversions (numpy float16) for the 16-bit format,
+  * invariants of Sec. 3.2: x = U(U^T x) + x_perp, U^T W_perp = 0, x_perp U = 0, Eq. (asp) with
+    Q = identity equals X W, r = 0 is plain per-group W4A4, r = K leaves a zero remainder,
+  * storage of Table 3 (4.50 bits per weight at group 32) and the isotropy share r/K of App. C.
+"""
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2609_33269_gb300 import workloads as wl
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "quant_cases.txt")
+
+
+# ---------------------------------------------------------------- exact helpers (tests only)
+
+def f32_bits(x: float) -> int:
+    return int(np.array([x], np.float32).view(np.uint32)[0])
+
+
+def f32_from_bits(b: int) -> float:
+    return float(np.array([b], np.uint32).view(np.float32)[0])
+
+
+def rn_binary(fr: Fraction, mant: int, emin: int) -> Fraction:
+    """Round |fr| to the nearest number with `mant` significant bits (ties to even), gradual
+    underflow below 2**emin; sign restored.  Exact, for pins only."""
+    if fr == 0:
+        return Fraction(0)
+    sgn = -1 if fr < 0 else 1
+    a = abs(fr)
+    e = a.numerator.bit_length() - a.denominator.bit_length()
+    if Fraction(2) ** e > a:
+        e -= 1
+    if Fraction(2) ** (e + 1) <= a:
+        e += 1
+    e = max(e, emin)
+    quantum = Fraction(2) ** (e - (mant - 1))
+    q = a / quantum
+    n = q.numerator // q.denominator
+    rem = q - n
+    if rem > Fraction(1, 2) or (rem == Fraction(1, 2) and n % 2 == 1):
+        n += 1
+    return sgn * n * quantum
+
+
+def rn_f32(fr):
+    return rn_binary(fr, 24, -126)
+
+
+def rn_f16(fr):
+    return rn_binary(fr, 11, -14)
+
+
+def brute_code(x: Fraction, s: Fraction) -> int:
+    """argmin over the 16 codes -8..7 of |x - c s|, ties to the even code; s == 0 -> 0."""
+    if s == 0:
+        return 0
+    best = None
+    for c in range(-8, 8):
+        d = abs(x - c * s)
+        if best is None or d < best[0] or (d == best[0] and c % 2 == 0):
+            best = (d, c)
+    return best[1]
+
+
+def bf16_frac(bits):
+    return Fraction(float(wl.bf16_bits_to_f32(np.array([bits], np.uint16))[0]))
+
+
+def f16_frac(bits):
+    return Fraction(float(np.array([bits], np.uint16).view(np.float16)[0]))
+
+
+# ---------------------------------------------------------------- number formats
+
+def test_f16_rounding_matches_numpy():
+    g = np.random.default_rng(7)
+    xs = np.concatenate([
+        g.standard_normal(20000) * 10.0 ** g.integers(-9, 5, 20000),
+        np.array([0.0, -0.0, 65504.0, 65519.99, 65520.0, -65520.0, 6.1e-5, 5.96e-8, 2.98e-8,
+                  2.9802322387695312e-08, 1.0 + 2.0 ** -11, 1.0 + 3 * 2.0 ** -11, 2.0 ** -25]),
+    ])
+    # exact ties of the 11-bit grid
+    xs = np.concatenate([xs, (1024 + np.arange(0, 1024) + 0.5) * 2.0 ** -10])
+    with np.errstate(over="ignore"):
+        want = xs.astype(np.float16).view(np.uint16)
+    got = np.array([oracle.f16_bits(x) for x in xs], np.uint16)
+    np.testing.assert_array_equal(got, want)
+    for h in (0, 1, 0x3c00, 0x3092, 0x7bff, 0x8001, 0x0400):
+        assert oracle.f16_value(h) == float(np.array([h], np.uint16).view(np.float16)[0])
+
+
+# ---------------------------------------------------------------- quantizer (Eq. (quant))
+
+def _golden_cases():
+    cases = []
+    for line in open(GOLDEN):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        kind, vals, sbits, codes = [t.strip() for t in line.split("|")]
+        cases.append((kind, [float(v) for v in vals.split(",")], int(sbits, 16),
+                      [int(c) for c in codes.split(",")]))
+    return cases
+
+
+@pytest.mark.parametrize("case", _golden_cases())
+def test_golden_group_cases(case):
+    kind, vals, sbits, codes = case
+    G = len(vals)
+    if kind == "act":
+        q, s = oracle.quantize_residual(np.array([vals], np.float32), G)
+        assert f32_bits(float(s[0, 0])) == sbits
+        assert q[0].tolist() == codes
+    else:
+        # weight path: one output channel, K = G, r = 0, W holds the values exactly in bf16
+        W = wl.f32_to_bf16_bits(np.array(vals, np.float32).reshape(G, 1))
+        assert np.array_equal(wl.bf16_bits_to_f32(W)[:, 0], np.array(vals, np.float32))
+        out = oracle.pack(W, np.zeros((G, 0), np.float32), G)
+        assert int(out["sw"][0, 0]) == sbits
+        assert out["qw"][0].tolist() == codes
+
+
+def test_nearest_code_bruteforce_with_ties():
+    g = np.random.default_rng(3)
+    checked = 0
+    for _ in range(3000):
+        # scales with few significant bits make exact ties x = (c + 1/2) s representable
+        s = float(np.float32(g.integers(1, 2 ** 10) * 2.0 ** int(g.integers(-20, 5))))
+        if g.random() < 0.5:
+            c = int(g.integers(-7, 7))
+            x = float(np.float32((c + 0.5) * s))
+        else:
+            x = float(np.float32(g.uniform(-7.4, 7.4) * s))
+        got = oracle.nearest_code(x, s)
+        assert got == brute_code(Fraction(x), Fraction(s)), (x, s)
+        checked += 1
+    assert checked == 3000
+
+
+def test_quantize_residual_bruteforce_and_error_bound():
+    g = np.random.default_rng(11)
+    for G in (32, 64):
+        R = (g.standard_normal((3, 128)) * np.exp(g.uniform(-3, 3, (3, 1)))).astype(np.float32)
+        R[1, :G] = 0.0  # an all-zero group
+        q, s = oracle.quantize_residual(R, G)
+        for m in range(R.shape[0]):
+            for gi in range(128 // G):
+                grp = [Fraction(float(v)) for v in R[m, gi * G:(gi + 1) * G]]
+                amax = max(abs(v) for v in grp)
+                s_exact = rn_f32(amax / 7)
+                assert Fraction(float(s[m, gi])) == s_exact
+                for k, v in enumerate(grp):
+                    c = brute_code(v, s_exact)
+                    assert int(q[m, gi * G + k]) == c
+                    assert -7 <= c <= 7  # -8 is never produced by absmax / 7
+                    assert abs(c * s_exact - v) <= s_exact / 2  # dequantization error <= s/2
+
+
+# ---------------------------------------------------------------- whole layer, exact arithmetic
+
+def _exact_layer(Xb, Wb, U, G):
+    """Eq. (xsplit) + Eq. (asp) + Eq. (quant) in exact rationals, with the stated readings."""
+    M, K = Xb.shape
+    N = Wb.shape[1]
+    r = U.shape[1]
+    X = [[bf16_frac(Xb[m, k]) for k in range(K)] for m in range(M)]
+    W = [[bf16_frac(Wb[k, n]) for n in range(N)] for k in range(K)]
+    Uf = [[Fraction(float(U[k, j])) for j in range(r)] for k in range(K)]
+    # pack
+    Bf = [[sum(Uf[k][j] * W[k][n] for k in range(K)) for n in range(N)] for j in range(r)]
+    Wp = [[W[k][n] - sum(Uf[k][j] * Bf[j][n] for j in range(r)) for n in range(N)] for k in range(K)]
+    ng = K // G
+    sw = [[rn_f16(max(abs(Wp[k][n]) for k in range(g * G, (g + 1) * G)) / 7) for n in range(N)]
+          for g in range(ng)]
+    qw = [[brute_code(Wp[k][n], sw[k // G][n]) for k in range(K)] for n in range(N)]
+    Bh = [[rn_f16(Bf[j][n]) for n in range(N)] for j in range(r)]
+    # activations
+    p = [[sum(X[m][k] * Uf[k][j] for k in range(K)) for j in range(r)] for m in range(M)]
+    Xp = [[X[m][k] - sum(p[m][j] * Uf[k][j] for j in range(r)) for k in range(K)] for m in range(M)]
+    sx = [[rn_f32(max(abs(Xp[m][k]) for k in range(g * G, (g + 1) * G)) / 7) for g in range(ng)]
+          for m in range(M)]
+    qx = [[brute_code(Xp[m][k], sx[m][k // G]) for k in range(K)] for m in range(M)]
+    ph = [[rn_f16(p[m][j]) for j in range(r)] for m in range(M)]
+    Y = [[sum(sx[m][g] * sw[g][n] * sum(qx[m][k] * qw[n][k] for k in range(g * G, (g + 1) * G))
+              for g in range(ng)) + sum(ph[m][j] * Bh[j][n] for j in range(r))
+          for n in range(N)] for m in range(M)]
+    return dict(qw=qw, sw=sw, Bh=Bh, qx=qx, sx=sx, ph=ph, Y=Y)
+
+
+@pytest.mark.parametrize("r", [0, 1, 2])
+@pytest.mark.parametrize("G", [32, 64])
+def test_layer_matches_exact_rational_arithmetic(r, G):
+    M, K, N = 4, 128, 8
+    Xb = wl.activations(M, K, seed=5, layer_id=r, dist="outlier", n_outlier=3)
+    Wb = wl.weight(K, N, seed=5, layer_id=r)
+    U = wl.basis(K, r, seed=5, layer_id=r)
+    ex = _exact_layer(Xb, Wb, U, G)
+    w = oracle.pack(Wb, U, G)
+    a = oracle.quantize_act(Xb, U, G)
+    Y = oracle.linear(a, w, G)
+    assert w["qw"].tolist() == ex["qw"]
+    assert [[f16_frac(b) for b in row] for row in w["sw"]] == ex["sw"]
+    assert [[f16_frac(b) for b in row] for row in w["Bh"]] == ex["Bh"]
+    assert a["qx"].tolist() == ex["qx"]
+    assert [[Fraction(float(v)) for v in row] for row in a["sx"]] == ex["sx"]
+    assert [[f16_frac(b) for b in row] for row in a["ph"]] == ex["ph"]
+    Yex = np.array([[float(v) for v in row] for row in ex["Y"]])
+    np.testing.assert_allclose(Y, Yex, rtol=1e-12, atol=1e-12 * np.abs(Yex).max())
+
+
+# ---------------------------------------------------------------- invariants of Sec. 3.2
+
+def _small_case(M=16, K=256, N=96, r=8, G=64, seed=1):
+    Xb = wl.activations(M, K, seed=seed, layer_id=7, dist="outlier", n_outlier=4)
+    Wb = wl.weight(K, N, seed=seed, layer_id=7)
+    U = wl.basis(K, r, seed=seed, layer_id=7)
+    return Xb, Wb, U
+
+
+def test_split_identity_and_projection_invariants():
+    Xb, Wb, U = _small_case()
+    G = 64
+    X = wl.bf16_bits_to_f32(Xb).astype(np.float64)
+    W = wl.bf16_bits_to_f32(Wb).astype(np.float64)
+    Ud = U.astype(np.float64)
+    w = oracle.pack(Wb, U, G, want_float64=True)
+    a = oracle.quantize_act(Xb, U, G, want_float64=True)
+    scale = np.abs(X).max()
+    # x = U (U^T x) + x_perp  (Eq. (xsplit))
+    np.testing.assert_allclose(a["p"] @ Ud.T + a["Xperp"], X, rtol=0, atol=1e-12 * scale)
+    # p = x U, B_f = U^T W (library matmul as an independent check)
+    np.testing.assert_allclose(a["p"], X @ Ud, rtol=0, atol=1e-12 * scale)
+    np.testing.assert_allclose(w["Bf"], Ud.T @ W, rtol=0, atol=1e-12 * np.abs(W).max())
+    # (I - Pi) removes span(U): x_perp U = p (I - U^T U) and U^T W_perp = (I - U^T U) B_f hold
+    # exactly for any U; with float32 U, I - U^T U is ~1e-7, so both are ~1e-7 and not 0.
+    D = np.eye(U.shape[1]) - Ud.T @ Ud
+    np.testing.assert_allclose(a["Xperp"] @ Ud, a["p"] @ D, rtol=0, atol=1e-12 * scale)
+    np.testing.assert_allclose(Ud.T @ w["Wperp"], D @ w["Bf"], rtol=0, atol=1e-12 * np.abs(W).max())
+    assert np.abs(a["Xperp"] @ Ud).max() <= 1e-5 * scale
+    # Eq. (asp) with Q = identity: (U^T W)^T (U^T x) + W_perp^T x_perp = W^T x for orthonormal U;
+    # for any U the two sides differ by exactly p (I - U^T U) B_f (expand the product).
+    Y = oracle.linear_split_exact(a["p"], a["Xperp"], w["Bf"], w["Wperp"])
+    ref = X @ W
+    np.testing.assert_allclose(Y, ref - a["p"] @ D @ w["Bf"], rtol=0, atol=1e-12 * np.abs(ref).max())
+    np.testing.assert_allclose(Y, ref, rtol=0, atol=1e-5 * np.abs(ref).max())
+
+
+def test_r0_is_plain_per_group_w4a4():
+    M, K, N, G = 64, 512, 128, 64
+    Xb = wl.activations(M, K, seed=2, layer_id=3)
+    Wb = wl.weight(K, N, seed=2, layer_id=3)
+    U0 = np.zeros((K, 0), np.float32)
+    Y, a, w = oracle.forward(Xb, Wb, U0, G)
+    # independent numpy statement of per-group W4A4 (Eq. (quant) on both operands)
+    X = wl.bf16_bits_to_f32(Xb).reshape(M, K // G, G)
+    amax = np.abs(X).max(axis=2)
+    sx = (amax.astype(np.float64) / 7.0).astype(np.float32)   # exact rounding: 53 >= 2*24+2
+    with np.errstate(invalid="ignore", divide="ignore"):
+        qx = np.where(sx[..., None] > 0, np.rint(X / sx[..., None].astype(np.float64)), 0).astype(np.int64)
+    np.testing.assert_array_equal(a["sx"], sx)
+    np.testing.assert_array_equal(a["qx"], qx.reshape(M, K))
+    Wt = wl.bf16_bits_to_f32(Wb).astype(np.float64).T.reshape(N, K // G, G)
+    swv = np.abs(Wt).max(axis=2) / 7.0
+    sw_bits = swv.astype(np.float16).view(np.uint16)
+    np.testing.assert_array_equal(w["sw"], sw_bits.T)
+    swf = sw_bits.view(np.float16).astype(np.float64)
+    with np.errstate(invalid="ignore", divide="ignore"):
+        qw = np.where(swf[..., None] > 0, np.rint(Wt / swf[..., None]), 0).astype(np.int64)
+    np.testing.assert_array_equal(w["qw"], qw.reshape(N, K))
+    P = np.einsum("mgk,ngk->mng", qx, qw)  # exact int64 group partial sums
+    ref = np.einsum("mng,mg,ng->mn", P.astype(np.float64), sx.astype(np.float64), swf)
+    np.testing.assert_allclose(Y, ref, rtol=1e-13, atol=1e-13 * np.abs(ref).max())
+    assert a["ph"].shape == (M, 0) and w["Bh"].shape == (0, N)
+
+
+def test_r_equals_K_zero_remainder_and_bf16_gemm():
+    M, K, N, G = 32, 128, 64, 64
+    Xb = wl.activations(M, K, seed=4, layer_id=9)
+    Wb = wl.weight(K, N, seed=4, layer_id=9)
+    U = wl.basis(K, K, seed=4, layer_id=9)
+    w = oracle.pack(Wb, U, G, want_float64=True)
+    a = oracle.quantize_act(Xb, U, G, want_float64=True)
+    X = wl.bf16_bits_to_f32(Xb).astype(np.float64)
+    W = wl.bf16_bits_to_f32(Wb).astype(np.float64)
+    assert np.abs(a["Xperp"]).max() <= 1e-5 * np.abs(X).max()  # only float32 U roundoff remains
+    assert np.abs(w["Wperp"]).max() <= 1e-5 * np.abs(W).max()
+    Y = oracle.linear(a, w, G)
+    ref = X @ W
+    err = np.abs(Y - ref).max(axis=1) / np.abs(ref).max(axis=1)
+    assert err.max() <= 1e-3, err.max()
+
+
+def test_codes_range_and_storage_table3():
+    Xb, Wb, U = _small_case(K=512, N=128, r=0)
+    for G in (32, 64):
+        w = oracle.pack(Wb, U, G)
+        assert w["qw"].min() >= -7 and w["qw"].max() <= 7
+        K, N = Wb.shape
+        bits = 4 * w["qw"].size + 16 * w["sw"].size  # 4-bit codes + 16-bit scales
+        bpw = bits / (K * N)
+        assert bpw == 4 + 16 / G
+    assert 4 + 16 / 32 == 4.50  # Table 3: per-group W4A4 at group 32
+
+
+def test_isotropy_share_of_the_4bit_residual():
+    """App. C: the rounding error of the 4-bit remainder puts about r/K of its squared norm in
+    span(U).  Loose statistical check on synthetic data (factor of 2)."""
+    M, K, r, G = 256, 1024, 32, 64
+    Xb = wl.activations(M, K, seed=6, layer_id=11)
+    U = wl.basis(K, r, seed=6, layer_id=11)
+    a = oracle.quantize_act(Xb, U, G, want_float64=True)
+    deq = a["qx"].astype(np.float64) * np.repeat(a["sx"].astype(np.float64), G, axis=1)
+    delta = deq - a["Xperp"]
+    share = (np.linalg.norm(delta @ U.astype(np.float64)) ** 2) / (np.linalg.norm(delta) ** 2)
+    assert 0.5 * r / K <= share <= 2.0 * r / K, share
