@@ -1,0 +1,401 @@
+"""Benchmark of the ASP W4A4 + low-rank linear layer on GB300.
+
+One step = one pass of the whole hot path -- kernel (a) (projection, remainder, 4-bit activation
+quantization) and kernel (b) (4-bit GEMM with the 16-bit branch in its epilogue) -- over one
+batch of the DiT attention-projection workload: X bf16 [M=4096, K=3072], W [3072, 3072],
+r = 32, group 64, seeded synthetic data (1% outlier channels x10..30).
+
+Output: one JSON line.  `value` is the effective TOPS (2*M*N*K per step over the device time of
+the timed steps, max over ranks, summed over ranks' work); `e2e` repeats the measurement through
+the C ABI with the activations copied from pinned host memory and the output copied back inside
+the timed region; `roofline` describes the dominant kernel; `cpu_baseline` times the CPU oracle
+on a bounded sample of rows.  `--impl reference` times the CPU oracle alone (the reference arm).
+
+Multi-GPU (torchrun): every rank runs the same per-GPU batch (token rows are independent, so
+the layer shards by rows with no collective); weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "ASP W4A4+low-rank linear effective TOPS (2*M*N*K per step)"
+UNIT = "TOPS"
+WORKLOAD = dict(workload="dit_attn_proj_M4096_K3072_N3072_r32_g64", M=4096, K=3072, N=3072, r=32, group=64)
+ROTATE_SETS = 6  # distinct input/output/workspace/weight sets cycled through (> L2 in total)
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--warmup", type=int, default=50)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--cpu-rows", type=int, default=0, help="oracle sample rows (0 = sized to ~10 s)")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+# ------------------------------------------------------------------ distributed plumbing
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def init_dist(world, backend):
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend)
+    return dist
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ------------------------------------------------------------------ clocks during the timed region
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons (read-only)."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.samples = []
+        self.proc = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu=timestamp,{self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), line.strip()))
+
+    def mark(self, which):
+        setattr(self, which, time.time())
+
+    def stop(self):
+        if self.proc:
+            time.sleep(0.12)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=2)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        for ts, line in self.samples:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[4:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        inside = [r for r in rows if self.t0 and self.t1 and self.t0 - 0.05 <= r[0] <= self.t1 + 0.05]
+        use = inside or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in use for i, v in enumerate(r[3][1:]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(r[1] for r in use), "sm_max_mhz": max(r[2] for r in use),
+                "reasons": reasons, "samples": len(use), "samples_in_timed_region": len(inside)}
+
+
+# ------------------------------------------------------------------ CPU oracle (baseline / reference arm)
+
+def oracle_sample(rows: int):
+    """Inputs and packed weights for the oracle timing: the workload's first `rows` tokens."""
+    import oracle
+    from paper_2609_33269_gb300 import workloads as wl
+    layer = wl.dit_attention().layers[0]
+    Xb = layer.x()[:rows].copy()
+    U = layer.u()
+    wts = oracle.pack(layer.w(), U, layer.G)  # offline packing: outside the timed sample
+    return Xb, U, wts, layer
+
+
+def oracle_step(Xb, U, wts, G):
+    import oracle
+    act = oracle.quantize_act(Xb, U, G)
+    return oracle.linear(act, wts, G)
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    K, N = WORKLOAD["K"], WORKLOAD["N"]
+    rows = args.cpu_rows
+    if not rows:  # size each step so that warm-up + timed steps take about two minutes
+        Xb, U, wts, layer = oracle_sample(8)
+        t0 = time.perf_counter()
+        oracle_step(Xb, U, wts, layer.G)
+        per_row = (time.perf_counter() - t0) / 8
+        rows = int(max(1, min(256, 120.0 / (max(1, args.steps + args.warmup) * per_row))))
+    Xb, U, wts, layer = oracle_sample(rows)
+    for _ in range(max(0, args.warmup)):
+        oracle_step(Xb, U, wts, layer.G)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(Xb, U, wts, layer.G)
+    dt = time.perf_counter() - t0
+    value = 2.0 * rows * N * K * args.steps / dt / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": dict(WORKLOAD, sample_rows_per_step=rows, parallelism="host cores"),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                         "sample": f"{rows} of 4096 token rows per step (quantize + output); packing offline"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def cpu_baseline(rows_req: int):
+    K, N = WORKLOAD["K"], WORKLOAD["N"]
+    rows = rows_req or 64
+    Xb, U, wts, layer = oracle_sample(rows)
+    t0 = time.perf_counter()
+    oracle_step(Xb, U, wts, layer.G)
+    dt = time.perf_counter() - t0
+    if not rows_req and dt < 10.0:  # size the sample to roughly 10-20 s of CPU work
+        rows = min(4096, max(rows, int(rows * 12.0 / max(dt, 1e-3))))
+        Xb, U, wts, layer = oracle_sample(rows)
+        t0 = time.perf_counter()
+        oracle_step(Xb, U, wts, layer.G)
+        dt = time.perf_counter() - t0
+    return {"value": 2.0 * rows * N * K / dt / 1e12, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"{rows} of 4096 token rows (quantize + output, {dt:.1f} s); weight packing offline"}
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def alg_bytes_actquant(M, K, r_pad, G):
+    """Kernel (a): read X (2MK) and U (hi/lo, twice), write codes (MK/2), scales (4MK/G), p_hat."""
+    return 2 * M * K + M * K // 2 + 4 * M * K // G + 2 * M * r_pad + 2 * (2 * K * r_pad) * 2
+
+
+def run_ours(args):
+    import torch
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    init_dist(world, "nccl")
+    dev = torch.device("cuda", local)
+
+    from paper_2609_33269_gb300 import asp, build
+    from paper_2609_33269_gb300 import workloads as wl
+    build.build()
+    asp.load()
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        pass
+    hbm_peak = peaks.get("hbm_gbs", 6800.0)
+    bf16_peak = peaks.get("bf16_tflops", 1900.0)
+    fp8_peak = 2.0 * bf16_peak  # dense fp8 = 2x dense bf16 (nominal 4.5 / 2.25 PFLOP/s)
+
+    layer_def = wl.dit_attention().layers[0]
+    M, K, N, r, G = layer_def.M, layer_def.K, layer_def.N, layer_def.r, layer_def.G
+    Xb = layer_def.x()
+    Wb = layer_def.w()
+    U = layer_def.u()
+
+    def dev_bf16(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    W = dev_bf16(Wb)
+    Ud = torch.from_numpy(U).to(dev)
+    # rotating sets: distinct weights (packed per set), activations, workspaces and outputs
+    sets = []
+    X0 = dev_bf16(Xb)
+    for i in range(ROTATE_SETS):
+        lin = asp.AspLinear(W, Ud, G)
+        X = X0 if i == 0 else X0.clone()
+        ws = lin.workspace(M)
+        Y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+        sets.append((lin, X, ws, Y))
+    working_mb = ROTATE_SETS * (2 * M * K + 2 * M * N + lin_ws_bytes(sets[0][0], M) + N * K // 2) / 1e6
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        lin, X, ws, Y = sets[i % ROTATE_SETS]
+        asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
+        asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    for lin, *_ in sets:
+        st = asp.qwam_asp_get_error(lin.h)
+        if st != asp.QWAM_OK:
+            raise RuntimeError(f"device error after warm-up: {asp.status_string(st)}")
+
+    # timed region: per-kernel events on the launching stream
+    nsteps = args.steps
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * nsteps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.mark("t0")
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(nsteps):
+        lin, X, ws, Y = sets[i % ROTATE_SETS]
+        ev[3 * i].record(stream)
+        asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
+        ev[3 * i + 1].record(stream)
+        asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
+        ev[3 * i + 2].record(stream)
+    end.record(stream)
+    torch.cuda.synchronize()
+    clocks.mark("t1")
+    barrier(world)
+    clocks.stop()
+    total_ms = start.elapsed_time(end)
+    t_a = sum(ev[3 * i].elapsed_time(ev[3 * i + 1]) for i in range(nsteps)) / nsteps
+    t_b = sum(ev[3 * i + 1].elapsed_time(ev[3 * i + 2]) for i in range(nsteps)) / nsteps
+    for lin, *_ in sets:
+        st = asp.qwam_asp_get_error(lin.h)
+        if st != asp.QWAM_OK:
+            raise RuntimeError(f"device error in the timed region: {asp.status_string(st)}")
+    total_ms = max_over_ranks(total_ms, world, dev)
+    flops = 2.0 * M * N * K
+    value = flops * nsteps * world / (total_ms * 1e-3) / 1e12
+
+    # end to end through the public API: pinned host X -> device, layer, Y -> pinned host
+    Xh = torch.from_numpy(np.ascontiguousarray(Xb).view(np.int16)).view(torch.bfloat16).pin_memory()
+    Yh = torch.empty((M, N), dtype=torch.bfloat16).pin_memory()
+    lin, Xd, ws, Yd = sets[0]
+    e2e_steps = max(3, min(nsteps, 200))
+    for _ in range(3):
+        Xd.copy_(Xh, non_blocking=True)
+        lin(Xd, out=Yd)
+        Yh.copy_(Yd, non_blocking=True)
+    torch.cuda.synchronize()
+    barrier(world)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        Xd.copy_(Xh, non_blocking=True)
+        lin(Xd, out=Yd)
+        Yh.copy_(Yd, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_value = flops * e2e_steps * world / (e2e_ms * 1e-3) / 1e12
+
+    # roofline of the dominant kernel (per-launch averages from the events above)
+    r_pad = sets[0][0].r_pad
+    a_bytes = alg_bytes_actquant(M, K, r_pad, G)
+    kern = {
+        "actquant": {"ms": t_a, "bound": "hbm", "alg_bytes": a_bytes,
+                     "achieved_gbs": a_bytes / (t_a * 1e-3) / 1e9, "peak_gbs": hbm_peak},
+        "gemm_w4a4_lr": {"ms": t_b, "bound": "tensor", "alg_flops": flops,
+                         "achieved_tflops": flops / (t_b * 1e-3) / 1e12, "peak_tflops_fp8": fp8_peak},
+    }
+    kern["actquant"]["frac"] = kern["actquant"]["achieved_gbs"] / hbm_peak
+    kern["gemm_w4a4_lr"]["frac"] = kern["gemm_w4a4_lr"]["achieved_tflops"] / fp8_peak
+    if t_b >= t_a:
+        roof = {"kernel": "gemm_w4a4_lr", "bound": "tensor", "achieved": kern["gemm_w4a4_lr"]["achieved_tflops"],
+                "peak": fp8_peak, "unit": "TFLOP/s", "frac": kern["gemm_w4a4_lr"]["frac"],
+                "traffic": None,
+                "peak_source": "measured bf16 burst x 2 (nominal fp8/bf16 dense ratio), of measured"}
+    else:
+        roof = {"kernel": "actquant", "bound": "hbm", "achieved": kern["actquant"]["achieved_gbs"],
+                "peak": hbm_peak, "unit": "GB/s", "frac": kern["actquant"]["frac"], "traffic": None,
+                "peak_source": "measured HBM copy, of measured"}
+
+    if rank != 0:
+        return 0
+    t_layer_roof = max((a_bytes + N * K // 2 + 2 * N * K // G + 2 * N * r_pad + 2 * M * N) / (hbm_peak * 1e9),
+                       flops / (fp8_peak * 1e12))
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": nsteps, "warmup": args.warmup,
+        "ms_per_step": total_ms / nsteps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int4 codes (e4m3 MMA) + f32 scales, bf16 out", "data": "synthetic",
+        "config": dict(WORKLOAD, parallelism=f"replicas by token rows x{world}",
+                       l2="rotating buffers: %d sets, %.0f MB > L2" % (ROTATE_SETS, working_mb)),
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 2 * M * K, "d2h_bytes_per_step": 2 * M * N},
+        "gpu_launches": 2 * nsteps,
+        "roofline": roof,
+        "layer_roofline_frac": (t_layer_roof * 1e3) / (total_ms / nsteps),
+        "kernels": kern,
+        "clocks": clocks.summary(),
+    }
+    if not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = cpu_baseline(args.cpu_rows)
+    print(json.dumps(line))
+    for s in sets:
+        s[0].close()
+    return 0
+
+
+def lin_ws_bytes(lin, M):
+    from paper_2609_33269_gb300 import asp
+    return asp.qwam_asp_act_workspace_bytes(lin.h, M)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,142 @@
+/*
+ * qwam_asp.h -- C ABI of the GB300 (sm_103a) implementation of the Action-Subspace Protection
+ * (ASP) linear layer of Q-WAM (arxiv 2609.33269).
+ *
+ * The layer (Sec. 3.2, Eq. (xsplit) and Eq. (asp)), in the row-major notation used here
+ * (X [M,K] = one token per row, W [K,N], U [K,r] = the paper's V with orthonormal columns):
+ *
+ *     p      = X U                       (protected coordinates, kept in 16 bits)
+ *     X_perp = X - p U^T                 (remainder, orthogonal to span(U))
+ *     W_perp = W - U (U^T W)             (deflated weight, Sec. 3.2 "Splitting the layer")
+ *     Y      = p_hat B_hat  +  Q4(X_perp) Q4(W_perp)
+ *
+ * with B_hat = RN_f16(U^T W), p_hat = RN_f16(p), and Q4 the symmetric group quantizer of
+ * Eq. (quant) (Sec. 2) with b = 4: scale s = absmax / 7 per group of `group` consecutive input
+ * channels (App. B.1), codes = nearest integer to x / s (exact quotient, ties to even), so codes
+ * lie in [-7, 7].  Activation scales are float32, weight scales float16 (Table 3: 4.50 bits per
+ * weight at group 32 implies a 16-bit weight scale).  r = 0 gives plain per-group W4A4 (experts
+ * that ASP does not select, Sec. 3.3).
+ *
+ * Conventions for every entry point:
+ *   - Pointers marked "device" are CUDA device pointers on the current device; "host" pointers
+ *     are ordinary host memory.  All device pointers must be 16-byte aligned.
+ *   - The caller owns every buffer it passes in (X, Y, W, U, act_ws).  The handle owns its packed
+ *     weights until qwam_asp_destroy.  No entry point retains a caller pointer after it returns.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).
+ *   - Arguments are validated on the host before anything is launched; an invalid argument
+ *     returns QWAM_ERR_INVALID_ARG and launches nothing.  A failed CUDA call returns
+ *     QWAM_ERR_CUDA.  Run-time entry points are asynchronous and allocate no device memory.
+ *   - Device-side waits are bounded.  A wait that runs out records QWAM_ERR_TIMEOUT in the
+ *     handle's sticky error word (read with qwam_asp_get_error) and the kernel returns.
+ *   - Inputs must be finite.  A handle may be used from one host thread at a time.
+ */
+#ifndef QWAM_ASP_H
+#define QWAM_ASP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st; /* cudaStream_t == struct CUstream_st* */
+
+typedef struct qwam_asp_handle_s* qwam_asp_handle;
+
+typedef enum {
+  QWAM_OK = 0,
+  QWAM_ERR_INVALID_ARG = -1,
+  QWAM_ERR_UNSUPPORTED = -2, /* valid request that this build does not implement (e.g. r > 64) */
+  QWAM_ERR_CUDA = -3,
+  QWAM_ERR_OOM = -4,
+  QWAM_ERR_TIMEOUT = -5,     /* a bounded device wait gave up */
+  QWAM_ERR_RANGE = -6        /* a scale or branch value does not fit its 16-bit format */
+} qwam_status;
+
+enum { QWAM_Y_BF16 = 0, QWAM_Y_FP32 = 1 };
+
+/* Offline packing (Sec. 3.2 Eq. (asp); the W_perp derivation; Eq. (quant) on the weight).
+ *   W_bf16 : device, bf16 [K, N] row-major (the paper's W~ in its transformed coordinates)
+ *   U      : device, float32 [K, r] row-major, orthonormal columns; may be NULL iff r == 0
+ *   K      : input dimension, K % 64 == 0;   N : output dimension, N % 8 == 0
+ *   r      : protected rank, 0 <= r <= min(K, 64) (larger r returns QWAM_ERR_UNSUPPORTED)
+ *   group  : quantization group along K, 32 or 64
+ *   out    : receives the new handle
+ * Computes, in float64 on the device: B_f = U^T W, W_perp = W - U B_f, per (output channel,
+ * group) s_w = RN_f16(absmax / 7) and the codes of W_perp / s_w, B_hat = RN_f16(B_f), and the
+ * bf16 hi/lo split of U used by the activation kernel.  Synchronizes `stream` before returning.
+ * Returns QWAM_ERR_RANGE if a weight scale or a branch value overflows float16. */
+qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int N, int r, int group,
+                                  struct CUstream_st* stream, qwam_asp_handle* out);
+
+/* Bytes of the caller-owned activation workspace needed for M tokens. */
+qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes);
+
+/* Layout of the activation workspace for M tokens (byte offsets from its start):
+ *   codes  : uint8 [M, K/2], two 4-bit two's-complement codes per byte, low nibble = even k
+ *   scales : float32 [K/group, M_pad] (M_pad = M rounded up to 128), s_x of token m, group g
+ *            at [g * M_pad + m]
+ *   p_hat  : float16 [M, r_pad] (r_pad = r rounded up to 16; columns >= r are zero) */
+qwam_status qwam_asp_act_layout(qwam_asp_handle h, int M, size_t* codes_off, size_t* scales_off,
+                                size_t* phat_off, int* M_pad, int* r_pad);
+
+/* Kernel (a): Eq. (xsplit) and the run-time half of Eq. (quant), one launch, asynchronous.
+ *   X_bf16 : device, bf16 [M, K] row-major;  act_ws : device workspace (see above), written
+ * Reads X once from HBM, forms p = X U on tensor cores (bf16 hi/lo split of U, float32
+ * accumulation), X_perp = X - p U^T in float32, and writes codes, float32 scales and p_hat. */
+qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws,
+                                  struct CUstream_st* stream);
+
+/* Kernel (b): the 4-bit GEMM with the low-rank branch in its epilogue, asynchronous.
+ *   act_ws : device workspace filled by qwam_asp_quantize_act for the same M
+ *   Y      : device [M, N] row-major, bf16 (y_dtype QWAM_Y_BF16) or float32 (QWAM_Y_FP32)
+ * Per group g the tensor cores form the exact integer partial sums P_g = sum_k qx qw (codes
+ * expanded to E4M3, which holds every integer in [-7, 7] exactly; float32 accumulation of
+ * integers below 2^12 is exact); the epilogue adds s_x[m,g] s_w[g,n] P_g in float32 and, last,
+ * the branch p_hat B_hat (float16 operands, float32 accumulation). */
+qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle h, void* Y, int y_dtype,
+                          struct CUstream_st* stream);
+
+/* The whole layer: qwam_asp_quantize_act followed by qwam_asp_gemm on `stream`. */
+qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
+                            void* act_ws, struct CUstream_st* stream);
+
+/* Sticky device-side error of the handle (QWAM_OK, QWAM_ERR_TIMEOUT or QWAM_ERR_RANGE);
+ * synchronizes the device.  The word is cleared by this call. */
+qwam_status qwam_asp_get_error(qwam_asp_handle h);
+
+/* Shape of a handle (any output pointer may be NULL). */
+qwam_status qwam_asp_shape(qwam_asp_handle h, int* K, int* N, int* r, int* group, int* r_pad);
+
+/* Copy the packed weights to HOST buffers (any may be NULL), synchronously:
+ *   qw  : uint8 [N, K/2] codes of W_perp, low nibble = even k (two's complement)
+ *   sw  : uint16 (float16 bits) [K/group, N]
+ *   Bh  : uint16 (float16 bits) [N, r_pad]   (B_hat transposed, zero beyond r)
+ *   Uhl : uint16 (bf16 bits) [2, K, r_pad]   (hi and lo parts of U, zero beyond r) */
+qwam_status qwam_asp_export(qwam_asp_handle h, void* qw, void* sw, void* Bh, void* Uhl);
+
+/* Free the handle and its device buffers (synchronizes the device). */
+qwam_status qwam_asp_destroy(qwam_asp_handle h);
+
+const char* qwam_status_string(qwam_status s);
+
+/* ---- test support ------------------------------------------------------------------------ */
+
+/* Kernel (a) with one more output: R, device float32 [M, K], receives X_perp exactly as the
+ * kernel forms it before quantization (so the quantizer can be checked bit for bit). */
+qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws, float* R,
+                                    struct CUstream_st* stream);
+
+/* Set the bound of every device wait of this handle's kernels, in seconds (default 2.0). */
+qwam_status qwam_asp_set_timeout(qwam_asp_handle h, double seconds);
+
+/* Launch one CTA that waits on a shared-memory barrier nothing arrives on, with a bound of
+ * `timeout_us` microseconds; the wait runs out, the kernel records QWAM_ERR_TIMEOUT in the
+ * handle's error word and returns.  Exercises the bounded-wait path without a fault. */
+qwam_status qwam_asp_debug_wait_timeout(qwam_asp_handle h, int timeout_us, struct CUstream_st* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* QWAM_ASP_H */

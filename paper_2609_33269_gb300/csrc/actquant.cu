@@ -1,0 +1,465 @@
+// actquant.cu -- kernel (a): the run-time activation path of the ASP layer.
+//
+//   p      = X U                (Sec. 3.2 Eq. (xsplit): the protected coordinates V^T x)
+//   X_perp = X - p U^T          (the remainder (I - V V^T) x)
+//   s_x    = RN_f32(absmax(X_perp over a group) / 7),  codes = nearest(X_perp / s_x)
+//                               (Eq. (quant) with b = 4; App. B.1: per token, per group)
+//   p_hat  = RN_f16(p)          (the 16-bit branch input of Eq. (asp))
+//
+// One CTA owns 128 token rows (one TMEM lane per row) and a slice of K; the C CTAs of a
+// thread-block cluster cover the whole of K for the same rows.  Each CTA streams its X slice
+// through a TMA ring twice: pass 1 feeds p_part = X_slice [U_hi | U_lo] into TMEM (bf16
+// tensor-core MMA, float32 accumulation); the partial projections are summed across the
+// cluster through distributed shared memory (fixed order, so every CTA sees the same p);
+// pass 2 re-reads the slice (L2-resident by then) while the tensor cores form
+// R = [p_hi | p_hi | p_lo] [U_hi | U_lo | U_hi]^T, and the epilogue warps form X_perp = X - R
+// in float32 and quantize it.  With r = 0 the kernel is a single streaming pass (no MMA).
+//
+// Warp roles (192 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner,
+// warps 2..5 epilogue (thread = token row).
+#include <algorithm>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace qwam {
+namespace {
+
+struct ActArgs {
+  int M, K, G, C, Kc, M_pad;
+  uint8_t* codes;   // [M, K/2]
+  float* scales;    // [K/G, M_pad]
+  __half* phat;     // [M, RP]
+  float* dump;      // optional [M, K]
+  int* err;
+  uint64_t timeout_ns;
+};
+
+template <int RP>
+struct ActCfg {
+  static constexpr int KU3 = RP == 0 ? 0 : ((3 * RP + 63) / 64) * 64;  // (hi, hi, lo) width, padded
+  static constexpr int X_BYTES = kBM * kChunk * 2;                     // 16 KB, 128-byte swizzle
+  static constexpr int U1_BYTES = 2 * RP * 128;                        // [U_hi|U_lo]^T chunk
+  static constexpr int U2_BYTES = kChunk * KU3 * 2;                    // Ucat3 chunk, KU3/64 atoms
+  static constexpr int U_BYTES = U1_BYTES > U2_BYTES ? U1_BYTES : U2_BYTES;
+  static constexpr int STAGE = X_BYTES + U_BYTES;
+  static constexpr int S = RP == 0 ? 6 : (RP <= 32 ? 4 : 2);
+  static constexpr int AREC_BYTES = kBM * KU3 * 2;
+  static constexpr int PP_BYTES = kBM * RP * 4;
+  static constexpr int NBAR = 2 * S + 7;
+  static constexpr int SMEM = 1024 + S * STAGE + AREC_BYTES + 2 * PP_BYTES + NBAR * 8 + 16;
+  static constexpr uint32_t TMEM_COLS = 256;  // proj at col 0 (2*RP <= 128), rec buffers at 128, 192
+};
+
+__device__ __forceinline__ int nearest_code_f32(float x, float s, float inv) {
+  // Nearest integer to the exact quotient x / s, ties to even.  c is within one of it; the
+  // remainder x - c s is exact in float32 (see the design notes), so it decides exactly.
+  float c = rintf(x * inv);
+  float e = fmaf(-c, s, x);
+  float t = 2.0f * fabsf(e);
+  int ci = static_cast<int>(c);
+  if (t > s || (t == s && (ci & 1))) ci += (e > 0.0f) ? 1 : -1;
+  return ci;
+}
+
+// One group of GS remainder values: s = RN_f32(absmax / 7) (IEEE division), codes packed two
+// per byte, low nibble first.
+template <int GS>
+__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* packed, float* scale_out) {
+  float amax = 0.0f;
+#pragma unroll
+  for (int i = 0; i < GS; ++i) amax = fmaxf(amax, fabsf(xp[i]));
+  const float sc = __fdiv_rn(amax, 7.0f);
+  const float inv = sc > 0.0f ? __frcp_rn(sc) : 0.0f;
+  *scale_out = sc;
+#pragma unroll
+  for (int w8 = 0; w8 < GS / 8; ++w8) {
+    uint32_t word = 0;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int ci = nearest_code_f32(xp[8 * w8 + u], sc, inv);
+      word |= (static_cast<uint32_t>(ci) & 0xFu) << (4 * u);
+    }
+    packed[w8] = word;
+  }
+}
+
+template <int RP>
+__global__ void __launch_bounds__(192, 1)
+    actquant_kernel(const __grid_constant__ CUtensorMap x_map, const __grid_constant__ CUtensorMap ut_map,
+                    const __grid_constant__ CUtensorMap u3_map, const ActArgs a) {
+  using Cfg = ActCfg<RP>;
+  constexpr int S = Cfg::S;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* stages = smem;
+  uint8_t* arec = stages + S * Cfg::STAGE;
+  float* ppart = reinterpret_cast<float*>(arec + Cfg::AREC_BYTES);
+  float* pred = ppart + kBM * RP;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(pred) + Cfg::PP_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + S;
+  uint64_t* proj_done = bars + 2 * S;
+  uint64_t* arec_ready = proj_done + 1;
+  uint64_t* tfull = proj_done + 2;
+  uint64_t* tempty = proj_done + 4;
+  uint64_t* drain = proj_done + 6;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + Cfg::NBAR);
+  int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+  const uint32_t wid = warp_id(), lane = lane_id();
+  const int C = a.C;
+  const uint32_t rank = (RP > 0 && C > 1) ? cluster_ctarank() : 0u;
+  const int cta_k = (RP > 0) ? static_cast<int>(rank) : static_cast<int>(blockIdx.x);
+  const int k0 = cta_k * a.Kc;
+  const int m0 = blockIdx.y * kBM;
+  const int nch = a.Kc / kChunk;
+  const int pass1 = RP > 0 ? nch : 0;  // pass-1 iterations before pass 2 in the ring order
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < S; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(proj_done, 1);
+    mbar_init(arec_ready, 128);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 128);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (RP > 0 && wid == 1) {
+    tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+    tmem_relinquish();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = (RP > 0) ? *tmem_slot : 0u;
+  const WaitCtl wc{abort_flag, a.err, globaltimer_ns() + a.timeout_ns};
+
+  auto stage_x = [&](int s) { return stages + s * Cfg::STAGE; };
+  auto stage_u = [&](int s) { return stages + s * Cfg::STAGE + Cfg::X_BYTES; };
+
+  if (wid == 0) {
+    // ------------------------------------------------------------- TMA producer
+    int it = 0, issued2 = 0;
+    bool ok = true;
+    auto produce = [&](bool first_pass, int c) {
+      const int s = it % S;
+      if (ok && it >= S) ok = mbar_wait(&empty[s], ((it / S) & 1) ^ 1, wc);
+      if (ok) {
+        const uint32_t bytes = Cfg::X_BYTES + (first_pass ? Cfg::U1_BYTES : (RP > 0 ? Cfg::U2_BYTES : 0));
+        mbar_arrive_expect_tx(&full[s], bytes);
+        tma_load_2d(stage_x(s), &x_map, &full[s], k0 + c * kChunk, m0);
+        if (first_pass) {
+          tma_load_2d(stage_u(s), &ut_map, &full[s], k0 + c * kChunk, 0);
+        } else if (RP > 0) {
+          for (int q = 0; q < Cfg::KU3 / 64; ++q)
+            tma_load_2d(stage_u(s) + q * 8192, &u3_map, &full[s], q * 64, k0 + c * kChunk);
+        }
+      }
+      ++it;
+    };
+    if (lane == 0) {
+      tma_prefetch_desc(&x_map);
+      for (int c = 0; c < pass1; ++c) produce(true, c);
+      for (; issued2 < nch && issued2 < S; ++issued2) produce(false, issued2);
+    }
+    __syncwarp();
+    if (RP > 0) {
+      cluster_sync();
+      cluster_sync();
+      cluster_sync();
+    }
+    if (lane == 0) {
+      for (; issued2 < nch; ++issued2) produce(false, issued2);
+      // Let every load issued into the ring land before the CTA can exit.
+      int never = 0;
+      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+      for (int j = std::max(0, it - S); j < it; ++j) mbar_wait(&full[j % S], (j / S) & 1, dc);
+    }
+  } else if (wid == 1) {
+    // ------------------------------------------------------------- MMA issuer
+    if constexpr (RP > 0) {
+      bool ok = true;
+      if (lane == 0) {
+        constexpr uint32_t idesc_proj = idesc_bf16(kBM, 2 * RP);
+        for (int c = 0; c < nch && ok; ++c) {
+          const int s = c % S;
+          ok = mbar_wait(&full[s], (c / S) & 1, wc);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t xa = smem_u32(stage_x(s)), ua = smem_u32(stage_u(s));
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            mma_f16(tmem, smem_desc(xa + kk * 32, 16, 1024, kSw128), smem_desc(ua + kk * 32, 16, 1024, kSw128),
+                    idesc_proj, (c | kk) != 0);
+          mma_commit(&empty[s]);
+        }
+        mma_commit(proj_done);
+      }
+      __syncwarp();
+      cluster_sync();
+      cluster_sync();
+      cluster_sync();
+      if (lane == 0) {
+        if (ok) ok = mbar_wait(arec_ready, 0, wc);
+        tc_fence_after();
+        constexpr uint32_t idesc_rec = idesc_bf16(kBM, kChunk);
+        const uint32_t ar = smem_u32(arec);
+        for (int c = 0; c < nch && ok; ++c) {
+          const int it = pass1 + c, s = it % S, b = c & 1;
+          ok = mbar_wait(&full[s], (it / S) & 1, wc);
+          if (ok && c >= 2) ok = mbar_wait(&tempty[b], ((c >> 1) & 1) ^ 1, wc);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t ua = smem_u32(stage_u(s));
+#pragma unroll
+          for (int kk = 0; kk < 3 * RP / 16; ++kk) {
+            const int q = kk >> 2, off = (kk & 3) * 32;
+            mma_f16(tmem + 128 + 64 * b, smem_desc(ar + q * 16384 + off, 16, 1024, kSw128),
+                    smem_desc(ua + q * 8192 + off, 16, 1024, kSw128), idesc_rec, kk != 0);
+          }
+          mma_commit(&tfull[b]);
+        }
+        // Make sure every MMA of this CTA has completed before TMEM is released.
+        mma_commit(drain);
+        int never = 0;
+        const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+        mbar_wait(drain, 0, dc);
+      }
+      __syncwarp();
+    }
+  } else {
+    // ------------------------------------------------------------- epilogue (thread = row)
+    const int quad = wid & 3;
+    const int row = quad * 32 + static_cast<int>(lane);
+    const int m = m0 + row;
+    const int et = static_cast<int>(wid - 2) * 32 + static_cast<int>(lane);
+    const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    bool ok = true;
+
+    if constexpr (RP > 0) {
+      // -- partial projection of this CTA's K slice: hi part + lo part
+      ok = mbar_wait(proj_done, 0, wc);
+      tc_fence_after();
+      float pp[RP];
+#pragma unroll
+      for (int q = 0; q < RP / 16; ++q) {
+        uint32_t vh[16], vl[16];
+        tmem_ld16(tlane + q * 16, vh);
+        tmem_ld16(tlane + RP + q * 16, vl);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) pp[q * 16 + i] = __uint_as_float(vh[i]) + __uint_as_float(vl[i]);
+      }
+      float4* prow = reinterpret_cast<float4*>(ppart + row * RP);
+#pragma unroll
+      for (int j = 0; j < RP / 4; ++j) prow[j] = make_float4(pp[4 * j], pp[4 * j + 1], pp[4 * j + 2], pp[4 * j + 3]);
+      cluster_sync();  // A: every CTA's partial is in its shared memory
+      // -- reduce-scatter: this CTA sums rows [rank*Rc, (rank+1)*Rc) over the cluster, in rank order
+      const int Rc = kBM / C;
+      const int n4 = Rc * RP / 4;
+      const uint32_t pp_base = smem_u32(ppart);
+      for (int i = et; i < n4; i += 128) {
+        const uint32_t off = static_cast<uint32_t>((static_cast<int>(rank) * Rc * RP + 4 * i) * 4);
+        float4 acc = ld_dsmem_f4(mapa_smem(pp_base + off, 0));
+        for (int q = 1; q < C; ++q) {
+          const float4 v = ld_dsmem_f4(mapa_smem(pp_base + off, static_cast<uint32_t>(q)));
+          acc.x += v.x;
+          acc.y += v.y;
+          acc.z += v.z;
+          acc.w += v.w;
+        }
+        reinterpret_cast<float4*>(pred)[i] = acc;
+        const int lr = (4 * i) / RP, col = (4 * i) % RP;
+        const int gm = m0 + static_cast<int>(rank) * Rc + lr;
+        if (gm < a.M) {
+          __half2 h01 = __floats2half2_rn(acc.x, acc.y), h23 = __floats2half2_rn(acc.z, acc.w);
+          uint2 hv;
+          hv.x = *reinterpret_cast<uint32_t*>(&h01);
+          hv.y = *reinterpret_cast<uint32_t*>(&h23);
+          *reinterpret_cast<uint2*>(a.phat + static_cast<size_t>(gm) * RP + col) = hv;
+        }
+      }
+      cluster_sync();  // B: the reduced rows are in their owners' shared memory
+      // -- gather this thread's row of p from its owner
+      const int owner = row / Rc, lr = row % Rc;
+      const uint32_t pr_base = smem_u32(pred);
+      float p[RP];
+#pragma unroll
+      for (int j = 0; j < RP / 4; ++j) {
+        const float4 v = ld_dsmem_f4(mapa_smem(pr_base + static_cast<uint32_t>((lr * RP + 4 * j) * 4),
+                                               static_cast<uint32_t>(owner)));
+        p[4 * j] = v.x;
+        p[4 * j + 1] = v.y;
+        p[4 * j + 2] = v.z;
+        p[4 * j + 3] = v.w;
+      }
+      cluster_sync();  // C: no CTA reads a peer's shared memory after this point
+      // -- A operand of the reconstruction: [p_hi | p_hi | p_lo | 0], 128-byte swizzle
+      __nv_bfloat16 hi[RP], lo[RP];
+#pragma unroll
+      for (int j = 0; j < RP; ++j) {
+        hi[j] = __float2bfloat16_rn(p[j]);
+        lo[j] = __float2bfloat16_rn(p[j] - __bfloat162float(hi[j]));
+      }
+#pragma unroll
+      for (int c8 = 0; c8 < Cfg::KU3 / 8; ++c8) {  // 16-byte chunk of 8 bf16
+        uint32_t w[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          __nv_bfloat16 e2[2];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int col = c8 * 8 + 2 * t + u;
+            e2[u] = col < RP ? hi[col % RP]
+                    : col < 2 * RP ? hi[col % RP]
+                    : col < 3 * RP ? lo[col % RP]
+                                   : __float2bfloat16_rn(0.0f);
+          }
+          w[t] = static_cast<uint32_t>(*reinterpret_cast<uint16_t*>(&e2[0])) |
+                 (static_cast<uint32_t>(*reinterpret_cast<uint16_t*>(&e2[1])) << 16);
+        }
+        const int q = c8 >> 3, j = c8 & 7;
+        *reinterpret_cast<uint4*>(arec + q * 16384 + row * 128 + ((j ^ (row & 7)) << 4)) =
+            make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(arec_ready);
+    }
+
+    // -- pass 2: remainder and quantization, one 64-column chunk at a time
+    const int half_k = a.K / 2;
+    for (int c = 0; c < nch; ++c) {
+      const int it = pass1 + c, s = it % S;
+      float xp[kChunk];
+      if constexpr (RP > 0) {
+        const int b = c & 1;
+        if (ok) ok = mbar_wait(&tfull[b], (c >> 1) & 1, wc);
+        tc_fence_after();
+        uint32_t r0[32], r1[32];
+        tmem_ld32(tlane + 128 + 64 * b, r0);
+        tmem_ld32(tlane + 128 + 64 * b + 32, r1);
+        tmem_ld_wait();
+        tc_fence_before();
+        mbar_arrive(&tempty[b]);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          xp[i] = __uint_as_float(r0[i]);
+          xp[32 + i] = __uint_as_float(r1[i]);
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < kChunk; ++i) xp[i] = 0.0f;
+      }
+      if (ok) ok = mbar_wait(&full[s], (it / S) & 1, wc);
+      const uint8_t* xs = stage_x(s) + row * 128;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const uint4 v = *reinterpret_cast<const uint4*>(xs + ((j ^ (row & 7)) << 4));
+        const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const float lo_f = __uint_as_float(wv[t] << 16);
+          const float hi_f = __uint_as_float(wv[t] & 0xFFFF0000u);
+          xp[8 * j + 2 * t] = lo_f - xp[8 * j + 2 * t];
+          xp[8 * j + 2 * t + 1] = hi_f - xp[8 * j + 2 * t + 1];
+        }
+      }
+      named_bar_sync(1, 128);
+      if (et == 0) mbar_arrive(&empty[s]);
+      if (!ok || m >= a.M) continue;
+
+      const int kc = k0 + c * kChunk;
+      if (a.dump) {
+        float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + kc);
+#pragma unroll
+        for (int i = 0; i < kChunk / 4; ++i) d[i] = make_float4(xp[4 * i], xp[4 * i + 1], xp[4 * i + 2], xp[4 * i + 3]);
+      }
+      uint32_t packed[8];
+      if (a.G == 64) {
+        quantize_group<64>(xp, packed, a.scales + static_cast<size_t>(kc / 64) * a.M_pad + m);
+      } else {
+        quantize_group<32>(xp, packed, a.scales + static_cast<size_t>(kc / 32) * a.M_pad + m);
+        quantize_group<32>(xp + 32, packed + 4, a.scales + static_cast<size_t>(kc / 32 + 1) * a.M_pad + m);
+      }
+      uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * half_k + kc / 2);
+      dst[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+      dst[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+    }
+    if constexpr (RP == 0) {
+      (void)tlane;
+    }
+  }
+
+  __syncthreads();
+  if (RP > 0 && wid == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Cfg::TMEM_COLS);
+  }
+}
+
+template <int RP>
+cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
+  using Cfg = ActCfg<RP>;
+  const ActLayout L = act_layout(h, M);
+  ActArgs a;
+  a.M = M;
+  a.K = h.K;
+  a.G = h.G;
+  const int chunks = h.K / kChunk;
+  const int tiles = (M + kBM - 1) / kBM;
+  int C = 1;
+  while (C < 8 && chunks % (2 * C) == 0 && tiles * C < 2 * 152) C *= 2;
+  a.C = C;
+  a.Kc = h.K / C;
+  a.M_pad = L.M_pad;
+  uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
+  a.codes = base + L.codes_off;
+  a.scales = reinterpret_cast<float*>(base + L.scales_off);
+  a.phat = reinterpret_cast<__half*>(base + L.phat_off);
+  a.dump = dump;
+  a.err = h.err;
+  a.timeout_ns = deadline_budget_ns(h);
+
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(actquant_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(C, tiles, 1);
+  cfg.blockDim = dim3(192, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (RP > 0) ? C : 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const CUtensorMap& ut = (RP > 0) ? h.ucat_t_map : am.x_map;
+  const CUtensorMap& u3 = (RP > 0) ? h.ucat3_map : am.x_map;
+  return cudaLaunchKernelEx(&cfg, actquant_kernel<RP>, am.x_map, ut, u3, a);
+}
+
+}  // namespace
+
+cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
+  switch (h.r_pad) {
+    case 0: return launch_rp<0>(h, am, ws, M, dump, s);
+    case 16: return launch_rp<16>(h, am, ws, M, dump, s);
+    case 32: return launch_rp<32>(h, am, ws, M, dump, s);
+    case 48: return launch_rp<48>(h, am, ws, M, dump, s);
+    case 64: return launch_rp<64>(h, am, ws, M, dump, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace qwam

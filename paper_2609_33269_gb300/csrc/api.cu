@@ -1,0 +1,336 @@
+// api.cu -- the C ABI declared in include/qwam_asp.h: argument validation, the handle's device
+// buffers, TMA tensor maps, and the launches.  No entry point on the run-time path allocates
+// device memory.
+#include <cudaTypedefs.h>
+
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace qwam {
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool ensure_encoder() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_encode != nullptr;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t up256(size_t b) { return (b + 255) & ~size_t(255); }
+
+__global__ void wait_probe_kernel(int* err, uint64_t timeout_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const WaitCtl wc{&abort_flag, err, globaltimer_ns() + timeout_ns};
+    mbar_wait(&bar, 0, wc);  // nothing arrives: the bound runs out and records kErrTimeout
+    mbar_arrive(&bar);       // complete the phase so the barrier is left consistent
+  }
+}
+
+}  // namespace
+
+bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint64_t inner, uint64_t outer,
+               uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle sw) {
+  if (!ensure_encoder()) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+ActLayout act_layout(const Handle& h, int M) {
+  ActLayout L;
+  L.M_pad = round_up(M > 0 ? M : 1, kBM);
+  L.codes_off = 0;
+  L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
+  L.phat_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
+  L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
+  return L;
+}
+
+uint64_t deadline_budget_ns(const Handle& h) { return static_cast<uint64_t>(h.timeout_s * 1e9); }
+
+const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
+  for (auto& c : h.act_cache)
+    if (c.ws == ws && c.M == M && (x == nullptr || c.x == x)) return &c;
+  ActMaps& c = h.act_cache[h.act_next];
+  h.act_next = (h.act_next + 1) % 4;
+  c.ws = nullptr;
+  const ActLayout L = act_layout(h, M);
+  const uint8_t* base = static_cast<const uint8_t*>(ws);
+  bool ok = true;
+  if (x) {
+    ok &= encode_2d(&c.x_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, h.K, M, static_cast<uint64_t>(h.K) * 2, kChunk, kBM,
+                    CU_TENSOR_MAP_SWIZZLE_128B);
+  }
+  ok &= encode_2d(&c.qx_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, kGemmKS / 2, kBM,
+                  CU_TENSOR_MAP_SWIZZLE_NONE);
+  ok &= encode_2d(&c.sx_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.scales_off, M, h.K / h.G,
+                  static_cast<uint64_t>(L.M_pad) * 4, kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
+  if (h.r_pad > 0)
+    ok &= encode_2d(&c.ph_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
+                    static_cast<uint64_t>(h.r_pad) * 2, 8, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+  if (!ok) return nullptr;
+  c.ws = ws;
+  c.x = x;
+  c.M = M;
+  return &c;
+}
+
+cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(h.err, static_cast<uint64_t>(timeout_us) * 1000ull);
+  return cudaGetLastError();
+}
+
+}  // namespace qwam
+
+using qwam::Handle;
+
+static qwam_status from_cuda_status(cudaError_t e) { return e == cudaSuccess ? QWAM_OK : QWAM_ERR_CUDA; }
+
+extern "C" {
+
+const char* qwam_status_string(qwam_status s) {
+  switch (s) {
+    case QWAM_OK: return "ok";
+    case QWAM_ERR_INVALID_ARG: return "invalid argument";
+    case QWAM_ERR_UNSUPPORTED: return "unsupported configuration";
+    case QWAM_ERR_CUDA: return "CUDA error";
+    case QWAM_ERR_OOM: return "out of device memory";
+    case QWAM_ERR_TIMEOUT: return "device wait timed out";
+    case QWAM_ERR_RANGE: return "value out of 16-bit range";
+  }
+  return "unknown status";
+}
+
+qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int N, int r, int group,
+                                  struct CUstream_st* stream, qwam_asp_handle* out) {
+  if (!out) return QWAM_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!W_bf16 || !qwam::aligned16(W_bf16)) return QWAM_ERR_INVALID_ARG;
+  if (K <= 0 || K % 64 != 0 || N <= 0 || N % 8 != 0) return QWAM_ERR_INVALID_ARG;
+  if (group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
+  if (r < 0 || r > K) return QWAM_ERR_INVALID_ARG;
+  if (r > 0 && (!U || !qwam::aligned16(U))) return QWAM_ERR_INVALID_ARG;
+  if (r > qwam::kMaxRank) return QWAM_ERR_UNSUPPORTED;
+  if (!qwam::ensure_encoder()) return QWAM_ERR_CUDA;
+
+  auto* hs = new (std::nothrow) qwam_asp_handle_s();
+  if (!hs) return QWAM_ERR_OOM;
+  Handle& h = hs->h;
+  h.K = K;
+  h.N = N;
+  h.r = r;
+  h.G = group;
+  h.r_pad = r == 0 ? 0 : qwam::round_up(r, 16);
+  h.N_pad = qwam::round_up(N, qwam::kGemmBN);
+  h.ku3 = h.r_pad == 0 ? 0 : qwam::round_up(3 * h.r_pad, 64);
+  cudaGetDevice(&h.device);
+
+  const size_t b_qw = qwam::up256(static_cast<size_t>(h.N_pad) * (K / 2));
+  const size_t b_sw = qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
+  const size_t b_bh = qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2);
+  const size_t b_ut = qwam::up256(static_cast<size_t>(2 * h.r_pad) * K * 2);
+  const size_t b_u3 = qwam::up256(static_cast<size_t>(K) * h.ku3 * 2);
+  const size_t total = b_qw + b_sw + b_bh + b_ut + b_u3 + 256;
+  if (cudaMalloc(&h.block, total) != cudaSuccess) {
+    cudaGetLastError();
+    delete hs;
+    return QWAM_ERR_OOM;
+  }
+  uint8_t* p = static_cast<uint8_t*>(h.block);
+  h.qw = p;
+  h.sw = reinterpret_cast<__half*>(p + b_qw);
+  h.Bh = reinterpret_cast<__half*>(p + b_qw + b_sw);
+  h.ucat_t = reinterpret_cast<__nv_bfloat16*>(p + b_qw + b_sw + b_bh);
+  h.ucat3 = reinterpret_cast<__nv_bfloat16*>(p + b_qw + b_sw + b_bh + b_ut);
+  h.err = reinterpret_cast<int*>(p + b_qw + b_sw + b_bh + b_ut + b_u3);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+  bool ok = true;
+  ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kGemmKS / 2, qwam::kBM,
+                        CU_TENSOR_MAP_SWIZZLE_NONE);
+  ok &= qwam::encode_2d(&h.sw_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.sw, N, K / group,
+                        static_cast<uint64_t>(h.N_pad) * 2, qwam::kGemmBN, qwam::kGemmKS / group,
+                        CU_TENSOR_MAP_SWIZZLE_NONE);
+  if (h.r_pad > 0) {
+    ok &= qwam::encode_2d(&h.Bh_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,
+                          static_cast<uint64_t>(h.r_pad) * 2, 8, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= qwam::encode_2d(&h.ucat_t_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h.ucat_t, K, 2 * h.r_pad,
+                          static_cast<uint64_t>(K) * 2, qwam::kChunk, 2 * h.r_pad, CU_TENSOR_MAP_SWIZZLE_128B);
+    ok &= qwam::encode_2d(&h.ucat3_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h.ucat3, h.ku3, K,
+                          static_cast<uint64_t>(h.ku3) * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
+  }
+  if (!ok) {
+    cudaFree(h.block);
+    delete hs;
+    return QWAM_ERR_CUDA;
+  }
+  cudaError_t e = cudaMemsetAsync(h.block, 0, total, s);
+  if (e == cudaSuccess)
+    e = qwam::launch_pack(h, static_cast<const __nv_bfloat16*>(W_bf16), r > 0 ? U : nullptr, s);
+  int herr = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&herr, h.err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess || herr != 0) {
+    cudaFree(h.block);
+    delete hs;
+    return e != cudaSuccess ? QWAM_ERR_CUDA : QWAM_ERR_RANGE;
+  }
+  *out = hs;
+  return QWAM_OK;
+}
+
+qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle hs, int M, size_t* bytes) {
+  if (!hs || !bytes || M < 0) return QWAM_ERR_INVALID_ARG;
+  *bytes = qwam::act_layout(hs->h, M).bytes;
+  return QWAM_OK;
+}
+
+qwam_status qwam_asp_act_layout(qwam_asp_handle hs, int M, size_t* codes_off, size_t* scales_off, size_t* phat_off,
+                                int* M_pad, int* r_pad) {
+  if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
+  const qwam::ActLayout L = qwam::act_layout(hs->h, M);
+  if (codes_off) *codes_off = L.codes_off;
+  if (scales_off) *scales_off = L.scales_off;
+  if (phat_off) *phat_off = L.phat_off;
+  if (M_pad) *M_pad = L.M_pad;
+  if (r_pad) *r_pad = hs->h.r_pad;
+  return QWAM_OK;
+}
+
+static qwam_status quantize_impl(const void* X, int M, qwam_asp_handle hs, void* ws, float* dump,
+                                 struct CUstream_st* stream) {
+  if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
+  if (M == 0) return QWAM_OK;
+  if (!X || !ws || !qwam::aligned16(X) || !qwam::aligned16(ws)) return QWAM_ERR_INVALID_ARG;
+  if (dump && !qwam::aligned16(dump)) return QWAM_ERR_INVALID_ARG;
+  Handle& h = hs->h;
+  const qwam::ActMaps* am = qwam::get_act_maps(h, X, ws, M);
+  if (!am) return QWAM_ERR_CUDA;
+  return from_cuda_status(qwam::launch_actquant(h, *am, ws, M, dump, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws,
+                                  struct CUstream_st* stream) {
+  return quantize_impl(X_bf16, M, h, act_ws, nullptr, stream);
+}
+
+qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws, float* R,
+                                    struct CUstream_st* stream) {
+  if (!R) return QWAM_ERR_INVALID_ARG;
+  return quantize_impl(X_bf16, M, h, act_ws, R, stream);
+}
+
+qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle hs, void* Y, int y_dtype,
+                          struct CUstream_st* stream) {
+  if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
+  if (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32) return QWAM_ERR_INVALID_ARG;
+  if (M == 0) return QWAM_OK;
+  if (!act_ws || !Y || !qwam::aligned16(act_ws) || !qwam::aligned16(Y)) return QWAM_ERR_INVALID_ARG;
+  Handle& h = hs->h;
+  const qwam::ActMaps* am = qwam::get_act_maps(h, nullptr, act_ws, M);
+  if (!am) return QWAM_ERR_CUDA;
+  return from_cuda_status(qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32,
+                                            reinterpret_cast<cudaStream_t>(stream)));
+}
+
+qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype, void* act_ws,
+                            struct CUstream_st* stream) {
+  if (!h || M < 0 || (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32)) return QWAM_ERR_INVALID_ARG;
+  if (M > 0 && (!Y || !qwam::aligned16(Y))) return QWAM_ERR_INVALID_ARG;
+  qwam_status st = qwam_asp_quantize_act(X_bf16, M, h, act_ws, stream);
+  if (st != QWAM_OK) return st;
+  return qwam_asp_gemm(act_ws, M, h, Y, y_dtype, stream);
+}
+
+qwam_status qwam_asp_get_error(qwam_asp_handle hs) {
+  if (!hs) return QWAM_ERR_INVALID_ARG;
+  if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, hs->h.err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return QWAM_ERR_CUDA;
+  if (cudaMemset(hs->h.err, 0, sizeof(int)) != cudaSuccess) return QWAM_ERR_CUDA;
+  if (v & qwam::kErrTimeout) return QWAM_ERR_TIMEOUT;
+  if (v & qwam::kErrRange) return QWAM_ERR_RANGE;
+  return QWAM_OK;
+}
+
+qwam_status qwam_asp_shape(qwam_asp_handle hs, int* K, int* N, int* r, int* group, int* r_pad) {
+  if (!hs) return QWAM_ERR_INVALID_ARG;
+  if (K) *K = hs->h.K;
+  if (N) *N = hs->h.N;
+  if (r) *r = hs->h.r;
+  if (group) *group = hs->h.G;
+  if (r_pad) *r_pad = hs->h.r_pad;
+  return QWAM_OK;
+}
+
+qwam_status qwam_asp_export(qwam_asp_handle hs, void* qw, void* sw, void* Bh, void* Uhl) {
+  if (!hs) return QWAM_ERR_INVALID_ARG;
+  Handle& h = hs->h;
+  if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
+  cudaError_t e = cudaSuccess;
+  if (qw) e = cudaMemcpy(qw, h.qw, static_cast<size_t>(h.N) * (h.K / 2), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && sw)
+    e = cudaMemcpy2D(sw, static_cast<size_t>(h.N) * 2, h.sw, static_cast<size_t>(h.N_pad) * 2,
+                     static_cast<size_t>(h.N) * 2, h.K / h.G, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && Bh && h.r_pad > 0)
+    e = cudaMemcpy(Bh, h.Bh, static_cast<size_t>(h.N) * h.r_pad * 2, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && Uhl && h.r_pad > 0) {
+    std::vector<uint16_t> t(static_cast<size_t>(2 * h.r_pad) * h.K);
+    e = cudaMemcpy(t.data(), h.ucat_t, t.size() * 2, cudaMemcpyDeviceToHost);
+    uint16_t* o = static_cast<uint16_t*>(Uhl);
+    for (int part = 0; part < 2 && e == cudaSuccess; ++part)
+      for (int k = 0; k < h.K; ++k)
+        for (int j = 0; j < h.r_pad; ++j)
+          o[(static_cast<size_t>(part) * h.K + k) * h.r_pad + j] =
+              t[static_cast<size_t>(part * h.r_pad + j) * h.K + k];
+  }
+  return from_cuda_status(e);
+}
+
+qwam_status qwam_asp_destroy(qwam_asp_handle hs) {
+  if (!hs) return QWAM_ERR_INVALID_ARG;
+  cudaDeviceSynchronize();
+  cudaError_t e = cudaFree(hs->h.block);
+  delete hs;
+  return from_cuda_status(e);
+}
+
+qwam_status qwam_asp_set_timeout(qwam_asp_handle hs, double seconds) {
+  if (!hs || !(seconds > 0.0) || seconds > 3600.0) return QWAM_ERR_INVALID_ARG;
+  hs->h.timeout_s = seconds;
+  return QWAM_OK;
+}
+
+qwam_status qwam_asp_debug_wait_timeout(qwam_asp_handle hs, int timeout_us, struct CUstream_st* stream) {
+  if (!hs || timeout_us <= 0 || timeout_us > 10000000) return QWAM_ERR_INVALID_ARG;
+  return from_cuda_status(qwam::launch_wait_probe(hs->h, timeout_us, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

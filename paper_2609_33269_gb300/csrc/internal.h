@@ -1,0 +1,73 @@
+// internal.h -- handle layout and kernel launchers shared by the translation units of the
+// library (never by the oracle).
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/qwam_asp.h"
+
+namespace qwam {
+
+constexpr int kBM = 128;        // token rows per CTA tile (one TMEM lane per row)
+constexpr int kChunk = 64;      // K columns per activation chunk (bf16: one 128-byte row)
+constexpr int kMaxRank = 64;    // largest protected rank of this build
+constexpr int kGemmBN = 128;    // output columns per GEMM CTA tile
+constexpr int kGemmKS = 128;    // K elements per GEMM pipeline stage
+
+inline int round_up(int a, int b) { return (a + b - 1) / b * b; }
+
+// Activation-side tensor maps for one (workspace, X, M) triple.
+struct ActMaps {
+  const void* ws = nullptr;
+  const void* x = nullptr;
+  int M = -1;
+  CUtensorMap x_map;    // X bf16 [M, K], box {64, 128}, 128-byte swizzle
+  CUtensorMap qx_map;   // codes u8 [M, K/2], box {64, 128}
+  CUtensorMap sx_map;   // scales f32 [K/G, M_pad] (dims {M, K/G}), box {128, KS/G}
+  CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128}
+};
+
+struct Handle {
+  int K = 0, N = 0, r = 0, G = 0, r_pad = 0, N_pad = 0, ku3 = 0;
+  int device = 0;
+  void* block = nullptr;             // one device allocation holding every buffer below
+  uint8_t* qw = nullptr;             // [N_pad, K/2]
+  __half* sw = nullptr;              // [K/G, N_pad]
+  __half* Bh = nullptr;              // [N_pad, r_pad]
+  __nv_bfloat16* ucat_t = nullptr;   // [2 r_pad, K]: rows 0..r_pad-1 = U_hi^T, then U_lo^T
+  __nv_bfloat16* ucat3 = nullptr;    // [K, ku3]: row k = U_hi[k,:], U_lo[k,:], U_hi[k,:], zeros
+  int* err = nullptr;                // sticky device error word
+  double timeout_s = 2.0;
+  CUtensorMap qw_map, sw_map, Bh_map, ucat_t_map, ucat3_map;
+  ActMaps act_cache[4];
+  int act_next = 0;
+};
+
+struct ActLayout {
+  size_t codes_off, scales_off, phat_off, bytes;
+  int M_pad;
+};
+ActLayout act_layout(const Handle& h, int M);
+
+// Tensor-map encoder (driver entry point fetched through the runtime).
+bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint64_t inner, uint64_t outer,
+               uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle sw);
+const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M);
+
+uint64_t deadline_budget_ns(const Handle& h);
+
+// Launchers (return cudaSuccess or the launch error).
+cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
+cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s);
+cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
+cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s);
+
+}  // namespace qwam
+
+struct qwam_asp_handle_s {
+  qwam::Handle h;
+};

@@ -1,0 +1,135 @@
+// pack.cu -- offline packing of one ASP layer (Sec. 3.2 Eq. (asp) and the derivation of the
+// deflated weight W_perp = (I - U U^T) W; Eq. (quant) of Sec. 2 applied to W_perp per output
+// channel and group, App. B.1).  float64 on the device, untimed.
+//
+// Every float64 operation is an explicit IEEE intrinsic (__dmul_rn, __dadd_rn, ...) so that no
+// multiply-add is contracted: sums run in index order, each product and sum rounded once.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace qwam {
+namespace {
+
+// B_f[j, n] = sum_k U[k, j] W[k, n]  (k ascending), float64.
+__global__ void branch_weight_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U, int K, int N,
+                                     int r, double* __restrict__ Bf) {
+  int n = blockIdx.x * blockDim.x + threadIdx.x;
+  int j = blockIdx.y;
+  if (n >= N) return;
+  double acc = 0.0;
+  for (int k = 0; k < K; ++k) {
+    double u = static_cast<double>(U[static_cast<size_t>(k) * r + j]);
+    double w = static_cast<double>(__bfloat162float(W[static_cast<size_t>(k) * N + n]));
+    acc = __dadd_rn(acc, __dmul_rn(u, w));
+  }
+  Bf[static_cast<size_t>(j) * N + n] = acc;
+}
+
+// W_perp[k, n] = W[k, n] - sum_j U[k, j] B_f[j, n]  (j ascending).
+__device__ __forceinline__ double wperp(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+                                        const double* __restrict__ Bf, int N, int r, int k, int n) {
+  double acc = 0.0;
+  for (int j = 0; j < r; ++j)
+    acc = __dadd_rn(acc, __dmul_rn(static_cast<double>(U[static_cast<size_t>(k) * r + j]),
+                                   Bf[static_cast<size_t>(j) * N + n]));
+  return __dsub_rn(static_cast<double>(__bfloat162float(W[static_cast<size_t>(k) * N + n])), acc);
+}
+
+// Nearest integer to the exact quotient w / s, ties to even.  s is a float16 value and w a
+// float64 with |w| <= ~7.5 s, so c * s and w - c * s are exact in float64 and the remainder
+// decides the rounding.
+__device__ __forceinline__ int nearest_code_f64(double w, double s) {
+  double c = rint(__ddiv_rn(w, s));
+  double e = __dsub_rn(w, __dmul_rn(c, s));
+  double t = 2.0 * fabs(e);
+  bool odd = (static_cast<long long>(c) & 1LL) != 0;
+  if (t > s || (t == s && odd)) c = __dadd_rn(c, e > 0.0 ? 1.0 : -1.0);
+  return static_cast<int>(c);
+}
+
+// One thread per (output channel n, group g): s_w = RN_f16(absmax / 7), codes packed two per
+// byte (low nibble = even k) into qw[n, k/2].
+__global__ void quantize_weight_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+                                       const double* __restrict__ Bf, int K, int N, int r, int G, int N_pad,
+                                       uint8_t* __restrict__ qw, __half* __restrict__ sw, int* err) {
+  int n = blockIdx.x * blockDim.x + threadIdx.x;
+  int g = blockIdx.y;
+  if (n >= N) return;
+  double amax = 0.0;
+  for (int k = g * G; k < (g + 1) * G; ++k) amax = fmax(amax, fabs(wperp(W, U, Bf, N, r, k, n)));
+  __half sh = __double2half(__ddiv_rn(amax, 7.0));
+  double s = static_cast<double>(__half2float(sh));
+  sw[static_cast<size_t>(g) * N_pad + n] = sh;
+  bool ok_scale = isfinite(s);
+  if (!ok_scale) atomicOr(err, kErrRange);
+  uint8_t* row = qw + static_cast<size_t>(n) * (K / 2);
+  for (int k = g * G; k < (g + 1) * G; k += 2) {
+    int c0 = 0, c1 = 0;
+    if (s > 0.0 && ok_scale) {
+      c0 = nearest_code_f64(wperp(W, U, Bf, N, r, k, n), s);
+      c1 = nearest_code_f64(wperp(W, U, Bf, N, r, k + 1, n), s);
+    }
+    if (c0 < -7 || c0 > 7 || c1 < -7 || c1 > 7) atomicOr(err, kErrRange);
+    row[k / 2] = static_cast<uint8_t>((c0 & 0xF) | ((c1 & 0xF) << 4));
+  }
+}
+
+// B_hat[n, j] = RN_f16(B_f[j, n]), K-major for the branch MMA, zero beyond r.
+__global__ void branch_half_kernel(const double* __restrict__ Bf, int N, int r, int r_pad, __half* __restrict__ Bh,
+                                   int* err) {
+  int n = blockIdx.x * blockDim.x + threadIdx.x;
+  if (n >= N) return;
+  for (int j = 0; j < r_pad; ++j) {
+    __half v = __float2half(0.0f);
+    if (j < r) {
+      v = __double2half(Bf[static_cast<size_t>(j) * N + n]);
+      if (!isfinite(__half2float(v))) atomicOr(err, kErrRange);
+    }
+    Bh[static_cast<size_t>(n) * r_pad + j] = v;
+  }
+}
+
+// bf16 hi/lo split of U: hi = RN_bf16(u), lo = RN_bf16(u - hi).  Written twice: transposed
+// [2 r_pad, K] for the projection X U, and [K, ku3] as (hi, lo, hi) for the reconstruction.
+__global__ void split_basis_kernel(const float* __restrict__ U, int K, int r, int r_pad, int ku3,
+                                   __nv_bfloat16* __restrict__ ucat_t, __nv_bfloat16* __restrict__ ucat3) {
+  int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= K) return;
+  for (int j = 0; j < r_pad; ++j) {
+    float u = (j < r) ? U[static_cast<size_t>(k) * r + j] : 0.0f;
+    __nv_bfloat16 hi = __float2bfloat16_rn(u);
+    __nv_bfloat16 lo = __float2bfloat16_rn(u - __bfloat162float(hi));
+    ucat_t[static_cast<size_t>(j) * K + k] = hi;
+    ucat_t[static_cast<size_t>(r_pad + j) * K + k] = lo;
+    __nv_bfloat16* row = ucat3 + static_cast<size_t>(k) * ku3;
+    row[j] = hi;
+    row[r_pad + j] = lo;
+    row[2 * r_pad + j] = hi;
+  }
+  for (int j = 3 * r_pad; j < ku3; ++j) ucat3[static_cast<size_t>(k) * ku3 + j] = __float2bfloat16_rn(0.0f);
+}
+
+}  // namespace
+
+cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s) {
+  const int K = h.K, N = h.N, r = h.r;
+  double* Bf = nullptr;
+  cudaError_t e = cudaMalloc(&Bf, sizeof(double) * static_cast<size_t>(r > 0 ? r : 1) * N);
+  if (e != cudaSuccess) return e;
+  const int T = 128;
+  if (r > 0) {
+    branch_weight_kernel<<<dim3((N + T - 1) / T, r), T, 0, s>>>(W, U, K, N, r, Bf);
+  }
+  quantize_weight_kernel<<<dim3((N + T - 1) / T, K / h.G), T, 0, s>>>(W, U, Bf, K, N, r, h.G, h.N_pad, h.qw, h.sw,
+                                                                     h.err);
+  if (r > 0) {
+    branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
+    split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(U, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+  }
+  e = cudaGetLastError();
+  cudaError_t e2 = cudaStreamSynchronize(s);
+  cudaFree(Bf);
+  return e != cudaSuccess ? e : e2;
+}
+
+}  // namespace qwam

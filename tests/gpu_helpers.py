@@ -1,0 +1,99 @@
+"""Shared helpers of the GPU parity tests: seeded inputs on both sides, workspace read-back,
+nibble unpacking and the comparison rules."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2609_33269_gb300 import asp
+from paper_2609_33269_gb300 import workloads as wl
+
+
+def to_dev_bf16(bits: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).cuda().view(torch.bfloat16)
+
+
+def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
+    """uint8 [R, K/2] -> int8 [R, K] (low nibble = even k, two's complement)."""
+    p = np.ascontiguousarray(packed)
+    lo = (p & 0xF).astype(np.int16)
+    hi = (p >> 4).astype(np.int16)
+    out = np.empty((p.shape[0], p.shape[1] * 2), np.int16)
+    out[:, 0::2] = lo
+    out[:, 1::2] = hi
+    return ((out ^ 8) - 8).astype(np.int8)
+
+
+class Case:
+    """One layer on both sides: host inputs, the packed GPU layer, oracle outputs on demand."""
+
+    def __init__(self, M, K, N, r, G=64, seed=0, layer_id=0, dist="outlier", n_outlier=None):
+        self.M, self.K, self.N, self.r, self.G = M, K, N, r, G
+        self.Xb = wl.activations(M, K, seed=seed, layer_id=layer_id, dist=dist, n_outlier=n_outlier)
+        self.Wb = wl.weight(K, N, seed=seed, layer_id=layer_id)
+        self.U = wl.basis(K, r, seed=seed, layer_id=layer_id)
+        self.X = to_dev_bf16(self.Xb)
+        self.W = to_dev_bf16(self.Wb)
+        self.Ud = torch.from_numpy(self.U).cuda() if r > 0 else None
+        self.layer = asp.AspLinear(self.W, self.Ud, G)
+        self._ow = None
+
+    # oracle side
+    def oracle_weights(self):
+        if self._ow is None:
+            self._ow = oracle.pack(self.Wb, self.U, self.G)
+        return self._ow
+
+    def oracle_act(self, rows=None, want_float64=True):
+        Xb = self.Xb if rows is None else self.Xb[rows]
+        return oracle.quantize_act(Xb, self.U, self.G, want_float64=want_float64)
+
+    # GPU side
+    def gpu_weights(self):
+        e = asp.qwam_asp_export(self.layer.h)
+        return dict(qw=unpack_nibbles(e["qw"]), sw=e["sw"], Bh=e["Bh"][:, :self.r].T.copy(), Uhl=e["Uhl"])
+
+    def gpu_act(self, rows=None):
+        codes, scales, ph = self.layer.act_views(self.M)
+        torch.cuda.synchronize()
+        qx = unpack_nibbles(codes.cpu().numpy())
+        sx = scales.cpu().numpy()[:, :self.M].T.copy()
+        phv = ph.cpu().numpy().view(np.uint16)[:, :self.r].copy()
+        if rows is not None:
+            qx, sx, phv = qx[rows], sx[rows], phv[rows]
+        return dict(qx=qx, sx=sx, ph=phv)
+
+    def run(self, fp32=True):
+        Y = self.layer(self.X, fp32=fp32)
+        torch.cuda.synchronize()
+        return Y
+
+    def residual(self):
+        R = torch.empty((self.M, self.K), dtype=torch.float32, device="cuda")
+        ws = self.layer.workspace(self.M)
+        asp.qwam_asp_debug_residual(self.X, self.M, self.layer.h, ws, R)
+        torch.cuda.synchronize()
+        return R.cpu().numpy()
+
+    def close(self):
+        self.layer.close()
+
+
+def rowwise_rel_err(Y, ref):
+    """max |Y - ref| / max |ref| per row."""
+    d = np.abs(np.asarray(Y, np.float64) - ref).max(axis=1)
+    n = np.abs(ref).max(axis=1)
+    return d / np.maximum(n, 1e-30)
+
+
+def near_tie_mismatches(q_gpu, q_ref, x_ref, s_ref, G, eps_rel):
+    """Indices where the codes differ, and whether each lies within eps (relative to the scale)
+    of a rounding boundary of the reference remainder x_ref / s_ref."""
+    bad = np.argwhere(q_gpu != q_ref)
+    ok = []
+    for m, k in bad:
+        s = float(s_ref[m, k // G])
+        t = abs(float(x_ref[m, k]) / s) if s > 0 else 0.0
+        ok.append(abs((t - np.floor(t)) - 0.5) <= eps_rel)
+    return bad, np.array(ok, bool)

@@ -1,0 +1,62 @@
+"""The C-ABI library loads and exports every entry point the header declares; host-side argument
+validation answers without touching a GPU (no compute call runs here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "qwam_asp.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(qwam_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_33269_gb300 import build as b
+    from paper_2609_33269_gb300 import asp
+    b.build()
+    return asp.load()
+
+
+def test_header_declares_the_boundary():
+    fns = declared_functions()
+    for name in ("qwam_asp_pack_weights", "qwam_asp_quantize_act", "qwam_asp_linear", "qwam_asp_gemm",
+                 "qwam_asp_act_workspace_bytes", "qwam_asp_get_error", "qwam_asp_export", "qwam_asp_destroy"):
+        assert name in fns
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    from paper_2609_33269_gb300 import asp
+    assert set(asp.EXPORTED) >= set(declared_functions())
+
+
+def test_host_validation_rejects_bad_arguments_without_a_launch(lib):
+    from paper_2609_33269_gb300 import asp
+    h = ctypes.c_void_p()
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+    V = ctypes.c_void_p
+    # NULL output handle
+    assert lib.qwam_asp_pack_weights(fake, None, 64, 64, 0, 64, None, None) == asp.QWAM_ERR_INVALID_ARG
+    # K not a multiple of 64, N not a multiple of 8, group not 32/64, r > K, r > 0 with NULL U
+    for K, N, r, G, U in ((100, 64, 0, 64, None), (64, 60, 0, 64, None), (64, 64, 0, 48, None),
+                          (64, 64, 65, 64, fake), (64, 64, 4, 64, None)):
+        st = lib.qwam_asp_pack_weights(fake, U, K, N, r, G, None, ctypes.byref(h))
+        assert st == asp.QWAM_ERR_INVALID_ARG, (K, N, r, G)
+    # misaligned W
+    assert lib.qwam_asp_pack_weights(V((1 << 20) + 2), None, 64, 64, 0, 64, None,
+                                     ctypes.byref(h)) == asp.QWAM_ERR_INVALID_ARG
+    # rank above this build's maximum (valid per the paper) is reported as unsupported
+    assert lib.qwam_asp_pack_weights(fake, fake, 256, 64, 65, 64, None, ctypes.byref(h)) == asp.QWAM_ERR_UNSUPPORTED
+    size = ctypes.c_size_t()
+    assert lib.qwam_asp_act_workspace_bytes(None, 4, ctypes.byref(size)) == asp.QWAM_ERR_INVALID_ARG
+    assert lib.qwam_asp_linear(None, 4, None, None, 0, None, None) == asp.QWAM_ERR_INVALID_ARG
+    assert lib.qwam_asp_get_error(None) == asp.QWAM_ERR_INVALID_ARG
+    assert asp.status_string(asp.QWAM_ERR_TIMEOUT) == "device wait timed out"
