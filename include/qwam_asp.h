@@ -74,12 +74,17 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
 qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes);
 
 /* Layout of the activation workspace for M tokens (byte offsets from its start):
- *   codes  : uint8 [M, K/2], two 4-bit two's-complement codes per byte, low nibble = even k
+ *   codes  : uint8 [M, K], one byte per activation code c in [-7, 7]: the E4M3 bit pattern of
+ *            c * 2^-9, i.e. (c < 0 ? 0x80 : 0) | |c| (an E4M3 subnormal; the GEMM's tensor cores
+ *            read these bytes as they are)
  *   scales : float32 [K/group, M_pad] (M_pad = M rounded up to 128), s_x of token m, group g
  *            at [g * M_pad + m]
- *   p_hat  : float16 [M, r_pad] (r_pad = r rounded up to 16; columns >= r are zero) */
+ *   csums  : float32 [K/group, M_pad], the sum of the group's codes (an exact integer)
+ *   p_hat  : float16 [M, r_pad] (r_pad = r rounded up to 16; columns >= r are zero)
+ * The workspace is transient (written by qwam_asp_quantize_act, read by qwam_asp_gemm); the
+ * weights are the part of the layer that stays packed at 4 bits. */
 qwam_status qwam_asp_act_layout(qwam_asp_handle h, int M, size_t* codes_off, size_t* scales_off,
-                                size_t* phat_off, int* M_pad, int* r_pad);
+                                size_t* csums_off, size_t* phat_off, int* M_pad, int* r_pad);
 
 /* Kernel (a): Eq. (xsplit) and the run-time half of Eq. (quant), one launch, asynchronous.
  *   X_bf16 : device, bf16 [M, K] row-major;  act_ws : device workspace (see above), written
@@ -91,10 +96,10 @@ qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, 
 /* Kernel (b): the 4-bit GEMM with the low-rank branch in its epilogue, asynchronous.
  *   act_ws : device workspace filled by qwam_asp_quantize_act for the same M
  *   Y      : device [M, N] row-major, bf16 (y_dtype QWAM_Y_BF16) or float32 (QWAM_Y_FP32)
- * Per group g the tensor cores form the exact integer partial sums P_g = sum_k qx qw (codes
- * expanded to E4M3, which holds every integer in [-7, 7] exactly; float32 accumulation of
- * integers below 2^12 is exact); the epilogue adds s_x[m,g] s_w[g,n] P_g in float32 and, last,
- * the branch p_hat B_hat (float16 operands, float32 accumulation). */
+ * Per group g the tensor cores form the exact integer partial sums P_g = sum_k qx qw (codes fed
+ * as E4M3 multiples of 2^-9, which E4M3 holds exactly; float32 accumulation of these integer
+ * multiples of 2^-18 below 2^-5 is exact); the epilogue adds s_x[m,g] s_w[g,n] P_g in float32
+ * and, last, the branch p_hat B_hat (float16 operands, float32 accumulation). */
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle h, void* Y, int y_dtype,
                           struct CUstream_st* stream);
 

@@ -59,7 +59,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_pack_weights.argtypes = [V, V, I, I, I, I, V, ctypes.POINTER(H)]
         lib.qwam_asp_act_workspace_bytes.argtypes = [H, I, ctypes.POINTER(S)]
         lib.qwam_asp_act_layout.argtypes = [H, I, ctypes.POINTER(S), ctypes.POINTER(S), ctypes.POINTER(S),
-                                            ctypes.POINTER(I), ctypes.POINTER(I)]
+                                            ctypes.POINTER(S), ctypes.POINTER(I), ctypes.POINTER(I)]
         lib.qwam_asp_quantize_act.argtypes = [V, I, H, V, V]
         lib.qwam_asp_gemm.argtypes = [V, I, H, V, I, V]
         lib.qwam_asp_linear.argtypes = [V, I, H, V, I, V, V]
@@ -117,11 +117,12 @@ def qwam_asp_act_workspace_bytes(h: int, M: int) -> int:
 
 
 def qwam_asp_act_layout(h: int, M: int) -> dict:
-    c, s, p = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t()
+    c, s, cs, p = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t()
     mp, rp = ctypes.c_int(), ctypes.c_int()
-    _check(load().qwam_asp_act_layout(h, M, ctypes.byref(c), ctypes.byref(s), ctypes.byref(p),
+    _check(load().qwam_asp_act_layout(h, M, ctypes.byref(c), ctypes.byref(s), ctypes.byref(cs), ctypes.byref(p),
                                       ctypes.byref(mp), ctypes.byref(rp)), "qwam_asp_act_layout")
-    return dict(codes_off=c.value, scales_off=s.value, phat_off=p.value, M_pad=mp.value, r_pad=rp.value)
+    return dict(codes_off=c.value, scales_off=s.value, csums_off=cs.value, phat_off=p.value, M_pad=mp.value,
+                r_pad=rp.value)
 
 
 def qwam_asp_quantize_act(X_bf16, M: int, h: int, act_ws, stream=None):
@@ -204,15 +205,16 @@ class AspLinear:
         return self._ws
 
     def act_views(self, M: int, ws: torch.Tensor | None = None):
-        """Views of the workspace for M tokens: codes uint8 [M, K/2], scales f32 [K/G, M_pad],
-        p_hat f16 [M, r_pad]."""
+        """Views of the workspace for M tokens: code bytes uint8 [M, K] (E4M3 of c * 2^-9),
+        scales f32 [K/G, M_pad], code sums f32 [K/G, M_pad], p_hat f16 [M, r_pad]."""
         ws = self.workspace(M) if ws is None else ws
         L = qwam_asp_act_layout(self.h, M)
-        codes = ws[L["codes_off"]:L["codes_off"] + M * self.K // 2].view(M, self.K // 2)
+        codes = ws[L["codes_off"]:L["codes_off"] + M * self.K].view(M, self.K)
         ns = self.K // self.group
         scales = ws[L["scales_off"]:L["scales_off"] + ns * L["M_pad"] * 4].view(torch.float32).view(ns, L["M_pad"])
+        csums = ws[L["csums_off"]:L["csums_off"] + ns * L["M_pad"] * 4].view(torch.float32).view(ns, L["M_pad"])
         ph = ws[L["phat_off"]:L["phat_off"] + M * self.r_pad * 2].view(torch.float16).view(M, self.r_pad)
-        return codes, scales, ph
+        return codes, scales, csums, ph
 
     def quantize(self, X: torch.Tensor, stream=None) -> torch.Tensor:
         M = X.shape[0]

@@ -12,11 +12,18 @@
 // tensor-core MMA, float32 accumulation); the partial projections are summed across the
 // cluster through distributed shared memory (fixed order, so every CTA sees the same p);
 // pass 2 re-reads the slice (L2-resident by then) while the tensor cores form
-// R = [p_hi | p_hi | p_lo] [U_hi | U_lo | U_hi]^T, and the epilogue warps form X_perp = X - R
-// in float32 and quantize it.  With r = 0 the kernel is a single streaming pass (no MMA).
+// R = [p_hi | p_hi | p_lo] [U_hi | U_lo | U_hi]^T chunk by chunk, and the epilogue warps form
+// X_perp = X - R in float32 and quantize it.  With r = 0 the kernel is one streaming pass.
 //
-// Warp roles (192 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner,
-// warps 2..5 epilogue (thread = token row).
+// Outputs per token row m and group g (the activation workspace):
+//   codes[m, k]   one byte per code, E4M3 bit pattern of c * 2^-9 (sign | magnitude, a
+//                 subnormal): the GEMM feeds these bytes to the tensor cores unchanged;
+//   s_x[g, m]     float32 scale;   csum[g, m]  float32 sum of the group's codes (exact);
+//   p_hat[m, :]   float16.
+//
+// Warp roles (320 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2..9
+// epilogue: warps 2..5 and 6..9 each cover the four 32-row TMEM quadrants and take the even
+// and the odd K chunks respectively.
 #include <algorithm>
 
 #include "internal.h"
@@ -27,13 +34,16 @@ namespace {
 
 struct ActArgs {
   int M, K, G, C, Kc, M_pad;
-  uint8_t* codes;   // [M, K/2]
+  uint8_t* codes;   // [M, K]
   float* scales;    // [K/G, M_pad]
+  float* csums;     // [K/G, M_pad]
   __half* phat;     // [M, RP]
   float* dump;      // optional [M, K]
   int* err;
   uint64_t timeout_ns;
 };
+
+constexpr int kNumRec = 4;  // TMEM reconstruction buffers (64 columns each)
 
 template <int RP>
 struct ActCfg {
@@ -43,49 +53,61 @@ struct ActCfg {
   static constexpr int U2_BYTES = kChunk * KU3 * 2;                    // Ucat3 chunk, KU3/64 atoms
   static constexpr int U_BYTES = U1_BYTES > U2_BYTES ? U1_BYTES : U2_BYTES;
   static constexpr int STAGE = X_BYTES + U_BYTES;
-  static constexpr int S = RP == 0 ? 6 : (RP <= 32 ? 4 : 2);
+  static constexpr int S = RP == 0 ? 8 : (RP <= 32 ? 4 : (RP <= 48 ? 3 : 2));
   static constexpr int AREC_BYTES = kBM * KU3 * 2;
   static constexpr int PP_BYTES = kBM * RP * 4;
-  static constexpr int NBAR = 2 * S + 7;
+  static constexpr int NBAR = 2 * S + 3 + 2 * kNumRec;
   static constexpr int SMEM = 1024 + S * STAGE + AREC_BYTES + 2 * PP_BYTES + NBAR * 8 + 16;
-  static constexpr uint32_t TMEM_COLS = 256;  // proj at col 0 (2*RP <= 128), rec buffers at 128, 192
+  static constexpr uint32_t TMEM_COLS = 512;  // proj at col 0 (2*RP <= 128), rec buffers at 128 + 64 b
+  static_assert(SMEM <= 232448, "kernel (a) shared memory above the 227 KB per-CTA limit");
 };
 
-__device__ __forceinline__ int nearest_code_f32(float x, float s, float inv) {
-  // Nearest integer to the exact quotient x / s, ties to even.  c is within one of it; the
-  // remainder x - c s is exact in float32 (see the design notes), so it decides exactly.
-  float c = rintf(x * inv);
-  float e = fmaf(-c, s, x);
-  float t = 2.0f * fabsf(e);
-  int ci = static_cast<int>(c);
-  if (t > s || (t == s && (ci & 1))) ci += (e > 0.0f) ? 1 : -1;
+constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23: adding it rounds to an integer (ties to even)
+constexpr int kMagicBits = 0x4B400000;
+
+// Nearest integer to the exact quotient x / s, ties to even (s > 0, |x| <= ~7.5 s).
+// c = rint(x * (1/s)) is the answer or its neighbour; the remainder e = x - c s is exact in
+// float32 (c and the true answer differ by at most one), and |e| < s/2 exactly when c is right
+// and not a tie, so only |e| >= s/2 (rare) needs the exact decision.
+__device__ __forceinline__ int nearest_code(float x, float s, float inv, float hs) {
+  const float t = fmaf(x, inv, kMagic);
+  const float c = t - kMagic;
+  const float e = fmaf(-c, s, x);
+  int ci = __float_as_int(t) - kMagicBits;
+  if (fabsf(e) >= hs) {
+    const float te = 2.0f * fabsf(e);
+    if (te > s || (te == s && (ci & 1))) ci += (e > 0.0f) ? 1 : -1;
+  }
   return ci;
 }
 
-// One group of GS remainder values: s = RN_f32(absmax / 7) (IEEE division), codes packed two
-// per byte, low nibble first.
+// One group of GS remainder values -> scale, code sum and GS code bytes (E4M3 of c * 2^-9).
 template <int GS>
-__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* packed, float* scale_out) {
+__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4, float* scale_out, float* csum_out) {
   float amax = 0.0f;
 #pragma unroll
   for (int i = 0; i < GS; ++i) amax = fmaxf(amax, fabsf(xp[i]));
   const float sc = __fdiv_rn(amax, 7.0f);
   const float inv = sc > 0.0f ? __frcp_rn(sc) : 0.0f;
-  *scale_out = sc;
+  const float hs = 0.5f * sc;
+  int sum = 0;
 #pragma unroll
-  for (int w8 = 0; w8 < GS / 8; ++w8) {
-    uint32_t word = 0;
+  for (int w = 0; w < GS / 4; ++w) {
+    uint32_t b[4];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int ci = nearest_code_f32(xp[8 * w8 + u], sc, inv);
-      word |= (static_cast<uint32_t>(ci) & 0xFu) << (4 * u);
+    for (int u = 0; u < 4; ++u) {
+      const int ci = nearest_code(xp[4 * w + u], sc, inv, hs);
+      sum += ci;
+      b[u] = static_cast<uint32_t>(abs(ci)) | (static_cast<uint32_t>(ci) & 0x80u);
     }
-    packed[w8] = word;
+    bytes4[w] = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
   }
+  *scale_out = sc;
+  *csum_out = static_cast<float>(sum);
 }
 
 template <int RP>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
     actquant_kernel(const __grid_constant__ CUtensorMap x_map, const __grid_constant__ CUtensorMap ut_map,
                     const __grid_constant__ CUtensorMap u3_map, const ActArgs a) {
   using Cfg = ActCfg<RP>;
@@ -101,9 +123,9 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* empty = bars + S;
   uint64_t* proj_done = bars + 2 * S;
   uint64_t* arec_ready = proj_done + 1;
-  uint64_t* tfull = proj_done + 2;
-  uint64_t* tempty = proj_done + 4;
-  uint64_t* drain = proj_done + 6;
+  uint64_t* drain = proj_done + 2;
+  uint64_t* tfull = proj_done + 3;
+  uint64_t* tempty = tfull + kNumRec;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + Cfg::NBAR);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
@@ -122,12 +144,12 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&empty[i], 1);
     }
     mbar_init(proj_done, 1);
-    mbar_init(arec_ready, 128);
-    for (int i = 0; i < 2; ++i) {
+    mbar_init(arec_ready, 256);
+    mbar_init(drain, 1);
+    for (int i = 0; i < kNumRec; ++i) {
       mbar_init(&tfull[i], 1);
       mbar_init(&tempty[i], 128);
     }
-    mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -179,7 +201,7 @@ __global__ void __launch_bounds__(192, 1)
       // Let every load issued into the ring land before the CTA can exit.
       int never = 0;
       const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-      for (int j = std::max(0, it - S); j < it; ++j) mbar_wait(&full[j % S], (j / S) & 1, dc);
+      for (int j = (it > S ? it - S : 0); j < it; ++j) mbar_wait(&full[j % S], (j / S) & 1, dc);
     }
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
@@ -211,9 +233,9 @@ __global__ void __launch_bounds__(192, 1)
         constexpr uint32_t idesc_rec = idesc_bf16(kBM, kChunk);
         const uint32_t ar = smem_u32(arec);
         for (int c = 0; c < nch && ok; ++c) {
-          const int it = pass1 + c, s = it % S, b = c & 1;
+          const int it = pass1 + c, s = it % S, b = c % kNumRec;
           ok = mbar_wait(&full[s], (it / S) & 1, wc);
-          if (ok && c >= 2) ok = mbar_wait(&tempty[b], ((c >> 1) & 1) ^ 1, wc);
+          if (ok && c >= kNumRec) ok = mbar_wait(&tempty[b], ((c / kNumRec) & 1) ^ 1, wc);
           if (!ok) break;
           tc_fence_after();
           const uint32_t ua = smem_u32(stage_u(s));
@@ -236,35 +258,46 @@ __global__ void __launch_bounds__(192, 1)
   } else {
     // ------------------------------------------------------------- epilogue (thread = row)
     const int quad = wid & 3;
+    const int par = (static_cast<int>(wid) - 2) >> 2;  // 0: even chunks, 1: odd chunks
     const int row = quad * 32 + static_cast<int>(lane);
     const int m = m0 + row;
-    const int et = static_cast<int>(wid - 2) * 32 + static_cast<int>(lane);
+    const int et = static_cast<int>(wid - 2) * 32 + static_cast<int>(lane);  // 0..255
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     bool ok = true;
 
     if constexpr (RP > 0) {
-      // -- partial projection of this CTA's K slice: hi part + lo part
+      constexpr int HR = RP / 2;  // projection columns handled by this thread (half of them)
+      const int j0 = par * HR;
+      // -- partial projection of this CTA's K slice: hi part + lo part, columns [j0, j0 + HR)
       ok = mbar_wait(proj_done, 0, wc);
       tc_fence_after();
-      float pp[RP];
+      float pp[HR];
 #pragma unroll
-      for (int q = 0; q < RP / 16; ++q) {
-        uint32_t vh[16], vl[16];
-        tmem_ld16(tlane + q * 16, vh);
-        tmem_ld16(tlane + RP + q * 16, vl);
+      for (int q = 0; q < HR / 8; ++q) {
+        uint32_t vh[8], vl[8];
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+            : "=r"(vh[0]), "=r"(vh[1]), "=r"(vh[2]), "=r"(vh[3]), "=r"(vh[4]), "=r"(vh[5]), "=r"(vh[6]), "=r"(vh[7])
+            : "r"(tlane + j0 + q * 8)
+            : "memory");
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+            : "=r"(vl[0]), "=r"(vl[1]), "=r"(vl[2]), "=r"(vl[3]), "=r"(vl[4]), "=r"(vl[5]), "=r"(vl[6]), "=r"(vl[7])
+            : "r"(tlane + RP + j0 + q * 8)
+            : "memory");
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 16; ++i) pp[q * 16 + i] = __uint_as_float(vh[i]) + __uint_as_float(vl[i]);
+        for (int i = 0; i < 8; ++i) pp[q * 8 + i] = __uint_as_float(vh[i]) + __uint_as_float(vl[i]);
       }
-      float4* prow = reinterpret_cast<float4*>(ppart + row * RP);
+      float4* prow = reinterpret_cast<float4*>(ppart + row * RP + j0);
 #pragma unroll
-      for (int j = 0; j < RP / 4; ++j) prow[j] = make_float4(pp[4 * j], pp[4 * j + 1], pp[4 * j + 2], pp[4 * j + 3]);
+      for (int j = 0; j < HR / 4; ++j) prow[j] = make_float4(pp[4 * j], pp[4 * j + 1], pp[4 * j + 2], pp[4 * j + 3]);
       cluster_sync();  // A: every CTA's partial is in its shared memory
       // -- reduce-scatter: this CTA sums rows [rank*Rc, (rank+1)*Rc) over the cluster, in rank order
       const int Rc = kBM / C;
       const int n4 = Rc * RP / 4;
       const uint32_t pp_base = smem_u32(ppart);
-      for (int i = et; i < n4; i += 128) {
+      for (int i = et; i < n4; i += 256) {
         const uint32_t off = static_cast<uint32_t>((static_cast<int>(rank) * Rc * RP + 4 * i) * 4);
         float4 acc = ld_dsmem_f4(mapa_smem(pp_base + off, 0));
         for (int q = 1; q < C; ++q) {
@@ -286,13 +319,13 @@ __global__ void __launch_bounds__(192, 1)
         }
       }
       cluster_sync();  // B: the reduced rows are in their owners' shared memory
-      // -- gather this thread's row of p from its owner
+      // -- gather this thread's half row of p from its owner
       const int owner = row / Rc, lr = row % Rc;
       const uint32_t pr_base = smem_u32(pred);
-      float p[RP];
+      float p[HR];
 #pragma unroll
-      for (int j = 0; j < RP / 4; ++j) {
-        const float4 v = ld_dsmem_f4(mapa_smem(pr_base + static_cast<uint32_t>((lr * RP + 4 * j) * 4),
+      for (int j = 0; j < HR / 4; ++j) {
+        const float4 v = ld_dsmem_f4(mapa_smem(pr_base + static_cast<uint32_t>((lr * RP + j0 + 4 * j) * 4),
                                                static_cast<uint32_t>(owner)));
         p[4 * j] = v.x;
         p[4 * j + 1] = v.y;
@@ -300,46 +333,45 @@ __global__ void __launch_bounds__(192, 1)
         p[4 * j + 3] = v.w;
       }
       cluster_sync();  // C: no CTA reads a peer's shared memory after this point
-      // -- A operand of the reconstruction: [p_hi | p_hi | p_lo | 0], 128-byte swizzle
-      __nv_bfloat16 hi[RP], lo[RP];
+      // -- A operand of the reconstruction: [p_hi | p_hi | p_lo | 0], 128-byte swizzle.
+      //    This thread writes its columns j0..j0+HR-1 of each segment (8 bf16 = one 16-byte chunk).
+      __nv_bfloat16 hi[HR], lo[HR];
 #pragma unroll
-      for (int j = 0; j < RP; ++j) {
+      for (int j = 0; j < HR; ++j) {
         hi[j] = __float2bfloat16_rn(p[j]);
         lo[j] = __float2bfloat16_rn(p[j] - __bfloat162float(hi[j]));
       }
-#pragma unroll
-      for (int c8 = 0; c8 < Cfg::KU3 / 8; ++c8) {  // 16-byte chunk of 8 bf16
+      auto put8 = [&](int col, const __nv_bfloat16* v) {  // col: multiple of 8
         uint32_t w[4];
 #pragma unroll
-        for (int t = 0; t < 4; ++t) {
-          __nv_bfloat16 e2[2];
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const int col = c8 * 8 + 2 * t + u;
-            e2[u] = col < RP ? hi[col % RP]
-                    : col < 2 * RP ? hi[col % RP]
-                    : col < 3 * RP ? lo[col % RP]
-                                   : __float2bfloat16_rn(0.0f);
-          }
-          w[t] = static_cast<uint32_t>(*reinterpret_cast<uint16_t*>(&e2[0])) |
-                 (static_cast<uint32_t>(*reinterpret_cast<uint16_t*>(&e2[1])) << 16);
-        }
-        const int q = c8 >> 3, j = c8 & 7;
+        for (int t = 0; t < 4; ++t)
+          w[t] = static_cast<uint32_t>(__bfloat16_as_ushort(v[2 * t])) |
+                 (static_cast<uint32_t>(__bfloat16_as_ushort(v[2 * t + 1])) << 16);
+        const int q = col >> 6, j = (col & 63) >> 3;
         *reinterpret_cast<uint4*>(arec + q * 16384 + row * 128 + ((j ^ (row & 7)) << 4)) =
             make_uint4(w[0], w[1], w[2], w[3]);
+      };
+#pragma unroll
+      for (int c8 = 0; c8 < HR / 8; ++c8) {
+        put8(j0 + 8 * c8, hi + 8 * c8);
+        put8(RP + j0 + 8 * c8, hi + 8 * c8);
+        put8(2 * RP + j0 + 8 * c8, lo + 8 * c8);
+      }
+      if (par == 1) {  // zero padding columns [3 RP, KU3)
+        const __nv_bfloat16 z[8] = {};
+        for (int col = 3 * RP; col < Cfg::KU3; col += 8) put8(col, z);
       }
       fence_proxy_async_smem();
       mbar_arrive(arec_ready);
     }
 
-    // -- pass 2: remainder and quantization, one 64-column chunk at a time
-    const int half_k = a.K / 2;
-    for (int c = 0; c < nch; ++c) {
+    // -- pass 2: remainder and quantization; this warp takes the chunks of its parity
+    for (int c = par; c < nch; c += 2) {
       const int it = pass1 + c, s = it % S;
       float xp[kChunk];
       if constexpr (RP > 0) {
-        const int b = c & 1;
-        if (ok) ok = mbar_wait(&tfull[b], (c >> 1) & 1, wc);
+        const int b = c % kNumRec;
+        if (ok) ok = mbar_wait(&tfull[b], (c / kNumRec) & 1, wc);
         tc_fence_after();
         uint32_t r0[32], r1[32];
         tmem_ld32(tlane + 128 + 64 * b, r0);
@@ -370,8 +402,11 @@ __global__ void __launch_bounds__(192, 1)
           xp[8 * j + 2 * t + 1] = hi_f - xp[8 * j + 2 * t + 1];
         }
       }
-      named_bar_sync(1, 128);
-      if (et == 0) mbar_arrive(&empty[s]);
+      // The stage goes back to the TMA producer: order these generic-proxy reads before the
+      // async-proxy write that will refill it, then release it once all 128 readers are done.
+      fence_proxy_async_smem();
+      named_bar_sync(1 + par, 128);
+      if (et == par * 128) mbar_arrive(&empty[s]);
       if (!ok || m >= a.M) continue;
 
       const int kc = k0 + c * kChunk;
@@ -380,19 +415,18 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
         for (int i = 0; i < kChunk / 4; ++i) d[i] = make_float4(xp[4 * i], xp[4 * i + 1], xp[4 * i + 2], xp[4 * i + 3]);
       }
-      uint32_t packed[8];
+      uint32_t bytes4[16];
       if (a.G == 64) {
-        quantize_group<64>(xp, packed, a.scales + static_cast<size_t>(kc / 64) * a.M_pad + m);
+        const size_t gi = static_cast<size_t>(kc / 64) * a.M_pad + m;
+        quantize_group<64>(xp, bytes4, a.scales + gi, a.csums + gi);
       } else {
-        quantize_group<32>(xp, packed, a.scales + static_cast<size_t>(kc / 32) * a.M_pad + m);
-        quantize_group<32>(xp + 32, packed + 4, a.scales + static_cast<size_t>(kc / 32 + 1) * a.M_pad + m);
+        const size_t gi = static_cast<size_t>(kc / 32) * a.M_pad + m;
+        quantize_group<32>(xp, bytes4, a.scales + gi, a.csums + gi);
+        quantize_group<32>(xp + 32, bytes4 + 8, a.scales + gi + a.M_pad, a.csums + gi + a.M_pad);
       }
-      uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * half_k + kc / 2);
-      dst[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
-      dst[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
-    }
-    if constexpr (RP == 0) {
-      (void)tlane;
+      uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * a.K + kc);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) dst[i] = make_uint4(bytes4[4 * i], bytes4[4 * i + 1], bytes4[4 * i + 2], bytes4[4 * i + 3]);
     }
   }
 
@@ -403,6 +437,15 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
+// Cluster size (CTAs along K per 128-row tile): as many as fit one wave of the GPU.
+int choose_split(int K, int tiles, int sms) {
+  const int chunks = K / kChunk;
+  int C = 1;
+  while (C < 8 && chunks % (2 * C) == 0 && tiles * 2 * C <= sms) C *= 2;
+  if (C == 1 && chunks % 2 == 0 && tiles < sms) C = 2;
+  return C;
+}
+
 template <int RP>
 cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
   using Cfg = ActCfg<RP>;
@@ -411,16 +454,15 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   a.M = M;
   a.K = h.K;
   a.G = h.G;
-  const int chunks = h.K / kChunk;
   const int tiles = (M + kBM - 1) / kBM;
-  int C = 1;
-  while (C < 8 && chunks % (2 * C) == 0 && tiles * C < 2 * 152) C *= 2;
+  const int C = choose_split(h.K, tiles, h.num_sms);
   a.C = C;
   a.Kc = h.K / C;
   a.M_pad = L.M_pad;
   uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
   a.codes = base + L.codes_off;
   a.scales = reinterpret_cast<float*>(base + L.scales_off);
+  a.csums = reinterpret_cast<float*>(base + L.csums_off);
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
   a.dump = dump;
   a.err = h.err;
@@ -434,7 +476,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(C, tiles, 1);
-  cfg.blockDim = dim3(192, 1, 1);
+  cfg.blockDim = dim3(320, 1, 1);
   cfg.dynamicSmemBytes = Cfg::SMEM;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];

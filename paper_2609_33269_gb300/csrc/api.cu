@@ -68,8 +68,9 @@ ActLayout act_layout(const Handle& h, int M) {
   ActLayout L;
   L.M_pad = round_up(M > 0 ? M : 1, kBM);
   L.codes_off = 0;
-  L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
-  L.phat_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
+  L.scales_off = up256(static_cast<size_t>(M) * h.K);
+  L.csums_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
+  L.phat_off = L.csums_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
   L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
   return L;
 }
@@ -89,9 +90,11 @@ const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
     ok &= encode_2d(&c.x_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, h.K, M, static_cast<uint64_t>(h.K) * 2, kChunk, kBM,
                     CU_TENSOR_MAP_SWIZZLE_128B);
   }
-  ok &= encode_2d(&c.qx_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, kGemmKS / 2, kBM,
-                  CU_TENSOR_MAP_SWIZZLE_NONE);
+  ok &= encode_2d(&c.qx_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K, M, h.K, kGemmKS, kBM,
+                  CU_TENSOR_MAP_SWIZZLE_128B);
   ok &= encode_2d(&c.sx_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.scales_off, M, h.K / h.G,
+                  static_cast<uint64_t>(L.M_pad) * 4, kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
+  ok &= encode_2d(&c.cs_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.csums_off, M, h.K / h.G,
                   static_cast<uint64_t>(L.M_pad) * 4, kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
   if (h.r_pad > 0)
     ok &= encode_2d(&c.ph_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
@@ -152,6 +155,7 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   h.N_pad = qwam::round_up(N, qwam::kGemmBN);
   h.ku3 = h.r_pad == 0 ? 0 : qwam::round_up(3 * h.r_pad, 64);
   cudaGetDevice(&h.device);
+  cudaDeviceGetAttribute(&h.num_sms, cudaDevAttrMultiProcessorCount, h.device);
 
   const size_t b_qw = qwam::up256(static_cast<size_t>(h.N_pad) * (K / 2));
   const size_t b_sw = qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
@@ -212,12 +216,13 @@ qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle hs, int M, size_t* byte
   return QWAM_OK;
 }
 
-qwam_status qwam_asp_act_layout(qwam_asp_handle hs, int M, size_t* codes_off, size_t* scales_off, size_t* phat_off,
-                                int* M_pad, int* r_pad) {
+qwam_status qwam_asp_act_layout(qwam_asp_handle hs, int M, size_t* codes_off, size_t* scales_off,
+                                size_t* csums_off, size_t* phat_off, int* M_pad, int* r_pad) {
   if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
   const qwam::ActLayout L = qwam::act_layout(hs->h, M);
   if (codes_off) *codes_off = L.codes_off;
   if (scales_off) *scales_off = L.scales_off;
+  if (csums_off) *csums_off = L.csums_off;
   if (phat_off) *phat_off = L.phat_off;
   if (M_pad) *M_pad = L.M_pad;
   if (r_pad) *r_pad = hs->h.r_pad;
@@ -295,7 +300,20 @@ qwam_status qwam_asp_export(qwam_asp_handle hs, void* qw, void* sw, void* Bh, vo
   Handle& h = hs->h;
   if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
   cudaError_t e = cudaSuccess;
-  if (qw) e = cudaMemcpy(qw, h.qw, static_cast<size_t>(h.N) * (h.K / 2), cudaMemcpyDeviceToHost);
+  if (qw) {
+    // device words hold k = 8j..8j+3 in low and 8j+4..8j+7 in high nibbles; export pairs (2q, 2q+1)
+    std::vector<uint8_t> t(static_cast<size_t>(h.N) * (h.K / 2));
+    e = cudaMemcpy(t.data(), h.qw, t.size(), cudaMemcpyDeviceToHost);
+    uint8_t* o = static_cast<uint8_t*>(qw);
+    for (size_t wd = 0; e == cudaSuccess && wd < t.size() / 4; ++wd) {
+      uint8_t c[8];
+      for (int i = 0; i < 4; ++i) {
+        c[i] = t[4 * wd + i] & 0xF;
+        c[4 + i] = t[4 * wd + i] >> 4;
+      }
+      for (int q = 0; q < 4; ++q) o[4 * wd + q] = static_cast<uint8_t>(c[2 * q] | (c[2 * q + 1] << 4));
+    }
+  }
   if (e == cudaSuccess && sw)
     e = cudaMemcpy2D(sw, static_cast<size_t>(h.N) * 2, h.sw, static_cast<size_t>(h.N_pad) * 2,
                      static_cast<size_t>(h.N) * 2, h.K / h.G, cudaMemcpyDeviceToHost);

@@ -5,18 +5,22 @@
 //   Y[m, n] = sum_g s_x[m, g] s_w[g, n] P_g[m, n]  +  sum_j p_hat[m, j] B_hat[n, j]
 //   P_g[m, n] = sum_{k in group g} q_x[m, k] q_w[n, k]          (exact integers)
 //
-// sm_103a has no integer tensor-core MMA, so the 4-bit codes (always in [-7, 7]) are expanded to
-// E4M3, which represents every integer in [-16, 16] exactly, and multiplied with
-// tcgen05.mma.kind::f8f6f4 into float32 TMEM accumulators.  Every product is an integer of
-// magnitude <= 49 and every per-group sum is below 2^12, so the float32 accumulator holds the
-// same integer an int32 accumulator would.  Each group gets its own accumulator (two TMEM
-// buffers, double-buffered); the epilogue warps apply s_x * s_w in float32 and accumulate in
-// registers.  After the last group, one kind::f16 MMA of K = r_pad forms p_hat B_hat^T into a
-// TMEM buffer that the epilogue adds with scale 1.
+// sm_103a has no integer tensor-core MMA, so the codes are fed to tcgen05.mma.kind::f8f6f4 as
+// E4M3 bit patterns of exact multiples of 2^-9 (E4M3 subnormals, which the tensor core keeps):
+//   A: activation byte = sign | |c|      -> value c * 2^-9     (written so by kernel (a))
+//   B: weight byte     = c + 8 in [1,15] -> value (c + 8) 2^-9 (expanded here from 4 bits)
+// so one group's float32 accumulator holds D = 2^-18 sum_k c_a (c_b + 8) = 2^-18 (P + 8 S_a)
+// exactly (S_a = the activation group's code sum, every partial sum an integer below 2^13 times
+// 2^-18).  The epilogue forms s_x P = alpha D + beta with alpha = 2^18 s_x, beta = -8 s_x S_a
+// (per row and group) and accumulates s_w * (s_x P) in float32 registers.  The 4-bit weights
+// stay packed in HBM; a nibble becomes its byte with three logic ops per eight nibbles because
+// the packing puts the codes of k = 8j..8j+3 in the low and of k = 8j+4..8j+7 in the high
+// nibbles of the four bytes of word j.  Each group has its own TMEM accumulator (four buffers);
+// after the last group one kind::f16 MMA of K = r_pad forms p_hat B_hat^T, added with scale 1.
 //
-// CTA tile 128 x 128 outputs; 448 threads: warp 0 TMA producer, warp 1 MMA issuer and TMEM
-// owner, warps 2..5 expand packed nibbles to E4M3 (128-byte swizzled, K-major) and stage the
-// group scales, warps 6..13 epilogue (thread = output row x 64 columns, float32 accumulators).
+// CTA tile 128 x 128 outputs, 384 threads: warp 0 TMA producer, warp 1 MMA issuer and TMEM
+// owner, warps 2..3 expand weight nibbles and stage the group scales, warps 4..11 epilogue
+// (thread = output row x 64 columns, float32 accumulators, packed f32x2 arithmetic).
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -31,61 +35,75 @@ struct GemmArgs {
   uint64_t timeout_ns;
 };
 
-constexpr int SP = 4;   // packed stages
-constexpr int SE = 2;   // expanded stages
-constexpr int NSL = 8;  // scale slots (one group each)
-constexpr int PA_BYTES = kBM * kGemmKS / 2;      // 8 KB packed A
+constexpr int SO = 3;    // operand stages (A by TMA, B expanded)
+constexpr int SP = 4;    // packed-weight stages
+constexpr int NSL = 8;   // scale slots (one group each)
+constexpr int NTB = 4;   // TMEM accumulator buffers (128 columns each)
+constexpr int NEXP = 64; // expander threads
+constexpr int NEPI = 256;// epilogue threads
+constexpr int OA_BYTES = kBM * kGemmKS;          // 16 KB E4M3 A, 128-byte swizzle
+constexpr int OB_BYTES = kGemmBN * kGemmKS;      // 16 KB E4M3 B, 128-byte swizzle
+constexpr int OSTAGE = OA_BYTES + OB_BYTES;
 constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;  // 8 KB packed B
 constexpr int PSX_BYTES = 4 * kBM * 4;           // up to 4 groups x 128 f32 activation scales
+constexpr int PCS_BYTES = 4 * kBM * 4;           // up to 4 groups x 128 f32 activation code sums
 constexpr int PSW_BYTES = 4 * kGemmBN * 2;       // up to 4 groups x 128 f16 weight scales
-constexpr int PSTAGE = PA_BYTES + PB_BYTES + PSX_BYTES + PSW_BYTES;  // 19 KB
-constexpr int XA_BYTES = kBM * kGemmKS;          // 16 KB E4M3 A
-constexpr int XB_BYTES = kGemmBN * kGemmKS;      // 16 KB E4M3 B
-constexpr int XSTAGE = XA_BYTES + XB_BYTES;
-constexpr int SLOT_BYTES = (kGemmBN + kBM) * 4;  // f32 weight scales + f32 activation scales
+constexpr int PSTAGE = PB_BYTES + PSX_BYTES + PCS_BYTES + PSW_BYTES;
+constexpr int SLOT_FLOATS = kGemmBN + 2 * kBM;   // s_w (f32) | s_x | code sums
 
 template <int RP>
 struct GemmCfg {
   static constexpr int BR_BYTES = RP * kBM * 2;  // p_hat tile (and the B_hat tile), RP/8 boxes of 2 KB
-  static constexpr int NBAR = 2 * SP + 2 * SE + 2 * NSL + 4 + 2;
-  static constexpr int SMEM = 1024 + SE * XSTAGE + SP * PSTAGE + NSL * SLOT_BYTES + 2 * BR_BYTES + NBAR * 8 + 16;
+  static constexpr int NBAR = 2 * SO + 2 * SP + 2 * NSL + 2 * NTB + 2;
+  static constexpr int SMEM =
+      1024 + SO * OSTAGE + SP * PSTAGE + NSL * SLOT_FLOATS * 4 + 2 * BR_BYTES + NBAR * 8 + 16;
+  static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 };
 
-// 4 two's-complement nibbles (low 16 bits of w) -> 4 E4M3 bytes of the same integers.
-__device__ __forceinline__ uint32_t nibbles_to_e4m3(uint32_t w) {
-  // E4M3 of 0..7 and of -8..-1 (indexed by the low three bits of the nibble).
-  constexpr uint32_t P0 = 0x44403800u, P1 = 0x4E4C4A48u;
-  constexpr uint32_t N0 = 0xCACCCED0u, N1 = 0xB8C0C4C8u;
-  const uint32_t sel = w & 0x7777u;
-  const uint32_t pos = __byte_perm(P0, P1, sel);
-  const uint32_t neg = __byte_perm(N0, N1, sel);
-  const uint32_t pick = ((w >> 1) & 0x4444u) | 0x3210u;
-  return __byte_perm(pos, neg, pick);
+typedef unsigned long long f2;  // two packed float32 (for the f32x2 instructions)
+
+__device__ __forceinline__ f2 pk(float lo, float hi) {
+  return static_cast<f2>(__float_as_uint(lo)) | (static_cast<f2>(__float_as_uint(hi)) << 32);
+}
+__device__ __forceinline__ f2 pku(uint32_t lo, uint32_t hi) {
+  return static_cast<f2>(lo) | (static_cast<f2>(hi) << 32);
+}
+__device__ __forceinline__ float lo_f(f2 v) { return __uint_as_float(static_cast<uint32_t>(v)); }
+__device__ __forceinline__ float hi_f(f2 v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
+__device__ __forceinline__ f2 fma2(f2 a, f2 b, f2 c) {
+  f2 d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ f2 add2(f2 a, f2 b) {
+  f2 d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
 }
 
 template <int RP>
-__global__ void __launch_bounds__(448, 1)
+__global__ void __launch_bounds__(384, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap qx_map, const __grid_constant__ CUtensorMap qw_map,
-                const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap sw_map,
-                const __grid_constant__ CUtensorMap ph_map, const __grid_constant__ CUtensorMap bh_map,
-                const GemmArgs a) {
+                const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap cs_map,
+                const __grid_constant__ CUtensorMap sw_map, const __grid_constant__ CUtensorMap ph_map,
+                const __grid_constant__ CUtensorMap bh_map, const GemmArgs a) {
   using Cfg = GemmCfg<RP>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* xring = smem;                          // SE x (A 16 KB | B 16 KB), 1024-aligned
-  uint8_t* pring = xring + SE * XSTAGE;           // SP x (A | B | sx | sw)
-  float* slots = reinterpret_cast<float*>(pring + SP * PSTAGE);  // NSL x (sw[128] | sx[128])
-  uint8_t* br = reinterpret_cast<uint8_t*>(slots) + NSL * SLOT_BYTES;  // p_hat tile | B_hat tile
+  uint8_t* oring = smem;                          // SO x (A 16 KB | B 16 KB), 1024-aligned
+  uint8_t* pring = oring + SO * OSTAGE;           // SP x (B packed | s_x | code sums | s_w)
+  float* slots = reinterpret_cast<float*>(pring + SP * PSTAGE);
+  uint8_t* br = reinterpret_cast<uint8_t*>(slots + NSL * SLOT_FLOATS);  // p_hat tile | B_hat tile
   uint64_t* bars = reinterpret_cast<uint64_t*>(br + 2 * Cfg::BR_BYTES);
-  uint64_t* pfull = bars;
+  uint64_t* ofull = bars;
+  uint64_t* oempty = ofull + SO;
+  uint64_t* pfull = oempty + SO;
   uint64_t* pempty = pfull + SP;
-  uint64_t* xfull = pempty + SP;
-  uint64_t* xempty = xfull + SE;
-  uint64_t* sfull = xempty + SE;
+  uint64_t* sfull = pempty + SP;
   uint64_t* sempty = sfull + NSL;
   uint64_t* tfull = sempty + NSL;
-  uint64_t* tempty = tfull + 2;
-  uint64_t* bfull = tempty + 2;
+  uint64_t* tempty = tfull + NTB;
+  uint64_t* bfull = tempty + NTB;
   uint64_t* drain = bfull + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + Cfg::NBAR);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
@@ -99,21 +117,21 @@ __global__ void __launch_bounds__(448, 1)
   const int nst = (a.K + kGemmKS - 1) / kGemmKS;  // the last stage may be partly past K (zero-filled)
 
   if (threadIdx.x == 0) {
+    for (int i = 0; i < SO; ++i) {
+      mbar_init(&ofull[i], 1 + NEXP);
+      mbar_init(&oempty[i], 1);
+    }
     for (int i = 0; i < SP; ++i) {
       mbar_init(&pfull[i], 1);
-      mbar_init(&pempty[i], 128);
-    }
-    for (int i = 0; i < SE; ++i) {
-      mbar_init(&xfull[i], 128);
-      mbar_init(&xempty[i], 1);
+      mbar_init(&pempty[i], NEXP);
     }
     for (int i = 0; i < NSL; ++i) {
-      mbar_init(&sfull[i], 128);
-      mbar_init(&sempty[i], 256);
+      mbar_init(&sfull[i], NEXP);
+      mbar_init(&sempty[i], NEPI);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < NTB; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], 256);
+      mbar_init(&tempty[i], NEPI);
     }
     mbar_init(bfull, 1);
     mbar_init(drain, 1);
@@ -121,7 +139,7 @@ __global__ void __launch_bounds__(448, 1)
     fence_mbar_init();
   }
   if (wid == 1) {
-    tmem_alloc(tmem_slot, 256);
+    tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
   __syncthreads();
@@ -140,17 +158,21 @@ __global__ void __launch_bounds__(448, 1)
           tma_load_2d(br + Cfg::BR_BYTES + b * 2048, &bh_map, bfull, b * 8, n0);
         }
       }
-      const uint32_t bytes = PA_BYTES + PB_BYTES + gps * (kBM * 4 + kGemmBN * 2);
+      const uint32_t pbytes = PB_BYTES + gps * (kBM * 8 + kGemmBN * 2);
       for (int st = 0; st < nst; ++st) {
-        const int s = st % SP;
-        if (st >= SP) ok = mbar_wait(&pempty[s], ((st / SP) & 1) ^ 1, wc);
+        const int sp = st % SP, so = st % SO;
+        if (st >= SP) ok = mbar_wait(&pempty[sp], ((st / SP) & 1) ^ 1, wc);
         if (!ok) break;
-        uint8_t* p = pring + s * PSTAGE;
-        mbar_arrive_expect_tx(&pfull[s], bytes);
-        tma_load_2d(p, &qx_map, &pfull[s], st * (kGemmKS / 2), m0);
-        tma_load_2d(p + PA_BYTES, &qw_map, &pfull[s], st * (kGemmKS / 2), n0);
-        tma_load_2d(p + PA_BYTES + PB_BYTES, &sx_map, &pfull[s], m0, st * gps);
-        tma_load_2d(p + PA_BYTES + PB_BYTES + PSX_BYTES, &sw_map, &pfull[s], n0, st * gps);
+        uint8_t* p = pring + sp * PSTAGE;
+        mbar_arrive_expect_tx(&pfull[sp], pbytes);
+        tma_load_2d(p, &qw_map, &pfull[sp], st * (kGemmKS / 2), n0);
+        tma_load_2d(p + PB_BYTES, &sx_map, &pfull[sp], m0, st * gps);
+        tma_load_2d(p + PB_BYTES + PSX_BYTES, &cs_map, &pfull[sp], m0, st * gps);
+        tma_load_2d(p + PB_BYTES + PSX_BYTES + PCS_BYTES, &sw_map, &pfull[sp], n0, st * gps);
+        if (st >= SO) ok = mbar_wait(&oempty[so], ((st / SO) & 1) ^ 1, wc);
+        if (!ok) break;
+        mbar_arrive_expect_tx(&ofull[so], OA_BYTES);
+        tma_load_2d(oring + so * OSTAGE, &qx_map, &ofull[so], st * kGemmKS, m0);
       }
       // Let every issued load land before the CTA can exit.
       int never = 0;
@@ -165,16 +187,16 @@ __global__ void __launch_bounds__(448, 1)
       bool ok = true;
       constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
       for (int st = 0; st < nst && ok; ++st) {
-        const int x = st % SE;
-        ok = mbar_wait(&xfull[x], (st / SE) & 1, wc);
+        const int so = st % SO;
+        ok = mbar_wait(&ofull[so], (st / SO) & 1, wc);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t xa = smem_u32(xring + x * XSTAGE), xb = xa + XA_BYTES;
+        const uint32_t xa = smem_u32(oring + so * OSTAGE), xb = xa + OA_BYTES;
         for (int gi = 0; gi < gps && ok; ++gi) {
           const int g = st * gps + gi;
           if (g >= ngroups) break;
-          const int b = g & 1;
-          if (g >= 2) ok = mbar_wait(&tempty[b], ((g >> 1) & 1) ^ 1, wc);
+          const int b = g % NTB;
+          if (g >= NTB) ok = mbar_wait(&tempty[b], ((g / NTB) & 1) ^ 1, wc);
           if (!ok) break;
           tc_fence_after();
           for (int kk = 0; kk < G / 32; ++kk) {
@@ -184,12 +206,12 @@ __global__ void __launch_bounds__(448, 1)
           }
           mma_commit(&tfull[b]);
         }
-        mma_commit(&xempty[x]);
+        mma_commit(&oempty[so]);
       }
       if constexpr (RP > 0) {
-        const int g = ngroups, b = g & 1;
+        const int g = ngroups, b = g % NTB;
         if (ok) ok = mbar_wait(bfull, 0, wc);
-        if (ok && g >= 2) ok = mbar_wait(&tempty[b], ((g >> 1) & 1) ^ 1, wc);
+        if (ok && g >= NTB) ok = mbar_wait(&tempty[b], ((g / NTB) & 1) ^ 1, wc);
         if (ok) {
           tc_fence_after();
           constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
@@ -207,99 +229,100 @@ __global__ void __launch_bounds__(448, 1)
       mbar_wait(drain, 0, dc);
     }
     __syncwarp();
-  } else if (wid < 6) {
-    // ------------------------------------------------------------- expanders
-    const int e = static_cast<int>(threadIdx.x) - 64;  // 0..127
+  } else if (wid < 4) {
+    // ------------------------------------------------------------- weight expanders + scales
+    const int e = static_cast<int>(threadIdx.x) - 64;  // 0..63
+    const uint32_t kX8 = 0x88888888u;
     bool ok = true;
     for (int st = 0; st < nst && ok; ++st) {
-      const int s = st % SP, x = st % SE;
-      ok = mbar_wait(&pfull[s], (st / SP) & 1, wc);
-      if (ok && st >= SE) ok = mbar_wait(&xempty[x], ((st / SE) & 1) ^ 1, wc);
+      const int sp = st % SP, so = st % SO;
+      ok = mbar_wait(&pfull[sp], (st / SP) & 1, wc);
+      if (ok && st >= SO) ok = mbar_wait(&oempty[so], ((st / SO) & 1) ^ 1, wc);
       if (!ok) break;
-      const uint8_t* p = pring + s * PSTAGE;
-      uint8_t* xs = xring + x * XSTAGE;
+      const uint8_t* p = pring + sp * PSTAGE;
+      uint8_t* xb = oring + so * OSTAGE + OA_BYTES;
 #pragma unroll 4
       for (int i = 0; i < 16; ++i) {
-        const int t = e + 128 * i;
-        const int mat = t >> 10, tt = t & 1023, row = tt >> 3, j = tt & 7;
-        const uint2 pk = *reinterpret_cast<const uint2*>(p + mat * PA_BYTES + row * 64 + j * 8);
+        const int t = e + NEXP * i;
+        const int row = t >> 3, j = t & 7;
+        const uint2 pkd = *reinterpret_cast<const uint2*>(p + row * 64 + j * 8);
         uint4 o;
-        o.x = nibbles_to_e4m3(pk.x);
-        o.y = nibbles_to_e4m3(pk.x >> 16);
-        o.z = nibbles_to_e4m3(pk.y);
-        o.w = nibbles_to_e4m3(pk.y >> 16);
-        *reinterpret_cast<uint4*>(xs + mat * XA_BYTES + (row >> 3) * 1024 + (row & 7) * 128 + ((j ^ (row & 7)) << 4)) = o;
+        o.x = (pkd.x ^ kX8) & 0x0F0F0F0Fu;
+        o.y = ((pkd.x >> 4) ^ kX8) & 0x0F0F0F0Fu;
+        o.z = (pkd.y ^ kX8) & 0x0F0F0F0Fu;
+        o.w = ((pkd.y >> 4) ^ kX8) & 0x0F0F0F0Fu;
+        *reinterpret_cast<uint4*>(xb + (row >> 3) * 1024 + (row & 7) * 128 + ((j ^ (row & 7)) << 4)) = o;
       }
       fence_proxy_async_smem();
-      mbar_arrive(&xfull[x]);
+      mbar_arrive(&ofull[so]);
       // group scales of this stage -> float32 slots for the epilogue
-      const float* psx = reinterpret_cast<const float*>(p + PA_BYTES + PB_BYTES);
-      const __half* psw = reinterpret_cast<const __half*>(p + PA_BYTES + PB_BYTES + PSX_BYTES);
+      const float* psx = reinterpret_cast<const float*>(p + PB_BYTES);
+      const float* pcs = reinterpret_cast<const float*>(p + PB_BYTES + PSX_BYTES);
+      const __half* psw = reinterpret_cast<const __half*>(p + PB_BYTES + PSX_BYTES + PCS_BYTES);
       for (int gi = 0; gi < gps && ok; ++gi) {
         const int g = st * gps + gi;
         if (g >= ngroups) break;
         const int sl = g % NSL;
         if (g >= NSL) ok = mbar_wait(&sempty[sl], ((g / NSL) & 1) ^ 1, wc);
         if (!ok) break;
-        float* slot = slots + sl * (kGemmBN + kBM);
-        slot[e] = __half2float(psw[gi * kGemmBN + e]);
-        slot[kGemmBN + e] = psx[gi * kBM + e];
+        float* slot = slots + sl * SLOT_FLOATS;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int i = e + NEXP * h;
+          slot[i] = __half2float(psw[gi * kGemmBN + i]);
+          slot[kGemmBN + i] = psx[gi * kBM + i];
+          slot[kGemmBN + kBM + i] = pcs[gi * kBM + i];
+        }
         mbar_arrive(&sfull[sl]);
       }
-      mbar_arrive(&pempty[s]);
+      fence_proxy_async_smem();  // reads of the packed stage before the TMA refills it
+      mbar_arrive(&pempty[sp]);
     }
   } else {
     // ------------------------------------------------------------- epilogue
-    // Warps 6..13: warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 64
-    // output columns [64*((w-6)/4), +64).
+    // Warps 4..11: warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 64 output
+    // columns [64*((w-4)/4), +64).
     const int quad = wid & 3;
     const int row = quad * 32 + static_cast<int>(lane);
     const int m = m0 + row;
-    const int col0 = 64 * ((static_cast<int>(wid) - 6) >> 2);
+    const int col0 = 64 * ((static_cast<int>(wid) - 4) >> 2);
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
-    float acc[64];
+    f2 acc[32];
 #pragma unroll
-    for (int i = 0; i < 64; ++i) acc[i] = 0.0f;
+    for (int i = 0; i < 32; ++i) acc[i] = 0ull;
     bool ok = true;
     const int ntot = ngroups + (RP > 0 ? 1 : 0);
     for (int g = 0; g < ntot; ++g) {
-      const int b = g & 1;
-      if (ok) ok = mbar_wait(&tfull[b], (g >> 1) & 1, wc);
+      const int b = g % NTB;
+      if (ok) ok = mbar_wait(&tfull[b], (g / NTB) & 1, wc);
       tc_fence_after();
+      uint32_t v[64];
+      tmem_ld32(tlane + b * 128, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
+      tmem_ld32(tlane + b * 128 + 32, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
+      tmem_ld_wait();
+      tc_fence_before();
+      mbar_arrive(&tempty[b]);
       if (g < ngroups) {
         const int sl = g % NSL;
         if (ok) ok = mbar_wait(&sfull[sl], (g / NSL) & 1, wc);
-        const float* slot = slots + sl * (kGemmBN + kBM);
+        const float* slot = slots + sl * SLOT_FLOATS;
         const float sxv = slot[kGemmBN + row];
+        const float alpha = sxv * 262144.0f;                       // 2^18 s_x (exact)
+        const float beta = -8.0f * sxv * slot[kGemmBN + kBM + row];  // -8 s_x S_a
+        const f2 al2 = pk(alpha, alpha), be2 = pk(beta, beta);
+        const float4* w4 = reinterpret_cast<const float4*>(slot + col0);
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          uint32_t v[32];
-          tmem_ld32(tlane + b * 128 + c * 32, v);
-          tmem_ld_wait();
-          const float4* w4 = reinterpret_cast<const float4*>(slot + col0 + c * 32);
-#pragma unroll
-          for (int i4 = 0; i4 < 8; ++i4) {
-            const float4 w = w4[i4];
-            acc[c * 32 + 4 * i4 + 0] = fmaf(__uint_as_float(v[4 * i4 + 0]) * w.x, sxv, acc[c * 32 + 4 * i4 + 0]);
-            acc[c * 32 + 4 * i4 + 1] = fmaf(__uint_as_float(v[4 * i4 + 1]) * w.y, sxv, acc[c * 32 + 4 * i4 + 1]);
-            acc[c * 32 + 4 * i4 + 2] = fmaf(__uint_as_float(v[4 * i4 + 2]) * w.z, sxv, acc[c * 32 + 4 * i4 + 2]);
-            acc[c * 32 + 4 * i4 + 3] = fmaf(__uint_as_float(v[4 * i4 + 3]) * w.w, sxv, acc[c * 32 + 4 * i4 + 3]);
-          }
+        for (int i4 = 0; i4 < 16; ++i4) {
+          const float4 w = w4[i4];
+          const f2 t0 = fma2(pku(v[4 * i4], v[4 * i4 + 1]), al2, be2);
+          const f2 t1 = fma2(pku(v[4 * i4 + 2], v[4 * i4 + 3]), al2, be2);
+          acc[2 * i4] = fma2(t0, pk(w.x, w.y), acc[2 * i4]);
+          acc[2 * i4 + 1] = fma2(t1, pk(w.z, w.w), acc[2 * i4 + 1]);
         }
-        tc_fence_before();
-        mbar_arrive(&tempty[b]);
         mbar_arrive(&sempty[sl]);
       } else {
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          uint32_t v[32];
-          tmem_ld32(tlane + b * 128 + c * 32, v);
-          tmem_ld_wait();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) acc[c * 32 + i] += __uint_as_float(v[i]);
-        }
-        tc_fence_before();
-        mbar_arrive(&tempty[b]);
+        for (int i = 0; i < 32; ++i) acc[i] = add2(acc[i], pku(v[2 * i], v[2 * i + 1]));
       }
     }
     if (ok && m < a.M) {
@@ -310,9 +333,9 @@ __global__ void __launch_bounds__(448, 1)
         for (int c8 = 0; c8 < 8; ++c8) {
           if (nb + c8 * 8 < a.N) {
             reinterpret_cast<float4*>(yr + c8 * 8)[0] =
-                make_float4(acc[c8 * 8], acc[c8 * 8 + 1], acc[c8 * 8 + 2], acc[c8 * 8 + 3]);
-            reinterpret_cast<float4*>(yr + c8 * 8)[1] =
-                make_float4(acc[c8 * 8 + 4], acc[c8 * 8 + 5], acc[c8 * 8 + 6], acc[c8 * 8 + 7]);
+                make_float4(lo_f(acc[4 * c8]), hi_f(acc[4 * c8]), lo_f(acc[4 * c8 + 1]), hi_f(acc[4 * c8 + 1]));
+            reinterpret_cast<float4*>(yr + c8 * 8)[1] = make_float4(lo_f(acc[4 * c8 + 2]), hi_f(acc[4 * c8 + 2]),
+                                                                    lo_f(acc[4 * c8 + 3]), hi_f(acc[4 * c8 + 3]));
           }
         }
       } else {
@@ -323,7 +346,7 @@ __global__ void __launch_bounds__(448, 1)
             uint32_t w[4];
 #pragma unroll
             for (int t = 0; t < 4; ++t) {
-              __nv_bfloat162 h2 = __floats2bfloat162_rn(acc[c8 * 8 + 2 * t], acc[c8 * 8 + 2 * t + 1]);
+              __nv_bfloat162 h2 = __floats2bfloat162_rn(lo_f(acc[4 * c8 + t]), hi_f(acc[4 * c8 + t]));
               w[t] = *reinterpret_cast<uint32_t*>(&h2);
             }
             *reinterpret_cast<uint4*>(yr + c8 * 8) = make_uint4(w[0], w[1], w[2], w[3]);
@@ -336,7 +359,7 @@ __global__ void __launch_bounds__(448, 1)
   __syncthreads();
   if (wid == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, 512);
   }
 }
 
@@ -361,7 +384,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
   dim3 grid((h.N + kGemmBN - 1) / kGemmBN, (M + kBM - 1) / kBM, 1);
   const CUtensorMap& ph = (RP > 0) ? am.ph_map : am.qx_map;
   const CUtensorMap& bh = (RP > 0) ? h.Bh_map : am.qx_map;
-  gemm_kernel<RP><<<grid, 448, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.sx_map, h.sw_map, ph, bh, a);
+  gemm_kernel<RP><<<grid, 384, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.sx_map, am.cs_map, h.sw_map, ph, bh, a);
   return cudaGetLastError();
 }
 

@@ -26,16 +26,19 @@ struct ActMaps {
   const void* x = nullptr;
   int M = -1;
   CUtensorMap x_map;    // X bf16 [M, K], box {64, 128}, 128-byte swizzle
-  CUtensorMap qx_map;   // codes u8 [M, K/2], box {64, 128}
+  CUtensorMap qx_map;   // code bytes [M, K], box {128, 128}, 128-byte swizzle
   CUtensorMap sx_map;   // scales f32 [K/G, M_pad] (dims {M, K/G}), box {128, KS/G}
+  CUtensorMap cs_map;   // code sums f32 [K/G, M_pad], same geometry as the scales
   CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128}
 };
 
 struct Handle {
   int K = 0, N = 0, r = 0, G = 0, r_pad = 0, N_pad = 0, ku3 = 0;
   int device = 0;
+  int num_sms = 148;
   void* block = nullptr;             // one device allocation holding every buffer below
-  uint8_t* qw = nullptr;             // [N_pad, K/2]
+  uint8_t* qw = nullptr;             // [N_pad, K/2]; word j of a row holds k = 8j..8j+3 in the low
+                                     // and 8j+4..8j+7 in the high nibbles of its bytes
   __half* sw = nullptr;              // [K/G, N_pad]
   __half* Bh = nullptr;              // [N_pad, r_pad]
   __nv_bfloat16* ucat_t = nullptr;   // [2 r_pad, K]: rows 0..r_pad-1 = U_hi^T, then U_lo^T
@@ -48,7 +51,7 @@ struct Handle {
 };
 
 struct ActLayout {
-  size_t codes_off, scales_off, phat_off, bytes;
+  size_t codes_off, scales_off, csums_off, phat_off, bytes;
   int M_pad;
 };
 ActLayout act_layout(const Handle& h, int M);

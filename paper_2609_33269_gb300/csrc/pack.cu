@@ -47,8 +47,9 @@ __device__ __forceinline__ int nearest_code_f64(double w, double s) {
   return static_cast<int>(c);
 }
 
-// One thread per (output channel n, group g): s_w = RN_f16(absmax / 7), codes packed two per
-// byte (low nibble = even k) into qw[n, k/2].
+// One thread per (output channel n, group g): s_w = RN_f16(absmax / 7), codes packed 4 bits
+// each into qw[n, :]: 32-bit word j holds k = 8j..8j+3 in the low nibbles and k = 8j+4..8j+7 in
+// the high nibbles of its four bytes (the GEMM expands a word to bytes with three logic ops).
 __global__ void quantize_weight_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
                                        const double* __restrict__ Bf, int K, int N, int r, int G, int N_pad,
                                        uint8_t* __restrict__ qw, __half* __restrict__ sw, int* err) {
@@ -62,15 +63,18 @@ __global__ void quantize_weight_kernel(const __nv_bfloat16* __restrict__ W, cons
   sw[static_cast<size_t>(g) * N_pad + n] = sh;
   bool ok_scale = isfinite(s);
   if (!ok_scale) atomicOr(err, kErrRange);
-  uint8_t* row = qw + static_cast<size_t>(n) * (K / 2);
-  for (int k = g * G; k < (g + 1) * G; k += 2) {
-    int c0 = 0, c1 = 0;
-    if (s > 0.0 && ok_scale) {
-      c0 = nearest_code_f64(wperp(W, U, Bf, N, r, k, n), s);
-      c1 = nearest_code_f64(wperp(W, U, Bf, N, r, k + 1, n), s);
+  uint32_t* row = reinterpret_cast<uint32_t*>(qw + static_cast<size_t>(n) * (K / 2));
+  for (int k = g * G; k < (g + 1) * G; k += 8) {
+    uint32_t word = 0;
+    for (int i = 0; i < 8; ++i) {
+      int c = 0;
+      if (s > 0.0 && ok_scale) c = nearest_code_f64(wperp(W, U, Bf, N, r, k + i, n), s);
+      if (c < -7 || c > 7) atomicOr(err, kErrRange);
+      // k + i (i < 4) -> low nibble of byte i; k + 4 + i -> high nibble of byte i
+      const int shift = (i < 4) ? 8 * i : 8 * (i - 4) + 4;
+      word |= (static_cast<uint32_t>(c) & 0xFu) << shift;
     }
-    if (c0 < -7 || c0 > 7 || c1 < -7 || c1 > 7) atomicOr(err, kErrRange);
-    row[k / 2] = static_cast<uint8_t>((c0 & 0xF) | ((c1 & 0xF) << 4));
+    row[k / 8] = word;
   }
 }
 

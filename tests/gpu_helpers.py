@@ -14,6 +14,14 @@ def to_dev_bf16(bits: np.ndarray) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).cuda().view(torch.bfloat16)
 
 
+def decode_code_bytes(b: np.ndarray) -> np.ndarray:
+    """Activation code bytes (E4M3 of c * 2^-9: sign bit | magnitude) -> int8 codes."""
+    b = np.ascontiguousarray(b, np.uint8)
+    assert not (b & 0x78).any(), "activation code byte outside the E4M3 subnormal code range"
+    mag = (b & 0x7).astype(np.int8)
+    return np.where(b & 0x80, -mag, mag).astype(np.int8)
+
+
 def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
     """uint8 [R, K/2] -> int8 [R, K] (low nibble = even k, two's complement)."""
     p = np.ascontiguousarray(packed)
@@ -55,11 +63,14 @@ class Case:
         return dict(qw=unpack_nibbles(e["qw"]), sw=e["sw"], Bh=e["Bh"][:, :self.r].T.copy(), Uhl=e["Uhl"])
 
     def gpu_act(self, rows=None):
-        codes, scales, ph = self.layer.act_views(self.M)
+        codes, scales, csums, ph = self.layer.act_views(self.M)
         torch.cuda.synchronize()
-        qx = unpack_nibbles(codes.cpu().numpy())
+        qx = decode_code_bytes(codes.cpu().numpy())
         sx = scales.cpu().numpy()[:, :self.M].T.copy()
+        cs = csums.cpu().numpy()[:, :self.M].T.copy()
         phv = ph.cpu().numpy().view(np.uint16)[:, :self.r].copy()
+        # the code sums the GEMM uses are the exact sums of the codes
+        np.testing.assert_array_equal(cs, qx.reshape(self.M, -1, self.G).sum(axis=2).astype(np.float32))
         if rows is not None:
             qx, sx, phv = qx[rows], sx[rows], phv[rows]
         return dict(qx=qx, sx=sx, ph=phv)
