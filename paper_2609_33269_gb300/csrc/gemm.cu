@@ -16,11 +16,16 @@
 // stay packed in HBM; a nibble becomes its byte with three logic ops per eight nibbles because
 // the packing puts the codes of k = 8j..8j+3 in the low and of k = 8j+4..8j+7 in the high
 // nibbles of the four bytes of word j.  Each group has its own TMEM accumulator (four buffers);
-// after the last group one kind::f16 MMA of K = r_pad forms p_hat B_hat^T, added with scale 1.
+// after the last group of a tile one kind::f16 MMA of K = r_pad forms p_hat B_hat^T, which the
+// epilogue adds with scale 1.
 //
-// CTA tile 128 x 128 outputs, 384 threads: warp 0 TMA producer, warp 1 MMA issuer and TMEM
-// owner, warps 2..3 expand weight nibbles and stage the group scales, warps 4..11 epilogue
-// (thread = output row x 64 columns, float32 accumulators, packed f32x2 arithmetic).
+// Persistent CTAs (one per SM) walk output tiles of 128 x 128 with a static stride; every ring
+// (activation tiles, packed weights with the group scales, expanded weights, branch tiles, scale
+// slots, TMEM accumulators) runs continuously across tiles, so loads for the next tile overlap
+// the epilogue of the current one.  448 threads: warp 0 TMA producer, warp 1 MMA issuer and TMEM
+// owner, warps 2..5 expand weight nibbles and stage the group scales, warps 6..13 epilogue
+// (thread = output row x 64 columns, packed f32x2).  Every ring has exactly one waiting role per
+// side, which waits for each phase in turn.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -29,34 +34,36 @@ namespace {
 
 struct GemmArgs {
   int M, N, K, G;
+  int m_tiles, n_tiles;
   void* Y;
   int y_f32;
   int* err;
   uint64_t timeout_ns;
 };
 
-constexpr int SO = 3;    // operand stages (A by TMA, B expanded)
-constexpr int SP = 4;    // packed-weight stages
-constexpr int NSL = 8;   // scale slots (one group each)
-constexpr int NTB = 4;   // TMEM accumulator buffers (128 columns each)
-constexpr int NEXP = 64; // expander threads
-constexpr int NEPI = 256;// epilogue threads
-constexpr int OA_BYTES = kBM * kGemmKS;          // 16 KB E4M3 A, 128-byte swizzle
-constexpr int OB_BYTES = kGemmBN * kGemmKS;      // 16 KB E4M3 B, 128-byte swizzle
-constexpr int OSTAGE = OA_BYTES + OB_BYTES;
-constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;  // 8 KB packed B
-constexpr int PSX_BYTES = 4 * kBM * 4;           // up to 4 groups x 128 f32 activation scales
-constexpr int PCS_BYTES = 4 * kBM * 4;           // up to 4 groups x 128 f32 activation code sums
-constexpr int PSW_BYTES = 4 * kGemmBN * 2;       // up to 4 groups x 128 f16 weight scales
+constexpr int SX = 3;     // expanded-weight stages (expanders -> MMA)
+constexpr int NSL = 8;    // scale slots (one group each)
+constexpr int NTB = 4;    // TMEM accumulator buffers (128 columns each)
+constexpr int NBR = 2;    // branch-operand stages (one per tile)
+constexpr int NEXP = 128; // expander threads
+constexpr int NEPI = 256; // epilogue threads
+constexpr int A_BYTES = kBM * kGemmKS;            // 16 KB, 128-byte swizzle
+constexpr int X_BYTES = kGemmBN * kGemmKS;        // 16 KB, 128-byte swizzle
+constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;   // 8 KB packed weights
+constexpr int PSX_BYTES = 4 * kBM * 4;            // up to 4 groups x 128 f32 activation scales
+constexpr int PCS_BYTES = 4 * kBM * 4;            // up to 4 groups x 128 f32 activation code sums
+constexpr int PSW_BYTES = 4 * kGemmBN * 2;        // up to 4 groups x 128 f16 weight scales
 constexpr int PSTAGE = PB_BYTES + PSX_BYTES + PCS_BYTES + PSW_BYTES;
-constexpr int SLOT_FLOATS = kGemmBN + 2 * kBM;   // s_w (f32) | s_x | code sums
+constexpr int SLOT_FLOATS = kGemmBN + 2 * kBM;    // s_w (f32) | s_x | code sums
 
 template <int RP>
 struct GemmCfg {
-  static constexpr int BR_BYTES = RP * kBM * 2;  // p_hat tile (and the B_hat tile), RP/8 boxes of 2 KB
-  static constexpr int NBAR = 2 * SO + 2 * SP + 2 * NSL + 2 * NTB + 2;
-  static constexpr int SMEM =
-      1024 + SO * OSTAGE + SP * PSTAGE + NSL * SLOT_FLOATS * 4 + 2 * BR_BYTES + NBAR * 8 + 16;
+  static constexpr int SA = RP <= 48 ? 4 : 3;                     // activation stages (TMA -> MMA)
+  static constexpr int SP = RP <= 16 ? 6 : (RP <= 32 ? 5 : 4);    // packed-weight stages
+  static constexpr int BR_BYTES = RP * kBM * 2;   // p_hat tile (and the B_hat tile), RP/8 boxes of 2 KB
+  static constexpr int NBAR = 2 * SA + 2 * SX + 2 * SP + 2 * NSL + 2 * NTB + 2 * NBR + 1;
+  static constexpr int SMEM = 1024 + SA * A_BYTES + SX * X_BYTES + SP * PSTAGE + NSL * SLOT_FLOATS * 4 +
+                              NBR * 2 * BR_BYTES + NBAR * 8 + 16;
   static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 };
 
@@ -82,44 +89,62 @@ __device__ __forceinline__ f2 add2(f2 a, f2 b) {
 }
 
 template <int RP>
-__global__ void __launch_bounds__(384, 1)
+__global__ void __launch_bounds__(448, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap qx_map, const __grid_constant__ CUtensorMap qw_map,
                 const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap cs_map,
                 const __grid_constant__ CUtensorMap sw_map, const __grid_constant__ CUtensorMap ph_map,
                 const __grid_constant__ CUtensorMap bh_map, const GemmArgs a) {
   using Cfg = GemmCfg<RP>;
+  constexpr int SP = Cfg::SP;
+  constexpr int SA = Cfg::SA;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* oring = smem;                          // SO x (A 16 KB | B 16 KB), 1024-aligned
-  uint8_t* pring = oring + SO * OSTAGE;           // SP x (B packed | s_x | code sums | s_w)
+  uint8_t* aring = smem;                           // SA x 16 KB, 1024-aligned
+  uint8_t* xring = aring + SA * A_BYTES;           // SX x 16 KB, 1024-aligned
+  uint8_t* pring = xring + SX * X_BYTES;           // SP x (weights packed | s_x | code sums | s_w)
   float* slots = reinterpret_cast<float*>(pring + SP * PSTAGE);
-  uint8_t* br = reinterpret_cast<uint8_t*>(slots + NSL * SLOT_FLOATS);  // p_hat tile | B_hat tile
-  uint64_t* bars = reinterpret_cast<uint64_t*>(br + 2 * Cfg::BR_BYTES);
-  uint64_t* ofull = bars;
-  uint64_t* oempty = ofull + SO;
-  uint64_t* pfull = oempty + SO;
+  uint8_t* br = reinterpret_cast<uint8_t*>(slots + NSL * SLOT_FLOATS);  // NBR x (p_hat | B_hat)
+  uint64_t* bars = reinterpret_cast<uint64_t*>(br + NBR * 2 * Cfg::BR_BYTES);
+  uint64_t* afull = bars;
+  uint64_t* aempty = afull + SA;
+  uint64_t* xfull = aempty + SA;
+  uint64_t* xempty = xfull + SX;
+  uint64_t* pfull = xempty + SX;
   uint64_t* pempty = pfull + SP;
   uint64_t* sfull = pempty + SP;
   uint64_t* sempty = sfull + NSL;
   uint64_t* tfull = sempty + NSL;
   uint64_t* tempty = tfull + NTB;
   uint64_t* bfull = tempty + NTB;
-  uint64_t* drain = bfull + 1;
+  uint64_t* bempty = bfull + NBR;
+  uint64_t* drain = bempty + NBR;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + Cfg::NBAR);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const uint32_t wid = warp_id(), lane = lane_id();
-  const int n0 = blockIdx.x * kGemmBN;
-  const int m0 = blockIdx.y * kBM;
   const int G = a.G;
   const int gps = kGemmKS / G;                    // groups per stage (2 or 4)
   const int ngroups = a.K / G;
   const int nst = (a.K + kGemmKS - 1) / kGemmKS;  // the last stage may be partly past K (zero-filled)
+  const int ntiles = a.m_tiles * a.n_tiles;
+  const int my_tiles = ntiles > static_cast<int>(blockIdx.x)
+                           ? (ntiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                                 static_cast<int>(gridDim.x)
+                           : 0;
+  auto tile_mn = [&](int i, int& m0, int& n0) {  // i-th tile of this CTA, m-major order
+    const int t = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
+    m0 = (t / a.n_tiles) * kBM;
+    n0 = (t % a.n_tiles) * kGemmBN;
+  };
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < SO; ++i) {
-      mbar_init(&ofull[i], 1 + NEXP);
-      mbar_init(&oempty[i], 1);
+    for (int i = 0; i < SA; ++i) {
+      mbar_init(&afull[i], 1);
+      mbar_init(&aempty[i], 1);
+    }
+    for (int i = 0; i < SX; ++i) {
+      mbar_init(&xfull[i], NEXP);
+      mbar_init(&xempty[i], 1);
     }
     for (int i = 0; i < SP; ++i) {
       mbar_init(&pfull[i], 1);
@@ -133,7 +158,10 @@ __global__ void __launch_bounds__(384, 1)
       mbar_init(&tfull[i], 1);
       mbar_init(&tempty[i], NEPI);
     }
-    mbar_init(bfull, 1);
+    for (int i = 0; i < NBR; ++i) {
+      mbar_init(&bfull[i], 1);
+      mbar_init(&bempty[i], 1);
+    }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -151,76 +179,97 @@ __global__ void __launch_bounds__(384, 1)
     // ------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
-      if constexpr (RP > 0) {
-        mbar_arrive_expect_tx(bfull, 2 * Cfg::BR_BYTES);
-        for (int b = 0; b < RP / 8; ++b) {
-          tma_load_2d(br + b * 2048, &ph_map, bfull, b * 8, m0);
-          tma_load_2d(br + Cfg::BR_BYTES + b * 2048, &bh_map, bfull, b * 8, n0);
-        }
-      }
       const uint32_t pbytes = PB_BYTES + gps * (kBM * 8 + kGemmBN * 2);
-      for (int st = 0; st < nst; ++st) {
-        const int sp = st % SP, so = st % SO;
-        if (st >= SP) ok = mbar_wait(&pempty[sp], ((st / SP) & 1) ^ 1, wc);
-        if (!ok) break;
-        uint8_t* p = pring + sp * PSTAGE;
-        mbar_arrive_expect_tx(&pfull[sp], pbytes);
-        tma_load_2d(p, &qw_map, &pfull[sp], st * (kGemmKS / 2), n0);
-        tma_load_2d(p + PB_BYTES, &sx_map, &pfull[sp], m0, st * gps);
-        tma_load_2d(p + PB_BYTES + PSX_BYTES, &cs_map, &pfull[sp], m0, st * gps);
-        tma_load_2d(p + PB_BYTES + PSX_BYTES + PCS_BYTES, &sw_map, &pfull[sp], n0, st * gps);
-        if (st >= SO) ok = mbar_wait(&oempty[so], ((st / SO) & 1) ^ 1, wc);
-        if (!ok) break;
-        mbar_arrive_expect_tx(&ofull[so], OA_BYTES);
-        tma_load_2d(oring + so * OSTAGE, &qx_map, &ofull[so], st * kGemmKS, m0);
+      int sa = 0, sp = 0;  // running stage counters (the same sequence every role walks)
+      for (int ti = 0; ti < my_tiles && ok; ++ti) {
+        int m0, n0;
+        tile_mn(ti, m0, n0);
+        if constexpr (RP > 0) {
+          const int bs = ti % NBR;
+          if (ti >= NBR) ok = mbar_wait(&bempty[bs], ((ti / NBR) & 1) ^ 1, wc);
+          if (!ok) break;
+          uint8_t* b = br + bs * 2 * Cfg::BR_BYTES;
+          mbar_arrive_expect_tx(&bfull[bs], 2 * Cfg::BR_BYTES);
+          for (int q = 0; q < RP / 8; ++q) {
+            tma_load_2d(b + q * 2048, &ph_map, &bfull[bs], q * 8, m0);
+            tma_load_2d(b + Cfg::BR_BYTES + q * 2048, &bh_map, &bfull[bs], q * 8, n0);
+          }
+        }
+        for (int st = 0; st < nst && ok; ++st) {
+          // packed weights and the group scales of this stage
+          const int ps = sp % SP;
+          if (sp >= SP) ok = mbar_wait(&pempty[ps], ((sp / SP) & 1) ^ 1, wc);
+          if (!ok) break;
+          uint8_t* p = pring + ps * PSTAGE;
+          mbar_arrive_expect_tx(&pfull[ps], pbytes);
+          tma_load_2d(p, &qw_map, &pfull[ps], st * (kGemmKS / 2), n0);
+          tma_load_2d(p + PB_BYTES, &sx_map, &pfull[ps], m0, st * gps);
+          tma_load_2d(p + PB_BYTES + PSX_BYTES, &cs_map, &pfull[ps], m0, st * gps);
+          tma_load_2d(p + PB_BYTES + PSX_BYTES + PCS_BYTES, &sw_map, &pfull[ps], n0, st * gps);
+          ++sp;
+          // activation codes of this stage
+          const int as = sa % SA;
+          if (sa >= SA) ok = mbar_wait(&aempty[as], ((sa / SA) & 1) ^ 1, wc);
+          if (!ok) break;
+          mbar_arrive_expect_tx(&afull[as], A_BYTES);
+          tma_load_2d(aring + as * A_BYTES, &qx_map, &afull[as], st * kGemmKS, m0);
+          ++sa;
+        }
       }
       // Let every issued load land before the CTA can exit.
       int never = 0;
       const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-      const int last = ok ? nst : 0;
-      for (int j = (last > SP ? last - SP : 0); j < last; ++j) mbar_wait(&pfull[j % SP], (j / SP) & 1, dc);
-      if (RP > 0) mbar_wait(bfull, 0, dc);
+      for (int j = (sp > SP ? sp - SP : 0); j < sp; ++j) mbar_wait(&pfull[j % SP], (j / SP) & 1, dc);
+      for (int j = (sa > SA ? sa - SA : 0); j < sa; ++j) mbar_wait(&afull[j % SA], (j / SA) & 1, dc);
     }
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       bool ok = true;
       constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
-      for (int st = 0; st < nst && ok; ++st) {
-        const int so = st % SO;
-        ok = mbar_wait(&ofull[so], (st / SO) & 1, wc);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t xa = smem_u32(oring + so * OSTAGE), xb = xa + OA_BYTES;
-        for (int gi = 0; gi < gps && ok; ++gi) {
-          const int g = st * gps + gi;
-          if (g >= ngroups) break;
-          const int b = g % NTB;
-          if (g >= NTB) ok = mbar_wait(&tempty[b], ((g / NTB) & 1) ^ 1, wc);
+      int s = 0, g_all = 0;  // running stage and accumulator counters
+      for (int ti = 0; ti < my_tiles && ok; ++ti) {
+        for (int st = 0; st < nst && ok; ++st, ++s) {
+          const int as = s % SA, xs = s % SX;
+          ok = mbar_wait(&afull[as], (s / SA) & 1, wc);
+          if (ok) ok = mbar_wait(&xfull[xs], (s / SX) & 1, wc);
           if (!ok) break;
           tc_fence_after();
-          for (int kk = 0; kk < G / 32; ++kk) {
-            const uint32_t off = static_cast<uint32_t>((gi * (G / 32) + kk) * 32);
-            mma_f8f6f4(tmem + b * 128, smem_desc(xa + off, 16, 1024, kSw128), smem_desc(xb + off, 16, 1024, kSw128),
-                       idesc, kk != 0);
+          const uint32_t aa = smem_u32(aring + as * A_BYTES), xa = smem_u32(xring + xs * X_BYTES);
+          for (int gi = 0; gi < gps && ok; ++gi) {
+            const int g = st * gps + gi;
+            if (g >= ngroups) break;
+            const int b = g_all % NTB;
+            if (g_all >= NTB) ok = mbar_wait(&tempty[b], ((g_all / NTB) & 1) ^ 1, wc);
+            if (!ok) break;
+            tc_fence_after();
+            for (int kk = 0; kk < G / 32; ++kk) {
+              const uint32_t off = static_cast<uint32_t>((gi * (G / 32) + kk) * 32);
+              mma_f8f6f4(tmem + b * 128, smem_desc(aa + off, 16, 1024, kSw128),
+                         smem_desc(xa + off, 16, 1024, kSw128), idesc, kk != 0);
+            }
+            mma_commit(&tfull[b]);
+            ++g_all;
           }
-          mma_commit(&tfull[b]);
+          mma_commit(&aempty[as]);
+          mma_commit(&xempty[xs]);
         }
-        mma_commit(&oempty[so]);
-      }
-      if constexpr (RP > 0) {
-        const int g = ngroups, b = g % NTB;
-        if (ok) ok = mbar_wait(bfull, 0, wc);
-        if (ok && g >= NTB) ok = mbar_wait(&tempty[b], ((g / NTB) & 1) ^ 1, wc);
-        if (ok) {
-          tc_fence_after();
-          constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
-          const uint32_t pa = smem_u32(br), pb = pa + Cfg::BR_BYTES;
+        if constexpr (RP > 0) {
+          const int bs = ti % NBR, b = g_all % NTB;
+          if (ok) ok = mbar_wait(&bfull[bs], (ti / NBR) & 1, wc);
+          if (ok && g_all >= NTB) ok = mbar_wait(&tempty[b], ((g_all / NTB) & 1) ^ 1, wc);
+          if (ok) {
+            tc_fence_after();
+            constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
+            const uint32_t pa = smem_u32(br + bs * 2 * Cfg::BR_BYTES), pb = pa + Cfg::BR_BYTES;
 #pragma unroll
-          for (int kk = 0; kk < RP / 16; ++kk)
-            mma_f16(tmem + b * 128, smem_desc(pa + kk * 4096, 2048, 128, kSwNone),
-                    smem_desc(pb + kk * 4096, 2048, 128, kSwNone), idesc_br, kk != 0);
-          mma_commit(&tfull[b]);
+            for (int kk = 0; kk < RP / 16; ++kk)
+              mma_f16(tmem + b * 128, smem_desc(pa + kk * 4096, 2048, 128, kSwNone),
+                      smem_desc(pb + kk * 4096, 2048, 128, kSwNone), idesc_br, kk != 0);
+            mma_commit(&tfull[b]);
+            mma_commit(&bempty[bs]);
+            ++g_all;
+          }
         }
       }
       mma_commit(drain);
@@ -229,127 +278,148 @@ __global__ void __launch_bounds__(384, 1)
       mbar_wait(drain, 0, dc);
     }
     __syncwarp();
-  } else if (wid < 4) {
+  } else if (wid < 6) {
     // ------------------------------------------------------------- weight expanders + scales
-    const int e = static_cast<int>(threadIdx.x) - 64;  // 0..63
+    // Thread e (0..127) owns the 16-byte chunk j = e % 8 of rows e/8 + 16 i (i = 0..7): its source
+    // and destination offsets only step by constants (1024 and 2048 bytes).
+    const int e = static_cast<int>(threadIdx.x) - 64;
+    const int r0 = e >> 3, j = e & 7;
+    const int src0 = r0 * 64 + j * 8;
+    const int dst0 = (r0 >> 3) * 1024 + (r0 & 7) * 128 + ((j ^ (r0 & 7)) << 4);
     const uint32_t kX8 = 0x88888888u;
     bool ok = true;
-    for (int st = 0; st < nst && ok; ++st) {
-      const int sp = st % SP, so = st % SO;
-      ok = mbar_wait(&pfull[sp], (st / SP) & 1, wc);
-      if (ok && st >= SO) ok = mbar_wait(&oempty[so], ((st / SO) & 1) ^ 1, wc);
-      if (!ok) break;
-      const uint8_t* p = pring + sp * PSTAGE;
-      uint8_t* xb = oring + so * OSTAGE + OA_BYTES;
-#pragma unroll 4
-      for (int i = 0; i < 16; ++i) {
-        const int t = e + NEXP * i;
-        const int row = t >> 3, j = t & 7;
-        const uint2 pkd = *reinterpret_cast<const uint2*>(p + row * 64 + j * 8);
-        uint4 o;
-        o.x = (pkd.x ^ kX8) & 0x0F0F0F0Fu;
-        o.y = ((pkd.x >> 4) ^ kX8) & 0x0F0F0F0Fu;
-        o.z = (pkd.y ^ kX8) & 0x0F0F0F0Fu;
-        o.w = ((pkd.y >> 4) ^ kX8) & 0x0F0F0F0Fu;
-        *reinterpret_cast<uint4*>(xb + (row >> 3) * 1024 + (row & 7) * 128 + ((j ^ (row & 7)) << 4)) = o;
-      }
-      fence_proxy_async_smem();
-      mbar_arrive(&ofull[so]);
-      // group scales of this stage -> float32 slots for the epilogue
-      const float* psx = reinterpret_cast<const float*>(p + PB_BYTES);
-      const float* pcs = reinterpret_cast<const float*>(p + PB_BYTES + PSX_BYTES);
-      const __half* psw = reinterpret_cast<const __half*>(p + PB_BYTES + PSX_BYTES + PCS_BYTES);
-      for (int gi = 0; gi < gps && ok; ++gi) {
-        const int g = st * gps + gi;
-        if (g >= ngroups) break;
-        const int sl = g % NSL;
-        if (g >= NSL) ok = mbar_wait(&sempty[sl], ((g / NSL) & 1) ^ 1, wc);
+    int s = 0, g_all = 0;
+    for (int ti = 0; ti < my_tiles && ok; ++ti) {
+      for (int st = 0; st < nst && ok; ++st, ++s) {
+        const int gn = (st * gps + gps <= ngroups) ? gps : ngroups - st * gps;  // groups in this stage
+        const int ps = s % SP, xs = s % SX;
+        ok = mbar_wait(&pfull[ps], (s / SP) & 1, wc);
+        if (ok && s >= SX) ok = mbar_wait(&xempty[xs], ((s / SX) & 1) ^ 1, wc);
         if (!ok) break;
-        float* slot = slots + sl * SLOT_FLOATS;
+        const uint8_t* p = pring + ps * PSTAGE;
+        uint8_t* xb = xring + xs * X_BYTES;
+        uint2 pkd[8];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int i = e + NEXP * h;
-          slot[i] = __half2float(psw[gi * kGemmBN + i]);
-          slot[kGemmBN + i] = psx[gi * kBM + i];
-          slot[kGemmBN + kBM + i] = pcs[gi * kBM + i];
+        for (int i = 0; i < 8; ++i) pkd[i] = *reinterpret_cast<const uint2*>(p + src0 + i * 1024);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          uint4 o;
+          o.x = (pkd[i].x ^ kX8) & 0x0F0F0F0Fu;
+          o.y = ((pkd[i].x >> 4) ^ kX8) & 0x0F0F0F0Fu;
+          o.z = (pkd[i].y ^ kX8) & 0x0F0F0F0Fu;
+          o.w = ((pkd[i].y >> 4) ^ kX8) & 0x0F0F0F0Fu;
+          *reinterpret_cast<uint4*>(xb + dst0 + i * 2048) = o;
         }
-        mbar_arrive(&sfull[sl]);
+        fence_proxy_async_smem();
+        mbar_arrive(&xfull[xs]);
+        // group scales of this stage -> float32 slots for the epilogue
+        const float* psx = reinterpret_cast<const float*>(p + PB_BYTES);
+        const float* pcs = reinterpret_cast<const float*>(p + PB_BYTES + PSX_BYTES);
+        const __half* psw = reinterpret_cast<const __half*>(p + PB_BYTES + PSX_BYTES + PCS_BYTES);
+        for (int gi = 0; gi < gn && ok; ++gi, ++g_all) {
+          const int sl = g_all % NSL;
+          if (g_all >= NSL) ok = mbar_wait(&sempty[sl], ((g_all / NSL) & 1) ^ 1, wc);
+          if (!ok) break;
+          float* slot = slots + sl * SLOT_FLOATS;
+          slot[e] = __half2float(psw[gi * kGemmBN + e]);
+          slot[kGemmBN + e] = psx[gi * kBM + e];
+          slot[kGemmBN + kBM + e] = pcs[gi * kBM + e];
+          mbar_arrive(&sfull[sl]);
+        }
+        fence_proxy_async_smem();  // reads of the packed stage before the TMA refills it
+        mbar_arrive(&pempty[ps]);
       }
-      fence_proxy_async_smem();  // reads of the packed stage before the TMA refills it
-      mbar_arrive(&pempty[sp]);
     }
   } else {
     // ------------------------------------------------------------- epilogue
-    // Warps 4..11: warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 64 output
-    // columns [64*((w-4)/4), +64).
+    // Warps 6..13: warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 64 output
+    // columns [64*((w-6)/4), +64).
     const int quad = wid & 3;
     const int row = quad * 32 + static_cast<int>(lane);
-    const int m = m0 + row;
-    const int col0 = 64 * ((static_cast<int>(wid) - 4) >> 2);
+    const int col0 = 64 * ((static_cast<int>(wid) - 6) >> 2);
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
-    f2 acc[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) acc[i] = 0ull;
     bool ok = true;
-    const int ntot = ngroups + (RP > 0 ? 1 : 0);
-    for (int g = 0; g < ntot; ++g) {
-      const int b = g % NTB;
-      if (ok) ok = mbar_wait(&tfull[b], (g / NTB) & 1, wc);
-      tc_fence_after();
-      uint32_t v[64];
-      tmem_ld32(tlane + b * 128, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
-      tmem_ld32(tlane + b * 128 + 32, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
-      tmem_ld_wait();
-      tc_fence_before();
-      mbar_arrive(&tempty[b]);
-      if (g < ngroups) {
-        const int sl = g % NSL;
-        if (ok) ok = mbar_wait(&sfull[sl], (g / NSL) & 1, wc);
-        const float* slot = slots + sl * SLOT_FLOATS;
-        const float sxv = slot[kGemmBN + row];
-        const float alpha = sxv * 262144.0f;                       // 2^18 s_x (exact)
-        const float beta = -8.0f * sxv * slot[kGemmBN + kBM + row];  // -8 s_x S_a
-        const f2 al2 = pk(alpha, alpha), be2 = pk(beta, beta);
-        const float4* w4 = reinterpret_cast<const float4*>(slot + col0);
+    int g_all = 0, gs_all = 0;  // accumulator and scale-slot counters
+    for (int ti = 0; ti < my_tiles; ++ti) {
+      int m0, n0;
+      tile_mn(ti, m0, n0);
+      f2 acc[32];
 #pragma unroll
-        for (int i4 = 0; i4 < 16; ++i4) {
-          const float4 w = w4[i4];
-          const f2 t0 = fma2(pku(v[4 * i4], v[4 * i4 + 1]), al2, be2);
-          const f2 t1 = fma2(pku(v[4 * i4 + 2], v[4 * i4 + 3]), al2, be2);
-          acc[2 * i4] = fma2(t0, pk(w.x, w.y), acc[2 * i4]);
-          acc[2 * i4 + 1] = fma2(t1, pk(w.z, w.w), acc[2 * i4 + 1]);
-        }
-        mbar_arrive(&sempty[sl]);
-      } else {
+      for (int i = 0; i < 32; ++i) acc[i] = 0ull;
+      const int ntot = ngroups + (RP > 0 ? 1 : 0);
+      for (int g = 0; g < ntot; ++g, ++g_all) {
+        const int b = g_all % NTB;
+        if (ok) ok = mbar_wait(&tfull[b], (g_all / NTB) & 1, wc);
+        tc_fence_after();
+        if (g < ngroups) {
+          const int sl = gs_all % NSL;
+          if (ok) ok = mbar_wait(&sfull[sl], (gs_all / NSL) & 1, wc);
+          const float* slot = slots + sl * SLOT_FLOATS;
+          const float sxv = slot[kGemmBN + row];
+          const float alpha = sxv * 262144.0f;                         // 2^18 s_x (exact)
+          const float beta = -8.0f * sxv * slot[kGemmBN + kBM + row];  // -8 s_x S_a
+          const f2 al2 = pk(alpha, alpha), be2 = pk(beta, beta);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) acc[i] = add2(acc[i], pku(v[2 * i], v[2 * i + 1]));
-      }
-    }
-    if (ok && m < a.M) {
-      const int nb = n0 + col0;
-      if (a.y_f32) {
-        float* yr = static_cast<float*>(a.Y) + static_cast<size_t>(m) * a.N + nb;
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          if (nb + c8 * 8 < a.N) {
-            reinterpret_cast<float4*>(yr + c8 * 8)[0] =
-                make_float4(lo_f(acc[4 * c8]), hi_f(acc[4 * c8]), lo_f(acc[4 * c8 + 1]), hi_f(acc[4 * c8 + 1]));
-            reinterpret_cast<float4*>(yr + c8 * 8)[1] = make_float4(lo_f(acc[4 * c8 + 2]), hi_f(acc[4 * c8 + 2]),
-                                                                    lo_f(acc[4 * c8 + 3]), hi_f(acc[4 * c8 + 3]));
-          }
-        }
-      } else {
-        __nv_bfloat16* yr = static_cast<__nv_bfloat16*>(a.Y) + static_cast<size_t>(m) * a.N + nb;
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          if (nb + c8 * 8 < a.N) {
-            uint32_t w[4];
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              __nv_bfloat162 h2 = __floats2bfloat162_rn(lo_f(acc[4 * c8 + t]), hi_f(acc[4 * c8 + t]));
-              w[t] = *reinterpret_cast<uint32_t*>(&h2);
+          for (int c = 0; c < 2; ++c) {
+            uint32_t v[32];
+            tmem_ld32(tlane + b * 128 + c * 32, v);
+            tmem_ld_wait();
+            if (c == 1) {
+              tc_fence_before();
+              mbar_arrive(&tempty[b]);
             }
-            *reinterpret_cast<uint4*>(yr + c8 * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+            const float4* w4 = reinterpret_cast<const float4*>(slot + col0 + c * 32);
+#pragma unroll
+            for (int i4 = 0; i4 < 8; ++i4) {
+              const float4 w = w4[i4];
+              const f2 t0 = fma2(pku(v[4 * i4], v[4 * i4 + 1]), al2, be2);
+              const f2 t1 = fma2(pku(v[4 * i4 + 2], v[4 * i4 + 3]), al2, be2);
+              acc[16 * c + 2 * i4] = fma2(t0, pk(w.x, w.y), acc[16 * c + 2 * i4]);
+              acc[16 * c + 2 * i4 + 1] = fma2(t1, pk(w.z, w.w), acc[16 * c + 2 * i4 + 1]);
+            }
+          }
+          mbar_arrive(&sempty[sl]);
+          ++gs_all;
+        } else {
+#pragma unroll
+          for (int c = 0; c < 2; ++c) {
+            uint32_t v[32];
+            tmem_ld32(tlane + b * 128 + c * 32, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) acc[16 * c + i] = add2(acc[16 * c + i], pku(v[2 * i], v[2 * i + 1]));
+          }
+          tc_fence_before();
+          mbar_arrive(&tempty[b]);
+        }
+      }
+      const int m = m0 + row;
+      if (ok && m < a.M) {
+        const int nb = n0 + col0;
+        if (a.y_f32) {
+          float* yr = static_cast<float*>(a.Y) + static_cast<size_t>(m) * a.N + nb;
+#pragma unroll
+          for (int c8 = 0; c8 < 8; ++c8) {
+            if (nb + c8 * 8 < a.N) {
+              reinterpret_cast<float4*>(yr + c8 * 8)[0] =
+                  make_float4(lo_f(acc[4 * c8]), hi_f(acc[4 * c8]), lo_f(acc[4 * c8 + 1]), hi_f(acc[4 * c8 + 1]));
+              reinterpret_cast<float4*>(yr + c8 * 8)[1] = make_float4(lo_f(acc[4 * c8 + 2]), hi_f(acc[4 * c8 + 2]),
+                                                                      lo_f(acc[4 * c8 + 3]), hi_f(acc[4 * c8 + 3]));
+            }
+          }
+        } else {
+          __nv_bfloat16* yr = static_cast<__nv_bfloat16*>(a.Y) + static_cast<size_t>(m) * a.N + nb;
+#pragma unroll
+          for (int c8 = 0; c8 < 8; ++c8) {
+            if (nb + c8 * 8 < a.N) {
+              uint32_t w[4];
+#pragma unroll
+              for (int t = 0; t < 4; ++t) {
+                __nv_bfloat162 h2 = __floats2bfloat162_rn(lo_f(acc[4 * c8 + t]), hi_f(acc[4 * c8 + t]));
+                w[t] = *reinterpret_cast<uint32_t*>(&h2);
+              }
+              *reinterpret_cast<uint4*>(yr + c8 * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+            }
           }
         }
       }
@@ -371,6 +441,8 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
   a.N = h.N;
   a.K = h.K;
   a.G = h.G;
+  a.m_tiles = (M + kBM - 1) / kBM;
+  a.n_tiles = (h.N + kGemmBN - 1) / kGemmBN;
   a.Y = Y;
   a.y_f32 = y_f32 ? 1 : 0;
   a.err = h.err;
@@ -381,10 +453,11 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  dim3 grid((h.N + kGemmBN - 1) / kGemmBN, (M + kBM - 1) / kBM, 1);
+  const int ntiles = a.m_tiles * a.n_tiles;
+  const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
   const CUtensorMap& ph = (RP > 0) ? am.ph_map : am.qx_map;
   const CUtensorMap& bh = (RP > 0) ? h.Bh_map : am.qx_map;
-  gemm_kernel<RP><<<grid, 384, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.sx_map, am.cs_map, h.sw_map, ph, bh, a);
+  gemm_kernel<RP><<<grid, 448, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.sx_map, am.cs_map, h.sw_map, ph, bh, a);
   return cudaGetLastError();
 }
 
