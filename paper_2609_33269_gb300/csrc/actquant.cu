@@ -144,11 +144,11 @@ __global__ void __launch_bounds__(320, 1)
       mbar_init(&empty[i], 1);
     }
     mbar_init(proj_done, 1);
-    mbar_init(arec_ready, 256);
+    mbar_init(arec_ready, 8);   // epilogue warps
     mbar_init(drain, 1);
     for (int i = 0; i < kNumRec; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], 128);
+      mbar_init(&tempty[i], 4);   // the four warps of one chunk parity
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -362,7 +362,7 @@ __global__ void __launch_bounds__(320, 1)
         for (int col = 3 * RP; col < Cfg::KU3; col += 8) put8(col, z);
       }
       fence_proxy_async_smem();
-      mbar_arrive(arec_ready);
+      warp_arrive(arec_ready);
     }
 
     // -- pass 2: remainder and quantization; this warp takes the chunks of its parity
@@ -378,7 +378,7 @@ __global__ void __launch_bounds__(320, 1)
         tmem_ld32(tlane + 128 + 64 * b + 32, r1);
         tmem_ld_wait();
         tc_fence_before();
-        mbar_arrive(&tempty[b]);
+        warp_arrive(&tempty[b]);
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           xp[i] = __uint_as_float(r0[i]);

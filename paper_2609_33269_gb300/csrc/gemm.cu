@@ -23,7 +23,8 @@
 // (activation tiles, packed weights with the group scales, expanded weights, branch tiles, scale
 // slots, TMEM accumulators) runs continuously across tiles, so loads for the next tile overlap
 // the epilogue of the current one.  448 threads: warp 0 TMA producer, warp 1 MMA issuer and TMEM
-// owner, warps 2..5 expand weight nibbles and stage the group scales, warps 6..13 epilogue
+// owner, warps 2..5 expand weight nibbles and stage the group scales (two teams taking alternate
+// stages), warps 6..13 epilogue
 // (thread = output row x 64 columns, packed f32x2).  Every ring has exactly one waiting role per
 // side, which waits for each phase in turn.
 #include "internal.h"
@@ -41,12 +42,16 @@ struct GemmArgs {
   uint64_t timeout_ns;
 };
 
-constexpr int SX = 3;     // expanded-weight stages (expanders -> MMA)
-constexpr int NSL = 8;    // scale slots (one group each)
-constexpr int NTB = 4;    // TMEM accumulator buffers (128 columns each)
+// Two expander teams take alternate stages.  Every ring a team touches therefore has an even
+// number of slots, so each slot always belongs to the same team and every waiter sees each of its
+// slot's phases in turn.
+constexpr int SX = 2;     // expanded-weight stages (expanders -> MMA): one per team
+constexpr int NSS = 2;    // scale slots, one per stage and team (up to 4 groups each)
+constexpr int NTB = 2;    // TMEM accumulator buffers, one per unit (2 x 128 columns each)
 constexpr int NBR = 2;    // branch-operand stages (one per tile)
-constexpr int NEXP = 128; // expander threads
-constexpr int NEPI = 256; // epilogue threads
+constexpr int NTEAM = 64; // threads per expander team
+constexpr int NTEAMW = 2; // warps per expander team
+constexpr int NEPIW = 8;  // epilogue warps (2 per row quadrant, 64 columns each)
 constexpr int A_BYTES = kBM * kGemmKS;            // 16 KB, 128-byte swizzle
 constexpr int X_BYTES = kGemmBN * kGemmKS;        // 16 KB, 128-byte swizzle
 constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;   // 8 KB packed weights
@@ -54,15 +59,16 @@ constexpr int PSX_BYTES = 4 * kBM * 4;            // up to 4 groups x 128 f32 ac
 constexpr int PCS_BYTES = 4 * kBM * 4;            // up to 4 groups x 128 f32 activation code sums
 constexpr int PSW_BYTES = 4 * kGemmBN * 2;        // up to 4 groups x 128 f16 weight scales
 constexpr int PSTAGE = PB_BYTES + PSX_BYTES + PCS_BYTES + PSW_BYTES;
-constexpr int SLOT_FLOATS = kGemmBN + 2 * kBM;    // s_w (f32) | s_x | code sums
+constexpr int GSLOT = kGemmBN + 2 * kBM;         // per group: s_w (f32) | s_x | code sums
+constexpr int SLOT_FLOATS = 4 * GSLOT;           // one stage (up to 4 groups)
 
 template <int RP>
 struct GemmCfg {
-  static constexpr int SA = RP <= 48 ? 4 : 3;                     // activation stages (TMA -> MMA)
-  static constexpr int SP = RP <= 16 ? 6 : (RP <= 32 ? 5 : 4);    // packed-weight stages
+  static constexpr int SA = 4;                  // activation stages (TMA -> MMA)
+  static constexpr int SP = RP <= 32 ? 6 : 4;   // packed-weight stages (even, see the teams)
   static constexpr int BR_BYTES = RP * kBM * 2;   // p_hat tile (and the B_hat tile), RP/8 boxes of 2 KB
-  static constexpr int NBAR = 2 * SA + 2 * SX + 2 * SP + 2 * NSL + 2 * NTB + 2 * NBR + 1;
-  static constexpr int SMEM = 1024 + SA * A_BYTES + SX * X_BYTES + SP * PSTAGE + NSL * SLOT_FLOATS * 4 +
+  static constexpr int NBAR = 2 * SA + 2 * SX + 2 * SP + 2 * NSS + 2 * NTB + 2 * NBR + 1;
+  static constexpr int SMEM = 1024 + SA * A_BYTES + SX * X_BYTES + SP * PSTAGE + NSS * SLOT_FLOATS * 4 +
                               NBR * 2 * BR_BYTES + NBAR * 8 + 16;
   static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 };
@@ -103,7 +109,7 @@ __global__ void __launch_bounds__(448, 1)
   uint8_t* xring = aring + SA * A_BYTES;           // SX x 16 KB, 1024-aligned
   uint8_t* pring = xring + SX * X_BYTES;           // SP x (weights packed | s_x | code sums | s_w)
   float* slots = reinterpret_cast<float*>(pring + SP * PSTAGE);
-  uint8_t* br = reinterpret_cast<uint8_t*>(slots + NSL * SLOT_FLOATS);  // NBR x (p_hat | B_hat)
+  uint8_t* br = reinterpret_cast<uint8_t*>(slots + NSS * SLOT_FLOATS);  // NBR x (p_hat | B_hat)
   uint64_t* bars = reinterpret_cast<uint64_t*>(br + NBR * 2 * Cfg::BR_BYTES);
   uint64_t* afull = bars;
   uint64_t* aempty = afull + SA;
@@ -112,8 +118,8 @@ __global__ void __launch_bounds__(448, 1)
   uint64_t* pfull = xempty + SX;
   uint64_t* pempty = pfull + SP;
   uint64_t* sfull = pempty + SP;
-  uint64_t* sempty = sfull + NSL;
-  uint64_t* tfull = sempty + NSL;
+  uint64_t* sempty = sfull + NSS;
+  uint64_t* tfull = sempty + NSS;
   uint64_t* tempty = tfull + NTB;
   uint64_t* bfull = tempty + NTB;
   uint64_t* bempty = bfull + NBR;
@@ -143,20 +149,20 @@ __global__ void __launch_bounds__(448, 1)
       mbar_init(&aempty[i], 1);
     }
     for (int i = 0; i < SX; ++i) {
-      mbar_init(&xfull[i], NEXP);
+      mbar_init(&xfull[i], NTEAMW);
       mbar_init(&xempty[i], 1);
     }
     for (int i = 0; i < SP; ++i) {
       mbar_init(&pfull[i], 1);
-      mbar_init(&pempty[i], NEXP);
+      mbar_init(&pempty[i], NTEAMW);
     }
-    for (int i = 0; i < NSL; ++i) {
-      mbar_init(&sfull[i], NEXP);
-      mbar_init(&sempty[i], NEPI);
+    for (int i = 0; i < NSS; ++i) {
+      mbar_init(&sfull[i], NTEAMW);
+      mbar_init(&sempty[i], NEPIW);
     }
     for (int i = 0; i < NTB; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], NEPI);
+      mbar_init(&tempty[i], NEPIW);
     }
     for (int i = 0; i < NBR; ++i) {
       mbar_init(&bfull[i], 1);
@@ -224,51 +230,52 @@ __global__ void __launch_bounds__(448, 1)
     }
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
+    // The epilogue consumes accumulators in units of two groups (one TMEM buffer of 2 x 128
+    // columns); a unit never straddles a stage because a stage holds an even number of groups.
+    // One tcgen05 fence per unit: fences and commits cost far more than an MMA issue.
     if (lane == 0) {
       bool ok = true;
       constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
-      int s = 0, g_all = 0;  // running stage and accumulator counters
+      int s = 0, u_all = 0;  // running stage and accumulator-unit counters
       for (int ti = 0; ti < my_tiles && ok; ++ti) {
         for (int st = 0; st < nst && ok; ++st, ++s) {
+          const int gn = (st * gps + gps <= ngroups) ? gps : ngroups - st * gps;  // groups in this stage
           const int as = s % SA, xs = s % SX;
           ok = mbar_wait(&afull[as], (s / SA) & 1, wc);
           if (ok) ok = mbar_wait(&xfull[xs], (s / SX) & 1, wc);
           if (!ok) break;
-          tc_fence_after();
           const uint32_t aa = smem_u32(aring + as * A_BYTES), xa = smem_u32(xring + xs * X_BYTES);
-          for (int gi = 0; gi < gps && ok; ++gi) {
-            const int g = st * gps + gi;
-            if (g >= ngroups) break;
-            const int b = g_all % NTB;
-            if (g_all >= NTB) ok = mbar_wait(&tempty[b], ((g_all / NTB) & 1) ^ 1, wc);
+          for (int g0 = 0; g0 < gn && ok; g0 += 2, ++u_all) {
+            const int ub = u_all % NTB;
+            if (u_all >= NTB) ok = mbar_wait(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
             if (!ok) break;
             tc_fence_after();
-            for (int kk = 0; kk < G / 32; ++kk) {
-              const uint32_t off = static_cast<uint32_t>((gi * (G / 32) + kk) * 32);
-              mma_f8f6f4(tmem + b * 128, smem_desc(aa + off, 16, 1024, kSw128),
-                         smem_desc(xa + off, 16, 1024, kSw128), idesc, kk != 0);
-            }
-            mma_commit(&tfull[b]);
-            ++g_all;
+            for (int gi = g0; gi < gn && gi < g0 + 2; ++gi)
+              for (int kk = 0; kk < G / 32; ++kk) {
+                const uint32_t off = static_cast<uint32_t>((gi * (G / 32) + kk) * 32);
+                mma_f8f6f4(tmem + ub * 256 + (gi - g0) * 128, smem_desc(aa + off, 16, 1024, kSw128),
+                           smem_desc(xa + off, 16, 1024, kSw128), idesc, kk != 0);
+              }
+            mma_commit(&tfull[ub]);
           }
           mma_commit(&aempty[as]);
           mma_commit(&xempty[xs]);
         }
         if constexpr (RP > 0) {
-          const int bs = ti % NBR, b = g_all % NTB;
+          const int bs = ti % NBR, ub = u_all % NTB;
           if (ok) ok = mbar_wait(&bfull[bs], (ti / NBR) & 1, wc);
-          if (ok && g_all >= NTB) ok = mbar_wait(&tempty[b], ((g_all / NTB) & 1) ^ 1, wc);
+          if (ok && u_all >= NTB) ok = mbar_wait(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
           if (ok) {
             tc_fence_after();
             constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
             const uint32_t pa = smem_u32(br + bs * 2 * Cfg::BR_BYTES), pb = pa + Cfg::BR_BYTES;
 #pragma unroll
             for (int kk = 0; kk < RP / 16; ++kk)
-              mma_f16(tmem + b * 128, smem_desc(pa + kk * 4096, 2048, 128, kSwNone),
+              mma_f16(tmem + ub * 256, smem_desc(pa + kk * 4096, 2048, 128, kSwNone),
                       smem_desc(pb + kk * 4096, 2048, 128, kSwNone), idesc_br, kk != 0);
-            mma_commit(&tfull[b]);
+            mma_commit(&tfull[ub]);
             mma_commit(&bempty[bs]);
-            ++g_all;
+            ++u_all;
           }
         }
       }
@@ -280,54 +287,62 @@ __global__ void __launch_bounds__(448, 1)
     __syncwarp();
   } else if (wid < 6) {
     // ------------------------------------------------------------- weight expanders + scales
-    // Thread e (0..127) owns the 16-byte chunk j = e % 8 of rows e/8 + 16 i (i = 0..7): its source
-    // and destination offsets only step by constants (1024 and 2048 bytes).
-    const int e = static_cast<int>(threadIdx.x) - 64;
+    // Team t (warps 2+2t, 3+2t) takes the stages s with s % 2 == t.  Thread e (0..63) of a team
+    // owns the 16-byte chunk j = e % 8 of rows e/8 + 8 i (i = 0..15): its source and destination
+    // offsets only step by constants (512 and 1024 bytes).
+    const int team = (static_cast<int>(wid) - 2) >> 1;
+    const int e = (static_cast<int>(threadIdx.x) - 64) & (NTEAM - 1);
     const int r0 = e >> 3, j = e & 7;
     const int src0 = r0 * 64 + j * 8;
-    const int dst0 = (r0 >> 3) * 1024 + (r0 & 7) * 128 + ((j ^ (r0 & 7)) << 4);
+    const int dst0 = r0 * 128 + ((j ^ r0) << 4);
     const uint32_t kX8 = 0x88888888u;
     bool ok = true;
-    int s = 0, g_all = 0;
+    int s = 0;
     for (int ti = 0; ti < my_tiles && ok; ++ti) {
       for (int st = 0; st < nst && ok; ++st, ++s) {
+        if ((s & 1) != team) continue;
         const int gn = (st * gps + gps <= ngroups) ? gps : ngroups - st * gps;  // groups in this stage
-        const int ps = s % SP, xs = s % SX;
+        const int ps = s % SP, xs = team;
         ok = mbar_wait(&pfull[ps], (s / SP) & 1, wc);
         if (ok && s >= SX) ok = mbar_wait(&xempty[xs], ((s / SX) & 1) ^ 1, wc);
         if (!ok) break;
         const uint8_t* p = pring + ps * PSTAGE;
         uint8_t* xb = xring + xs * X_BYTES;
-        uint2 pkd[8];
+        uint2 pkd[16];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) pkd[i] = *reinterpret_cast<const uint2*>(p + src0 + i * 1024);
+        for (int i = 0; i < 16; ++i) pkd[i] = *reinterpret_cast<const uint2*>(p + src0 + i * 512);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
+        for (int i = 0; i < 16; ++i) {
           uint4 o;
           o.x = (pkd[i].x ^ kX8) & 0x0F0F0F0Fu;
           o.y = ((pkd[i].x >> 4) ^ kX8) & 0x0F0F0F0Fu;
           o.z = (pkd[i].y ^ kX8) & 0x0F0F0F0Fu;
           o.w = ((pkd[i].y >> 4) ^ kX8) & 0x0F0F0F0Fu;
-          *reinterpret_cast<uint4*>(xb + dst0 + i * 2048) = o;
+          *reinterpret_cast<uint4*>(xb + dst0 + i * 1024) = o;
         }
         fence_proxy_async_smem();
-        mbar_arrive(&xfull[xs]);
-        // group scales of this stage -> float32 slots for the epilogue
+        warp_arrive(&xfull[xs]);
+        // group scales of this stage -> the team's float32 scale slot for the epilogue
         const float* psx = reinterpret_cast<const float*>(p + PB_BYTES);
         const float* pcs = reinterpret_cast<const float*>(p + PB_BYTES + PSX_BYTES);
         const __half* psw = reinterpret_cast<const __half*>(p + PB_BYTES + PSX_BYTES + PCS_BYTES);
-        for (int gi = 0; gi < gn && ok; ++gi, ++g_all) {
-          const int sl = g_all % NSL;
-          if (g_all >= NSL) ok = mbar_wait(&sempty[sl], ((g_all / NSL) & 1) ^ 1, wc);
-          if (!ok) break;
-          float* slot = slots + sl * SLOT_FLOATS;
-          slot[e] = __half2float(psw[gi * kGemmBN + e]);
-          slot[kGemmBN + e] = psx[gi * kBM + e];
-          slot[kGemmBN + kBM + e] = pcs[gi * kBM + e];
-          mbar_arrive(&sfull[sl]);
+        const int ss = team;
+        if (s >= NSS) ok = mbar_wait(&sempty[ss], ((s / NSS) & 1) ^ 1, wc);
+        if (!ok) break;
+        float* slot = slots + ss * SLOT_FLOATS;
+        for (int gi = 0; gi < gn; ++gi) {
+          float* sg = slot + gi * GSLOT;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int i = e + NTEAM * h;
+            sg[i] = __half2float(psw[gi * kGemmBN + i]);
+            sg[kGemmBN + i] = psx[gi * kBM + i];
+            sg[kGemmBN + kBM + i] = pcs[gi * kBM + i];
+          }
         }
+        warp_arrive(&sfull[ss]);
         fence_proxy_async_smem();  // reads of the packed stage before the TMA refills it
-        mbar_arrive(&pempty[ps]);
+        warp_arrive(&pempty[ps]);
       }
     }
   } else {
@@ -339,59 +354,67 @@ __global__ void __launch_bounds__(448, 1)
     const int col0 = 64 * ((static_cast<int>(wid) - 6) >> 2);
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
     bool ok = true;
-    int g_all = 0, gs_all = 0;  // accumulator and scale-slot counters
+    int u_all = 0, s = 0;  // accumulator-unit and stage counters
     for (int ti = 0; ti < my_tiles; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
       f2 acc[32];
 #pragma unroll
       for (int i = 0; i < 32; ++i) acc[i] = 0ull;
-      const int ntot = ngroups + (RP > 0 ? 1 : 0);
-      for (int g = 0; g < ntot; ++g, ++g_all) {
-        const int b = g_all % NTB;
-        if (ok) ok = mbar_wait(&tfull[b], (g_all / NTB) & 1, wc);
-        tc_fence_after();
-        if (g < ngroups) {
-          const int sl = gs_all % NSL;
-          if (ok) ok = mbar_wait(&sfull[sl], (gs_all / NSL) & 1, wc);
-          const float* slot = slots + sl * SLOT_FLOATS;
-          const float sxv = slot[kGemmBN + row];
-          const float alpha = sxv * 262144.0f;                         // 2^18 s_x (exact)
-          const float beta = -8.0f * sxv * slot[kGemmBN + kBM + row];  // -8 s_x S_a
-          const f2 al2 = pk(alpha, alpha), be2 = pk(beta, beta);
+      for (int st = 0; st < nst; ++st, ++s) {
+        const int gn = (st * gps + gps <= ngroups) ? gps : ngroups - st * gps;  // groups in this stage
+        const int ss = s % NSS;
+        if (ok) ok = mbar_wait(&sfull[ss], (s / NSS) & 1, wc);
+        const float* slot = slots + ss * SLOT_FLOATS;
+        for (int g0 = 0; g0 < gn; g0 += 2, ++u_all) {
+          const int ub = u_all % NTB;
+          const int nmem = (g0 + 1 < gn) ? 2 : 1;
+          if (ok) ok = mbar_wait(&tfull[ub], (u_all / NTB) & 1, wc);
+          tc_fence_after();
+          for (int mi = 0; mi < nmem; ++mi) {
+            const float* sg = slot + (g0 + mi) * GSLOT;
+            const float sxv = sg[kGemmBN + row];
+            const float alpha = sxv * 262144.0f;                       // 2^18 s_x (exact)
+            const float beta = -8.0f * sxv * sg[kGemmBN + kBM + row];  // -8 s_x S_a
+            const f2 al2 = pk(alpha, alpha), be2 = pk(beta, beta);
 #pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            uint32_t v[32];
-            tmem_ld32(tlane + b * 128 + c * 32, v);
-            tmem_ld_wait();
-            if (c == 1) {
-              tc_fence_before();
-              mbar_arrive(&tempty[b]);
-            }
-            const float4* w4 = reinterpret_cast<const float4*>(slot + col0 + c * 32);
+            for (int c = 0; c < 2; ++c) {
+              uint32_t v[32];
+              tmem_ld32(tlane + ub * 256 + mi * 128 + c * 32, v);
+              tmem_ld_wait();
+              if (mi == nmem - 1 && c == 1) {
+                tc_fence_before();
+                warp_arrive(&tempty[ub]);
+              }
+              const float4* w4 = reinterpret_cast<const float4*>(sg + col0 + c * 32);
 #pragma unroll
-            for (int i4 = 0; i4 < 8; ++i4) {
-              const float4 w = w4[i4];
-              const f2 t0 = fma2(pku(v[4 * i4], v[4 * i4 + 1]), al2, be2);
-              const f2 t1 = fma2(pku(v[4 * i4 + 2], v[4 * i4 + 3]), al2, be2);
-              acc[16 * c + 2 * i4] = fma2(t0, pk(w.x, w.y), acc[16 * c + 2 * i4]);
-              acc[16 * c + 2 * i4 + 1] = fma2(t1, pk(w.z, w.w), acc[16 * c + 2 * i4 + 1]);
+              for (int i4 = 0; i4 < 8; ++i4) {
+                const float4 w = w4[i4];
+                const f2 t0 = fma2(pku(v[4 * i4], v[4 * i4 + 1]), al2, be2);
+                const f2 t1 = fma2(pku(v[4 * i4 + 2], v[4 * i4 + 3]), al2, be2);
+                acc[16 * c + 2 * i4] = fma2(t0, pk(w.x, w.y), acc[16 * c + 2 * i4]);
+                acc[16 * c + 2 * i4 + 1] = fma2(t1, pk(w.z, w.w), acc[16 * c + 2 * i4 + 1]);
+              }
             }
           }
-          mbar_arrive(&sempty[sl]);
-          ++gs_all;
-        } else {
-#pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            uint32_t v[32];
-            tmem_ld32(tlane + b * 128 + c * 32, v);
-            tmem_ld_wait();
-#pragma unroll
-            for (int i = 0; i < 16; ++i) acc[16 * c + i] = add2(acc[16 * c + i], pku(v[2 * i], v[2 * i + 1]));
-          }
-          tc_fence_before();
-          mbar_arrive(&tempty[b]);
         }
+        warp_arrive(&sempty[ss]);
+      }
+      if constexpr (RP > 0) {
+        const int ub = u_all % NTB;
+        if (ok) ok = mbar_wait(&tfull[ub], (u_all / NTB) & 1, wc);
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tlane + ub * 256 + c * 32, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) acc[16 * c + i] = add2(acc[16 * c + i], pku(v[2 * i], v[2 * i + 1]));
+        }
+        tc_fence_before();
+        warp_arrive(&tempty[ub]);
+        ++u_all;
       }
       const int m = m0 + row;
       if (ok && m < a.M) {
