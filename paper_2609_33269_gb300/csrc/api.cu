@@ -159,10 +159,11 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
 
   const size_t b_qw = qwam::up256(static_cast<size_t>(h.N_pad) * (K / 2));
   const size_t b_sw = qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
+  const size_t b_s32 = qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 4);
   const size_t b_bh = qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2);
   const size_t b_ut = qwam::up256(static_cast<size_t>(2 * h.r_pad) * K * 2);
   const size_t b_u3 = qwam::up256(static_cast<size_t>(K) * h.ku3 * 2);
-  const size_t total = b_qw + b_sw + b_bh + b_ut + b_u3 + 256;
+  const size_t total = b_qw + b_sw + b_s32 + b_bh + b_ut + b_u3 + 256;
   if (cudaMalloc(&h.block, total) != cudaSuccess) {
     cudaGetLastError();
     delete hs;
@@ -171,17 +172,19 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   uint8_t* p = static_cast<uint8_t*>(h.block);
   h.qw = p;
   h.sw = reinterpret_cast<__half*>(p + b_qw);
-  h.Bh = reinterpret_cast<__half*>(p + b_qw + b_sw);
-  h.ucat_t = reinterpret_cast<__nv_bfloat16*>(p + b_qw + b_sw + b_bh);
-  h.ucat3 = reinterpret_cast<__nv_bfloat16*>(p + b_qw + b_sw + b_bh + b_ut);
-  h.err = reinterpret_cast<int*>(p + b_qw + b_sw + b_bh + b_ut + b_u3);
+  h.sw32 = reinterpret_cast<float*>(p + b_qw + b_sw);
+  uint8_t* q = p + b_qw + b_sw + b_s32;
+  h.Bh = reinterpret_cast<__half*>(q);
+  h.ucat_t = reinterpret_cast<__nv_bfloat16*>(q + b_bh);
+  h.ucat3 = reinterpret_cast<__nv_bfloat16*>(q + b_bh + b_ut);
+  h.err = reinterpret_cast<int*>(q + b_bh + b_ut + b_u3);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   bool ok = true;
   ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kGemmKS / 2, qwam::kBM,
                         CU_TENSOR_MAP_SWIZZLE_NONE);
-  ok &= qwam::encode_2d(&h.sw_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.sw, N, K / group,
-                        static_cast<uint64_t>(h.N_pad) * 2, qwam::kGemmBN, qwam::kGemmKS / group,
+  ok &= qwam::encode_2d(&h.sw32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, h.sw32, N, K / group,
+                        static_cast<uint64_t>(h.N_pad) * 4, qwam::kGemmBN, qwam::kGemmKS / group,
                         CU_TENSOR_MAP_SWIZZLE_NONE);
   if (h.r_pad > 0) {
     ok &= qwam::encode_2d(&h.Bh_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,

@@ -20,13 +20,23 @@
 // epilogue adds with scale 1.
 //
 // Persistent CTAs (one per SM) walk output tiles of 128 x 128 with a static stride; every ring
-// (activation tiles, packed weights with the group scales, expanded weights, branch tiles, scale
-// slots, TMEM accumulators) runs continuously across tiles, so loads for the next tile overlap
-// the epilogue of the current one.  448 threads: warp 0 TMA producer, warp 1 MMA issuer and TMEM
-// owner, warps 2..5 expand weight nibbles and stage the group scales (two teams taking alternate
-// stages), warps 6..13 epilogue
-// (thread = output row x 64 columns, packed f32x2).  Every ring has exactly one waiting role per
-// side, which waits for each phase in turn.
+// runs continuously across tiles, so loads for the next tile overlap the epilogue of the current
+// one.  640 threads in five warpgroups:
+//   warpgroup 0 (56 registers): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2-3
+//     expand weight nibbles into the operand stage;
+//   warpgroups 1-4 (104 registers): warps 4..19 epilogue.  A warp owns 32 rows x 32 columns of
+//     the tile; TMEM is read with the 16x256b shape, so a thread holds 4 rows x 8 columns (as
+//     packed f32x2 pairs) and needs only 8 column scales s_w and 4 row scales (alpha, beta) per
+//     group: the scales reaching registers, not the arithmetic, bound a one-row-per-thread
+//     epilogue.  The floor is the FMA pipe: two operations per output and group.
+// Rings (each waiter waits for every phase of its slots in turn):
+//   O  operand stage = activation codes (TMA) + expanded weights (expanders)  -> MMA     SO slots
+//   P  packed weights (-> expanders) + s_x, S_a, s_w of the stage (-> epilogue)         SP slots
+//   T  TMEM accumulators, units of two groups (2 x 128 columns)  MMA -> epilogue        NTB units
+//   B  p_hat / B_hat tiles  TMA -> MMA, loaded after the tile's stages                   one per tile
+// Every barrier operation costs on the order of 100 cycles, so each role touches as few as
+// possible per stage: the MMA warp waits twice and commits twice, the expanders wait twice and
+// arrive once, the epilogue waits twice and arrives twice.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -42,34 +52,29 @@ struct GemmArgs {
   uint64_t timeout_ns;
 };
 
-// Two expander teams take alternate stages.  Every ring a team touches therefore has an even
-// number of slots, so each slot always belongs to the same team and every waiter sees each of its
-// slot's phases in turn.
-constexpr int SX = 2;     // expanded-weight stages (expanders -> MMA): one per team
-constexpr int NSS = 2;    // scale slots, one per stage and team (up to 4 groups each)
-constexpr int NTB = 2;    // TMEM accumulator buffers, one per unit (2 x 128 columns each)
-constexpr int NBR = 2;    // branch-operand stages (one per tile)
-constexpr int NTEAM = 64; // threads per expander team
-constexpr int NTEAMW = 2; // warps per expander team
-constexpr int NEPIW = 8;  // epilogue warps (2 per row quadrant, 64 columns each)
+constexpr int kThreads = 640;
+constexpr int kLaunchRegs = 96;  // 65536 / 640 rounded down to a multiple of 8
+constexpr int kRegsCtl = 56;     // warpgroup 0
+constexpr int kRegsEpi = 104;    // warpgroups 1-4
+static_assert(128 * kRegsCtl + 512 * kRegsEpi <= kThreads * kLaunchRegs, "register split above the launch allocation");
+constexpr int SO = 3;     // operand stages
+constexpr int SP = 6;     // packed-weight + scale stages
+constexpr int NTB = 2;    // TMEM accumulator units (2 x 128 columns each)
+constexpr int NBR = 1;    // branch-operand stages (one per tile)
+constexpr int NXW = 2;    // expander warps
+constexpr int NEPIW = 16; // epilogue warps (4 per row quadrant, 32 columns each)
 constexpr int A_BYTES = kBM * kGemmKS;            // 16 KB, 128-byte swizzle
 constexpr int X_BYTES = kGemmBN * kGemmKS;        // 16 KB, 128-byte swizzle
+constexpr int OSTAGE = A_BYTES + X_BYTES;
 constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;   // 8 KB packed weights
-constexpr int PSX_BYTES = 4 * kBM * 4;            // up to 4 groups x 128 f32 activation scales
-constexpr int PCS_BYTES = 4 * kBM * 4;            // up to 4 groups x 128 f32 activation code sums
-constexpr int PSW_BYTES = 4 * kGemmBN * 2;        // up to 4 groups x 128 f16 weight scales
-constexpr int PSTAGE = PB_BYTES + PSX_BYTES + PCS_BYTES + PSW_BYTES;
-constexpr int GSLOT = kGemmBN + 2 * kBM;         // per group: s_w (f32) | s_x | code sums
-constexpr int SLOT_FLOATS = 4 * GSLOT;           // one stage (up to 4 groups)
+constexpr int PSC_BYTES = 4 * 128 * 4;            // up to 4 groups x 128 f32 (each of s_x, S_a, s_w)
+constexpr int PSTAGE = PB_BYTES + 3 * PSC_BYTES;
 
 template <int RP>
 struct GemmCfg {
-  static constexpr int SA = 4;                  // activation stages (TMA -> MMA)
-  static constexpr int SP = RP <= 32 ? 6 : 4;   // packed-weight stages (even, see the teams)
   static constexpr int BR_BYTES = RP * kBM * 2;   // p_hat tile (and the B_hat tile), RP/8 boxes of 2 KB
-  static constexpr int NBAR = 2 * SA + 2 * SX + 2 * SP + 2 * NSS + 2 * NTB + 2 * NBR + 1;
-  static constexpr int SMEM = 1024 + SA * A_BYTES + SX * X_BYTES + SP * PSTAGE + NSS * SLOT_FLOATS * 4 +
-                              NBR * 2 * BR_BYTES + NBAR * 8 + 16;
+  static constexpr int NBAR = 2 * SO + 2 * SP + 2 * NTB + 2 * NBR + 1;
+  static constexpr int SMEM = 1024 + SO * OSTAGE + SP * PSTAGE + NBR * 2 * BR_BYTES + NBAR * 8 + 16;
   static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 };
 
@@ -95,31 +100,23 @@ __device__ __forceinline__ f2 add2(f2 a, f2 b) {
 }
 
 template <int RP>
-__global__ void __launch_bounds__(448, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap qx_map, const __grid_constant__ CUtensorMap qw_map,
                 const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap cs_map,
                 const __grid_constant__ CUtensorMap sw_map, const __grid_constant__ CUtensorMap ph_map,
                 const __grid_constant__ CUtensorMap bh_map, const GemmArgs a) {
   using Cfg = GemmCfg<RP>;
-  constexpr int SP = Cfg::SP;
-  constexpr int SA = Cfg::SA;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* aring = smem;                           // SA x 16 KB, 1024-aligned
-  uint8_t* xring = aring + SA * A_BYTES;           // SX x 16 KB, 1024-aligned
-  uint8_t* pring = xring + SX * X_BYTES;           // SP x (weights packed | s_x | code sums | s_w)
-  float* slots = reinterpret_cast<float*>(pring + SP * PSTAGE);
-  uint8_t* br = reinterpret_cast<uint8_t*>(slots + NSS * SLOT_FLOATS);  // NBR x (p_hat | B_hat)
+  uint8_t* oring = smem;                           // SO x (A 16 KB | X 16 KB), 1024-aligned
+  uint8_t* pring = oring + SO * OSTAGE;            // SP x (weights packed | s_x | S_a | s_w)
+  uint8_t* br = pring + SP * PSTAGE;               // NBR x (p_hat | B_hat)
   uint64_t* bars = reinterpret_cast<uint64_t*>(br + NBR * 2 * Cfg::BR_BYTES);
-  uint64_t* afull = bars;
-  uint64_t* aempty = afull + SA;
-  uint64_t* xfull = aempty + SA;
-  uint64_t* xempty = xfull + SX;
-  uint64_t* pfull = xempty + SX;
+  uint64_t* ofull = bars;
+  uint64_t* oempty = ofull + SO;
+  uint64_t* pfull = oempty + SO;
   uint64_t* pempty = pfull + SP;
-  uint64_t* sfull = pempty + SP;
-  uint64_t* sempty = sfull + NSS;
-  uint64_t* tfull = sempty + NSS;
+  uint64_t* tfull = pempty + SP;
   uint64_t* tempty = tfull + NTB;
   uint64_t* bfull = tempty + NTB;
   uint64_t* bempty = bfull + NBR;
@@ -142,23 +139,16 @@ __global__ void __launch_bounds__(448, 1)
     m0 = (t / a.n_tiles) * kBM;
     n0 = (t % a.n_tiles) * kGemmBN;
   };
+  auto groups_in = [&](int st) { return (st * gps + gps <= ngroups) ? gps : ngroups - st * gps; };
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < SA; ++i) {
-      mbar_init(&afull[i], 1);
-      mbar_init(&aempty[i], 1);
-    }
-    for (int i = 0; i < SX; ++i) {
-      mbar_init(&xfull[i], NTEAMW);
-      mbar_init(&xempty[i], 1);
+    for (int i = 0; i < SO; ++i) {
+      mbar_init(&ofull[i], 1 + NXW);  // the producer's expect-tx arrival + one per expander warp
+      mbar_init(&oempty[i], 1);
     }
     for (int i = 0; i < SP; ++i) {
       mbar_init(&pfull[i], 1);
-      mbar_init(&pempty[i], NTEAMW);
-    }
-    for (int i = 0; i < NSS; ++i) {
-      mbar_init(&sfull[i], NTEAMW);
-      mbar_init(&sempty[i], NEPIW);
+      mbar_init(&pempty[i], NEPIW);
     }
     for (int i = 0; i < NTB; ++i) {
       mbar_init(&tfull[i], 1);
@@ -181,267 +171,258 @@ __global__ void __launch_bounds__(448, 1)
   const uint32_t tmem = *tmem_slot;
   const WaitCtl wc{abort_flag, a.err, globaltimer_ns() + a.timeout_ns};
 
-  if (wid == 0) {
-    // ------------------------------------------------------------- TMA producer
-    if (lane == 0) {
-      bool ok = true;
-      const uint32_t pbytes = PB_BYTES + gps * (kBM * 8 + kGemmBN * 2);
-      int sa = 0, sp = 0;  // running stage counters (the same sequence every role walks)
-      for (int ti = 0; ti < my_tiles && ok; ++ti) {
-        int m0, n0;
-        tile_mn(ti, m0, n0);
-        if constexpr (RP > 0) {
-          const int bs = ti % NBR;
-          if (ti >= NBR) ok = mbar_wait(&bempty[bs], ((ti / NBR) & 1) ^ 1, wc);
-          if (!ok) break;
-          uint8_t* b = br + bs * 2 * Cfg::BR_BYTES;
-          mbar_arrive_expect_tx(&bfull[bs], 2 * Cfg::BR_BYTES);
-          for (int q = 0; q < RP / 8; ++q) {
-            tma_load_2d(b + q * 2048, &ph_map, &bfull[bs], q * 8, m0);
-            tma_load_2d(b + Cfg::BR_BYTES + q * 2048, &bh_map, &bfull[bs], q * 8, n0);
+  if (wid < 4) {
+    setmaxnreg_dec<kRegsCtl>();
+    if (wid == 0) {
+      // ----------------------------------------------------------- TMA producer
+      if (lane == 0) {
+        bool ok = true;
+        const uint32_t pbytes = PB_BYTES + gps * 3 * 128 * 4;
+        int s = 0;  // running stage counter (the same sequence every role walks)
+        for (int ti = 0; ti < my_tiles && ok; ++ti) {
+          int m0, n0;
+          tile_mn(ti, m0, n0);
+          for (int st = 0; st < nst && ok; ++st, ++s) {
+            // packed weights and the group scales of this stage
+            const int ps = s % SP;
+            if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
+            if (!ok) break;
+            uint8_t* p = pring + ps * PSTAGE;
+            mbar_arrive_expect_tx(&pfull[ps], pbytes);
+            tma_load_2d(p, &qw_map, &pfull[ps], st * (kGemmKS / 2), n0);
+            tma_load_2d(p + PB_BYTES, &sx_map, &pfull[ps], m0, st * gps);
+            tma_load_2d(p + PB_BYTES + PSC_BYTES, &cs_map, &pfull[ps], m0, st * gps);
+            tma_load_2d(p + PB_BYTES + 2 * PSC_BYTES, &sw_map, &pfull[ps], n0, st * gps);
+            // activation codes of this stage
+            const int os = s % SO;
+            if (s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
+            if (!ok) break;
+            mbar_arrive_expect_tx(&ofull[os], A_BYTES);
+            tma_load_2d(oring + os * OSTAGE, &qx_map, &ofull[os], st * kGemmKS, m0);
+          }
+          if constexpr (RP > 0) {
+            // the branch operands are needed only after the tile's last stage
+            const int bs = ti % NBR;
+            if (ok && ti >= NBR) ok = mbar_wait_inline(&bempty[bs], ((ti / NBR) & 1) ^ 1, wc);
+            if (!ok) break;
+            uint8_t* b = br + bs * 2 * Cfg::BR_BYTES;
+            mbar_arrive_expect_tx(&bfull[bs], 2 * Cfg::BR_BYTES);
+            for (int q = 0; q < RP / 8; ++q) {
+              tma_load_2d(b + q * 2048, &ph_map, &bfull[bs], q * 8, m0);
+              tma_load_2d(b + Cfg::BR_BYTES + q * 2048, &bh_map, &bfull[bs], q * 8, n0);
+            }
           }
         }
-        for (int st = 0; st < nst && ok; ++st) {
-          // packed weights and the group scales of this stage
-          const int ps = sp % SP;
-          if (sp >= SP) ok = mbar_wait(&pempty[ps], ((sp / SP) & 1) ^ 1, wc);
-          if (!ok) break;
-          uint8_t* p = pring + ps * PSTAGE;
-          mbar_arrive_expect_tx(&pfull[ps], pbytes);
-          tma_load_2d(p, &qw_map, &pfull[ps], st * (kGemmKS / 2), n0);
-          tma_load_2d(p + PB_BYTES, &sx_map, &pfull[ps], m0, st * gps);
-          tma_load_2d(p + PB_BYTES + PSX_BYTES, &cs_map, &pfull[ps], m0, st * gps);
-          tma_load_2d(p + PB_BYTES + PSX_BYTES + PCS_BYTES, &sw_map, &pfull[ps], n0, st * gps);
-          ++sp;
-          // activation codes of this stage
-          const int as = sa % SA;
-          if (sa >= SA) ok = mbar_wait(&aempty[as], ((sa / SA) & 1) ^ 1, wc);
-          if (!ok) break;
-          mbar_arrive_expect_tx(&afull[as], A_BYTES);
-          tma_load_2d(aring + as * A_BYTES, &qx_map, &afull[as], st * kGemmKS, m0);
-          ++sa;
+        // Let every issued load land before the CTA can exit (these phases complete in the
+        // normal course; after an abort the waits end at the deadline).
+        int never = 0;
+        const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+        for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
+        // An operand stage also needs the expanders' arrivals: in the normal course they come;
+        // after an abort the wait ends at the deadline, long after the tile has landed.
+        for (int j = (s > SO ? s - SO : 0); j < s; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
+        if constexpr (RP > 0) {
+          for (int t = (my_tiles > NBR ? my_tiles - NBR : 0); t < my_tiles; ++t)
+            mbar_wait_inline(&bfull[t % NBR], (t / NBR) & 1, dc);
         }
       }
-      // Let every issued load land before the CTA can exit.
-      int never = 0;
-      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-      for (int j = (sp > SP ? sp - SP : 0); j < sp; ++j) mbar_wait(&pfull[j % SP], (j / SP) & 1, dc);
-      for (int j = (sa > SA ? sa - SA : 0); j < sa; ++j) mbar_wait(&afull[j % SA], (j / SA) & 1, dc);
-    }
-  } else if (wid == 1) {
-    // ------------------------------------------------------------- MMA issuer
-    // The epilogue consumes accumulators in units of two groups (one TMEM buffer of 2 x 128
-    // columns); a unit never straddles a stage because a stage holds an even number of groups.
-    // One tcgen05 fence per unit: fences and commits cost far more than an MMA issue.
-    if (lane == 0) {
+    } else if (wid == 1) {
+      // ----------------------------------------------------------- MMA issuer
+      // The epilogue consumes accumulators in units of two groups (one TMEM buffer of 2 x 128
+      // columns); a unit never straddles a stage because a full stage holds an even number of
+      // groups.  One tcgen05 fence per unit: fences and commits cost far more than an MMA issue.
+      if (lane == 0) {
+        bool ok = true;
+        constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
+        int s = 0, u_all = 0;  // running stage and accumulator-unit counters
+        for (int ti = 0; ti < my_tiles && ok; ++ti) {
+          for (int st = 0; st < nst && ok; ++st, ++s) {
+            const int gn = groups_in(st);
+            const int os = s % SO;
+            ok = mbar_wait_inline(&ofull[os], (s / SO) & 1, wc);
+            if (!ok) break;
+            const uint32_t aa = smem_u32(oring + os * OSTAGE), xa = aa + A_BYTES;
+            for (int g0 = 0; g0 < gn && ok; g0 += 2, ++u_all) {
+              const int ub = u_all % NTB;
+              if (u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
+              if (!ok) break;
+              tc_fence_after();
+              for (int gi = g0; gi < gn && gi < g0 + 2; ++gi)
+                for (int kk = 0; kk < G / 32; ++kk) {
+                  const uint32_t off = static_cast<uint32_t>((gi * (G / 32) + kk) * 32);
+                  mma_f8f6f4(tmem + ub * 256 + (gi - g0) * 128, smem_desc(aa + off, 16, 1024, kSw128),
+                             smem_desc(xa + off, 16, 1024, kSw128), idesc, kk != 0);
+                }
+              mma_commit(&tfull[ub]);
+            }
+            mma_commit(&oempty[os]);
+          }
+          if constexpr (RP > 0) {
+            const int bs = ti % NBR, ub = u_all % NTB;
+            if (ok) ok = mbar_wait_inline(&bfull[bs], (ti / NBR) & 1, wc);
+            if (ok && u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
+            if (ok) {
+              tc_fence_after();
+              constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
+              const uint32_t pa = smem_u32(br + bs * 2 * Cfg::BR_BYTES), pb = pa + Cfg::BR_BYTES;
+#pragma unroll
+              for (int kk = 0; kk < RP / 16; ++kk)
+                mma_f16(tmem + ub * 256, smem_desc(pa + kk * 4096, 2048, 128, kSwNone),
+                        smem_desc(pb + kk * 4096, 2048, 128, kSwNone), idesc_br, kk != 0);
+              mma_commit(&tfull[ub]);
+              mma_commit(&bempty[bs]);
+              ++u_all;
+            }
+          }
+        }
+        mma_commit(drain);
+        int never = 0;
+        const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+        mbar_wait_inline(drain, 0, dc);
+      }
+      __syncwarp();
+    } else {
+      // ----------------------------------------------------------- weight expanders
+      // Thread e (0..63) owns the 16-byte chunk j = e % 8 of rows e/8 + 8 i (i = 0..15): its source
+      // and destination offsets only step by constants (512 and 1024 bytes).
+      const int e = static_cast<int>(threadIdx.x) - 64;
+      const int r0 = e >> 3, j = e & 7;
+      const int src0 = r0 * 64 + j * 8;
+      const int dst0 = r0 * 128 + ((j ^ r0) << 4);
+      const uint32_t kX8 = 0x88888888u;
       bool ok = true;
-      constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
-      int s = 0, u_all = 0;  // running stage and accumulator-unit counters
+      int s = 0;
       for (int ti = 0; ti < my_tiles && ok; ++ti) {
         for (int st = 0; st < nst && ok; ++st, ++s) {
-          const int gn = (st * gps + gps <= ngroups) ? gps : ngroups - st * gps;  // groups in this stage
-          const int as = s % SA, xs = s % SX;
-          ok = mbar_wait(&afull[as], (s / SA) & 1, wc);
-          if (ok) ok = mbar_wait(&xfull[xs], (s / SX) & 1, wc);
+          const int ps = s % SP, os = s % SO;
+          ok = mbar_wait_inline(&pfull[ps], (s / SP) & 1, wc);
+          if (ok && s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
           if (!ok) break;
-          const uint32_t aa = smem_u32(aring + as * A_BYTES), xa = smem_u32(xring + xs * X_BYTES);
-          for (int g0 = 0; g0 < gn && ok; g0 += 2, ++u_all) {
-            const int ub = u_all % NTB;
-            if (u_all >= NTB) ok = mbar_wait(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
-            if (!ok) break;
-            tc_fence_after();
-            for (int gi = g0; gi < gn && gi < g0 + 2; ++gi)
-              for (int kk = 0; kk < G / 32; ++kk) {
-                const uint32_t off = static_cast<uint32_t>((gi * (G / 32) + kk) * 32);
-                mma_f8f6f4(tmem + ub * 256 + (gi - g0) * 128, smem_desc(aa + off, 16, 1024, kSw128),
-                           smem_desc(xa + off, 16, 1024, kSw128), idesc, kk != 0);
-              }
-            mma_commit(&tfull[ub]);
+          const uint8_t* p = pring + ps * PSTAGE;
+          uint8_t* xb = oring + os * OSTAGE + A_BYTES;
+#pragma unroll
+          for (int h8 = 0; h8 < 16; h8 += 8) {
+            uint2 pkd[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) pkd[i] = *reinterpret_cast<const uint2*>(p + src0 + (h8 + i) * 512);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              uint4 o;
+              o.x = (pkd[i].x ^ kX8) & 0x0F0F0F0Fu;
+              o.y = ((pkd[i].x >> 4) ^ kX8) & 0x0F0F0F0Fu;
+              o.z = (pkd[i].y ^ kX8) & 0x0F0F0F0Fu;
+              o.w = ((pkd[i].y >> 4) ^ kX8) & 0x0F0F0F0Fu;
+              *reinterpret_cast<uint4*>(xb + dst0 + (h8 + i) * 1024) = o;
+            }
           }
-          mma_commit(&aempty[as]);
-          mma_commit(&xempty[xs]);
+          // Orders the generic writes of the expanded weights before the MMA reads them, and the
+          // generic reads of the packed stage before TMA refills it (the epilogue releases it).
+          fence_proxy_async_smem();
+          warp_arrive(&ofull[os]);
         }
-        if constexpr (RP > 0) {
-          const int bs = ti % NBR, ub = u_all % NTB;
-          if (ok) ok = mbar_wait(&bfull[bs], (ti / NBR) & 1, wc);
-          if (ok && u_all >= NTB) ok = mbar_wait(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
-          if (ok) {
-            tc_fence_after();
-            constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
-            const uint32_t pa = smem_u32(br + bs * 2 * Cfg::BR_BYTES), pb = pa + Cfg::BR_BYTES;
-#pragma unroll
-            for (int kk = 0; kk < RP / 16; ++kk)
-              mma_f16(tmem + ub * 256, smem_desc(pa + kk * 4096, 2048, 128, kSwNone),
-                      smem_desc(pb + kk * 4096, 2048, 128, kSwNone), idesc_br, kk != 0);
-            mma_commit(&tfull[ub]);
-            mma_commit(&bempty[bs]);
-            ++u_all;
-          }
-        }
-      }
-      mma_commit(drain);
-      int never = 0;
-      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-      mbar_wait(drain, 0, dc);
-    }
-    __syncwarp();
-  } else if (wid < 6) {
-    // ------------------------------------------------------------- weight expanders + scales
-    // Team t (warps 2+2t, 3+2t) takes the stages s with s % 2 == t.  Thread e (0..63) of a team
-    // owns the 16-byte chunk j = e % 8 of rows e/8 + 8 i (i = 0..15): its source and destination
-    // offsets only step by constants (512 and 1024 bytes).
-    const int team = (static_cast<int>(wid) - 2) >> 1;
-    const int e = (static_cast<int>(threadIdx.x) - 64) & (NTEAM - 1);
-    const int r0 = e >> 3, j = e & 7;
-    const int src0 = r0 * 64 + j * 8;
-    const int dst0 = r0 * 128 + ((j ^ r0) << 4);
-    const uint32_t kX8 = 0x88888888u;
-    bool ok = true;
-    int s = 0;
-    for (int ti = 0; ti < my_tiles && ok; ++ti) {
-      for (int st = 0; st < nst && ok; ++st, ++s) {
-        if ((s & 1) != team) continue;
-        const int gn = (st * gps + gps <= ngroups) ? gps : ngroups - st * gps;  // groups in this stage
-        const int ps = s % SP, xs = team;
-        ok = mbar_wait(&pfull[ps], (s / SP) & 1, wc);
-        if (ok && s >= SX) ok = mbar_wait(&xempty[xs], ((s / SX) & 1) ^ 1, wc);
-        if (!ok) break;
-        const uint8_t* p = pring + ps * PSTAGE;
-        uint8_t* xb = xring + xs * X_BYTES;
-        uint2 pkd[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) pkd[i] = *reinterpret_cast<const uint2*>(p + src0 + i * 512);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          uint4 o;
-          o.x = (pkd[i].x ^ kX8) & 0x0F0F0F0Fu;
-          o.y = ((pkd[i].x >> 4) ^ kX8) & 0x0F0F0F0Fu;
-          o.z = (pkd[i].y ^ kX8) & 0x0F0F0F0Fu;
-          o.w = ((pkd[i].y >> 4) ^ kX8) & 0x0F0F0F0Fu;
-          *reinterpret_cast<uint4*>(xb + dst0 + i * 1024) = o;
-        }
-        fence_proxy_async_smem();
-        warp_arrive(&xfull[xs]);
-        // group scales of this stage -> the team's float32 scale slot for the epilogue
-        const float* psx = reinterpret_cast<const float*>(p + PB_BYTES);
-        const float* pcs = reinterpret_cast<const float*>(p + PB_BYTES + PSX_BYTES);
-        const __half* psw = reinterpret_cast<const __half*>(p + PB_BYTES + PSX_BYTES + PCS_BYTES);
-        const int ss = team;
-        if (s >= NSS) ok = mbar_wait(&sempty[ss], ((s / NSS) & 1) ^ 1, wc);
-        if (!ok) break;
-        float* slot = slots + ss * SLOT_FLOATS;
-        for (int gi = 0; gi < gn; ++gi) {
-          float* sg = slot + gi * GSLOT;
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int i = e + NTEAM * h;
-            sg[i] = __half2float(psw[gi * kGemmBN + i]);
-            sg[kGemmBN + i] = psx[gi * kBM + i];
-            sg[kGemmBN + kBM + i] = pcs[gi * kBM + i];
-          }
-        }
-        warp_arrive(&sfull[ss]);
-        fence_proxy_async_smem();  // reads of the packed stage before the TMA refills it
-        warp_arrive(&pempty[ps]);
       }
     }
   } else {
+    setmaxnreg_inc<kRegsEpi>();
     // ------------------------------------------------------------- epilogue
-    // Warps 6..13: warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 64 output
-    // columns [64*((w-6)/4), +64).
+    // Warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 32 output columns
+    // [32*((w-4)/4), +32).  Thread t holds rows rq + 8k (k = 0..3, rq = t/4 within the quadrant)
+    // and columns 8j + 2 cq + {0, 1} (j = 0..3, cq = t % 4): acc[4k + j] is that pair.
     const int quad = wid & 3;
-    const int row = quad * 32 + static_cast<int>(lane);
-    const int col0 = 64 * ((static_cast<int>(wid) - 6) >> 2);
-    const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
+    const int col0 = 32 * ((static_cast<int>(wid) - 4) >> 2);
+    const int rq = static_cast<int>(lane) >> 2, cq = static_cast<int>(lane) & 3;
+    const int rbase = quad * 32 + rq;
+    const uint32_t tq = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
     bool ok = true;
     int u_all = 0, s = 0;  // accumulator-unit and stage counters
     for (int ti = 0; ti < my_tiles; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
-      f2 acc[32];
+      f2 acc[16];
 #pragma unroll
-      for (int i = 0; i < 32; ++i) acc[i] = 0ull;
+      for (int i = 0; i < 16; ++i) acc[i] = 0ull;
       for (int st = 0; st < nst; ++st, ++s) {
-        const int gn = (st * gps + gps <= ngroups) ? gps : ngroups - st * gps;  // groups in this stage
-        const int ss = s % NSS;
-        if (ok) ok = mbar_wait(&sfull[ss], (s / NSS) & 1, wc);
-        const float* slot = slots + ss * SLOT_FLOATS;
+        const int gn = groups_in(st);
+        const int ps = s % SP;
+        if (ok) ok = mbar_wait_inline(&pfull[ps], (s / SP) & 1, wc);
+        const float* psx = reinterpret_cast<const float*>(pring + ps * PSTAGE + PB_BYTES);
+        const float* pcs = psx + 4 * 128;
+        const float* psw = psx + 8 * 128;
         for (int g0 = 0; g0 < gn; g0 += 2, ++u_all) {
           const int ub = u_all % NTB;
           const int nmem = (g0 + 1 < gn) ? 2 : 1;
-          if (ok) ok = mbar_wait(&tfull[ub], (u_all / NTB) & 1, wc);
+          if (ok) ok = mbar_wait_inline(&tfull[ub], (u_all / NTB) & 1, wc);
           tc_fence_after();
           for (int mi = 0; mi < nmem; ++mi) {
-            const float* sg = slot + (g0 + mi) * GSLOT;
-            const float sxv = sg[kGemmBN + row];
-            const float alpha = sxv * 262144.0f;                       // 2^18 s_x (exact)
-            const float beta = -8.0f * sxv * sg[kGemmBN + kBM + row];  // -8 s_x S_a
-            const f2 al2 = pk(alpha, alpha), be2 = pk(beta, beta);
+            const int gi = g0 + mi;
+            uint32_t v0[16], v1[16];
+            tmem_ld16x256_x4(tq + ub * 256 + mi * 128, v0);
+            tmem_ld16x256_x4(tq + (16u << 16) + ub * 256 + mi * 128, v1);
+            float sxr[4], csr[4];
 #pragma unroll
-            for (int c = 0; c < 2; ++c) {
-              uint32_t v[32];
-              tmem_ld32(tlane + ub * 256 + mi * 128 + c * 32, v);
-              tmem_ld_wait();
-              if (mi == nmem - 1 && c == 1) {
-                tc_fence_before();
-                warp_arrive(&tempty[ub]);
-              }
-              const float4* w4 = reinterpret_cast<const float4*>(sg + col0 + c * 32);
+            for (int k = 0; k < 4; ++k) {
+              sxr[k] = psx[gi * 128 + rbase + 8 * k];
+              csr[k] = pcs[gi * 128 + rbase + 8 * k];
+            }
+            f2 sw2[4];
 #pragma unroll
-              for (int i4 = 0; i4 < 8; ++i4) {
-                const float4 w = w4[i4];
-                const f2 t0 = fma2(pku(v[4 * i4], v[4 * i4 + 1]), al2, be2);
-                const f2 t1 = fma2(pku(v[4 * i4 + 2], v[4 * i4 + 3]), al2, be2);
-                acc[16 * c + 2 * i4] = fma2(t0, pk(w.x, w.y), acc[16 * c + 2 * i4]);
-                acc[16 * c + 2 * i4 + 1] = fma2(t1, pk(w.z, w.w), acc[16 * c + 2 * i4 + 1]);
+            for (int j = 0; j < 4; ++j) sw2[j] = *reinterpret_cast<const f2*>(psw + gi * 128 + col0 + 8 * j + 2 * cq);
+            f2 d[16];  // d[8h + 2j + rr] = columns (8j + 2cq, +1) of row rq + 16h + 8rr
+            tmem_ld_wait_pairs(v0, v1, d);
+            if (mi == nmem - 1) {
+              tc_fence_before();
+              warp_arrive(&tempty[ub]);  // every load of the unit has landed
+            }
+            // acc += (alpha D + beta) * s_w, alpha = 2^18 s_x (exact), beta = -8 s_x S_a
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float alpha = sxr[k] * 262144.0f;
+              const float beta = -8.0f * sxr[k] * csr[k];
+              const f2 al2 = dup2(alpha), be2 = dup2(beta);
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                const f2 t = fma2(d[8 * (k >> 1) + 2 * j + (k & 1)], al2, be2);
+                acc[4 * k + j] = fma2(t, sw2[j], acc[4 * k + j]);
               }
             }
           }
         }
-        warp_arrive(&sempty[ss]);
+        fence_proxy_async_smem();  // reads of the TMA-written scales before the stage is refilled
+        warp_arrive(&pempty[ps]);
       }
       if constexpr (RP > 0) {
         const int ub = u_all % NTB;
-        if (ok) ok = mbar_wait(&tfull[ub], (u_all / NTB) & 1, wc);
+        if (ok) ok = mbar_wait_inline(&tfull[ub], (u_all / NTB) & 1, wc);
         tc_fence_after();
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          uint32_t v[32];
-          tmem_ld32(tlane + ub * 256 + c * 32, v);
-          tmem_ld_wait();
-#pragma unroll
-          for (int i = 0; i < 16; ++i) acc[16 * c + i] = add2(acc[16 * c + i], pku(v[2 * i], v[2 * i + 1]));
-        }
+        uint32_t v0[16], v1[16];
+        tmem_ld16x256_x4(tq + ub * 256, v0);
+        tmem_ld16x256_x4(tq + (16u << 16) + ub * 256, v1);
+        f2 d[16];
+        tmem_ld_wait_pairs(v0, v1, d);
         tc_fence_before();
         warp_arrive(&tempty[ub]);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+#pragma unroll
+          for (int j = 0; j < 4; ++j) acc[4 * k + j] = add2(acc[4 * k + j], d[8 * (k >> 1) + 2 * j + (k & 1)]);
         ++u_all;
       }
-      const int m = m0 + row;
-      if (ok && m < a.M) {
-        const int nb = n0 + col0;
-        if (a.y_f32) {
-          float* yr = static_cast<float*>(a.Y) + static_cast<size_t>(m) * a.N + nb;
+      if (ok) {
 #pragma unroll
-          for (int c8 = 0; c8 < 8; ++c8) {
-            if (nb + c8 * 8 < a.N) {
-              reinterpret_cast<float4*>(yr + c8 * 8)[0] =
-                  make_float4(lo_f(acc[4 * c8]), hi_f(acc[4 * c8]), lo_f(acc[4 * c8 + 1]), hi_f(acc[4 * c8 + 1]));
-              reinterpret_cast<float4*>(yr + c8 * 8)[1] = make_float4(lo_f(acc[4 * c8 + 2]), hi_f(acc[4 * c8 + 2]),
-                                                                      lo_f(acc[4 * c8 + 3]), hi_f(acc[4 * c8 + 3]));
-            }
-          }
-        } else {
-          __nv_bfloat16* yr = static_cast<__nv_bfloat16*>(a.Y) + static_cast<size_t>(m) * a.N + nb;
+        for (int k = 0; k < 4; ++k) {
+          const int m = m0 + rbase + 8 * k;
+          if (m >= a.M) continue;
 #pragma unroll
-          for (int c8 = 0; c8 < 8; ++c8) {
-            if (nb + c8 * 8 < a.N) {
-              uint32_t w[4];
-#pragma unroll
-              for (int t = 0; t < 4; ++t) {
-                __nv_bfloat162 h2 = __floats2bfloat162_rn(lo_f(acc[4 * c8 + t]), hi_f(acc[4 * c8 + t]));
-                w[t] = *reinterpret_cast<uint32_t*>(&h2);
-              }
-              *reinterpret_cast<uint4*>(yr + c8 * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+          for (int j = 0; j < 4; ++j) {
+            const int n = n0 + col0 + 8 * j + 2 * cq;  // even; N is a multiple of 8
+            if (n >= a.N) continue;
+            const size_t off = static_cast<size_t>(m) * a.N + n;
+            if (a.y_f32) {
+              *reinterpret_cast<float2*>(static_cast<float*>(a.Y) + off) =
+                  make_float2(lo_f(acc[4 * k + j]), hi_f(acc[4 * k + j]));
+            } else {
+              *reinterpret_cast<__nv_bfloat162*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
+                  __floats2bfloat162_rn(lo_f(acc[4 * k + j]), hi_f(acc[4 * k + j]));
             }
           }
         }
@@ -480,7 +461,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
   const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
   const CUtensorMap& ph = (RP > 0) ? am.ph_map : am.qx_map;
   const CUtensorMap& bh = (RP > 0) ? h.Bh_map : am.qx_map;
-  gemm_kernel<RP><<<grid, 448, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.sx_map, am.cs_map, h.sw_map, ph, bh, a);
+  gemm_kernel<RP><<<grid, kThreads, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.sx_map, am.cs_map, h.sw32_map, ph, bh, a);
   return cudaGetLastError();
 }
 

@@ -40,12 +40,13 @@ struct Handle {
   uint8_t* qw = nullptr;             // [N_pad, K/2]; word j of a row holds k = 8j..8j+3 in the low
                                      // and 8j+4..8j+7 in the high nibbles of its bytes
   __half* sw = nullptr;              // [K/G, N_pad]
+  float* sw32 = nullptr;             // [K/G, N_pad]: the same scales widened to float32 (GEMM epilogue)
   __half* Bh = nullptr;              // [N_pad, r_pad]
   __nv_bfloat16* ucat_t = nullptr;   // [2 r_pad, K]: rows 0..r_pad-1 = U_hi^T, then U_lo^T
   __nv_bfloat16* ucat3 = nullptr;    // [K, ku3]: row k = U_hi[k,:], U_lo[k,:], U_hi[k,:], zeros
   int* err = nullptr;                // sticky device error word
   double timeout_s = 2.0;
-  CUtensorMap qw_map, sw_map, Bh_map, ucat_t_map, ucat3_map;
+  CUtensorMap qw_map, sw32_map, Bh_map, ucat_t_map, ucat3_map;
   ActMaps act_cache[4];
   int act_next = 0;
 };

@@ -52,7 +52,8 @@ __device__ __forceinline__ int nearest_code_f64(double w, double s) {
 // the high nibbles of its four bytes (the GEMM expands a word to bytes with three logic ops).
 __global__ void quantize_weight_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
                                        const double* __restrict__ Bf, int K, int N, int r, int G, int N_pad,
-                                       uint8_t* __restrict__ qw, __half* __restrict__ sw, int* err) {
+                                       uint8_t* __restrict__ qw, __half* __restrict__ sw, float* __restrict__ sw32,
+                                       int* err) {
   int n = blockIdx.x * blockDim.x + threadIdx.x;
   int g = blockIdx.y;
   if (n >= N) return;
@@ -61,6 +62,7 @@ __global__ void quantize_weight_kernel(const __nv_bfloat16* __restrict__ W, cons
   __half sh = __double2half(__ddiv_rn(amax, 7.0));
   double s = static_cast<double>(__half2float(sh));
   sw[static_cast<size_t>(g) * N_pad + n] = sh;
+  sw32[static_cast<size_t>(g) * N_pad + n] = static_cast<float>(s);
   bool ok_scale = isfinite(s);
   if (!ok_scale) atomicOr(err, kErrRange);
   uint32_t* row = reinterpret_cast<uint32_t*>(qw + static_cast<size_t>(n) * (K / 2));
@@ -124,7 +126,7 @@ cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaS
   if (r > 0) {
     branch_weight_kernel<<<dim3((N + T - 1) / T, r), T, 0, s>>>(W, U, K, N, r, Bf);
   }
-  quantize_weight_kernel<<<dim3((N + T - 1) / T, K / h.G), T, 0, s>>>(W, U, Bf, K, N, r, h.G, h.N_pad, h.qw, h.sw,
+  quantize_weight_kernel<<<dim3((N + T - 1) / T, K / h.G), T, 0, s>>>(W, U, Bf, K, N, r, h.G, h.N_pad, h.qw, h.sw, h.sw32,
                                                                      h.err);
   if (r > 0) {
     branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);

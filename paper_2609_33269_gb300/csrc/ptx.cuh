@@ -76,7 +76,7 @@ struct WaitCtl {
   uint64_t deadline_ns;      // %globaltimer value after which waits give up
 };
 
-static __device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
+__device__ __forceinline__ bool wait_loop(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 127) == 0) {
@@ -89,9 +89,18 @@ static __device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, co
     }
   }
 }
+static __device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
+  return wait_loop(bar, parity, c);
+}
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
   if (mbar_try_wait(bar, parity)) return true;
   return wait_slow(bar, parity, c);
+}
+// The same wait with the slow loop inlined, for kernels that set per-warpgroup register budgets
+// (setmaxnreg): ptxas cannot allocate registers for a function called from such regions.
+__device__ __forceinline__ bool mbar_wait_inline(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return wait_loop(bar, parity, c);
 }
 
 // ---------------------------------------------------------------- fences
@@ -227,5 +236,88 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "memory");
 }
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// The same wait, naming the 32 registers of one tcgen05.ld as its operands: the compiler then
+// cannot move a use of those registers above the wait, so loads can be issued ahead (software
+// pipelining) while other registers are being consumed.
+__device__ __forceinline__ void tmem_ld_wait_dep(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+
+// tcgen05.ld.16x256b.x4: 16 TMEM lanes x 32 columns.  Thread t receives register 4j + q =
+// (lane t/4 + 8 [q >= 2], column 8j + 2 (t % 4) + (q & 1)), j = 0..3: four threads share a lane
+// (row) and eight share a column pair.
+__device__ __forceinline__ void tmem_ld16x256_x4(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x4.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+}
+// Wait for outstanding tcgen05.ld, naming both destination arrays (see tmem_ld_wait_dep).
+__device__ __forceinline__ void tmem_ld_wait_dep2(uint32_t (&a)[16], uint32_t (&b)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(a[0]), "+r"(a[1]), "+r"(a[2]), "+r"(a[3]), "+r"(a[4]), "+r"(a[5]), "+r"(a[6]), "+r"(a[7]),
+                 "+r"(a[8]), "+r"(a[9]), "+r"(a[10]), "+r"(a[11]), "+r"(a[12]), "+r"(a[13]), "+r"(a[14]),
+                 "+r"(a[15]), "+r"(b[0]), "+r"(b[1]), "+r"(b[2]), "+r"(b[3]), "+r"(b[4]), "+r"(b[5]), "+r"(b[6]),
+                 "+r"(b[7]), "+r"(b[8]), "+r"(b[9]), "+r"(b[10]), "+r"(b[11]), "+r"(b[12]), "+r"(b[13]),
+                 "+r"(b[14]), "+r"(b[15])
+               :
+               : "memory");
+}
+
+// Wait for outstanding tcgen05.ld and hand the two 16-register results on as 16 packed pairs
+// p[i] = {r[2i], r[2i + 1]} (a then b): the pairing happens after the wait, in the form the
+// register allocator maps onto aligned register pairs.
+__device__ __forceinline__ void tmem_ld_wait_pairs(const uint32_t (&a)[16], const uint32_t (&b)[16],
+                                                   unsigned long long (&p)[16]) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;\n"
+      "mov.b64 %0, {%16, %17};\n"
+      "mov.b64 %1, {%18, %19};\n"
+      "mov.b64 %2, {%20, %21};\n"
+      "mov.b64 %3, {%22, %23};\n"
+      "mov.b64 %4, {%24, %25};\n"
+      "mov.b64 %5, {%26, %27};\n"
+      "mov.b64 %6, {%28, %29};\n"
+      "mov.b64 %7, {%30, %31};\n"
+      "mov.b64 %8, {%32, %33};\n"
+      "mov.b64 %9, {%34, %35};\n"
+      "mov.b64 %10, {%36, %37};\n"
+      "mov.b64 %11, {%38, %39};\n"
+      "mov.b64 %12, {%40, %41};\n"
+      "mov.b64 %13, {%42, %43};\n"
+      "mov.b64 %14, {%44, %45};\n"
+      "mov.b64 %15, {%46, %47};\n"
+      : "=l"(p[0]), "=l"(p[1]), "=l"(p[2]), "=l"(p[3]), "=l"(p[4]), "=l"(p[5]), "=l"(p[6]), "=l"(p[7]), "=l"(p[8]), "=l"(p[9]), "=l"(p[10]), "=l"(p[11]), "=l"(p[12]), "=l"(p[13]), "=l"(p[14]), "=l"(p[15])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(a[4]), "r"(a[5]), "r"(a[6]), "r"(a[7]), "r"(a[8]), "r"(a[9]), "r"(a[10]), "r"(a[11]), "r"(a[12]), "r"(a[13]), "r"(a[14]), "r"(a[15]), "r"(b[0]), "r"(b[1]), "r"(b[2]), "r"(b[3]), "r"(b[4]), "r"(b[5]), "r"(b[6]), "r"(b[7]), "r"(b[8]), "r"(b[9]), "r"(b[10]), "r"(b[11]), "r"(b[12]), "r"(b[13]), "r"(b[14]), "r"(b[15])
+      : "memory");
+}
+// {x, x} as a packed pair.
+__device__ __forceinline__ unsigned long long dup2(float x) {
+  unsigned long long d;
+  asm("mov.b64 %0, {%1, %1};" : "=l"(d) : "f"(x));
+  return d;
+}
+
+// Per-warpgroup register budgets (all four warps of a warpgroup execute the same instruction).
+// The sum over the CTA's warps must not exceed what the CTA was launched with (threads x the
+// kernel's register count), or an increase would wait for registers that never come free.
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
 
 }  // namespace qwam
