@@ -51,7 +51,8 @@ typedef enum {
   QWAM_ERR_CUDA = -3,
   QWAM_ERR_OOM = -4,
   QWAM_ERR_TIMEOUT = -5,     /* a bounded device wait gave up */
-  QWAM_ERR_RANGE = -6        /* a scale or branch value does not fit its 16-bit format */
+  QWAM_ERR_RANGE = -6,       /* a scale or branch value does not fit its 16-bit format */
+  QWAM_ERR_TOO_LARGE = -7    /* the activation workspace would exceed QWAM_STATIC_WS_BYTES */
 } qwam_status;
 
 enum { QWAM_Y_BF16 = 0, QWAM_Y_FP32 = 1 };
@@ -106,6 +107,33 @@ qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle h, void* Y,
 /* The whole layer: qwam_asp_quantize_act followed by qwam_asp_gemm on `stream`. */
 qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
                             void* act_ws, struct CUstream_st* stream);
+
+/* ---- the layer without a caller-provided workspace ---------------------------------------
+ * The paper has no counterpart to this call: it is a convenience of this library.
+ *
+ * qwam_asp_linear needs the caller to hand it `act_ws`, a device buffer.  Some callers cannot
+ * provide one: a plain C host without a device allocator of its own, or a serving loop that
+ * must not allocate on its hot path (cudaMalloc and cudaFree may synchronize the device and
+ * fragment memory).  qwam_asp_linear_static runs the same two kernels as qwam_asp_linear, on
+ * `stream`, but with a scratch buffer that the library reserves statically in device memory
+ * (QWAM_STATIC_WS_BYTES per device, set aside when the library's device code is loaded).  It
+ * allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ *   - Size limit: the workspace qwam_asp_act_workspace_bytes(h, M) reports must fit in
+ *     QWAM_STATIC_WS_BYTES (16 MiB: e.g. M = 4096 tokens at K = 3072, group 32 or 64, r <= 64).
+ *     Larger requests return QWAM_ERR_TOO_LARGE before anything is launched.
+ *   - Nothing in the scratch needs to start at zero: kernel (a) writes every byte the GEMM
+ *     then reads, on every call, so the scratch is never cleared.
+ *   - One scratch per device: calls that may overlap in time on one device (different streams
+ *     without ordering between them, or different host threads) race on it and give wrong
+ *     results.  Order such calls, e.g. issue them on one stream.
+ *   - The first call on each device looks the scratch's device address up (cudaGetSymbolAddress,
+ *     with that device current) and keeps it; later calls reuse it.  Make that first call
+ *     before any stream capture begins on the stream you pass.
+ * Other arguments and errors are those of qwam_asp_linear; the handle's device must be current. */
+#define QWAM_STATIC_WS_BYTES (16u * 1024u * 1024u)
+qwam_status qwam_asp_linear_static(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
+                                   struct CUstream_st* stream);
 
 /* Sticky device-side error of the handle (QWAM_OK, QWAM_ERR_TIMEOUT or QWAM_ERR_RANGE);
  * synchronizes the device.  The word is cleared by this call. */

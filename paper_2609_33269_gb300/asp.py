@@ -25,6 +25,8 @@ QWAM_ERR_CUDA = -3
 QWAM_ERR_OOM = -4
 QWAM_ERR_TIMEOUT = -5
 QWAM_ERR_RANGE = -6
+QWAM_ERR_TOO_LARGE = -7
+STATIC_WS_BYTES = 16 * 1024 * 1024  # QWAM_STATIC_WS_BYTES of the header
 QWAM_Y_BF16 = 0
 QWAM_Y_FP32 = 1
 
@@ -33,6 +35,7 @@ EXPORTED = [
     "qwam_asp_quantize_act", "qwam_asp_gemm", "qwam_asp_linear", "qwam_asp_get_error",
     "qwam_asp_shape", "qwam_asp_export", "qwam_asp_destroy", "qwam_status_string",
     "qwam_asp_debug_residual", "qwam_asp_set_timeout", "qwam_asp_debug_wait_timeout",
+    "qwam_asp_linear_static",
 ]
 
 _lib = None
@@ -63,6 +66,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_quantize_act.argtypes = [V, I, H, V, V]
         lib.qwam_asp_gemm.argtypes = [V, I, H, V, I, V]
         lib.qwam_asp_linear.argtypes = [V, I, H, V, I, V, V]
+        lib.qwam_asp_linear_static.argtypes = [V, I, H, V, I, V]
         lib.qwam_asp_get_error.argtypes = [H]
         lib.qwam_asp_shape.argtypes = [H] + [ctypes.POINTER(I)] * 5
         lib.qwam_asp_export.argtypes = [H, V, V, V, V]
@@ -136,6 +140,12 @@ def qwam_asp_gemm(act_ws, M: int, h: int, Y, y_dtype: int, stream=None):
 def qwam_asp_linear(X_bf16, M: int, h: int, Y, y_dtype: int, act_ws, stream=None):
     _check(load().qwam_asp_linear(_ptr(X_bf16), M, h, _ptr(Y), y_dtype, _ptr(act_ws), _stream(stream)),
            "qwam_asp_linear")
+
+
+def qwam_asp_linear_static(X_bf16, M: int, h: int, Y, y_dtype: int, stream=None):
+    """The layer with the library's static scratch workspace (no act_ws; see the header)."""
+    _check(load().qwam_asp_linear_static(_ptr(X_bf16), M, h, _ptr(Y), y_dtype, _stream(stream)),
+           "qwam_asp_linear_static")
 
 
 def qwam_asp_get_error(h: int) -> int:

@@ -128,6 +128,7 @@ const char* qwam_status_string(qwam_status s) {
     case QWAM_ERR_OOM: return "out of device memory";
     case QWAM_ERR_TIMEOUT: return "device wait timed out";
     case QWAM_ERR_RANGE: return "value out of 16-bit range";
+    case QWAM_ERR_TOO_LARGE: return "activation workspace larger than the static scratch (QWAM_STATIC_WS_BYTES)";
   }
   return "unknown status";
 }
