@@ -52,17 +52,20 @@ struct GemmArgs {
   uint64_t timeout_ns;
 };
 
-constexpr int kThreads = 640;
-constexpr int kLaunchRegs = 96;  // 65536 / 640 rounded down to a multiple of 8
-constexpr int kRegsCtl = 56;     // warpgroup 0
-constexpr int kRegsEpi = 104;    // warpgroups 1-4
-static_assert(128 * kRegsCtl + 512 * kRegsEpi <= kThreads * kLaunchRegs, "register split above the launch allocation");
+constexpr int kEpiWarpsPerQuad = 2;                 // epilogue warps per 32-row quadrant (2 or 4)
+constexpr int CBW = 4 / kEpiWarpsPerQuad;           // 32-column blocks per epilogue warp
+constexpr int kThreads = 128 + 128 * kEpiWarpsPerQuad;
+constexpr int kLaunchRegs = kEpiWarpsPerQuad == 4 ? 96 : 168;  // 65536 / threads, multiple of 8
+constexpr int kRegsCtl = kEpiWarpsPerQuad == 4 ? 56 : 80;     // warpgroup 0
+constexpr int kRegsEpi = kEpiWarpsPerQuad == 4 ? 104 : 208;   // the epilogue warpgroups
+static_assert(128 * kRegsCtl + (kThreads - 128) * kRegsEpi <= kThreads * kLaunchRegs,
+              "register split above the launch allocation");
 constexpr int SO = 3;     // operand stages
 constexpr int SP = 6;     // packed-weight + scale stages
 constexpr int NTB = 2;    // TMEM accumulator units (2 x 128 columns each)
 constexpr int NBR = 1;    // branch-operand stages (one per tile)
 constexpr int NXW = 2;    // expander warps
-constexpr int NEPIW = 16; // epilogue warps (4 per row quadrant, 32 columns each)
+constexpr int NEPIW = 4 * kEpiWarpsPerQuad;  // epilogue warps (32 * CBW columns each)
 constexpr int A_BYTES = kBM * kGemmKS;            // 16 KB, 128-byte swizzle
 constexpr int X_BYTES = kGemmBN * kGemmKS;        // 16 KB, 128-byte swizzle
 constexpr int OSTAGE = A_BYTES + X_BYTES;
@@ -325,11 +328,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     setmaxnreg_inc<kRegsEpi>();
     // ------------------------------------------------------------- epilogue
-    // Warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 32 output columns
-    // [32*((w-4)/4), +32).  Thread t holds rows rq + 8k (k = 0..3, rq = t/4 within the quadrant)
-    // and columns 8j + 2 cq + {0, 1} (j = 0..3, cq = t % 4): acc[4k + j] is that pair.
+    // Warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 32 CBW output columns
+    // from 32 CBW ((w-4)/4).  Thread t holds rows rq + 8k (k = 0..3, rq = t/4 within the
+    // quadrant) and, in each 32-column block cb, columns 8j + 2 cq + {0, 1} (j = 0..3,
+    // cq = t % 4): acc[16 cb + 4k + j] is that pair.
     const int quad = wid & 3;
-    const int col0 = 32 * ((static_cast<int>(wid) - 4) >> 2);
+    const int col0 = 32 * CBW * ((static_cast<int>(wid) - 4) >> 2);
     const int rq = static_cast<int>(lane) >> 2, cq = static_cast<int>(lane) & 3;
     const int rbase = quad * 32 + rq;
     const uint32_t tq = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
@@ -338,9 +342,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int ti = 0; ti < my_tiles; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
-      f2 acc[16];
+      f2 acc[16 * CBW];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) acc[i] = 0ull;
+      for (int i = 0; i < 16 * CBW; ++i) acc[i] = 0ull;
       for (int st = 0; st < nst; ++st, ++s) {
         const int gn = groups_in(st);
         const int ps = s % SP;
@@ -355,20 +359,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
           for (int mi = 0; mi < nmem; ++mi) {
             const int gi = g0 + mi;
-            uint32_t v0[16], v1[16];
-            tmem_ld16x256_x4(tq + ub * 256 + mi * 128, v0);
-            tmem_ld16x256_x4(tq + (16u << 16) + ub * 256 + mi * 128, v1);
+            uint32_t v0[CBW][16], v1[CBW][16];
+#pragma unroll
+            for (int cb = 0; cb < CBW; ++cb) {
+              tmem_ld16x256_x4(tq + ub * 256 + mi * 128 + 32 * cb, v0[cb]);
+              tmem_ld16x256_x4(tq + (16u << 16) + ub * 256 + mi * 128 + 32 * cb, v1[cb]);
+            }
             float sxr[4], csr[4];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               sxr[k] = psx[gi * 128 + rbase + 8 * k];
               csr[k] = pcs[gi * 128 + rbase + 8 * k];
             }
-            f2 sw2[4];
+            f2 sw2[4 * CBW];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) sw2[j] = *reinterpret_cast<const f2*>(psw + gi * 128 + col0 + 8 * j + 2 * cq);
-            f2 d[16];  // d[8h + 2j + rr] = columns (8j + 2cq, +1) of row rq + 16h + 8rr
-            tmem_ld_wait_pairs(v0, v1, d);
+            for (int j = 0; j < 4 * CBW; ++j)
+              sw2[j] = *reinterpret_cast<const f2*>(psw + gi * 128 + col0 + 8 * j + 2 * cq);
+            f2 d[CBW][16];  // d[cb][8h + 2j + rr] = columns (8j + 2cq, +1) of row rq + 16h + 8rr
+#pragma unroll
+            for (int cb = 0; cb < CBW; ++cb) tmem_ld_wait_pairs(v0[cb], v1[cb], d[cb]);
             if (mi == nmem - 1) {
               tc_fence_before();
               warp_arrive(&tempty[ub]);  // every load of the unit has landed
@@ -380,10 +389,12 @@ __global__ void __launch_bounds__(kThreads, 1)
               const float beta = -8.0f * sxr[k] * csr[k];
               const f2 al2 = dup2(alpha), be2 = dup2(beta);
 #pragma unroll
-              for (int j = 0; j < 4; ++j) {
-                const f2 t = fma2(d[8 * (k >> 1) + 2 * j + (k & 1)], al2, be2);
-                acc[4 * k + j] = fma2(t, sw2[j], acc[4 * k + j]);
-              }
+              for (int cb = 0; cb < CBW; ++cb)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                  const f2 t = fma2(d[cb][8 * (k >> 1) + 2 * j + (k & 1)], al2, be2);
+                  acc[16 * cb + 4 * k + j] = fma2(t, sw2[4 * cb + j], acc[16 * cb + 4 * k + j]);
+                }
             }
           }
         }
@@ -394,17 +405,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int ub = u_all % NTB;
         if (ok) ok = mbar_wait_inline(&tfull[ub], (u_all / NTB) & 1, wc);
         tc_fence_after();
-        uint32_t v0[16], v1[16];
-        tmem_ld16x256_x4(tq + ub * 256, v0);
-        tmem_ld16x256_x4(tq + (16u << 16) + ub * 256, v1);
-        f2 d[16];
-        tmem_ld_wait_pairs(v0, v1, d);
+#pragma unroll
+        for (int cb = 0; cb < CBW; ++cb) {
+          uint32_t v0[16], v1[16];
+          tmem_ld16x256_x4(tq + ub * 256 + 32 * cb, v0);
+          tmem_ld16x256_x4(tq + (16u << 16) + ub * 256 + 32 * cb, v1);
+          f2 d[16];
+          tmem_ld_wait_pairs(v0, v1, d);
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              acc[16 * cb + 4 * k + j] = add2(acc[16 * cb + 4 * k + j], d[8 * (k >> 1) + 2 * j + (k & 1)]);
+        }
         tc_fence_before();
         warp_arrive(&tempty[ub]);
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-#pragma unroll
-          for (int j = 0; j < 4; ++j) acc[4 * k + j] = add2(acc[4 * k + j], d[8 * (k >> 1) + 2 * j + (k & 1)]);
         ++u_all;
       }
       if (ok) {
@@ -413,18 +428,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int m = m0 + rbase + 8 * k;
           if (m >= a.M) continue;
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int n = n0 + col0 + 8 * j + 2 * cq;  // even; N is a multiple of 8
-            if (n >= a.N) continue;
-            const size_t off = static_cast<size_t>(m) * a.N + n;
-            if (a.y_f32) {
-              *reinterpret_cast<float2*>(static_cast<float*>(a.Y) + off) =
-                  make_float2(lo_f(acc[4 * k + j]), hi_f(acc[4 * k + j]));
-            } else {
-              *reinterpret_cast<__nv_bfloat162*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
-                  __floats2bfloat162_rn(lo_f(acc[4 * k + j]), hi_f(acc[4 * k + j]));
+          for (int cb = 0; cb < CBW; ++cb)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const int n = n0 + col0 + 32 * cb + 8 * j + 2 * cq;  // even; N is a multiple of 8
+              if (n >= a.N) continue;
+              const size_t off = static_cast<size_t>(m) * a.N + n;
+              const f2 y = acc[16 * cb + 4 * k + j];
+              if (a.y_f32) {
+                *reinterpret_cast<float2*>(static_cast<float*>(a.Y) + off) = make_float2(lo_f(y), hi_f(y));
+              } else {
+                *reinterpret_cast<__nv_bfloat162*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
+                    __floats2bfloat162_rn(lo_f(y), hi_f(y));
+              }
             }
-          }
         }
       }
     }
