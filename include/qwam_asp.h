@@ -80,17 +80,21 @@ qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes
  *            read these bytes as they are)
  *   scales : float32 [K/group, M_pad] (M_pad = M rounded up to 128), s_x of token m, group g
  *            at [g * M_pad + m]
- *   csums  : float32 [K/group, M_pad], the sum of the group's codes (an exact integer)
+ *   ab     : float32 [K/group, M_pad, 2], for token m and group g at [(g * M_pad + m) * 2]:
+ *            (alpha, beta) with alpha = 2^18 s_x and beta = -8 s_x S_a, S_a the sum of the
+ *            group's codes.  These are the GEMM epilogue's per-row constants (see
+ *            qwam_asp_gemm), formed here once per token and group, each with one rounding.
  *   p_hat  : float16 [M, r_pad] (r_pad = r rounded up to 16; columns >= r are zero)
  * The workspace is transient (written by qwam_asp_quantize_act, read by qwam_asp_gemm); the
  * weights are the part of the layer that stays packed at 4 bits. */
 qwam_status qwam_asp_act_layout(qwam_asp_handle h, int M, size_t* codes_off, size_t* scales_off,
-                                size_t* csums_off, size_t* phat_off, int* M_pad, int* r_pad);
+                                size_t* ab_off, size_t* phat_off, int* M_pad, int* r_pad);
 
 /* Kernel (a): Eq. (xsplit) and the run-time half of Eq. (quant), one launch, asynchronous.
  *   X_bf16 : device, bf16 [M, K] row-major;  act_ws : device workspace (see above), written
  * Reads X once from HBM, forms p = X U on tensor cores (bf16 hi/lo split of U, float32
- * accumulation), X_perp = X - p U^T in float32, and writes codes, float32 scales and p_hat. */
+ * accumulation), X_perp = X - p U^T in float32, and writes codes, float32 scales, the epilogue
+ * constants and p_hat. */
 qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws,
                                   struct CUstream_st* stream);
 
@@ -99,8 +103,10 @@ qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, 
  *   Y      : device [M, N] row-major, bf16 (y_dtype QWAM_Y_BF16) or float32 (QWAM_Y_FP32)
  * Per group g the tensor cores form the exact integer partial sums P_g = sum_k qx qw (codes fed
  * as E4M3 multiples of 2^-9, which E4M3 holds exactly; float32 accumulation of these integer
- * multiples of 2^-18 below 2^-5 is exact); the epilogue adds s_x[m,g] s_w[g,n] P_g in float32
- * and, last, the branch p_hat B_hat (float16 operands, float32 accumulation). */
+ * multiples of 2^-18 below 2^-5 is exact); the weight bytes carry an offset of 8, so the
+ * accumulator is D = 2^-18 (P_g + 8 S_a), and the epilogue adds s_w[g,n] (alpha D + beta) =
+ * s_w[g,n] s_x[m,g] P_g in float32 and, last, the branch p_hat B_hat (float16 operands,
+ * float32 accumulation). */
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle h, void* Y, int y_dtype,
                           struct CUstream_st* stream);
 
@@ -120,7 +126,7 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
  * allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
  *
  *   - Size limit: the workspace qwam_asp_act_workspace_bytes(h, M) reports must fit in
- *     QWAM_STATIC_WS_BYTES (16 MiB: e.g. M = 4096 tokens at K = 3072, group 32 or 64, r <= 64).
+ *     QWAM_STATIC_WS_BYTES (24 MiB: e.g. M = 4096 tokens at K = 3072, group 32 or 64, r <= 64).
  *     Larger requests return QWAM_ERR_TOO_LARGE before anything is launched.
  *   - Nothing in the scratch needs to start at zero: kernel (a) writes every byte the GEMM
  *     then reads, on every call, so the scratch is never cleared.
@@ -131,7 +137,7 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
  *     with that device current) and keeps it; later calls reuse it.  Make that first call
  *     before any stream capture begins on the stream you pass.
  * Other arguments and errors are those of qwam_asp_linear; the handle's device must be current. */
-#define QWAM_STATIC_WS_BYTES (16u * 1024u * 1024u)
+#define QWAM_STATIC_WS_BYTES (24u * 1024u * 1024u)
 qwam_status qwam_asp_linear_static(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
                                    struct CUstream_st* stream);
 

@@ -26,7 +26,7 @@ QWAM_ERR_OOM = -4
 QWAM_ERR_TIMEOUT = -5
 QWAM_ERR_RANGE = -6
 QWAM_ERR_TOO_LARGE = -7
-STATIC_WS_BYTES = 16 * 1024 * 1024  # QWAM_STATIC_WS_BYTES of the header
+STATIC_WS_BYTES = 24 * 1024 * 1024  # QWAM_STATIC_WS_BYTES of the header
 QWAM_Y_BF16 = 0
 QWAM_Y_FP32 = 1
 
@@ -125,7 +125,7 @@ def qwam_asp_act_layout(h: int, M: int) -> dict:
     mp, rp = ctypes.c_int(), ctypes.c_int()
     _check(load().qwam_asp_act_layout(h, M, ctypes.byref(c), ctypes.byref(s), ctypes.byref(cs), ctypes.byref(p),
                                       ctypes.byref(mp), ctypes.byref(rp)), "qwam_asp_act_layout")
-    return dict(codes_off=c.value, scales_off=s.value, csums_off=cs.value, phat_off=p.value, M_pad=mp.value,
+    return dict(codes_off=c.value, scales_off=s.value, ab_off=cs.value, phat_off=p.value, M_pad=mp.value,
                 r_pad=rp.value)
 
 
@@ -216,15 +216,16 @@ class AspLinear:
 
     def act_views(self, M: int, ws: torch.Tensor | None = None):
         """Views of the workspace for M tokens: code bytes uint8 [M, K] (E4M3 of c * 2^-9),
-        scales f32 [K/G, M_pad], code sums f32 [K/G, M_pad], p_hat f16 [M, r_pad]."""
+        scales f32 [K/G, M_pad], epilogue constants f32 [K/G, M_pad, 2] = (alpha, beta) with
+        alpha = 2^18 s_x and beta = -8 s_x S_a, p_hat f16 [M, r_pad]."""
         ws = self.workspace(M) if ws is None else ws
         L = qwam_asp_act_layout(self.h, M)
         codes = ws[L["codes_off"]:L["codes_off"] + M * self.K].view(M, self.K)
         ns = self.K // self.group
         scales = ws[L["scales_off"]:L["scales_off"] + ns * L["M_pad"] * 4].view(torch.float32).view(ns, L["M_pad"])
-        csums = ws[L["csums_off"]:L["csums_off"] + ns * L["M_pad"] * 4].view(torch.float32).view(ns, L["M_pad"])
+        ab = ws[L["ab_off"]:L["ab_off"] + ns * L["M_pad"] * 8].view(torch.float32).view(ns, L["M_pad"], 2)
         ph = ws[L["phat_off"]:L["phat_off"] + M * self.r_pad * 2].view(torch.float16).view(M, self.r_pad)
-        return codes, scales, csums, ph
+        return codes, scales, ab, ph
 
     def quantize(self, X: torch.Tensor, stream=None) -> torch.Tensor:
         M = X.shape[0]

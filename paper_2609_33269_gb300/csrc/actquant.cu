@@ -36,7 +36,7 @@ struct ActArgs {
   int M, K, G, C, Kc, M_pad;
   uint8_t* codes;   // [M, K]
   float* scales;    // [K/G, M_pad]
-  float* csums;     // [K/G, M_pad]
+  float2* ab;       // [K/G, M_pad]: (alpha, beta)
   __half* phat;     // [M, RP]
   float* dump;      // optional [M, K]
   int* err;
@@ -83,7 +83,7 @@ __device__ __forceinline__ int nearest_code(float x, float s, float inv, float h
 
 // One group of GS remainder values -> scale, code sum and GS code bytes (E4M3 of c * 2^-9).
 template <int GS>
-__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4, float* scale_out, float* csum_out) {
+__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4, float* scale_out, float2* ab_out) {
   float amax = 0.0f;
 #pragma unroll
   for (int i = 0; i < GS; ++i) amax = fmaxf(amax, fabsf(xp[i]));
@@ -103,7 +103,9 @@ __device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4
     bytes4[w] = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
   }
   *scale_out = sc;
-  *csum_out = static_cast<float>(sum);
+  // the GEMM epilogue's constants for this token and group: alpha = 2^18 s_x (exact) and
+  // beta = -8 s_x S_a (-8 s_x is exact; one rounding)
+  *ab_out = make_float2(sc * 262144.0f, (-8.0f * sc) * static_cast<float>(sum));
 }
 
 template <int RP>
@@ -418,11 +420,11 @@ __global__ void __launch_bounds__(320, 1)
       uint32_t bytes4[16];
       if (a.G == 64) {
         const size_t gi = static_cast<size_t>(kc / 64) * a.M_pad + m;
-        quantize_group<64>(xp, bytes4, a.scales + gi, a.csums + gi);
+        quantize_group<64>(xp, bytes4, a.scales + gi, a.ab + gi);
       } else {
         const size_t gi = static_cast<size_t>(kc / 32) * a.M_pad + m;
-        quantize_group<32>(xp, bytes4, a.scales + gi, a.csums + gi);
-        quantize_group<32>(xp + 32, bytes4 + 8, a.scales + gi + a.M_pad, a.csums + gi + a.M_pad);
+        quantize_group<32>(xp, bytes4, a.scales + gi, a.ab + gi);
+        quantize_group<32>(xp + 32, bytes4 + 8, a.scales + gi + a.M_pad, a.ab + gi + a.M_pad);
       }
       uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * a.K + kc);
 #pragma unroll
@@ -462,7 +464,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
   a.codes = base + L.codes_off;
   a.scales = reinterpret_cast<float*>(base + L.scales_off);
-  a.csums = reinterpret_cast<float*>(base + L.csums_off);
+  a.ab = reinterpret_cast<float2*>(base + L.ab_off);
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
   a.dump = dump;
   a.err = h.err;

@@ -64,13 +64,25 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint6
   return r == CUDA_SUCCESS;
 }
 
+bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const uint64_t dims[3],
+               const uint64_t strides_bytes[2], const uint32_t box[3]) {
+  if (!ensure_encoder()) return false;
+  cuuint64_t d[3] = {dims[0], dims[1], dims[2]};
+  cuuint64_t st[2] = {strides_bytes[0], strides_bytes[1]};
+  cuuint32_t b[3] = {box[0], box[1], box[2]};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, dt, 3, const_cast<void*>(base), d, st, b, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 ActLayout act_layout(const Handle& h, int M) {
   ActLayout L;
   L.M_pad = round_up(M > 0 ? M : 1, kBM);
   L.codes_off = 0;
   L.scales_off = up256(static_cast<size_t>(M) * h.K);
-  L.csums_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
-  L.phat_off = L.csums_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
+  L.ab_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
+  L.phat_off = L.ab_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 8);
   L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
   return L;
 }
@@ -94,8 +106,8 @@ const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
                   CU_TENSOR_MAP_SWIZZLE_128B);
   ok &= encode_2d(&c.sx_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.scales_off, M, h.K / h.G,
                   static_cast<uint64_t>(L.M_pad) * 4, kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
-  ok &= encode_2d(&c.cs_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.csums_off, M, h.K / h.G,
-                  static_cast<uint64_t>(L.M_pad) * 4, kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
+  ok &= encode_2d(&c.ab_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.ab_off, 2 * static_cast<uint64_t>(M), h.K / h.G,
+                  static_cast<uint64_t>(L.M_pad) * 8, 2 * kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
   if (h.r_pad > 0)
     ok &= encode_2d(&c.ph_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
                     static_cast<uint64_t>(h.r_pad) * 2, 8, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
@@ -221,12 +233,12 @@ qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle hs, int M, size_t* byte
 }
 
 qwam_status qwam_asp_act_layout(qwam_asp_handle hs, int M, size_t* codes_off, size_t* scales_off,
-                                size_t* csums_off, size_t* phat_off, int* M_pad, int* r_pad) {
+                                size_t* ab_off, size_t* phat_off, int* M_pad, int* r_pad) {
   if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
   const qwam::ActLayout L = qwam::act_layout(hs->h, M);
   if (codes_off) *codes_off = L.codes_off;
   if (scales_off) *scales_off = L.scales_off;
-  if (csums_off) *csums_off = L.csums_off;
+  if (ab_off) *ab_off = L.ab_off;
   if (phat_off) *phat_off = L.phat_off;
   if (M_pad) *M_pad = L.M_pad;
   if (r_pad) *r_pad = hs->h.r_pad;

@@ -21,17 +21,18 @@
 //
 // Persistent CTAs (one per SM) walk output tiles of 128 x 128 with a static stride; every ring
 // runs continuously across tiles, so loads for the next tile overlap the epilogue of the current
-// one.  640 threads in five warpgroups:
-//   warpgroup 0 (56 registers): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2-3
+// one.  384 threads in three warpgroups (kEpiWarpsPerQuad = 2; 4 gives 640 threads):
+//   warpgroup 0 (80 registers): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2-3
 //     expand weight nibbles into the operand stage;
-//   warpgroups 1-4 (104 registers): warps 4..19 epilogue.  A warp owns 32 rows x 32 columns of
-//     the tile; TMEM is read with the 16x256b shape, so a thread holds 4 rows x 8 columns (as
-//     packed f32x2 pairs) and needs only 8 column scales s_w and 4 row scales (alpha, beta) per
-//     group: the scales reaching registers, not the arithmetic, bound a one-row-per-thread
-//     epilogue.  The floor is the FMA pipe: two operations per output and group.
+//   warpgroups 1-2 (208 registers): warps 4..11 epilogue.  A warp owns 32 rows x 64 columns of
+//     the tile; TMEM is read with the 16x256b shape, so a thread holds 4 rows x 16 columns (as
+//     packed f32x2 pairs) and, per group, loads 16 column scales s_w and the constants
+//     (alpha, beta) of its 4 rows, which kernel (a) wrote.  With one row per
+//     thread, moving the scales into registers cost as much as the arithmetic; here the floor is
+//     the FMA pipe, two operations per output and group, and the issue of everything around it.
 // Rings (each waiter waits for every phase of its slots in turn):
 //   O  operand stage = activation codes (TMA) + expanded weights (expanders)  -> MMA     SO slots
-//   P  packed weights (-> expanders) + s_x, S_a, s_w of the stage (-> epilogue)         SP slots
+//   P  packed weights (-> expanders) + alpha, beta, s_w of the stage (-> epilogue)      SP slots
 //   T  TMEM accumulators, units of two groups (2 x 128 columns)  MMA -> epilogue        NTB units
 //   B  p_hat / B_hat tiles  TMA -> MMA, loaded after the tile's stages                   one per tile
 // Every barrier operation costs on the order of 100 cycles, so each role touches as few as
@@ -70,8 +71,9 @@ constexpr int A_BYTES = kBM * kGemmKS;            // 16 KB, 128-byte swizzle
 constexpr int X_BYTES = kGemmBN * kGemmKS;        // 16 KB, 128-byte swizzle
 constexpr int OSTAGE = A_BYTES + X_BYTES;
 constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;   // 8 KB packed weights
-constexpr int PSC_BYTES = 4 * 128 * 4;            // up to 4 groups x 128 f32 (each of s_x, S_a, s_w)
-constexpr int PSTAGE = PB_BYTES + 3 * PSC_BYTES;
+constexpr int PAB_BYTES = 4 * 128 * 8;            // up to 4 groups x 128 rows x (alpha, beta)
+constexpr int PSW_BYTES = 4 * 128 * 4;            // up to 4 groups x 128 f32 s_w
+constexpr int PSTAGE = PB_BYTES + PAB_BYTES + PSW_BYTES;
 
 template <int RP>
 struct GemmCfg {
@@ -105,8 +107,7 @@ __device__ __forceinline__ f2 add2(f2 a, f2 b) {
 template <int RP>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap qx_map, const __grid_constant__ CUtensorMap qw_map,
-                const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap cs_map,
-                const __grid_constant__ CUtensorMap sw_map, const __grid_constant__ CUtensorMap ph_map,
+                const __grid_constant__ CUtensorMap ab_map, const __grid_constant__ CUtensorMap sw_map, const __grid_constant__ CUtensorMap ph_map,
                 const __grid_constant__ CUtensorMap bh_map, const GemmArgs a) {
   using Cfg = GemmCfg<RP>;
   extern __shared__ uint8_t smem_raw[];
@@ -180,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ----------------------------------------------------------- TMA producer
       if (lane == 0) {
         bool ok = true;
-        const uint32_t pbytes = PB_BYTES + gps * 3 * 128 * 4;
+        const uint32_t pbytes = PB_BYTES + gps * 128 * (8 + 4);
         int s = 0;  // running stage counter (the same sequence every role walks)
         for (int ti = 0; ti < my_tiles && ok; ++ti) {
           int m0, n0;
@@ -193,9 +194,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint8_t* p = pring + ps * PSTAGE;
             mbar_arrive_expect_tx(&pfull[ps], pbytes);
             tma_load_2d(p, &qw_map, &pfull[ps], st * (kGemmKS / 2), n0);
-            tma_load_2d(p + PB_BYTES, &sx_map, &pfull[ps], m0, st * gps);
-            tma_load_2d(p + PB_BYTES + PSC_BYTES, &cs_map, &pfull[ps], m0, st * gps);
-            tma_load_2d(p + PB_BYTES + 2 * PSC_BYTES, &sw_map, &pfull[ps], n0, st * gps);
+            tma_load_2d(p + PB_BYTES, &ab_map, &pfull[ps], 2 * m0, st * gps);
+            tma_load_2d(p + PB_BYTES + PAB_BYTES, &sw_map, &pfull[ps], n0, st * gps);
             // activation codes of this stage
             const int os = s % SO;
             if (s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
@@ -349,9 +349,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int gn = groups_in(st);
         const int ps = s % SP;
         if (ok) ok = mbar_wait_inline(&pfull[ps], (s / SP) & 1, wc);
-        const float* psx = reinterpret_cast<const float*>(pring + ps * PSTAGE + PB_BYTES);
-        const float* pcs = psx + 4 * 128;
-        const float* psw = psx + 8 * 128;
+        const float2* pab = reinterpret_cast<const float2*>(pring + ps * PSTAGE + PB_BYTES);
+        const float* psw = reinterpret_cast<const float*>(pring + ps * PSTAGE + PB_BYTES + PAB_BYTES);
         for (int g0 = 0; g0 < gn; g0 += 2, ++u_all) {
           const int ub = u_all % NTB;
           const int nmem = (g0 + 1 < gn) ? 2 : 1;
@@ -365,12 +364,9 @@ __global__ void __launch_bounds__(kThreads, 1)
               tmem_ld16x256_x4(tq + ub * 256 + mi * 128 + 32 * cb, v0[cb]);
               tmem_ld16x256_x4(tq + (16u << 16) + ub * 256 + mi * 128 + 32 * cb, v1[cb]);
             }
-            float sxr[4], csr[4];
+            float2 abr[4];  // (alpha, beta) of rows rbase + 8k
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              sxr[k] = psx[gi * 128 + rbase + 8 * k];
-              csr[k] = pcs[gi * 128 + rbase + 8 * k];
-            }
+            for (int k = 0; k < 4; ++k) abr[k] = pab[gi * 128 + rbase + 8 * k];
             f2 sw2[4 * CBW];
 #pragma unroll
             for (int j = 0; j < 4 * CBW; ++j)
@@ -382,12 +378,10 @@ __global__ void __launch_bounds__(kThreads, 1)
               tc_fence_before();
               warp_arrive(&tempty[ub]);  // every load of the unit has landed
             }
-            // acc += (alpha D + beta) * s_w, alpha = 2^18 s_x (exact), beta = -8 s_x S_a
+            // acc += (alpha D + beta) * s_w, alpha = 2^18 s_x, beta = -8 s_x S_a (from kernel (a))
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-              const float alpha = sxr[k] * 262144.0f;
-              const float beta = -8.0f * sxr[k] * csr[k];
-              const f2 al2 = dup2(alpha), be2 = dup2(beta);
+              const f2 al2 = dup2(abr[k].x), be2 = dup2(abr[k].y);
 #pragma unroll
               for (int cb = 0; cb < CBW; ++cb)
 #pragma unroll
@@ -478,7 +472,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
   const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
   const CUtensorMap& ph = (RP > 0) ? am.ph_map : am.qx_map;
   const CUtensorMap& bh = (RP > 0) ? h.Bh_map : am.qx_map;
-  gemm_kernel<RP><<<grid, kThreads, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.sx_map, am.cs_map, h.sw32_map, ph, bh, a);
+  gemm_kernel<RP><<<grid, kThreads, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.ab_map, h.sw32_map, ph, bh, a);
   return cudaGetLastError();
 }
 

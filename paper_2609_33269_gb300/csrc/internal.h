@@ -28,7 +28,7 @@ struct ActMaps {
   CUtensorMap x_map;    // X bf16 [M, K], box {64, 128}, 128-byte swizzle
   CUtensorMap qx_map;   // code bytes [M, K], box {128, 128}, 128-byte swizzle
   CUtensorMap sx_map;   // scales f32 [K/G, M_pad] (dims {M, K/G}), box {128, KS/G}
-  CUtensorMap cs_map;   // code sums f32 [K/G, M_pad], same geometry as the scales
+  CUtensorMap ab_map;   // epilogue constants f32 [K/G, M_pad, 2] (dims {2M, K/G}), box {256, KS/G}
   CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128}
 };
 
@@ -52,7 +52,7 @@ struct Handle {
 };
 
 struct ActLayout {
-  size_t codes_off, scales_off, csums_off, phat_off, bytes;
+  size_t codes_off, scales_off, ab_off, phat_off, bytes;
   int M_pad;
 };
 ActLayout act_layout(const Handle& h, int M);
@@ -60,6 +60,8 @@ ActLayout act_layout(const Handle& h, int M);
 // Tensor-map encoder (driver entry point fetched through the runtime).
 bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint64_t inner, uint64_t outer,
                uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle sw);
+bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const uint64_t dims[3],
+               const uint64_t strides_bytes[2], const uint32_t box[3]);
 const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M);
 
 uint64_t deadline_budget_ns(const Handle& h);

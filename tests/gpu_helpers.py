@@ -63,14 +63,19 @@ class Case:
         return dict(qw=unpack_nibbles(e["qw"]), sw=e["sw"], Bh=e["Bh"][:, :self.r].T.copy(), Uhl=e["Uhl"])
 
     def gpu_act(self, rows=None):
-        codes, scales, csums, ph = self.layer.act_views(self.M)
+        codes, scales, ab, ph = self.layer.act_views(self.M)
         torch.cuda.synchronize()
         qx = decode_code_bytes(codes.cpu().numpy())
         sx = scales.cpu().numpy()[:, :self.M].T.copy()
-        cs = csums.cpu().numpy()[:, :self.M].T.copy()
+        abv = ab.cpu().numpy()[:, :self.M, :].transpose(1, 0, 2).copy()  # [M, K/G, 2]
         phv = ph.cpu().numpy().view(np.uint16)[:, :self.r].copy()
-        # the code sums the GEMM uses are the exact sums of the codes
-        np.testing.assert_array_equal(cs, qx.reshape(self.M, -1, self.G).sum(axis=2).astype(np.float32))
+        # the epilogue constants are (2^18 s_x, -8 s_x S_a) with S_a the exact sum of the group's
+        # codes, each rounded once in float32
+        sa = qx.reshape(self.M, -1, self.G).sum(axis=2).astype(np.float32)
+        alpha = (sx * np.float32(262144.0)).astype(np.float32)
+        beta = ((np.float32(-8.0) * sx).astype(np.float32) * sa).astype(np.float32)
+        for i, want in enumerate((alpha, beta)):
+            np.testing.assert_array_equal(abv[:, :, i].view(np.uint32), want.view(np.uint32))
         if rows is not None:
             qx, sx, phv = qx[rows], sx[rows], phv[rows]
         return dict(qx=qx, sx=sx, ph=phv)
