@@ -18,7 +18,8 @@
 // Outputs per token row m and group g (the activation workspace):
 //   codes[m, k]   one byte per code, E4M3 bit pattern of c * 2^-9 (sign | magnitude, a
 //                 subnormal): the GEMM feeds these bytes to the tensor cores unchanged;
-//   s_x[g, m]     float32 scale;   csum[g, m]  float32 sum of the group's codes (exact);
+//   s_x[g, m]     float32 scale;   ab[g, m]  (2^18 s_x, -8 s_x S_a), S_a the group's code sum:
+//                 the GEMM epilogue's per-row constants, each rounded once;
 //   p_hat[m, :]   float16.
 //
 // Warp roles (320 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2..9
@@ -80,28 +81,49 @@ __device__ __forceinline__ int nearest_code(float x, float s, float inv, float h
   }
   return ci;
 }
+// Approximate reciprocal (the hardware's single-instruction estimate).  It only seeds the
+// rounding in nearest_code, whose exact remainder test corrects a seed that is off by one.
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
 
-// One group of GS remainder values -> scale, code sum and GS code bytes (E4M3 of c * 2^-9).
+// One group of GS remainder values -> scale, epilogue constants and GS code bytes (E4M3 of
+// c * 2^-9).  The absmax and the code sum are formed as trees (max is exact and the sum is of
+// integers, so the order does not matter), which keeps the dependency chains short.
 template <int GS>
 __device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4, float* scale_out, float2* ab_out) {
-  float amax = 0.0f;
+  float mx[8];
 #pragma unroll
-  for (int i = 0; i < GS; ++i) amax = fmaxf(amax, fabsf(xp[i]));
+  for (int j = 0; j < 8; ++j) mx[j] = fabsf(xp[j]);
+#pragma unroll
+  for (int i = 8; i < GS; ++i) mx[i & 7] = fmaxf(mx[i & 7], fabsf(xp[i]));
+#pragma unroll
+  for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+    for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
+  const float amax = mx[0];
   const float sc = __fdiv_rn(amax, 7.0f);
-  const float inv = sc > 0.0f ? __frcp_rn(sc) : 0.0f;
-  const float hs = 0.5f * sc;
-  int sum = 0;
+  // Codes are invariant under a common power-of-two scaling of the values and the scale (exact
+  // in float32), which keeps 1/s finite for the rare group whose scale is tiny.
+  const float k = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100
+  const float scs = sc * k;
+  const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
+  const float hs = 0.5f * scs;
+  int sums[4] = {0, 0, 0, 0};
 #pragma unroll
   for (int w = 0; w < GS / 4; ++w) {
     uint32_t b[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      const int ci = nearest_code(xp[4 * w + u], sc, inv, hs);
-      sum += ci;
+      const int ci = nearest_code(xp[4 * w + u] * k, scs, inv, hs);
+      sums[u] += ci;
       b[u] = static_cast<uint32_t>(abs(ci)) | (static_cast<uint32_t>(ci) & 0x80u);
     }
     bytes4[w] = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
   }
+  const int sum = (sums[0] + sums[1]) + (sums[2] + sums[3]);
   *scale_out = sc;
   // the GEMM epilogue's constants for this token and group: alpha = 2^18 s_x (exact) and
   // beta = -8 s_x S_a (-8 s_x is exact; one rounding)
