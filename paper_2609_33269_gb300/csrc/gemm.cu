@@ -179,111 +179,127 @@ __global__ void __launch_bounds__(kThreads, 1)
     setmaxnreg_dec<kRegsCtl>();
     if (wid == 0) {
       // ----------------------------------------------------------- TMA producer
-      if (lane == 0) {
-        bool ok = true;
-        const uint32_t pbytes = PB_BYTES + gps * 128 * (8 + 4);
-        int s = 0;  // running stage counter (the same sequence every role walks)
-        for (int ti = 0; ti < my_tiles && ok; ++ti) {
-          int m0, n0;
-          tile_mn(ti, m0, n0);
-          for (int st = 0; st < nst && ok; ++st, ++s) {
-            // packed weights and the group scales of this stage
-            const int ps = s % SP;
-            if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
-            if (!ok) break;
-            uint8_t* p = pring + ps * PSTAGE;
+      // The whole warp walks the loop (so addresses, coordinates and barrier phases are
+      // warp-uniform and stay in uniform registers); one elected lane issues each copy.
+      bool ok = true;
+      const uint32_t pbytes = PB_BYTES + gps * 128 * (8 + 4);
+      int s = 0;  // running stage counter (the same sequence every role walks)
+      for (int ti = 0; ti < my_tiles && ok; ++ti) {
+        int m0, n0;
+        tile_mn(ti, m0, n0);
+        for (int st = 0; st < nst && ok; ++st, ++s) {
+          // packed weights and the group scales of this stage
+          const int ps = s % SP;
+          if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
+          if (!ok) break;
+          uint8_t* p = pring + ps * PSTAGE;
+          if (elect_one()) {
             mbar_arrive_expect_tx(&pfull[ps], pbytes);
             tma_load_2d(p, &qw_map, &pfull[ps], st * (kGemmKS / 2), n0);
             tma_load_2d(p + PB_BYTES, &ab_map, &pfull[ps], 2 * m0, st * gps);
             tma_load_2d(p + PB_BYTES + PAB_BYTES, &sw_map, &pfull[ps], n0, st * gps);
-            // activation codes of this stage
-            const int os = s % SO;
-            if (s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
-            if (!ok) break;
+          }
+          __syncwarp();
+          // activation codes of this stage
+          const int os = s % SO;
+          if (s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
+          if (!ok) break;
+          if (elect_one()) {
             mbar_arrive_expect_tx(&ofull[os], A_BYTES);
             tma_load_2d(oring + os * OSTAGE, &qx_map, &ofull[os], st * kGemmKS, m0);
           }
-          if constexpr (RP > 0) {
-            // the branch operands are needed only after the tile's last stage
-            const int bs = ti % NBR;
-            if (ok && ti >= NBR) ok = mbar_wait_inline(&bempty[bs], ((ti / NBR) & 1) ^ 1, wc);
-            if (!ok) break;
-            uint8_t* b = br + bs * 2 * Cfg::BR_BYTES;
+          __syncwarp();
+        }
+        if constexpr (RP > 0) {
+          // the branch operands are needed only after the tile's last stage
+          const int bs = ti % NBR;
+          if (ok && ti >= NBR) ok = mbar_wait_inline(&bempty[bs], ((ti / NBR) & 1) ^ 1, wc);
+          if (!ok) break;
+          uint8_t* b = br + bs * 2 * Cfg::BR_BYTES;
+          if (elect_one()) {
             mbar_arrive_expect_tx(&bfull[bs], 2 * Cfg::BR_BYTES);
             for (int q = 0; q < RP / 8; ++q) {
               tma_load_2d(b + q * 2048, &ph_map, &bfull[bs], q * 8, m0);
               tma_load_2d(b + Cfg::BR_BYTES + q * 2048, &bh_map, &bfull[bs], q * 8, n0);
             }
           }
+          __syncwarp();
         }
-        // Let every issued load land before the CTA can exit (these phases complete in the
-        // normal course; after an abort the waits end at the deadline).
-        int never = 0;
-        const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-        for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
-        // An operand stage also needs the expanders' arrivals: in the normal course they come;
-        // after an abort the wait ends at the deadline, long after the tile has landed.
-        for (int j = (s > SO ? s - SO : 0); j < s; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
-        if constexpr (RP > 0) {
-          for (int t = (my_tiles > NBR ? my_tiles - NBR : 0); t < my_tiles; ++t)
-            mbar_wait_inline(&bfull[t % NBR], (t / NBR) & 1, dc);
-        }
+      }
+      // Let every issued load land before the CTA can exit (these phases complete in the
+      // normal course; after an abort the waits end at the deadline).
+      int never = 0;
+      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+      for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
+      // An operand stage also needs the expanders' arrivals: in the normal course they come;
+      // after an abort the wait ends at the deadline, long after the tile has landed.
+      for (int j = (s > SO ? s - SO : 0); j < s; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
+      if constexpr (RP > 0) {
+        for (int t = (my_tiles > NBR ? my_tiles - NBR : 0); t < my_tiles; ++t)
+          mbar_wait_inline(&bfull[t % NBR], (t / NBR) & 1, dc);
       }
     } else if (wid == 1) {
       // ----------------------------------------------------------- MMA issuer
       // The epilogue consumes accumulators in units of two groups (one TMEM buffer of 2 x 128
       // columns); a unit never straddles a stage because a full stage holds an even number of
-      // groups.  One tcgen05 fence per unit: fences and commits cost far more than an MMA issue.
-      if (lane == 0) {
-        bool ok = true;
-        constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
-        int s = 0, u_all = 0;  // running stage and accumulator-unit counters
-        for (int ti = 0; ti < my_tiles && ok; ++ti) {
-          for (int st = 0; st < nst && ok; ++st, ++s) {
-            const int gn = groups_in(st);
-            const int os = s % SO;
-            ok = mbar_wait_inline(&ofull[os], (s / SO) & 1, wc);
+      // groups.  The whole warp walks the loop and forms the descriptors (warp-uniform values);
+      // one elected lane (the same one throughout, as the commits track its MMAs) issues.
+      bool ok = true;
+      constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
+      int s = 0, u_all = 0;  // running stage and accumulator-unit counters
+      for (int ti = 0; ti < my_tiles && ok; ++ti) {
+        for (int st = 0; st < nst && ok; ++st, ++s) {
+          const int gn = groups_in(st);
+          const int os = s % SO;
+          ok = mbar_wait_inline(&ofull[os], (s / SO) & 1, wc);
+          if (!ok) break;
+          const uint32_t aa = smem_u32(oring + os * OSTAGE), xa = aa + A_BYTES;
+          const uint64_t adesc0 = smem_desc(aa, 16, 1024, kSw128), xdesc0 = smem_desc(xa, 16, 1024, kSw128);
+          for (int g0 = 0; g0 < gn && ok; g0 += 2, ++u_all) {
+            const int ub = u_all % NTB;
+            if (u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
             if (!ok) break;
-            const uint32_t aa = smem_u32(oring + os * OSTAGE), xa = aa + A_BYTES;
-            for (int g0 = 0; g0 < gn && ok; g0 += 2, ++u_all) {
-              const int ub = u_all % NTB;
-              if (u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
-              if (!ok) break;
-              tc_fence_after();
-              for (int gi = g0; gi < gn && gi < g0 + 2; ++gi)
+            tc_fence_after();
+            const int g1 = (g0 + 2 < gn) ? g0 + 2 : gn;
+            if (elect_one()) {
+              for (int gi = g0; gi < g1; ++gi)
                 for (int kk = 0; kk < G / 32; ++kk) {
-                  const uint32_t off = static_cast<uint32_t>((gi * (G / 32) + kk) * 32);
-                  mma_f8f6f4(tmem + ub * 256 + (gi - g0) * 128, smem_desc(aa + off, 16, 1024, kSw128),
-                             smem_desc(xa + off, 16, 1024, kSw128), idesc, kk != 0);
+                  const uint64_t off = static_cast<uint64_t>((gi * (G / 32) + kk) * 32) >> 4;  // 16-byte units
+                  mma_f8f6f4(tmem + ub * 256 + (gi - g0) * 128, adesc0 + off, xdesc0 + off, idesc, kk != 0);
                 }
               mma_commit(&tfull[ub]);
             }
-            mma_commit(&oempty[os]);
+            __syncwarp();
           }
-          if constexpr (RP > 0) {
-            const int bs = ti % NBR, ub = u_all % NTB;
-            if (ok) ok = mbar_wait_inline(&bfull[bs], (ti / NBR) & 1, wc);
-            if (ok && u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
-            if (ok) {
-              tc_fence_after();
-              constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
-              const uint32_t pa = smem_u32(br + bs * 2 * Cfg::BR_BYTES), pb = pa + Cfg::BR_BYTES;
+          if (elect_one()) mma_commit(&oempty[os]);
+          __syncwarp();
+        }
+        if constexpr (RP > 0) {
+          const int bs = ti % NBR, ub = u_all % NTB;
+          if (ok) ok = mbar_wait_inline(&bfull[bs], (ti / NBR) & 1, wc);
+          if (ok && u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
+          if (ok) {
+            tc_fence_after();
+            constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
+            const uint32_t pa = smem_u32(br + bs * 2 * Cfg::BR_BYTES), pb = pa + Cfg::BR_BYTES;
+            const uint64_t pdesc0 = smem_desc(pa, 2048, 128, kSwNone), bdesc0 = smem_desc(pb, 2048, 128, kSwNone);
+            if (elect_one()) {
 #pragma unroll
               for (int kk = 0; kk < RP / 16; ++kk)
-                mma_f16(tmem + ub * 256, smem_desc(pa + kk * 4096, 2048, 128, kSwNone),
-                        smem_desc(pb + kk * 4096, 2048, 128, kSwNone), idesc_br, kk != 0);
+                mma_f16(tmem + ub * 256, pdesc0 + kk * 256, bdesc0 + kk * 256, idesc_br, kk != 0);  // 4096 B
               mma_commit(&tfull[ub]);
               mma_commit(&bempty[bs]);
-              ++u_all;
             }
+            __syncwarp();
+            ++u_all;
           }
         }
-        mma_commit(drain);
-        int never = 0;
-        const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-        mbar_wait_inline(drain, 0, dc);
       }
+      if (elect_one()) mma_commit(drain);
       __syncwarp();
+      int never = 0;
+      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+      mbar_wait_inline(drain, 0, dc);
     } else {
       // ----------------------------------------------------------- weight expanders
       // Thread e (0..63) owns the 16-byte chunk j = e % 8 of rows e/8 + 8 i (i = 0..15): its source
