@@ -36,9 +36,10 @@ def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
 class Case:
     """One layer on both sides: host inputs, the packed GPU layer, oracle outputs on demand."""
 
-    def __init__(self, M, K, N, r, G=64, seed=0, layer_id=0, dist="outlier", n_outlier=None):
+    def __init__(self, M, K, N, r, G=64, seed=0, layer_id=0, dist="outlier", n_outlier=None, Xb=None):
         self.M, self.K, self.N, self.r, self.G = M, K, N, r, G
-        self.Xb = wl.activations(M, K, seed=seed, layer_id=layer_id, dist=dist, n_outlier=n_outlier)
+        self.Xb = (wl.activations(M, K, seed=seed, layer_id=layer_id, dist=dist, n_outlier=n_outlier)
+                   if Xb is None else np.ascontiguousarray(Xb, np.uint16))
         self.Wb = wl.weight(K, N, seed=seed, layer_id=layer_id)
         self.U = wl.basis(K, r, seed=seed, layer_id=layer_id)
         self.X = to_dev_bf16(self.Xb)

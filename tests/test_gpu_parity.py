@@ -188,19 +188,21 @@ def test_gpu_handles_reject_bad_arguments():
         c.close()
 
 
-FULL = [  # (name, M, K, N, r, dist) in the launch configuration the benchmark times
-    ("dit_attn", 4096, 3072, 3072, 32, "outlier"),
-    ("ffn_up", 4096, 3072, 12288, 32, "outlier"),
-    ("ffn_down", 4096, 12288, 3072, 32, "student_t"),
-    ("small_M32_r16", 32, 1024, 1024, 16, "outlier"),
-    ("small_M128_N4096_r0", 128, 1024, 4096, 0, "outlier"),
+FULL = [  # (name, M, K, N, r, dist, G) in the launch configuration the benchmark times
+    ("dit_attn", 4096, 3072, 3072, 32, "outlier", 64),
+    ("dit_attn_g32", 4096, 3072, 3072, 32, "outlier", 32),
+    ("dit_qkv", 4096, 3072, 9216, 32, "outlier", 64),
+    ("ffn_up", 4096, 3072, 12288, 32, "outlier", 64),
+    ("ffn_down", 4096, 12288, 3072, 32, "student_t", 64),
+    ("small_M32_r16", 32, 1024, 1024, 16, "outlier", 64),
+    ("small_M128_N4096_r0", 128, 1024, 4096, 0, "outlier", 64),
 ]
 
 
 @pytest.mark.parametrize("cfg", FULL, ids=lambda c: c[0])
 def test_full_size_sampled_rows(cfg):
-    name, M, K, N, r, dist = cfg
-    c = Case(M, K, N, r, 64, seed=0, layer_id=FULL.index(cfg) + 1, dist=dist)
+    name, M, K, N, r, dist, G = cfg
+    c = Case(M, K, N, r, G, seed=0, layer_id=FULL.index(cfg) + 1, dist=dist)
     try:
         Y = c.run(fp32=True).cpu().numpy()
         rows = np.unique(np.random.default_rng(0).choice(M, size=min(M, 48), replace=False))
@@ -211,14 +213,14 @@ def test_full_size_sampled_rows(cfg):
         np.testing.assert_array_equal(gw["qw"], ow["qw"])
         np.testing.assert_array_equal(gw["sw"], ow["sw"])
         oa = c.oracle_act(rows)
-        Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), 64)
+        Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), G)
         assert rowwise_rel_err(Y[rows], Yk).max() <= 1e-5
-        Yo = oracle.linear(oa, ow, 64)
+        Yo = oracle.linear(oa, ow, G)
         check_layer_output(Y[rows], Yo, Yk, ga["qx"], oa["qx"])
         if r == 0:
             np.testing.assert_array_equal(ga["qx"], oa["qx"])
         else:
-            bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], 64, 1e-3)
+            bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], G, 1e-3)
             assert len(bad) <= max(2, 1e-4 * ga["qx"].size) and near.all()
     finally:
         c.close()
