@@ -104,10 +104,8 @@ const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
   }
   ok &= encode_2d(&c.qx_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K, M, h.K, kGemmKS, kBM,
                   CU_TENSOR_MAP_SWIZZLE_128B);
-  ok &= encode_2d(&c.sx_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.scales_off, M, h.K / h.G,
-                  static_cast<uint64_t>(L.M_pad) * 4, kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
   ok &= encode_2d(&c.ab_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.ab_off, 2 * static_cast<uint64_t>(M), h.K / h.G,
-                  static_cast<uint64_t>(L.M_pad) * 8, 2 * kBM, kGemmKS / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
+                  static_cast<uint64_t>(L.M_pad) * 8, 2 * kBM, kScaleGroups, CU_TENSOR_MAP_SWIZZLE_NONE);
   if (h.r_pad > 0)
     ok &= encode_2d(&c.ph_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
                     static_cast<uint64_t>(h.r_pad) * 2, 8, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
@@ -197,7 +195,7 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kGemmKS / 2, qwam::kBM,
                         CU_TENSOR_MAP_SWIZZLE_NONE);
   ok &= qwam::encode_2d(&h.sw32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, h.sw32, N, K / group,
-                        static_cast<uint64_t>(h.N_pad) * 4, qwam::kGemmBN, qwam::kGemmKS / group,
+                        static_cast<uint64_t>(h.N_pad) * 4, qwam::kGemmBN, qwam::kScaleGroups,
                         CU_TENSOR_MAP_SWIZZLE_NONE);
   if (h.r_pad > 0) {
     ok &= qwam::encode_2d(&h.Bh_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,

@@ -32,12 +32,13 @@
 //     the FMA pipe, two operations per output and group, and the issue of everything around it.
 // Rings (each waiter waits for every phase of its slots in turn):
 //   O  operand stage = activation codes (TMA) + expanded weights (expanders)  -> MMA     SO slots
-//   P  packed weights (-> expanders) + alpha, beta, s_w of the stage (-> epilogue)      SP slots
+//   P  packed weights of a stage  TMA -> expanders                                      SP slots
+//   S  alpha, beta, s_w of eight groups  TMA -> epilogue                                SS slots
 //   T  TMEM accumulators, units of two groups (2 x 128 columns)  MMA -> epilogue        NTB units
 //   B  p_hat / B_hat tiles  TMA -> MMA, loaded after the tile's stages                   one per tile
 // Every barrier operation costs on the order of 100 cycles, so each role touches as few as
 // possible per stage: the MMA warp waits twice and commits twice, the expanders wait twice and
-// arrive once, the epilogue waits twice and arrives twice.
+// arrive twice, the epilogue waits once and arrives once per unit, plus once each per S slot.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -62,7 +63,8 @@ constexpr int kRegsEpi = kEpiWarpsPerQuad == 4 ? 104 : 208;   // the epilogue wa
 static_assert(128 * kRegsCtl + (kThreads - 128) * kRegsEpi <= kThreads * kLaunchRegs,
               "register split above the launch allocation");
 constexpr int SO = 3;     // operand stages
-constexpr int SP = 6;     // packed-weight + scale stages
+constexpr int SP = 6;     // packed-weight stages
+constexpr int SS = 3;     // scale stages (kScaleGroups groups each)
 constexpr int NTB = 2;    // TMEM accumulator units (2 x 128 columns each)
 constexpr int NBR = 1;    // branch-operand stages (one per tile)
 constexpr int NXW = 2;    // expander warps
@@ -71,15 +73,16 @@ constexpr int A_BYTES = kBM * kGemmKS;            // 16 KB, 128-byte swizzle
 constexpr int X_BYTES = kGemmBN * kGemmKS;        // 16 KB, 128-byte swizzle
 constexpr int OSTAGE = A_BYTES + X_BYTES;
 constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;   // 8 KB packed weights
-constexpr int PAB_BYTES = 4 * 128 * 8;            // up to 4 groups x 128 rows x (alpha, beta)
-constexpr int PSW_BYTES = 4 * 128 * 4;            // up to 4 groups x 128 f32 s_w
-constexpr int PSTAGE = PB_BYTES + PAB_BYTES + PSW_BYTES;
+constexpr int PSTAGE = PB_BYTES;
+constexpr int SAB_BYTES = kScaleGroups * 128 * 8;  // 8 groups x 128 rows x (alpha, beta)
+constexpr int SSW_BYTES = kScaleGroups * 128 * 4;  // 8 groups x 128 f32 s_w
+constexpr int SSTAGE = SAB_BYTES + SSW_BYTES;      // 12 KB
 
 template <int RP>
 struct GemmCfg {
   static constexpr int BR_BYTES = RP * kBM * 2;   // p_hat tile (and the B_hat tile), RP/8 boxes of 2 KB
-  static constexpr int NBAR = 2 * SO + 2 * SP + 2 * NTB + 2 * NBR + 1;
-  static constexpr int SMEM = 1024 + SO * OSTAGE + SP * PSTAGE + NBR * 2 * BR_BYTES + NBAR * 8 + 16;
+  static constexpr int NBAR = 2 * SO + 2 * SP + 2 * SS + 2 * NTB + 2 * NBR + 1;
+  static constexpr int SMEM = 1024 + SO * OSTAGE + SP * PSTAGE + SS * SSTAGE + NBR * 2 * BR_BYTES + NBAR * 8 + 16;
   static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 };
 
@@ -113,14 +116,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* oring = smem;                           // SO x (A 16 KB | X 16 KB), 1024-aligned
-  uint8_t* pring = oring + SO * OSTAGE;            // SP x (weights packed | s_x | S_a | s_w)
-  uint8_t* br = pring + SP * PSTAGE;               // NBR x (p_hat | B_hat)
+  uint8_t* pring = oring + SO * OSTAGE;            // SP x packed weights
+  uint8_t* sring = pring + SP * PSTAGE;            // SS x ((alpha, beta) | s_w)
+  uint8_t* br = sring + SS * SSTAGE;               // NBR x (p_hat | B_hat)
   uint64_t* bars = reinterpret_cast<uint64_t*>(br + NBR * 2 * Cfg::BR_BYTES);
   uint64_t* ofull = bars;
   uint64_t* oempty = ofull + SO;
   uint64_t* pfull = oempty + SO;
   uint64_t* pempty = pfull + SP;
-  uint64_t* tfull = pempty + SP;
+  uint64_t* sfull = pempty + SP;
+  uint64_t* sempty = sfull + SS;
+  uint64_t* tfull = sempty + SS;
   uint64_t* tempty = tfull + NTB;
   uint64_t* bfull = tempty + NTB;
   uint64_t* bempty = bfull + NBR;
@@ -144,6 +150,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     n0 = (t % a.n_tiles) * kGemmBN;
   };
   auto groups_in = [&](int st) { return (st * gps + gps <= ngroups) ? gps : ngroups - st * gps; };
+  // A scale stage starts with every K stage whose first group is a multiple of kScaleGroups
+  // (gps divides kScaleGroups) and ends with the K stage that reaches the next one, or K.
+  auto scale_starts = [&](int st) { return (st * gps) % kScaleGroups == 0; };
+  auto scale_ends = [&](int st) { return ((st + 1) * gps) % kScaleGroups == 0 || st + 1 == nst; };
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < SO; ++i) {
@@ -152,7 +162,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < SP; ++i) {
       mbar_init(&pfull[i], 1);
-      mbar_init(&pempty[i], NEPIW);
+      mbar_init(&pempty[i], NXW);
+    }
+    for (int i = 0; i < SS; ++i) {
+      mbar_init(&sfull[i], 1);
+      mbar_init(&sempty[i], NEPIW);
     }
     for (int i = 0; i < NTB; ++i) {
       mbar_init(&tfull[i], 1);
@@ -182,22 +196,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       // The whole warp walks the loop (so addresses, coordinates and barrier phases are
       // warp-uniform and stay in uniform registers); one elected lane issues each copy.
       bool ok = true;
-      const uint32_t pbytes = PB_BYTES + gps * 128 * (8 + 4);
-      int s = 0;  // running stage counter (the same sequence every role walks)
+      int s = 0, ss = 0;  // running K-stage and scale-stage counters (every role walks the same)
       for (int ti = 0; ti < my_tiles && ok; ++ti) {
         int m0, n0;
         tile_mn(ti, m0, n0);
         for (int st = 0; st < nst && ok; ++st, ++s) {
-          // packed weights and the group scales of this stage
+          if (scale_starts(st)) {
+            // (alpha, beta) and s_w of the next kScaleGroups groups (zero-filled past K)
+            const int sb = ss % SS;
+            if (ss >= SS) ok = mbar_wait_inline(&sempty[sb], ((ss / SS) & 1) ^ 1, wc);
+            if (!ok) break;
+            uint8_t* q = sring + sb * SSTAGE;
+            if (elect_one()) {
+              mbar_arrive_expect_tx(&sfull[sb], SSTAGE);
+              tma_load_2d(q, &ab_map, &sfull[sb], 2 * m0, st * gps);
+              tma_load_2d(q + SAB_BYTES, &sw_map, &sfull[sb], n0, st * gps);
+            }
+            __syncwarp();
+            ++ss;
+          }
+          // packed weights of this stage
           const int ps = s % SP;
           if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
           if (!ok) break;
           uint8_t* p = pring + ps * PSTAGE;
           if (elect_one()) {
-            mbar_arrive_expect_tx(&pfull[ps], pbytes);
+            mbar_arrive_expect_tx(&pfull[ps], PB_BYTES);
             tma_load_2d(p, &qw_map, &pfull[ps], st * (kGemmKS / 2), n0);
-            tma_load_2d(p + PB_BYTES, &ab_map, &pfull[ps], 2 * m0, st * gps);
-            tma_load_2d(p + PB_BYTES + PAB_BYTES, &sw_map, &pfull[ps], n0, st * gps);
           }
           __syncwarp();
           // activation codes of this stage
@@ -231,6 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int never = 0;
       const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
       for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
+      for (int j = (ss > SS ? ss - SS : 0); j < ss; ++j) mbar_wait_inline(&sfull[j % SS], (j / SS) & 1, dc);
       // An operand stage also needs the expanders' arrivals: in the normal course they come;
       // after an abort the wait ends at the deadline, long after the tile has landed.
       for (int j = (s > SO ? s - SO : 0); j < s; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
@@ -335,9 +361,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           // Orders the generic writes of the expanded weights before the MMA reads them, and the
-          // generic reads of the packed stage before TMA refills it (the epilogue releases it).
+          // generic reads of the packed stage before TMA refills it.
           fence_proxy_async_smem();
           warp_arrive(&ofull[os]);
+          if (lane == 0) mbar_arrive(&pempty[ps]);
         }
       }
     }
@@ -354,7 +381,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rbase = quad * 32 + rq;
     const uint32_t tq = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
     bool ok = true;
-    int u_all = 0, s = 0;  // accumulator-unit and stage counters
+    int u_all = 0, s = 0, ss = 0;  // accumulator-unit, K-stage and scale-stage counters
     for (int ti = 0; ti < my_tiles; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
@@ -363,10 +390,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = 0; i < 16 * CBW; ++i) acc[i] = 0ull;
       for (int st = 0; st < nst; ++st, ++s) {
         const int gn = groups_in(st);
-        const int ps = s % SP;
-        if (ok) ok = mbar_wait_inline(&pfull[ps], (s / SP) & 1, wc);
-        const float2* pab = reinterpret_cast<const float2*>(pring + ps * PSTAGE + PB_BYTES);
-        const float* psw = reinterpret_cast<const float*>(pring + ps * PSTAGE + PB_BYTES + PAB_BYTES);
+        const int sb = ss % SS;
+        if (scale_starts(st) && ok) ok = mbar_wait_inline(&sfull[sb], (ss / SS) & 1, wc);
+        const int gl0 = (st * gps) % kScaleGroups;  // the stage's first group within the scale stage
+        const float2* pab = reinterpret_cast<const float2*>(sring + sb * SSTAGE) + gl0 * 128;
+        const float* psw = reinterpret_cast<const float*>(sring + sb * SSTAGE + SAB_BYTES) + gl0 * 128;
         for (int g0 = 0; g0 < gn; g0 += 2, ++u_all) {
           const int ub = u_all % NTB;
           const int nmem = (g0 + 1 < gn) ? 2 : 1;
@@ -408,8 +436,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        fence_proxy_async_smem();  // reads of the TMA-written scales before the stage is refilled
-        warp_arrive(&pempty[ps]);
+        if (scale_ends(st)) {
+          fence_proxy_async_smem();  // reads of the TMA-written scales before the slot is refilled
+          warp_arrive(&sempty[sb]);
+          ++ss;
+        }
       }
       if constexpr (RP > 0) {
         const int ub = u_all % NTB;

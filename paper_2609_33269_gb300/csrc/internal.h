@@ -17,6 +17,7 @@ constexpr int kChunk = 64;      // K columns per activation chunk (bf16: one 128
 constexpr int kMaxRank = 64;    // largest protected rank of this build
 constexpr int kGemmBN = 128;    // output columns per GEMM CTA tile
 constexpr int kGemmKS = 128;    // K elements per GEMM pipeline stage
+constexpr int kScaleGroups = 8; // groups per GEMM scale stage (epilogue constants and s_w)
 
 inline int round_up(int a, int b) { return (a + b - 1) / b * b; }
 
@@ -27,8 +28,7 @@ struct ActMaps {
   int M = -1;
   CUtensorMap x_map;    // X bf16 [M, K], box {64, 128}, 128-byte swizzle
   CUtensorMap qx_map;   // code bytes [M, K], box {128, 128}, 128-byte swizzle
-  CUtensorMap sx_map;   // scales f32 [K/G, M_pad] (dims {M, K/G}), box {128, KS/G}
-  CUtensorMap ab_map;   // epilogue constants f32 [K/G, M_pad, 2] (dims {2M, K/G}), box {256, KS/G}
+  CUtensorMap ab_map;   // epilogue constants f32 [K/G, M_pad, 2] (dims {2M, K/G}), box {256, 8}
   CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128}
 };
 
