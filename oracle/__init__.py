@@ -5,6 +5,10 @@ load this module; the library under ``paper_2609_33269_gb300`` never imports it 
 code with it.  The arithmetic lives in ``qwam_oracle.c`` (float64 / int64, OpenMP over rows);
 this file only compiles it with gcc and marshals numpy arrays through ctypes.
 
+The NVFP4 variant (App. B.1's Blackwell format) has its own entry points with the suffix
+``_nvfp4``: E2M1 codes (one 4-bit code per uint8), E4M3 block scales (uint8 bits, one per 16
+consecutive K entries) and one float32 scale per weight tensor.
+
 Every function returns semantic arrays in the paper's row-major notation:
 X [M,K] tokens, W [K,N], U [K,r] (the paper's V), codes as int8 in [-7, 7], activation scales
 float32 [M, K/G], weight scales float16 [K/G, N], branch factors float16.
@@ -58,6 +62,18 @@ def _load():
             lib.qo_f16_value.restype = ctypes.c_double
             lib.qo_nearest_code.argtypes = [ctypes.c_double, ctypes.c_double]
             lib.qo_nearest_code.restype = ctypes.c_int
+            lib.qo_pack_nvfp4.argtypes = [P, P, I, I, I, P, P, P, P]
+            lib.qo_quantize_act_nvfp4.argtypes = [P, P, I, I, I, P, P, P]
+            lib.qo_quantize_residual_nvfp4_f32.argtypes = [P, I, I, P, P]
+            lib.qo_linear_nvfp4.argtypes = [P, P, P, P, P, ctypes.c_float, P, I, I, I, I, P]
+            lib.qo_e2m1_value.argtypes = [I]
+            lib.qo_e2m1_value.restype = ctypes.c_double
+            lib.qo_e2m1_code_rn.argtypes = [ctypes.c_double]
+            lib.qo_e2m1_code_rn.restype = I
+            lib.qo_e4m3_value.argtypes = [ctypes.c_uint8]
+            lib.qo_e4m3_value.restype = ctypes.c_double
+            lib.qo_e4m3_bits_rn.argtypes = [ctypes.c_double]
+            lib.qo_e4m3_bits_rn.restype = ctypes.c_uint8
             _lib = lib
     return _lib
 
@@ -180,3 +196,89 @@ def f16_value(h: int) -> float:
 
 def nearest_code(x: float, s: float) -> int:
     return int(_load().qo_nearest_code(float(x), float(s)))
+
+
+# ---- NVFP4 variant (App. B.1) ----------------------------------------------------------------
+
+FP4_BLOCK = 16
+
+
+def pack_nvfp4(W_bf16_bits, U):
+    """Offline packing of the NVFP4 variant (readings N1, N2, N4 of qwam_oracle.c).
+
+    Returns dict(qw uint8 E2M1 codes [N,K], sfw uint8 E4M3 bits [N,K/16], sg float32,
+    Bh uint16 fp16-bits [r,N])."""
+    W = _c(W_bf16_bits, np.uint16)
+    K, N = W.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qw = np.empty((N, K), np.uint8)
+    sfw = np.empty((N, K // FP4_BLOCK), np.uint8)
+    sg = ctypes.c_float(0.0)
+    Bh = np.empty((r, N), np.uint16)
+    _check(_load().qo_pack_nvfp4(_ptr(W), _ptr(U), K, N, r, _ptr(qw), _ptr(sfw), ctypes.byref(sg), _ptr(Bh)),
+           "pack_nvfp4")
+    return dict(qw=qw, sfw=sfw, sg=np.float32(sg.value), Bh=Bh)
+
+
+def quantize_act_nvfp4(X_bf16_bits, U):
+    """Activation path of the NVFP4 variant (Eq. (xsplit), reading N3).
+
+    Returns dict(qx uint8 E2M1 codes [M,K], sfx uint8 E4M3 bits [M,K/16], ph uint16 [M,r])."""
+    X = _c(X_bf16_bits, np.uint16)
+    M, K = X.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qx = np.empty((M, K), np.uint8)
+    sfx = np.empty((M, K // FP4_BLOCK), np.uint8)
+    ph = np.empty((M, r), np.uint16)
+    _check(_load().qo_quantize_act_nvfp4(_ptr(X), _ptr(U), M, K, r, _ptr(qx), _ptr(sfx), _ptr(ph)),
+           "quantize_act_nvfp4")
+    return dict(qx=qx, sfx=sfx, ph=ph)
+
+
+def quantize_residual_nvfp4(R_f32):
+    """Reading N3 alone on a float32 remainder R [M,K] -> (codes uint8 [M,K], E4M3 bits [M,K/16])."""
+    R = _c(R_f32, np.float32)
+    M, K = R.shape
+    q = np.empty((M, K), np.uint8)
+    sf = np.empty((M, K // FP4_BLOCK), np.uint8)
+    _check(_load().qo_quantize_residual_nvfp4_f32(_ptr(R), M, K, _ptr(q), _ptr(sf)), "quantize_residual_nvfp4")
+    return q, sf
+
+
+def linear_nvfp4(act, wts):
+    """Layer output of the NVFP4 variant (reading N5) -> float64 Y [M,N]."""
+    qx = _c(act["qx"], np.uint8)
+    M, K = qx.shape
+    qw = _c(wts["qw"], np.uint8)
+    N = qw.shape[0]
+    r = wts["Bh"].shape[0]
+    Y = np.empty((M, N), np.float64)
+    _check(_load().qo_linear_nvfp4(_ptr(qx), _ptr(_c(act["sfx"], np.uint8)), _ptr(_c(act["ph"], np.uint16)),
+                                   _ptr(qw), _ptr(_c(wts["sfw"], np.uint8)), float(wts["sg"]),
+                                   _ptr(_c(wts["Bh"], np.uint16)), M, K, N, r, _ptr(Y)), "linear_nvfp4")
+    return Y
+
+
+def forward_nvfp4(X_bf16_bits, W_bf16_bits, U):
+    """Whole NVFP4 layer: pack, quantize the activations, output.  Returns (Y, act, wts)."""
+    wts = pack_nvfp4(W_bf16_bits, U)
+    act = quantize_act_nvfp4(X_bf16_bits, U)
+    return linear_nvfp4(act, wts), act, wts
+
+
+def e2m1_value(c: int) -> float:
+    return float(_load().qo_e2m1_value(int(c)))
+
+
+def e2m1_code(x: float) -> int:
+    return int(_load().qo_e2m1_code_rn(float(x)))
+
+
+def e4m3_value(b: int) -> float:
+    return float(_load().qo_e4m3_value(int(b)))
+
+
+def e4m3_bits(x: float) -> int:
+    return int(_load().qo_e4m3_bits_rn(float(x)))

@@ -305,3 +305,246 @@ int qo_linear_split_exact(const double* p, const double* Xperp, const double* Bf
 uint16_t qo_f16_bits_rn(double x) { return f16_bits_rn(x); }
 double qo_f16_value(uint16_t h) { return f16_value(h); }
 int qo_nearest_code(double x, double s) { return nearest_code(x, s); }
+
+/* ==== NVFP4 variant (App. B.1: on Blackwell GPUs the paper stores E2M1 values with an E4M3
+ * scale per group of 16 elements, for weights and activations, and one extra float32 scale per
+ * weight tensor).  The paper gives the storage format only; the readings below fix the rest.
+ *   N1  E2M1 (OCP FP4): sign | 2-bit exponent (bias 1) | 1-bit mantissa.  Magnitudes of codes
+ *       0..7: 0, 0.5, 1, 1.5, 2, 3, 4, 6.  Rounding to E2M1 is to nearest, ties to an even
+ *       mantissa bit, and saturates at 6.
+ *   N2  E4M3 (OCP FP8, "FN"): sign | 4-bit exponent (bias 7) | 3-bit mantissa; no infinities;
+ *       largest finite 448; subnormals m * 2^-9.  Rounding is to nearest, ties to even, and
+ *       saturates at 448.
+ *   N3  activations, per token and block b of 16 consecutive K entries of x_perp (float32):
+ *       s = RN_e4m3(RN_f32(amax_b / 6)),  code = RN_e2m1(RN_f32(x / s)),  s == 0 -> codes 0.
+ *   N4  weights: s_g = RN_f32(amax(W_perp) / (6 * 448)); per output channel n and block b,
+ *       s_b = RN_e4m3(amax_b / (6 s_g)) and code = RN_e2m1(w / (s_b s_g)), both from the
+ *       float64 quotient (whose one rounding cannot change a 4-bit or 2-bit result:
+ *       53 >= 2 * 4 + 2); s_g == 0 or s_b == 0 -> codes 0.
+ *   N5  output: y = s_g * sum_b s_a s_b sum_{k in b} e2m1(qa) e2m1(qb)  +  sum_j p_hat_j B_hat_j.
+ * Block length is 16; K must be a multiple of 16. */
+
+#define QO_FP4_BLOCK 16
+
+/* E2M1 code (4 bits) -> value. */
+static double e2m1_value(int c) {
+  static const double mag[8] = {0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0};
+  double v = mag[c & 7];
+  return (c & 8) ? -v : v;
+}
+
+/* E4M3 bits -> value (reading N2).  0x7f / 0xff are NaN. */
+static double e4m3_value(uint8_t b) {
+  int s = b >> 7, e = (b >> 3) & 15, m = b & 7;
+  double v;
+  if (e == 15 && m == 7)
+    v = NAN;
+  else if (e == 0)
+    v = ldexp((double)m, -9);
+  else
+    v = ldexp((double)(8 + m), e - 10);
+  return s ? -v : v;
+}
+
+/* value -> E4M3 bits, nearest, ties to even, saturating at 448 (reading N2).  As in f16_bits_rn:
+ * scale by a power of two so that one quantum of the binade is 1, then nearbyint(). */
+static uint8_t e4m3_bits_rn(double x) {
+  uint8_t sign = signbit(x) ? 0x80 : 0;
+  double a = fabs(x);
+  if (isnan(x)) return 0x7f;
+  if (a == 0.0) return sign;
+  if (a >= 448.0) return sign | 0x7e; /* saturate */
+  int e2;
+  frexp(a, &e2);
+  int E = e2 - 1;        /* a in [2^E, 2^(E+1)) */
+  if (E < -6) E = -6;    /* subnormal binade: quantum 2^-9 */
+  double q = nearbyint(ldexp(a, 3 - E)); /* quanta of 2^(E-3): 0 .. 16 */
+  if (q >= 16.0) {
+    q = 8.0;
+    E += 1;
+  }
+  if (E == -6 && q < 8.0) return sign | (uint8_t)q; /* subnormal (or zero) */
+  if (E > 8) return sign | 0x7e;                   /* 2^9 and beyond: above 448 */
+  int code = ((E + 7) << 3) | ((int)q - 8);
+  if (code > 0x7e) code = 0x7e;                    /* 464 .. 480 round to 448 by saturation */
+  return sign | (uint8_t)code;
+}
+
+/* value -> E2M1 code, nearest, ties to even mantissa, saturating at 6 (reading N1).
+ * Exhaustive over the eight magnitudes: the nearest one wins; on a tie the one whose code is
+ * even (mantissa bit 0). */
+static int e2m1_code_rn(double x) {
+  double a = fabs(x);
+  int best = 0;
+  double bestd = INFINITY;
+  if (a >= 6.0) {
+    best = 7;
+  } else {
+    for (int c = 0; c < 8; ++c) {
+      double d = fabs(a - e2m1_value(c));
+      if (d < bestd || (d == bestd && (c & 1) == 0)) {
+        best = c;
+        bestd = d;
+      }
+    }
+  }
+  if (best == 0) return 0; /* +0 for any sign */
+  return (x < 0.0) ? (best | 8) : best;
+}
+
+/* Offline packing of the NVFP4 variant: W_perp as in qo_pack, then reading N4.
+ * Outputs: qw [N,K] E2M1 codes (one per byte), sfw [N,K/16] E4M3 bits, *sg, Bh [r,N]. */
+int qo_pack_nvfp4(const uint16_t* W_bf16, const float* U, int K, int N, int r, uint8_t* qw, uint8_t* sfw,
+                  float* sg_out, uint16_t* Bh) {
+  if (K <= 0 || N <= 0 || r < 0 || r > K || K % QO_FP4_BLOCK) return QO_EINVAL;
+  int status = QO_OK;
+  double* Bf = (double*)calloc((size_t)(r > 0 ? r : 1) * N, sizeof(double));
+  double* Wp = (double*)malloc((size_t)K * N * sizeof(double));
+  if (!Bf || !Wp) {
+    free(Bf);
+    free(Wp);
+    return QO_EINVAL;
+  }
+#pragma omp parallel for schedule(static)
+  for (int n = 0; n < N; ++n)
+    for (int j = 0; j < r; ++j) {
+      double acc = 0.0;
+      for (int k = 0; k < K; ++k) acc += (double)U[(size_t)k * r + j] * bf16_value(W_bf16[(size_t)k * N + n]);
+      Bf[(size_t)j * N + n] = acc;
+    }
+#pragma omp parallel for schedule(static)
+  for (int k = 0; k < K; ++k)
+    for (int n = 0; n < N; ++n) {
+      double acc = 0.0;
+      for (int j = 0; j < r; ++j) acc += (double)U[(size_t)k * r + j] * Bf[(size_t)j * N + n];
+      Wp[(size_t)k * N + n] = bf16_value(W_bf16[(size_t)k * N + n]) - acc;
+    }
+  double amax = 0.0;
+  for (size_t i = 0; i < (size_t)K * N; ++i)
+    if (fabs(Wp[i]) > amax) amax = fabs(Wp[i]);
+  const float sg = (float)(amax / (6.0 * 448.0));
+  *sg_out = sg;
+  const int nb = K / QO_FP4_BLOCK;
+#pragma omp parallel for schedule(static)
+  for (int n = 0; n < N; ++n)
+    for (int b = 0; b < nb; ++b) {
+      double ab = 0.0;
+      for (int k = b * QO_FP4_BLOCK; k < (b + 1) * QO_FP4_BLOCK; ++k)
+        if (fabs(Wp[(size_t)k * N + n]) > ab) ab = fabs(Wp[(size_t)k * N + n]);
+      uint8_t sb = (sg > 0.0f) ? e4m3_bits_rn(ab / (6.0 * (double)sg)) : 0;
+      sfw[(size_t)n * nb + b] = sb;
+      double scale = e4m3_value(sb) * (double)sg; /* exact: 4 x 24 significant bits */
+      for (int k = b * QO_FP4_BLOCK; k < (b + 1) * QO_FP4_BLOCK; ++k)
+        qw[(size_t)n * K + k] = (uint8_t)((scale > 0.0) ? e2m1_code_rn(Wp[(size_t)k * N + n] / scale) : 0);
+    }
+  for (size_t i = 0; i < (size_t)r * N; ++i) {
+    Bh[i] = f16_bits_rn(Bf[i]);
+    if ((Bh[i] & 0x7c00) == 0x7c00) status = QO_ERANGE;
+  }
+  free(Bf);
+  free(Wp);
+  return status;
+}
+
+/* Reading N3 on one float32 remainder row segment of 16 entries. */
+static void quantize_block_nvfp4(const float* x, uint8_t* q, uint8_t* sf) {
+  float amax = 0.0f;
+  for (int k = 0; k < QO_FP4_BLOCK; ++k)
+    if (fabsf(x[k]) > amax) amax = fabsf(x[k]);
+  const float t = (float)((double)amax / 6.0); /* RN_f32(amax / 6): innocuous double rounding */
+  const uint8_t sb = e4m3_bits_rn((double)t);
+  *sf = sb;
+  const double s = e4m3_value(sb);
+  for (int k = 0; k < QO_FP4_BLOCK; ++k) {
+    if (s > 0.0) {
+      const float u = (float)((double)x[k] / s); /* RN_f32(x / s) */
+      q[k] = (uint8_t)e2m1_code_rn((double)u);
+    } else {
+      q[k] = 0;
+    }
+  }
+}
+
+/* Run-time activation path of the NVFP4 variant: Eq. (xsplit) as in qo_quantize_act, with the
+ * remainder rounded to float32 (the precision in which the GPU forms it), then reading N3.
+ * Outputs: qx [M,K] E2M1 codes, sfx [M,K/16] E4M3 bits, ph [M,r] float16 bits. */
+int qo_quantize_act_nvfp4(const uint16_t* X_bf16, const float* U, int M, int K, int r, uint8_t* qx,
+                          uint8_t* sfx, uint16_t* ph) {
+  if (M < 0 || K <= 0 || r < 0 || r > K || K % QO_FP4_BLOCK) return QO_EINVAL;
+  int status = QO_OK;
+  const int nb = K / QO_FP4_BLOCK;
+#pragma omp parallel reduction(min : status)
+  {
+    double* x = (double*)malloc((size_t)K * sizeof(double));
+    float* xf = (float*)malloc((size_t)K * sizeof(float));
+    double* p = (double*)malloc((size_t)(r > 0 ? r : 1) * sizeof(double));
+#pragma omp for schedule(static)
+    for (int m = 0; m < M; ++m) {
+      for (int k = 0; k < K; ++k) x[k] = bf16_value(X_bf16[(size_t)m * K + k]);
+      for (int j = 0; j < r; ++j) {
+        double acc = 0.0;
+        for (int k = 0; k < K; ++k) acc += x[k] * (double)U[(size_t)k * r + j];
+        p[j] = acc;
+      }
+      for (int k = 0; k < K; ++k) {
+        double acc = 0.0;
+        for (int j = 0; j < r; ++j) acc += p[j] * (double)U[(size_t)k * r + j];
+        xf[k] = (float)(x[k] - acc);
+      }
+      for (int j = 0; j < r; ++j) {
+        ph[(size_t)m * r + j] = f16_bits_rn(p[j]);
+        if ((ph[(size_t)m * r + j] & 0x7c00) == 0x7c00) status = QO_ERANGE;
+      }
+      for (int b = 0; b < nb; ++b)
+        quantize_block_nvfp4(xf + b * QO_FP4_BLOCK, qx + (size_t)m * K + b * QO_FP4_BLOCK, sfx + (size_t)m * nb + b);
+    }
+    free(x);
+    free(xf);
+    free(p);
+  }
+  return status;
+}
+
+/* Reading N3 alone on a given float32 remainder R [M,K] -> qx [M,K], sfx [M,K/16]. */
+int qo_quantize_residual_nvfp4_f32(const float* R, int M, int K, uint8_t* qx, uint8_t* sfx) {
+  if (M < 0 || K <= 0 || K % QO_FP4_BLOCK) return QO_EINVAL;
+  const int nb = K / QO_FP4_BLOCK;
+#pragma omp parallel for schedule(static)
+  for (int m = 0; m < M; ++m)
+    for (int b = 0; b < nb; ++b)
+      quantize_block_nvfp4(R + (size_t)m * K + b * QO_FP4_BLOCK, qx + (size_t)m * K + b * QO_FP4_BLOCK,
+                           sfx + (size_t)m * nb + b);
+  return QO_OK;
+}
+
+/* Reading N5: the layer output of the NVFP4 variant in float64. */
+int qo_linear_nvfp4(const uint8_t* qx, const uint8_t* sfx, const uint16_t* ph, const uint8_t* qw,
+                    const uint8_t* sfw, float sg, const uint16_t* Bh, int M, int K, int N, int r, double* Y) {
+  if (M < 0 || K <= 0 || N <= 0 || r < 0 || K % QO_FP4_BLOCK) return QO_EINVAL;
+  const int nb = K / QO_FP4_BLOCK;
+  double* bhv = (double*)malloc((size_t)(r > 0 ? r : 1) * N * sizeof(double));
+  if (!bhv) return QO_EINVAL;
+  for (size_t i = 0; i < (size_t)r * N; ++i) bhv[i] = f16_value(Bh[i]);
+#pragma omp parallel for schedule(dynamic, 4)
+  for (int m = 0; m < M; ++m)
+    for (int n = 0; n < N; ++n) {
+      double y = 0.0;
+      for (int b = 0; b < nb; ++b) {
+        double P = 0.0; /* sum of 16 products of E2M1 values: exact (quarter-integers below 600) */
+        for (int k = b * QO_FP4_BLOCK; k < (b + 1) * QO_FP4_BLOCK; ++k)
+          P += e2m1_value(qx[(size_t)m * K + k]) * e2m1_value(qw[(size_t)n * K + k]);
+        y += e4m3_value(sfx[(size_t)m * nb + b]) * e4m3_value(sfw[(size_t)n * nb + b]) * P;
+      }
+      double br = 0.0;
+      for (int j = 0; j < r; ++j) br += f16_value(ph[(size_t)m * r + j]) * bhv[(size_t)j * N + n];
+      Y[(size_t)m * N + n] = (double)sg * y + br;
+    }
+  free(bhv);
+  return QO_OK;
+}
+
+/* NVFP4 number formats exposed for the pins. */
+double qo_e2m1_value(int c) { return e2m1_value(c); }
+int qo_e2m1_code_rn(double x) { return e2m1_code_rn(x); }
+double qo_e4m3_value(uint8_t b) { return e4m3_value(b); }
+uint8_t qo_e4m3_bits_rn(double x) { return e4m3_bits_rn(x); }
