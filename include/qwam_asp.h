@@ -141,11 +141,59 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
 qwam_status qwam_asp_linear_static(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
                                    struct CUstream_st* stream);
 
+/* ---- NVFP4 variant (App. B.1) -----------------------------------------------------------
+ * On Blackwell GPUs the paper stores the 4-bit operands as NVFP4: E2M1 values with an E4M3
+ * scale for every 16 consecutive input channels, for weights and activations, and one more
+ * float32 scale per weight tensor.  The paper fixes that storage format only; this library
+ * reads the rest as follows (each exactly as the CPU reference computes it):
+ *   - E2M1 values 0, 0.5, 1, 1.5, 2, 3, 4, 6 (and negatives); E4M3 the OCP FP8 "FN" format
+ *     (largest finite 448).  Rounding to either is to nearest, ties to even, saturating; a code
+ *     of magnitude zero is stored as 0.
+ *   - Activations, per token and block b of 16: s = RN_e4m3(RN_f32(amax_b / 6)),
+ *     code = RN_e2m1(RN_f32(x_perp / s)) (float32 IEEE division); s == 0 gives zero codes.
+ *   - Weights: s_g = RN_f32(amax(W_perp) / (6 * 448)); per output channel and block,
+ *     s_b = RN_e4m3(amax_b / (6 s_g)) and code = RN_e2m1(w / (s_b s_g)), both from the float64
+ *     quotient.
+ *   - Y = s_g sum_b s_a s_b sum_{k in b} qa qb  +  p_hat B_hat.  The block scales are applied by
+ *     the tensor cores (tcgen05.mma kind::mxf4nvf4 block_scale, float32 accumulation); the
+ *     epilogue multiplies by s_g and adds the branch.
+ * The projection, the remainder, p_hat and the branch are those of the INT4 layer above.
+ *
+ * A handle made by qwam_asp_pack_weights_nvfp4 is used with the same calls as an INT4 handle
+ * (qwam_asp_act_workspace_bytes, qwam_asp_act_layout, qwam_asp_quantize_act, qwam_asp_gemm,
+ * qwam_asp_linear, qwam_asp_linear_static, qwam_asp_debug_residual), which dispatch on its
+ * format.  Its activation workspace for M tokens holds:
+ *   codes  : uint8 [M, K/2], two E2M1 codes per byte, low nibble = even k
+ *   scales : uint8 E4M3 block scales, M_pad * K/16 bytes, in 512-byte atoms: atom
+ *            (m / 128, k / 64) starts at ((m / 128) * (K / 64) + k / 64) * 512, and within it the
+ *            four scales of token m (k / 16 in order) start at byte (m % 32) * 16 +
+ *            ((m % 128) / 32) * 4.  This is the order in which tcgen05.cp.32x128b.warpx4 places
+ *            them in tensor memory where the block-scaled MMA reads them.
+ *   ab     : empty (qwam_asp_act_layout reports ab_off == phat_off)
+ *   p_hat  : float16 [M, r_pad], as for INT4.                                              */
+enum { QWAM_FMT_INT4 = 0, QWAM_FMT_NVFP4 = 1 };
+
+/* Offline packing of the NVFP4 variant.  Arguments as for qwam_asp_pack_weights, without the
+ * group (the block is 16); K % 256 == 0.  Synchronizes `stream` before returning. */
+qwam_status qwam_asp_pack_weights_nvfp4(const void* W_bf16, const float* U, int K, int N, int r,
+                                        struct CUstream_st* stream, qwam_asp_handle* out);
+
+/* The handle's format: QWAM_FMT_INT4 or QWAM_FMT_NVFP4. */
+qwam_status qwam_asp_format(qwam_asp_handle h, int* format);
+
+/* Copy the packed NVFP4 weights to HOST buffers (any may be NULL), synchronously:
+ *   qw  : uint8 [N, K/2] E2M1 codes of W_perp, low nibble = even k
+ *   sfw : uint8 [N, K/16] E4M3 block scales, row-major
+ *   sg  : the float32 per-tensor scale
+ *   Bh  : uint16 (float16 bits) [N, r_pad]
+ * Returns QWAM_ERR_INVALID_ARG for an INT4 handle (and qwam_asp_export does for an NVFP4 one). */
+qwam_status qwam_asp_export_nvfp4(qwam_asp_handle h, void* qw, void* sfw, float* sg, void* Bh);
+
 /* Sticky device-side error of the handle (QWAM_OK, QWAM_ERR_TIMEOUT or QWAM_ERR_RANGE);
  * synchronizes the device.  The word is cleared by this call. */
 qwam_status qwam_asp_get_error(qwam_asp_handle h);
 
-/* Shape of a handle (any output pointer may be NULL). */
+/* Shape of a handle (any output pointer may be NULL); `group` is 16 for an NVFP4 handle. */
 qwam_status qwam_asp_shape(qwam_asp_handle h, int* K, int* N, int* r, int* group, int* r_pad);
 
 /* Copy the packed weights to HOST buffers (any may be NULL), synchronously:

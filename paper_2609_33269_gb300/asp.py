@@ -29,13 +29,15 @@ QWAM_ERR_TOO_LARGE = -7
 STATIC_WS_BYTES = 24 * 1024 * 1024  # QWAM_STATIC_WS_BYTES of the header
 QWAM_Y_BF16 = 0
 QWAM_Y_FP32 = 1
+QWAM_FMT_INT4 = 0
+QWAM_FMT_NVFP4 = 1
 
 EXPORTED = [
     "qwam_asp_pack_weights", "qwam_asp_act_workspace_bytes", "qwam_asp_act_layout",
     "qwam_asp_quantize_act", "qwam_asp_gemm", "qwam_asp_linear", "qwam_asp_get_error",
     "qwam_asp_shape", "qwam_asp_export", "qwam_asp_destroy", "qwam_status_string",
     "qwam_asp_debug_residual", "qwam_asp_set_timeout", "qwam_asp_debug_wait_timeout",
-    "qwam_asp_linear_static",
+    "qwam_asp_linear_static", "qwam_asp_pack_weights_nvfp4", "qwam_asp_format", "qwam_asp_export_nvfp4",
 ]
 
 _lib = None
@@ -76,6 +78,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_debug_residual.argtypes = [V, I, H, V, V, V]
         lib.qwam_asp_set_timeout.argtypes = [H, ctypes.c_double]
         lib.qwam_asp_debug_wait_timeout.argtypes = [H, I, V]
+        lib.qwam_asp_pack_weights_nvfp4.argtypes = [V, V, I, I, I, V, ctypes.POINTER(H)]
+        lib.qwam_asp_format.argtypes = [H, ctypes.POINTER(I)]
+        lib.qwam_asp_export_nvfp4.argtypes = [H, V, V, ctypes.POINTER(ctypes.c_float), V]
         for name in EXPORTED:
             if name != "qwam_status_string":
                 getattr(lib, name).restype = I
@@ -112,6 +117,19 @@ def qwam_asp_pack_weights(W_bf16, U, K: int, N: int, r: int, group: int, stream=
     _check(load().qwam_asp_pack_weights(_ptr(W_bf16), _ptr(U), K, N, r, group, _stream(stream),
                                         ctypes.byref(h)), "qwam_asp_pack_weights")
     return h.value
+
+
+def qwam_asp_pack_weights_nvfp4(W_bf16, U, K: int, N: int, r: int, stream=None) -> int:
+    h = ctypes.c_void_p()
+    _check(load().qwam_asp_pack_weights_nvfp4(_ptr(W_bf16), _ptr(U), K, N, r, _stream(stream), ctypes.byref(h)),
+           "qwam_asp_pack_weights_nvfp4")
+    return h.value
+
+
+def qwam_asp_format(h: int) -> int:
+    f = ctypes.c_int()
+    _check(load().qwam_asp_format(h, ctypes.byref(f)), "qwam_asp_format")
+    return f.value
 
 
 def qwam_asp_act_workspace_bytes(h: int, M: int) -> int:
@@ -173,6 +191,21 @@ def qwam_asp_export(h: int):
     return dict(qw=qw, sw=sw, Bh=Bh, Uhl=Uhl)
 
 
+def qwam_asp_export_nvfp4(h: int):
+    """Packed NVFP4 weights on the host: qw uint8 [N, K/2] (low nibble = even k), sfw uint8
+    E4M3 bits [N, K/16], sg float32, Bh float16-bits [N, r_pad] (numpy)."""
+    import numpy as np
+    sh = qwam_asp_shape(h)
+    K, N, rp = sh["K"], sh["N"], sh["r_pad"]
+    qw = np.empty((N, K // 2), np.uint8)
+    sfw = np.empty((N, K // 16), np.uint8)
+    sg = ctypes.c_float()
+    Bh = np.empty((N, rp), np.uint16)
+    _check(load().qwam_asp_export_nvfp4(h, qw.ctypes.data, sfw.ctypes.data, ctypes.byref(sg),
+                                        Bh.ctypes.data if rp else None), "qwam_asp_export_nvfp4")
+    return dict(qw=qw, sfw=sfw, sg=np.float32(sg.value), Bh=Bh)
+
+
 def qwam_asp_destroy(h: int):
     _check(load().qwam_asp_destroy(h), "qwam_asp_destroy")
 
@@ -195,14 +228,22 @@ def qwam_asp_debug_wait_timeout(h: int, timeout_us: int, stream=None):
 class AspLinear:
     """One packed ASP layer plus a reusable activation workspace on the current device."""
 
-    def __init__(self, W_bf16: torch.Tensor, U: torch.Tensor | None, group: int = 64, stream=None):
+    def __init__(self, W_bf16: torch.Tensor, U: torch.Tensor | None, group: int = 64, stream=None,
+                 fmt: int = QWAM_FMT_INT4):
+        """fmt QWAM_FMT_INT4 (group 32 or 64) or QWAM_FMT_NVFP4 (App. B.1's Blackwell format;
+        `group` is then ignored: the block is 16)."""
         assert W_bf16.is_cuda and W_bf16.dtype == torch.bfloat16 and W_bf16.is_contiguous()
         K, N = W_bf16.shape
         r = 0 if U is None else U.shape[1]
         if U is not None:
             assert U.is_cuda and U.dtype == torch.float32 and U.is_contiguous() and U.shape[0] == K
-        self.K, self.N, self.r, self.group = K, N, r, group
-        self.h = qwam_asp_pack_weights(W_bf16, U if r > 0 else None, K, N, r, group, stream)
+        self.fmt = fmt
+        self.K, self.N, self.r = K, N, r
+        self.group = 16 if fmt == QWAM_FMT_NVFP4 else group
+        if fmt == QWAM_FMT_NVFP4:
+            self.h = qwam_asp_pack_weights_nvfp4(W_bf16, U if r > 0 else None, K, N, r, stream)
+        else:
+            self.h = qwam_asp_pack_weights(W_bf16, U if r > 0 else None, K, N, r, group, stream)
         self.r_pad = qwam_asp_shape(self.h)["r_pad"]
         self._ws = None
         self._ws_M = -1
@@ -220,12 +261,24 @@ class AspLinear:
         alpha = 2^18 s_x and beta = -8 s_x S_a, p_hat f16 [M, r_pad]."""
         ws = self.workspace(M) if ws is None else ws
         L = qwam_asp_act_layout(self.h, M)
+        if self.fmt == QWAM_FMT_NVFP4:
+            return self.act_views_nvfp4(M, ws)
         codes = ws[L["codes_off"]:L["codes_off"] + M * self.K].view(M, self.K)
         ns = self.K // self.group
         scales = ws[L["scales_off"]:L["scales_off"] + ns * L["M_pad"] * 4].view(torch.float32).view(ns, L["M_pad"])
         ab = ws[L["ab_off"]:L["ab_off"] + ns * L["M_pad"] * 8].view(torch.float32).view(ns, L["M_pad"], 2)
         ph = ws[L["phat_off"]:L["phat_off"] + M * self.r_pad * 2].view(torch.float16).view(M, self.r_pad)
         return codes, scales, ab, ph
+
+    def act_views_nvfp4(self, M: int, ws: torch.Tensor | None = None):
+        """NVFP4 workspace views: packed codes uint8 [M, K/2] (low nibble = even k), the scale
+        atoms uint8 [M_pad * K/16] (see the header for their order), p_hat f16 [M, r_pad]."""
+        ws = self.workspace(M) if ws is None else ws
+        L = qwam_asp_act_layout(self.h, M)
+        codes = ws[L["codes_off"]:L["codes_off"] + M * (self.K // 2)].view(M, self.K // 2)
+        atoms = ws[L["scales_off"]:L["scales_off"] + L["M_pad"] * (self.K // 16)]
+        ph = ws[L["phat_off"]:L["phat_off"] + M * self.r_pad * 2].view(torch.float16).view(M, self.r_pad)
+        return codes, atoms, ph
 
     def quantize(self, X: torch.Tensor, stream=None) -> torch.Tensor:
         M = X.shape[0]

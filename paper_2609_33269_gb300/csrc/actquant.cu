@@ -21,6 +21,8 @@
 //   s_x[g, m]     float32 scale;   ab[g, m]  (2^18 s_x, -8 s_x S_a), S_a the group's code sum:
 //                 the GEMM epilogue's per-row constants, each rounded once;
 //   p_hat[m, :]   float16.
+// NVFP4 variant (App. B.1, the same kernel with one template flag): per block of 16 K an E4M3
+// scale (in the 512-byte atoms the GEMM copies to tensor memory) and E2M1 codes, two per byte.
 //
 // Warp roles (320 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2..9
 // epilogue: warps 2..5 and 6..9 each cover the four 32-row TMEM quadrants and take the even
@@ -35,7 +37,8 @@ namespace {
 
 struct ActArgs {
   int M, K, G, C, Kc, M_pad;
-  uint8_t* codes;   // [M, K]
+  uint8_t* codes;   // [M, K] (NVFP4: [M, K/2], two codes per byte, low nibble = even k)
+  uint8_t* sf;      // NVFP4: E4M3 block scales in 512-byte atoms
   float* scales;    // [K/G, M_pad]
   float2* ab;       // [K/G, M_pad]: (alpha, beta)
   __half* phat;     // [M, RP]
@@ -130,7 +133,51 @@ __device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4
   *ab_out = make_float2(sc * 262144.0f, (-8.0f * sc) * static_cast<float>(sum));
 }
 
-template <int RP>
+// ---- NVFP4 variant (App. B.1): one block of 16 remainder values -> E4M3 scale and E2M1 codes.
+//   s = RN_e4m3(RN_f32(amax / 6)) (saturating at 448),  code = RN_e2m1(RN_f32(x / s)) (saturating
+//   at 6; s == 0 gives zero codes; a result of magnitude zero is stored as code 0).
+// The conversions are the hardware's round-to-nearest-even cvt forms; each is given the same
+// value twice so that the result does not depend on which half of the pair a value lands in.
+__device__ __forceinline__ uint32_t cvt_e4m3(float t) {
+  uint16_t v;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %1;" : "=h"(v) : "f"(t));
+  return v & 0xFFu;
+}
+__device__ __forceinline__ float e4m3_value(uint32_t b) {
+  const uint16_t pair = static_cast<uint16_t>(b | (b << 8));
+  uint32_t h2;
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"(pair));
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(h2 & 0xFFFFu)));
+}
+__device__ __forceinline__ uint32_t cvt_e2m1(float u) {
+  uint32_t v;
+  asm("{.reg .b8 t;\ncvt.rn.satfinite.e2m1x2.f32 t, %1, %1;\ncvt.u32.u8 %0, t;}" : "=r"(v) : "f"(u));
+  return v & 0xFu;
+}
+// 16 values -> two words of codes (k order, four bits each, low nibble first) and the scale byte.
+__device__ __forceinline__ uint32_t quantize_block_nvfp4(const float* x, uint32_t* w2) {
+  float mx[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) mx[j] = fmaxf(fmaxf(fabsf(x[j]), fabsf(x[j + 4])), fmaxf(fabsf(x[j + 8]), fabsf(x[j + 12])));
+  const float amax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+  const uint32_t sb = cvt_e4m3(__fdiv_rn(amax, 6.0f));
+  const float sc = e4m3_value(sb);
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint32_t w = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float u = sc > 0.0f ? __fdiv_rn(x[8 * h + i], sc) : 0.0f;
+      w |= cvt_e2m1(u) << (4 * i);
+    }
+    // a code whose magnitude bits are zero loses its sign bit
+    const uint32_t nz = ((w & 0x77777777u) + 0x77777777u) & 0x88888888u;
+    w2[h] = w & (0x77777777u | nz);
+  }
+  return sb;
+}
+
+template <int RP, bool NV>
 __global__ void __launch_bounds__(320, 1)
     actquant_kernel(const __grid_constant__ CUtensorMap x_map, const __grid_constant__ CUtensorMap ut_map,
                     const __grid_constant__ CUtensorMap u3_map, const ActArgs a) {
@@ -439,6 +486,19 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
         for (int i = 0; i < kChunk / 4; ++i) d[i] = make_float4(xp[4 * i], xp[4 * i + 1], xp[4 * i + 2], xp[4 * i + 3]);
       }
+      if constexpr (NV) {
+        uint32_t w[8];
+        uint32_t sf4 = 0;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) sf4 |= quantize_block_nvfp4(xp + 16 * b, w + 2 * b) << (8 * b);
+        uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * (a.K / 2) + kc / 2);
+        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+        dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+        const int mr = m % kBM;
+        *reinterpret_cast<uint32_t*>(a.sf + (static_cast<size_t>(m / kBM) * (a.K / 64) + kc / 64) * kSfAtom +
+                                     (mr % 32) * 16 + (mr / 32) * 4) = sf4;
+        continue;
+      }
       uint32_t bytes4[16];
       if (a.G == 64) {
         const size_t gi = static_cast<size_t>(kc / 64) * a.M_pad + m;
@@ -470,7 +530,7 @@ int choose_split(int K, int tiles, int sms) {
   return C;
 }
 
-template <int RP>
+template <int RP, bool NV>
 cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
   using Cfg = ActCfg<RP>;
   const ActLayout L = act_layout(h, M);
@@ -485,6 +545,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   a.M_pad = L.M_pad;
   uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
   a.codes = base + L.codes_off;
+  a.sf = base + L.scales_off;
   a.scales = reinterpret_cast<float*>(base + L.scales_off);
   a.ab = reinterpret_cast<float2*>(base + L.ab_off);
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
@@ -494,7 +555,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
 
   static bool attr_done = false;
   if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(actquant_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(actquant_kernel<RP, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
@@ -512,20 +573,25 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   cfg.numAttrs = 1;
   const CUtensorMap& ut = (RP > 0) ? h.ucat_t_map : am.x_map;
   const CUtensorMap& u3 = (RP > 0) ? h.ucat3_map : am.x_map;
-  return cudaLaunchKernelEx(&cfg, actquant_kernel<RP>, am.x_map, ut, u3, a);
+  return cudaLaunchKernelEx(&cfg, actquant_kernel<RP, NV>, am.x_map, ut, u3, a);
+}
+
+template <bool NV>
+cudaError_t launch_fmt(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
+  switch (h.r_pad) {
+    case 0: return launch_rp<0, NV>(h, am, ws, M, dump, s);
+    case 16: return launch_rp<16, NV>(h, am, ws, M, dump, s);
+    case 32: return launch_rp<32, NV>(h, am, ws, M, dump, s);
+    case 48: return launch_rp<48, NV>(h, am, ws, M, dump, s);
+    case 64: return launch_rp<64, NV>(h, am, ws, M, dump, s);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace
 
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
-  switch (h.r_pad) {
-    case 0: return launch_rp<0>(h, am, ws, M, dump, s);
-    case 16: return launch_rp<16>(h, am, ws, M, dump, s);
-    case 32: return launch_rp<32>(h, am, ws, M, dump, s);
-    case 48: return launch_rp<48>(h, am, ws, M, dump, s);
-    case 64: return launch_rp<64>(h, am, ws, M, dump, s);
-    default: return cudaErrorInvalidValue;
-  }
+  return h.fmt == kFmtNvfp4 ? launch_fmt<true>(h, am, ws, M, dump, s) : launch_fmt<false>(h, am, ws, M, dump, s);
 }
 
 }  // namespace qwam

@@ -80,6 +80,13 @@ ActLayout act_layout(const Handle& h, int M) {
   ActLayout L;
   L.M_pad = round_up(M > 0 ? M : 1, kBM);
   L.codes_off = 0;
+  if (h.fmt == kFmtNvfp4) {  // packed codes [M, K/2], scale atoms (M_pad rows), no epilogue constants
+    L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
+    L.ab_off = L.scales_off + up256(static_cast<size_t>(L.M_pad) * (h.K / kFp4Block));
+    L.phat_off = L.ab_off;
+    L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
+    return L;
+  }
   L.scales_off = up256(static_cast<size_t>(M) * h.K);
   L.ab_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
   L.phat_off = L.ab_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 8);
@@ -102,10 +109,15 @@ const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
     ok &= encode_2d(&c.x_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, x, h.K, M, static_cast<uint64_t>(h.K) * 2, kChunk, kBM,
                     CU_TENSOR_MAP_SWIZZLE_128B);
   }
-  ok &= encode_2d(&c.qx_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K, M, h.K, kGemmKS, kBM,
-                  CU_TENSOR_MAP_SWIZZLE_128B);
-  ok &= encode_2d(&c.ab_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.ab_off, 2 * static_cast<uint64_t>(M), h.K / h.G,
-                  static_cast<uint64_t>(L.M_pad) * 8, 2 * kBM, kScaleGroups, CU_TENSOR_MAP_SWIZZLE_NONE);
+  if (h.fmt == kFmtNvfp4) {
+    ok &= encode_2d(&c.qx4_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, kFp4KS / 2,
+                    kBM, CU_TENSOR_MAP_SWIZZLE_128B);
+  } else {
+    ok &= encode_2d(&c.qx_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K, M, h.K, kGemmKS, kBM,
+                    CU_TENSOR_MAP_SWIZZLE_128B);
+    ok &= encode_2d(&c.ab_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.ab_off, 2 * static_cast<uint64_t>(M),
+                    h.K / h.G, static_cast<uint64_t>(L.M_pad) * 8, 2 * kBM, kScaleGroups, CU_TENSOR_MAP_SWIZZLE_NONE);
+  }
   if (h.r_pad > 0)
     ok &= encode_2d(&c.ph_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
                     static_cast<uint64_t>(h.r_pad) * 2, 8, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
@@ -143,13 +155,14 @@ const char* qwam_status_string(qwam_status s) {
   return "unknown status";
 }
 
-qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int N, int r, int group,
-                                  struct CUstream_st* stream, qwam_asp_handle* out) {
+static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K, int N, int r, int group,
+                             struct CUstream_st* stream, qwam_asp_handle* out) {
   if (!out) return QWAM_ERR_INVALID_ARG;
   *out = nullptr;
   if (!W_bf16 || !qwam::aligned16(W_bf16)) return QWAM_ERR_INVALID_ARG;
   if (K <= 0 || K % 64 != 0 || N <= 0 || N % 8 != 0) return QWAM_ERR_INVALID_ARG;
-  if (group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
+  if (fmt == qwam::kFmtNvfp4 && K % qwam::kFp4KS != 0) return QWAM_ERR_INVALID_ARG;
+  if (fmt == qwam::kFmtInt4 && group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
   if (r < 0 || r > K) return QWAM_ERR_INVALID_ARG;
   if (r > 0 && (!U || !qwam::aligned16(U))) return QWAM_ERR_INVALID_ARG;
   if (r > qwam::kMaxRank) return QWAM_ERR_UNSUPPORTED;
@@ -158,6 +171,7 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   auto* hs = new (std::nothrow) qwam_asp_handle_s();
   if (!hs) return QWAM_ERR_OOM;
   Handle& h = hs->h;
+  h.fmt = fmt;
   h.K = K;
   h.N = N;
   h.r = r;
@@ -168,9 +182,12 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   cudaGetDevice(&h.device);
   cudaDeviceGetAttribute(&h.num_sms, cudaDevAttrMultiProcessorCount, h.device);
 
+  const bool nv = fmt == qwam::kFmtNvfp4;
   const size_t b_qw = qwam::up256(static_cast<size_t>(h.N_pad) * (K / 2));
-  const size_t b_sw = qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
-  const size_t b_s32 = qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 4);
+  // INT4: float16 scales and their float32 copy; NVFP4: E4M3 scale atoms (N_pad rows)
+  const size_t b_sw = nv ? qwam::up256(static_cast<size_t>(h.N_pad) * (K / qwam::kFp4Block))
+                         : qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
+  const size_t b_s32 = nv ? 0 : qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 4);
   const size_t b_bh = qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2);
   const size_t b_ut = qwam::up256(static_cast<size_t>(2 * h.r_pad) * K * 2);
   const size_t b_u3 = qwam::up256(static_cast<size_t>(K) * h.ku3 * 2);
@@ -182,8 +199,12 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   }
   uint8_t* p = static_cast<uint8_t*>(h.block);
   h.qw = p;
-  h.sw = reinterpret_cast<__half*>(p + b_qw);
-  h.sw32 = reinterpret_cast<float*>(p + b_qw + b_sw);
+  if (nv) {
+    h.sfw = p + b_qw;
+  } else {
+    h.sw = reinterpret_cast<__half*>(p + b_qw);
+    h.sw32 = reinterpret_cast<float*>(p + b_qw + b_sw);
+  }
   uint8_t* q = p + b_qw + b_sw + b_s32;
   h.Bh = reinterpret_cast<__half*>(q);
   h.ucat_t = reinterpret_cast<__nv_bfloat16*>(q + b_bh);
@@ -192,11 +213,16 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   bool ok = true;
-  ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kGemmKS / 2, qwam::kBM,
-                        CU_TENSOR_MAP_SWIZZLE_NONE);
-  ok &= qwam::encode_2d(&h.sw32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, h.sw32, N, K / group,
-                        static_cast<uint64_t>(h.N_pad) * 4, qwam::kGemmBN, qwam::kScaleGroups,
-                        CU_TENSOR_MAP_SWIZZLE_NONE);
+  if (nv) {
+    ok &= qwam::encode_2d(&h.qw4_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kFp4KS / 2,
+                          qwam::kGemmBN, CU_TENSOR_MAP_SWIZZLE_128B);
+  } else {
+    ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kGemmKS / 2,
+                          qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= qwam::encode_2d(&h.sw32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, h.sw32, N, K / group,
+                          static_cast<uint64_t>(h.N_pad) * 4, qwam::kGemmBN, qwam::kScaleGroups,
+                          CU_TENSOR_MAP_SWIZZLE_NONE);
+  }
   if (h.r_pad > 0) {
     ok &= qwam::encode_2d(&h.Bh_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,
                           static_cast<uint64_t>(h.r_pad) * 2, 8, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
@@ -212,7 +238,8 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
   }
   cudaError_t e = cudaMemsetAsync(h.block, 0, total, s);
   if (e == cudaSuccess)
-    e = qwam::launch_pack(h, static_cast<const __nv_bfloat16*>(W_bf16), r > 0 ? U : nullptr, s);
+    e = nv ? qwam::launch_pack_nvfp4(h, static_cast<const __nv_bfloat16*>(W_bf16), r > 0 ? U : nullptr, s)
+           : qwam::launch_pack(h, static_cast<const __nv_bfloat16*>(W_bf16), r > 0 ? U : nullptr, s);
   int herr = 0;
   if (e == cudaSuccess) e = cudaMemcpy(&herr, h.err, sizeof(int), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess || herr != 0) {
@@ -221,6 +248,22 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
     return e != cudaSuccess ? QWAM_ERR_CUDA : QWAM_ERR_RANGE;
   }
   *out = hs;
+  return QWAM_OK;
+}
+
+qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int N, int r, int group,
+                                  struct CUstream_st* stream, qwam_asp_handle* out) {
+  return pack_impl(qwam::kFmtInt4, W_bf16, U, K, N, r, group, stream, out);
+}
+
+qwam_status qwam_asp_pack_weights_nvfp4(const void* W_bf16, const float* U, int K, int N, int r,
+                                        struct CUstream_st* stream, qwam_asp_handle* out) {
+  return pack_impl(qwam::kFmtNvfp4, W_bf16, U, K, N, r, qwam::kFp4Block, stream, out);
+}
+
+qwam_status qwam_asp_format(qwam_asp_handle hs, int* format) {
+  if (!hs || !format) return QWAM_ERR_INVALID_ARG;
+  *format = hs->h.fmt == qwam::kFmtNvfp4 ? QWAM_FMT_NVFP4 : QWAM_FMT_INT4;
   return QWAM_OK;
 }
 
@@ -275,6 +318,9 @@ qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle hs, void* Y
   Handle& h = hs->h;
   const qwam::ActMaps* am = qwam::get_act_maps(h, nullptr, act_ws, M);
   if (!am) return QWAM_ERR_CUDA;
+  if (h.fmt == qwam::kFmtNvfp4)
+    return from_cuda_status(qwam::launch_gemm_nvfp4(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32,
+                                                    reinterpret_cast<cudaStream_t>(stream)));
   return from_cuda_status(qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32,
                                             reinterpret_cast<cudaStream_t>(stream)));
 }
@@ -312,6 +358,7 @@ qwam_status qwam_asp_shape(qwam_asp_handle hs, int* K, int* N, int* r, int* grou
 qwam_status qwam_asp_export(qwam_asp_handle hs, void* qw, void* sw, void* Bh, void* Uhl) {
   if (!hs) return QWAM_ERR_INVALID_ARG;
   Handle& h = hs->h;
+  if (h.fmt != qwam::kFmtInt4) return QWAM_ERR_INVALID_ARG;
   if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
   cudaError_t e = cudaSuccess;
   if (qw) {
@@ -343,6 +390,32 @@ qwam_status qwam_asp_export(qwam_asp_handle hs, void* qw, void* sw, void* Bh, vo
           o[(static_cast<size_t>(part) * h.K + k) * h.r_pad + j] =
               t[static_cast<size_t>(part * h.r_pad + j) * h.K + k];
   }
+  return from_cuda_status(e);
+}
+
+qwam_status qwam_asp_export_nvfp4(qwam_asp_handle hs, void* qw, void* sfw, float* sg, void* Bh) {
+  if (!hs) return QWAM_ERR_INVALID_ARG;
+  Handle& h = hs->h;
+  if (h.fmt != qwam::kFmtNvfp4) return QWAM_ERR_INVALID_ARG;
+  if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
+  cudaError_t e = cudaSuccess;
+  if (qw) e = cudaMemcpy(qw, h.qw, static_cast<size_t>(h.N) * (h.K / 2), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && sfw) {
+    // atoms -> row-major [N, K/16]
+    const int nb = h.K / qwam::kFp4Block;
+    std::vector<uint8_t> t(static_cast<size_t>(h.N_pad) * nb);
+    e = cudaMemcpy(t.data(), h.sfw, t.size(), cudaMemcpyDeviceToHost);
+    uint8_t* o = static_cast<uint8_t*>(sfw);
+    for (int n = 0; e == cudaSuccess && n < h.N; ++n)
+      for (int b = 0; b < nb; ++b) {
+        const int nr = n % 128;
+        o[static_cast<size_t>(n) * nb + b] =
+            t[(static_cast<size_t>(n / 128) * (h.K / 64) + b / 4) * qwam::kSfAtom + (nr % 32) * 16 + (nr / 32) * 4 + b % 4];
+      }
+  }
+  if (e == cudaSuccess && sg) *sg = h.sg;
+  if (e == cudaSuccess && Bh && h.r_pad > 0)
+    e = cudaMemcpy(Bh, h.Bh, static_cast<size_t>(h.N) * h.r_pad * 2, cudaMemcpyDeviceToHost);
   return from_cuda_status(e);
 }
 

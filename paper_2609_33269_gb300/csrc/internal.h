@@ -19,6 +19,15 @@ constexpr int kGemmBN = 128;    // output columns per GEMM CTA tile
 constexpr int kGemmKS = 128;    // K elements per GEMM pipeline stage
 constexpr int kScaleGroups = 8; // groups per GEMM scale stage (epilogue constants and s_w)
 
+// NVFP4 variant (App. B.1): E2M1 codes, one E4M3 scale per 16 consecutive K, one float32 scale per
+// weight tensor.  Block scales are stored in 512-byte atoms, one per 128 rows x 64 K: the four
+// scales of row r (r = row % 128) sit at bytes (r % 32) * 16 + (r / 32) * 4 .. +3, K order, and
+// atom (row / 128, k / 64) starts at ((row / 128) * (K / 64) + k / 64) * 512.
+constexpr int kFp4Block = 16;   // K entries per E4M3 scale
+constexpr int kFp4KS = 256;     // K entries per NVFP4 GEMM stage (128 bytes of codes per row)
+constexpr int kSfAtom = 512;    // bytes per scale atom (128 rows x 64 K)
+enum Format : int { kFmtInt4 = 0, kFmtNvfp4 = 1 };
+
 inline int round_up(int a, int b) { return (a + b - 1) / b * b; }
 
 // Activation-side tensor maps for one (workspace, X, M) triple.
@@ -30,9 +39,11 @@ struct ActMaps {
   CUtensorMap qx_map;   // code bytes [M, K], box {128, 128}, 128-byte swizzle
   CUtensorMap ab_map;   // epilogue constants f32 [K/G, M_pad, 2] (dims {2M, K/G}), box {256, 8}
   CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128}
+  CUtensorMap qx4_map;  // NVFP4 codes [M, K/2] bytes, box {128, 128}, 128-byte swizzle
 };
 
 struct Handle {
+  int fmt = kFmtInt4;
   int K = 0, N = 0, r = 0, G = 0, r_pad = 0, N_pad = 0, ku3 = 0;
   int device = 0;
   int num_sms = 148;
@@ -44,9 +55,12 @@ struct Handle {
   __half* Bh = nullptr;              // [N_pad, r_pad]
   __nv_bfloat16* ucat_t = nullptr;   // [2 r_pad, K]: rows 0..r_pad-1 = U_hi^T, then U_lo^T
   __nv_bfloat16* ucat3 = nullptr;    // [K, ku3]: row k = U_hi[k,:], U_lo[k,:], U_hi[k,:], zeros
+  uint8_t* sfw = nullptr;            // NVFP4: E4M3 block scales of W_perp in atoms (N_pad rows)
+  float sg = 0.0f;                   // NVFP4: float32 per-tensor weight scale
   int* err = nullptr;                // sticky device error word
   double timeout_s = 2.0;
   CUtensorMap qw_map, sw32_map, Bh_map, ucat_t_map, ucat3_map;
+  CUtensorMap qw4_map;               // NVFP4 weight codes [N, K/2], box {128, 128}, 128-byte swizzle
   ActMaps act_cache[4];
   int act_next = 0;
 };
@@ -68,8 +82,10 @@ uint64_t deadline_budget_ns(const Handle& h);
 
 // Launchers (return cudaSuccess or the launch error).
 cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
+cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s);
 cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
+cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
 cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s);
 
 }  // namespace qwam

@@ -1,9 +1,13 @@
 // pack.cu -- offline packing of one ASP layer (Sec. 3.2 Eq. (asp) and the derivation of the
 // deflated weight W_perp = (I - U U^T) W; Eq. (quant) of Sec. 2 applied to W_perp per output
-// channel and group, App. B.1).  float64 on the device, untimed.
+// channel and group, App. B.1; or, for the NVFP4 variant of App. B.1, E2M1 codes with an E4M3
+// scale per 16 K and one float32 scale per tensor).  float64 on the device, untimed.
 //
 // Every float64 operation is an explicit IEEE intrinsic (__dmul_rn, __dadd_rn, ...) so that no
 // multiply-add is contracted: sums run in index order, each product and sum rounded once.
+#include <cuda_fp4.h>
+#include <cuda_fp8.h>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -115,7 +119,103 @@ __global__ void split_basis_kernel(const float* __restrict__ U, int K, int r, in
   for (int j = 3 * r_pad; j < ku3; ++j) ucat3[static_cast<size_t>(k) * ku3 + j] = __float2bfloat16_rn(0.0f);
 }
 
+// ---- NVFP4 variant (App. B.1: E2M1 codes, an E4M3 scale per 16 K, one float32 scale per tensor)
+
+// One thread per (output channel n, block b of 16 K): the block's absmax of |W_perp| (float64),
+// and the tensor's absmax by an atomic max on the bit pattern (non-negative doubles order as
+// unsigned integers).
+__global__ void block_amax_nvfp4_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+                                        const double* __restrict__ Bf, int K, int N, int r, double* __restrict__ bam,
+                                        unsigned long long* __restrict__ amax_bits) {
+  int n = blockIdx.x * blockDim.x + threadIdx.x;
+  int b = blockIdx.y;
+  if (n >= N) return;
+  double a = 0.0;
+  for (int k = b * kFp4Block; k < (b + 1) * kFp4Block; ++k) a = fmax(a, fabs(wperp(W, U, Bf, N, r, k, n)));
+  bam[static_cast<size_t>(n) * (K / kFp4Block) + b] = a;
+  atomicMax(amax_bits, static_cast<unsigned long long>(__double_as_longlong(a)));
+}
+
+// E4M3 bits -> value (exact in float64).
+__device__ __forceinline__ double e4m3_to_double(__nv_fp8_storage_t b) {
+  __half_raw hr = __nv_cvt_fp8_to_halfraw(b, __NV_E4M3);
+  return static_cast<double>(__half2float(__half(hr)));
+}
+
+// One thread per (n, b): s_g = RN_f32(amax / (6 * 448)); s_b = RN_e4m3(amax_b / (6 s_g)) and the
+// codes RN_e2m1(w / (s_b s_g)), each from the float64 quotient (one rounding to a 4-bit format),
+// saturating; a code of magnitude zero is stored as 0.  Codes are packed two per byte, low nibble =
+// even k; the block scale goes to its atom (see internal.h).
+__global__ void quantize_weight_nvfp4_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+                                             const double* __restrict__ Bf, int K, int N, int r,
+                                             const double* __restrict__ bam,
+                                             const unsigned long long* __restrict__ amax_bits,
+                                             uint8_t* __restrict__ qw, uint8_t* __restrict__ sfw,
+                                             float* __restrict__ sg_out) {
+  int n = blockIdx.x * blockDim.x + threadIdx.x;
+  int b = blockIdx.y;
+  if (n >= N) return;
+  const double amax = __longlong_as_double(static_cast<long long>(*amax_bits));
+  const float sg = __double2float_rn(__ddiv_rn(amax, 2688.0));  // 6 * 448
+  if (n == 0 && b == 0) *sg_out = sg;
+  __nv_fp8_storage_t sb = 0;
+  if (sg > 0.0f) {
+    const double q = __ddiv_rn(bam[static_cast<size_t>(n) * (K / kFp4Block) + b], __dmul_rn(6.0, static_cast<double>(sg)));
+    sb = __nv_cvt_double_to_fp8(q, __NV_SATFINITE, __NV_E4M3);
+  }
+  const int nr = n % 128;
+  sfw[(static_cast<size_t>(n / 128) * (K / 64) + b / 4) * kSfAtom + (nr % 32) * 16 + (nr / 32) * 4 + (b % 4)] = sb;
+  const double scale = __dmul_rn(e4m3_to_double(sb), static_cast<double>(sg));  // exact
+  uint32_t lo = 0, hi = 0;
+  for (int i = 0; i < kFp4Block; ++i) {
+    uint32_t c = 0;
+    if (scale > 0.0) {
+      const double u = __ddiv_rn(wperp(W, U, Bf, N, r, b * kFp4Block + i, n), scale);
+      c = static_cast<uint32_t>(__nv_cvt_double_to_fp4(u, __NV_E2M1, cudaRoundNearest)) & 0xFu;
+      if ((c & 7u) == 0u) c = 0u;  // zero has one code
+    }
+    if (i < 8)
+      lo |= c << (4 * i);
+    else
+      hi |= c << (4 * (i - 8));
+  }
+  *reinterpret_cast<uint2*>(qw + static_cast<size_t>(n) * (K / 2) + b * (kFp4Block / 2)) = make_uint2(lo, hi);
+}
+
 }  // namespace
+
+cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s) {
+  const int K = h.K, N = h.N, r = h.r;
+  const int nb = K / kFp4Block;
+  double* Bf = nullptr;
+  double* bam = nullptr;
+  unsigned long long* amax = nullptr;
+  float* sg_dev = nullptr;
+  cudaError_t e = cudaMalloc(&Bf, sizeof(double) * static_cast<size_t>(r > 0 ? r : 1) * N);
+  if (e == cudaSuccess) e = cudaMalloc(&bam, sizeof(double) * static_cast<size_t>(N) * nb);
+  if (e == cudaSuccess) e = cudaMalloc(&amax, 16);
+  if (e == cudaSuccess) e = cudaMemsetAsync(amax, 0, 16, s);
+  if (e == cudaSuccess) {
+    sg_dev = reinterpret_cast<float*>(amax + 1);
+    const int T = 128;
+    if (r > 0) branch_weight_kernel<<<dim3((N + T - 1) / T, r), T, 0, s>>>(W, U, K, N, r, Bf);
+    block_amax_nvfp4_kernel<<<dim3((N + T - 1) / T, nb), T, 0, s>>>(W, U, Bf, K, N, r, bam, amax);
+    quantize_weight_nvfp4_kernel<<<dim3((N + T - 1) / T, nb), T, 0, s>>>(W, U, Bf, K, N, r, bam, amax, h.qw, h.sfw,
+                                                                          sg_dev);
+    if (r > 0) {
+      branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
+      split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(U, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+    }
+    e = cudaGetLastError();
+    cudaError_t e2 = cudaStreamSynchronize(s);
+    if (e == cudaSuccess) e = e2;
+    if (e == cudaSuccess) e = cudaMemcpy(&h.sg, sg_dev, sizeof(float), cudaMemcpyDeviceToHost);
+  }
+  cudaFree(Bf);
+  cudaFree(bam);
+  cudaFree(amax);
+  return e;
+}
 
 cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s) {
   const int K = h.K, N = h.N, r = h.r;

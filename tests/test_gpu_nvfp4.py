@@ -1,0 +1,228 @@
+"""GPU parity of the NVFP4 variant (App. B.1: E2M1 codes, an E4M3 scale per 16 K, one float32
+scale per weight tensor) against the CPU oracle, through the C ABI.
+
+Bars (as for the INT4 layer):
+  * weight codes, block scales, the per-tensor scale and the branch weights: bit-exact;
+  * activation codes and block scales: bit-exact when r = 0 (the remainder is X itself), and,
+    for r > 0, bit-exact given the kernel's own float32 remainder (qwam_asp_debug_residual);
+  * the float32 output within 1e-5 * max |y| per row of the oracle evaluated on the kernel's
+    own codes and scales (float32 accumulation order only), and within 1e-3 * max |y| per row
+    of the end-to-end oracle for rows whose codes equal the oracle's;
+  * the bf16 output equals RN_bf16 of the float32 output bit for bit.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_33269_gb300 import asp
+from paper_2609_33269_gb300 import workloads as wl
+
+from gpu_helpers import rowwise_rel_err, to_dev_bf16
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2609_33269_gb300 import build
+    build.build()
+    asp.load()
+
+
+def unpack_e2m1(packed):
+    """uint8 [R, K/2] -> E2M1 codes uint8 [R, K], low nibble = even k."""
+    p = np.ascontiguousarray(packed)
+    out = np.empty((p.shape[0], p.shape[1] * 2), np.uint8)
+    out[:, 0::2] = p & 0xF
+    out[:, 1::2] = p >> 4
+    return out
+
+
+def atoms_to_rows(atoms, rows, K):
+    """Scale atoms (512 bytes per 128 rows x 64 K; row r's four scales at (r % 32) * 16 +
+    (r % 128 // 32) * 4) -> row-major uint8 [rows, K/16]."""
+    a = np.asarray(atoms, np.uint8)
+    r = np.arange(rows)[:, None]
+    b = np.arange(K // 16)[None, :]
+    idx = ((r // 128) * (K // 64) + b // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + b % 4
+    return a[idx]
+
+
+class NvCase:
+    def __init__(self, M, K, N, r, seed=0, layer_id=0, dist="outlier"):
+        self.M, self.K, self.N, self.r = M, K, N, r
+        self.Xb = wl.activations(M, K, seed=seed, layer_id=layer_id, dist=dist)
+        self.Wb = wl.weight(K, N, seed=seed, layer_id=layer_id)
+        self.U = wl.basis(K, r, seed=seed, layer_id=layer_id)
+        self.X = to_dev_bf16(self.Xb)
+        W = to_dev_bf16(self.Wb)
+        Ud = torch.from_numpy(self.U).cuda() if r > 0 else None
+        self.layer = asp.AspLinear(W, Ud, fmt=asp.QWAM_FMT_NVFP4)
+        self._ow = None
+
+    def oracle_weights(self):
+        if self._ow is None:
+            self._ow = oracle.pack_nvfp4(self.Wb, self.U)
+        return self._ow
+
+    def gpu_weights(self):
+        e = asp.qwam_asp_export_nvfp4(self.layer.h)
+        return dict(qw=unpack_e2m1(e["qw"]), sfw=e["sfw"], sg=e["sg"], Bh=e["Bh"][:, :self.r].T.copy())
+
+    def gpu_act(self):
+        codes, atoms, ph = self.layer.act_views_nvfp4(self.M)
+        torch.cuda.synchronize()
+        return dict(qx=unpack_e2m1(codes.cpu().numpy()),
+                    sfx=atoms_to_rows(atoms.cpu().numpy(), self.M, self.K),
+                    ph=ph.cpu().numpy().view(np.uint16)[:, :self.r].copy())
+
+    def residual(self):
+        R = torch.empty((self.M, self.K), dtype=torch.float32, device="cuda")
+        asp.qwam_asp_debug_residual(self.X, self.M, self.layer.h, self.layer.workspace(self.M), R)
+        torch.cuda.synchronize()
+        return R.cpu().numpy()
+
+    def run(self, fp32=True):
+        Y = self.layer(self.X, fp32=fp32)
+        torch.cuda.synchronize()
+        return Y
+
+    def close(self):
+        self.layer.close()
+
+
+PACK_SHAPES = [(512, 512, 16), (256, 136, 0), (1024, 384, 48), (256, 64, 64), (768, 264, 32)]
+
+
+@pytest.mark.parametrize("shape", PACK_SHAPES, ids=lambda s: "K%d_N%d_r%d" % s)
+def test_nvfp4_pack_bit_exact(shape):
+    K, N, r = shape
+    c = NvCase(8, K, N, r, seed=5, layer_id=K + r)
+    try:
+        assert asp.qwam_asp_format(c.layer.h) == asp.QWAM_FMT_NVFP4
+        gw, ow = c.gpu_weights(), c.oracle_weights()
+        assert gw["sg"].view(np.uint32) == np.float32(ow["sg"]).view(np.uint32)
+        np.testing.assert_array_equal(gw["sfw"], ow["sfw"])
+        np.testing.assert_array_equal(gw["qw"], ow["qw"])
+        if r > 0:
+            np.testing.assert_array_equal(gw["Bh"], ow["Bh"])
+    finally:
+        c.close()
+
+
+@pytest.mark.parametrize("M", [1, 33, 256, 300])
+def test_nvfp4_activation_codes_bit_exact_r0(M):
+    c = NvCase(M, 512, 128, 0, seed=6, layer_id=M)
+    try:
+        c.layer.quantize(c.X)
+        ga = c.gpu_act()
+        oa = oracle.quantize_act_nvfp4(c.Xb, c.U)
+        np.testing.assert_array_equal(ga["sfx"], oa["sfx"])
+        np.testing.assert_array_equal(ga["qx"], oa["qx"])
+    finally:
+        c.close()
+
+
+@pytest.mark.parametrize("shape", [(128, 512, 128, 16), (100, 1024, 128, 64)], ids=lambda s: "M%d_K%d_N%d_r%d" % s)
+def test_nvfp4_quantizer_bit_exact_given_residual(shape):
+    M, K, N, r = shape
+    c = NvCase(M, K, N, r, seed=7, layer_id=r)
+    try:
+        R = c.residual()
+        ga = c.gpu_act()
+        q, sf = oracle.quantize_residual_nvfp4(R)
+        np.testing.assert_array_equal(ga["sfx"], sf)
+        np.testing.assert_array_equal(ga["qx"], q)
+    finally:
+        c.close()
+
+
+LAYER_SHAPES = [  # M, K, N, r
+    (256, 512, 512, 16),    # the tiny workload's shape
+    (33, 512, 200, 32),     # ragged M and N
+    (1, 256, 136, 0),       # one token, r = 0
+    (200, 1024, 384, 48),
+    (130, 768, 264, 64),
+    (300, 2048, 640, 0),    # several tiles per CTA row and column, ragged M
+]
+
+
+@pytest.mark.parametrize("shape", LAYER_SHAPES, ids=lambda s: "M%d_K%d_N%d_r%d" % s)
+def test_nvfp4_layer_parity(shape):
+    M, K, N, r = shape
+    c = NvCase(M, K, N, r, seed=8, layer_id=M + r)
+    try:
+        Y = c.run(fp32=True).cpu().numpy()
+        ga = c.gpu_act()
+        gw = c.gpu_weights()
+        ow = c.oracle_weights()
+        # the oracle's output on the kernel's own codes and scales
+        Yk = oracle.linear_nvfp4(ga, dict(qw=gw["qw"], sfw=gw["sfw"], sg=gw["sg"], Bh=ow["Bh"]))
+        assert rowwise_rel_err(Y, Yk).max() <= 1e-5
+        # end to end: rows whose codes equal the oracle's are within 1e-3 of the oracle
+        oa = oracle.quantize_act_nvfp4(c.Xb, c.U)
+        Yo = oracle.linear_nvfp4(oa, ow)
+        same = np.all(ga["qx"] == oa["qx"], axis=1) & np.all(ga["sfx"] == oa["sfx"], axis=1)
+        if r == 0:
+            assert same.all()
+        assert same.mean() >= 0.9
+        assert rowwise_rel_err(Y[same], Yo[same]).max() <= 1e-3
+        # bf16 output = RN_bf16(float32 output)
+        Yb = c.run(fp32=False).float().cpu().numpy()
+        np.testing.assert_array_equal(Yb, torch.from_numpy(Y).to(torch.bfloat16).float().numpy())
+    finally:
+        c.close()
+
+
+def test_nvfp4_full_size_dit_attention_sampled_rows():
+    """M = 4096, K = N = 3072, r = 32 (the DiT attention projection), in the launch configuration
+    the benchmark times; 48 sampled rows against the oracle."""
+    L = wl.dit_attention().layers[0]
+    X = to_dev_bf16(L.x())
+    layer = asp.AspLinear(to_dev_bf16(L.w()), torch.from_numpy(L.u()).cuda(), fmt=asp.QWAM_FMT_NVFP4)
+    try:
+        Y = layer(X, fp32=True)
+        torch.cuda.synchronize()
+        rows = np.sort(np.random.default_rng(0).choice(L.M, 48, replace=False))
+        rows[0], rows[-1] = 0, L.M - 1
+        Ys = Y[torch.from_numpy(rows).cuda()].cpu().numpy()
+        ow = oracle.pack_nvfp4(L.w(), L.u())
+        gw = asp.qwam_asp_export_nvfp4(layer.h)
+        np.testing.assert_array_equal(unpack_e2m1(gw["qw"]), ow["qw"])
+        oa = oracle.quantize_act_nvfp4(L.x()[rows], L.u())
+        Yo = oracle.linear_nvfp4(oa, ow)
+        codes, atoms, _ = layer.act_views_nvfp4(L.M)
+        qx = unpack_e2m1(codes.cpu().numpy()[rows])
+        sfx = atoms_to_rows(atoms.cpu().numpy(), L.M, L.K)[rows]
+        same = np.all(qx == oa["qx"], axis=1) & np.all(sfx == oa["sfx"], axis=1)
+        assert same.mean() >= 0.9
+        assert rowwise_rel_err(Ys[same], Yo[same]).max() <= 1e-3
+        # rows with a near-tie flip: the oracle on the kernel's own codes
+        if (~same).any():
+            Yk = oracle.linear_nvfp4(dict(qx=qx, sfx=sfx, ph=oa["ph"]), ow)
+            assert rowwise_rel_err(Ys[~same], Yk[~same]).max() <= 1e-3
+        assert asp.qwam_asp_get_error(layer.h) == asp.QWAM_OK
+    finally:
+        layer.close()
+
+
+def test_nvfp4_empty_input_and_bad_k():
+    K, N = 256, 64
+    W = to_dev_bf16(wl.weight(K, N, seed=1, layer_id=0))
+    layer = asp.AspLinear(W, None, fmt=asp.QWAM_FMT_NVFP4)
+    try:
+        X = torch.empty((0, K), dtype=torch.bfloat16, device="cuda")
+        Y = torch.empty((0, N), dtype=torch.float32, device="cuda")
+        ws = torch.zeros(16, dtype=torch.uint8, device="cuda")
+        asp.qwam_asp_linear(X, 0, layer.h, Y, asp.QWAM_Y_FP32, ws)
+        torch.cuda.synchronize()
+        assert asp.qwam_asp_get_error(layer.h) == asp.QWAM_OK
+        with pytest.raises(asp.QwamError):  # an INT4 export of an NVFP4 handle is refused
+            asp.qwam_asp_export(layer.h)
+    finally:
+        layer.close()
+    W2 = to_dev_bf16(wl.weight(320, N, seed=1, layer_id=0))
+    with pytest.raises(asp.QwamError) as ei:  # K must be a multiple of 256
+        asp.qwam_asp_pack_weights_nvfp4(W2, None, 320, N, 0)
+    assert ei.value.status == asp.QWAM_ERR_INVALID_ARG
