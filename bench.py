@@ -13,6 +13,10 @@ on a bounded sample of rows.  `--impl reference` times the CPU oracle alone (the
 
 Multi-GPU (torchrun): every rank runs the same per-GPU batch (token rows are independent, so
 the layer shards by rows with no collective); weak scaling.
+
+The NVFP4 variant (App. B.1: E2M1 with an E4M3 scale per 16 K, block scales applied by the
+tensor cores) is timed on the same workload and reported under `variants`; `--format nvfp4` makes
+it the headline.
 """
 from __future__ import annotations
 
@@ -45,6 +49,9 @@ def parse():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--cpu-rows", type=int, default=0, help="oracle sample rows (0 = sized to ~10 s)")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--format", choices=["int4", "nvfp4"], default="int4",
+                   help="4-bit format of the headline: INT4 group 64 (the configuration's), or NVFP4 "
+                        "(App. B.1's Blackwell format, also measured as a variant of the INT4 run)")
     return p.parse_args()
 
 
@@ -149,19 +156,22 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ CPU oracle (baseline / reference arm)
 
-def oracle_sample(rows: int):
+def oracle_sample(rows: int, nvfp4: bool = False):
     """Inputs and packed weights for the oracle timing: the workload's first `rows` tokens."""
     import oracle
     from paper_2609_33269_gb300 import workloads as wl
     layer = wl.dit_attention().layers[0]
     Xb = layer.x()[:rows].copy()
     U = layer.u()
-    wts = oracle.pack(layer.w(), U, layer.G)  # offline packing: outside the timed sample
+    # offline packing: outside the timed sample
+    wts = oracle.pack_nvfp4(layer.w(), U) if nvfp4 else oracle.pack(layer.w(), U, layer.G)
     return Xb, U, wts, layer
 
 
-def oracle_step(Xb, U, wts, G):
+def oracle_step(Xb, U, wts, G, nvfp4: bool = False):
     import oracle
+    if nvfp4:
+        return oracle.linear_nvfp4(oracle.quantize_act_nvfp4(Xb, U), wts)
     act = oracle.quantize_act(Xb, U, G)
     return oracle.linear(act, wts, G)
 
@@ -178,26 +188,28 @@ def run_reference(args):
     if rank != 0:
         return 0
     K, N = WORKLOAD["K"], WORKLOAD["N"]
+    nv = args.format == "nvfp4"
     rows = args.cpu_rows
     if not rows:  # size each step so that warm-up + timed steps take about two minutes
-        Xb, U, wts, layer = oracle_sample(8)
+        Xb, U, wts, layer = oracle_sample(8, nv)
         t0 = time.perf_counter()
-        oracle_step(Xb, U, wts, layer.G)
+        oracle_step(Xb, U, wts, layer.G, nv)
         per_row = (time.perf_counter() - t0) / 8
         rows = int(max(1, min(256, 120.0 / (max(1, args.steps + args.warmup) * per_row))))
-    Xb, U, wts, layer = oracle_sample(rows)
+    Xb, U, wts, layer = oracle_sample(rows, nv)
     for _ in range(max(0, args.warmup)):
-        oracle_step(Xb, U, wts, layer.G)
+        oracle_step(Xb, U, wts, layer.G, nv)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle_step(Xb, U, wts, layer.G)
+        oracle_step(Xb, U, wts, layer.G, nv)
     dt = time.perf_counter() - t0
     value = 2.0 * rows * N * K * args.steps / dt / 1e12
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": dict(WORKLOAD, sample_rows_per_step=rows, parallelism="host cores"),
+        "data": "synthetic", "config": dict(WORKLOAD, sample_rows_per_step=rows, parallelism="host cores",
+                                            format="nvfp4 (block 16)" if nv else "int4 (group 64)"),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                          "sample": f"{rows} of 4096 token rows per step (quantize + output); packing offline"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -206,15 +218,15 @@ def run_reference(args):
     return 0
 
 
-def cpu_baseline(rows_req: int):
+def cpu_baseline(rows_req: int, nvfp4: bool = False):
     """The oracle as it stands on the host cores: whole passes over a sample of the workload's
     rows, repeated until about ten seconds of CPU work (packing excluded, as on the GPU)."""
     K, N = WORKLOAD["K"], WORKLOAD["N"]
     rows = rows_req or WORKLOAD["M"]
-    Xb, U, wts, layer = oracle_sample(rows)
+    Xb, U, wts, layer = oracle_sample(rows, nvfp4)
     reps, t0 = 0, time.perf_counter()
     while True:
-        oracle_step(Xb, U, wts, layer.G)
+        oracle_step(Xb, U, wts, layer.G, nvfp4)
         reps += 1
         dt = time.perf_counter() - t0
         if dt >= 10.0 or reps >= 50:
@@ -241,9 +253,11 @@ def kernel_traffic(kernel: str):
 
 # ------------------------------------------------------------------ GPU arm
 
-def alg_bytes_actquant(M, K, r_pad, G):
-    """Kernel (a): read X (2MK) and U (hi/lo, twice), write codes (MK/2), scales (4MK/G), p_hat."""
-    return 2 * M * K + M * K // 2 + 4 * M * K // G + 2 * M * r_pad + 2 * (2 * K * r_pad) * 2
+def alg_bytes_actquant(M, K, r_pad, G, nvfp4=False):
+    """Kernel (a): read X (2MK) and U (hi/lo, twice), write codes (MK/2), scales (INT4: float32
+    per group, 4MK/G; NVFP4: one E4M3 byte per 16, MK/16), p_hat."""
+    scales = M * K // 16 if nvfp4 else 4 * M * K // G
+    return 2 * M * K + M * K // 2 + scales + 2 * M * r_pad + 2 * (2 * K * r_pad) * 2
 
 
 def run_ours(args):
@@ -266,6 +280,8 @@ def run_ours(args):
     bf16_peak = peaks.get("bf16_tflops", 1900.0)
     fp8_peak = 2.0 * bf16_peak  # dense fp8 = 2x dense bf16 (nominal 4.5 / 2.25 PFLOP/s)
 
+    fp4_peak = 6.0 * bf16_peak  # dense fp4 = 6x dense bf16 (nominal 13.5 / 2.25 PFLOP/s)
+
     layer_def = wl.dit_attention().layers[0]
     M, K, N, r, G = layer_def.M, layer_def.K, layer_def.N, layer_def.r, layer_def.G
     Xb = layer_def.x()
@@ -277,65 +293,102 @@ def run_ours(args):
 
     W = dev_bf16(Wb)
     Ud = torch.from_numpy(U).to(dev)
-    # rotating sets: distinct weights (packed per set), activations, workspaces and outputs
-    sets = []
     X0 = dev_bf16(Xb)
-    for i in range(ROTATE_SETS):
-        lin = asp.AspLinear(W, Ud, G)
-        X = X0 if i == 0 else X0.clone()
-        ws = lin.workspace(M)
-        Y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
-        sets.append((lin, X, ws, Y))
-    working_mb = ROTATE_SETS * (2 * M * K + 2 * M * N + lin_ws_bytes(sets[0][0], M) + N * K // 2) / 1e6
     stream = torch.cuda.current_stream(dev)
-
-    def step(i):
-        lin, X, ws, Y = sets[i % ROTATE_SETS]
-        asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
-        asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
-
-    for i in range(args.warmup):
-        step(i)
-    torch.cuda.synchronize()
-    for lin, *_ in sets:
-        st = asp.qwam_asp_get_error(lin.h)
-        if st != asp.QWAM_OK:
-            raise RuntimeError(f"device error after warm-up: {asp.status_string(st)}")
-
-    # timed region: per-kernel events on the launching stream
-    nsteps = args.steps
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * nsteps)]
-    clocks = ClockSampler(local)
-    clocks.start()
-    time.sleep(0.3)
-    barrier(world)
-    torch.cuda.synchronize()
-    clocks.mark("t0")
-    start = torch.cuda.Event(enable_timing=True)
-    end = torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for i in range(nsteps):
-        lin, X, ws, Y = sets[i % ROTATE_SETS]
-        ev[3 * i].record(stream)
-        asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
-        ev[3 * i + 1].record(stream)
-        asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
-        ev[3 * i + 2].record(stream)
-    end.record(stream)
-    torch.cuda.synchronize()
-    clocks.mark("t1")
-    barrier(world)
-    clocks.stop()
-    total_ms = start.elapsed_time(end)
-    t_a = sum(ev[3 * i].elapsed_time(ev[3 * i + 1]) for i in range(nsteps)) / nsteps
-    t_b = sum(ev[3 * i + 1].elapsed_time(ev[3 * i + 2]) for i in range(nsteps)) / nsteps
-    for lin, *_ in sets:
-        st = asp.qwam_asp_get_error(lin.h)
-        if st != asp.QWAM_OK:
-            raise RuntimeError(f"device error in the timed region: {asp.status_string(st)}")
-    total_ms = max_over_ranks(total_ms, world, dev)
     flops = 2.0 * M * N * K
-    value = aggregate_value(flops, nsteps, world, total_ms)
+
+    def timed(fmt, nsteps, warmup, clocks=None):
+        """Per-kernel CUDA-event times of `nsteps` steps over rotating sets (weights packed per
+        set, activations, workspaces, outputs), after `warmup` untimed steps."""
+        sets = []
+        for i in range(ROTATE_SETS):
+            lin = asp.AspLinear(W, Ud, G, fmt=fmt)
+            X = X0 if i == 0 else X0.clone()
+            sets.append((lin, X, lin.workspace(M), torch.empty((M, N), dtype=torch.bfloat16, device=dev)))
+        mb = ROTATE_SETS * (2 * M * K + 2 * M * N + lin_ws_bytes(sets[0][0], M) + N * K // 2) / 1e6
+        for i in range(warmup):
+            lin, X, ws, Y = sets[i % ROTATE_SETS]
+            asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
+            asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
+        torch.cuda.synchronize()
+        for lin, *_ in sets:
+            st = asp.qwam_asp_get_error(lin.h)
+            if st != asp.QWAM_OK:
+                raise RuntimeError(f"device error after warm-up: {asp.status_string(st)}")
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * nsteps)]
+        if clocks is not None:
+            clocks.start()
+            time.sleep(0.3)
+        barrier(world)
+        torch.cuda.synchronize()
+        if clocks is not None:
+            clocks.mark("t0")
+        start = torch.cuda.Event(enable_timing=True)
+        end = torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for i in range(nsteps):
+            lin, X, ws, Y = sets[i % ROTATE_SETS]
+            ev[3 * i].record(stream)
+            asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
+            ev[3 * i + 1].record(stream)
+            asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
+            ev[3 * i + 2].record(stream)
+        end.record(stream)
+        torch.cuda.synchronize()
+        if clocks is not None:
+            clocks.mark("t1")
+        barrier(world)
+        if clocks is not None:
+            clocks.stop()
+        total_ms = start.elapsed_time(end)
+        t_a = sum(ev[3 * i].elapsed_time(ev[3 * i + 1]) for i in range(nsteps)) / nsteps
+        t_b = sum(ev[3 * i + 1].elapsed_time(ev[3 * i + 2]) for i in range(nsteps)) / nsteps
+        for lin, *_ in sets:
+            st = asp.qwam_asp_get_error(lin.h)
+            if st != asp.QWAM_OK:
+                raise RuntimeError(f"device error in the timed region: {asp.status_string(st)}")
+        total_ms = max_over_ranks(total_ms, world, dev)
+        return dict(sets=sets, total_ms=total_ms, t_a=t_a, t_b=t_b, mb=mb,
+                    value=aggregate_value(flops, nsteps, world, total_ms))
+
+    def rooflines(fmt, t_a, t_b, step_ms, r_pad):
+        """Per-kernel achieved vs peak, the dominant kernel's roofline object and the layer's
+        roofline fraction (slower of the algorithmic bytes over HBM and the MMA kind's peak)."""
+        nv = fmt == asp.QWAM_FMT_NVFP4
+        a_bytes = alg_bytes_actquant(M, K, r_pad, G, nv)
+        peak, pname = (fp4_peak, "fp4") if nv else (fp8_peak, "fp8")
+        gname = "gemm_nvfp4" if nv else "gemm_w4a4_lr"
+        kern = {
+            "actquant": {"ms": t_a, "bound": "hbm", "alg_bytes": a_bytes,
+                         "achieved_gbs": a_bytes / (t_a * 1e-3) / 1e9, "peak_gbs": hbm_peak},
+            gname: {"ms": t_b, "bound": "tensor", "alg_flops": flops,
+                    "achieved_tflops": flops / (t_b * 1e-3) / 1e12, f"peak_tflops_{pname}": peak},
+        }
+        kern["actquant"]["frac"] = kern["actquant"]["achieved_gbs"] / hbm_peak
+        kern[gname]["frac"] = kern[gname]["achieved_tflops"] / peak
+        if t_b >= t_a:
+            roof = {"kernel": gname, "bound": "tensor", "achieved": kern[gname]["achieved_tflops"],
+                    "peak": peak, "unit": "TFLOP/s", "frac": kern[gname]["frac"],
+                    "traffic": kernel_traffic("gemm_nvfp4_kernel" if nv else "gemm_kernel"),
+                    "peak_source": "measured bf16 burst x %d (nominal %s/bf16 dense ratio), of measured"
+                                   % (6 if nv else 2, pname)}
+        else:
+            roof = {"kernel": "actquant", "bound": "hbm", "achieved": kern["actquant"]["achieved_gbs"],
+                    "peak": hbm_peak, "unit": "GB/s", "frac": kern["actquant"]["frac"],
+                    "traffic": kernel_traffic("actquant_kernel"),
+                    "peak_source": "measured HBM copy, of measured"}
+        w_bytes = N * K // 2 + (N * K // 16 if nv else 2 * N * K // G)
+        t_roof = max((2 * M * K + w_bytes + 2 * K * r_pad + 2 * N * r_pad + 2 * M * N) / (hbm_peak * 1e9),
+                     flops / (peak * 1e12))
+        return kern, roof, (t_roof * 1e3) / step_ms
+
+    fmt = asp.QWAM_FMT_NVFP4 if args.format == "nvfp4" else asp.QWAM_FMT_INT4
+    nsteps = args.steps
+    clocks = ClockSampler(local)
+    main_run = timed(fmt, nsteps, args.warmup, clocks)
+    sets, total_ms, t_a, t_b = main_run["sets"], main_run["total_ms"], main_run["t_a"], main_run["t_b"]
+    value = main_run["value"]
+    working_mb = main_run["mb"]
 
     # End to end through the public API, as a serving loop would run it: every step copies its
     # activations from pinned host memory to the device, runs the layer (qwam_asp_linear) and
@@ -385,52 +438,47 @@ def run_ours(args):
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     e2e_value = aggregate_value(flops, e2e_steps, world, e2e_ms)
 
-    # roofline of the dominant kernel (per-launch averages from the events above)
     r_pad = sets[0][0].r_pad
-    a_bytes = alg_bytes_actquant(M, K, r_pad, G)
-    kern = {
-        "actquant": {"ms": t_a, "bound": "hbm", "alg_bytes": a_bytes,
-                     "achieved_gbs": a_bytes / (t_a * 1e-3) / 1e9, "peak_gbs": hbm_peak},
-        "gemm_w4a4_lr": {"ms": t_b, "bound": "tensor", "alg_flops": flops,
-                         "achieved_tflops": flops / (t_b * 1e-3) / 1e12, "peak_tflops_fp8": fp8_peak},
-    }
-    kern["actquant"]["frac"] = kern["actquant"]["achieved_gbs"] / hbm_peak
-    kern["gemm_w4a4_lr"]["frac"] = kern["gemm_w4a4_lr"]["achieved_tflops"] / fp8_peak
-    if t_b >= t_a:
-        roof = {"kernel": "gemm_w4a4_lr", "bound": "tensor", "achieved": kern["gemm_w4a4_lr"]["achieved_tflops"],
-                "peak": fp8_peak, "unit": "TFLOP/s", "frac": kern["gemm_w4a4_lr"]["frac"],
-                "traffic": kernel_traffic("gemm_kernel"),
-                "peak_source": "measured bf16 burst x 2 (nominal fp8/bf16 dense ratio), of measured"}
-    else:
-        roof = {"kernel": "actquant", "bound": "hbm", "achieved": kern["actquant"]["achieved_gbs"],
-                "peak": hbm_peak, "unit": "GB/s", "frac": kern["actquant"]["frac"],
-                "traffic": kernel_traffic("actquant_kernel"),
-                "peak_source": "measured HBM copy, of measured"}
+    kern, roof, layer_frac = rooflines(fmt, t_a, t_b, total_ms / nsteps, r_pad)
+    variants = {}
+    if fmt == asp.QWAM_FMT_INT4:
+        for lin_, *_ in sets:
+            lin_.close()
+        sets = []
+        vsteps = max(3, min(nsteps, 500))
+        vr = timed(asp.QWAM_FMT_NVFP4, vsteps, max(3, min(args.warmup, 20)))
+        vk, vroof, vfrac = rooflines(asp.QWAM_FMT_NVFP4, vr["t_a"], vr["t_b"], vr["total_ms"] / vsteps, r_pad)
+        variants["nvfp4"] = {"value": vr["value"], "unit": UNIT, "steps": vsteps,
+                             "ms_per_step": vr["total_ms"] / vsteps, "dtype": "e2m1",
+                             "format": "NVFP4 (App. B.1): E2M1, E4M3 scale per 16 K, float32 per-tensor weight scale",
+                             "roofline": vroof, "layer_roofline_frac": vfrac, "kernels": vk}
+        for s_ in vr["sets"]:
+            s_[0].close()
 
     if rank != 0:
         return 0
-    t_layer_roof = max((a_bytes + N * K // 2 + 2 * N * K // G + 2 * N * r_pad + 2 * M * N) / (hbm_peak * 1e9),
-                       flops / (fp8_peak * 1e12))
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": nsteps, "warmup": args.warmup,
         "ms_per_step": total_ms / nsteps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "e4m3", "data": "synthetic",
+        "dtype": "e2m1" if fmt == asp.QWAM_FMT_NVFP4 else "e4m3", "data": "synthetic",
         "config": dict(WORKLOAD, parallelism=f"replicas by token rows x{world}",
+                       format="nvfp4 (block 16)" if fmt == asp.QWAM_FMT_NVFP4 else "int4 (group 64)",
                        l2="rotating buffers: %d sets, %.0f MB > L2" % (ROTATE_SETS, working_mb)),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 2 * M * K, "d2h_bytes_per_step": 2 * M * N,
                 "steps": e2e_steps,
                 "pipeline": "copies on their own streams, overlapping the layer of the neighbouring steps"},
         "gpu_launches": 2 * nsteps,
         "roofline": roof,
-        "layer_roofline_frac": (t_layer_roof * 1e3) / (total_ms / nsteps),
+        "layer_roofline_frac": layer_frac,
         "kernels": kern,
+        "variants": variants,
         "clocks": clocks.summary(),
     }
     if not args.no_cpu_baseline and world == 1:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_rows)
+        line["cpu_baseline"] = cpu_baseline(args.cpu_rows, fmt == asp.QWAM_FMT_NVFP4)
     print(json.dumps(line))
-    for s in sets:
-        s[0].close()
+    for s_ in sets:
+        s_[0].close()
     return 0
 
 
