@@ -12,12 +12,13 @@
 // Persistent CTAs (one per SM) walk 128 x 128 output tiles with a static stride.  192 threads:
 //   warp 0   TMA producer: per stage of 256 K, the two 16 KB code tiles (128-byte swizzle) and
 //            the two 2 KB scale-atom blocks (plain bulk copies; see internal.h for the atom);
-//   warp 1   MMA issuer and TMEM owner: copies a stage's scale atoms into TMEM
+//   warp 1   MMA issuer and TMEM owner (lane 0): copies a stage's scale atoms into TMEM
 //            (tcgen05.cp.32x128b.warpx4, which puts the 32 x 16 bytes of an atom into all four
 //            lane quarters, where the MMA reads them), then issues four 128x128x64 MMAs;
 //            tcgen05 operations of one thread run in issue order, so a scale slot is rewritten
 //            only after the MMAs that read it;
-//   warps 2-5 epilogue: one TMEM lane quarter each (thread = output row), 32x32b loads.
+//   warps 2-5 epilogue: one TMEM lane quarter each (thread = output row), 32x32b loads; warp 2
+//            also issues each tile's branch MMA, so the MMA issuer never waits on the branch.
 // TMEM: two accumulators (columns 0..255), the branch accumulator (256..383), four scale slots
 // of 32 columns (384..511: A at +0, B at +16, four columns per MMA).
 #include "internal.h"
@@ -165,57 +166,53 @@ __global__ void __launch_bounds__(kThreads4, 1)
     }
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
+    // The whole warp walks the loop (warp-uniform counters and descriptors); one elected lane
+    // issues.  The tensor pipe queues little ahead of the issuing thread, so the work between
+    // MMAs is kept small: counters advance by increments, descriptors are offsets from
+    // precomputed bases, and the 16-bit branch MMA is issued by an epilogue warp instead.
     bool ok = true;
     constexpr uint32_t idesc = idesc_nvf4(kBM, kGemmBN);
-    int s = 0;
+    const uint32_t s0 = smem_u32(stages);
+    const uint64_t adesc_base = smem_desc(s0, 16, 1024, kSw128);
+    const uint64_t bdesc_base = smem_desc(s0 + A4_BYTES, 16, 1024, kSw128);
+    const uint64_t sadesc_base = smem_desc(s0 + A4_BYTES + B4_BYTES, 128, 128, kSwNone);
+    const uint64_t sbdesc_base = smem_desc(s0 + A4_BYTES + B4_BYTES + SF4_BYTES, 128, 128, kSwNone);
+    int slot = 0, phase = 0, sfs = 0;  // operand slot, its phase bit, scale slot
     for (int ti = 0; ti < my_tiles && ok; ++ti) {
-      const int ub = ti & 1;
-      if (ti >= 2) ok = mbar_wait_inline(&tempty[ub], ((ti >> 1) & 1) ^ 1, wc);
-      if (!ok) break;
-      tc_fence_after();
-      for (int st = 0; st < nst && ok; ++st, ++s) {
-        const int slot = s % NS4;
-        ok = mbar_wait_inline(&full[slot], (s / NS4) & 1, wc);
+      const uint32_t d = tmem + 128u * static_cast<uint32_t>(ti & 1);
+      if (ti >= 2) {
+        ok = mbar_wait_inline(&tempty[ti & 1], ((ti >> 1) & 1) ^ 1, wc);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t pa = smem_u32(stage(slot)), pb = pa + A4_BYTES;
-        const uint32_t psa = pb + B4_BYTES, psb = psa + SF4_BYTES;
-        const uint64_t adesc0 = smem_desc(pa, 16, 1024, kSw128), bdesc0 = smem_desc(pb, 16, 1024, kSw128);
-        const uint32_t ta = tmem + kColScale + 32u * static_cast<uint32_t>(s % NSF), tb = ta + 16;
+      }
+      for (int st = 0; st < nst; ++st) {
+        ok = mbar_wait_inline(&full[slot], phase, wc);
+        if (!ok) break;
+        tc_fence_after();
+        const uint64_t soff = static_cast<uint64_t>(slot) * (STAGE4 >> 4);
+        const uint32_t ta = tmem + kColScale + 32u * static_cast<uint32_t>(sfs), tb = ta + 16;
         if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {
-            tc_cp_32x128b_x4(ta + 4 * kk, smem_desc(psa + kk * kSfAtom, 128, 128, kSwNone));
-            tc_cp_32x128b_x4(tb + 4 * kk, smem_desc(psb + kk * kSfAtom, 128, 128, kSwNone));
+            tc_cp_32x128b_x4(ta + 4 * kk, sadesc_base + soff + kk * (kSfAtom >> 4));
+            tc_cp_32x128b_x4(tb + 4 * kk, sbdesc_base + soff + kk * (kSfAtom >> 4));
           }
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)  // 32 bytes (64 codes) of each row per MMA
-            mma_nvf4(tmem + 128u * ub, adesc0 + 2 * kk, bdesc0 + 2 * kk, idesc, ta + 4 * kk, tb + 4 * kk,
+            mma_nvf4(d, adesc_base + soff + 2 * kk, bdesc_base + soff + 2 * kk, idesc, ta + 4 * kk, tb + 4 * kk,
                      (st | kk) != 0);
           mma_commit(&empty[slot]);
         }
         __syncwarp();
+        if (++slot == NS4) {
+          slot = 0;
+          phase ^= 1;
+        }
+        sfs = (sfs + 1) & (NSF - 1);
       }
       if (!ok) break;
-      if (elect_one()) mma_commit(&tfull[ub]);
+      if (elect_one()) mma_commit(&tfull[ti & 1]);
       __syncwarp();
-      if constexpr (RP > 0) {
-        ok = mbar_wait_inline(bfull, ti & 1, wc);
-        if (ok && ti >= 1) ok = mbar_wait_inline(brempty, (ti & 1) ^ 1, wc);
-        if (!ok) break;
-        tc_fence_after();
-        constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
-        const uint32_t pp = smem_u32(br), pw = pp + Cfg::BR_BYTES;
-        const uint64_t pdesc0 = smem_desc(pp, 2048, 128, kSwNone), wdesc0 = smem_desc(pw, 2048, 128, kSwNone);
-        if (elect_one()) {
-#pragma unroll
-          for (int kk = 0; kk < RP / 16; ++kk)
-            mma_f16(tmem + kColBranch, pdesc0 + kk * 256, wdesc0 + kk * 256, idesc_br, kk != 0);  // 4096 B
-          mma_commit(brfull);
-          mma_commit(bempty);
-        }
-        __syncwarp();
-      }
     }
     if (elect_one()) mma_commit(drain);
     __syncwarp();
@@ -228,6 +225,27 @@ __global__ void __launch_bounds__(kThreads4, 1)
     const int row = quad * 32 + static_cast<int>(lane);
     const uint32_t tq = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     bool ok = true;
+    // Warp 2 issues the branch MMA p_hat B_hat^T of tile t (kind::f16, K = RP) into the branch
+    // accumulator once the four epilogue warps have read tile t - 1's and the operands have landed.
+    auto issue_branch = [&](int t) {
+      if constexpr (RP > 0) {
+        if (ok && t >= 1) ok = mbar_wait_inline(brempty, (t - 1) & 1, wc);
+        if (ok) ok = mbar_wait_inline(bfull, t & 1, wc);
+        tc_fence_after();
+        if (ok && lane == 0) {
+          constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
+          const uint32_t pp = smem_u32(br), pw = pp + Cfg::BR_BYTES;
+          const uint64_t pdesc0 = smem_desc(pp, 2048, 128, kSwNone), wdesc0 = smem_desc(pw, 2048, 128, kSwNone);
+#pragma unroll
+          for (int kk = 0; kk < RP / 16; ++kk)
+            mma_f16(tmem + kColBranch, pdesc0 + kk * 256, wdesc0 + kk * 256, idesc_br, kk != 0);  // 4096 B
+          mma_commit(brfull);
+          mma_commit(bempty);
+        }
+        __syncwarp();
+      }
+    };
+    if (wid == 2 && my_tiles > 0) issue_branch(0);
     for (int ti = 0; ti < my_tiles; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
@@ -273,6 +291,7 @@ __global__ void __launch_bounds__(kThreads4, 1)
           }
         }
       }
+      if (wid == 2 && ti + 1 < my_tiles) issue_branch(ti + 1);
     }
   }
 
