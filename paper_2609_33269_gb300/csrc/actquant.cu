@@ -243,7 +243,7 @@ __global__ void __launch_bounds__(320, 1)
     auto produce = [&](bool first_pass, int c) {
       const int s = it % S;
       if (ok && it >= S) ok = mbar_wait(&empty[s], ((it / S) & 1) ^ 1, wc);
-      if (ok) {
+      if (ok && elect_one()) {
         const uint32_t bytes = Cfg::X_BYTES + (first_pass ? Cfg::U1_BYTES : (RP > 0 ? Cfg::U2_BYTES : 0));
         mbar_arrive_expect_tx(&full[s], bytes);
         tma_load_2d(stage_x(s), &x_map, &full[s], k0 + c * kChunk, m0);
@@ -254,31 +254,30 @@ __global__ void __launch_bounds__(320, 1)
             tma_load_2d(stage_u(s) + q * 8192, &u3_map, &full[s], q * 64, k0 + c * kChunk);
         }
       }
+      __syncwarp();
       ++it;
     };
-    if (lane == 0) {
-      tma_prefetch_desc(&x_map);
-      for (int c = 0; c < pass1; ++c) produce(true, c);
-      for (; issued2 < nch && issued2 < S; ++issued2) produce(false, issued2);
-    }
+    // The whole warp walks the ring (warp-uniform state); one elected lane issues each copy.
+    if (elect_one()) tma_prefetch_desc(&x_map);
     __syncwarp();
+    for (int c = 0; c < pass1; ++c) produce(true, c);
+    for (; issued2 < nch && issued2 < S; ++issued2) produce(false, issued2);
     if (RP > 0) {
       cluster_sync();
       cluster_sync();
       cluster_sync();
     }
-    if (lane == 0) {
-      for (; issued2 < nch; ++issued2) produce(false, issued2);
-      // Let every load issued into the ring land before the CTA can exit.
-      int never = 0;
-      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-      for (int j = (it > S ? it - S : 0); j < it; ++j) mbar_wait(&full[j % S], (j / S) & 1, dc);
-    }
+    for (; issued2 < nch; ++issued2) produce(false, issued2);
+    // Let every load issued into the ring land before the CTA can exit.
+    int never = 0;
+    const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+    for (int j = (it > S ? it - S : 0); j < it; ++j) mbar_wait(&full[j % S], (j / S) & 1, dc);
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
     if constexpr (RP > 0) {
+      // The whole warp walks both passes (warp-uniform state); one elected lane issues.
       bool ok = true;
-      if (lane == 0) {
+      {
         constexpr uint32_t idesc_proj = idesc_bf16(kBM, 2 * RP);
         for (int c = 0; c < nch && ok; ++c) {
           const int s = c % S;
@@ -286,19 +285,22 @@ __global__ void __launch_bounds__(320, 1)
           if (!ok) break;
           tc_fence_after();
           const uint32_t xa = smem_u32(stage_x(s)), ua = smem_u32(stage_u(s));
+          if (elect_one()) {
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            mma_f16(tmem, smem_desc(xa + kk * 32, 16, 1024, kSw128), smem_desc(ua + kk * 32, 16, 1024, kSw128),
-                    idesc_proj, (c | kk) != 0);
-          mma_commit(&empty[s]);
+            for (int kk = 0; kk < 4; ++kk)
+              mma_f16(tmem, smem_desc(xa + kk * 32, 16, 1024, kSw128), smem_desc(ua + kk * 32, 16, 1024, kSw128),
+                      idesc_proj, (c | kk) != 0);
+            mma_commit(&empty[s]);
+          }
+          __syncwarp();
         }
-        mma_commit(proj_done);
+        if (elect_one()) mma_commit(proj_done);
       }
       __syncwarp();
       cluster_sync();
       cluster_sync();
       cluster_sync();
-      if (lane == 0) {
+      {
         if (ok) ok = mbar_wait(arec_ready, 0, wc);
         tc_fence_after();
         constexpr uint32_t idesc_rec = idesc_bf16(kBM, kChunk);
@@ -310,16 +312,20 @@ __global__ void __launch_bounds__(320, 1)
           if (!ok) break;
           tc_fence_after();
           const uint32_t ua = smem_u32(stage_u(s));
+          if (elect_one()) {
 #pragma unroll
-          for (int kk = 0; kk < 3 * RP / 16; ++kk) {
-            const int q = kk >> 2, off = (kk & 3) * 32;
-            mma_f16(tmem + 128 + 64 * b, smem_desc(ar + q * 16384 + off, 16, 1024, kSw128),
-                    smem_desc(ua + q * 8192 + off, 16, 1024, kSw128), idesc_rec, kk != 0);
+            for (int kk = 0; kk < 3 * RP / 16; ++kk) {
+              const int q = kk >> 2, off = (kk & 3) * 32;
+              mma_f16(tmem + 128 + 64 * b, smem_desc(ar + q * 16384 + off, 16, 1024, kSw128),
+                      smem_desc(ua + q * 8192 + off, 16, 1024, kSw128), idesc_rec, kk != 0);
+            }
+            mma_commit(&tfull[b]);
           }
-          mma_commit(&tfull[b]);
+          __syncwarp();
         }
         // Make sure every MMA of this CTA has completed before TMEM is released.
-        mma_commit(drain);
+        if (elect_one()) mma_commit(drain);
+        __syncwarp();
         int never = 0;
         const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
         mbar_wait(drain, 0, dc);

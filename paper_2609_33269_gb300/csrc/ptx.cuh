@@ -92,12 +92,18 @@ __device__ __forceinline__ bool wait_loop(uint64_t* bar, uint32_t parity, const 
 static __device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
   return wait_loop(bar, parity, c);
 }
+// Every lane that calls a wait together gets the same answer: a lane that saw the phase complete
+// and one that gave up at the deadline would otherwise part ways before a warp-wide instruction
+// (elect.sync, a warp barrier) that needs them all.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
-  if (mbar_try_wait(bar, parity)) return true;
-  return wait_slow(bar, parity, c);
+  const bool r = mbar_try_wait(bar, parity) || wait_slow(bar, parity, c);
+  return __all_sync(__activemask(), r) != 0;
 }
 // The same wait with the slow loop inlined, for kernels that set per-warpgroup register budgets
-// (setmaxnreg): ptxas cannot allocate registers for a function called from such regions.
+// (setmaxnreg): ptxas cannot allocate registers for a function called from such regions.  It is
+// on the hot paths, so it takes no vote: a warp that enters it converged stays converged, because
+// each try is one warp instruction on one barrier (every lane gets the same result) and the loop's
+// deadline checks fall on the same iteration for every lane.
 __device__ __forceinline__ bool mbar_wait_inline(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
   if (mbar_try_wait(bar, parity)) return true;
   return wait_loop(bar, parity, c);
