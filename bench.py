@@ -375,7 +375,7 @@ def run_ours(args):
         else:
             roof = {"kernel": "actquant", "bound": "hbm", "achieved": kern["actquant"]["achieved_gbs"],
                     "peak": hbm_peak, "unit": "GB/s", "frac": kern["actquant"]["frac"],
-                    "traffic": kernel_traffic("actquant_kernel"),
+                    "traffic": kernel_traffic("actquant_kernel_nvfp4" if nv else "actquant_kernel"),
                     "peak_source": "measured HBM copy, of measured"}
         w_bytes = N * K // 2 + (N * K // 16 if nv else 2 * N * K // G)
         t_roof = max((2 * M * K + w_bytes + 2 * K * r_pad + 2 * N * r_pad + 2 * M * N) / (hbm_peak * 1e9),

@@ -12,7 +12,8 @@
 // Persistent CTAs (one per SM) walk 128 x 128 output tiles with a static stride.  192 threads:
 //   warp 0   TMA producer: per stage of 256 K, the two 16 KB code tiles (128-byte swizzle) and
 //            the two 2 KB scale-atom blocks (plain bulk copies; see internal.h for the atom);
-//   warp 1   MMA issuer and TMEM owner (lane 0): copies a stage's scale atoms into TMEM
+//   warp 1   MMA issuer and TMEM owner (warp-wide loop, one elected lane issues): copies a
+//            stage's scale atoms into TMEM
 //            (tcgen05.cp.32x128b.warpx4, which puts the 32 x 16 bytes of an atom into all four
 //            lane quarters, where the MMA reads them), then issues four 128x128x64 MMAs;
 //            tcgen05 operations of one thread run in issue order, so a scale slot is rewritten
