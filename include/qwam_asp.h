@@ -215,6 +215,22 @@ const char* qwam_status_string(qwam_status s);
 qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws, float* R,
                                     struct CUstream_st* stream);
 
+/* Test support: kernel (a)'s quantizer alone (Eq. (quant) with the rounding of readings R2, R3
+ * and R5; for fmt == QWAM_FMT_NVFP4 the block rule of App. B.1 read as N1-N3) applied to
+ * caller-given float32 rows, so that its rounding can be checked on chosen values such as exact
+ * ties and values a few units in the last place from a rounding boundary.  No handle is needed.
+ *   R      : device float32 [M, K], row-major, 16-byte aligned; K % 64 == 0
+ *   fmt    : QWAM_FMT_INT4 or QWAM_FMT_NVFP4
+ *   group  : 32 or 64 for INT4 (ignored for NVFP4, whose block is 16)
+ *   codes  : device, 16-byte aligned.  INT4: uint8 [M, K], each the E4M3 bit pattern of c * 2^-9
+ *            (sign bit | magnitude), as in the activation workspace.  NVFP4: uint8 [M, K/2], two
+ *            E2M1 codes per byte, low nibble = even k.
+ *   scales : device.  INT4: float32 [M, K/group] row-major (4-byte aligned).  NVFP4: uint8 E4M3
+ *            bit patterns [M, K/16] row-major.
+ * Asynchronous on `stream`; QWAM_ERR_INVALID_ARG for bad sizes, formats or alignment. */
+qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, int group, void* codes,
+                                         void* scales, struct CUstream_st* stream);
+
 /* Set the bound of every device wait of this handle's kernels, in seconds (default 2.0). */
 qwam_status qwam_asp_set_timeout(qwam_asp_handle h, double seconds);
 

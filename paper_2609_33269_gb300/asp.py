@@ -38,6 +38,7 @@ EXPORTED = [
     "qwam_asp_shape", "qwam_asp_export", "qwam_asp_destroy", "qwam_status_string",
     "qwam_asp_debug_residual", "qwam_asp_set_timeout", "qwam_asp_debug_wait_timeout",
     "qwam_asp_linear_static", "qwam_asp_pack_weights_nvfp4", "qwam_asp_format", "qwam_asp_export_nvfp4",
+    "qwam_asp_debug_quantize_rows",
 ]
 
 _lib = None
@@ -76,6 +77,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_status_string.argtypes = [I]
         lib.qwam_status_string.restype = ctypes.c_char_p
         lib.qwam_asp_debug_residual.argtypes = [V, I, H, V, V, V]
+        lib.qwam_asp_debug_quantize_rows.argtypes = [V, I, I, I, I, V, V, V]
         lib.qwam_asp_set_timeout.argtypes = [H, ctypes.c_double]
         lib.qwam_asp_debug_wait_timeout.argtypes = [H, I, V]
         lib.qwam_asp_pack_weights_nvfp4.argtypes = [V, V, I, I, I, V, ctypes.POINTER(H)]
@@ -213,6 +215,11 @@ def qwam_asp_destroy(h: int):
 def qwam_asp_debug_residual(X_bf16, M: int, h: int, act_ws, R, stream=None):
     _check(load().qwam_asp_debug_residual(_ptr(X_bf16), M, h, _ptr(act_ws), _ptr(R), _stream(stream)),
            "qwam_asp_debug_residual")
+
+
+def qwam_asp_debug_quantize_rows(R, M: int, K: int, fmt: int, group: int, codes, scales, stream=None):
+    _check(load().qwam_asp_debug_quantize_rows(_ptr(R), M, K, fmt, group, _ptr(codes), _ptr(scales),
+                                               _stream(stream)), "qwam_asp_debug_quantize_rows")
 
 
 def qwam_asp_set_timeout(h: int, seconds: float):

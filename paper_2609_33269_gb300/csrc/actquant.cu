@@ -72,17 +72,17 @@ constexpr int kMagicBits = 0x4B400000;
 // Nearest integer to the exact quotient x / s, ties to even (s > 0, |x| <= ~7.5 s).
 // c = rint(x * (1/s)) is the answer or its neighbour; the remainder e = x - c s is exact in
 // float32 (c and the true answer differ by at most one), and |e| < s/2 exactly when c is right
-// and not a tie, so only |e| >= s/2 (rare) needs the exact decision.
+// and not a tie.  The correction is taken with selects rather than a branch: a branch per value
+// keeps the compiler from overlapping the 64 independent roundings of a group.
 __device__ __forceinline__ int nearest_code(float x, float s, float inv, float hs) {
   const float t = fmaf(x, inv, kMagic);
   const float c = t - kMagic;
   const float e = fmaf(-c, s, x);
-  int ci = __float_as_int(t) - kMagicBits;
-  if (fabsf(e) >= hs) {
-    const float te = 2.0f * fabsf(e);
-    if (te > s || (te == s && (ci & 1))) ci += (e > 0.0f) ? 1 : -1;
-  }
-  return ci;
+  const int ci = __float_as_int(t) - kMagicBits;
+  const float ae = fabsf(e);
+  // |e| > s/2: the neighbour on e's side; |e| == s/2 (a tie): the even one of the two
+  const int adj = static_cast<int>(ae > hs) | (static_cast<int>(ae == hs) & ci & 1);
+  return ci + (e > 0.0f ? adj : -adj);
 }
 // Approximate reciprocal (the hardware's single-instruction estimate).  It only seeds the
 // rounding in nearest_code, whose exact remainder test corrects a seed that is off by one.
@@ -154,7 +154,19 @@ __device__ __forceinline__ uint32_t cvt_e2m1(float u) {
   asm("{.reg .b8 t;\ncvt.rn.satfinite.e2m1x2.f32 t, %1, %1;\ncvt.u32.u8 %0, t;}" : "=r"(v) : "f"(u));
   return v & 0xFu;
 }
+// Two values -> their E2M1 codes in one byte, the first in the low nibble (cvt puts its first
+// source operand in the upper half of the destination).
+__device__ __forceinline__ uint32_t cvt_e2m1x2(float lo, float hi) {
+  uint32_t v;
+  asm("{.reg .b8 t;\ncvt.rn.satfinite.e2m1x2.f32 t, %1, %2;\ncvt.u32.u8 %0, t;}" : "=r"(v) : "f"(hi), "f"(lo));
+  return v;
+}
 // 16 values -> two words of codes (k order, four bits each, low nibble first) and the scale byte.
+// The codes are RN_e2m1 of the float32 quotient RN_f32(x / s).  The fast path rounds q = x * r
+// (r the approximate reciprocal of s: |q - RN_f32(x / s)| < 2^-21 |q|) bracketed by the factors
+// (1 -+ 2^-19): when both ends round to the same code, so does every value between them, the
+// float32 quotient included.  A block with an end pair that differs (a quotient within 2^-19 of
+// an E2M1 midpoint, rare) is recomputed with the correctly rounded division.
 __device__ __forceinline__ uint32_t quantize_block_nvfp4(const float* x, uint32_t* w2) {
   float mx[4];
 #pragma unroll
@@ -162,17 +174,35 @@ __device__ __forceinline__ uint32_t quantize_block_nvfp4(const float* x, uint32_
   const float amax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
   const uint32_t sb = cvt_e4m3(__fdiv_rn(amax, 6.0f));
   const float sc = e4m3_value(sb);
+  const float r = sc > 0.0f ? rcp_approx(sc) : 0.0f;
+  constexpr float kDn = 1.0f - 1.0f / 524288.0f, kUp = 1.0f + 1.0f / 524288.0f;  // 1 -+ 2^-19
+  uint32_t w[2] = {0u, 0u};
+  bool near_mid = false;
+#pragma unroll
+  for (int h = 0; h < 2; ++h)
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+      const float q0 = x[8 * h + i] * r, q1 = x[8 * h + i + 1] * r;
+      const uint32_t lo = cvt_e2m1x2(q0 * kDn, q1 * kDn), hi = cvt_e2m1x2(q0 * kUp, q1 * kUp);
+      near_mid |= lo != hi;
+      w[h] |= lo << (4 * i);
+    }
+  if (near_mid) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      w[h] = 0u;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float u = sc > 0.0f ? __fdiv_rn(x[8 * h + i], sc) : 0.0f;
+        w[h] |= cvt_e2m1(u) << (4 * i);
+      }
+    }
+  }
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    uint32_t w = 0;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float u = sc > 0.0f ? __fdiv_rn(x[8 * h + i], sc) : 0.0f;
-      w |= cvt_e2m1(u) << (4 * i);
-    }
     // a code whose magnitude bits are zero loses its sign bit
-    const uint32_t nz = ((w & 0x77777777u) + 0x77777777u) & 0x88888888u;
-    w2[h] = w & (0x77777777u | nz);
+    const uint32_t nz = ((w[h] & 0x77777777u) + 0x77777777u) & 0x88888888u;
+    w2[h] = w[h] & (0x77777777u | nz);
   }
   return sb;
 }
@@ -527,6 +557,49 @@ __global__ void __launch_bounds__(320, 1)
   }
 }
 
+// Test support: the quantizers above applied to caller-given float32 rows (one thread per row
+// and 64-value chunk), so that their rounding can be checked on chosen values.
+template <bool NV>
+__global__ void __launch_bounds__(128) debug_quantize_kernel(const float* R, int M, int K, int G, uint8_t* codes,
+                                                               void* scales) {
+  const int nch = K / kChunk;
+  const long long idx = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (idx >= static_cast<long long>(M) * nch) return;
+  const int m = static_cast<int>(idx / nch), c = static_cast<int>(idx % nch);
+  float xp[kChunk];
+  const float4* src = reinterpret_cast<const float4*>(R + static_cast<size_t>(m) * K + static_cast<size_t>(c) * kChunk);
+#pragma unroll
+  for (int i = 0; i < kChunk / 4; ++i) {
+    const float4 v = src[i];
+    xp[4 * i] = v.x;
+    xp[4 * i + 1] = v.y;
+    xp[4 * i + 2] = v.z;
+    xp[4 * i + 3] = v.w;
+  }
+  if constexpr (NV) {
+    uint32_t w[8];
+    uint8_t* sf = static_cast<uint8_t*>(scales) + static_cast<size_t>(m) * (K / kFp4Block) + c * (kChunk / kFp4Block);
+#pragma unroll
+    for (int b = 0; b < 4; ++b) sf[b] = static_cast<uint8_t>(quantize_block_nvfp4(xp + 16 * b, w + 2 * b));
+    uint4* dst = reinterpret_cast<uint4*>(codes + static_cast<size_t>(m) * (K / 2) + c * (kChunk / 2));
+    dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+  } else {
+    uint32_t bytes4[16];
+    float2 ab[2];
+    float* sc = static_cast<float*>(scales) + static_cast<size_t>(m) * (K / G) + c * (kChunk / G);
+    if (G == 64) {
+      quantize_group<64>(xp, bytes4, sc, ab);
+    } else {
+      quantize_group<32>(xp, bytes4, sc, ab);
+      quantize_group<32>(xp + 32, bytes4 + 8, sc + 1, ab + 1);
+    }
+    uint4* dst = reinterpret_cast<uint4*>(codes + static_cast<size_t>(m) * K + c * kChunk);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(bytes4[4 * i], bytes4[4 * i + 1], bytes4[4 * i + 2], bytes4[4 * i + 3]);
+  }
+}
+
 // Cluster size (CTAs along K per 128-row tile): as many as fit one wave of the GPU.
 int choose_split(int K, int tiles, int sms) {
   const int chunks = K / kChunk;
@@ -595,6 +668,17 @@ cudaError_t launch_fmt(Handle& h, const ActMaps& am, const void* ws, int M, floa
 }
 
 }  // namespace
+
+cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
+                                       void* scales, cudaStream_t s) {
+  const long long n = static_cast<long long>(M) * (K / kChunk);
+  const int grid = static_cast<int>((n + 127) / 128);
+  if (nvfp4)
+    debug_quantize_kernel<true><<<grid, 128, 0, s>>>(R, M, K, G, codes, scales);
+  else
+    debug_quantize_kernel<false><<<grid, 128, 0, s>>>(R, M, K, G, codes, scales);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
   return h.fmt == kFmtNvfp4 ? launch_fmt<true>(h, am, ws, M, dump, s) : launch_fmt<false>(h, am, ws, M, dump, s);

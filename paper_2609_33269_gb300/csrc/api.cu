@@ -309,6 +309,19 @@ qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h
   return quantize_impl(X_bf16, M, h, act_ws, R, stream);
 }
 
+qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, int group, void* codes,
+                                         void* scales, struct CUstream_st* stream) {
+  if (M < 0 || K <= 0 || K % qwam::kChunk != 0) return QWAM_ERR_INVALID_ARG;
+  if (fmt != QWAM_FMT_INT4 && fmt != QWAM_FMT_NVFP4) return QWAM_ERR_INVALID_ARG;
+  if (fmt == QWAM_FMT_INT4 && group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
+  if (M == 0) return QWAM_OK;
+  if (!R || !codes || !scales || !qwam::aligned16(R) || !qwam::aligned16(codes)) return QWAM_ERR_INVALID_ARG;
+  if (fmt == QWAM_FMT_INT4 && reinterpret_cast<uintptr_t>(scales) % 4 != 0) return QWAM_ERR_INVALID_ARG;
+  return from_cuda_status(qwam::launch_debug_quantize_rows(R, M, K, fmt == QWAM_FMT_NVFP4, group,
+                                                           static_cast<uint8_t*>(codes), scales,
+                                                           reinterpret_cast<cudaStream_t>(stream)));
+}
+
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle hs, void* Y, int y_dtype,
                           struct CUstream_st* stream) {
   if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
