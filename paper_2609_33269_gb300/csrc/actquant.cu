@@ -214,6 +214,7 @@ __global__ void __launch_bounds__(320, 1)
   using Cfg = ActCfg<RP>;
   constexpr int S = Cfg::S;
   extern __shared__ uint8_t smem_raw[];
+  pdl_launch_dependents();
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* stages = smem;
   uint8_t* arec = stages + S * Cfg::STAGE;
@@ -262,6 +263,7 @@ __global__ void __launch_bounds__(320, 1)
   tc_fence_after();
   const uint32_t tmem = (RP > 0) ? *tmem_slot : 0u;
   const WaitCtl wc{abort_flag, a.err, globaltimer_ns() + a.timeout_ns};
+  pdl_wait();  // every global access of this kernel comes after the previous kernel's
 
   auto stage_x = [&](int s) { return stages + s * Cfg::STAGE; };
   auto stage_u = [&](int s) { return stages + s * Cfg::STAGE + Cfg::X_BYTES; };
@@ -643,13 +645,15 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   cfg.blockDim = dim3(320, 1, 1);
   cfg.dynamicSmemBytes = Cfg::SMEM;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (RP > 0) ? C : 1;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   const CUtensorMap& ut = (RP > 0) ? h.ucat_t_map : am.x_map;
   const CUtensorMap& u3 = (RP > 0) ? h.ucat3_map : am.x_map;
   return cudaLaunchKernelEx(&cfg, actquant_kernel<RP, NV>, am.x_map, ut, u3, a);

@@ -114,6 +114,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const __grid_constant__ CUtensorMap bh_map, const GemmArgs a) {
   using Cfg = GemmCfg<RP>;
   extern __shared__ uint8_t smem_raw[];
+  pdl_launch_dependents();
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* oring = smem;                           // SO x (A 16 KB | X 16 KB), 1024-aligned
   uint8_t* pring = oring + SO * OSTAGE;            // SP x packed weights
@@ -188,6 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const WaitCtl wc{abort_flag, a.err, globaltimer_ns() + a.timeout_ns};
+  pdl_wait();  // every global access of this kernel comes after the previous kernel's
 
   if (wid < 4) {
     setmaxnreg_dec<kRegsCtl>();
@@ -519,8 +521,17 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
   const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
   const CUtensorMap& ph = (RP > 0) ? am.ph_map : am.qx_map;
   const CUtensorMap& bh = (RP > 0) ? h.Bh_map : am.qx_map;
-  gemm_kernel<RP><<<grid, kThreads, Cfg::SMEM, s>>>(am.qx_map, h.qw_map, am.ab_map, h.sw32_map, ph, bh, a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<RP>, am.qx_map, h.qw_map, am.ab_map, h.sw32_map, ph, bh, a);
 }
 
 }  // namespace

@@ -64,6 +64,7 @@ __global__ void __launch_bounds__(kThreads4, 1)
                       const Gemm4Args a) {
   using Cfg = Gemm4Cfg<RP>;
   extern __shared__ uint8_t smem_raw[];
+  pdl_launch_dependents();
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* stages = smem;                       // NS4 x (A | B | SF_A | SF_B)
   uint8_t* br = stages + NS4 * STAGE4;          // p_hat | B_hat
@@ -120,6 +121,7 @@ __global__ void __launch_bounds__(kThreads4, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const WaitCtl wc{abort_flag, a.err, globaltimer_ns() + a.timeout_ns};
+  pdl_wait();  // every global access of this kernel comes after the previous kernel's
 
   if (wid == 0) {
     // ------------------------------------------------------------- TMA producer
@@ -330,8 +332,17 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, void*
   const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
   const CUtensorMap& ph = (RP > 0) ? am.ph_map : am.qx4_map;
   const CUtensorMap& bh = (RP > 0) ? h.Bh_map : am.qx4_map;
-  gemm_nvfp4_kernel<RP><<<grid, kThreads4, Cfg::SMEM, s>>>(am.qx4_map, h.qw4_map, ph, bh, a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kThreads4, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemm_nvfp4_kernel<RP>, am.qx4_map, h.qw4_map, ph, bh, a);
 }
 
 }  // namespace

@@ -109,6 +109,14 @@ __device__ __forceinline__ bool mbar_wait_inline(uint64_t* bar, uint32_t parity,
   return wait_loop(bar, parity, c);
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// The layer's kernels are launched with programmatic stream serialization: each lets the next
+// kernel of the stream be scheduled as soon as it starts (its CTAs then set up barriers and
+// tensor memory while this one runs), and waits, before it touches global memory, until the
+// previous kernel has completed and its writes are visible.
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------- fences
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
