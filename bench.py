@@ -260,6 +260,47 @@ def alg_bytes_actquant(M, K, r_pad, G, nvfp4=False):
     return 2 * M * K + M * K // 2 + scales + 2 * M * r_pad + 2 * (2 * K * r_pad) * 2
 
 
+def small_m_latencies(asp, wl, dev, stream, dev_bf16):
+    """The action-expert small-M layers (K = 1024; M 32 and 128; N 1024 and 4096; r 16 and 0), the
+    latency-bound regime: the time of one qwam_asp_linear call in each format, from a CUDA graph of
+    20 calls replayed 10 times, with the inputs resident on the device."""
+    import torch
+    out = {}
+    side = torch.cuda.Stream(dev)
+    for L in wl.action_expert_small_m().layers:
+        if L.M not in (32, 128):
+            continue
+        Xs, Ws = dev_bf16(L.x()), dev_bf16(L.w())
+        Us = torch.from_numpy(L.u()).to(dev) if L.r else None
+        for fmt, fname in ((asp.QWAM_FMT_INT4, "int4"), (asp.QWAM_FMT_NVFP4, "nvfp4")):
+            lin = asp.AspLinear(Ws, Us, L.G, fmt=fmt)
+            Ys = torch.empty((L.M, L.N), dtype=torch.bfloat16, device=dev)
+            side.wait_stream(stream)
+            with torch.cuda.stream(side):
+                for _ in range(3):
+                    lin(Xs, out=Ys, stream=side)
+            side.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                for _ in range(20):
+                    lin(Xs, out=Ys, stream=side)
+            g.replay()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(10):
+                g.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            us = e0.elapsed_time(e1) / 200 * 1e3
+            out["%s_%s" % (fname, L.name)] = {"us_per_layer": round(us, 2),
+                                              "tops": round(2.0 * L.M * L.N * L.K / us / 1e6, 2)}
+            del g
+            lin.close()
+    return {"what": "one qwam_asp_linear call of an action-expert layer (K=1024), CUDA graph of 20 calls",
+            "layers": out}
+
+
 def run_ours(args):
     import torch
     rank, world, local = dist_env()
@@ -454,6 +495,7 @@ def run_ours(args):
                              "roofline": vroof, "layer_roofline_frac": vfrac, "kernels": vk}
         for s_ in vr["sets"]:
             s_[0].close()
+        variants["small_m"] = small_m_latencies(asp, wl, dev, stream, dev_bf16)
 
     if rank != 0:
         return 0
