@@ -48,9 +48,15 @@ def block_hadamard(d: int) -> np.ndarray:
 
 
 def smoothing_factors(xmax: np.ndarray, W: np.ndarray, alpha: float = 0.5) -> np.ndarray:
-    """App. B.1: s_j = max|X_j|^alpha / max|W_j,:|^(1 - alpha) for W [d, d'] (row j = channel j)."""
+    """App. B.1: s_j = max|X_j|^alpha / max|W_j,:|^(1 - alpha) for W [d, d'] (row j = channel j).
+    A channel whose activation or weight maximum is zero carries nothing and is left unsmoothed
+    (s_j = 1): the factor is undefined there and the paper does not say."""
     wmax = np.abs(np.asarray(W, np.float64)).max(axis=1)
-    return np.asarray(xmax, np.float64) ** alpha / wmax ** (1.0 - alpha)
+    xm = np.asarray(xmax, np.float64)
+    ok = (xm > 0) & (wmax > 0)
+    s = np.ones_like(xm)
+    s[ok] = xm[ok] ** alpha / wmax[ok] ** (1.0 - alpha)
+    return s
 
 
 def rotated_gramian(G: np.ndarray, gamma: np.ndarray | None = None) -> np.ndarray:

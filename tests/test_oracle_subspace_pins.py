@@ -71,6 +71,15 @@ def test_smoothing_factor_closed_forms_and_exactness():
     np.testing.assert_allclose(sub.smoothing_factors(xmax, W, 0.5), np.sqrt(xmax / wmax), rtol=1e-14)
     np.testing.assert_allclose(sub.smoothing_factors(xmax, W, 1.0), xmax, rtol=1e-14)
     np.testing.assert_allclose(sub.smoothing_factors(xmax, W, 0.0), 1.0 / wmax, rtol=1e-14)
+    # a channel with a zero maximum is left unsmoothed
+    W0 = W.copy()
+    W0[3] = 0.0
+    xm0 = xmax.copy()
+    xm0[5] = 0.0
+    s0 = sub.smoothing_factors(xm0, W0, 0.5)
+    assert s0[3] == 1.0 and s0[5] == 1.0
+    np.testing.assert_allclose(np.delete(s0, [3, 5]), np.delete(np.sqrt(xm0 / np.abs(W0).max(axis=1).clip(1e-300)), [3, 5]),
+                               rtol=1e-14)
     # Eq. (pair): x~ = H diag(s)^-1 x and W~ = H diag(s) W leave W^T x unchanged
     s = sub.smoothing_factors(xmax, W, 0.5)
     H = sub.block_hadamard(d)
