@@ -231,6 +231,52 @@ qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h
 qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, int group, void* codes,
                                          void* scales, struct CUstream_st* stream);
 
+/* ---- The offline choice of what to protect (Sec. 3.2-3.3; App. A; App. B.1) -----------------
+ * Calibration-time steps that pick U (the paper's V) and which experts carry a branch, from a given
+ * Action Observability Gramian G (the AOG of Sec. 3.1, estimated elsewhere).  None of them needs a
+ * handle.  All matrices are float32, row-major, on the device unless stated otherwise.        */
+
+/* Smoothing factors of App. B.1: s_j = xmax_j^alpha / max_n |W[j, n]|^(1 - alpha) for every input
+ * channel j (row j of W).  xmax [K] (device float32): each channel's calibration maximum |x_j|;
+ * W_bf16 [K, N] device; alpha in [0, 1]; s [K] device float32 output.  A channel whose activation
+ * or weight maximum is zero is left unsmoothed (s_j = 1).  Computed in float64, rounded once.
+ * Asynchronous on `stream`. */
+qwam_status qwam_asp_smoothing_factors(const float* xmax, const void* W_bf16, int K, int N, double alpha, float* s,
+                                       struct CUstream_st* stream);
+
+/* The AOG in the rotated coordinates (Sec. 3.2): Gt = H diag(gamma) G diag(gamma) H, with H the block
+ * Hadamard rotation of Eq. (pair) (normalised Sylvester blocks of size B, the largest power of two
+ * dividing d, at most 1024).  G, Gt, work: [d, d] (work is scratch); gamma [d] or NULL for no
+ * smoothing.  G, Gt and work must be distinct.  d <= 32768.  Asynchronous on `stream`. */
+qwam_status qwam_asp_rotated_gramian(const float* G, const float* gamma, int d, float* Gt, float* work,
+                                     struct CUstream_st* stream);
+
+/* tr(A) of a [d, d] device matrix, accumulated in float64 and returned in *trace (host): the
+ * per-layer term of an expert's action mass mu_E = sum of tr Gt (Sec. 3.3, Eq. (mass)).
+ * Synchronizes `stream`. */
+qwam_status qwam_asp_gramian_trace(const float* A, int d, double* trace, struct CUstream_st* stream);
+
+/* Scratch bytes of qwam_asp_action_subspace for a [d, d] matrix and rank r (1 <= r <= min(d, 96)). */
+qwam_status qwam_asp_subspace_workspace_bytes(int d, int r, size_t* bytes);
+
+/* The action subspace (Sec. 3.2, Eq. (gtilde); App. A): the eigenvectors of the r largest
+ * eigenvalues of the symmetric positive semidefinite Gt [d, d].  V [d, r] receives them as columns
+ * (decreasing eigenvalue, orthonormal; each column's sign is arbitrary) and lambda [r] (device)
+ * the eigenvalues.  Subspace iteration with r + max(8, r/2) vectors (at most 96) for `iters`
+ * steps, then a Rayleigh-Ritz step: the subspace's error falls like (lambda_{p+1}/lambda_r)^iters,
+ * so a spectrum with a gap after the r-th eigenvalue converges in few steps.  work: device scratch
+ * of qwam_asp_subspace_workspace_bytes, 16-byte aligned.  Synchronizes `stream`. */
+qwam_status qwam_asp_action_subspace(const float* Gt, int d, int r, int iters, float* V, float* lambda, void* work,
+                                     struct CUstream_st* stream);
+
+/* Which experts to protect (Sec. 3.3): in decreasing order of action mass per added 16-bit value,
+ * mass[i] / cost[i] (equal ratios: lower index first), each expert whose added values still fit the
+ * budget.  mass[n] >= 0, cost[n] > 0 (the 16-bit values its branches add, r (d + d') per layer),
+ * host arrays; chosen[n] (host) receives the chosen indices in that order and *n_chosen their count.
+ * Host only. */
+qwam_status qwam_asp_select_experts(const double* mass, const double* cost, int n, double budget, int* chosen,
+                                    int* n_chosen);
+
 /* Set the bound of every device wait of this handle's kernels, in seconds (default 2.0). */
 qwam_status qwam_asp_set_timeout(qwam_asp_handle h, double seconds);
 

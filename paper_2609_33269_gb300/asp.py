@@ -38,7 +38,9 @@ EXPORTED = [
     "qwam_asp_shape", "qwam_asp_export", "qwam_asp_destroy", "qwam_status_string",
     "qwam_asp_debug_residual", "qwam_asp_set_timeout", "qwam_asp_debug_wait_timeout",
     "qwam_asp_linear_static", "qwam_asp_pack_weights_nvfp4", "qwam_asp_format", "qwam_asp_export_nvfp4",
-    "qwam_asp_debug_quantize_rows",
+    "qwam_asp_debug_quantize_rows", "qwam_asp_smoothing_factors", "qwam_asp_rotated_gramian",
+    "qwam_asp_gramian_trace", "qwam_asp_subspace_workspace_bytes", "qwam_asp_action_subspace",
+    "qwam_asp_select_experts",
 ]
 
 _lib = None
@@ -78,6 +80,12 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_status_string.restype = ctypes.c_char_p
         lib.qwam_asp_debug_residual.argtypes = [V, I, H, V, V, V]
         lib.qwam_asp_debug_quantize_rows.argtypes = [V, I, I, I, I, V, V, V]
+        lib.qwam_asp_smoothing_factors.argtypes = [V, V, I, I, ctypes.c_double, V, V]
+        lib.qwam_asp_rotated_gramian.argtypes = [V, V, I, V, V, V]
+        lib.qwam_asp_gramian_trace.argtypes = [V, I, V, V]
+        lib.qwam_asp_subspace_workspace_bytes.argtypes = [I, I, V]
+        lib.qwam_asp_action_subspace.argtypes = [V, I, I, I, V, V, V, V]
+        lib.qwam_asp_select_experts.argtypes = [V, V, I, ctypes.c_double, V, V]
         lib.qwam_asp_set_timeout.argtypes = [H, ctypes.c_double]
         lib.qwam_asp_debug_wait_timeout.argtypes = [H, I, V]
         lib.qwam_asp_pack_weights_nvfp4.argtypes = [V, V, I, I, I, V, ctypes.POINTER(H)]
@@ -220,6 +228,46 @@ def qwam_asp_debug_residual(X_bf16, M: int, h: int, act_ws, R, stream=None):
 def qwam_asp_debug_quantize_rows(R, M: int, K: int, fmt: int, group: int, codes, scales, stream=None):
     _check(load().qwam_asp_debug_quantize_rows(_ptr(R), M, K, fmt, group, _ptr(codes), _ptr(scales),
                                                _stream(stream)), "qwam_asp_debug_quantize_rows")
+
+
+def qwam_asp_smoothing_factors(xmax, W_bf16, K: int, N: int, alpha: float, s, stream=None):
+    _check(load().qwam_asp_smoothing_factors(_ptr(xmax), _ptr(W_bf16), K, N, float(alpha), _ptr(s), _stream(stream)),
+           "qwam_asp_smoothing_factors")
+
+
+def qwam_asp_rotated_gramian(G, gamma, d: int, Gt, work, stream=None):
+    _check(load().qwam_asp_rotated_gramian(_ptr(G), None if gamma is None else _ptr(gamma), d, _ptr(Gt), _ptr(work),
+                                           _stream(stream)), "qwam_asp_rotated_gramian")
+
+
+def qwam_asp_gramian_trace(A, d: int, stream=None) -> float:
+    out = ctypes.c_double(0.0)
+    _check(load().qwam_asp_gramian_trace(_ptr(A), d, ctypes.byref(out), _stream(stream)), "qwam_asp_gramian_trace")
+    return out.value
+
+
+def qwam_asp_subspace_workspace_bytes(d: int, r: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check(load().qwam_asp_subspace_workspace_bytes(d, r, ctypes.byref(out)), "qwam_asp_subspace_workspace_bytes")
+    return out.value
+
+
+def qwam_asp_action_subspace(Gt, d: int, r: int, iters: int, V, lam, work, stream=None):
+    _check(load().qwam_asp_action_subspace(_ptr(Gt), d, r, iters, _ptr(V), _ptr(lam), _ptr(work), _stream(stream)),
+           "qwam_asp_action_subspace")
+
+
+def qwam_asp_select_experts(mass, cost, budget: float):
+    """Host-only: the chosen expert indices, in the order chosen (Sec. 3.3)."""
+    import numpy as np
+    m = np.ascontiguousarray(mass, np.float64)
+    c = np.ascontiguousarray(cost, np.float64)
+    n = m.shape[0]
+    chosen = np.zeros(max(n, 1), np.int32)
+    k = ctypes.c_int(0)
+    _check(load().qwam_asp_select_experts(m.ctypes.data, c.ctypes.data, n, float(budget), chosen.ctypes.data,
+                                          ctypes.byref(k)), "qwam_asp_select_experts")
+    return [int(v) for v in chosen[:k.value]]
 
 
 def qwam_asp_set_timeout(h: int, seconds: float):

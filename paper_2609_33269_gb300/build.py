@@ -13,7 +13,7 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libqwam_asp.so")
-SOURCES = ["api.cu", "pack.cu", "actquant.cu", "gemm.cu", "gemm_nvfp4.cu", "static_ws.cu"]
+SOURCES = ["api.cu", "pack.cu", "actquant.cu", "gemm.cu", "gemm_nvfp4.cu", "static_ws.cu", "subspace.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

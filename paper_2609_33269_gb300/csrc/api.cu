@@ -3,6 +3,7 @@
 // device memory.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -320,6 +321,59 @@ qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, 
   return from_cuda_status(qwam::launch_debug_quantize_rows(R, M, K, fmt == QWAM_FMT_NVFP4, group,
                                                            static_cast<uint8_t*>(codes), scales,
                                                            reinterpret_cast<cudaStream_t>(stream)));
+}
+
+qwam_status qwam_asp_smoothing_factors(const float* xmax, const void* W_bf16, int K, int N, double alpha, float* s,
+                                       struct CUstream_st* stream) {
+  if (K <= 0 || N <= 0 || !xmax || !W_bf16 || !s || !(alpha >= 0.0 && alpha <= 1.0)) return QWAM_ERR_INVALID_ARG;
+  return from_cuda_status(qwam::launch_smoothing(xmax, static_cast<const __nv_bfloat16*>(W_bf16), K, N, alpha, s,
+                                                 reinterpret_cast<cudaStream_t>(stream)));
+}
+
+qwam_status qwam_asp_rotated_gramian(const float* G, const float* gamma, int d, float* Gt, float* work,
+                                     struct CUstream_st* stream) {
+  if (d <= 0 || d > 32768 || !G || !Gt || !work || G == Gt || G == work || Gt == work) return QWAM_ERR_INVALID_ARG;
+  return from_cuda_status(qwam::launch_rotated_gramian(G, gamma, d, Gt, work, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+qwam_status qwam_asp_gramian_trace(const float* A, int d, double* trace, struct CUstream_st* stream) {
+  if (d <= 0 || !A || !trace) return QWAM_ERR_INVALID_ARG;
+  return from_cuda_status(qwam::gramian_trace(A, d, trace, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+qwam_status qwam_asp_subspace_workspace_bytes(int d, int r, size_t* bytes) {
+  if (d <= 0 || r <= 0 || r > d || r > qwam::subspace_width(d, r) || !bytes) return QWAM_ERR_INVALID_ARG;
+  *bytes = qwam::subspace_workspace_bytes(d, r);
+  return QWAM_OK;
+}
+
+qwam_status qwam_asp_action_subspace(const float* Gt, int d, int r, int iters, float* V, float* lambda, void* work,
+                                     struct CUstream_st* stream) {
+  if (d <= 0 || r <= 0 || r > d || r > qwam::subspace_width(d, r) || iters < 0 || !Gt || !V || !lambda || !work ||
+      !qwam::aligned16(work))
+    return QWAM_ERR_INVALID_ARG;
+  return from_cuda_status(qwam::action_subspace(Gt, d, r, iters, V, lambda, work, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+qwam_status qwam_asp_select_experts(const double* mass, const double* cost, int n, double budget, int* chosen,
+                                    int* n_chosen) {
+  if (n < 0 || (n > 0 && (!mass || !cost || !chosen)) || !n_chosen) return QWAM_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i)
+    if (!(cost[i] > 0.0) || !(mass[i] >= 0.0)) return QWAM_ERR_INVALID_ARG;
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  // decreasing action mass per added 16-bit value; equal ratios keep the lower index first
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int a, int b) { return mass[a] / cost[a] > mass[b] / cost[b]; });
+  double used = 0.0;
+  int k = 0;
+  for (int i : order)
+    if (used + cost[i] <= budget) {
+      chosen[k++] = i;
+      used += cost[i];
+    }
+  *n_chosen = k;
+  return QWAM_OK;
 }
 
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle hs, void* Y, int y_dtype,

@@ -89,6 +89,15 @@ cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int 
 cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s);
 cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
                                        void* scales, cudaStream_t s);
+// The offline choice of what to protect (subspace.cu).
+int subspace_width(int d, int r);
+size_t subspace_workspace_bytes(int d, int r);
+cudaError_t launch_smoothing(const float* xmax, const __nv_bfloat16* W, int K, int N, double alpha, float* s,
+                             cudaStream_t st);
+cudaError_t launch_rotated_gramian(const float* G, const float* gamma, int d, float* Gt, float* work, cudaStream_t st);
+cudaError_t gramian_trace(const float* A, int d, double* host_out, cudaStream_t st);
+cudaError_t action_subspace(const float* Gt, int d, int r, int iters, float* V_out, float* lambda, void* work,
+                            cudaStream_t st);
 
 }  // namespace qwam
 
