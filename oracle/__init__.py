@@ -74,6 +74,9 @@ def _load():
             lib.qo_e4m3_value.restype = ctypes.c_double
             lib.qo_e4m3_bits_rn.argtypes = [ctypes.c_double]
             lib.qo_e4m3_bits_rn.restype = ctypes.c_uint8
+            lib.qo_pack_f64.argtypes = [P, P, I, I, I, I, P, P, P, P, P]
+            lib.qo_quantize_act_f64.argtypes = [P, P, I, I, I, I, P, P, P, P, P]
+            lib.qo_block_fwht.argtypes = [P, I, I, ctypes.c_long, ctypes.c_long, P, I]
             _lib = lib
     return _lib
 
@@ -138,6 +141,76 @@ def quantize_act(X_bf16_bits, U, G, want_float64=False):
     if want_float64:
         out.update(p=p, Xperp=Xp)
     return out
+
+
+def pack_f64(W, U, G, want_float64=False):
+    """pack() of a float64 weight W [K,N] (the smoothed and rotated W~ of Sec. 2 Eq. (pair))."""
+    W = _c(W, np.float64)
+    K, N = W.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qw = np.empty((N, K), np.int8)
+    sw = np.empty((K // G, N), np.uint16)
+    Bh = np.empty((r, N), np.uint16)
+    Bf = np.empty((r, N), np.float64) if want_float64 else None
+    Wp = np.empty((K, N), np.float64) if want_float64 else None
+    _check(_load().qo_pack_f64(_ptr(W), _ptr(U), K, N, r, G, _ptr(qw), _ptr(sw), _ptr(Bh), _ptr(Bf), _ptr(Wp)),
+           "pack_f64")
+    out = dict(qw=qw, sw=sw, Bh=Bh)
+    if want_float64:
+        out.update(Bf=Bf, Wperp=Wp)
+    return out
+
+
+def quantize_act_f64(X, U, G, want_float64=False):
+    """quantize_act() of float64 activations X [M,K] (the smoothed and rotated x~)."""
+    X = _c(X, np.float64)
+    M, K = X.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qx = np.empty((M, K), np.int8)
+    sx = np.empty((M, K // G), np.float32)
+    ph = np.empty((M, r), np.uint16)
+    p = np.empty((M, r), np.float64) if want_float64 else None
+    Xp = np.empty((M, K), np.float64) if want_float64 else None
+    _check(_load().qo_quantize_act_f64(_ptr(X), _ptr(U), M, K, r, G, _ptr(qx), _ptr(sx), _ptr(ph), _ptr(p), _ptr(Xp)),
+           "quantize_act_f64")
+    out = dict(qx=qx, sx=sx, ph=ph)
+    if want_float64:
+        out.update(p=p, Xperp=Xp)
+    return out
+
+
+def rotate_weights(W_bf16_bits, s=None):
+    """Sec. 2 Eq. (pair), weight side: W~ = H diag(s) W in float64 ([K,N]; H along K by the block
+    fast Walsh-Hadamard transform of App. B.1, in a fixed butterfly order)."""
+    W = bf16_bits_to_f64(W_bf16_bits)
+    K, N = W.shape
+    sc = None if s is None else _c(s, np.float64)
+    _check(_load().qo_block_fwht(_ptr(W), N, K, 1, N, _ptr(sc), 0), "block_fwht")
+    return W
+
+
+def rotate_acts(X_bf16_bits, s=None):
+    """Sec. 2 Eq. (pair), activation side: x~ = H diag(s)^-1 x for every token row, float64 [M,K]."""
+    X = bf16_bits_to_f64(X_bf16_bits)
+    M, K = X.shape
+    sc = None if s is None else _c(s, np.float64)
+    _check(_load().qo_block_fwht(_ptr(X), M, K, K, 1, _ptr(sc), 1), "block_fwht")
+    return X
+
+
+def forward_rotated(X_bf16_bits, W_bf16_bits, s, U, G):
+    """The layer with smoothing and rotation (Eq. (pair)) in front of ASP: x~ and W~ first, then
+    the same pack, activation path and output on them.  U lives in the rotated coordinates."""
+    wts = pack_f64(rotate_weights(W_bf16_bits, s), U, G)
+    act = quantize_act_f64(rotate_acts(X_bf16_bits, s), U, G)
+    return linear(act, wts, G), act, wts
+
+
+def bf16_bits_to_f64(bits):
+    b = _c(bits, np.uint16)
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
 def quantize_residual(R_f32, G):

@@ -20,6 +20,10 @@
  *       x = V(V^T x) + x_perp,  x_perp = (I - VV^T) x,
  *       W^T x ~= (V^T W)^T (V^T x) + Q4(W_perp)^T Q4(x_perp),  W_perp = (I - VV^T) W.
  *   - Table 3: per-group W4A4 costs 4.50 bits per weight at group 32, i.e. a 16-bit weight scale.
+ *   - Sec. 2 Eq. (pair) and App. B.1: smoothing and a block Hadamard rotation in front of the
+ *     quantizer, x~ = H diag(s)^-1 x and W~ = H diag(s) W, H applied by the fast Walsh-Hadamard
+ *     transform in blocks of B (qo_block_fwht); the layer then runs on x~ and W~ (the *_f64 entry
+ *     points take float64 inputs).
  *
  * Row-major notation of this file: X [M,K] holds one token per row, W [K,N] maps K inputs to N
  * outputs (Y = X W is the paper's y = W^T x for every token), U [K,r] is the paper's V.
@@ -32,6 +36,7 @@
  *   R5  codes are taken against the stored (rounded) scale; a zero scale gives zero codes.
  *   R6  the "16-bit" branch is float16: p_hat = RN_f16(x U), B_hat = RN_f16(U^T W).
  *   R7  the branch uses float64 B_f = U^T W for the deflation, B_hat only for the output.
+ *   R8  on float64 activations (the rotated x~) the scale is RN_f32(RN_f64(amax / 7)).
  */
 #include <math.h>
 #include <stdint.h>
@@ -109,8 +114,8 @@ static int nearest_code(double x, double s) {
 /* W_bf16 [K,N] bf16 bits; U [K,r] float32 (orthonormal columns; ignored when r == 0).
  * Outputs: qw [N,K] int8 codes, sw [K/G,N] float16 bits, Bh [r,N] float16 bits,
  *          Bf [r,N] float64 (optional), Wperp [K,N] float64 (optional). */
-int qo_pack(const uint16_t* W_bf16, const float* U, int K, int N, int r, int G, int8_t* qw,
-            uint16_t* sw, uint16_t* Bh, double* Bf_out, double* Wperp_out) {
+static int pack_core(const double* W, const float* U, int K, int N, int r, int G, int8_t* qw, uint16_t* sw,
+                     uint16_t* Bh, double* Bf_out, double* Wperp_out) {
   if (K <= 0 || N <= 0 || r < 0 || r > K || G <= 0 || K % G) return QO_EINVAL;
   int status = QO_OK;
   double* Bf = (double*)calloc((size_t)(r > 0 ? r : 1) * N, sizeof(double));
@@ -125,7 +130,7 @@ int qo_pack(const uint16_t* W_bf16, const float* U, int K, int N, int r, int G, 
   for (int n = 0; n < N; ++n)
     for (int j = 0; j < r; ++j) {
       double acc = 0.0;
-      for (int k = 0; k < K; ++k) acc += (double)U[(size_t)k * r + j] * bf16_value(W_bf16[(size_t)k * N + n]);
+      for (int k = 0; k < K; ++k) acc += (double)U[(size_t)k * r + j] * W[(size_t)k * N + n];
       Bf[(size_t)j * N + n] = acc;
     }
   /* W_perp = (I - U U^T) W = W - U B_f. */
@@ -134,7 +139,7 @@ int qo_pack(const uint16_t* W_bf16, const float* U, int K, int N, int r, int G, 
     for (int n = 0; n < N; ++n) {
       double acc = 0.0;
       for (int j = 0; j < r; ++j) acc += (double)U[(size_t)k * r + j] * Bf[(size_t)j * N + n];
-      Wp[(size_t)k * N + n] = bf16_value(W_bf16[(size_t)k * N + n]) - acc;
+      Wp[(size_t)k * N + n] = W[(size_t)k * N + n] - acc;
     }
   /* Per output channel n and group g of G consecutive inputs: s_w = RN_f16(amax/7), codes. */
   int ng = K / G;
@@ -167,13 +172,30 @@ int qo_pack(const uint16_t* W_bf16, const float* U, int K, int N, int r, int G, 
   return status;
 }
 
+int qo_pack(const uint16_t* W_bf16, const float* U, int K, int N, int r, int G, int8_t* qw,
+            uint16_t* sw, uint16_t* Bh, double* Bf_out, double* Wperp_out) {
+  if (K <= 0 || N <= 0) return QO_EINVAL;
+  double* W = (double*)malloc((size_t)K * N * sizeof(double));
+  if (!W) return QO_EINVAL;
+  for (size_t i = 0; i < (size_t)K * N; ++i) W[i] = bf16_value(W_bf16[i]);
+  int st = pack_core(W, U, K, N, r, G, qw, sw, Bh, Bf_out, Wperp_out);
+  free(W);
+  return st;
+}
+
+/* The same packing of a float64 weight W [K,N] (the smoothed and rotated W~ of Eq. (pair)). */
+int qo_pack_f64(const double* W, const float* U, int K, int N, int r, int G, int8_t* qw, uint16_t* sw,
+                uint16_t* Bh, double* Bf_out, double* Wperp_out) {
+  return pack_core(W, U, K, N, r, G, qw, sw, Bh, Bf_out, Wperp_out);
+}
+
 /* ---- run-time activation path: Eq. (xsplit), then Eq. (quant) per token and group ------- */
 
 /* X_bf16 [M,K] bf16 bits; U [K,r] float32.
  * Outputs: qx [M,K] int8 codes, sx [M,K/G] float32 scales, ph [M,r] float16 bits,
  *          p [M,r] float64 (optional), Xperp [M,K] float64 (optional). */
-int qo_quantize_act(const uint16_t* X_bf16, const float* U, int M, int K, int r, int G, int8_t* qx,
-                    float* sx, uint16_t* ph, double* p_out, double* Xperp_out) {
+static int quantize_act_core(const uint16_t* X_bf16, const double* X_f64, const float* U, int M, int K, int r,
+                             int G, int8_t* qx, float* sx, uint16_t* ph, double* p_out, double* Xperp_out) {
   if (M < 0 || K <= 0 || r < 0 || r > K || G <= 0 || K % G) return QO_EINVAL;
   int status = QO_OK;
   int ng = K / G;
@@ -183,7 +205,7 @@ int qo_quantize_act(const uint16_t* X_bf16, const float* U, int M, int K, int r,
     double* p = (double*)malloc((size_t)(r > 0 ? r : 1) * sizeof(double));
 #pragma omp for schedule(static)
     for (int m = 0; m < M; ++m) {
-      for (int k = 0; k < K; ++k) x[k] = bf16_value(X_bf16[(size_t)m * K + k]);
+      for (int k = 0; k < K; ++k) x[k] = X_bf16 ? bf16_value(X_bf16[(size_t)m * K + k]) : X_f64[(size_t)m * K + k];
       /* protected coordinates p = x U (r values), the V^T x of Eq. (xsplit) */
       for (int j = 0; j < r; ++j) {
         double acc = 0.0;
@@ -219,6 +241,51 @@ int qo_quantize_act(const uint16_t* X_bf16, const float* U, int M, int K, int r,
     free(p);
   }
   return status;
+}
+
+int qo_quantize_act(const uint16_t* X_bf16, const float* U, int M, int K, int r, int G, int8_t* qx,
+                    float* sx, uint16_t* ph, double* p_out, double* Xperp_out) {
+  return quantize_act_core(X_bf16, NULL, U, M, K, r, G, qx, sx, ph, p_out, Xperp_out);
+}
+
+/* The same activation path on float64 activations X [M,K] (the smoothed and rotated x~). */
+int qo_quantize_act_f64(const double* X, const float* U, int M, int K, int r, int G, int8_t* qx, float* sx,
+                        uint16_t* ph, double* p_out, double* Xperp_out) {
+  if (!X && M > 0) return QO_EINVAL;
+  return quantize_act_core(NULL, X, U, M, K, r, G, qx, sx, ph, p_out, Xperp_out);
+}
+
+/* The rotation H of Eq. (pair) applied with the fast Walsh-Hadamard transform, the method the paper
+ * names for it (App. B.1: blocks of B, the largest power of two dividing n, at most 1024).  For
+ * each of `count` vectors of length n (element i of vector v at data[v * vstride + i * estride]):
+ * y_i = x_i * scale[i] (or x_i / scale[i] when divide != 0; no scaling when scale is NULL), then
+ * butterflies (a + b, a - b) at spans 1, 2, 4, ..., B/2 inside each block, then each entry times
+ * 1/sqrt(B).  Every product and sum is one float64 rounding, in this order, in place. */
+int qo_block_fwht(double* data, int count, int n, long vstride, long estride, const double* scale, int divide) {
+  if (count < 0 || n <= 0) return QO_EINVAL;
+  int B = 1;
+  while (n % (2 * B) == 0 && 2 * B <= 1024) B *= 2;
+  const double nrm = 1.0 / sqrt((double)B);
+#pragma omp parallel for schedule(static)
+  for (int v = 0; v < count; ++v) {
+    double* x = data + (long)v * vstride;
+    if (scale)
+      for (int i = 0; i < n; ++i) {
+        const long a = (long)i * estride;
+        x[a] = divide ? x[a] / scale[i] : x[a] * scale[i];
+      }
+    for (int h = 1; h < B; h *= 2)
+      for (int b0 = 0; b0 < n; b0 += B)
+        for (int u0 = 0; u0 < B; u0 += 2 * h)
+          for (int q = 0; q < h; ++q) {
+            const long a = (long)(b0 + u0 + q) * estride, c = (long)(b0 + u0 + q + h) * estride;
+            const double xa = x[a], xc = x[c];
+            x[a] = xa + xc;
+            x[c] = xa - xc;
+          }
+    for (int i = 0; i < n; ++i) x[(long)i * estride] *= nrm;
+  }
+  return QO_OK;
 }
 
 /* The quantizer alone, applied to a given float32 remainder R [M,K] (reading R3 with an exact

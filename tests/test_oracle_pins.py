@@ -174,9 +174,15 @@ def _exact_layer(Xb, Wb, U, G):
     """Eq. (xsplit) + Eq. (asp) + Eq. (quant) in exact rationals, with the stated readings."""
     M, K = Xb.shape
     N = Wb.shape[1]
-    r = U.shape[1]
     X = [[bf16_frac(Xb[m, k]) for k in range(K)] for m in range(M)]
     W = [[bf16_frac(Wb[k, n]) for n in range(N)] for k in range(K)]
+    return _exact_layer_values(X, W, U, G)
+
+
+def _exact_layer_values(X, W, U, G):
+    """_exact_layer on inputs given as lists of exact rationals X [M][K], W [K][N]."""
+    M, K, N = len(X), len(W), len(W[0])
+    r = U.shape[1]
     Uf = [[Fraction(float(U[k, j])) for j in range(r)] for k in range(K)]
     # pack
     Bf = [[sum(Uf[k][j] * W[k][n] for k in range(K)) for n in range(N)] for j in range(r)]
@@ -325,3 +331,110 @@ def test_isotropy_share_of_the_4bit_residual():
     delta = deq - a["Xperp"]
     share = (np.linalg.norm(delta @ U.astype(np.float64)) ** 2) / (np.linalg.norm(delta) ** 2)
     assert 0.5 * r / K <= share <= 2.0 * r / K, share
+
+
+# ---------------------------------------------------------------- smoothing and rotation (Eq. (pair))
+
+def _hadamard_dense(d):
+    """Block-diagonal H from the bit formula H[i, j] = (-1)^popcount(i & j) / sqrt(B) per block of
+    B (the largest power of two dividing d, at most 1024), written out element by element."""
+    b = 1
+    while d % (2 * b) == 0 and 2 * b <= 1024:
+        b *= 2
+    H = np.zeros((d, d))
+    for i in range(d):
+        for j in range(d):
+            if i // b == j // b:
+                H[i, j] = (-1) ** bin((i % b) & (j % b)).count("1") / math.sqrt(b)
+    return H
+
+
+@pytest.mark.parametrize("K", [64, 96, 640])
+def test_rotation_is_the_dense_block_hadamard_and_keeps_the_product(K):
+    M, N = 5, 12
+    Xb = wl.activations(M, K, seed=8, layer_id=K, dist="outlier", n_outlier=3)
+    Wb = wl.weight(K, N, seed=8, layer_id=K)
+    s = np.exp(np.random.default_rng(K).uniform(-2, 2, K))
+    X = wl.bf16_bits_to_f32(Xb).astype(np.float64)
+    W = wl.bf16_bits_to_f32(Wb).astype(np.float64)
+    H = _hadamard_dense(K)
+    Wt = oracle.rotate_weights(Wb, s)
+    Xt = oracle.rotate_acts(Xb, s)
+    np.testing.assert_allclose(Wt, H @ (s[:, None] * W), rtol=0, atol=1e-13 * np.abs(Wt).max())
+    np.testing.assert_allclose(Xt, (X / s[None, :]) @ H.T, rtol=0, atol=1e-13 * np.abs(Xt).max())
+    # Eq. (pair): W~^T x~ = W^T diag(s) H^T H diag(s)^-1 x = W^T x
+    ref = X @ W
+    np.testing.assert_allclose(Xt @ Wt, ref, rtol=0, atol=1e-12 * np.abs(ref).max())
+    # without smoothing factors the rotation alone; H is an involution: rotating twice is identity
+    np.testing.assert_allclose(oracle.rotate_weights(Wb), H @ W, rtol=0, atol=1e-13 * np.abs(W).max())
+    Xb2 = wl.f32_to_bf16_bits(np.eye(K, dtype=np.float32)[:3])
+    np.testing.assert_allclose(oracle.rotate_acts(Xb2), H[:3], rtol=0, atol=1e-15)
+
+
+def test_float64_entry_points_reduce_to_the_bf16_ones():
+    """pack_f64 / quantize_act_f64 on the float64 values of bf16 inputs are the bf16 entry points,
+    bit for bit (the bf16 ones are pinned above by exact rational arithmetic)."""
+    M, K, N, r, G = 8, 256, 32, 4, 64
+    Xb = wl.activations(M, K, seed=9, layer_id=2, dist="outlier", n_outlier=3)
+    Wb = wl.weight(K, N, seed=9, layer_id=2)
+    U = wl.basis(K, r, seed=9, layer_id=2)
+    X = wl.bf16_bits_to_f32(Xb).astype(np.float64)
+    W = wl.bf16_bits_to_f32(Wb).astype(np.float64)
+    a, a64 = oracle.quantize_act(Xb, U, G, True), oracle.quantize_act_f64(X, U, G, True)
+    w, w64 = oracle.pack(Wb, U, G, True), oracle.pack_f64(W, U, G, True)
+    for k in a:
+        np.testing.assert_array_equal(a[k], a64[k])
+    for k in w:
+        np.testing.assert_array_equal(w[k], w64[k])
+
+
+@pytest.mark.parametrize("r", [0, 2])
+def test_rotated_layer_matches_exact_rational_arithmetic(r):
+    """The layer on x~ and W~ (float64 values that are not bf16) against exact rationals."""
+    M, K, N, G = 3, 64, 4, 32
+    Xb = wl.activations(M, K, seed=10, layer_id=r, dist="outlier", n_outlier=2)
+    Wb = wl.weight(K, N, seed=10, layer_id=r)
+    U = wl.basis(K, r, seed=10, layer_id=r)
+    s = np.exp(np.random.default_rng(r).uniform(-1, 1, K))
+    Y, a, w = oracle.forward_rotated(Xb, Wb, s, U, G)
+    Xt, Wt = oracle.rotate_acts(Xb, s), oracle.rotate_weights(Wb, s)
+    ex = _exact_layer_values([[Fraction(float(v)) for v in row] for row in Xt],
+                             [[Fraction(float(v)) for v in row] for row in Wt], U, G)
+    assert w["qw"].tolist() == ex["qw"]
+    assert [[f16_frac(b) for b in row] for row in w["sw"]] == ex["sw"]
+    assert [[f16_frac(b) for b in row] for row in w["Bh"]] == ex["Bh"]
+    assert a["qx"].tolist() == ex["qx"]
+    assert [[Fraction(float(v)) for v in row] for row in a["sx"]] == ex["sx"]
+    assert [[f16_frac(b) for b in row] for row in a["ph"]] == ex["ph"]
+    Yex = np.array([[float(v) for v in row] for row in ex["Y"]])
+    np.testing.assert_allclose(Y, Yex, rtol=1e-12, atol=1e-12 * np.abs(Yex).max())
+
+
+def test_rotation_with_full_rank_protection_is_the_plain_product():
+    """r = K in the rotated coordinates: the 4-bit remainder vanishes and the output is X W up to
+    the float16 branch rounding, whatever the smoothing factors."""
+    M, K, N, G = 16, 128, 32, 64
+    Xb = wl.activations(M, K, seed=12, layer_id=1, dist="outlier", n_outlier=4)
+    Wb = wl.weight(K, N, seed=12, layer_id=1)
+    U = wl.basis(K, K, seed=12, layer_id=1)
+    s = np.exp(np.random.default_rng(3).uniform(-1, 1, K))
+    Y, _, _ = oracle.forward_rotated(Xb, Wb, s, U, G)
+    ref = wl.bf16_bits_to_f32(Xb).astype(np.float64) @ wl.bf16_bits_to_f32(Wb).astype(np.float64)
+    err = np.abs(Y - ref).max(axis=1) / np.abs(ref).max(axis=1)
+    assert err.max() <= 1e-3, err.max()
+
+
+def test_rotation_spreads_an_outlier_channel():
+    """Sec. 2: the rotation spreads one large channel over its Hadamard block: every rotated entry
+    is at most ||x||_1 / sqrt(B) (each is a +-1/sqrt(B) combination of the block), and the norm is
+    kept (H is orthogonal)."""
+    K = 256
+    X = np.zeros((1, K), np.float32)
+    X[0, 5] = 64.0
+    X[0, 6:] = np.random.default_rng(1).uniform(-0.5, 0.5, K - 6).astype(np.float32)
+    Xb = wl.f32_to_bf16_bits(X)
+    Xd = wl.bf16_bits_to_f32(Xb).astype(np.float64)
+    Xt = oracle.rotate_acts(Xb)
+    assert np.abs(Xt).max() <= np.abs(Xd).sum() / math.sqrt(K) * (1 + 1e-15)
+    assert np.abs(Xt).max() < 64.0 / 4
+    np.testing.assert_allclose(np.linalg.norm(Xt), np.linalg.norm(Xd), rtol=1e-14)
