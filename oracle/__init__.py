@@ -64,6 +64,8 @@ def _load():
             lib.qo_nearest_code.restype = ctypes.c_int
             lib.qo_pack_nvfp4.argtypes = [P, P, I, I, I, P, P, P, P]
             lib.qo_quantize_act_nvfp4.argtypes = [P, P, I, I, I, P, P, P]
+            lib.qo_pack_nvfp4_f64.argtypes = [P, P, I, I, I, P, P, P, P]
+            lib.qo_quantize_act_nvfp4_f64.argtypes = [P, P, I, I, I, P, P, P]
             lib.qo_quantize_residual_nvfp4_f32.argtypes = [P, I, I, P, P]
             lib.qo_linear_nvfp4.argtypes = [P, P, P, P, P, ctypes.c_float, P, I, I, I, I, P]
             lib.qo_e2m1_value.argtypes = [I]
@@ -181,6 +183,15 @@ def quantize_act_f64(X, U, G, want_float64=False):
     return out
 
 
+def fwht_cols(A, s=None):
+    """H diag(s) A for a float64 A [K,n] (the transform of rotate_weights on any float64 input)."""
+    A = np.array(A, np.float64, order="C", copy=True)
+    K, n = A.shape
+    sc = None if s is None else _c(s, np.float64)
+    _check(_load().qo_block_fwht(_ptr(A), n, K, 1, n, _ptr(sc), 0), "block_fwht")
+    return A
+
+
 def rotate_weights(W_bf16_bits, s=None):
     """Sec. 2 Eq. (pair), weight side: W~ = H diag(s) W in float64 ([K,N]; H along K by the block
     fast Walsh-Hadamard transform of App. B.1, in a fixed butterfly order)."""
@@ -274,6 +285,42 @@ def nearest_code(x: float, s: float) -> int:
 # ---- NVFP4 variant (App. B.1) ----------------------------------------------------------------
 
 FP4_BLOCK = 16
+
+
+def pack_nvfp4_f64(W, U):
+    """pack_nvfp4() of a float64 weight W [K,N] (the smoothed and rotated W~ of Eq. (pair))."""
+    W = _c(W, np.float64)
+    K, N = W.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qw = np.empty((N, K), np.uint8)
+    sfw = np.empty((N, K // FP4_BLOCK), np.uint8)
+    sg = ctypes.c_float(0.0)
+    Bh = np.empty((r, N), np.uint16)
+    _check(_load().qo_pack_nvfp4_f64(_ptr(W), _ptr(U), K, N, r, _ptr(qw), _ptr(sfw), ctypes.byref(sg), _ptr(Bh)),
+           "pack_nvfp4_f64")
+    return dict(qw=qw, sfw=sfw, sg=np.float32(sg.value), Bh=Bh)
+
+
+def quantize_act_nvfp4_f64(X, U):
+    """quantize_act_nvfp4() of float64 activations X [M,K] (the smoothed and rotated x~)."""
+    X = _c(X, np.float64)
+    M, K = X.shape
+    U = _c(U, np.float32).reshape(K, -1)
+    r = U.shape[1]
+    qx = np.empty((M, K), np.uint8)
+    sfx = np.empty((M, K // FP4_BLOCK), np.uint8)
+    ph = np.empty((M, r), np.uint16)
+    _check(_load().qo_quantize_act_nvfp4_f64(_ptr(X), _ptr(U), M, K, r, _ptr(qx), _ptr(sfx), _ptr(ph)),
+           "quantize_act_nvfp4_f64")
+    return dict(qx=qx, sfx=sfx, ph=ph)
+
+
+def forward_rotated_nvfp4(X_bf16_bits, W_bf16_bits, s, U):
+    """The NVFP4 layer on x~ and W~ (Eq. (pair)).  Returns (Y, act, wts)."""
+    wts = pack_nvfp4_f64(rotate_weights(W_bf16_bits, s), U)
+    act = quantize_act_nvfp4_f64(rotate_acts(X_bf16_bits, s), U)
+    return linear_nvfp4(act, wts), act, wts
 
 
 def pack_nvfp4(W_bf16_bits, U):

@@ -461,8 +461,8 @@ static int e2m1_code_rn(double x) {
 
 /* Offline packing of the NVFP4 variant: W_perp as in qo_pack, then reading N4.
  * Outputs: qw [N,K] E2M1 codes (one per byte), sfw [N,K/16] E4M3 bits, *sg, Bh [r,N]. */
-int qo_pack_nvfp4(const uint16_t* W_bf16, const float* U, int K, int N, int r, uint8_t* qw, uint8_t* sfw,
-                  float* sg_out, uint16_t* Bh) {
+static int pack_nvfp4_core(const double* W, const float* U, int K, int N, int r, uint8_t* qw, uint8_t* sfw,
+                           float* sg_out, uint16_t* Bh) {
   if (K <= 0 || N <= 0 || r < 0 || r > K || K % QO_FP4_BLOCK) return QO_EINVAL;
   int status = QO_OK;
   double* Bf = (double*)calloc((size_t)(r > 0 ? r : 1) * N, sizeof(double));
@@ -476,7 +476,7 @@ int qo_pack_nvfp4(const uint16_t* W_bf16, const float* U, int K, int N, int r, u
   for (int n = 0; n < N; ++n)
     for (int j = 0; j < r; ++j) {
       double acc = 0.0;
-      for (int k = 0; k < K; ++k) acc += (double)U[(size_t)k * r + j] * bf16_value(W_bf16[(size_t)k * N + n]);
+      for (int k = 0; k < K; ++k) acc += (double)U[(size_t)k * r + j] * W[(size_t)k * N + n];
       Bf[(size_t)j * N + n] = acc;
     }
 #pragma omp parallel for schedule(static)
@@ -484,7 +484,7 @@ int qo_pack_nvfp4(const uint16_t* W_bf16, const float* U, int K, int N, int r, u
     for (int n = 0; n < N; ++n) {
       double acc = 0.0;
       for (int j = 0; j < r; ++j) acc += (double)U[(size_t)k * r + j] * Bf[(size_t)j * N + n];
-      Wp[(size_t)k * N + n] = bf16_value(W_bf16[(size_t)k * N + n]) - acc;
+      Wp[(size_t)k * N + n] = W[(size_t)k * N + n] - acc;
     }
   double amax = 0.0;
   for (size_t i = 0; i < (size_t)K * N; ++i)
@@ -513,6 +513,24 @@ int qo_pack_nvfp4(const uint16_t* W_bf16, const float* U, int K, int N, int r, u
   return status;
 }
 
+int qo_pack_nvfp4(const uint16_t* W_bf16, const float* U, int K, int N, int r, uint8_t* qw, uint8_t* sfw,
+                  float* sg_out, uint16_t* Bh) {
+  if (K <= 0 || N <= 0) return QO_EINVAL;
+  double* W = (double*)malloc((size_t)K * N * sizeof(double));
+  if (!W) return QO_EINVAL;
+  for (size_t i = 0; i < (size_t)K * N; ++i) W[i] = bf16_value(W_bf16[i]);
+  const int st = pack_nvfp4_core(W, U, K, N, r, qw, sfw, sg_out, Bh);
+  free(W);
+  return st;
+}
+
+/* The NVFP4 pack of a float64 weight (the smoothed and rotated W~). */
+int qo_pack_nvfp4_f64(const double* W, const float* U, int K, int N, int r, uint8_t* qw, uint8_t* sfw,
+                      float* sg_out, uint16_t* Bh) {
+  if (!W) return QO_EINVAL;
+  return pack_nvfp4_core(W, U, K, N, r, qw, sfw, sg_out, Bh);
+}
+
 /* Reading N3 on one float32 remainder row segment of 16 entries. */
 static void quantize_block_nvfp4(const float* x, uint8_t* q, uint8_t* sf) {
   float amax = 0.0f;
@@ -535,8 +553,8 @@ static void quantize_block_nvfp4(const float* x, uint8_t* q, uint8_t* sf) {
 /* Run-time activation path of the NVFP4 variant: Eq. (xsplit) as in qo_quantize_act, with the
  * remainder rounded to float32 (the precision in which the GPU forms it), then reading N3.
  * Outputs: qx [M,K] E2M1 codes, sfx [M,K/16] E4M3 bits, ph [M,r] float16 bits. */
-int qo_quantize_act_nvfp4(const uint16_t* X_bf16, const float* U, int M, int K, int r, uint8_t* qx,
-                          uint8_t* sfx, uint16_t* ph) {
+static int quantize_act_nvfp4_core(const uint16_t* X_bf16, const double* X_f64, const float* U, int M, int K, int r,
+                                   uint8_t* qx, uint8_t* sfx, uint16_t* ph) {
   if (M < 0 || K <= 0 || r < 0 || r > K || K % QO_FP4_BLOCK) return QO_EINVAL;
   int status = QO_OK;
   const int nb = K / QO_FP4_BLOCK;
@@ -547,7 +565,7 @@ int qo_quantize_act_nvfp4(const uint16_t* X_bf16, const float* U, int M, int K, 
     double* p = (double*)malloc((size_t)(r > 0 ? r : 1) * sizeof(double));
 #pragma omp for schedule(static)
     for (int m = 0; m < M; ++m) {
-      for (int k = 0; k < K; ++k) x[k] = bf16_value(X_bf16[(size_t)m * K + k]);
+      for (int k = 0; k < K; ++k) x[k] = X_bf16 ? bf16_value(X_bf16[(size_t)m * K + k]) : X_f64[(size_t)m * K + k];
       for (int j = 0; j < r; ++j) {
         double acc = 0.0;
         for (int k = 0; k < K; ++k) acc += x[k] * (double)U[(size_t)k * r + j];
@@ -570,6 +588,18 @@ int qo_quantize_act_nvfp4(const uint16_t* X_bf16, const float* U, int M, int K, 
     free(p);
   }
   return status;
+}
+
+int qo_quantize_act_nvfp4(const uint16_t* X_bf16, const float* U, int M, int K, int r, uint8_t* qx,
+                          uint8_t* sfx, uint16_t* ph) {
+  return quantize_act_nvfp4_core(X_bf16, NULL, U, M, K, r, qx, sfx, ph);
+}
+
+/* The NVFP4 activation path on float64 activations (the smoothed and rotated x~). */
+int qo_quantize_act_nvfp4_f64(const double* X, const float* U, int M, int K, int r, uint8_t* qx, uint8_t* sfx,
+                              uint16_t* ph) {
+  if (!X && M > 0) return QO_EINVAL;
+  return quantize_act_nvfp4_core(NULL, X, U, M, K, r, qx, sfx, ph);
 }
 
 /* Reading N3 alone on a given float32 remainder R [M,K] -> qx [M,K], sfx [M,K/16]. */

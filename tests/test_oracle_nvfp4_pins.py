@@ -202,3 +202,55 @@ def test_nvfp4_layer_is_a_4_bit_approximation_of_xw():
     e0 = (np.abs(Y0 - exact).max(axis=1) / np.abs(exact).max(axis=1)).mean()
     e1 = (np.abs(Y1 - exact).max(axis=1) / np.abs(exact).max(axis=1)).mean()
     assert e0 < 0.2 and e1 < 0.2
+
+
+# ---- smoothing and rotation in front of the NVFP4 layer (Eq. (pair)) --------------------------
+
+def test_float64_entry_points_reduce_to_the_bf16_ones():
+    M, K, N, r = 9, 256, 24, 4
+    X = wl.activations(M, K, seed=51, layer_id=4, dist="outlier", n_outlier=3)
+    W = wl.weight(K, N, seed=51, layer_id=4)
+    U = wl.basis(K, r, seed=51, layer_id=4)
+    a, a64 = oracle.quantize_act_nvfp4(X, U), oracle.quantize_act_nvfp4_f64(oracle.bf16_bits_to_f64(X), U)
+    w, w64 = oracle.pack_nvfp4(W, U), oracle.pack_nvfp4_f64(oracle.bf16_bits_to_f64(W), U)
+    for k in a:
+        np.testing.assert_array_equal(a[k], a64[k])
+    for k in w:
+        np.testing.assert_array_equal(w[k], w64[k])
+
+
+@pytest.mark.parametrize("r", [0, 5])
+def test_rotated_layer_equals_matrix_product_of_dequantized_operands(r):
+    """On x~ and W~ the layer is still sg * deq(qx) deq(qw)^T + p_hat B_hat, and the codes of W~
+    follow reading N4 (brute force, r = 0)."""
+    M, K, N = 5, 256, 8
+    X = wl.activations(M, K, seed=61, layer_id=r, dist="outlier", n_outlier=3)
+    W = wl.weight(K, N, seed=61, layer_id=r)
+    U = wl.basis(K, r, seed=61, layer_id=r) if r else np.zeros((K, 0), np.float32)
+    s = np.exp(np.random.default_rng(r).uniform(-1, 1, K))
+    Y, act, wts = oracle.forward_rotated_nvfp4(X, W, s, U)
+    ref = float(wts["sg"]) * (_deq(act["qx"], act["sfx"]) @ _deq(wts["qw"], wts["sfw"]).T)
+    if r:
+        ref = ref + _f16(act["ph"]) @ _f16(wts["Bh"])
+    np.testing.assert_allclose(Y, ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max())
+    if r == 0:
+        Wt = oracle.rotate_weights(W, s)
+        sg = np.float32(np.abs(Wt).max() / (6.0 * 448.0))
+        assert wts["sg"] == sg
+        for n in range(N):
+            for b in range(K // 16):
+                blk = Wt[16 * b:16 * b + 16, n]
+                s_bits = nearest_even(np.abs(blk).max() / (6.0 * float(sg)), E4M3_POS)[0]
+                assert wts["sfw"][n, b] == s_bits
+
+
+def test_rotated_full_rank_protection_gives_the_16_bit_product():
+    M, K, N = 6, 256, 12
+    X = wl.activations(M, K, seed=71, layer_id=2)
+    W = wl.weight(K, N, seed=71, layer_id=2)
+    U = wl.basis(K, K, seed=71, layer_id=2)
+    s = np.exp(np.random.default_rng(5).uniform(-1, 1, K))
+    Y, _, _ = oracle.forward_rotated_nvfp4(X, W, s, U)
+    exact = wl.bf16_bits_to_f32(X).astype(np.float64) @ wl.bf16_bits_to_f32(W).astype(np.float64)
+    err = np.abs(Y - exact).max(axis=1) / np.abs(exact).max(axis=1)
+    assert err.max() <= 1e-3
