@@ -178,6 +178,38 @@ enum { QWAM_FMT_INT4 = 0, QWAM_FMT_NVFP4 = 1 };
 qwam_status qwam_asp_pack_weights_nvfp4(const void* W_bf16, const float* U, int K, int N, int r,
                                         struct CUstream_st* stream, qwam_asp_handle* out);
 
+/* ---- Smoothing and block Hadamard rotation in front of the layer (Sec. 2 Eq. (pair); App. B.1)
+ * The paper quantizes in rotated coordinates: with per-channel smoothing factors s (App. B.1:
+ * s_j = max|X_j|^alpha / max|W_j,:|^(1-alpha), see qwam_asp_smoothing_factors) and the block
+ * Hadamard matrix H (block-diagonal, each block the Sylvester Hadamard matrix of size B divided by
+ * sqrt(B), B the largest power of two dividing K, at most 1024; H is symmetric and orthogonal),
+ *   x~ = H diag(s)^-1 x,   W~ = H diag(s) W,   so that W~^T x~ = W^T x,
+ * and ASP runs on x~ and W~ with a basis U given in the rotated coordinates (for instance the one
+ * qwam_asp_action_subspace returns for the rotated Gramian).
+ *
+ * These two calls pack W~ (formed in float64 on the device: W times s_k, the fast Walsh-Hadamard
+ * butterflies at spans 1, 2, ..., B/2 inside each block, then times 1/sqrt(B); every operation one
+ * float64 rounding) exactly as qwam_asp_pack_weights / qwam_asp_pack_weights_nvfp4 pack a weight,
+ * against U.  The handle's activation calls (qwam_asp_quantize_act, qwam_asp_linear,
+ * qwam_asp_linear_static, qwam_asp_debug_residual) then take X in the ORIGINAL coordinates and
+ * rotate it at run time: the projection p = x~ U is computed as x (diag(s)^-1 H U), the remainder
+ * as H diag(s)^-1 (x - diag(s) H U p) = x~ - U p in float32 (the fast Walsh-Hadamard transform,
+ * float32), and that is quantized.  With r > 0 the activation workspace also holds the float32
+ * remainder before the rotation (M * K * 4 more bytes; qwam_asp_act_workspace_bytes includes
+ * them).  qwam_asp_debug_residual writes the rotated remainder x~_perp.
+ *   W_bf16, U, K, N, r, group, stream, out: as for qwam_asp_pack_weights (or _nvfp4), and
+ *     K % 256 == 0 (QWAM_ERR_INVALID_ARG otherwise).
+ *   s : device float32 [K], 16-byte aligned, the smoothing factors; NULL for the rotation alone.
+ *       A factor that is not a positive finite number gives QWAM_ERR_RANGE.
+ * Synchronizes `stream` before returning; the temporary float64 W~ (K * N * 8 bytes) is freed. */
+qwam_status qwam_asp_pack_weights_rotated(const void* W_bf16, const float* s, const float* U, int K, int N, int r,
+                                          int group, struct CUstream_st* stream, qwam_asp_handle* out);
+qwam_status qwam_asp_pack_weights_nvfp4_rotated(const void* W_bf16, const float* s, const float* U, int K, int N,
+                                                int r, struct CUstream_st* stream, qwam_asp_handle* out);
+
+/* The Hadamard block B of a rotated handle, 0 for a handle without rotation. */
+qwam_status qwam_asp_rotation(qwam_asp_handle h, int* hadamard_block);
+
 /* The handle's format: QWAM_FMT_INT4 or QWAM_FMT_NVFP4. */
 qwam_status qwam_asp_format(qwam_asp_handle h, int* format);
 

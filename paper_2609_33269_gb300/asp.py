@@ -40,7 +40,8 @@ EXPORTED = [
     "qwam_asp_linear_static", "qwam_asp_pack_weights_nvfp4", "qwam_asp_format", "qwam_asp_export_nvfp4",
     "qwam_asp_debug_quantize_rows", "qwam_asp_smoothing_factors", "qwam_asp_rotated_gramian",
     "qwam_asp_gramian_trace", "qwam_asp_subspace_workspace_bytes", "qwam_asp_action_subspace",
-    "qwam_asp_select_experts",
+    "qwam_asp_select_experts", "qwam_asp_pack_weights_rotated", "qwam_asp_pack_weights_nvfp4_rotated",
+    "qwam_asp_rotation",
 ]
 
 _lib = None
@@ -90,6 +91,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_debug_wait_timeout.argtypes = [H, I, V]
         lib.qwam_asp_pack_weights_nvfp4.argtypes = [V, V, I, I, I, V, ctypes.POINTER(H)]
         lib.qwam_asp_format.argtypes = [H, ctypes.POINTER(I)]
+        lib.qwam_asp_pack_weights_rotated.argtypes = [V, V, V, I, I, I, I, V, ctypes.POINTER(H)]
+        lib.qwam_asp_pack_weights_nvfp4_rotated.argtypes = [V, V, V, I, I, I, V, ctypes.POINTER(H)]
+        lib.qwam_asp_rotation.argtypes = [H, ctypes.POINTER(I)]
         lib.qwam_asp_export_nvfp4.argtypes = [H, V, V, ctypes.POINTER(ctypes.c_float), V]
         for name in EXPORTED:
             if name != "qwam_status_string":
@@ -134,6 +138,26 @@ def qwam_asp_pack_weights_nvfp4(W_bf16, U, K: int, N: int, r: int, stream=None) 
     _check(load().qwam_asp_pack_weights_nvfp4(_ptr(W_bf16), _ptr(U), K, N, r, _stream(stream), ctypes.byref(h)),
            "qwam_asp_pack_weights_nvfp4")
     return h.value
+
+
+def qwam_asp_pack_weights_rotated(W_bf16, s, U, K: int, N: int, r: int, group: int, stream=None) -> int:
+    h = ctypes.c_void_p()
+    _check(load().qwam_asp_pack_weights_rotated(_ptr(W_bf16), _ptr(s), _ptr(U), K, N, r, group, _stream(stream),
+                                                ctypes.byref(h)), "qwam_asp_pack_weights_rotated")
+    return h.value
+
+
+def qwam_asp_pack_weights_nvfp4_rotated(W_bf16, s, U, K: int, N: int, r: int, stream=None) -> int:
+    h = ctypes.c_void_p()
+    _check(load().qwam_asp_pack_weights_nvfp4_rotated(_ptr(W_bf16), _ptr(s), _ptr(U), K, N, r, _stream(stream),
+                                                      ctypes.byref(h)), "qwam_asp_pack_weights_nvfp4_rotated")
+    return h.value
+
+
+def qwam_asp_rotation(h: int) -> int:
+    b = ctypes.c_int()
+    _check(load().qwam_asp_rotation(h, ctypes.byref(b)), "qwam_asp_rotation")
+    return b.value
 
 
 def qwam_asp_format(h: int) -> int:
@@ -284,9 +308,11 @@ class AspLinear:
     """One packed ASP layer plus a reusable activation workspace on the current device."""
 
     def __init__(self, W_bf16: torch.Tensor, U: torch.Tensor | None, group: int = 64, stream=None,
-                 fmt: int = QWAM_FMT_INT4):
+                 fmt: int = QWAM_FMT_INT4, rotate: bool = False, s: torch.Tensor | None = None):
         """fmt QWAM_FMT_INT4 (group 32 or 64) or QWAM_FMT_NVFP4 (App. B.1's Blackwell format;
-        `group` is then ignored: the block is 16)."""
+        `group` is then ignored: the block is 16).  rotate=True packs W~ = H diag(s) W (Sec. 2
+        Eq. (pair); s float32 [K] smoothing factors or None) and rotates X at run time; U is then
+        the basis in the rotated coordinates."""
         assert W_bf16.is_cuda and W_bf16.dtype == torch.bfloat16 and W_bf16.is_contiguous()
         K, N = W_bf16.shape
         r = 0 if U is None else U.shape[1]
@@ -295,7 +321,14 @@ class AspLinear:
         self.fmt = fmt
         self.K, self.N, self.r = K, N, r
         self.group = 16 if fmt == QWAM_FMT_NVFP4 else group
-        if fmt == QWAM_FMT_NVFP4:
+        if s is not None:
+            assert rotate and s.is_cuda and s.dtype == torch.float32 and s.is_contiguous() and s.numel() == K
+        self.rotate = rotate
+        if rotate and fmt == QWAM_FMT_NVFP4:
+            self.h = qwam_asp_pack_weights_nvfp4_rotated(W_bf16, s, U if r > 0 else None, K, N, r, stream)
+        elif rotate:
+            self.h = qwam_asp_pack_weights_rotated(W_bf16, s, U if r > 0 else None, K, N, r, group, stream)
+        elif fmt == QWAM_FMT_NVFP4:
             self.h = qwam_asp_pack_weights_nvfp4(W_bf16, U if r > 0 else None, K, N, r, stream)
         else:
             self.h = qwam_asp_pack_weights(W_bf16, U if r > 0 else None, K, N, r, group, stream)

@@ -43,6 +43,7 @@ struct ActArgs {
   float2* ab;       // [K/G, M_pad]: (alpha, beta)
   __half* phat;     // [M, RP]
   float* dump;      // optional [M, K]
+  int resid_only;   // rotated layer: write the remainder to dump and stop (the rotation kernel quantizes)
   int* err;
   uint64_t timeout_ns;
 };
@@ -523,6 +524,7 @@ __global__ void __launch_bounds__(320, 1)
         float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + kc);
 #pragma unroll
         for (int i = 0; i < kChunk / 4; ++i) d[i] = make_float4(xp[4 * i], xp[4 * i + 1], xp[4 * i + 2], xp[4 * i + 3]);
+        if (a.resid_only) continue;
       }
       if constexpr (NV) {
         uint32_t w[8];
@@ -602,6 +604,194 @@ __global__ void __launch_bounds__(128) debug_quantize_kernel(const float* R, int
   }
 }
 
+// ---- run-time smoothing and block Hadamard rotation (Sec. 2 Eq. (pair); App. B.1) ----------
+//
+//   x~_perp = H diag(s)^-1 v,  v = x (r = 0) or v = x - diag(s) H U p (r > 0, from kernel (a))
+//
+// then the same quantizers as kernel (a).  One warp per token row walks K in Hadamard blocks of
+// B = 256 NSUB channels; lane l holds channels 256 c + 8 l .. + 7 of sub-block c.  The fast
+// Walsh-Hadamard butterflies run at spans 1, 2, 4 inside a lane, 8 .. 128 across lanes
+// (shuffles) and 256, 512 across the lane's sub-blocks, then every value is scaled by
+// RN_f32(1/sqrt(B)).  A quantization group (32 or 64 channels) is 4 or 8 neighbouring lanes, an
+// NVFP4 block (16) two.
+struct RotArgs {
+  int M, K, G, M_pad;
+  float nrm;
+  const float* inv_s;
+  uint8_t* codes;
+  uint8_t* sf;
+  float* scales;
+  float2* ab;
+  float* dump;
+};
+
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float* v) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int t = 0; t < 4; ++t) {
+    v[2 * t] = __uint_as_float(w[t] << 16);
+    v[2 * t + 1] = __uint_as_float(w[t] & 0xFFFF0000u);
+  }
+}
+__device__ __forceinline__ void load8(const float* p, float* v) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0], b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+// The lane's 8 values of an NVFP4 block half: one word of E2M1 codes (low nibble first), with the
+// same bracketed fast path and exact fallback as quantize_block_nvfp4.
+__device__ __forceinline__ uint32_t codes8_nvfp4(const float* x, float sc, float r) {
+  constexpr float kDn = 1.0f - 1.0f / 524288.0f, kUp = 1.0f + 1.0f / 524288.0f;
+  uint32_t w = 0u;
+  bool near_mid = false;
+#pragma unroll
+  for (int i = 0; i < 8; i += 2) {
+    const float q0 = x[i] * r, q1 = x[i + 1] * r;
+    const uint32_t lo = cvt_e2m1x2(q0 * kDn, q1 * kDn), hi = cvt_e2m1x2(q0 * kUp, q1 * kUp);
+    near_mid |= lo != hi;
+    w |= lo << (4 * i);
+  }
+  if (near_mid) {
+    w = 0u;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) w |= cvt_e2m1(sc > 0.0f ? __fdiv_rn(x[i], sc) : 0.0f) << (4 * i);
+  }
+  const uint32_t nz = ((w & 0x77777777u) + 0x77777777u) & 0x88888888u;
+  return w & (0x77777777u | nz);
+}
+
+template <typename TIn, int NSUB, bool NV>
+__global__ void __launch_bounds__(256) rotquant_kernel(const TIn* __restrict__ in, const RotArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = static_cast<int>(threadIdx.x & 31);
+  const int m = blockIdx.x * 8 + static_cast<int>(threadIdx.x >> 5);
+  if (m >= a.M) return;
+  const TIn* row = in + static_cast<size_t>(m) * a.K;
+  constexpr unsigned kAll = 0xFFFFFFFFu;
+  for (int kb = 0; kb < a.K; kb += 256 * NSUB) {
+    float v[NSUB][8];
+#pragma unroll
+    for (int c = 0; c < NSUB; ++c) {
+      const int k = kb + 256 * c + 8 * lane;
+      float is[8];
+      load8(row + k, v[c]);
+      load8(a.inv_s + k, is);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[c][i] *= is[i];
+    }
+#pragma unroll
+    for (int h = 1; h < 8; h *= 2)
+#pragma unroll
+      for (int c = 0; c < NSUB; ++c)
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if ((i & h) == 0) {
+            const float x0 = v[c][i], x1 = v[c][i + h];
+            v[c][i] = x0 + x1;
+            v[c][i + h] = x0 - x1;
+          }
+#pragma unroll
+    for (int x = 1; x < 32; x *= 2) {
+      const bool upper = (lane & x) != 0;
+#pragma unroll
+      for (int c = 0; c < NSUB; ++c)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float o = __shfl_xor_sync(kAll, v[c][i], x);
+          v[c][i] = upper ? o - v[c][i] : v[c][i] + o;
+        }
+    }
+#pragma unroll
+    for (int h = 1; h < NSUB; h *= 2)
+#pragma unroll
+      for (int c = 0; c < NSUB; ++c)
+        if ((c & h) == 0)
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float x0 = v[c][i], x1 = v[c + h][i];
+            v[c][i] = x0 + x1;
+            v[c + h][i] = x0 - x1;
+          }
+#pragma unroll
+    for (int c = 0; c < NSUB; ++c) {
+      const int k = kb + 256 * c + 8 * lane;
+      float* x = v[c];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] *= a.nrm;
+      if (a.dump) {
+        float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + k);
+        d[0] = make_float4(x[0], x[1], x[2], x[3]);
+        d[1] = make_float4(x[4], x[5], x[6], x[7]);
+      }
+      float am = 0.0f;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
+      if constexpr (NV) {
+        am = fmaxf(am, __shfl_xor_sync(kAll, am, 1));
+        const uint32_t sb = cvt_e4m3(__fdiv_rn(am, 6.0f));
+        const float sc = e4m3_value(sb);
+        const uint32_t w = codes8_nvfp4(x, sc, sc > 0.0f ? rcp_approx(sc) : 0.0f);
+        *reinterpret_cast<uint32_t*>(a.codes + static_cast<size_t>(m) * (a.K / 2) + k / 2) = w;
+        if ((lane & 1) == 0) {
+          const int mr = m % kBM;
+          a.sf[(static_cast<size_t>(m / kBM) * (a.K / 64) + k / 64) * kSfAtom + (mr % 32) * 16 + (mr / 32) * 4 +
+               (k % 64) / kFp4Block] = static_cast<uint8_t>(sb);
+        }
+      } else {
+        am = fmaxf(am, __shfl_xor_sync(kAll, am, 1));
+        am = fmaxf(am, __shfl_xor_sync(kAll, am, 2));
+        if (a.G == 64) am = fmaxf(am, __shfl_xor_sync(kAll, am, 4));
+        const float sc = __fdiv_rn(am, 7.0f);
+        const float ks = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100 (see quantize_group)
+        const float scs = sc * ks;
+        const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
+        const float hs = 0.5f * scs;
+        uint32_t b[8];
+        int sum = 0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int ci = nearest_code(x[i] * ks, scs, inv, hs);
+          sum += ci;
+          b[i] = static_cast<uint32_t>(abs(ci)) | (static_cast<uint32_t>(ci) & 0x80u);
+        }
+        sum += __shfl_xor_sync(kAll, sum, 1);
+        sum += __shfl_xor_sync(kAll, sum, 2);
+        if (a.G == 64) sum += __shfl_xor_sync(kAll, sum, 4);
+        const uint32_t w0 = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+        const uint32_t w1 = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
+        *reinterpret_cast<uint2*>(a.codes + static_cast<size_t>(m) * a.K + k) = make_uint2(w0, w1);
+        if ((lane & (a.G / 8 - 1)) == 0) {
+          const size_t gi = static_cast<size_t>(k / a.G) * a.M_pad + m;
+          a.scales[gi] = sc;
+          a.ab[gi] = make_float2(sc * 262144.0f, (-8.0f * sc) * static_cast<float>(sum));
+        }
+      }
+    }
+  }
+}
+
+template <typename TIn, bool NV>
+cudaError_t launch_rotquant_t(const Handle& h, const TIn* in, const RotArgs& a, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((a.M + 7) / 8, 1, 1);
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  switch (h.hb) {
+    case 256: return cudaLaunchKernelEx(&cfg, rotquant_kernel<TIn, 1, NV>, in, a);
+    case 512: return cudaLaunchKernelEx(&cfg, rotquant_kernel<TIn, 2, NV>, in, a);
+    case 1024: return cudaLaunchKernelEx(&cfg, rotquant_kernel<TIn, 4, NV>, in, a);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 // Cluster size (CTAs along K per 128-row tile): as many as fit one wave of the GPU.
 int choose_split(int K, int tiles, int sms) {
   const int chunks = K / kChunk;
@@ -612,7 +802,8 @@ int choose_split(int K, int tiles, int sms) {
 }
 
 template <int RP, bool NV>
-cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
+cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, bool resid_only,
+                      cudaStream_t s) {
   using Cfg = ActCfg<RP>;
   const ActLayout L = act_layout(h, M);
   ActArgs a;
@@ -631,6 +822,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   a.ab = reinterpret_cast<float2*>(base + L.ab_off);
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
   a.dump = dump;
+  a.resid_only = resid_only ? 1 : 0;
   a.err = h.err;
   a.timeout_ns = deadline_budget_ns(h);
 
@@ -660,15 +852,43 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
 }
 
 template <bool NV>
-cudaError_t launch_fmt(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
+cudaError_t launch_fmt(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, bool resid_only,
+                       cudaStream_t s) {
   switch (h.r_pad) {
-    case 0: return launch_rp<0, NV>(h, am, ws, M, dump, s);
-    case 16: return launch_rp<16, NV>(h, am, ws, M, dump, s);
-    case 32: return launch_rp<32, NV>(h, am, ws, M, dump, s);
-    case 48: return launch_rp<48, NV>(h, am, ws, M, dump, s);
-    case 64: return launch_rp<64, NV>(h, am, ws, M, dump, s);
+    case 0: return launch_rp<0, NV>(h, am, ws, M, dump, resid_only, s);
+    case 16: return launch_rp<16, NV>(h, am, ws, M, dump, resid_only, s);
+    case 32: return launch_rp<32, NV>(h, am, ws, M, dump, resid_only, s);
+    case 48: return launch_rp<48, NV>(h, am, ws, M, dump, resid_only, s);
+    case 64: return launch_rp<64, NV>(h, am, ws, M, dump, resid_only, s);
     default: return cudaErrorInvalidValue;
   }
+}
+
+// Rotated layer: kernel (a) forms the remainder v = x - diag(s) H U p (and p_hat) into the
+// workspace, then the rotation kernel maps it to x~_perp and quantizes; with r = 0 the rotation
+// kernel reads X itself.  `dump` (optional) receives x~_perp.
+template <bool NV>
+cudaError_t launch_rotated(Handle& h, const ActMaps& am, const void* X, const void* ws, int M, float* dump,
+                           cudaStream_t s) {
+  const ActLayout L = act_layout(h, M);
+  uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
+  RotArgs a;
+  a.M = M;
+  a.K = h.K;
+  a.G = h.G;
+  a.M_pad = L.M_pad;
+  a.nrm = h.hnrm;
+  a.inv_s = h.inv_s;
+  a.codes = base + L.codes_off;
+  a.sf = base + L.scales_off;
+  a.scales = reinterpret_cast<float*>(base + L.scales_off);
+  a.ab = reinterpret_cast<float2*>(base + L.ab_off);
+  a.dump = dump;
+  if (h.r == 0) return launch_rotquant_t<__nv_bfloat16, NV>(h, static_cast<const __nv_bfloat16*>(X), a, s);
+  float* resid = reinterpret_cast<float*>(base + L.resid_off);
+  cudaError_t e = launch_fmt<NV>(h, am, ws, M, resid, true, s);
+  if (e != cudaSuccess) return e;
+  return launch_rotquant_t<float, NV>(h, resid, a, s);
 }
 
 }  // namespace
@@ -685,7 +905,9 @@ cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4,
 }
 
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
-  return h.fmt == kFmtNvfp4 ? launch_fmt<true>(h, am, ws, M, dump, s) : launch_fmt<false>(h, am, ws, M, dump, s);
+  const bool nv = h.fmt == kFmtNvfp4;
+  if (h.rot) return nv ? launch_rotated<true>(h, am, am.x, ws, M, dump, s) : launch_rotated<false>(h, am, am.x, ws, M, dump, s);
+  return nv ? launch_fmt<true>(h, am, ws, M, dump, false, s) : launch_fmt<false>(h, am, ws, M, dump, false, s);
 }
 
 }  // namespace qwam

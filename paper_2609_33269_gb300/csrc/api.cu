@@ -4,6 +4,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -86,12 +87,22 @@ ActLayout act_layout(const Handle& h, int M) {
     L.ab_off = L.scales_off + up256(static_cast<size_t>(L.M_pad) * (h.K / kFp4Block));
     L.phat_off = L.ab_off;
     L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
+    L.resid_off = 0;
+    if (h.rot && h.r > 0) {
+      L.resid_off = L.bytes;
+      L.bytes += up256(static_cast<size_t>(M) * h.K * 4);
+    }
     return L;
   }
   L.scales_off = up256(static_cast<size_t>(M) * h.K);
   L.ab_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
   L.phat_off = L.ab_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 8);
   L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
+  L.resid_off = 0;
+  if (h.rot && h.r > 0) {
+    L.resid_off = L.bytes;
+    L.bytes += up256(static_cast<size_t>(M) * h.K * 4);
+  }
   return L;
 }
 
@@ -156,8 +167,8 @@ const char* qwam_status_string(qwam_status s) {
   return "unknown status";
 }
 
-static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K, int N, int r, int group,
-                             struct CUstream_st* stream, qwam_asp_handle* out) {
+static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const float* sm, bool rot, int K, int N,
+                             int r, int group, struct CUstream_st* stream, qwam_asp_handle* out) {
   if (!out) return QWAM_ERR_INVALID_ARG;
   *out = nullptr;
   if (!W_bf16 || !qwam::aligned16(W_bf16)) return QWAM_ERR_INVALID_ARG;
@@ -167,6 +178,8 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K,
   if (r < 0 || r > K) return QWAM_ERR_INVALID_ARG;
   if (r > 0 && (!U || !qwam::aligned16(U))) return QWAM_ERR_INVALID_ARG;
   if (r > qwam::kMaxRank) return QWAM_ERR_UNSUPPORTED;
+  // the run-time rotation works on sub-blocks of 256 channels (one warp, eight per lane)
+  if (rot && (K % 256 != 0 || (sm && !qwam::aligned16(sm)))) return QWAM_ERR_INVALID_ARG;
   if (!qwam::ensure_encoder()) return QWAM_ERR_CUDA;
 
   auto* hs = new (std::nothrow) qwam_asp_handle_s();
@@ -180,6 +193,12 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K,
   h.r_pad = r == 0 ? 0 : qwam::round_up(r, 16);
   h.N_pad = qwam::round_up(N, qwam::kGemmBN);
   h.ku3 = h.r_pad == 0 ? 0 : qwam::round_up(3 * h.r_pad, 64);
+  h.rot = rot;
+  if (rot) {
+    h.hb = 1;
+    while (K % (2 * h.hb) == 0 && 2 * h.hb <= 1024) h.hb *= 2;
+    h.hnrm = static_cast<float>(1.0 / std::sqrt(static_cast<double>(h.hb)));
+  }
   cudaGetDevice(&h.device);
   cudaDeviceGetAttribute(&h.num_sms, cudaDevAttrMultiProcessorCount, h.device);
 
@@ -192,7 +211,8 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K,
   const size_t b_bh = qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2);
   const size_t b_ut = qwam::up256(static_cast<size_t>(2 * h.r_pad) * K * 2);
   const size_t b_u3 = qwam::up256(static_cast<size_t>(K) * h.ku3 * 2);
-  const size_t total = b_qw + b_sw + b_s32 + b_bh + b_ut + b_u3 + 256;
+  const size_t b_is = rot ? qwam::up256(static_cast<size_t>(K) * 4) : 0;
+  const size_t total = b_qw + b_sw + b_s32 + b_bh + b_ut + b_u3 + b_is + 256;
   if (cudaMalloc(&h.block, total) != cudaSuccess) {
     cudaGetLastError();
     delete hs;
@@ -210,7 +230,8 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K,
   h.Bh = reinterpret_cast<__half*>(q);
   h.ucat_t = reinterpret_cast<__nv_bfloat16*>(q + b_bh);
   h.ucat3 = reinterpret_cast<__nv_bfloat16*>(q + b_bh + b_ut);
-  h.err = reinterpret_cast<int*>(q + b_bh + b_ut + b_u3);
+  if (rot) h.inv_s = reinterpret_cast<float*>(q + b_bh + b_ut + b_u3);
+  h.err = reinterpret_cast<int*>(q + b_bh + b_ut + b_u3 + b_is);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   bool ok = true;
@@ -238,9 +259,13 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K,
     return QWAM_ERR_CUDA;
   }
   cudaError_t e = cudaMemsetAsync(h.block, 0, total, s);
-  if (e == cudaSuccess)
-    e = nv ? qwam::launch_pack_nvfp4(h, static_cast<const __nv_bfloat16*>(W_bf16), r > 0 ? U : nullptr, s)
-           : qwam::launch_pack(h, static_cast<const __nv_bfloat16*>(W_bf16), r > 0 ? U : nullptr, s);
+  if (e == cudaSuccess) {
+    const auto* W = static_cast<const __nv_bfloat16*>(W_bf16);
+    if (rot)
+      e = qwam::launch_pack_rotated(h, W, sm, r > 0 ? U : nullptr, s);
+    else
+      e = nv ? qwam::launch_pack_nvfp4(h, W, r > 0 ? U : nullptr, s) : qwam::launch_pack(h, W, r > 0 ? U : nullptr, s);
+  }
   int herr = 0;
   if (e == cudaSuccess) e = cudaMemcpy(&herr, h.err, sizeof(int), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess || herr != 0) {
@@ -254,12 +279,28 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, int K,
 
 qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int N, int r, int group,
                                   struct CUstream_st* stream, qwam_asp_handle* out) {
-  return pack_impl(qwam::kFmtInt4, W_bf16, U, K, N, r, group, stream, out);
+  return pack_impl(qwam::kFmtInt4, W_bf16, U, nullptr, false, K, N, r, group, stream, out);
+}
+
+qwam_status qwam_asp_pack_weights_rotated(const void* W_bf16, const float* s, const float* U, int K, int N, int r,
+                                          int group, struct CUstream_st* stream, qwam_asp_handle* out) {
+  return pack_impl(qwam::kFmtInt4, W_bf16, U, s, true, K, N, r, group, stream, out);
+}
+
+qwam_status qwam_asp_pack_weights_nvfp4_rotated(const void* W_bf16, const float* s, const float* U, int K, int N,
+                                                int r, struct CUstream_st* stream, qwam_asp_handle* out) {
+  return pack_impl(qwam::kFmtNvfp4, W_bf16, U, s, true, K, N, r, qwam::kFp4Block, stream, out);
+}
+
+qwam_status qwam_asp_rotation(qwam_asp_handle hs, int* hadamard_block) {
+  if (!hs || !hadamard_block) return QWAM_ERR_INVALID_ARG;
+  *hadamard_block = hs->h.rot ? hs->h.hb : 0;
+  return QWAM_OK;
 }
 
 qwam_status qwam_asp_pack_weights_nvfp4(const void* W_bf16, const float* U, int K, int N, int r,
                                         struct CUstream_st* stream, qwam_asp_handle* out) {
-  return pack_impl(qwam::kFmtNvfp4, W_bf16, U, K, N, r, qwam::kFp4Block, stream, out);
+  return pack_impl(qwam::kFmtNvfp4, W_bf16, U, nullptr, false, K, N, r, qwam::kFp4Block, stream, out);
 }
 
 qwam_status qwam_asp_format(qwam_asp_handle hs, int* format) {

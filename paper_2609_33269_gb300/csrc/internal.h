@@ -58,6 +58,14 @@ struct Handle {
   uint8_t* sfw = nullptr;            // NVFP4: E4M3 block scales of W_perp in atoms (N_pad rows)
   float sg = 0.0f;                   // NVFP4: float32 per-tensor weight scale
   int* err = nullptr;                // sticky device error word
+  // Smoothing and block Hadamard rotation in front of the layer (Sec. 2 Eq. (pair)): the packed
+  // weight is W~ = H diag(s) W, the activations are rotated at run time, x~ = H diag(s)^-1 x.
+  // ucat_t then holds diag(s)^-1 H U (the projection x~ U = x (diag(s)^-1 H U)) and ucat3 holds
+  // diag(s) H U (the remainder x - diag(s) H U p, which H diag(s)^-1 maps to x~ - U p).
+  bool rot = false;
+  int hb = 0;                        // Hadamard block: largest power of two dividing K, <= 1024
+  float hnrm = 0.0f;                 // RN_f32(1 / sqrt(hb))
+  float* inv_s = nullptr;            // [K]: RN_f32(1 / s_k) (1 without smoothing)
   double timeout_s = 2.0;
   CUtensorMap qw_map, sw32_map, Bh_map, ucat_t_map, ucat3_map;
   CUtensorMap qw4_map;               // NVFP4 weight codes [N, K/2], box {128, 128}, 128-byte swizzle
@@ -67,6 +75,7 @@ struct Handle {
 
 struct ActLayout {
   size_t codes_off, scales_off, ab_off, phat_off, bytes;
+  size_t resid_off;  // rotated handles with r > 0: float32 [M, K] remainder before the rotation
   int M_pad;
 };
 ActLayout act_layout(const Handle& h, int M);
@@ -83,6 +92,7 @@ uint64_t deadline_budget_ns(const Handle& h);
 // Launchers (return cudaSuccess or the launch error).
 cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
 cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
+cudaError_t launch_pack_rotated(Handle& h, const __nv_bfloat16* W, const float* s, const float* U, cudaStream_t st);
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s);
 cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
 cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);

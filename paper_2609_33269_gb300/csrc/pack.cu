@@ -5,6 +5,7 @@
 //
 // Every float64 operation is an explicit IEEE intrinsic (__dmul_rn, __dadd_rn, ...) so that no
 // multiply-add is contracted: sums run in index order, each product and sum rounded once.
+#include <cmath>
 #include <cuda_fp4.h>
 #include <cuda_fp8.h>
 
@@ -14,8 +15,15 @@
 namespace qwam {
 namespace {
 
+// The weight entering the pack: bf16 W, or the float64 smoothed and rotated W~ (exact either way).
+__device__ __forceinline__ double wval(const __nv_bfloat16* W, size_t i) {
+  return static_cast<double>(__bfloat162float(W[i]));
+}
+__device__ __forceinline__ double wval(const double* W, size_t i) { return W[i]; }
+
 // B_f[j, n] = sum_k U[k, j] W[k, n]  (k ascending), float64.
-__global__ void branch_weight_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U, int K, int N,
+template <typename WT>
+__global__ void branch_weight_kernel(const WT* __restrict__ W, const float* __restrict__ U, int K, int N,
                                      int r, double* __restrict__ Bf) {
   int n = blockIdx.x * blockDim.x + threadIdx.x;
   int j = blockIdx.y;
@@ -23,20 +31,21 @@ __global__ void branch_weight_kernel(const __nv_bfloat16* __restrict__ W, const 
   double acc = 0.0;
   for (int k = 0; k < K; ++k) {
     double u = static_cast<double>(U[static_cast<size_t>(k) * r + j]);
-    double w = static_cast<double>(__bfloat162float(W[static_cast<size_t>(k) * N + n]));
+    double w = wval(W, static_cast<size_t>(k) * N + n);
     acc = __dadd_rn(acc, __dmul_rn(u, w));
   }
   Bf[static_cast<size_t>(j) * N + n] = acc;
 }
 
 // W_perp[k, n] = W[k, n] - sum_j U[k, j] B_f[j, n]  (j ascending).
-__device__ __forceinline__ double wperp(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+template <typename WT>
+__device__ __forceinline__ double wperp(const WT* __restrict__ W, const float* __restrict__ U,
                                         const double* __restrict__ Bf, int N, int r, int k, int n) {
   double acc = 0.0;
   for (int j = 0; j < r; ++j)
     acc = __dadd_rn(acc, __dmul_rn(static_cast<double>(U[static_cast<size_t>(k) * r + j]),
                                    Bf[static_cast<size_t>(j) * N + n]));
-  return __dsub_rn(static_cast<double>(__bfloat162float(W[static_cast<size_t>(k) * N + n])), acc);
+  return __dsub_rn(wval(W, static_cast<size_t>(k) * N + n), acc);
 }
 
 // Nearest integer to the exact quotient w / s, ties to even.  s is a float16 value and w a
@@ -54,7 +63,8 @@ __device__ __forceinline__ int nearest_code_f64(double w, double s) {
 // One thread per (output channel n, group g): s_w = RN_f16(absmax / 7), codes packed 4 bits
 // each into qw[n, :]: 32-bit word j holds k = 8j..8j+3 in the low nibbles and k = 8j+4..8j+7 in
 // the high nibbles of its four bytes (the GEMM expands a word to bytes with three logic ops).
-__global__ void quantize_weight_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+template <typename WT>
+__global__ void quantize_weight_kernel(const WT* __restrict__ W, const float* __restrict__ U,
                                        const double* __restrict__ Bf, int K, int N, int r, int G, int N_pad,
                                        uint8_t* __restrict__ qw, __half* __restrict__ sw, float* __restrict__ sw32,
                                        int* err) {
@@ -101,20 +111,25 @@ __global__ void branch_half_kernel(const double* __restrict__ Bf, int N, int r, 
 
 // bf16 hi/lo split of U: hi = RN_bf16(u), lo = RN_bf16(u - hi).  Written twice: transposed
 // [2 r_pad, K] for the projection X U, and [K, ku3] as (hi, lo, hi) for the reconstruction.
-__global__ void split_basis_kernel(const float* __restrict__ U, int K, int r, int r_pad, int ku3,
-                                   __nv_bfloat16* __restrict__ ucat_t, __nv_bfloat16* __restrict__ ucat3) {
+// Up is the basis of the projection and Ur that of the reconstruction: both U, or, for a rotated
+// layer, diag(s)^-1 H U and diag(s) H U.
+__global__ void split_basis_kernel(const float* __restrict__ Up, const float* __restrict__ Ur, int K, int r, int r_pad,
+                                   int ku3, __nv_bfloat16* __restrict__ ucat_t, __nv_bfloat16* __restrict__ ucat3) {
   int k = blockIdx.x * blockDim.x + threadIdx.x;
   if (k >= K) return;
   for (int j = 0; j < r_pad; ++j) {
-    float u = (j < r) ? U[static_cast<size_t>(k) * r + j] : 0.0f;
-    __nv_bfloat16 hi = __float2bfloat16_rn(u);
-    __nv_bfloat16 lo = __float2bfloat16_rn(u - __bfloat162float(hi));
-    ucat_t[static_cast<size_t>(j) * K + k] = hi;
-    ucat_t[static_cast<size_t>(r_pad + j) * K + k] = lo;
+    const float up = (j < r) ? Up[static_cast<size_t>(k) * r + j] : 0.0f;
+    const float ur = (j < r) ? Ur[static_cast<size_t>(k) * r + j] : 0.0f;
+    const __nv_bfloat16 phi = __float2bfloat16_rn(up);
+    const __nv_bfloat16 plo = __float2bfloat16_rn(up - __bfloat162float(phi));
+    const __nv_bfloat16 rhi = __float2bfloat16_rn(ur);
+    const __nv_bfloat16 rlo = __float2bfloat16_rn(ur - __bfloat162float(rhi));
+    ucat_t[static_cast<size_t>(j) * K + k] = phi;
+    ucat_t[static_cast<size_t>(r_pad + j) * K + k] = plo;
     __nv_bfloat16* row = ucat3 + static_cast<size_t>(k) * ku3;
-    row[j] = hi;
-    row[r_pad + j] = lo;
-    row[2 * r_pad + j] = hi;
+    row[j] = rhi;
+    row[r_pad + j] = rlo;
+    row[2 * r_pad + j] = rhi;
   }
   for (int j = 3 * r_pad; j < ku3; ++j) ucat3[static_cast<size_t>(k) * ku3 + j] = __float2bfloat16_rn(0.0f);
 }
@@ -124,7 +139,8 @@ __global__ void split_basis_kernel(const float* __restrict__ U, int K, int r, in
 // One thread per (output channel n, block b of 16 K): the block's absmax of |W_perp| (float64),
 // and the tensor's absmax by an atomic max on the bit pattern (non-negative doubles order as
 // unsigned integers).
-__global__ void block_amax_nvfp4_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+template <typename WT>
+__global__ void block_amax_nvfp4_kernel(const WT* __restrict__ W, const float* __restrict__ U,
                                         const double* __restrict__ Bf, int K, int N, int r, double* __restrict__ bam,
                                         unsigned long long* __restrict__ amax_bits) {
   int n = blockIdx.x * blockDim.x + threadIdx.x;
@@ -146,7 +162,8 @@ __device__ __forceinline__ double e4m3_to_double(__nv_fp8_storage_t b) {
 // codes RN_e2m1(w / (s_b s_g)), each from the float64 quotient (one rounding to a 4-bit format),
 // saturating; a code of magnitude zero is stored as 0.  Codes are packed two per byte, low nibble =
 // even k; the block scale goes to its atom (see internal.h).
-__global__ void quantize_weight_nvfp4_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ U,
+template <typename WT>
+__global__ void quantize_weight_nvfp4_kernel(const WT* __restrict__ W, const float* __restrict__ U,
                                              const double* __restrict__ Bf, int K, int N, int r,
                                              const double* __restrict__ bam,
                                              const unsigned long long* __restrict__ amax_bits,
@@ -182,9 +199,68 @@ __global__ void quantize_weight_nvfp4_kernel(const __nv_bfloat16* __restrict__ W
   *reinterpret_cast<uint2*>(qw + static_cast<size_t>(n) * (K / 2) + b * (kFp4Block / 2)) = make_uint2(lo, hi);
 }
 
-}  // namespace
+// ---- smoothing and block Hadamard rotation (Sec. 2 Eq. (pair); App. B.1), float64
 
-cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s) {
+// Columns n0 .. n0+15 of rows [kb, kb + B) of A [K, N] (bf16 or float32), each times scale[k]
+// when scale is given, through the block Walsh-Hadamard butterflies (a + b, a - b) at spans
+// 1, 2, ..., B/2, then times nrm = 1/sqrt(B): out [K, N] float64.  Within one span the pairs are
+// disjoint, so every entry sees the same float64 operations in the same order as a sequential
+// transform, whatever thread takes it.
+constexpr int kRotCols = 16;
+template <typename AT>
+__global__ void __launch_bounds__(256) rotate_cols_kernel(const AT* __restrict__ A, const float* __restrict__ scale,
+                                                          int N, int B, double nrm, double* __restrict__ out) {
+  extern __shared__ double tile[];  // [B][kRotCols]
+  const int kb = blockIdx.x * B, n0 = blockIdx.y * kRotCols;
+  for (int i = threadIdx.x; i < B * kRotCols; i += blockDim.x) {
+    const int k = i / kRotCols, c = i % kRotCols, n = n0 + c;
+    double v = 0.0;
+    if (n < N) {
+      v = static_cast<double>(static_cast<float>(A[static_cast<size_t>(kb + k) * N + n]));
+      if (scale) v = __dmul_rn(v, static_cast<double>(scale[kb + k]));
+    }
+    tile[i] = v;
+  }
+  for (int h = 1; h < B; h *= 2) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < (B / 2) * kRotCols; i += blockDim.x) {
+      const int pr = i / kRotCols, c = i % kRotCols;
+      const int a = (pr / h) * 2 * h + pr % h, b = a + h;
+      const double xa = tile[a * kRotCols + c], xb = tile[b * kRotCols + c];
+      tile[a * kRotCols + c] = __dadd_rn(xa, xb);
+      tile[b * kRotCols + c] = __dsub_rn(xa, xb);
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < B * kRotCols; i += blockDim.x) {
+    const int k = i / kRotCols, n = n0 + i % kRotCols;
+    if (n < N) out[static_cast<size_t>(kb + k) * N + n] = __dmul_rn(tile[i], nrm);
+  }
+}
+
+// From HU [K, r] (float64): the projection basis diag(s)^-1 H U and the reconstruction basis
+// diag(s) H U, each rounded once to float32; and RN_f32(1 / s_k) for the run-time rotation.
+__global__ void rotated_bases_kernel(const double* __restrict__ HU, const float* __restrict__ sm, int K, int r,
+                                     float* __restrict__ Up, float* __restrict__ Ur, float* __restrict__ inv_s) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= K) return;
+  const double sk = sm ? static_cast<double>(sm[k]) : 1.0;
+  inv_s[k] = sm ? __frcp_rn(sm[k]) : 1.0f;
+  for (int j = 0; j < r; ++j) {
+    const double v = HU[static_cast<size_t>(k) * r + j];
+    Up[static_cast<size_t>(k) * r + j] = __double2float_rn(__ddiv_rn(v, sk));
+    Ur[static_cast<size_t>(k) * r + j] = __double2float_rn(__dmul_rn(v, sk));
+  }
+}
+
+// Every factor must be a positive finite number.
+__global__ void check_scale_kernel(const float* __restrict__ sm, int K, int* err) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k < K && !(sm[k] > 0.0f && isfinite(sm[k]))) atomicOr(err, kErrRange);
+}
+
+template <typename WT>
+cudaError_t pack_nvfp4(Handle& h, const WT* W, const float* U, const float* Up, const float* Ur, cudaStream_t s) {
   const int K = h.K, N = h.N, r = h.r;
   const int nb = K / kFp4Block;
   double* Bf = nullptr;
@@ -204,7 +280,7 @@ cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U,
                                                                           sg_dev);
     if (r > 0) {
       branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
-      split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(U, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+      split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
     }
     e = cudaGetLastError();
     cudaError_t e2 = cudaStreamSynchronize(s);
@@ -217,7 +293,8 @@ cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U,
   return e;
 }
 
-cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s) {
+template <typename WT>
+cudaError_t pack_int4(Handle& h, const WT* W, const float* U, const float* Up, const float* Ur, cudaStream_t s) {
   const int K = h.K, N = h.N, r = h.r;
   double* Bf = nullptr;
   cudaError_t e = cudaMalloc(&Bf, sizeof(double) * static_cast<size_t>(r > 0 ? r : 1) * N);
@@ -230,12 +307,60 @@ cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaS
                                                                      h.err);
   if (r > 0) {
     branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
-    split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(U, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+    split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
   }
   e = cudaGetLastError();
   cudaError_t e2 = cudaStreamSynchronize(s);
   cudaFree(Bf);
   return e != cudaSuccess ? e : e2;
+}
+
+}  // namespace
+
+cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s) {
+  return pack_nvfp4(h, W, U, U, U, s);
+}
+
+cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s) {
+  return pack_int4(h, W, U, U, U, s);
+}
+
+// W~ = H diag(s) W and H U in float64, the two run-time bases and 1/s, then the ordinary pack of
+// W~ against U (U spans the protected directions in the rotated coordinates).
+cudaError_t launch_pack_rotated(Handle& h, const __nv_bfloat16* W, const float* sm, const float* U, cudaStream_t s) {
+  const int K = h.K, N = h.N, r = h.r, B = h.hb;
+  const double nrm = 1.0 / std::sqrt(static_cast<double>(B));
+  const size_t smem = sizeof(double) * B * kRotCols;
+  double* Wt = nullptr;
+  double* HU = nullptr;
+  float* Upr = nullptr;
+  cudaError_t e = cudaFuncSetAttribute(rotate_cols_kernel<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(rotate_cols_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+  if (e == cudaSuccess) e = cudaMalloc(&Wt, sizeof(double) * static_cast<size_t>(K) * N);
+  if (e == cudaSuccess) e = cudaMalloc(&HU, sizeof(double) * static_cast<size_t>(K) * (r > 0 ? r : 1));
+  if (e == cudaSuccess) e = cudaMalloc(&Upr, sizeof(float) * 2 * static_cast<size_t>(K) * (r > 0 ? r : 1));
+  if (e == cudaSuccess) {
+    const int T = 128;
+    if (sm) check_scale_kernel<<<(K + T - 1) / T, T, 0, s>>>(sm, K, h.err);
+    rotate_cols_kernel<__nv_bfloat16><<<dim3(K / B, (N + kRotCols - 1) / kRotCols), 256, smem, s>>>(W, sm, N, B, nrm, Wt);
+    if (r > 0)
+      rotate_cols_kernel<float><<<dim3(K / B, (r + kRotCols - 1) / kRotCols), 256, smem, s>>>(U, nullptr, r, B, nrm, HU);
+    float* Up = Upr;
+    float* Ur = Upr + static_cast<size_t>(K) * (r > 0 ? r : 1);
+    rotated_bases_kernel<<<(K + T - 1) / T, T, 0, s>>>(HU, sm, K, r, Up, Ur, h.inv_s);
+    e = cudaGetLastError();
+    if (e == cudaSuccess)
+      e = h.fmt == kFmtNvfp4 ? pack_nvfp4(h, static_cast<const double*>(Wt), U, Up, Ur, s)
+                             : pack_int4(h, static_cast<const double*>(Wt), U, Up, Ur, s);
+  }
+  cudaStreamSynchronize(s);
+  cudaFree(Wt);
+  cudaFree(HU);
+  cudaFree(Upr);
+  return e;
 }
 
 }  // namespace qwam
