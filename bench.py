@@ -338,12 +338,16 @@ def run_ours(args):
     stream = torch.cuda.current_stream(dev)
     flops = 2.0 * M * N * K
 
-    def timed(fmt, nsteps, warmup, clocks=None):
+    def timed(fmt, nsteps, warmup, clocks=None, smooth=None):
         """Per-kernel CUDA-event times of `nsteps` steps over rotating sets (weights packed per
-        set, activations, workspaces, outputs), after `warmup` untimed steps."""
+        set, activations, workspaces, outputs), after `warmup` untimed steps.  `smooth`: pack
+        rotated layers (Eq. (pair)) with these smoothing factors."""
         sets = []
         for i in range(ROTATE_SETS):
-            lin = asp.AspLinear(W, Ud, G, fmt=fmt)
+            if smooth is None:
+                lin = asp.AspLinear(W, Ud, G, fmt=fmt)
+            else:
+                lin = asp.AspLinear(W, Ud, G, fmt=fmt, rotate=True, s=smooth)
             X = X0 if i == 0 else X0.clone()
             sets.append((lin, X, lin.workspace(M), torch.empty((M, N), dtype=torch.bfloat16, device=dev)))
         mb = ROTATE_SETS * (2 * M * K + 2 * M * N + lin_ws_bytes(sets[0][0], M) + N * K // 2) / 1e6
@@ -496,6 +500,24 @@ def run_ours(args):
         for s_ in vr["sets"]:
             s_[0].close()
         variants["small_m"] = small_m_latencies(asp, wl, dev, stream, dev_bf16)
+        # Smoothing (alpha = 0.5, factors from this batch's channel maxima) and the block Hadamard
+        # rotation (B = 1024) in front of the same layer: kernel (a) writes the float32 remainder,
+        # the rotation kernel rotates and quantizes it (two launches in qwam_asp_quantize_act).
+        xmax = X0.float().abs().amax(dim=0).contiguous()
+        smooth = torch.empty(K, dtype=torch.float32, device=dev)
+        asp.qwam_asp_smoothing_factors(xmax, W, K, N, 0.5, smooth, stream)
+        rr = timed(asp.QWAM_FMT_INT4, vsteps, max(3, min(args.warmup, 20)), smooth=smooth)
+        a_fused = alg_bytes_actquant(M, K, r_pad, G)
+        a_split = a_fused + 4 * M * K * 2 + 4 * K  # the float32 remainder written and read back, 1/s
+        variants["rotated_int4"] = {
+            "value": rr["value"], "unit": UNIT, "steps": vsteps, "ms_per_step": rr["total_ms"] / vsteps,
+            "what": "smoothing (alpha 0.5) + block Hadamard (B 1024) in front of the INT4 layer (Eq. (pair))",
+            "act_path_ms": rr["t_a"], "gemm_ms": rr["t_b"],
+            "act_path_gbs_of_fused_bytes": a_fused / (rr["t_a"] * 1e-3) / 1e9,
+            "act_path_gbs_of_moved_bytes": a_split / (rr["t_a"] * 1e-3) / 1e9, "peak_gbs": hbm_peak,
+            "launches_per_step": 3}
+        for s_ in rr["sets"]:
+            s_[0].close()
 
     if rank != 0:
         return 0

@@ -608,16 +608,15 @@ __global__ void __launch_bounds__(128) debug_quantize_kernel(const float* R, int
 //
 //   x~_perp = H diag(s)^-1 v,  v = x (r = 0) or v = x - diag(s) H U p (r > 0, from kernel (a))
 //
-// then the same quantizers as kernel (a).  One warp per token row walks K in Hadamard blocks of
+// then the same quantizers as kernel (a).  One warp takes one token row and one Hadamard block of
 // B = 256 NSUB channels; lane l holds channels 256 c + 8 l .. + 7 of sub-block c.  The fast
 // Walsh-Hadamard butterflies run at spans 1, 2, 4 inside a lane, 8 .. 128 across lanes
-// (shuffles) and 256, 512 across the lane's sub-blocks, then every value is scaled by
-// RN_f32(1/sqrt(B)).  A quantization group (32 or 64 channels) is 4 or 8 neighbouring lanes, an
-// NVFP4 block (16) two.
+// (shuffles) and 256, 512 across the lane's sub-blocks.  The normalisation 1/sqrt(B) is folded
+// into the per-channel factor applied first, RN_f32(1 / (sqrt(B) s_k)).  A quantization group
+// (32 or 64 channels) is 4 or 8 neighbouring lanes, an NVFP4 block (16) two.
 struct RotArgs {
   int M, K, G, M_pad;
-  float nrm;
-  const float* inv_s;
+  const float* inv_s;  // [K]: RN_f32(1 / (sqrt(B) s_k))
   uint8_t* codes;
   uint8_t* sf;
   float* scales;
@@ -663,15 +662,19 @@ __device__ __forceinline__ uint32_t codes8_nvfp4(const float* x, float sc, float
 }
 
 template <typename TIn, int NSUB, bool NV>
-__global__ void __launch_bounds__(256) rotquant_kernel(const TIn* __restrict__ in, const RotArgs a) {
+__global__ void __launch_bounds__(256, 4) rotquant_kernel(const TIn* __restrict__ in, const RotArgs a) {
   pdl_launch_dependents();
   pdl_wait();
   const int lane = static_cast<int>(threadIdx.x & 31);
-  const int m = blockIdx.x * 8 + static_cast<int>(threadIdx.x >> 5);
-  if (m >= a.M) return;
+  // one warp per (token row, Hadamard block): many warps in flight, each with one block's work
+  const int nblk = a.K / (256 * NSUB);
+  const long long wg = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (wg >= static_cast<long long>(a.M) * nblk) return;
+  const int m = static_cast<int>(wg / nblk);
   const TIn* row = in + static_cast<size_t>(m) * a.K;
   constexpr unsigned kAll = 0xFFFFFFFFu;
-  for (int kb = 0; kb < a.K; kb += 256 * NSUB) {
+  {
+    const int kb = static_cast<int>(wg % nblk) * (256 * NSUB);
     float v[NSUB][8];
 #pragma unroll
     for (int c = 0; c < NSUB; ++c) {
@@ -695,14 +698,12 @@ __global__ void __launch_bounds__(256) rotquant_kernel(const TIn* __restrict__ i
           }
 #pragma unroll
     for (int x = 1; x < 32; x *= 2) {
-      const bool upper = (lane & x) != 0;
+      // lower lane: v + o; upper lane: o - v; both one exactly rounded fma with a +-1 factor
+      const float sgn = (lane & x) ? -1.0f : 1.0f;
 #pragma unroll
       for (int c = 0; c < NSUB; ++c)
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const float o = __shfl_xor_sync(kAll, v[c][i], x);
-          v[c][i] = upper ? o - v[c][i] : v[c][i] + o;
-        }
+        for (int i = 0; i < 8; ++i) v[c][i] = fmaf(v[c][i], sgn, __shfl_xor_sync(kAll, v[c][i], x));
     }
 #pragma unroll
     for (int h = 1; h < NSUB; h *= 2)
@@ -719,8 +720,6 @@ __global__ void __launch_bounds__(256) rotquant_kernel(const TIn* __restrict__ i
     for (int c = 0; c < NSUB; ++c) {
       const int k = kb + 256 * c + 8 * lane;
       float* x = v[c];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) x[i] *= a.nrm;
       if (a.dump) {
         float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + k);
         d[0] = make_float4(x[0], x[1], x[2], x[3]);
@@ -776,7 +775,8 @@ __global__ void __launch_bounds__(256) rotquant_kernel(const TIn* __restrict__ i
 template <typename TIn, bool NV>
 cudaError_t launch_rotquant_t(const Handle& h, const TIn* in, const RotArgs& a, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((a.M + 7) / 8, 1, 1);
+  const long long warps = static_cast<long long>(a.M) * (a.K / h.hb);
+  cfg.gridDim = dim3(static_cast<unsigned>((warps + 7) / 8), 1, 1);
   cfg.blockDim = dim3(256, 1, 1);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -877,7 +877,6 @@ cudaError_t launch_rotated(Handle& h, const ActMaps& am, const void* X, const vo
   a.K = h.K;
   a.G = h.G;
   a.M_pad = L.M_pad;
-  a.nrm = h.hnrm;
   a.inv_s = h.inv_s;
   a.codes = base + L.codes_off;
   a.sf = base + L.scales_off;

@@ -197,7 +197,6 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
   if (rot) {
     h.hb = 1;
     while (K % (2 * h.hb) == 0 && 2 * h.hb <= 1024) h.hb *= 2;
-    h.hnrm = static_cast<float>(1.0 / std::sqrt(static_cast<double>(h.hb)));
   }
   cudaGetDevice(&h.device);
   cudaDeviceGetAttribute(&h.num_sms, cudaDevAttrMultiProcessorCount, h.device);

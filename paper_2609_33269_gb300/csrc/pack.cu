@@ -239,13 +239,15 @@ __global__ void __launch_bounds__(256) rotate_cols_kernel(const AT* __restrict__
 }
 
 // From HU [K, r] (float64): the projection basis diag(s)^-1 H U and the reconstruction basis
-// diag(s) H U, each rounded once to float32; and RN_f32(1 / s_k) for the run-time rotation.
+// diag(s) H U, each rounded once to float32; and RN_f32(nrm / s_k), nrm = 1/sqrt(B), the factor
+// the run-time rotation applies before its butterflies.
 __global__ void rotated_bases_kernel(const double* __restrict__ HU, const float* __restrict__ sm, int K, int r,
-                                     float* __restrict__ Up, float* __restrict__ Ur, float* __restrict__ inv_s) {
+                                     double nrm, float* __restrict__ Up, float* __restrict__ Ur,
+                                     float* __restrict__ inv_s) {
   const int k = blockIdx.x * blockDim.x + threadIdx.x;
   if (k >= K) return;
   const double sk = sm ? static_cast<double>(sm[k]) : 1.0;
-  inv_s[k] = sm ? __frcp_rn(sm[k]) : 1.0f;
+  inv_s[k] = __double2float_rn(__ddiv_rn(nrm, sk));
   for (int j = 0; j < r; ++j) {
     const double v = HU[static_cast<size_t>(k) * r + j];
     Up[static_cast<size_t>(k) * r + j] = __double2float_rn(__ddiv_rn(v, sk));
@@ -350,7 +352,7 @@ cudaError_t launch_pack_rotated(Handle& h, const __nv_bfloat16* W, const float* 
       rotate_cols_kernel<float><<<dim3(K / B, (r + kRotCols - 1) / kRotCols), 256, smem, s>>>(U, nullptr, r, B, nrm, HU);
     float* Up = Upr;
     float* Ur = Upr + static_cast<size_t>(K) * (r > 0 ? r : 1);
-    rotated_bases_kernel<<<(K + T - 1) / T, T, 0, s>>>(HU, sm, K, r, Up, Ur, h.inv_s);
+    rotated_bases_kernel<<<(K + T - 1) / T, T, 0, s>>>(HU, sm, K, r, nrm, Up, Ur, h.inv_s);
     e = cudaGetLastError();
     if (e == cudaSuccess)
       e = h.fmt == kFmtNvfp4 ? pack_nvfp4(h, static_cast<const double*>(Wt), U, Up, Ur, s)
