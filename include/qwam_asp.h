@@ -238,6 +238,14 @@ qwam_status qwam_asp_export(qwam_asp_handle h, void* qw, void* sw, void* Bh, voi
 /* Free the handle and its device buffers (synchronizes the device). */
 qwam_status qwam_asp_destroy(qwam_asp_handle h);
 
+/* Bias of the layer (App. B.1: the GEMM kernel adds the bias in its epilogue).  `bias` is a
+ * device float32 [N], 16-byte aligned; it is copied into the handle (synchronously on `stream`),
+ * and every later qwam_asp_gemm / qwam_asp_linear / qwam_asp_linear_static of the handle stores
+ * Y[m, n] = RN(acc[m, n] + bias[n]) with acc the float32 result described above (one float32
+ * addition, then the conversion to the output type).  NULL removes the bias.  Errors:
+ * QWAM_ERR_INVALID_ARG (no handle, unaligned bias), QWAM_ERR_OOM, QWAM_ERR_CUDA. */
+qwam_status qwam_asp_set_bias(qwam_asp_handle h, const float* bias, struct CUstream_st* stream);
+
 const char* qwam_status_string(qwam_status s);
 
 /* ---- test support ------------------------------------------------------------------------ */

@@ -41,7 +41,7 @@ EXPORTED = [
     "qwam_asp_debug_quantize_rows", "qwam_asp_smoothing_factors", "qwam_asp_rotated_gramian",
     "qwam_asp_gramian_trace", "qwam_asp_subspace_workspace_bytes", "qwam_asp_action_subspace",
     "qwam_asp_select_experts", "qwam_asp_pack_weights_rotated", "qwam_asp_pack_weights_nvfp4_rotated",
-    "qwam_asp_rotation",
+    "qwam_asp_rotation", "qwam_asp_set_bias",
 ]
 
 _lib = None
@@ -94,6 +94,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_pack_weights_rotated.argtypes = [V, V, V, I, I, I, I, V, ctypes.POINTER(H)]
         lib.qwam_asp_pack_weights_nvfp4_rotated.argtypes = [V, V, V, I, I, I, V, ctypes.POINTER(H)]
         lib.qwam_asp_rotation.argtypes = [H, ctypes.POINTER(I)]
+        lib.qwam_asp_set_bias.argtypes = [H, V, V]
         lib.qwam_asp_export_nvfp4.argtypes = [H, V, V, ctypes.POINTER(ctypes.c_float), V]
         for name in EXPORTED:
             if name != "qwam_status_string":
@@ -152,6 +153,11 @@ def qwam_asp_pack_weights_nvfp4_rotated(W_bf16, s, U, K: int, N: int, r: int, st
     _check(load().qwam_asp_pack_weights_nvfp4_rotated(_ptr(W_bf16), _ptr(s), _ptr(U), K, N, r, _stream(stream),
                                                       ctypes.byref(h)), "qwam_asp_pack_weights_nvfp4_rotated")
     return h.value
+
+
+def qwam_asp_set_bias(h: int, bias, stream=None):
+    """Bias [N] float32 (device) added in the GEMM epilogue; None removes it."""
+    _check(load().qwam_asp_set_bias(h, _ptr(bias), _stream(stream)), "qwam_asp_set_bias")
 
 
 def qwam_asp_rotation(h: int) -> int:

@@ -530,7 +530,36 @@ qwam_status qwam_asp_destroy(qwam_asp_handle hs) {
   if (!hs) return QWAM_ERR_INVALID_ARG;
   cudaDeviceSynchronize();
   cudaError_t e = cudaFree(hs->h.block);
+  if (hs->h.bias) cudaFree(hs->h.bias);
   delete hs;
+  return from_cuda_status(e);
+}
+
+qwam_status qwam_asp_set_bias(qwam_asp_handle hs, const float* bias, struct CUstream_st* stream) {
+  if (!hs) return QWAM_ERR_INVALID_ARG;
+  Handle& h = hs->h;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (!bias) {
+    if (h.bias) {
+      if (cudaStreamSynchronize(s) != cudaSuccess) return QWAM_ERR_CUDA;
+      cudaFree(h.bias);
+      h.bias = nullptr;
+    }
+    return QWAM_OK;
+  }
+  if (!qwam::aligned16(bias)) return QWAM_ERR_INVALID_ARG;
+  if (!h.bias) {
+    // 16-byte aligned rows of 8 floats: the epilogues read N rounded up to 8
+    if (cudaMalloc(&h.bias, sizeof(float) * static_cast<size_t>(h.N_pad)) != cudaSuccess) {
+      cudaGetLastError();
+      h.bias = nullptr;
+      return QWAM_ERR_OOM;
+    }
+    if (cudaMemsetAsync(h.bias, 0, sizeof(float) * static_cast<size_t>(h.N_pad), s) != cudaSuccess)
+      return QWAM_ERR_CUDA;
+  }
+  cudaError_t e = cudaMemcpyAsync(h.bias, bias, sizeof(float) * static_cast<size_t>(h.N), cudaMemcpyDeviceToDevice, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   return from_cuda_status(e);
 }
 

@@ -50,6 +50,7 @@ struct GemmArgs {
   int m_tiles, n_tiles;
   void* Y;
   int y_f32;
+  const float* bias;  // optional [N], added to the float32 result before it is stored
   int* err;
   uint64_t timeout_ns;
 };
@@ -478,11 +479,17 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (n >= a.N) continue;
               const size_t off = static_cast<size_t>(m) * a.N + n;
               const f2 y = acc[16 * cb + 4 * k + j];
+              float y0 = lo_f(y), y1 = hi_f(y);
+              if (a.bias) {
+                const float2 bb = *reinterpret_cast<const float2*>(a.bias + n);
+                y0 += bb.x;
+                y1 += bb.y;
+              }
               if (a.y_f32) {
-                *reinterpret_cast<float2*>(static_cast<float*>(a.Y) + off) = make_float2(lo_f(y), hi_f(y));
+                *reinterpret_cast<float2*>(static_cast<float*>(a.Y) + off) = make_float2(y0, y1);
               } else {
                 *reinterpret_cast<__nv_bfloat162*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
-                    __floats2bfloat162_rn(lo_f(y), hi_f(y));
+                    __floats2bfloat162_rn(y0, y1);
               }
             }
         }
@@ -509,6 +516,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
   a.n_tiles = (h.N + kGemmBN - 1) / kGemmBN;
   a.Y = Y;
   a.y_f32 = y_f32 ? 1 : 0;
+  a.bias = h.bias;
   a.err = h.err;
   a.timeout_ns = deadline_budget_ns(h);
   static bool attr_done = false;

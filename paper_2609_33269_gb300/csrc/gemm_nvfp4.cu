@@ -36,6 +36,7 @@ struct Gemm4Args {
   float sg;            // per-tensor weight scale
   void* Y;
   int y_f32;
+  const float* bias;  // optional [N], added to the float32 result before it is stored
   int* err;
   uint64_t timeout_ns;
 };
@@ -274,6 +275,17 @@ __global__ void __launch_bounds__(kThreads4, 1)
         float y[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) y[i] = fmaf(a.sg, __uint_as_float(v[i]), RP > 0 ? __uint_as_float(b[i]) : 0.0f);
+        if (a.bias) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int n = n0 + 32 * c + 8 * j;
+            if (n >= a.N) continue;
+            const float4 b0 = reinterpret_cast<const float4*>(a.bias + n)[0];
+            const float4 b1 = reinterpret_cast<const float4*>(a.bias + n)[1];
+            y[8 * j] += b0.x; y[8 * j + 1] += b0.y; y[8 * j + 2] += b0.z; y[8 * j + 3] += b0.w;
+            y[8 * j + 4] += b1.x; y[8 * j + 5] += b1.y; y[8 * j + 6] += b1.z; y[8 * j + 7] += b1.w;
+          }
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const int n = n0 + 32 * c + 8 * j;  // N is a multiple of 8
@@ -320,6 +332,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, void*
   a.sg = h.sg;
   a.Y = Y;
   a.y_f32 = y_f32 ? 1 : 0;
+  a.bias = h.bias;
   a.err = h.err;
   a.timeout_ns = deadline_budget_ns(h);
   static bool attr_done = false;
