@@ -16,7 +16,8 @@ the layer shards by rows with no collective); weak scaling.
 
 The NVFP4 variant (App. B.1: E2M1 with an E4M3 scale per 16 K, block scales applied by the
 tensor cores) is timed on the same workload and reported under `variants`; `--format nvfp4` makes
-it the headline.
+it the headline.  So is the layer with smoothing and the block Hadamard rotation in front (Sec. 2
+Eq. (pair)); `--rotate` makes that the headline (three launches per step with r > 0).
 """
 from __future__ import annotations
 
@@ -39,6 +40,7 @@ METRIC = "ASP W4A4+low-rank linear effective TOPS (2*M*N*K per step)"
 UNIT = "TOPS"
 WORKLOAD = dict(workload="dit_attn_proj_M4096_K3072_N3072_r32_g64", M=4096, K=3072, N=3072, r=32, group=64)
 ROTATE_SETS = 6  # distinct input/output/workspace/weight sets cycled through (> L2 in total)
+ROTATION = "smoothing alpha 0.5 + block Hadamard B 1024 in front of the layer (Eq. (pair))"
 
 
 def parse():
@@ -49,6 +51,9 @@ def parse():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--cpu-rows", type=int, default=0, help="oracle sample rows (0 = sized to ~10 s)")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--rotate", action="store_true",
+                   help="headline layer with smoothing (alpha 0.5) and the block Hadamard rotation in front "
+                        "(Eq. (pair)); also measured as a variant of the default run")
     p.add_argument("--format", choices=["int4", "nvfp4"], default="int4",
                    help="4-bit format of the headline: INT4 group 64 (the configuration's), or NVFP4 "
                         "(App. B.1's Blackwell format, also measured as a variant of the INT4 run)")
@@ -156,20 +161,38 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ CPU oracle (baseline / reference arm)
 
-def oracle_sample(rows: int, nvfp4: bool = False):
-    """Inputs and packed weights for the oracle timing: the workload's first `rows` tokens."""
+def oracle_sample(rows: int, nvfp4: bool = False, rotate: bool = False):
+    """Inputs and packed weights for the oracle timing: the workload's first `rows` tokens; with
+    `rotate`, smoothing factors (alpha 0.5, from the batch's channel maxima) for Eq. (pair)."""
     import oracle
+    from oracle import subspace
     from paper_2609_33269_gb300 import workloads as wl
     layer = wl.dit_attention().layers[0]
-    Xb = layer.x()[:rows].copy()
+    Xall = layer.x()
+    Xb = Xall[:rows].copy()
     U = layer.u()
+    s = None
+    W = layer.w()
+    if rotate:
+        xmax = np.abs(oracle.bf16_bits_to_f64(Xall)).max(axis=0)
+        s = subspace.smoothing_factors(xmax, oracle.bf16_bits_to_f64(W), 0.5)
     # offline packing: outside the timed sample
-    wts = oracle.pack_nvfp4(layer.w(), U) if nvfp4 else oracle.pack(layer.w(), U, layer.G)
+    if rotate:
+        Wt = oracle.rotate_weights(W, s)
+        wts = oracle.pack_nvfp4_f64(Wt, U) if nvfp4 else oracle.pack_f64(Wt, U, layer.G)
+    else:
+        wts = oracle.pack_nvfp4(W, U) if nvfp4 else oracle.pack(W, U, layer.G)
+    layer.s = s
     return Xb, U, wts, layer
 
 
-def oracle_step(Xb, U, wts, G, nvfp4: bool = False):
+def oracle_step(Xb, U, wts, G, nvfp4: bool = False, s=None, rotate: bool = False):
     import oracle
+    if rotate:
+        Xt = oracle.rotate_acts(Xb, s)
+        if nvfp4:
+            return oracle.linear_nvfp4(oracle.quantize_act_nvfp4_f64(Xt, U), wts)
+        return oracle.linear(oracle.quantize_act_f64(Xt, U, G), wts, G)
     if nvfp4:
         return oracle.linear_nvfp4(oracle.quantize_act_nvfp4(Xb, U), wts)
     act = oracle.quantize_act(Xb, U, G)
@@ -189,19 +212,20 @@ def run_reference(args):
         return 0
     K, N = WORKLOAD["K"], WORKLOAD["N"]
     nv = args.format == "nvfp4"
+    rot = args.rotate
     rows = args.cpu_rows
     if not rows:  # size each step so that warm-up + timed steps take about two minutes
-        Xb, U, wts, layer = oracle_sample(8, nv)
+        Xb, U, wts, layer = oracle_sample(8, nv, rot)
         t0 = time.perf_counter()
-        oracle_step(Xb, U, wts, layer.G, nv)
+        oracle_step(Xb, U, wts, layer.G, nv, layer.s, rot)
         per_row = (time.perf_counter() - t0) / 8
         rows = int(max(1, min(256, 120.0 / (max(1, args.steps + args.warmup) * per_row))))
-    Xb, U, wts, layer = oracle_sample(rows, nv)
+    Xb, U, wts, layer = oracle_sample(rows, nv, rot)
     for _ in range(max(0, args.warmup)):
-        oracle_step(Xb, U, wts, layer.G, nv)
+        oracle_step(Xb, U, wts, layer.G, nv, layer.s, rot)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle_step(Xb, U, wts, layer.G, nv)
+        oracle_step(Xb, U, wts, layer.G, nv, layer.s, rot)
     dt = time.perf_counter() - t0
     value = 2.0 * rows * N * K * args.steps / dt / 1e12
     line = {
@@ -209,7 +233,8 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": dict(WORKLOAD, sample_rows_per_step=rows, parallelism="host cores",
-                                            format="nvfp4 (block 16)" if nv else "int4 (group 64)"),
+                                            format="nvfp4 (block 16)" if nv else "int4 (group 64)",
+                                            **({"rotation": ROTATION} if rot else {})),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                          "sample": f"{rows} of 4096 token rows per step (quantize + output); packing offline"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -218,15 +243,15 @@ def run_reference(args):
     return 0
 
 
-def cpu_baseline(rows_req: int, nvfp4: bool = False):
+def cpu_baseline(rows_req: int, nvfp4: bool = False, rotate: bool = False):
     """The oracle as it stands on the host cores: whole passes over a sample of the workload's
     rows, repeated until about ten seconds of CPU work (packing excluded, as on the GPU)."""
     K, N = WORKLOAD["K"], WORKLOAD["N"]
     rows = rows_req or WORKLOAD["M"]
-    Xb, U, wts, layer = oracle_sample(rows, nvfp4)
+    Xb, U, wts, layer = oracle_sample(rows, nvfp4, rotate)
     reps, t0 = 0, time.perf_counter()
     while True:
-        oracle_step(Xb, U, wts, layer.G, nvfp4)
+        oracle_step(Xb, U, wts, layer.G, nvfp4, layer.s, rotate)
         reps += 1
         dt = time.perf_counter() - t0
         if dt >= 10.0 or reps >= 50:
@@ -429,8 +454,12 @@ def run_ours(args):
 
     fmt = asp.QWAM_FMT_NVFP4 if args.format == "nvfp4" else asp.QWAM_FMT_INT4
     nsteps = args.steps
+    # smoothing factors (alpha = 0.5, from this batch's channel maxima) for the rotated layer
+    xmax = X0.float().abs().amax(dim=0).contiguous()
+    smooth = torch.empty(K, dtype=torch.float32, device=dev)
+    asp.qwam_asp_smoothing_factors(xmax, W, K, N, 0.5, smooth, stream)
     clocks = ClockSampler(local)
-    main_run = timed(fmt, nsteps, args.warmup, clocks)
+    main_run = timed(fmt, nsteps, args.warmup, clocks, smooth=smooth if args.rotate else None)
     sets, total_ms, t_a, t_b = main_run["sets"], main_run["total_ms"], main_run["t_a"], main_run["t_b"]
     value = main_run["value"]
     working_mb = main_run["mb"]
@@ -486,7 +515,7 @@ def run_ours(args):
     r_pad = sets[0][0].r_pad
     kern, roof, layer_frac = rooflines(fmt, t_a, t_b, total_ms / nsteps, r_pad)
     variants = {}
-    if fmt == asp.QWAM_FMT_INT4:
+    if fmt == asp.QWAM_FMT_INT4 and not args.rotate:
         for lin_, *_ in sets:
             lin_.close()
         sets = []
@@ -500,12 +529,9 @@ def run_ours(args):
         for s_ in vr["sets"]:
             s_[0].close()
         variants["small_m"] = small_m_latencies(asp, wl, dev, stream, dev_bf16)
-        # Smoothing (alpha = 0.5, factors from this batch's channel maxima) and the block Hadamard
-        # rotation (B = 1024) in front of the same layer: kernel (a) writes the float32 remainder,
-        # the rotation kernel rotates and quantizes it (two launches in qwam_asp_quantize_act).
-        xmax = X0.float().abs().amax(dim=0).contiguous()
-        smooth = torch.empty(K, dtype=torch.float32, device=dev)
-        asp.qwam_asp_smoothing_factors(xmax, W, K, N, 0.5, smooth, stream)
+        # Smoothing and the block Hadamard rotation (B = 1024) in front of the same layer: kernel (a)
+        # writes the float32 remainder, the rotation kernel rotates and quantizes it (two launches
+        # in qwam_asp_quantize_act).
         rr = timed(asp.QWAM_FMT_INT4, vsteps, max(3, min(args.warmup, 20)), smooth=smooth)
         a_fused = alg_bytes_actquant(M, K, r_pad, G)
         a_split = a_fused + 4 * M * K * 2 + 4 * K  # the float32 remainder written and read back, 1/s
@@ -527,11 +553,12 @@ def run_ours(args):
         "dtype": "e2m1" if fmt == asp.QWAM_FMT_NVFP4 else "e4m3", "data": "synthetic",
         "config": dict(WORKLOAD, parallelism=f"replicas by token rows x{world}",
                        format="nvfp4 (block 16)" if fmt == asp.QWAM_FMT_NVFP4 else "int4 (group 64)",
-                       l2="rotating buffers: %d sets, %.0f MB > L2" % (ROTATE_SETS, working_mb)),
+                       l2="rotating buffers: %d sets, %.0f MB > L2" % (ROTATE_SETS, working_mb),
+                       **({"rotation": ROTATION} if args.rotate else {})),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 2 * M * K, "d2h_bytes_per_step": 2 * M * N,
                 "steps": e2e_steps,
                 "pipeline": "copies on their own streams, overlapping the layer of the neighbouring steps"},
-        "gpu_launches": 2 * nsteps,
+        "gpu_launches": (3 if args.rotate and r > 0 else 2) * nsteps,
         "roofline": roof,
         "layer_roofline_frac": layer_frac,
         "kernels": kern,
@@ -539,7 +566,7 @@ def run_ours(args):
         "clocks": clocks.summary(),
     }
     if not args.no_cpu_baseline and world == 1:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_rows, fmt == asp.QWAM_FMT_NVFP4)
+        line["cpu_baseline"] = cpu_baseline(args.cpu_rows, fmt == asp.QWAM_FMT_NVFP4, args.rotate)
     print(json.dumps(line))
     for s_ in sets:
         s_[0].close()
