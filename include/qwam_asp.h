@@ -232,7 +232,8 @@ qwam_status qwam_asp_shape(qwam_asp_handle h, int* K, int* N, int* r, int* group
  *   qw  : uint8 [N, K/2] codes of W_perp, low nibble = even k (two's complement)
  *   sw  : uint16 (float16 bits) [K/group, N]
  *   Bh  : uint16 (float16 bits) [N, r_pad]   (B_hat transposed, zero beyond r)
- *   Uhl : uint16 (bf16 bits) [2, K, r_pad]   (hi and lo parts of U, zero beyond r) */
+ *   Uhl : uint16 (bf16 bits) [2, K, r_pad]   (hi and lo parts of the projection basis: U, or
+ *         diag(s)^-1 H U for a rotated handle; zero beyond r) */
 qwam_status qwam_asp_export(qwam_asp_handle h, void* qw, void* sw, void* Bh, void* Uhl);
 
 /* Free the handle and its device buffers (synchronizes the device). */

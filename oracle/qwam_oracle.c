@@ -36,7 +36,7 @@
  *   R5  codes are taken against the stored (rounded) scale; a zero scale gives zero codes.
  *   R6  the "16-bit" branch is float16: p_hat = RN_f16(x U), B_hat = RN_f16(U^T W).
  *   R7  the branch uses float64 B_f = U^T W for the deflation, B_hat only for the output.
- *   R8  on float64 activations (the rotated x~) the scale is RN_f32(RN_f64(amax / 7)).
+ *   R11 on float64 activations (the rotated x~) the scale is RN_f32(RN_f64(amax / 7)).
  */
 #include <math.h>
 #include <stdint.h>
