@@ -321,6 +321,13 @@ qwam_status qwam_asp_select_experts(const double* mass, const double* cost, int 
 /* Set the bound of every device wait of this handle's kernels, in seconds (default 2.0). */
 qwam_status qwam_asp_set_timeout(qwam_asp_handle h, double seconds);
 
+/* Activation path for few tokens.  Calls with M <= max_rows tokens (default 256) on a handle
+ * without rotation and with K % 256 == 0 run the activation side on the CUDA cores, one CTA per
+ * token (float32 projection and remainder, the same quantizers); larger M take the tensor-core
+ * kernel.  Both meet the same parity bars; max_rows = 0 always takes the tensor-core kernel.
+ * Errors: QWAM_ERR_INVALID_ARG (no handle, max_rows < 0). */
+qwam_status qwam_asp_set_small_m(qwam_asp_handle h, int max_rows);
+
 /* Launch one CTA that waits on a shared-memory barrier nothing arrives on, with a bound of
  * `timeout_us` microseconds; the wait runs out, the kernel records QWAM_ERR_TIMEOUT in the
  * handle's error word and returns.  Exercises the bounded-wait path without a fault. */

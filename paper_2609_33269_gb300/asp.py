@@ -41,7 +41,7 @@ EXPORTED = [
     "qwam_asp_debug_quantize_rows", "qwam_asp_smoothing_factors", "qwam_asp_rotated_gramian",
     "qwam_asp_gramian_trace", "qwam_asp_subspace_workspace_bytes", "qwam_asp_action_subspace",
     "qwam_asp_select_experts", "qwam_asp_pack_weights_rotated", "qwam_asp_pack_weights_nvfp4_rotated",
-    "qwam_asp_rotation", "qwam_asp_set_bias",
+    "qwam_asp_rotation", "qwam_asp_set_bias", "qwam_asp_set_small_m",
 ]
 
 _lib = None
@@ -95,6 +95,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_pack_weights_nvfp4_rotated.argtypes = [V, V, V, I, I, I, V, ctypes.POINTER(H)]
         lib.qwam_asp_rotation.argtypes = [H, ctypes.POINTER(I)]
         lib.qwam_asp_set_bias.argtypes = [H, V, V]
+        lib.qwam_asp_set_small_m.argtypes = [H, I]
         lib.qwam_asp_export_nvfp4.argtypes = [H, V, V, ctypes.POINTER(ctypes.c_float), V]
         for name in EXPORTED:
             if name != "qwam_status_string":
@@ -158,6 +159,11 @@ def qwam_asp_pack_weights_nvfp4_rotated(W_bf16, s, U, K: int, N: int, r: int, st
 def qwam_asp_set_bias(h: int, bias, stream=None):
     """Bias [N] float32 (device) added in the GEMM epilogue; None removes it."""
     _check(load().qwam_asp_set_bias(h, _ptr(bias), _stream(stream)), "qwam_asp_set_bias")
+
+
+def qwam_asp_set_small_m(h: int, max_rows: int):
+    """Token counts up to max_rows take the small-M (CUDA-core) activation kernel; 0 never."""
+    _check(load().qwam_asp_set_small_m(h, int(max_rows)), "qwam_asp_set_small_m")
 
 
 def qwam_asp_rotation(h: int) -> int:

@@ -614,14 +614,20 @@ __global__ void __launch_bounds__(128) debug_quantize_kernel(const float* R, int
 // (shuffles) and 256, 512 across the lane's sub-blocks.  The normalisation 1/sqrt(B) is folded
 // into the per-channel factor applied first, RN_f32(1 / (sqrt(B) s_k)).  A quantization group
 // (32 or 64 channels) is 4 or 8 neighbouring lanes, an NVFP4 block (16) two.
-struct RotArgs {
-  int M, K, G, M_pad;
-  const float* inv_s;  // [K]: RN_f32(1 / (sqrt(B) s_k))
+// Where the lane quantizers below write: the activation workspace of one handle.
+struct QuantOut {
+  int K, G, M_pad;
   uint8_t* codes;
   uint8_t* sf;
   float* scales;
   float2* ab;
+};
+
+struct RotArgs {
+  int M, K;
+  const float* inv_s;  // [K]: RN_f32(1 / (sqrt(B) s_k))
   float* dump;
+  QuantOut q;
 };
 
 __device__ __forceinline__ void load8(const __nv_bfloat16* p, float* v) {
@@ -659,6 +665,59 @@ __device__ __forceinline__ uint32_t codes8_nvfp4(const float* x, float sc, float
   }
   const uint32_t nz = ((w & 0x77777777u) + 0x77777777u) & 0x88888888u;
   return w & (0x77777777u | nz);
+}
+
+// The quantizers of kernel (a) on a warp-wide layout: each lane holds 8 consecutive remainder
+// values x (channels k .. k+7 of token row m, k a multiple of 8) and the lanes of one quantization
+// group (INT4: G/8 lanes; NVFP4: 2 lanes per block of 16) are neighbours.  Writes the codes and,
+// from the group's first lane, its scale (and, for INT4, the epilogue constants).  The scale, the
+// codes and the constants are those of quantize_group / quantize_block_nvfp4, bit for bit.
+template <bool NV>
+__device__ __forceinline__ void quantize8_lanes(const float* x, int lane, int m, int k, const QuantOut& o) {
+  constexpr unsigned kAll = 0xFFFFFFFFu;
+  float am = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
+  if constexpr (NV) {
+    am = fmaxf(am, __shfl_xor_sync(kAll, am, 1));
+    const uint32_t sb = cvt_e4m3(__fdiv_rn(am, 6.0f));
+    const float sc = e4m3_value(sb);
+    const uint32_t w = codes8_nvfp4(x, sc, sc > 0.0f ? rcp_approx(sc) : 0.0f);
+    *reinterpret_cast<uint32_t*>(o.codes + static_cast<size_t>(m) * (o.K / 2) + k / 2) = w;
+    if ((lane & 1) == 0) {
+      const int mr = m % kBM;
+      o.sf[(static_cast<size_t>(m / kBM) * (o.K / 64) + k / 64) * kSfAtom + (mr % 32) * 16 + (mr / 32) * 4 +
+           (k % 64) / kFp4Block] = static_cast<uint8_t>(sb);
+    }
+  } else {
+    am = fmaxf(am, __shfl_xor_sync(kAll, am, 1));
+    am = fmaxf(am, __shfl_xor_sync(kAll, am, 2));
+    if (o.G == 64) am = fmaxf(am, __shfl_xor_sync(kAll, am, 4));
+    const float sc = __fdiv_rn(am, 7.0f);
+    const float ks = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100 (see quantize_group)
+    const float scs = sc * ks;
+    const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
+    const float hs = 0.5f * scs;
+    uint32_t b[8];
+    int sum = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int ci = nearest_code(x[i] * ks, scs, inv, hs);
+      sum += ci;
+      b[i] = static_cast<uint32_t>(abs(ci)) | (static_cast<uint32_t>(ci) & 0x80u);
+    }
+    sum += __shfl_xor_sync(kAll, sum, 1);
+    sum += __shfl_xor_sync(kAll, sum, 2);
+    if (o.G == 64) sum += __shfl_xor_sync(kAll, sum, 4);
+    const uint32_t w0 = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+    const uint32_t w1 = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
+    *reinterpret_cast<uint2*>(o.codes + static_cast<size_t>(m) * o.K + k) = make_uint2(w0, w1);
+    if ((lane & (o.G / 8 - 1)) == 0) {
+      const size_t gi = static_cast<size_t>(k / o.G) * o.M_pad + m;
+      o.scales[gi] = sc;
+      o.ab[gi] = make_float2(sc * 262144.0f, (-8.0f * sc) * static_cast<float>(sum));
+    }
+  }
 }
 
 template <typename TIn, int NSUB, bool NV>
@@ -725,51 +784,21 @@ __global__ void __launch_bounds__(256, 4) rotquant_kernel(const TIn* __restrict_
         d[0] = make_float4(x[0], x[1], x[2], x[3]);
         d[1] = make_float4(x[4], x[5], x[6], x[7]);
       }
-      float am = 0.0f;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
-      if constexpr (NV) {
-        am = fmaxf(am, __shfl_xor_sync(kAll, am, 1));
-        const uint32_t sb = cvt_e4m3(__fdiv_rn(am, 6.0f));
-        const float sc = e4m3_value(sb);
-        const uint32_t w = codes8_nvfp4(x, sc, sc > 0.0f ? rcp_approx(sc) : 0.0f);
-        *reinterpret_cast<uint32_t*>(a.codes + static_cast<size_t>(m) * (a.K / 2) + k / 2) = w;
-        if ((lane & 1) == 0) {
-          const int mr = m % kBM;
-          a.sf[(static_cast<size_t>(m / kBM) * (a.K / 64) + k / 64) * kSfAtom + (mr % 32) * 16 + (mr / 32) * 4 +
-               (k % 64) / kFp4Block] = static_cast<uint8_t>(sb);
-        }
-      } else {
-        am = fmaxf(am, __shfl_xor_sync(kAll, am, 1));
-        am = fmaxf(am, __shfl_xor_sync(kAll, am, 2));
-        if (a.G == 64) am = fmaxf(am, __shfl_xor_sync(kAll, am, 4));
-        const float sc = __fdiv_rn(am, 7.0f);
-        const float ks = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100 (see quantize_group)
-        const float scs = sc * ks;
-        const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
-        const float hs = 0.5f * scs;
-        uint32_t b[8];
-        int sum = 0;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int ci = nearest_code(x[i] * ks, scs, inv, hs);
-          sum += ci;
-          b[i] = static_cast<uint32_t>(abs(ci)) | (static_cast<uint32_t>(ci) & 0x80u);
-        }
-        sum += __shfl_xor_sync(kAll, sum, 1);
-        sum += __shfl_xor_sync(kAll, sum, 2);
-        if (a.G == 64) sum += __shfl_xor_sync(kAll, sum, 4);
-        const uint32_t w0 = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
-        const uint32_t w1 = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
-        *reinterpret_cast<uint2*>(a.codes + static_cast<size_t>(m) * a.K + k) = make_uint2(w0, w1);
-        if ((lane & (a.G / 8 - 1)) == 0) {
-          const size_t gi = static_cast<size_t>(k / a.G) * a.M_pad + m;
-          a.scales[gi] = sc;
-          a.ab[gi] = make_float2(sc * 262144.0f, (-8.0f * sc) * static_cast<float>(sum));
-        }
-      }
+      quantize8_lanes<NV>(x, lane, m, k, a.q);
     }
   }
+}
+
+QuantOut quant_out(const Handle& h, const ActLayout& L, uint8_t* base) {
+  QuantOut q;
+  q.K = h.K;
+  q.G = h.G;
+  q.M_pad = L.M_pad;
+  q.codes = base + L.codes_off;
+  q.sf = base + L.scales_off;
+  q.scales = reinterpret_cast<float*>(base + L.scales_off);
+  q.ab = reinterpret_cast<float2*>(base + L.ab_off);
+  return q;
 }
 
 template <typename TIn, bool NV>
@@ -788,6 +817,137 @@ cudaError_t launch_rotquant_t(const Handle& h, const TIn* in, const RotArgs& a, 
     case 256: return cudaLaunchKernelEx(&cfg, rotquant_kernel<TIn, 1, NV>, in, a);
     case 512: return cudaLaunchKernelEx(&cfg, rotquant_kernel<TIn, 2, NV>, in, a);
     case 1024: return cudaLaunchKernelEx(&cfg, rotquant_kernel<TIn, 4, NV>, in, a);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+// ---- small-M activation path ------------------------------------------------------------------
+//
+// For a few token rows (the action-expert layers) the phases of kernel (a) -- TMA ring, tensor-core
+// projection, cluster reduction, tensor-core reconstruction -- are mostly latency in series.  Here
+// one CTA of four warps takes one token row on the CUDA cores, in float32:
+//   p = x U        (per column, fma over the lane's channels in ascending order, then a fixed tree
+//                   over the lanes and the four warps),
+//   p_hat = RN_f16(p),
+//   x_perp = x - p U^T  (per channel, fma over j ascending, then one subtraction),
+// and the quantizers of kernel (a).  Lane l of warp w holds channels 256 c + 8 l .. + 7 of the
+// 256-channel chunks c = w, w + 4, ...  The bases are the handle's float32 copies, transposed
+// ([RP, K], zero rows beyond r), so that a warp reads 1 KB of one column per load.
+struct SmallArgs {
+  int M, K;
+  const float* up;  // [RP, K] projection basis
+  const float* ur;  // [RP, K] reconstruction basis
+  __half* phat;     // [M, RP]
+  float* dump;      // optional [M, K]: x_perp
+  QuantOut q;
+};
+
+template <int RP, bool NV>
+__global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __restrict__ X, const SmallArgs a) {
+  constexpr int RPS = RP > 0 ? RP : 1;
+  __shared__ float red[4][RPS];
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = static_cast<int>(threadIdx.x & 31), w = static_cast<int>(threadIdx.x >> 5);
+  const int m = blockIdx.x;
+  const __nv_bfloat16* row = X + static_cast<size_t>(m) * a.K;
+  const int nc = a.K / 256;
+  float p[RPS];
+  if constexpr (RP > 0) {
+    float pp[RP];
+#pragma unroll
+    for (int j = 0; j < RP; ++j) pp[j] = 0.0f;
+    for (int c = w; c < nc; c += 4) {
+      const int k = 256 * c + 8 * lane;
+      float x[8];
+      load8(row + k, x);
+      // columns in batches of 8: all of a batch's loads are issued before its fmas
+#pragma unroll
+      for (int jb = 0; jb < RP; jb += 8) {
+        float u[8][8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) load8(a.up + static_cast<size_t>(jb + j) * a.K + k, u[j]);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+#pragma unroll
+          for (int i = 0; i < 8; ++i) pp[jb + j] = fmaf(x[i], u[j][i], pp[jb + j]);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < RP; ++j)
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) pp[j] += __shfl_xor_sync(0xFFFFFFFFu, pp[j], off);
+    if (lane == 0)
+#pragma unroll
+      for (int j = 0; j < RP; ++j) red[w][j] = pp[j];
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < RP; ++j) p[j] = (red[0][j] + red[1][j]) + (red[2][j] + red[3][j]);
+    if (threadIdx.x < RP) {
+      const int j = static_cast<int>(threadIdx.x);
+      a.phat[static_cast<size_t>(m) * RP + j] = __float2half_rn((red[0][j] + red[1][j]) + (red[2][j] + red[3][j]));
+    }
+  }
+  for (int c = w; c < nc; c += 4) {
+    const int k = 256 * c + 8 * lane;
+    float x[8];
+    load8(row + k, x);
+    if constexpr (RP > 0) {
+      float acc[8] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+      for (int jb = 0; jb < RP; jb += 8) {
+        float u[8][8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) load8(a.ur + static_cast<size_t>(jb + j) * a.K + k, u[j]);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+#pragma unroll
+          for (int i = 0; i < 8; ++i) acc[i] = fmaf(p[jb + j], u[j][i], acc[i]);
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] -= acc[i];
+    }
+    if (a.dump) {
+      float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + k);
+      d[0] = make_float4(x[0], x[1], x[2], x[3]);
+      d[1] = make_float4(x[4], x[5], x[6], x[7]);
+    }
+    quantize8_lanes<NV>(x, lane, m, k, a.q);
+  }
+}
+
+template <int RP, bool NV>
+cudaError_t launch_smallq_rp(const Handle& h, const void* X, const void* ws, int M, float* dump, cudaStream_t s) {
+  const ActLayout L = act_layout(h, M);
+  uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
+  SmallArgs a;
+  a.M = M;
+  a.K = h.K;
+  a.up = h.up32;
+  a.ur = h.ur32;
+  a.phat = reinterpret_cast<__half*>(base + L.phat_off);
+  a.dump = dump;
+  a.q = quant_out(h, L, base);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(M, 1, 1);
+  cfg.blockDim = dim3(128, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, smallq_kernel<RP, NV>, static_cast<const __nv_bfloat16*>(X), a);
+}
+
+template <bool NV>
+cudaError_t launch_smallq(const Handle& h, const void* X, const void* ws, int M, float* dump, cudaStream_t s) {
+  switch (h.r_pad) {
+    case 0: return launch_smallq_rp<0, NV>(h, X, ws, M, dump, s);
+    case 16: return launch_smallq_rp<16, NV>(h, X, ws, M, dump, s);
+    case 32: return launch_smallq_rp<32, NV>(h, X, ws, M, dump, s);
+    case 48: return launch_smallq_rp<48, NV>(h, X, ws, M, dump, s);
+    case 64: return launch_smallq_rp<64, NV>(h, X, ws, M, dump, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -875,14 +1035,9 @@ cudaError_t launch_rotated(Handle& h, const ActMaps& am, const void* X, const vo
   RotArgs a;
   a.M = M;
   a.K = h.K;
-  a.G = h.G;
-  a.M_pad = L.M_pad;
   a.inv_s = h.inv_s;
-  a.codes = base + L.codes_off;
-  a.sf = base + L.scales_off;
-  a.scales = reinterpret_cast<float*>(base + L.scales_off);
-  a.ab = reinterpret_cast<float2*>(base + L.ab_off);
   a.dump = dump;
+  a.q = quant_out(h, L, base);
   if (h.r == 0) return launch_rotquant_t<__nv_bfloat16, NV>(h, static_cast<const __nv_bfloat16*>(X), a, s);
   float* resid = reinterpret_cast<float*>(base + L.resid_off);
   cudaError_t e = launch_fmt<NV>(h, am, ws, M, resid, true, s);
@@ -906,6 +1061,8 @@ cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4,
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
   const bool nv = h.fmt == kFmtNvfp4;
   if (h.rot) return nv ? launch_rotated<true>(h, am, am.x, ws, M, dump, s) : launch_rotated<false>(h, am, am.x, ws, M, dump, s);
+  if (M <= h.small_m && h.K % 256 == 0)
+    return nv ? launch_smallq<true>(h, am.x, ws, M, dump, s) : launch_smallq<false>(h, am.x, ws, M, dump, s);
   return nv ? launch_fmt<true>(h, am, ws, M, dump, false, s) : launch_fmt<false>(h, am, ws, M, dump, false, s);
 }
 

@@ -211,7 +211,8 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
   const size_t b_ut = qwam::up256(static_cast<size_t>(2 * h.r_pad) * K * 2);
   const size_t b_u3 = qwam::up256(static_cast<size_t>(K) * h.ku3 * 2);
   const size_t b_is = rot ? qwam::up256(static_cast<size_t>(K) * 4) : 0;
-  const size_t total = b_qw + b_sw + b_s32 + b_bh + b_ut + b_u3 + b_is + 256;
+  const size_t b_u32 = qwam::up256(static_cast<size_t>(K) * h.r_pad * 4);
+  const size_t total = b_qw + b_sw + b_s32 + b_bh + b_ut + b_u3 + b_is + 2 * b_u32 + 256;
   if (cudaMalloc(&h.block, total) != cudaSuccess) {
     cudaGetLastError();
     delete hs;
@@ -230,7 +231,13 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
   h.ucat_t = reinterpret_cast<__nv_bfloat16*>(q + b_bh);
   h.ucat3 = reinterpret_cast<__nv_bfloat16*>(q + b_bh + b_ut);
   if (rot) h.inv_s = reinterpret_cast<float*>(q + b_bh + b_ut + b_u3);
-  h.err = reinterpret_cast<int*>(q + b_bh + b_ut + b_u3 + b_is);
+  if (h.r_pad > 0) {
+    // without rotation both bases are U: one copy, so the small-M kernel's reconstruction reads
+    // what its projection just brought into L1
+    h.up32 = reinterpret_cast<float*>(q + b_bh + b_ut + b_u3 + b_is);
+    h.ur32 = rot ? reinterpret_cast<float*>(q + b_bh + b_ut + b_u3 + b_is + b_u32) : h.up32;
+  }
+  h.err = reinterpret_cast<int*>(q + b_bh + b_ut + b_u3 + b_is + 2 * b_u32);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   bool ok = true;
@@ -561,6 +568,12 @@ qwam_status qwam_asp_set_bias(qwam_asp_handle hs, const float* bias, struct CUst
   cudaError_t e = cudaMemcpyAsync(h.bias, bias, sizeof(float) * static_cast<size_t>(h.N), cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   return from_cuda_status(e);
+}
+
+qwam_status qwam_asp_set_small_m(qwam_asp_handle hs, int max_rows) {
+  if (!hs || max_rows < 0) return QWAM_ERR_INVALID_ARG;
+  hs->h.small_m = max_rows;
+  return QWAM_OK;
 }
 
 qwam_status qwam_asp_set_timeout(qwam_asp_handle hs, double seconds) {

@@ -66,6 +66,9 @@ struct Handle {
   int hb = 0;                        // Hadamard block: largest power of two dividing K, <= 1024
   float* inv_s = nullptr;            // [K]: RN_f32(1 / (sqrt(hb) s_k)) (s_k = 1 without smoothing)
   float* bias = nullptr;             // optional float32 [N], added in the GEMM epilogue (own allocation)
+  float* up32 = nullptr;             // [r_pad, K] float32 projection basis (U, or diag(s)^-1 H U), transposed
+  float* ur32 = nullptr;             // [r_pad, K] float32 reconstruction basis (U, or diag(s) H U), transposed
+  int small_m = 256;                 // token counts up to this take the small-M activation kernel
   double timeout_s = 2.0;
   CUtensorMap qw_map, sw32_map, Bh_map, ucat_t_map, ucat3_map;
   CUtensorMap qw4_map;               // NVFP4 weight codes [N, K/2], box {128, 128}, 128-byte swizzle

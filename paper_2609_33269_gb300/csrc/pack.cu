@@ -134,6 +134,18 @@ __global__ void split_basis_kernel(const float* __restrict__ Up, const float* __
   for (int j = 3 * r_pad; j < ku3; ++j) ucat3[static_cast<size_t>(k) * ku3 + j] = __float2bfloat16_rn(0.0f);
 }
 
+// The same two bases in float32, transposed to [r_pad, K] (zero rows beyond r), for the small-M
+// activation kernel: its lanes then read consecutive channels of one column.
+__global__ void basis32_kernel(const float* __restrict__ Up, const float* __restrict__ Ur, int K, int r, int r_pad,
+                               float* __restrict__ up32, float* __restrict__ ur32) {
+  int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= K) return;
+  for (int j = 0; j < r_pad; ++j) {
+    up32[static_cast<size_t>(j) * K + k] = (j < r) ? Up[static_cast<size_t>(k) * r + j] : 0.0f;
+    if (ur32 != up32) ur32[static_cast<size_t>(j) * K + k] = (j < r) ? Ur[static_cast<size_t>(k) * r + j] : 0.0f;
+  }
+}
+
 // ---- NVFP4 variant (App. B.1: E2M1 codes, an E4M3 scale per 16 K, one float32 scale per tensor)
 
 // One thread per (output channel n, block b of 16 K): the block's absmax of |W_perp| (float64),
@@ -283,6 +295,7 @@ cudaError_t pack_nvfp4(Handle& h, const WT* W, const float* U, const float* Up, 
     if (r > 0) {
       branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
       split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+      basis32_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.up32, h.ur32);
     }
     e = cudaGetLastError();
     cudaError_t e2 = cudaStreamSynchronize(s);
@@ -310,6 +323,7 @@ cudaError_t pack_int4(Handle& h, const WT* W, const float* U, const float* Up, c
   if (r > 0) {
     branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
     split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+    basis32_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.up32, h.ur32);
   }
   e = cudaGetLastError();
   cudaError_t e2 = cudaStreamSynchronize(s);
