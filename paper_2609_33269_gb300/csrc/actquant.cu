@@ -845,6 +845,7 @@ struct SmallArgs {
 template <int RP, bool NV>
 __global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __restrict__ X, const SmallArgs a) {
   constexpr int RPS = RP > 0 ? RP : 1;
+  constexpr int JB = RP <= 16 ? RPS : 8;  // basis columns loaded per batch
   __shared__ float red[4][RPS];
   pdl_launch_dependents();
   pdl_wait();
@@ -861,14 +862,14 @@ __global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __rest
       const int k = 256 * c + 8 * lane;
       float x[8];
       load8(row + k, x);
-      // columns in batches of 8: all of a batch's loads are issued before its fmas
+      // columns in batches of JB: all of a batch's loads are issued before its fmas
 #pragma unroll
-      for (int jb = 0; jb < RP; jb += 8) {
-        float u[8][8];
+      for (int jb = 0; jb < RP; jb += JB) {
+        float u[JB][8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) load8(a.up + static_cast<size_t>(jb + j) * a.K + k, u[j]);
+        for (int j = 0; j < JB; ++j) load8(a.up + static_cast<size_t>(jb + j) * a.K + k, u[j]);
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
+        for (int j = 0; j < JB; ++j)
 #pragma unroll
           for (int i = 0; i < 8; ++i) pp[jb + j] = fmaf(x[i], u[j][i], pp[jb + j]);
       }
@@ -895,12 +896,12 @@ __global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __rest
     if constexpr (RP > 0) {
       float acc[8] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-      for (int jb = 0; jb < RP; jb += 8) {
-        float u[8][8];
+      for (int jb = 0; jb < RP; jb += JB) {
+        float u[JB][8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) load8(a.ur + static_cast<size_t>(jb + j) * a.K + k, u[j]);
+        for (int j = 0; j < JB; ++j) load8(a.ur + static_cast<size_t>(jb + j) * a.K + k, u[j]);
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
+        for (int j = 0; j < JB; ++j)
 #pragma unroll
           for (int i = 0; i < 8; ++i) acc[i] = fmaf(p[jb + j], u[j][i], acc[i]);
       }
