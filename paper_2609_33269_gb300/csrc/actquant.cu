@@ -244,7 +244,7 @@ __global__ void __launch_bounds__(320, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1);
+      mbar_init(&empty[i], 4);  // pass 2: the four warps of one chunk parity; pass 1: the MMA commit + 3
     }
     mbar_init(proj_done, 1);
     mbar_init(arec_ready, 8);   // epilogue warps
@@ -323,6 +323,10 @@ __global__ void __launch_bounds__(320, 1)
             for (int kk = 0; kk < 4; ++kk)
               mma_f16(tmem, smem_desc(xa + kk * 32, 16, 1024, kSw128), smem_desc(ua + kk * 32, 16, 1024, kSw128),
                       idesc_proj, (c | kk) != 0);
+            // the stage frees when these MMAs complete (the commit is the last of four arrivals)
+            mbar_arrive(&empty[s]);
+            mbar_arrive(&empty[s]);
+            mbar_arrive(&empty[s]);
             mma_commit(&empty[s]);
           }
           __syncwarp();
@@ -513,10 +517,9 @@ __global__ void __launch_bounds__(320, 1)
         }
       }
       // The stage goes back to the TMA producer: order these generic-proxy reads before the
-      // async-proxy write that will refill it, then release it once all 128 readers are done.
+      // async-proxy write that will refill it; each of the four warps that read it releases it.
       fence_proxy_async_smem();
-      named_bar_sync(1 + par, 128);
-      if (et == par * 128) mbar_arrive(&empty[s]);
+      warp_arrive(&empty[s]);
       if (!ok || m >= a.M) continue;
 
       const int kc = k0 + c * kChunk;
