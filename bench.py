@@ -17,7 +17,9 @@ the layer shards by rows with no collective); weak scaling.
 The NVFP4 variant (App. B.1: E2M1 with an E4M3 scale per 16 K, block scales applied by the
 tensor cores) is timed on the same workload and reported under `variants`; `--format nvfp4` makes
 it the headline.  So is the layer with smoothing and the block Hadamard rotation in front (Sec. 2
-Eq. (pair)); `--rotate` makes that the headline (three launches per step with r > 0).
+Eq. (pair)); `--rotate` makes that the headline (three launches per step with r > 0).  The
+denoising-step layer sweep (30 DiT blocks, ASP on a third of them) is reported per format under
+`variants.sweep_int4` / `variants.sweep_nvfp4`.
 """
 from __future__ import annotations
 
@@ -326,6 +328,85 @@ def small_m_latencies(asp, wl, dev, stream, dev_bf16):
             "layers": out}
 
 
+def denoise_sweep(asp, wl, dev, stream, fmt, steps):
+    """The denoising-step layer sweep: 30 DiT blocks x {qkv 3072->9216, o 3072->3072, up
+    3072->12288, down 12288->3072} at M = 4096 tokens, ASP (r = 32) on the workload's seeded third of
+    the blocks and r = 0 elsewhere, over `steps` denoising steps with a fresh activation set each
+    step.  Weights, bases and activations are drawn on the device (seeded torch generator) with the
+    recipe's distributions, so that the 120 layers pack in seconds; every layer is packed once.
+    Two activation sets per input width alternate, so a layer's input may still be in L2 from an
+    earlier layer, as the previous layer's output would be in a model.  Returns aggregate effective
+    TOPS over all layer calls and a breakdown by layer kind and rank."""
+    import torch
+    W = wl.denoise_sweep(steps=steps)
+    g = torch.Generator(device=dev)
+    g.manual_seed(0)
+    lins = []
+    for L in W.layers:
+        Wt = (torch.randn((L.K, L.N), generator=g, device=dev) / np.sqrt(L.K)).to(torch.bfloat16)
+        U = None
+        if L.r:
+            q, rr = torch.linalg.qr(torch.randn((L.K, L.r), generator=g, device=dev, dtype=torch.float64))
+            U = (q * torch.sign(torch.diagonal(rr))[None, :]).float().contiguous()
+        lins.append(asp.AspLinear(Wt, U, L.G, fmt=fmt))
+        del Wt
+    # activation sets: two per input width and step parity, 1 % outlier channels x U(10, 30), and
+    # Student-t (nu = 4) for the down projections' input
+    def draw(K, student):
+        if student:  # t(4) = N(0, 1) / sqrt(chi2(4) / 4)
+            z = torch.randn((5, 4096, K), generator=g, device=dev)
+            x = z[0] / torch.sqrt((z[1:] ** 2).sum(dim=0) / 4.0)
+            del z
+        else:
+            x = torch.randn((4096, K), generator=g, device=dev)
+            ch = torch.randperm(K, generator=g, device=dev)[: K // 100]
+            x[:, ch] *= torch.empty(K // 100, device=dev).uniform_(10.0, 30.0, generator=g)
+        return x.to(torch.bfloat16).contiguous()
+    xs = {(K, st, i): draw(K, st) for K, st in ((3072, False), (12288, True)) for i in range(2)}
+    outs = {N: torch.empty((4096, N), dtype=torch.bfloat16, device=dev) for N in (3072, 9216, 12288)}
+    ws = torch.empty(max(asp.qwam_asp_act_workspace_bytes(l.h, 4096) for l in lins), dtype=torch.uint8, device=dev)
+
+    def one_step(i, ev=None):
+        for j, (L, lin) in enumerate(zip(W.layers, lins)):
+            X = xs[(L.K, L.dist == "student_t", i % 2)]
+            if ev is not None:
+                ev[2 * j].record(stream)
+            asp.qwam_asp_linear(X, 4096, lin.h, outs[L.N], asp.QWAM_Y_BF16, ws, stream)
+            if ev is not None:
+                ev[2 * j + 1].record(stream)
+
+    one_step(0)
+    torch.cuda.synchronize()
+    for lin in lins:
+        if asp.qwam_asp_get_error(lin.h) != asp.QWAM_OK:
+            raise RuntimeError("device error in the sweep warm-up")
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * len(lins))] for _ in range(steps)]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(steps):
+        one_step(i, evs[i])
+    e1.record(stream)
+    torch.cuda.synchronize()
+    total_ms = e0.elapsed_time(e1)
+    flops = sum(2.0 * L.M * L.N * L.K for L in W.layers) * steps
+    kinds = {}
+    for j, L in enumerate(W.layers):
+        key = "%s_r%d" % (L.name.split("_", 1)[1], L.r)
+        t = sum(evs[i][2 * j].elapsed_time(evs[i][2 * j + 1]) for i in range(steps))
+        k = kinds.setdefault(key, [0.0, 0.0, 0])
+        k[0] += t
+        k[1] += 2.0 * L.M * L.N * L.K * steps
+        k[2] += steps
+    for lin in lins:
+        lin.close()
+    return {"value": flops / (total_ms * 1e-3) / 1e12, "unit": UNIT, "steps": steps,
+            "ms_per_denoising_step": total_ms / steps, "layers_per_step": len(W.layers),
+            "asp_blocks": W.note, "what": "30 DiT blocks x {qkv, o, up, down} at M = 4096, r = 32 on a third "
+            "of the blocks, r = 0 elsewhere; one qwam_asp_linear per layer; device-drawn synthetic data",
+            "by_layer": {k: {"us_per_call": round(v[0] / v[2] * 1e3, 1), "tops": round(v[1] / (v[0] * 1e-3) / 1e12, 1)}
+                         for k, v in sorted(kinds.items())}}
+
+
 def run_ours(args):
     import torch
     rank, world, local = dist_env()
@@ -529,6 +610,8 @@ def run_ours(args):
         for s_ in vr["sets"]:
             s_[0].close()
         variants["small_m"] = small_m_latencies(asp, wl, dev, stream, dev_bf16)
+        variants["sweep_int4"] = denoise_sweep(asp, wl, dev, stream, asp.QWAM_FMT_INT4, 10)
+        variants["sweep_nvfp4"] = denoise_sweep(asp, wl, dev, stream, asp.QWAM_FMT_NVFP4, 10)
         # Smoothing and the block Hadamard rotation (B = 1024) in front of the same layer: kernel (a)
         # writes the float32 remainder, the rotation kernel rotates and quantizes it (two launches
         # in qwam_asp_quantize_act).

@@ -178,6 +178,7 @@ FULL = [  # (name, M, K, N, r, dist, G) in the launch configuration the benchmar
     ("dit_attn", 4096, 3072, 3072, 32, "outlier", 64),
     ("dit_attn_g32", 4096, 3072, 3072, 32, "outlier", 32),
     ("dit_qkv", 4096, 3072, 9216, 32, "outlier", 64),
+    ("dit_qkv_r0", 4096, 3072, 9216, 0, "outlier", 64),    # the sweep's layers without ASP
     ("ffn_up", 4096, 3072, 12288, 32, "outlier", 64),
     ("ffn_down", 4096, 12288, 3072, 32, "student_t", 64),
     ("small_M32_r16", 32, 1024, 1024, 16, "outlier", 64),
