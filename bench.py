@@ -332,8 +332,9 @@ def denoise_sweep(asp, wl, dev, stream, fmt, steps):
     """The denoising-step layer sweep: 30 DiT blocks x {qkv 3072->9216, o 3072->3072, up
     3072->12288, down 12288->3072} at M = 4096 tokens, ASP (r = 32) on the workload's seeded third of
     the blocks and r = 0 elsewhere, over `steps` denoising steps with a fresh activation set each
-    step.  Weights, bases and activations are drawn on the device (seeded torch generator) with the
-    recipe's distributions, so that the 120 layers pack in seconds; every layer is packed once.
+    step.  Weights and activations are drawn on the device (seeded torch generator) with the
+    recipe's distributions, so that the 120 layers pack in seconds (the bases are the workload's
+    own); every layer is packed once.
     Two activation sets per input width alternate, so a layer's input may still be in L2 from an
     earlier layer, as the previous layer's output would be in a model.  Returns aggregate effective
     TOPS over all layer calls and a breakdown by layer kind and rank."""
@@ -344,10 +345,7 @@ def denoise_sweep(asp, wl, dev, stream, fmt, steps):
     lins = []
     for L in W.layers:
         Wt = (torch.randn((L.K, L.N), generator=g, device=dev) / np.sqrt(L.K)).to(torch.bfloat16)
-        U = None
-        if L.r:
-            q, rr = torch.linalg.qr(torch.randn((L.K, L.r), generator=g, device=dev, dtype=torch.float64))
-            U = (q * torch.sign(torch.diagonal(rr))[None, :]).float().contiguous()
+        U = torch.from_numpy(L.u()).to(dev) if L.r else None  # the workload's seeded basis (host QR)
         lins.append(asp.AspLinear(Wt, U, L.G, fmt=fmt))
         del Wt
     # activation sets: two per input width and step parity, 1 % outlier channels x U(10, 30), and

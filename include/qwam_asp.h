@@ -272,6 +272,18 @@ qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h
 qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, int group, void* codes,
                                          void* scales, struct CUstream_st* stream);
 
+/* Test support: the warp-wide quantizers of the small-M and rotation kernels (8 consecutive values
+ * per lane, a group over neighbouring lanes) on caller-given float32 rows, with the same rounding
+ * rules as qwam_asp_debug_quantize_rows; K % 256 == 0.  Outputs are written in the activation
+ * workspace's layouts with M_pad = ceil(M / 128) * 128 rows:
+ *   INT4:  codes uint8 [M, K] (E4M3 bytes of c * 2^-9), scales float32 [K/group, M_pad],
+ *          ab float32 [K/group, M_pad, 2] (the GEMM epilogue constants);
+ *   NVFP4: codes uint8 [M, K/2] (two per byte, low nibble = even k), scales uint8 E4M3 in the
+ *          512-byte atoms described above (M_pad * K/16 bytes); ab unused (may be NULL).
+ * Device pointers; codes 16-byte aligned.  Errors: QWAM_ERR_INVALID_ARG, QWAM_ERR_CUDA. */
+qwam_status qwam_asp_debug_quantize_lanes(const float* R, int M, int K, int fmt, int group, void* codes,
+                                          void* scales, void* ab, struct CUstream_st* stream);
+
 /* ---- The offline choice of what to protect (Sec. 3.2-3.3; App. A; App. B.1) -----------------
  * Calibration-time steps that pick U (the paper's V) and which experts carry a branch, from a given
  * Action Observability Gramian G (the AOG of Sec. 3.1, estimated elsewhere).  None of them needs a

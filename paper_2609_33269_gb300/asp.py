@@ -41,7 +41,7 @@ EXPORTED = [
     "qwam_asp_debug_quantize_rows", "qwam_asp_smoothing_factors", "qwam_asp_rotated_gramian",
     "qwam_asp_gramian_trace", "qwam_asp_subspace_workspace_bytes", "qwam_asp_action_subspace",
     "qwam_asp_select_experts", "qwam_asp_pack_weights_rotated", "qwam_asp_pack_weights_nvfp4_rotated",
-    "qwam_asp_rotation", "qwam_asp_set_bias", "qwam_asp_set_small_m",
+    "qwam_asp_rotation", "qwam_asp_set_bias", "qwam_asp_set_small_m", "qwam_asp_debug_quantize_lanes",
 ]
 
 _lib = None
@@ -96,6 +96,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_rotation.argtypes = [H, ctypes.POINTER(I)]
         lib.qwam_asp_set_bias.argtypes = [H, V, V]
         lib.qwam_asp_set_small_m.argtypes = [H, I]
+        lib.qwam_asp_debug_quantize_lanes.argtypes = [V, I, I, I, I, V, V, V, V]
         lib.qwam_asp_export_nvfp4.argtypes = [H, V, V, ctypes.POINTER(ctypes.c_float), V]
         for name in EXPORTED:
             if name != "qwam_status_string":
@@ -264,6 +265,11 @@ def qwam_asp_debug_residual(X_bf16, M: int, h: int, act_ws, R, stream=None):
 def qwam_asp_debug_quantize_rows(R, M: int, K: int, fmt: int, group: int, codes, scales, stream=None):
     _check(load().qwam_asp_debug_quantize_rows(_ptr(R), M, K, fmt, group, _ptr(codes), _ptr(scales),
                                                _stream(stream)), "qwam_asp_debug_quantize_rows")
+
+
+def qwam_asp_debug_quantize_lanes(R, M: int, K: int, fmt: int, group: int, codes, scales, ab=None, stream=None):
+    _check(load().qwam_asp_debug_quantize_lanes(_ptr(R), M, K, fmt, group, _ptr(codes), _ptr(scales), _ptr(ab),
+                                                _stream(stream)), "qwam_asp_debug_quantize_lanes")
 
 
 def qwam_asp_smoothing_factors(xmax, W_bf16, K: int, N: int, alpha: float, s, stream=None):

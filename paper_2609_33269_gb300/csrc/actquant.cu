@@ -956,6 +956,20 @@ cudaError_t launch_smallq(const Handle& h, const void* X, const void* ws, int M,
   }
 }
 
+// Test support: the lane quantizers (quantize8_lanes, as the small-M and rotation kernels run
+// them) applied to caller-given float32 rows, one warp per row and 256 values.
+template <bool NV>
+__global__ void __launch_bounds__(256) debug_lanes_kernel(const float* __restrict__ R, int M, const QuantOut q) {
+  const long long wg = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  const int nc = q.K / 256;
+  if (wg >= static_cast<long long>(M) * nc) return;
+  const int lane = static_cast<int>(threadIdx.x & 31);
+  const int m = static_cast<int>(wg / nc), k = static_cast<int>(wg % nc) * 256 + 8 * lane;
+  float x[8];
+  load8(R + static_cast<size_t>(m) * q.K + k, x);
+  quantize8_lanes<NV>(x, lane, m, k, q);
+}
+
 // Cluster size (CTAs along K per 128-row tile): as many as fit one wave of the GPU.
 int choose_split(int K, int tiles, int sms) {
   const int chunks = K / kChunk;
@@ -1059,6 +1073,25 @@ cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4,
     debug_quantize_kernel<true><<<grid, 128, 0, s>>>(R, M, K, G, codes, scales);
   else
     debug_quantize_kernel<false><<<grid, 128, 0, s>>>(R, M, K, G, codes, scales);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
+                                        uint8_t* scales, float2* ab, int M_pad, cudaStream_t s) {
+  QuantOut q;
+  q.K = K;
+  q.G = G;
+  q.M_pad = M_pad;
+  q.codes = codes;
+  q.sf = scales;
+  q.scales = reinterpret_cast<float*>(scales);
+  q.ab = ab;
+  const long long warps = static_cast<long long>(M) * (K / 256);
+  const int grid = static_cast<int>((warps + 7) / 8);
+  if (nvfp4)
+    debug_lanes_kernel<true><<<grid, 256, 0, s>>>(R, M, q);
+  else
+    debug_lanes_kernel<false><<<grid, 256, 0, s>>>(R, M, q);
   return cudaGetLastError();
 }
 

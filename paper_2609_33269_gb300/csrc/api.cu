@@ -370,6 +370,22 @@ qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, 
                                                            reinterpret_cast<cudaStream_t>(stream)));
 }
 
+qwam_status qwam_asp_debug_quantize_lanes(const float* R, int M, int K, int fmt, int group, void* codes, void* scales,
+                                          void* ab, struct CUstream_st* stream) {
+  if (M < 0 || K <= 0 || K % 256 != 0) return QWAM_ERR_INVALID_ARG;
+  if (fmt != QWAM_FMT_INT4 && fmt != QWAM_FMT_NVFP4) return QWAM_ERR_INVALID_ARG;
+  if (fmt == QWAM_FMT_INT4 && group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
+  if (M == 0) return QWAM_OK;
+  if (!R || !codes || !scales || !qwam::aligned16(R) || !qwam::aligned16(codes)) return QWAM_ERR_INVALID_ARG;
+  if (fmt == QWAM_FMT_INT4 && (!ab || reinterpret_cast<uintptr_t>(scales) % 4 != 0 ||
+                               reinterpret_cast<uintptr_t>(ab) % 8 != 0))
+    return QWAM_ERR_INVALID_ARG;
+  const int M_pad = qwam::round_up(M, qwam::kBM);
+  return from_cuda_status(qwam::launch_debug_quantize_lanes(
+      R, M, K, fmt == QWAM_FMT_NVFP4, fmt == QWAM_FMT_NVFP4 ? qwam::kFp4Block : group, static_cast<uint8_t*>(codes),
+      static_cast<uint8_t*>(scales), static_cast<float2*>(ab), M_pad, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 qwam_status qwam_asp_smoothing_factors(const float* xmax, const void* W_bf16, int K, int N, double alpha, float* s,
                                        struct CUstream_st* stream) {
   if (K <= 0 || N <= 0 || !xmax || !W_bf16 || !s || !(alpha >= 0.0 && alpha <= 1.0)) return QWAM_ERR_INVALID_ARG;

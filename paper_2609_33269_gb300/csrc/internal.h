@@ -100,6 +100,8 @@ cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M,
 cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
 cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
 cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s);
+cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
+                                        uint8_t* scales, float2* ab, int M_pad, cudaStream_t s);
 cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
                                        void* scales, cudaStream_t s);
 // The offline choice of what to protect (subspace.cu).

@@ -4,7 +4,9 @@
   r = 0 the remainder is X itself, so scales and codes must equal the oracle's bit for bit
   (Eq. (quant) with the stored scale; a zero scale gives zero codes).  The kernel takes a
   different internal route for scales below 2^-100; this covers it.
-* An empty input (M = 0) is accepted and launches nothing.
+* An empty input (M = 0) is accepted and launches nothing, in both formats, with and without the
+  rotation.
+* Both activation kernels (the small-M one and kernel (a)) take the tiny-group cases.
 """
 import numpy as np
 import pytest
@@ -39,11 +41,13 @@ def _tiny_rows(M, K, seed):
     return wl.f32_to_bf16_bits(x)
 
 
+@pytest.mark.parametrize("small", [256, 0], ids=["small_m", "kernel_a"])
 @pytest.mark.parametrize("G", [32, 64])
-def test_tiny_and_zero_groups_bit_exact_r0(G):
+def test_tiny_and_zero_groups_bit_exact_r0(G, small):
     M, K, N = 24, 512, 128
     c = Case(M, K, N, 0, G, seed=5, layer_id=7, Xb=_tiny_rows(M, K, seed=G))
     try:
+        asp.qwam_asp_set_small_m(c.layer.h, small)
         c.layer.quantize(c.X)
         ga = c.gpu_act()  # also checks (alpha, beta) against the codes and scales, bit for bit
         oa = c.oracle_act(want_float64=False)
@@ -61,10 +65,12 @@ def test_tiny_and_zero_groups_bit_exact_r0(G):
         c.close()
 
 
-def test_empty_input_launches_nothing():
+@pytest.mark.parametrize("kind", ["int4", "nvfp4", "int4_rotated", "nvfp4_rotated"])
+def test_empty_input_launches_nothing(kind):
     K, N, G = 256, 64, 64
     W = torch.from_numpy(wl.weight(K, N, seed=1, layer_id=0).view(np.int16)).cuda().view(torch.bfloat16)
-    layer = asp.AspLinear(W, None, G)
+    fmt = asp.QWAM_FMT_NVFP4 if kind.startswith("nvfp4") else asp.QWAM_FMT_INT4
+    layer = asp.AspLinear(W, None, G, fmt=fmt, rotate=kind.endswith("rotated"))
     try:
         X = torch.empty((0, K), dtype=torch.bfloat16, device="cuda")
         Y = torch.empty((0, N), dtype=torch.float32, device="cuda")

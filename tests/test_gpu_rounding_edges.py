@@ -1,5 +1,7 @@
-"""Directed rounding cases for kernel (a)'s quantizers, through qwam_asp_debug_quantize_rows
-(the same device functions kernel (a) runs), against the CPU oracle, bit for bit.
+"""Directed rounding cases for both quantizer implementations, against the CPU oracle, bit for bit:
+kernel (a)'s thread-per-row quantizers through qwam_asp_debug_quantize_rows, and the warp-wide ones
+of the small-M and rotation kernels through qwam_asp_debug_quantize_lanes (the same device
+functions those kernels run).
 
 Random activations reach a rounding boundary too rarely to exercise the kernels' fast paths
 where they hand over to exact decisions, so the values here are placed on and next to the
@@ -137,7 +139,45 @@ def as_rows(chunks, width, K):
     return np.concatenate(chunks).reshape(-1, K)
 
 
-def run(R, fmt, G):
+def run_lanes(R, fmt, G):
+    """The warp-wide quantizers (small-M and rotation kernels): outputs in the workspace layouts,
+    returned row-major like run()."""
+    M, K = R.shape
+    M_pad = -(-M // 128) * 128
+    Rd = torch.from_numpy(R).cuda()
+    if fmt == asp.QWAM_FMT_NVFP4:
+        codes = torch.zeros((M, K // 2), dtype=torch.uint8, device="cuda")
+        atoms = torch.zeros(M_pad * K // 16, dtype=torch.uint8, device="cuda")
+        asp.qwam_asp_debug_quantize_lanes(Rd, M, K, fmt, 16, codes, atoms)
+        torch.cuda.synchronize()
+        a = atoms.cpu().numpy()
+        r = np.arange(M)[:, None]
+        b = np.arange(K // 16)[None, :]
+        sf = a[((r // 128) * (K // 64) + b // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + b % 4]
+        return codes.cpu().numpy(), sf
+    codes = torch.zeros((M, K), dtype=torch.uint8, device="cuda")
+    scales = torch.zeros((K // G, M_pad), dtype=torch.float32, device="cuda")
+    ab = torch.zeros((K // G, M_pad, 2), dtype=torch.float32, device="cuda")
+    asp.qwam_asp_debug_quantize_lanes(Rd, M, K, fmt, G, codes, scales, ab)
+    torch.cuda.synchronize()
+    c = codes.cpu().numpy()
+    sx = scales.cpu().numpy()[:, :M].T.copy()
+    # the epilogue constants: (2^18 s_x, -8 s_x S_a), S_a the group's code sum, each rounded once
+    q = (c & 0x7F).astype(np.int32) * np.where(c & 0x80, -1, 1)
+    sa = q.reshape(M, -1, G).sum(axis=2).astype(np.float32)
+    abv = ab.cpu().numpy()[:, :M, :].transpose(1, 0, 2)
+    np.testing.assert_array_equal(abv[:, :, 0].view(np.uint32), (sx * np.float32(262144.0)).view(np.uint32))
+    np.testing.assert_array_equal(abv[:, :, 1].view(np.uint32),
+                                  ((np.float32(-8.0) * sx).astype(np.float32) * sa).astype(np.float32).view(np.uint32))
+    return c, sx
+
+
+IMPLS = {"thread_rows": None, "warp_lanes": run_lanes}
+
+
+def run(R, fmt, G, impl="thread_rows"):
+    if IMPLS[impl] is not None:
+        return IMPLS[impl](R, fmt, G)
     M, K = R.shape
     Rd = torch.from_numpy(R).cuda()
     if fmt == asp.QWAM_FMT_NVFP4:
@@ -151,11 +191,12 @@ def run(R, fmt, G):
     return codes.cpu().numpy(), scales.cpu().numpy()
 
 
+@pytest.mark.parametrize("impl", list(IMPLS))
 @pytest.mark.parametrize("G", [64, 32])
-def test_int4_rounding_on_and_next_to_ties(G):
+def test_int4_rounding_on_and_next_to_ties(G, impl):
     rng = np.random.default_rng(100 + G)
     R = as_rows(int4_groups(G, rng), G, 256)
-    b, s = run(R, asp.QWAM_FMT_INT4, G)
+    b, s = run(R, asp.QWAM_FMT_INT4, G, impl)
     q = (b & 0x7F).astype(np.int16) * np.where(b & 0x80, -1, 1)
     oq, os_ = oracle.quantize_residual(R, G)
     np.testing.assert_array_equal(s.view(np.uint32), os_.view(np.uint32))
@@ -164,10 +205,11 @@ def test_int4_rounding_on_and_next_to_ties(G):
     assert np.abs(q).max() == 7 and (q == 0).any()
 
 
-def test_nvfp4_rounding_on_and_next_to_midpoints():
+@pytest.mark.parametrize("impl", list(IMPLS))
+def test_nvfp4_rounding_on_and_next_to_midpoints(impl):
     rng = np.random.default_rng(7)
     R = as_rows(nvfp4_blocks(rng), 16, 256)
-    packed, sf = run(R, asp.QWAM_FMT_NVFP4, 16)
+    packed, sf = run(R, asp.QWAM_FMT_NVFP4, 16, impl)
     q = np.empty((R.shape[0], R.shape[1]), np.uint8)
     q[:, 0::2] = packed & 0xF
     q[:, 1::2] = packed >> 4
