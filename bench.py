@@ -299,8 +299,13 @@ def small_m_latencies(asp, wl, dev, stream, dev_bf16):
             continue
         Xs, Ws = dev_bf16(L.x()), dev_bf16(L.w())
         Us = torch.from_numpy(L.u()).to(dev) if L.r else None
-        for fmt, fname in ((asp.QWAM_FMT_INT4, "int4"), (asp.QWAM_FMT_NVFP4, "nvfp4")):
-            lin = asp.AspLinear(Ws, Us, L.G, fmt=fmt)
+        variants = [(asp.QWAM_FMT_INT4, "int4", False), (asp.QWAM_FMT_NVFP4, "nvfp4", False)]
+        if L.r:  # the same layers with smoothing (from the batch's channel maxima) and the rotation
+            variants += [(asp.QWAM_FMT_INT4, "int4_rotated", True), (asp.QWAM_FMT_NVFP4, "nvfp4_rotated", True)]
+            sm = torch.empty(L.K, dtype=torch.float32, device=dev)
+            asp.qwam_asp_smoothing_factors(Xs.float().abs().amax(dim=0).contiguous(), Ws, L.K, L.N, 0.5, sm, stream)
+        for fmt, fname, rot in variants:
+            lin = asp.AspLinear(Ws, Us, L.G, fmt=fmt, rotate=rot, s=sm if rot else None)
             Ys = torch.empty((L.M, L.N), dtype=torch.bfloat16, device=dev)
             side.wait_stream(stream)
             with torch.cuda.stream(side):
@@ -324,7 +329,8 @@ def small_m_latencies(asp, wl, dev, stream, dev_bf16):
                                               "tops": round(2.0 * L.M * L.N * L.K / us / 1e6, 2)}
             del g
             lin.close()
-    return {"what": "one qwam_asp_linear call of an action-expert layer (K=1024), CUDA graph of 20 calls",
+    return {"what": "one qwam_asp_linear call of an action-expert layer (K=1024), CUDA graph of 20 calls; "
+                    "*_rotated: with smoothing and the block Hadamard rotation in front (Eq. (pair))",
             "layers": out}
 
 

@@ -835,21 +835,27 @@ cudaError_t launch_rotquant_t(const Handle& h, const TIn* in, const RotArgs& a, 
 //   x_perp = x - p U^T  (per channel, fma over j ascending, then one subtraction),
 // and the quantizers of kernel (a).  Lane l of warp w holds channels 256 c + 8 l .. + 7 of the
 // 256-channel chunks c = w, w + 4, ...  The bases are the handle's float32 copies, transposed
-// ([RP, K], zero rows beyond r), so that a warp reads 1 KB of one column per load.
+// ([RP, K], zero rows beyond r), so that a warp reads 1 KB of one column per load.  For a rotated
+// layer the bases are diag(s)^-1 H U and diag(s) H U (as for kernel (a)), and the remainder is
+// rotated before it is quantized (the rotation kernel's transform, the cross-chunk spans of a
+// Hadamard block through shared memory).
 struct SmallArgs {
   int M, K;
   const float* up;  // [RP, K] projection basis
   const float* ur;  // [RP, K] reconstruction basis
+  const float* inv_s;  // rotated layer: [K] RN_f32(1 / (sqrt(B) s_k)); the remainder is then rotated
+  int hb;              // rotated layer: Hadamard block B (256, 512 or 1024)
   __half* phat;     // [M, RP]
   float* dump;      // optional [M, K]: x_perp
   QuantOut q;
 };
 
-template <int RP, bool NV>
+template <int RP, bool NV, bool ROT>
 __global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __restrict__ X, const SmallArgs a) {
   constexpr int RPS = RP > 0 ? RP : 1;
   constexpr int JB = RP <= 16 ? RPS : 8;  // basis columns loaded per batch
   __shared__ float red[4][RPS];
+  __shared__ float4 xch[ROT ? 4 : 1][ROT ? 32 : 1][2];  // rotated layer: the four warps' chunks
   pdl_launch_dependents();
   pdl_wait();
   const int lane = static_cast<int>(threadIdx.x & 31), w = static_cast<int>(threadIdx.x >> 5);
@@ -892,8 +898,12 @@ __global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __rest
       a.phat[static_cast<size_t>(m) * RP + j] = __float2half_rn((red[0][j] + red[1][j]) + (red[2][j] + red[3][j]));
     }
   }
-  for (int c = w; c < nc; c += 4) {
-    const int k = 256 * c + 8 * lane;
+  // A rotated layer walks the chunks in rounds of four (one per warp) so that the chunks of a
+  // Hadamard block (B / 256 of them, aligned) are in the CTA at the same time.
+  const int rounds = ROT ? (nc + 3) / 4 : 0;
+  for (int c = w; ROT ? c < 4 * rounds : c < nc; c += 4) {
+    const bool live = c < nc;
+    const int k = 256 * (live ? c : 0) + 8 * lane;
     float x[8];
     load8(row + k, x);
     if constexpr (RP > 0) {
@@ -911,6 +921,55 @@ __global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __rest
 #pragma unroll
       for (int i = 0; i < 8; ++i) x[i] -= acc[i];
     }
+    if constexpr (ROT) {
+      // x~_perp = H diag(s)^-1 (x - diag(s) H U p): the channel factor (1/sqrt(B) folded in), the
+      // butterflies at spans 1, 2, 4 in the lane and 8 .. 128 across the lanes, then the
+      // chunks of one block combined through shared memory (spans 256 and 512 as one sum with
+      // the Sylvester signs).
+      float is[8];
+      load8(a.inv_s + k, is);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] *= is[i];
+#pragma unroll
+      for (int h = 1; h < 8; h *= 2)
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if ((i & h) == 0) {
+            const float x0 = x[i], x1 = x[i + h];
+            x[i] = x0 + x1;
+            x[i + h] = x0 - x1;
+          }
+#pragma unroll
+      for (int sh = 1; sh < 32; sh *= 2) {
+        const float sgn = (lane & sh) ? -1.0f : 1.0f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = fmaf(x[i], sgn, __shfl_xor_sync(0xFFFFFFFFu, x[i], sh));
+      }
+      const int nb = a.hb / 256;  // chunks per Hadamard block: 1, 2 or 4
+      if (nb > 1) {
+        xch[w][lane][0] = make_float4(x[0], x[1], x[2], x[3]);
+        xch[w][lane][1] = make_float4(x[4], x[5], x[6], x[7]);
+        __syncthreads();
+        const int cl = w & (nb - 1), w0 = w - cl;  // this chunk's index in its block, the block's first warp
+        float y[8] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+        for (int b = 0; b < nb; ++b) {
+          const float sg = (__popc(cl & b) & 1) ? -1.0f : 1.0f;
+          const float4 v0 = xch[w0 + b][lane][0], v1 = xch[w0 + b][lane][1];
+          y[0] = fmaf(sg, v0.x, y[0]);
+          y[1] = fmaf(sg, v0.y, y[1]);
+          y[2] = fmaf(sg, v0.z, y[2]);
+          y[3] = fmaf(sg, v0.w, y[3]);
+          y[4] = fmaf(sg, v1.x, y[4]);
+          y[5] = fmaf(sg, v1.y, y[5]);
+          y[6] = fmaf(sg, v1.z, y[6]);
+          y[7] = fmaf(sg, v1.w, y[7]);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = y[i];
+        __syncthreads();  // the exchange buffer is free for the next round
+      }
+    }
+    if (!live) continue;
     if (a.dump) {
       float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + k);
       d[0] = make_float4(x[0], x[1], x[2], x[3]);
@@ -922,6 +981,7 @@ __global__ void __launch_bounds__(128) smallq_kernel(const __nv_bfloat16* __rest
 
 template <int RP, bool NV>
 cudaError_t launch_smallq_rp(const Handle& h, const void* X, const void* ws, int M, float* dump, cudaStream_t s) {
+  const bool rot = h.rot;
   const ActLayout L = act_layout(h, M);
   uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
   SmallArgs a;
@@ -932,6 +992,8 @@ cudaError_t launch_smallq_rp(const Handle& h, const void* X, const void* ws, int
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
   a.dump = dump;
   a.q = quant_out(h, L, base);
+  a.inv_s = h.inv_s;
+  a.hb = h.hb;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(M, 1, 1);
   cfg.blockDim = dim3(128, 1, 1);
@@ -941,7 +1003,8 @@ cudaError_t launch_smallq_rp(const Handle& h, const void* X, const void* ws, int
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, smallq_kernel<RP, NV>, static_cast<const __nv_bfloat16*>(X), a);
+  if (rot) return cudaLaunchKernelEx(&cfg, smallq_kernel<RP, NV, true>, static_cast<const __nv_bfloat16*>(X), a);
+  return cudaLaunchKernelEx(&cfg, smallq_kernel<RP, NV, false>, static_cast<const __nv_bfloat16*>(X), a);
 }
 
 template <bool NV>
@@ -1097,9 +1160,9 @@ cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4
 
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
   const bool nv = h.fmt == kFmtNvfp4;
-  if (h.rot) return nv ? launch_rotated<true>(h, am, am.x, ws, M, dump, s) : launch_rotated<false>(h, am, am.x, ws, M, dump, s);
   if (M <= h.small_m && h.K % 256 == 0)
     return nv ? launch_smallq<true>(h, am.x, ws, M, dump, s) : launch_smallq<false>(h, am.x, ws, M, dump, s);
+  if (h.rot) return nv ? launch_rotated<true>(h, am, am.x, ws, M, dump, s) : launch_rotated<false>(h, am, am.x, ws, M, dump, s);
   return nv ? launch_fmt<true>(h, am, ws, M, dump, false, s) : launch_fmt<false>(h, am, ws, M, dump, false, s);
 }
 

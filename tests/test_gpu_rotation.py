@@ -55,9 +55,15 @@ SHAPES = [  # M, K, N, r, G, smoothing
 IDS = ["M%d_K%d_N%d_r%d_g%d_s%d" % s for s in SHAPES]
 
 
-def make_case(shape, seed):
+def make_case(shape, seed, small=256):
+    """small: token counts up to which the small-M kernel runs (0: kernel (a) + rotation kernel)."""
     M, K, N, r, G, sm = shape
-    return Case(M, K, N, r, G, seed=seed, layer_id=K + r, rotate=True, s=smoothing(K, seed) if sm else None)
+    c = Case(M, K, N, r, G, seed=seed, layer_id=K + r, rotate=True, s=smoothing(K, seed) if sm else None)
+    asp.qwam_asp_set_small_m(c.layer.h, small)
+    return c
+
+
+PATHS = pytest.mark.parametrize("small", [256, 0], ids=["small_m", "kernel_a"])
 
 
 @pytest.mark.parametrize("shape", SHAPES, ids=IDS)
@@ -82,10 +88,11 @@ def test_rotated_pack_bit_exact(shape):
         c.close()
 
 
+@PATHS
 @pytest.mark.parametrize("shape", SHAPES, ids=IDS)
-def test_rotated_quantizer_bit_exact_on_kernel_remainder(shape):
+def test_rotated_quantizer_bit_exact_on_kernel_remainder(shape, small):
     M, K, N, r, G, sm = shape
-    c = make_case(shape, 4)
+    c = make_case(shape, 4, small)
     try:
         R = c.residual()
         ga = c.gpu_act()
@@ -106,10 +113,11 @@ def test_rotated_quantizer_bit_exact_on_kernel_remainder(shape):
         c.close()
 
 
+@PATHS
 @pytest.mark.parametrize("shape", SHAPES, ids=IDS)
-def test_rotated_end_to_end(shape):
+def test_rotated_end_to_end(shape, small):
     M, K, N, r, G, sm = shape
-    c = make_case(shape, 6)
+    c = make_case(shape, 6, small)
     try:
         Y = c.run(fp32=True).cpu().numpy()
         ga, gw = c.gpu_act(), c.gpu_weights()
@@ -179,9 +187,10 @@ def atoms_to_rows(atoms, rows, K):
     return a[idx]
 
 
+@PATHS
 @pytest.mark.parametrize("shape", [(200, 512, 256, 16), (65, 1536, 136, 0), (130, 3072, 128, 32)],
                          ids=lambda s: "M%d_K%d_N%d_r%d" % s)
-def test_rotated_nvfp4(shape):
+def test_rotated_nvfp4(shape, small):
     M, K, N, r = shape
     Xb = wl.activations(M, K, seed=9, layer_id=K, dist="outlier")
     Wb = wl.weight(K, N, seed=9, layer_id=K)
@@ -192,6 +201,7 @@ def test_rotated_nvfp4(shape):
     layer = asp.AspLinear(to_dev_bf16(Wb), torch.from_numpy(U).cuda() if r else None, fmt=asp.QWAM_FMT_NVFP4,
                           rotate=True, s=torch.from_numpy(s).cuda())
     try:
+        asp.qwam_asp_set_small_m(layer.h, small)
         e = asp.qwam_asp_export_nvfp4(layer.h)
         gw = dict(qw=unpack_e2m1(e["qw"]), sfw=e["sfw"], sg=e["sg"], Bh=e["Bh"][:, :r].T.copy())
         ow = oracle.pack_nvfp4_f64(oracle.rotate_weights(Wb, s64), U)
