@@ -9,6 +9,12 @@ The NVFP4 variant (App. B.1's Blackwell format) has its own entry points with th
 ``_nvfp4``: E2M1 codes (one 4-bit code per uint8), E4M3 block scales (uint8 bits, one per 16
 consecutive K entries) and one float32 scale per weight tensor.
 
+Smoothing and the block Hadamard rotation in front of the layer (Sec. 2 Eq. (pair)):
+``rotate_weights`` / ``rotate_acts`` / ``fwht_cols`` form W~ = H diag(s) W and x~ = H diag(s)^-1 x
+in float64 (the block fast Walsh-Hadamard transform of ``qo_block_fwht``), the ``*_f64`` entry
+points run the pack and the activation path on those float64 values, and ``forward_rotated`` /
+``forward_rotated_nvfp4`` chain them.  The offline choice of what to protect is in ``subspace``.
+
 Every function returns semantic arrays in the paper's row-major notation:
 X [M,K] tokens, W [K,N], U [K,r] (the paper's V), codes as int8 in [-7, 7], activation scales
 float32 [M, K/G], weight scales float16 [K/G, N], branch factors float16.
