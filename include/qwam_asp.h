@@ -333,10 +333,12 @@ qwam_status qwam_asp_select_experts(const double* mass, const double* cost, int 
 /* Set the bound of every device wait of this handle's kernels, in seconds (default 2.0). */
 qwam_status qwam_asp_set_timeout(qwam_asp_handle h, double seconds);
 
-/* Activation path for few tokens.  Calls with M <= max_rows tokens (default 256) on a handle
- * without rotation and with K % 256 == 0 run the activation side on the CUDA cores, one CTA per
- * token (float32 projection and remainder, the same quantizers); larger M take the tensor-core
- * kernel.  Both meet the same parity bars; max_rows = 0 always takes the tensor-core kernel.
+/* Activation path for few tokens.  On a handle with K % 256 == 0, calls with M <= max_rows tokens
+ * (default 256), and calls of any M on an r = 0 handle without rotation, run the activation side
+ * on the CUDA cores, one CTA per token (float32 projection and remainder, the rotation of a
+ * rotated handle, the same quantizers); other calls take the tensor-core kernel (and, for a
+ * rotated handle, the rotation kernel).  Both meet the same parity bars; max_rows = 0 always
+ * takes the tensor-core kernel.
  * Errors: QWAM_ERR_INVALID_ARG (no handle, max_rows < 0). */
 qwam_status qwam_asp_set_small_m(qwam_asp_handle h, int max_rows);
 
