@@ -27,6 +27,14 @@
 // Warp roles (320 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2..9
 // epilogue: warps 2..5 and 6..9 each cover the four 32-row TMEM quadrants and take the even
 // and the odd K chunks respectively.
+//
+// Also in this file, sharing kernel (a)'s quantizers (the same rounding, bit for bit):
+//   rotquant_kernel  smoothing and block Hadamard rotation of the remainder (Sec. 2 Eq. (pair)),
+//                    then quantization, one warp per token row and Hadamard block;
+//   smallq_kernel    the whole activation path on the CUDA cores, one CTA per token row, for few
+//                    tokens and for r = 0 layers (with the rotation for rotated layers);
+//   debug kernels    the thread-per-row and warp-wide quantizers on caller-given rows (tests).
+// launch_actquant at the end of the file chooses among them.
 #include <algorithm>
 
 #include "internal.h"
