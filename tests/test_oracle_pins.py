@@ -438,3 +438,30 @@ def test_rotation_spreads_an_outlier_channel():
     assert np.abs(Xt).max() <= np.abs(Xd).sum() / math.sqrt(K) * (1 + 1e-15)
     assert np.abs(Xt).max() < 64.0 / 4
     np.testing.assert_allclose(np.linalg.norm(Xt), np.linalg.norm(Xd), rtol=1e-14)
+
+
+def _hadamard_dense_vec(d):
+    """The same block-diagonal H as _hadamard_dense, from the bit formula with numpy bit counts."""
+    b = 1
+    while d % (2 * b) == 0 and 2 * b <= 1024:
+        b *= 2
+    i = np.arange(b)
+    x = np.bitwise_and(i[:, None], i[None, :]).astype(np.uint32)
+    pc = np.zeros_like(x)
+    while x.any():
+        pc += x & 1
+        x >>= 1
+    blk = np.where(pc % 2 == 0, 1.0, -1.0) / math.sqrt(b)
+    return np.kron(np.eye(d // b), blk), b
+
+
+@pytest.mark.parametrize("K,B", [(1536, 512), (3072, 1024), (768, 256)])
+def test_rotation_blocks_of_the_bench_shapes(K, B):
+    """The block sizes of the benchmark's shapes (B = 256, 512, 1024) against the bit formula."""
+    H, b = _hadamard_dense_vec(K)
+    assert b == B
+    Xb = wl.activations(3, K, seed=K, layer_id=2, dist="outlier")
+    s = np.exp(np.random.default_rng(K).uniform(-1, 1, K))
+    X = wl.bf16_bits_to_f32(Xb).astype(np.float64)
+    Xt = oracle.rotate_acts(Xb, s)
+    np.testing.assert_allclose(Xt, (X / s[None, :]) @ H.T, rtol=0, atol=1e-12 * np.abs(Xt).max())
