@@ -11,16 +11,16 @@
  * aarch64 alike.
  *
  * What it follows (paper: "Q-WAM", arxiv 2609.33269):
- *   - Sec. 2 "Post-Training Quantization", Eq. (quant): Q_b(X) = s * round(X / s) with
+ *   - Sec. 3 "Post-Training Quantization", Eq. (quant): Q_b(X) = s * round(X / s) with
  *     s = max|X| / (2^(b-1) - 1), one scale per group of consecutive entries; b = 4 gives /7.
  *   - App. B.1 "Quantization settings and kernels": symmetric, round to nearest, one scale per
  *     group of consecutive input channels, weights offline, activations per token at run time,
  *     activation scale = group absmax / 7; weight codes stored as 4-bit values.
- *   - Sec. 3.2 "Splitting the layer", Eq. (xsplit) and Eq. (asp):
+ *   - Sec. 4.2 "Splitting the layer", Eq. (xsplit) and Eq. (asp):
  *       x = V(V^T x) + x_perp,  x_perp = (I - VV^T) x,
  *       W^T x ~= (V^T W)^T (V^T x) + Q4(W_perp)^T Q4(x_perp),  W_perp = (I - VV^T) W.
  *   - Table 3: per-group W4A4 costs 4.50 bits per weight at group 32, i.e. a 16-bit weight scale.
- *   - Sec. 2 Eq. (pair) and App. B.1: smoothing and a block Hadamard rotation in front of the
+ *   - Sec. 3 Eq. (pair) and App. B.1: smoothing and a block Hadamard rotation in front of the
  *     quantizer, x~ = H diag(s)^-1 x and W~ = H diag(s) W, H applied by the fast Walsh-Hadamard
  *     transform in blocks of B (qo_block_fwht); the layer then runs on x~ and W~ (the *_f64 entry
  *     points take float64 inputs).
@@ -382,8 +382,13 @@ int qo_nearest_code(double x, double s) { return nearest_code(x, s); }
  *   N2  E4M3 (OCP FP8, "FN"): sign | 4-bit exponent (bias 7) | 3-bit mantissa; no infinities;
  *       largest finite 448; subnormals m * 2^-9.  Rounding is to nearest, ties to even, and
  *       saturates at 448.
- *   N3  activations, per token and block b of 16 consecutive K entries of x_perp (float32):
- *       s = RN_e4m3(RN_f32(amax_b / 6)),  code = RN_e2m1(RN_f32(x / s)),  s == 0 -> codes 0.
+ *   N3  activations, per token and block b of 16 consecutive K entries of x_perp:
+ *       s = RN_e4m3(RN_f32(amax_b / 6)),  code = RN_e2m1(x / s) of the exact quotient,
+ *       s == 0 -> codes 0.  The remainder x_perp stays in float64 (Eq. (xsplit) in exact
+ *       arithmetic, as for the INT4 activations); amax_b / 6 is rounded to float64 and then
+ *       to float32.  For a float32 x, RN_e2m1(RN_f32(x / s)) = RN_e2m1(x / s): a float32 step
+ *       next to a midpoint product moves x / s by more than half a float32 unit of it, so the
+ *       float32 quotient lands on an E2M1 midpoint only when x / s is that midpoint.
  *   N4  weights: s_g = RN_f32(amax(W_perp) / (6 * 448)); per output channel n and block b,
  *       s_b = RN_e4m3(amax_b / (6 s_g)) and code = RN_e2m1(w / (s_b s_g)), both from the
  *       float64 quotient (whose one rounding cannot change a 4-bit or 2-bit result:
@@ -435,6 +440,29 @@ static uint8_t e4m3_bits_rn(double x) {
   int code = ((E + 7) << 3) | ((int)q - 8);
   if (code > 0x7e) code = 0x7e;                    /* 464 .. 480 round to 448 by saturation */
   return sign | (uint8_t)code;
+}
+
+/* RN_e2m1(x / s) of the exact quotient (s > 0), readings N1 and N3: |x| is compared with the
+ * midpoints 0.25, 0.75, ..., 5 of the magnitude grid times s (products of at most 3 and 4
+ * significant bits, exact in float64); on a midpoint the code with the even mantissa bit wins,
+ * and beyond 5 s the code saturates at 6. */
+static int e2m1_code_ratio(double x, double s) {
+  static const double mid[7] = {0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0};
+  const double a = fabs(x);
+  int c = 7;
+  for (int i = 0; i < 7; ++i) {
+    const double ms = mid[i] * s;
+    if (a < ms) {
+      c = i;
+      break;
+    }
+    if (a == ms) {
+      c = (i & 1) ? i + 1 : i; /* codes i and i + 1 differ in the mantissa bit: keep the even */
+      break;
+    }
+  }
+  if (c == 0) return 0; /* +0 for any sign */
+  return (x < 0.0) ? (c | 8) : c;
 }
 
 /* value -> E2M1 code, nearest, ties to even mantissa, saturating at 6 (reading N1).
@@ -531,27 +559,21 @@ int qo_pack_nvfp4_f64(const double* W, const float* U, int K, int N, int r, uint
   return pack_nvfp4_core(W, U, K, N, r, qw, sfw, sg_out, Bh);
 }
 
-/* Reading N3 on one float32 remainder row segment of 16 entries. */
-static void quantize_block_nvfp4(const float* x, uint8_t* q, uint8_t* sf) {
-  float amax = 0.0f;
+/* Reading N3 on one remainder row segment of 16 entries. */
+static void quantize_block_nvfp4(const double* x, uint8_t* q, uint8_t* sf) {
+  double amax = 0.0;
   for (int k = 0; k < QO_FP4_BLOCK; ++k)
-    if (fabsf(x[k]) > amax) amax = fabsf(x[k]);
-  const float t = (float)((double)amax / 6.0); /* RN_f32(amax / 6): innocuous double rounding */
+    if (fabs(x[k]) > amax) amax = fabs(x[k]);
+  /* RN_f32(amax / 6): for a float32 amax the double rounding through float64 is innocuous */
+  const float t = (float)(amax / 6.0);
   const uint8_t sb = e4m3_bits_rn((double)t);
   *sf = sb;
   const double s = e4m3_value(sb);
-  for (int k = 0; k < QO_FP4_BLOCK; ++k) {
-    if (s > 0.0) {
-      const float u = (float)((double)x[k] / s); /* RN_f32(x / s) */
-      q[k] = (uint8_t)e2m1_code_rn((double)u);
-    } else {
-      q[k] = 0;
-    }
-  }
+  for (int k = 0; k < QO_FP4_BLOCK; ++k) q[k] = (uint8_t)((s > 0.0) ? e2m1_code_ratio(x[k], s) : 0);
 }
 
-/* Run-time activation path of the NVFP4 variant: Eq. (xsplit) as in qo_quantize_act, with the
- * remainder rounded to float32 (the precision in which the GPU forms it), then reading N3.
+/* Run-time activation path of the NVFP4 variant: Eq. (xsplit) as in qo_quantize_act (the
+ * remainder in float64), then reading N3.
  * Outputs: qx [M,K] E2M1 codes, sfx [M,K/16] E4M3 bits, ph [M,r] float16 bits. */
 static int quantize_act_nvfp4_core(const uint16_t* X_bf16, const double* X_f64, const float* U, int M, int K, int r,
                                    uint8_t* qx, uint8_t* sfx, uint16_t* ph) {
@@ -561,7 +583,7 @@ static int quantize_act_nvfp4_core(const uint16_t* X_bf16, const double* X_f64, 
 #pragma omp parallel reduction(min : status)
   {
     double* x = (double*)malloc((size_t)K * sizeof(double));
-    float* xf = (float*)malloc((size_t)K * sizeof(float));
+    double* xp = (double*)malloc((size_t)K * sizeof(double));
     double* p = (double*)malloc((size_t)(r > 0 ? r : 1) * sizeof(double));
 #pragma omp for schedule(static)
     for (int m = 0; m < M; ++m) {
@@ -574,17 +596,17 @@ static int quantize_act_nvfp4_core(const uint16_t* X_bf16, const double* X_f64, 
       for (int k = 0; k < K; ++k) {
         double acc = 0.0;
         for (int j = 0; j < r; ++j) acc += p[j] * (double)U[(size_t)k * r + j];
-        xf[k] = (float)(x[k] - acc);
+        xp[k] = x[k] - acc;
       }
       for (int j = 0; j < r; ++j) {
         ph[(size_t)m * r + j] = f16_bits_rn(p[j]);
         if ((ph[(size_t)m * r + j] & 0x7c00) == 0x7c00) status = QO_ERANGE;
       }
       for (int b = 0; b < nb; ++b)
-        quantize_block_nvfp4(xf + b * QO_FP4_BLOCK, qx + (size_t)m * K + b * QO_FP4_BLOCK, sfx + (size_t)m * nb + b);
+        quantize_block_nvfp4(xp + b * QO_FP4_BLOCK, qx + (size_t)m * K + b * QO_FP4_BLOCK, sfx + (size_t)m * nb + b);
     }
     free(x);
-    free(xf);
+    free(xp);
     free(p);
   }
   return status;
@@ -608,9 +630,11 @@ int qo_quantize_residual_nvfp4_f32(const float* R, int M, int K, uint8_t* qx, ui
   const int nb = K / QO_FP4_BLOCK;
 #pragma omp parallel for schedule(static)
   for (int m = 0; m < M; ++m)
-    for (int b = 0; b < nb; ++b)
-      quantize_block_nvfp4(R + (size_t)m * K + b * QO_FP4_BLOCK, qx + (size_t)m * K + b * QO_FP4_BLOCK,
-                           sfx + (size_t)m * nb + b);
+    for (int b = 0; b < nb; ++b) {
+      double x[QO_FP4_BLOCK]; /* float32 values, widened exactly */
+      for (int k = 0; k < QO_FP4_BLOCK; ++k) x[k] = (double)R[(size_t)m * K + b * QO_FP4_BLOCK + k];
+      quantize_block_nvfp4(x, qx + (size_t)m * K + b * QO_FP4_BLOCK, sfx + (size_t)m * nb + b);
+    }
   return QO_OK;
 }
 

@@ -6,6 +6,7 @@ dequantized operands, and the special cases r = 0 and r = K of Eq. (asp)."""
 from __future__ import annotations
 
 import math
+from fractions import Fraction
 
 import numpy as np
 import pytest
@@ -150,6 +151,79 @@ def test_weight_pack_r0_brute_force():
                 code, _ = nearest_even(u, E2M1_POS) if abs(u) < 6 else (7, 6.0)
                 want = 0 if code == 0 else (code | 8 if u < 0 else code)
                 assert out["qw"][n, 16 * b + k] == want
+
+
+def nearest_even_exact(x: float, s: float, table):
+    """Brute force on the exact quotient x / s (rational arithmetic): the entry of `table`
+    nearest to |x| / s, ties to the even code."""
+    u = abs(Fraction(x)) / Fraction(s)
+    return min(table, key=lambda cv: (abs(u - Fraction(cv[1])), cv[0] & 1))
+
+
+@pytest.mark.parametrize("r", [1, 5])
+def test_activation_path_brute_force_on_the_pinned_remainder(r):
+    """0 < r < K: the NVFP4 activation path follows reading N3 on the remainder of Eq. (xsplit),
+    recomputed here by brute force from the INT4 oracle's float64 remainder (which the exact
+    rational test of the INT4 layer pins).  Scales: RN_e4m3 of RN_f32(amax / 6); codes: nearest
+    E2M1 value to the exact quotient, ties to even, saturating at 6."""
+    M, K = 6, 128
+    X = wl.activations(M, K, seed=81, layer_id=r, dist="outlier", n_outlier=3)
+    U = wl.basis(K, r, seed=81, layer_id=r)
+    Xp = oracle.quantize_act(X, U, 64, want_float64=True)["Xperp"]
+    out = oracle.quantize_act_nvfp4(X, U)
+    for m in range(M):
+        for b in range(K // 16):
+            blk = Xp[m, 16 * b:16 * b + 16]
+            t = float(np.float32(np.abs(blk).max() / 6.0))
+            s_bits = nearest_even(t, E4M3_POS)[0] if t < 448 else 0x7e
+            assert out["sfx"][m, b] == s_bits, (m, b)
+            s = e4m3_from_fields(s_bits)
+            for k in range(16):
+                x = float(blk[k])
+                code = 0 if s == 0 else (7 if abs(Fraction(x)) / Fraction(s) >= 6 else
+                                         nearest_even_exact(x, s, E2M1_POS)[0])
+                want = 0 if code == 0 else (code | 8 if x < 0 else code)
+                assert out["qx"][m, 16 * b + k] == want, (m, b, k)
+
+
+@pytest.mark.parametrize("r", [1, 5])
+def test_weight_pack_brute_force_on_the_pinned_deflated_weight(r):
+    """0 < r < K: every code and scale of the NVFP4 pack follows reading N4 on W_perp, recomputed by
+    brute force from the INT4 oracle's float64 W_perp (pinned by the exact rational test)."""
+    K, N = 128, 6
+    W = wl.weight(K, N, seed=82, layer_id=r)
+    U = wl.basis(K, r, seed=82, layer_id=r)
+    Wp = oracle.pack(W, U, 64, want_float64=True)["Wperp"]
+    out = oracle.pack_nvfp4(W, U)
+    sg = np.float32(np.abs(Wp).max() / (6.0 * 448.0))
+    assert out["sg"] == sg
+    for n in range(N):
+        for b in range(K // 16):
+            blk = Wp[16 * b:16 * b + 16, n]
+            s_bits = nearest_even(np.abs(blk).max() / (6.0 * float(sg)), E4M3_POS)[0]
+            assert out["sfw"][n, b] == s_bits, (n, b)
+            scale = e4m3_from_fields(s_bits) * float(sg)
+            for k in range(16):
+                u = blk[k] / scale
+                code, _ = nearest_even(u, E2M1_POS) if abs(u) < 6 else (7, 6.0)
+                want = 0 if code == 0 else (code | 8 if u < 0 else code)
+                assert out["qw"][n, 16 * b + k] == want, (n, b, k)
+
+
+def test_activation_quantizer_rounds_the_exact_quotient():
+    """A float64 remainder just above or below an E2M1 midpoint product m * s rounds by its exact
+    quotient (a float32 rounding of x / s would land on the midpoint and go to the even code)."""
+    s_bits = 0x38  # s = 1
+    for mid, lo_code, hi_code in ((0.25, 0, 1), (0.75, 1, 2), (1.25, 2, 3), (2.5, 4, 5), (5.0, 6, 7)):
+        R = np.zeros((1, 16), np.float64)
+        R[0, 0] = 6.0  # amax 6 -> s = 1 exactly
+        R[0, 1] = mid * (1 + 2.0 ** -40)
+        R[0, 2] = mid * (1 - 2.0 ** -40)
+        R[0, 3] = mid
+        q = oracle.quantize_act_nvfp4_f64(R, np.zeros((16, 0), np.float32))
+        assert q["sfx"][0, 0] == s_bits
+        tie = lo_code if lo_code % 2 == 0 else hi_code
+        assert list(q["qx"][0, 1:4]) == [hi_code, lo_code, tie], mid
 
 
 # ---- the layer (reading N5) -----------------------------------------------------------------
