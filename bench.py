@@ -16,7 +16,7 @@ the layer shards by rows with no collective); weak scaling.
 
 The NVFP4 variant (App. B.1: E2M1 with an E4M3 scale per 16 K, block scales applied by the
 tensor cores) is timed on the same workload and reported under `variants`; `--format nvfp4` makes
-it the headline.  So is the layer with smoothing and the block Hadamard rotation in front (Sec. 2
+it the headline.  So is the layer with smoothing and the block Hadamard rotation in front (Sec. 3
 Eq. (pair)); `--rotate` makes that the headline (three launches per step with r > 0).  The
 denoising-step layer sweep (30 DiT blocks, ASP on a third of them) is reported per format under
 `variants.sweep_int4` / `variants.sweep_nvfp4`.

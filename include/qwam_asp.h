@@ -2,20 +2,20 @@
  * qwam_asp.h -- C ABI of the GB300 (sm_103a) implementation of the Action-Subspace Protection
  * (ASP) linear layer of Q-WAM (arxiv 2609.33269).
  *
- * The layer (Sec. 3.2, Eq. (xsplit) and Eq. (asp)), in the row-major notation used here
+ * The layer (Sec. 4.2, Eq. (xsplit) and Eq. (asp)), in the row-major notation used here
  * (X [M,K] = one token per row, W [K,N], U [K,r] = the paper's V with orthonormal columns):
  *
  *     p      = X U                       (protected coordinates, kept in 16 bits)
  *     X_perp = X - p U^T                 (remainder, orthogonal to span(U))
- *     W_perp = W - U (U^T W)             (deflated weight, Sec. 3.2 "Splitting the layer")
+ *     W_perp = W - U (U^T W)             (deflated weight, Sec. 4.2 "Splitting the layer")
  *     Y      = p_hat B_hat  +  Q4(X_perp) Q4(W_perp)
  *
  * with B_hat = RN_f16(U^T W), p_hat = RN_f16(p), and Q4 the symmetric group quantizer of
- * Eq. (quant) (Sec. 2) with b = 4: scale s = absmax / 7 per group of `group` consecutive input
+ * Eq. (quant) (Sec. 3) with b = 4: scale s = absmax / 7 per group of `group` consecutive input
  * channels (App. B.1), codes = nearest integer to x / s (exact quotient, ties to even), so codes
  * lie in [-7, 7].  Activation scales are float32, weight scales float16 (Table 3: 4.50 bits per
  * weight at group 32 implies a 16-bit weight scale).  r = 0 gives plain per-group W4A4 (experts
- * that ASP does not select, Sec. 3.3).
+ * that ASP does not select, Sec. 4.3).
  *
  * Conventions for every entry point:
  *   - Pointers marked "device" are CUDA device pointers on the current device; "host" pointers
@@ -57,7 +57,7 @@ typedef enum {
 
 enum { QWAM_Y_BF16 = 0, QWAM_Y_FP32 = 1 };
 
-/* Offline packing (Sec. 3.2 Eq. (asp); the W_perp derivation; Eq. (quant) on the weight).
+/* Offline packing (Sec. 4.2 Eq. (asp); the W_perp derivation; Eq. (quant) on the weight).
  *   W_bf16 : device, bf16 [K, N] row-major (the paper's W~ in its transformed coordinates)
  *   U      : device, float32 [K, r] row-major, orthonormal columns; may be NULL iff r == 0
  *   K      : input dimension, K % 64 == 0;   N : output dimension, N % 8 == 0
@@ -75,15 +75,16 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
 qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes);
 
 /* Layout of the activation workspace for M tokens (byte offsets from its start):
- *   codes  : uint8 [M, K], one byte per activation code c in [-7, 7]: the E4M3 bit pattern of
- *            c * 2^-9, i.e. (c < 0 ? 0x80 : 0) | |c| (an E4M3 subnormal; the GEMM's tensor cores
- *            read these bytes as they are)
+ *   codes  : uint8 [M, K/2], the activation codes c in [-7, 7] packed at four bits as SM4 words:
+ *            the little-endian 32-bit word j of a row holds k = 8j .. 8j+7.  Byte i of the word
+ *            carries code 8j+i in its sign bit 7 and magnitude bits 0-2, the magnitude of code
+ *            8j+4+i in bits 4-6, and in bit 3 the sign of code 8j+4+((i+3) mod 4).  With lo and
+ *            hi the words of E4M3 bytes (c < 0 ? 0x80 : 0) | |c| of k = 8j..8j+3 and 8j+4..8j+7,
+ *            word = lo | rotl(hi, 4), and back lo = word & 0x87878787, hi = rotr(word, 4) &
+ *            0x87878787 (the GEMM expands the words this way, with one funnel shift and two masks)
  *   scales : float32 [K/group, M_pad] (M_pad = M rounded up to 128), s_x of token m, group g
  *            at [g * M_pad + m]
- *   ab     : float32 [K/group, M_pad, 2], for token m and group g at [(g * M_pad + m) * 2]:
- *            (alpha, beta) with alpha = 2^18 s_x and beta = -8 s_x S_a, S_a the sum of the
- *            group's codes.  These are the GEMM epilogue's per-row constants (see
- *            qwam_asp_gemm), formed here once per token and group, each with one rounding.
+ *   ab     : no region (ab_off == phat_off); kept in the call for the layout's stability
  *   p_hat  : float16 [M, r_pad] (r_pad = r rounded up to 16; columns >= r are zero)
  * The workspace is transient (written by qwam_asp_quantize_act, read by qwam_asp_gemm); the
  * weights are the part of the layer that stays packed at 4 bits. */
@@ -93,20 +94,20 @@ qwam_status qwam_asp_act_layout(qwam_asp_handle h, int M, size_t* codes_off, siz
 /* Kernel (a): Eq. (xsplit) and the run-time half of Eq. (quant), one launch, asynchronous.
  *   X_bf16 : device, bf16 [M, K] row-major;  act_ws : device workspace (see above), written
  * Reads X once from HBM, forms p = X U on tensor cores (bf16 hi/lo split of U, float32
- * accumulation), X_perp = X - p U^T in float32, and writes codes, float32 scales, the epilogue
- * constants and p_hat. */
+ * accumulation), X_perp = X - p U^T in float32, and writes the packed codes, float32 scales and
+ * p_hat. */
 qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws,
                                   struct CUstream_st* stream);
 
 /* Kernel (b): the 4-bit GEMM with the low-rank branch in its epilogue, asynchronous.
  *   act_ws : device workspace filled by qwam_asp_quantize_act for the same M
  *   Y      : device [M, N] row-major, bf16 (y_dtype QWAM_Y_BF16) or float32 (QWAM_Y_FP32)
- * Per group g the tensor cores form the exact integer partial sums P_g = sum_k qx qw (codes fed
- * as E4M3 multiples of 2^-9, which E4M3 holds exactly; float32 accumulation of these integer
- * multiples of 2^-18 below 2^-5 is exact); the weight bytes carry an offset of 8, so the
- * accumulator is D = 2^-18 (P_g + 8 S_a), and the epilogue adds s_w[g,n] (alpha D + beta) =
- * s_w[g,n] s_x[m,g] P_g in float32 and, last, the branch p_hat B_hat (float16 operands,
- * float32 accumulation). */
+ * Both operands stay packed at four bits in HBM and are expanded to E4M3 bytes of c * 2^-9 in
+ * shared memory.  Per group g the tensor cores form the exact integer partial sums
+ * D = 2^-18 P_g, P_g = sum_k qx qw (E4M3 holds the codes exactly; float32 accumulation of these
+ * integer multiples of 2^-18 below 2^-5 is exact), and the epilogue adds (D s_x[m,g]) sigma[g,n]
+ * in float32, sigma = 2^18 s_w (= s_w[g,n] s_x[m,g] P_g with two roundings), and, last, the
+ * branch p_hat B_hat (float16 operands, float32 accumulation; any r_pad). */
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle h, void* Y, int y_dtype,
                           struct CUstream_st* stream);
 
@@ -178,7 +179,7 @@ enum { QWAM_FMT_INT4 = 0, QWAM_FMT_NVFP4 = 1 };
 qwam_status qwam_asp_pack_weights_nvfp4(const void* W_bf16, const float* U, int K, int N, int r,
                                         struct CUstream_st* stream, qwam_asp_handle* out);
 
-/* ---- Smoothing and block Hadamard rotation in front of the layer (Sec. 2 Eq. (pair); App. B.1)
+/* ---- Smoothing and block Hadamard rotation in front of the layer (Sec. 3 Eq. (pair); App. B.1)
  * The paper quantizes in rotated coordinates: with per-channel smoothing factors s (App. B.1:
  * s_j = max|X_j|^alpha / max|W_j,:|^(1-alpha), see qwam_asp_smoothing_factors) and the block
  * Hadamard matrix H (block-diagonal, each block the Sylvester Hadamard matrix of size B divided by
@@ -263,9 +264,8 @@ qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h
  *   R      : device float32 [M, K], row-major, 16-byte aligned; K % 64 == 0
  *   fmt    : QWAM_FMT_INT4 or QWAM_FMT_NVFP4
  *   group  : 32 or 64 for INT4 (ignored for NVFP4, whose block is 16)
- *   codes  : device, 16-byte aligned.  INT4: uint8 [M, K], each the E4M3 bit pattern of c * 2^-9
- *            (sign bit | magnitude), as in the activation workspace.  NVFP4: uint8 [M, K/2], two
- *            E2M1 codes per byte, low nibble = even k.
+ *   codes  : device, 16-byte aligned.  INT4: uint8 [M, K/2], SM4 words as in the activation
+ *            workspace.  NVFP4: uint8 [M, K/2], two E2M1 codes per byte, low nibble = even k.
  *   scales : device.  INT4: float32 [M, K/group] row-major (4-byte aligned).  NVFP4: uint8 E4M3
  *            bit patterns [M, K/16] row-major.
  * Asynchronous on `stream`; QWAM_ERR_INVALID_ARG for bad sizes, formats or alignment. */
@@ -276,17 +276,17 @@ qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, 
  * per lane, a group over neighbouring lanes) on caller-given float32 rows, with the same rounding
  * rules as qwam_asp_debug_quantize_rows; K % 256 == 0.  Outputs are written in the activation
  * workspace's layouts with M_pad = ceil(M / 128) * 128 rows:
- *   INT4:  codes uint8 [M, K] (E4M3 bytes of c * 2^-9), scales float32 [K/group, M_pad],
- *          ab float32 [K/group, M_pad, 2] (the GEMM epilogue constants);
+ *   INT4:  codes uint8 [M, K/2] (SM4 words, described at qwam_asp_act_layout), scales float32
+ *          [K/group, M_pad];
  *   NVFP4: codes uint8 [M, K/2] (two per byte, low nibble = even k), scales uint8 E4M3 in the
- *          512-byte atoms described above (M_pad * K/16 bytes); ab unused (may be NULL).
+ *          512-byte atoms described above (M_pad * K/16 bytes).
  * Device pointers; codes 16-byte aligned.  Errors: QWAM_ERR_INVALID_ARG, QWAM_ERR_CUDA. */
 qwam_status qwam_asp_debug_quantize_lanes(const float* R, int M, int K, int fmt, int group, void* codes,
-                                          void* scales, void* ab, struct CUstream_st* stream);
+                                          void* scales, struct CUstream_st* stream);
 
-/* ---- The offline choice of what to protect (Sec. 3.2-3.3; App. A; App. B.1) -----------------
+/* ---- The offline choice of what to protect (Sec. 4.2-4.3; App. A; App. B.1) -----------------
  * Calibration-time steps that pick U (the paper's V) and which experts carry a branch, from a given
- * Action Observability Gramian G (the AOG of Sec. 3.1, estimated elsewhere).  None of them needs a
+ * Action Observability Gramian G (the AOG of Sec. 4.1, estimated elsewhere).  None of them needs a
  * handle.  All matrices are float32, row-major, on the device unless stated otherwise.        */
 
 /* Smoothing factors of App. B.1: s_j = xmax_j^alpha / max_n |W[j, n]|^(1 - alpha) for every input
@@ -297,7 +297,7 @@ qwam_status qwam_asp_debug_quantize_lanes(const float* R, int M, int K, int fmt,
 qwam_status qwam_asp_smoothing_factors(const float* xmax, const void* W_bf16, int K, int N, double alpha, float* s,
                                        struct CUstream_st* stream);
 
-/* The AOG in the rotated coordinates (Sec. 3.2): Gt = H diag(gamma) G diag(gamma) H, with H the block
+/* The AOG in the rotated coordinates (Sec. 4.2): Gt = H diag(gamma) G diag(gamma) H, with H the block
  * Hadamard rotation of Eq. (pair) (normalised Sylvester blocks of size B, the largest power of two
  * dividing d, at most 1024).  G, Gt, work: [d, d] (work is scratch); gamma [d] or NULL for no
  * smoothing.  G, Gt and work must be distinct.  d <= 32768.  Asynchronous on `stream`. */
@@ -305,14 +305,14 @@ qwam_status qwam_asp_rotated_gramian(const float* G, const float* gamma, int d, 
                                      struct CUstream_st* stream);
 
 /* tr(A) of a [d, d] device matrix, accumulated in float64 and returned in *trace (host): the
- * per-layer term of an expert's action mass mu_E = sum of tr Gt (Sec. 3.3, Eq. (mass)).
+ * per-layer term of an expert's action mass mu_E = sum of tr Gt (Sec. 4.3, Eq. (mass)).
  * Synchronizes `stream`. */
 qwam_status qwam_asp_gramian_trace(const float* A, int d, double* trace, struct CUstream_st* stream);
 
 /* Scratch bytes of qwam_asp_action_subspace for a [d, d] matrix and rank r (1 <= r <= min(d, 96)). */
 qwam_status qwam_asp_subspace_workspace_bytes(int d, int r, size_t* bytes);
 
-/* The action subspace (Sec. 3.2, Eq. (gtilde); App. A): the eigenvectors of the r largest
+/* The action subspace (Sec. 4.2, Eq. (gtilde); App. A): the eigenvectors of the r largest
  * eigenvalues of the symmetric positive semidefinite Gt [d, d].  V [d, r] receives them as columns
  * (decreasing eigenvalue, orthonormal; each column's sign is arbitrary) and lambda [r] (device)
  * the eigenvalues.  Subspace iteration with r + max(8, r/2) vectors (at most 96) for `iters`
@@ -322,7 +322,7 @@ qwam_status qwam_asp_subspace_workspace_bytes(int d, int r, size_t* bytes);
 qwam_status qwam_asp_action_subspace(const float* Gt, int d, int r, int iters, float* V, float* lambda, void* work,
                                      struct CUstream_st* stream);
 
-/* Which experts to protect (Sec. 3.3): in decreasing order of action mass per added 16-bit value,
+/* Which experts to protect (Sec. 4.3): in decreasing order of action mass per added 16-bit value,
  * mass[i] / cost[i] (equal ratios: lower index first), each expert whose added values still fit the
  * budget.  mass[n] >= 0, cost[n] > 0 (the 16-bit values its branches add, r (d + d') per layer),
  * host arrays; chosen[n] (host) receives the chosen indices in that order and *n_chosen their count.

@@ -1,4 +1,4 @@
-"""CPU oracle for the ASP linear layer (Q-WAM, Sec. 3.2 Eq. (asp); Sec. 2 Eq. (quant); App. B.1).
+"""CPU oracle for the ASP linear layer (Q-WAM, Sec. 4.2 Eq. (asp); Sec. 3 Eq. (quant); App. B.1).
 
 TEST INFRASTRUCTURE ONLY.  The tests, the smoke check and the CPU-baseline leg of the benchmark
 load this module; the library under ``paper_2609_33269_gb300`` never imports it and shares no
@@ -9,7 +9,7 @@ The NVFP4 variant (App. B.1's Blackwell format) has its own entry points with th
 ``_nvfp4``: E2M1 codes (one 4-bit code per uint8), E4M3 block scales (uint8 bits, one per 16
 consecutive K entries) and one float32 scale per weight tensor.
 
-Smoothing and the block Hadamard rotation in front of the layer (Sec. 2 Eq. (pair)):
+Smoothing and the block Hadamard rotation in front of the layer (Sec. 3 Eq. (pair)):
 ``rotate_weights`` / ``rotate_acts`` / ``fwht_cols`` form W~ = H diag(s) W and x~ = H diag(s)^-1 x
 in float64 (the block fast Walsh-Hadamard transform of ``qo_block_fwht``), the ``*_f64`` entry
 points run the pack and the activation path on those float64 values, and ``forward_rotated`` /
@@ -107,7 +107,7 @@ def _check(rc, what):
 
 
 def pack(W_bf16_bits, U, G, want_float64=False):
-    """Offline packing (Sec. 3.2 Eq. (asp) and the W_perp derivation; Eq. (quant) on weights).
+    """Offline packing (Sec. 4.2 Eq. (asp) and the W_perp derivation; Eq. (quant) on weights).
 
     W_bf16_bits: uint16 [K,N]; U: float32 [K,r] (r may be 0).
     Returns dict(qw int8 [N,K], sw uint16 fp16-bits [K/G,N], Bh uint16 fp16-bits [r,N],
@@ -152,7 +152,7 @@ def quantize_act(X_bf16_bits, U, G, want_float64=False):
 
 
 def pack_f64(W, U, G, want_float64=False):
-    """pack() of a float64 weight W [K,N] (the smoothed and rotated W~ of Sec. 2 Eq. (pair))."""
+    """pack() of a float64 weight W [K,N] (the smoothed and rotated W~ of Sec. 3 Eq. (pair))."""
     W = _c(W, np.float64)
     K, N = W.shape
     U = _c(U, np.float32).reshape(K, -1)
@@ -199,7 +199,7 @@ def fwht_cols(A, s=None):
 
 
 def rotate_weights(W_bf16_bits, s=None):
-    """Sec. 2 Eq. (pair), weight side: W~ = H diag(s) W in float64 ([K,N]; H along K by the block
+    """Sec. 3 Eq. (pair), weight side: W~ = H diag(s) W in float64 ([K,N]; H along K by the block
     fast Walsh-Hadamard transform of App. B.1, in a fixed butterfly order)."""
     W = bf16_bits_to_f64(W_bf16_bits)
     K, N = W.shape
@@ -209,7 +209,7 @@ def rotate_weights(W_bf16_bits, s=None):
 
 
 def rotate_acts(X_bf16_bits, s=None):
-    """Sec. 2 Eq. (pair), activation side: x~ = H diag(s)^-1 x for every token row, float64 [M,K]."""
+    """Sec. 3 Eq. (pair), activation side: x~ = H diag(s)^-1 x for every token row, float64 [M,K]."""
     X = bf16_bits_to_f64(X_bf16_bits)
     M, K = X.shape
     sc = None if s is None else _c(s, np.float64)

@@ -1,4 +1,4 @@
-"""CPU oracle for the offline choice of what ASP protects (Q-WAM Sec. 3.2 and 3.3; App. B.1).
+"""CPU oracle for the offline choice of what ASP protects (Q-WAM Sec. 4.2 and 3.3; App. B.1).
 
 TEST INFRASTRUCTURE ONLY, like the rest of ``oracle``: the tests and the smoke check load it; the
 library never imports it.  Everything is float64 numpy; the one library routine used as a step is
@@ -9,14 +9,14 @@ The steps, in the paper's order and notation (d = the layer's input width, row-m
 * smoothing factor per input channel j (App. B.1): s_j = max|X_j|^alpha / max|W_j,:|^(1 - alpha),
   with max|X_j| the channel's calibration maximum and max|W_j,:| the largest weight of that input
   channel (the row of W that multiplies x_j here, the paper's "matching weight column");
-* block Hadamard rotation H (Sec. 2 Eq. (pair); App. B.1): block-diagonal, each block the
+* block Hadamard rotation H (Sec. 3 Eq. (pair); App. B.1): block-diagonal, each block the
   Sylvester Hadamard matrix of size B divided by sqrt(B), B the largest power of two that divides
   d, at most 1024.  H is symmetric and orthogonal;
-* the AOG in the rotated coordinates (Sec. 3.2): G~ = H diag(gamma) G diag(gamma) H;
-* the action subspace (Sec. 3.2, Eq. (gtilde)): the eigenvectors of the r largest eigenvalues of
+* the AOG in the rotated coordinates (Sec. 4.2): G~ = H diag(gamma) G diag(gamma) H;
+* the action subspace (Sec. 4.2, Eq. (gtilde)): the eigenvectors of the r largest eigenvalues of
   G~, which the Ky Fan maximum principle (App. A) makes the best rank-r protection;
-* the action mass of an expert E (Sec. 3.3, Eq. (mass)): mu_E = sum over its layers of tr G~;
-* which experts to protect (Sec. 3.3): those with the largest action mass per added 16-bit value,
+* the action mass of an expert E (Sec. 4.3, Eq. (mass)): mu_E = sum over its layers of tr G~;
+* which experts to protect (Sec. 4.3): those with the largest action mass per added 16-bit value,
   read here as a greedy choice in decreasing mu_E / c_E while the added values fit a budget
   (c_E = the 16-bit values the branches of E add, r (d + d') per layer).
 """
@@ -60,7 +60,7 @@ def smoothing_factors(xmax: np.ndarray, W: np.ndarray, alpha: float = 0.5) -> np
 
 
 def rotated_gramian(G: np.ndarray, gamma: np.ndarray | None = None) -> np.ndarray:
-    """Sec. 3.2: G~ = H diag(gamma) G diag(gamma) H (gamma = 1 when None)."""
+    """Sec. 4.2: G~ = H diag(gamma) G diag(gamma) H (gamma = 1 when None)."""
     G = np.asarray(G, np.float64)
     d = G.shape[0]
     g = np.ones(d) if gamma is None else np.asarray(gamma, np.float64)
@@ -69,7 +69,7 @@ def rotated_gramian(G: np.ndarray, gamma: np.ndarray | None = None) -> np.ndarra
 
 
 def action_subspace(Gt: np.ndarray, r: int):
-    """Sec. 3.2: the top-r eigenvectors V [d, r] (columns in decreasing eigenvalue order) and the
+    """Sec. 4.2: the top-r eigenvectors V [d, r] (columns in decreasing eigenvalue order) and the
     eigenvalues lambda_1 >= ... >= lambda_r of the symmetric matrix G~."""
     w, Q = np.linalg.eigh(np.asarray(Gt, np.float64))
     order = np.argsort(w)[::-1][:r]
@@ -77,7 +77,7 @@ def action_subspace(Gt: np.ndarray, r: int):
 
 
 def action_mass(gramians) -> float:
-    """Sec. 3.3 Eq. (mass): mu_E = sum of tr G~ over the layers of the expert."""
+    """Sec. 4.3 Eq. (mass): mu_E = sum of tr G~ over the layers of the expert."""
     return float(sum(np.trace(np.asarray(g, np.float64)) for g in gramians))
 
 
@@ -87,7 +87,7 @@ def branch_cost(shapes, r: int) -> int:
 
 
 def select_experts(masses, costs, budget: float):
-    """Sec. 3.3: protect in decreasing order of action mass per added 16-bit value, while the added
+    """Sec. 4.3: protect in decreasing order of action mass per added 16-bit value, while the added
     values fit the budget; an expert that does not fit is skipped and the next one is tried.
     Returns the indices chosen, in the order chosen."""
     order = sorted(range(len(masses)), key=lambda i: (-masses[i] / costs[i], i))

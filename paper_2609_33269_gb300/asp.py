@@ -96,7 +96,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.qwam_asp_rotation.argtypes = [H, ctypes.POINTER(I)]
         lib.qwam_asp_set_bias.argtypes = [H, V, V]
         lib.qwam_asp_set_small_m.argtypes = [H, I]
-        lib.qwam_asp_debug_quantize_lanes.argtypes = [V, I, I, I, I, V, V, V, V]
+        lib.qwam_asp_debug_quantize_lanes.argtypes = [V, I, I, I, I, V, V, V]
         lib.qwam_asp_export_nvfp4.argtypes = [H, V, V, ctypes.POINTER(ctypes.c_float), V]
         for name in EXPORTED:
             if name != "qwam_status_string":
@@ -267,8 +267,8 @@ def qwam_asp_debug_quantize_rows(R, M: int, K: int, fmt: int, group: int, codes,
                                                _stream(stream)), "qwam_asp_debug_quantize_rows")
 
 
-def qwam_asp_debug_quantize_lanes(R, M: int, K: int, fmt: int, group: int, codes, scales, ab=None, stream=None):
-    _check(load().qwam_asp_debug_quantize_lanes(_ptr(R), M, K, fmt, group, _ptr(codes), _ptr(scales), _ptr(ab),
+def qwam_asp_debug_quantize_lanes(R, M: int, K: int, fmt: int, group: int, codes, scales, stream=None):
+    _check(load().qwam_asp_debug_quantize_lanes(_ptr(R), M, K, fmt, group, _ptr(codes), _ptr(scales),
                                                 _stream(stream)), "qwam_asp_debug_quantize_lanes")
 
 
@@ -300,7 +300,7 @@ def qwam_asp_action_subspace(Gt, d: int, r: int, iters: int, V, lam, work, strea
 
 
 def qwam_asp_select_experts(mass, cost, budget: float):
-    """Host-only: the chosen expert indices, in the order chosen (Sec. 3.3)."""
+    """Host-only: the chosen expert indices, in the order chosen (Sec. 4.3)."""
     import numpy as np
     m = np.ascontiguousarray(mass, np.float64)
     c = np.ascontiguousarray(cost, np.float64)
@@ -328,7 +328,7 @@ class AspLinear:
     def __init__(self, W_bf16: torch.Tensor, U: torch.Tensor | None, group: int = 64, stream=None,
                  fmt: int = QWAM_FMT_INT4, rotate: bool = False, s: torch.Tensor | None = None):
         """fmt QWAM_FMT_INT4 (group 32 or 64) or QWAM_FMT_NVFP4 (App. B.1's Blackwell format;
-        `group` is then ignored: the block is 16).  rotate=True packs W~ = H diag(s) W (Sec. 2
+        `group` is then ignored: the block is 16).  rotate=True packs W~ = H diag(s) W (Sec. 3
         Eq. (pair); s float32 [K] smoothing factors or None) and rotates X at run time; U is then
         the basis in the rotated coordinates."""
         assert W_bf16.is_cuda and W_bf16.dtype == torch.bfloat16 and W_bf16.is_contiguous()
@@ -362,19 +362,18 @@ class AspLinear:
         return self._ws
 
     def act_views(self, M: int, ws: torch.Tensor | None = None):
-        """Views of the workspace for M tokens: code bytes uint8 [M, K] (E4M3 of c * 2^-9),
-        scales f32 [K/G, M_pad], epilogue constants f32 [K/G, M_pad, 2] = (alpha, beta) with
-        alpha = 2^18 s_x and beta = -8 s_x S_a, p_hat f16 [M, r_pad]."""
+        """Views of the workspace for M tokens: packed codes uint8 [M, K/2] (SM4 words: word j of a
+        row holds k = 8j..8j+7, see qwam_asp_act_layout), scales f32 [K/G, M_pad], p_hat f16
+        [M, r_pad]."""
         ws = self.workspace(M) if ws is None else ws
         L = qwam_asp_act_layout(self.h, M)
         if self.fmt == QWAM_FMT_NVFP4:
             return self.act_views_nvfp4(M, ws)
-        codes = ws[L["codes_off"]:L["codes_off"] + M * self.K].view(M, self.K)
+        codes = ws[L["codes_off"]:L["codes_off"] + M * (self.K // 2)].view(M, self.K // 2)
         ns = self.K // self.group
         scales = ws[L["scales_off"]:L["scales_off"] + ns * L["M_pad"] * 4].view(torch.float32).view(ns, L["M_pad"])
-        ab = ws[L["ab_off"]:L["ab_off"] + ns * L["M_pad"] * 8].view(torch.float32).view(ns, L["M_pad"], 2)
         ph = ws[L["phat_off"]:L["phat_off"] + M * self.r_pad * 2].view(torch.float16).view(M, self.r_pad)
-        return codes, scales, ab, ph
+        return codes, scales, ph
 
     def act_views_nvfp4(self, M: int, ws: torch.Tensor | None = None):
         """NVFP4 workspace views: packed codes uint8 [M, K/2] (low nibble = even k), the scale

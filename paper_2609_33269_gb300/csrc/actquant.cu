@@ -1,6 +1,6 @@
 // actquant.cu -- kernel (a): the run-time activation path of the ASP layer.
 //
-//   p      = X U                (Sec. 3.2 Eq. (xsplit): the protected coordinates V^T x)
+//   p      = X U                (Sec. 4.2 Eq. (xsplit): the protected coordinates V^T x)
 //   X_perp = X - p U^T          (the remainder (I - V V^T) x)
 //   s_x    = RN_f32(absmax(X_perp over a group) / 7),  codes = nearest(X_perp / s_x)
 //                               (Eq. (quant) with b = 4; App. B.1: per token, per group)
@@ -16,10 +16,9 @@
 // X_perp = X - R in float32 and quantize it.  With r = 0 the kernel is one streaming pass.
 //
 // Outputs per token row m and group g (the activation workspace):
-//   codes[m, k]   one byte per code, E4M3 bit pattern of c * 2^-9 (sign | magnitude, a
-//                 subnormal): the GEMM feeds these bytes to the tensor cores unchanged;
-//   s_x[g, m]     float32 scale;   ab[g, m]  (2^18 s_x, -8 s_x S_a), S_a the group's code sum:
-//                 the GEMM epilogue's per-row constants, each rounded once;
+//   codes[m, :]   packed at four bits, SM4 words (sm4_pack: word j holds k = 8j..8j+7,
+//                 sign-magnitude), which the GEMM expands to E4M3 bytes of c * 2^-9;
+//   s_x[g, m]     float32 scale;
 //   p_hat[m, :]   float16.
 // NVFP4 variant (App. B.1, the same kernel with one template flag): per block of 16 K an E4M3
 // scale (in the 512-byte atoms the GEMM copies to tensor memory) and E2M1 codes, two per byte.
@@ -29,7 +28,7 @@
 // and the odd K chunks respectively.
 //
 // Also in this file, sharing kernel (a)'s quantizers (the same rounding, bit for bit):
-//   rotquant_kernel  smoothing and block Hadamard rotation of the remainder (Sec. 2 Eq. (pair)),
+//   rotquant_kernel  smoothing and block Hadamard rotation of the remainder (Sec. 3 Eq. (pair)),
 //                    then quantization, one warp per token row and Hadamard block;
 //   smallq_kernel    the whole activation path on the CUDA cores, one CTA per token row, for few
 //                    tokens and for r = 0 layers (with the rotation for rotated layers);
@@ -45,10 +44,9 @@ namespace {
 
 struct ActArgs {
   int M, K, G, C, Kc, M_pad;
-  uint8_t* codes;   // [M, K] (NVFP4: [M, K/2], two codes per byte, low nibble = even k)
+  uint8_t* codes;   // [M, K/2]: SM4 words (NVFP4: E2M1 codes, two per byte, low nibble = even k)
   uint8_t* sf;      // NVFP4: E4M3 block scales in 512-byte atoms
   float* scales;    // [K/G, M_pad]
-  float2* ab;       // [K/G, M_pad]: (alpha, beta)
   __half* phat;     // [M, RP]
   float* dump;      // optional [M, K]
   int resid_only;   // rotated layer: write the remainder to dump and stop (the rotation kernel quantizes)
@@ -101,11 +99,10 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return r;
 }
 
-// One group of GS remainder values -> scale, epilogue constants and GS code bytes (E4M3 of
-// c * 2^-9).  The absmax and the code sum are formed as trees (max is exact and the sum is of
-// integers, so the order does not matter), which keeps the dependency chains short.
+// One group of GS remainder values -> scale and GS/8 SM4 words of codes.  The absmax is formed
+// as a tree (max is exact, so the order does not matter), which keeps the dependency chain short.
 template <int GS>
-__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4, float* scale_out, float2* ab_out) {
+__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words, float* scale_out) {
   float mx[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) mx[j] = fabsf(xp[j]);
@@ -123,23 +120,16 @@ __device__ __forceinline__ void quantize_group(const float* xp, uint32_t* bytes4
   const float scs = sc * k;
   const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
   const float hs = 0.5f * scs;
-  int sums[4] = {0, 0, 0, 0};
 #pragma unroll
-  for (int w = 0; w < GS / 4; ++w) {
-    uint32_t b[4];
+  for (int w = 0; w < GS / 8; ++w) {
+    uint32_t b[8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int ci = nearest_code(xp[4 * w + u] * k, scs, inv, hs);
-      sums[u] += ci;
-      b[u] = static_cast<uint32_t>(abs(ci)) | (static_cast<uint32_t>(ci) & 0x80u);
-    }
-    bytes4[w] = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+    for (int u = 0; u < 8; ++u) b[u] = sm4_byte(nearest_code(xp[8 * w + u] * k, scs, inv, hs));
+    const uint32_t lo = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+    const uint32_t hi = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
+    words[w] = sm4_pack(lo, hi);
   }
-  const int sum = (sums[0] + sums[1]) + (sums[2] + sums[3]);
   *scale_out = sc;
-  // the GEMM epilogue's constants for this token and group: alpha = 2^18 s_x (exact) and
-  // beta = -8 s_x S_a (-8 s_x is exact; one rounding)
-  *ab_out = make_float2(sc * 262144.0f, (-8.0f * sc) * static_cast<float>(sum));
 }
 
 // ---- NVFP4 variant (App. B.1): one block of 16 remainder values -> E4M3 scale and E2M1 codes.
@@ -550,18 +540,17 @@ __global__ void __launch_bounds__(320, 1)
                                      (mr % 32) * 16 + (mr / 32) * 4) = sf4;
         continue;
       }
-      uint32_t bytes4[16];
+      uint32_t words[8];
       if (a.G == 64) {
-        const size_t gi = static_cast<size_t>(kc / 64) * a.M_pad + m;
-        quantize_group<64>(xp, bytes4, a.scales + gi, a.ab + gi);
+        quantize_group<64>(xp, words, a.scales + static_cast<size_t>(kc / 64) * a.M_pad + m);
       } else {
         const size_t gi = static_cast<size_t>(kc / 32) * a.M_pad + m;
-        quantize_group<32>(xp, bytes4, a.scales + gi, a.ab + gi);
-        quantize_group<32>(xp + 32, bytes4 + 8, a.scales + gi + a.M_pad, a.ab + gi + a.M_pad);
+        quantize_group<32>(xp, words, a.scales + gi);
+        quantize_group<32>(xp + 32, words + 4, a.scales + gi + a.M_pad);
       }
-      uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * a.K + kc);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) dst[i] = make_uint4(bytes4[4 * i], bytes4[4 * i + 1], bytes4[4 * i + 2], bytes4[4 * i + 3]);
+      uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * (a.K / 2) + kc / 2);
+      dst[0] = make_uint4(words[0], words[1], words[2], words[3]);
+      dst[1] = make_uint4(words[4], words[5], words[6], words[7]);
     }
   }
 
@@ -600,22 +589,21 @@ __global__ void __launch_bounds__(128) debug_quantize_kernel(const float* R, int
     dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
     dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
   } else {
-    uint32_t bytes4[16];
-    float2 ab[2];
+    uint32_t words[8];
     float* sc = static_cast<float*>(scales) + static_cast<size_t>(m) * (K / G) + c * (kChunk / G);
     if (G == 64) {
-      quantize_group<64>(xp, bytes4, sc, ab);
+      quantize_group<64>(xp, words, sc);
     } else {
-      quantize_group<32>(xp, bytes4, sc, ab);
-      quantize_group<32>(xp + 32, bytes4 + 8, sc + 1, ab + 1);
+      quantize_group<32>(xp, words, sc);
+      quantize_group<32>(xp + 32, words + 4, sc + 1);
     }
-    uint4* dst = reinterpret_cast<uint4*>(codes + static_cast<size_t>(m) * K + c * kChunk);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(bytes4[4 * i], bytes4[4 * i + 1], bytes4[4 * i + 2], bytes4[4 * i + 3]);
+    uint4* dst = reinterpret_cast<uint4*>(codes + static_cast<size_t>(m) * (K / 2) + c * (kChunk / 2));
+    dst[0] = make_uint4(words[0], words[1], words[2], words[3]);
+    dst[1] = make_uint4(words[4], words[5], words[6], words[7]);
   }
 }
 
-// ---- run-time smoothing and block Hadamard rotation (Sec. 2 Eq. (pair); App. B.1) ----------
+// ---- run-time smoothing and block Hadamard rotation (Sec. 3 Eq. (pair); App. B.1) ----------
 //
 //   x~_perp = H diag(s)^-1 v,  v = x (r = 0) or v = x - diag(s) H U p (r > 0, from kernel (a))
 //
@@ -631,7 +619,6 @@ struct QuantOut {
   uint8_t* codes;
   uint8_t* sf;
   float* scales;
-  float2* ab;
 };
 
 struct RotArgs {
@@ -680,9 +667,9 @@ __device__ __forceinline__ uint32_t codes8_nvfp4(const float* x, float sc, float
 
 // The quantizers of kernel (a) on a warp-wide layout: each lane holds 8 consecutive remainder
 // values x (channels k .. k+7 of token row m, k a multiple of 8) and the lanes of one quantization
-// group (INT4: G/8 lanes; NVFP4: 2 lanes per block of 16) are neighbours.  Writes the codes and,
-// from the group's first lane, its scale (and, for INT4, the epilogue constants).  The scale, the
-// codes and the constants are those of quantize_group / quantize_block_nvfp4, bit for bit.
+// group (INT4: G/8 lanes; NVFP4: 2 lanes per block of 16) are neighbours.  Writes the codes (INT4:
+// the lane's SM4 word) and, from the group's first lane, its scale.  The scale and the codes are
+// those of quantize_group / quantize_block_nvfp4, bit for bit.
 template <bool NV>
 __device__ __forceinline__ void quantize8_lanes(const float* x, int lane, int m, int k, const QuantOut& o) {
   constexpr unsigned kAll = 0xFFFFFFFFu;
@@ -710,24 +697,12 @@ __device__ __forceinline__ void quantize8_lanes(const float* x, int lane, int m,
     const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
     const float hs = 0.5f * scs;
     uint32_t b[8];
-    int sum = 0;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int ci = nearest_code(x[i] * ks, scs, inv, hs);
-      sum += ci;
-      b[i] = static_cast<uint32_t>(abs(ci)) | (static_cast<uint32_t>(ci) & 0x80u);
-    }
-    sum += __shfl_xor_sync(kAll, sum, 1);
-    sum += __shfl_xor_sync(kAll, sum, 2);
-    if (o.G == 64) sum += __shfl_xor_sync(kAll, sum, 4);
-    const uint32_t w0 = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
-    const uint32_t w1 = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
-    *reinterpret_cast<uint2*>(o.codes + static_cast<size_t>(m) * o.K + k) = make_uint2(w0, w1);
-    if ((lane & (o.G / 8 - 1)) == 0) {
-      const size_t gi = static_cast<size_t>(k / o.G) * o.M_pad + m;
-      o.scales[gi] = sc;
-      o.ab[gi] = make_float2(sc * 262144.0f, (-8.0f * sc) * static_cast<float>(sum));
-    }
+    for (int i = 0; i < 8; ++i) b[i] = sm4_byte(nearest_code(x[i] * ks, scs, inv, hs));
+    const uint32_t lo = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+    const uint32_t hi = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
+    *reinterpret_cast<uint32_t*>(o.codes + static_cast<size_t>(m) * (o.K / 2) + k / 2) = sm4_pack(lo, hi);
+    if ((lane & (o.G / 8 - 1)) == 0) o.scales[static_cast<size_t>(k / o.G) * o.M_pad + m] = sc;
   }
 }
 
@@ -808,7 +783,6 @@ QuantOut quant_out(const Handle& h, const ActLayout& L, uint8_t* base) {
   q.codes = base + L.codes_off;
   q.sf = base + L.scales_off;
   q.scales = reinterpret_cast<float*>(base + L.scales_off);
-  q.ab = reinterpret_cast<float2*>(base + L.ab_off);
   return q;
 }
 
@@ -1068,7 +1042,6 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   a.codes = base + L.codes_off;
   a.sf = base + L.scales_off;
   a.scales = reinterpret_cast<float*>(base + L.scales_off);
-  a.ab = reinterpret_cast<float2*>(base + L.ab_off);
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
   a.dump = dump;
   a.resid_only = resid_only ? 1 : 0;
@@ -1148,7 +1121,7 @@ cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4,
 }
 
 cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
-                                        uint8_t* scales, float2* ab, int M_pad, cudaStream_t s) {
+                                        uint8_t* scales, int M_pad, cudaStream_t s) {
   QuantOut q;
   q.K = K;
   q.G = G;
@@ -1156,7 +1129,6 @@ cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4
   q.codes = codes;
   q.sf = scales;
   q.scales = reinterpret_cast<float*>(scales);
-  q.ab = ab;
   const long long warps = static_cast<long long>(M) * (K / 256);
   const int grid = static_cast<int>((warps + 7) / 8);
   if (nvfp4)

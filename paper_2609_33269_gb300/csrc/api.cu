@@ -94,9 +94,9 @@ ActLayout act_layout(const Handle& h, int M) {
     }
     return L;
   }
-  L.scales_off = up256(static_cast<size_t>(M) * h.K);
+  L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
   L.ab_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
-  L.phat_off = L.ab_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 8);
+  L.phat_off = L.ab_off;
   L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
   L.resid_off = 0;
   if (h.rot && h.r > 0) {
@@ -125,14 +125,17 @@ const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
     ok &= encode_2d(&c.qx4_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, kFp4KS / 2,
                     kBM, CU_TENSOR_MAP_SWIZZLE_128B);
   } else {
-    ok &= encode_2d(&c.qx_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K, M, h.K, kGemmKS, kBM,
-                    CU_TENSOR_MAP_SWIZZLE_128B);
-    ok &= encode_2d(&c.ab_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.ab_off, 2 * static_cast<uint64_t>(M),
-                    h.K / h.G, static_cast<uint64_t>(L.M_pad) * 8, 2 * kBM, kScaleGroups, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= encode_2d(&c.qa_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, 64, kBM,
+                    CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= encode_2d(&c.sx_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.scales_off, M, h.K / h.G,
+                    static_cast<uint64_t>(L.M_pad) * 4, kBM, kScaleGroups, CU_TENSOR_MAP_SWIZZLE_NONE);
   }
-  if (h.r_pad > 0)
+  if (h.r_pad > 0) {
     ok &= encode_2d(&c.ph_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
                     static_cast<uint64_t>(h.r_pad) * 2, 8, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= encode_2d(&c.ph32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
+                    static_cast<uint64_t>(h.r_pad) * 2, 32, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+  }
   if (!ok) return nullptr;
   c.ws = ws;
   c.x = x;
@@ -245,15 +248,18 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
     ok &= qwam::encode_2d(&h.qw4_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kFp4KS / 2,
                           qwam::kGemmBN, CU_TENSOR_MAP_SWIZZLE_128B);
   } else {
-    ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kGemmKS / 2,
-                          qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
-    ok &= qwam::encode_2d(&h.sw32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, h.sw32, N, K / group,
-                          static_cast<uint64_t>(h.N_pad) * 4, qwam::kGemmBN, qwam::kScaleGroups,
+    ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, 64, qwam::kBM,
+                          CU_TENSOR_MAP_SWIZZLE_NONE);
+    // sigma is permuted within 32-column blocks, so the map spans every column of N_pad
+    ok &= qwam::encode_2d(&h.sw32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, h.sw32, h.N_pad, K / group,
+                          static_cast<uint64_t>(h.N_pad) * 4, qwam::kBM, qwam::kScaleGroups,
                           CU_TENSOR_MAP_SWIZZLE_NONE);
   }
   if (h.r_pad > 0) {
     ok &= qwam::encode_2d(&h.Bh_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,
                           static_cast<uint64_t>(h.r_pad) * 2, 8, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= qwam::encode_2d(&h.bh32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,
+                          static_cast<uint64_t>(h.r_pad) * 2, 32, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
     ok &= qwam::encode_2d(&h.ucat_t_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h.ucat_t, K, 2 * h.r_pad,
                           static_cast<uint64_t>(K) * 2, qwam::kChunk, 2 * h.r_pad, CU_TENSOR_MAP_SWIZZLE_128B);
     ok &= qwam::encode_2d(&h.ucat3_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h.ucat3, h.ku3, K,
@@ -371,19 +377,17 @@ qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, 
 }
 
 qwam_status qwam_asp_debug_quantize_lanes(const float* R, int M, int K, int fmt, int group, void* codes, void* scales,
-                                          void* ab, struct CUstream_st* stream) {
+                                          struct CUstream_st* stream) {
   if (M < 0 || K <= 0 || K % 256 != 0) return QWAM_ERR_INVALID_ARG;
   if (fmt != QWAM_FMT_INT4 && fmt != QWAM_FMT_NVFP4) return QWAM_ERR_INVALID_ARG;
   if (fmt == QWAM_FMT_INT4 && group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
   if (M == 0) return QWAM_OK;
   if (!R || !codes || !scales || !qwam::aligned16(R) || !qwam::aligned16(codes)) return QWAM_ERR_INVALID_ARG;
-  if (fmt == QWAM_FMT_INT4 && (!ab || reinterpret_cast<uintptr_t>(scales) % 4 != 0 ||
-                               reinterpret_cast<uintptr_t>(ab) % 8 != 0))
-    return QWAM_ERR_INVALID_ARG;
+  if (fmt == QWAM_FMT_INT4 && reinterpret_cast<uintptr_t>(scales) % 4 != 0) return QWAM_ERR_INVALID_ARG;
   const int M_pad = qwam::round_up(M, qwam::kBM);
   return from_cuda_status(qwam::launch_debug_quantize_lanes(
       R, M, K, fmt == QWAM_FMT_NVFP4, fmt == QWAM_FMT_NVFP4 ? qwam::kFp4Block : group, static_cast<uint8_t*>(codes),
-      static_cast<uint8_t*>(scales), static_cast<float2*>(ab), M_pad, reinterpret_cast<cudaStream_t>(stream)));
+      static_cast<uint8_t*>(scales), M_pad, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 qwam_status qwam_asp_smoothing_factors(const float* xmax, const void* W_bf16, int K, int N, double alpha, float* s,
@@ -492,15 +496,18 @@ qwam_status qwam_asp_export(qwam_asp_handle hs, void* qw, void* sw, void* Bh, vo
   if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
   cudaError_t e = cudaSuccess;
   if (qw) {
-    // device words hold k = 8j..8j+3 in low and 8j+4..8j+7 in high nibbles; export pairs (2q, 2q+1)
-    std::vector<uint8_t> t(static_cast<size_t>(h.N) * (h.K / 2));
-    e = cudaMemcpy(t.data(), h.qw, t.size(), cudaMemcpyDeviceToHost);
+    // device rows are SM4 words (word j: k = 8j..8j+7, sign-magnitude); export two's-complement
+    // nibbles, low nibble = even k
+    std::vector<uint32_t> t(static_cast<size_t>(h.N) * (h.K / 8));
+    e = cudaMemcpy(t.data(), h.qw, t.size() * 4, cudaMemcpyDeviceToHost);
     uint8_t* o = static_cast<uint8_t*>(qw);
-    for (size_t wd = 0; e == cudaSuccess && wd < t.size() / 4; ++wd) {
+    for (size_t wd = 0; e == cudaSuccess && wd < t.size(); ++wd) {
+      const uint32_t lo = t[wd] & 0x87878787u, hi = ((t[wd] >> 4) | (t[wd] << 28)) & 0x87878787u;
       uint8_t c[8];
-      for (int i = 0; i < 4; ++i) {
-        c[i] = t[4 * wd + i] & 0xF;
-        c[4 + i] = t[4 * wd + i] >> 4;
+      for (int i = 0; i < 8; ++i) {
+        const uint32_t b = ((i < 4 ? lo : hi) >> (8 * (i & 3))) & 0xFFu;
+        const int v = (b & 0x80u) ? -static_cast<int>(b & 7u) : static_cast<int>(b & 7u);
+        c[i] = static_cast<uint8_t>(v & 0xF);
       }
       for (int q = 0; q < 4; ++q) o[4 * wd + q] = static_cast<uint8_t>(c[2 * q] | (c[2 * q + 1] << 4));
     }

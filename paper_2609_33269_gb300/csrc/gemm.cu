@@ -1,44 +1,44 @@
 // gemm.cu -- kernel (b): the 4-bit deflated path of Eq. (asp) with the 16-bit branch fused into
-// the epilogue (Sec. 3.2; App. B.1 describes the paper's GEMM as one that keeps the weights
+// the same kernel (Sec. 4.2; App. B.1 describes the paper's GEMM as one that keeps the weights
 // packed at 4 bits and adds the protected branch in its epilogue).
 //
 //   Y[m, n] = sum_g s_x[m, g] s_w[g, n] P_g[m, n]  +  sum_j p_hat[m, j] B_hat[n, j]
 //   P_g[m, n] = sum_{k in group g} q_x[m, k] q_w[n, k]          (exact integers)
 //
-// sm_103a has no integer tensor-core MMA, so the codes are fed to tcgen05.mma.kind::f8f6f4 as
-// E4M3 bit patterns of exact multiples of 2^-9 (E4M3 subnormals, which the tensor core keeps):
-//   A: activation byte = sign | |c|      -> value c * 2^-9     (written so by kernel (a))
-//   B: weight byte     = c + 8 in [1,15] -> value (c + 8) 2^-9 (expanded here from 4 bits)
-// so one group's float32 accumulator holds D = 2^-18 sum_k c_a (c_b + 8) = 2^-18 (P + 8 S_a)
-// exactly (S_a = the activation group's code sum, every partial sum an integer below 2^13 times
-// 2^-18).  The epilogue forms s_x P = alpha D + beta with alpha = 2^18 s_x, beta = -8 s_x S_a
-// (per row and group) and accumulates s_w * (s_x P) in float32 registers.  The 4-bit weights
-// stay packed in HBM; a nibble becomes its byte with three logic ops per eight nibbles because
-// the packing puts the codes of k = 8j..8j+3 in the low and of k = 8j+4..8j+7 in the high
-// nibbles of the four bytes of word j.  Each group has its own TMEM accumulator (four buffers);
-// after the last group of a tile one kind::f16 MMA of K = r_pad forms p_hat B_hat^T, which the
-// epilogue adds with scale 1.
+// sm_103a has no integer tensor-core MMA, so both operands go to tcgen05.mma.kind::f8f6f4 as
+// E4M3 bytes of c * 2^-9 (sign | |c|: E4M3 subnormals, which the tensor core keeps exactly).  One
+// group's float32 accumulator then holds D = 2^-18 P_g exactly (every partial sum is an integer
+// below 2^13 times 2^-18).  The epilogue accumulates s_x s_w P_g as (D s_x) sigma, where
+// sigma = 2^18 s_w is the handle's float32 copy of the weight scale: two float32 roundings per
+// output and group, the float32 running sum a third.
 //
-// Persistent CTAs (one per SM) walk output tiles of 128 x 128 with a static stride; every ring
-// runs continuously across tiles, so loads for the next tile overlap the epilogue of the current
-// one.  384 threads in three warpgroups (kEpiWarpsPerQuad = 2; 4 gives 640 threads):
-//   warpgroup 0 (80 registers): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2-3
-//     expand weight nibbles into the operand stage;
-//   warpgroups 1-2 (208 registers): warps 4..11 epilogue.  A warp owns 32 rows x 64 columns of
-//     the tile; TMEM is read with the 16x256b shape, so a thread holds 4 rows x 16 columns (as
-//     packed f32x2 pairs) and, per group, loads 16 column scales s_w and the constants
-//     (alpha, beta) of its 4 rows, which kernel (a) wrote.  With one row per
-//     thread, moving the scales into registers cost as much as the arithmetic; here the floor is
-//     the FMA pipe, two operations per output and group, and the issue of everything around it.
-// Rings (each waiter waits for every phase of its slots in turn):
-//   O  operand stage = activation codes (TMA) + expanded weights (expanders)  -> MMA     SO slots
-//   P  packed weights of a stage  TMA -> expanders                                      SP slots
-//   S  alpha, beta, s_w of eight groups  TMA -> epilogue                                SS slots
-//   T  TMEM accumulators, units of two groups (2 x 128 columns)  MMA -> epilogue        NTB units
-//   B  p_hat / B_hat tiles  TMA -> MMA, loaded after the tile's stages                   one per tile
-// Every barrier operation costs on the order of 100 cycles, so each role touches as few as
-// possible per stage: the MMA warp waits twice and commits twice, the expanders wait twice and
-// arrive twice, the epilogue waits once and arrives once per unit, plus once each per S slot.
+// Both operands stay packed at 4 bits in HBM (SM4 words, see sm4_pack) and are expanded to bytes
+// in shared memory: lo = w & 0x87878787 (k = 8j..8j+3), hi = rotr(w, 4) & 0x87878787 (k = 8j+4..).
+//
+// Persistent CTAs (one per SM) walk output tiles of 128 x 128 with a static stride (row-block
+// major, so the CTAs working at one time share the activation rows in L2).  Every ring runs
+// continuously across tiles.  384 threads:
+//   warp 0        TMA producer: packed codes of both operands per stage, scale slots;
+//   warp 1        MMA issuer and TMEM owner;
+//   warps 2, 3    expanders: packed stage -> byte operand stage (128-byte swizzle);
+//   warps 4..11   epilogue: warp 4 + 4h + q reads TMEM lane quadrant q, columns 64h .. 64h + 63.
+// Stages cover 128 K (two groups of 64 or four of 32).  After a tile's K stages come r_pad / 32
+// branch stages: the producer brings 32 columns of p_hat and B_hat (float16) through the same
+// packed ring, the expanders copy them into the operand layout, and the MMA issuer runs two
+// kind::f16 MMAs (K = 16 each); the branch accumulates in its own TMEM unit, which the epilogue
+// adds with scale 1.  Any r_pad works.
+// TMEM holds four units of 128 columns, one group each (unit g mod 4), so the MMA issuer runs up
+// to four groups ahead of the epilogue.  An mbarrier wait costs on the order of a hundred cycles
+// even when its phase has completed, so each role waits as little as possible: the MMA issuer
+// once per stage for its operands and once for the last TMEM unit the stage writes (the epilogue
+// releases units in order); each epilogue warp once per group, for the unit after the one it is
+// about to compute (its TMEM loads are double-buffered across groups, so a group's load latency
+// overlaps the arithmetic of the previous one).
+// Rings (every wait is bounded):
+//   P  packed stage (A and B codes, or p_hat / B_hat)   TMA -> expanders          SP slots
+//   O  operand stage (A and B bytes)                    expanders -> MMA          SO slots
+//   S  scale slot: s_x and sigma of kSG groups           TMA -> epilogue           SS slots
+//   T  TMEM units                                       MMA -> epilogue           4 units
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -46,7 +46,8 @@ namespace qwam {
 namespace {
 
 struct GemmArgs {
-  int M, N, K, G;
+  int M, N, K;
+  int nbs;  // branch stages per tile (r_pad / 32, rounded up)
   int m_tiles, n_tiles;
   void* Y;
   int y_f32;
@@ -55,46 +56,31 @@ struct GemmArgs {
   uint64_t timeout_ns;
 };
 
-constexpr int kEpiWarpsPerQuad = 2;                 // epilogue warps per 32-row quadrant (2 or 4)
-constexpr int CBW = 4 / kEpiWarpsPerQuad;           // 32-column blocks per epilogue warp
-constexpr int kThreads = 128 + 128 * kEpiWarpsPerQuad;
-constexpr int kLaunchRegs = kEpiWarpsPerQuad == 4 ? 96 : 168;  // 65536 / threads, multiple of 8
-constexpr int kRegsCtl = kEpiWarpsPerQuad == 4 ? 56 : 80;     // warpgroup 0
-constexpr int kRegsEpi = kEpiWarpsPerQuad == 4 ? 104 : 208;   // the epilogue warpgroups
-static_assert(128 * kRegsCtl + (kThreads - 128) * kRegsEpi <= kThreads * kLaunchRegs,
-              "register split above the launch allocation");
-constexpr int SO = 3;     // operand stages
-constexpr int SP = 6;     // packed-weight stages
-constexpr int SS = 3;     // scale stages (kScaleGroups groups each)
-constexpr int NTB = 2;    // TMEM accumulator units (2 x 128 columns each)
-constexpr int NBR = 1;    // branch-operand stages (one per tile)
-constexpr int NXW = 2;    // expander warps
-constexpr int NEPIW = 4 * kEpiWarpsPerQuad;  // epilogue warps (32 * CBW columns each)
-constexpr int A_BYTES = kBM * kGemmKS;            // 16 KB, 128-byte swizzle
-constexpr int X_BYTES = kGemmBN * kGemmKS;        // 16 KB, 128-byte swizzle
-constexpr int OSTAGE = A_BYTES + X_BYTES;
-constexpr int PB_BYTES = kGemmBN * kGemmKS / 2;   // 8 KB packed weights
-constexpr int PSTAGE = PB_BYTES;
-constexpr int SAB_BYTES = kScaleGroups * 128 * 8;  // 8 groups x 128 rows x (alpha, beta)
-constexpr int SSW_BYTES = kScaleGroups * 128 * 4;  // 8 groups x 128 f32 s_w
-constexpr int SSTAGE = SAB_BYTES + SSW_BYTES;      // 12 KB
-
-template <int RP>
-struct GemmCfg {
-  static constexpr int BR_BYTES = RP * kBM * 2;   // p_hat tile (and the B_hat tile), RP/8 boxes of 2 KB
-  static constexpr int NBAR = 2 * SO + 2 * SP + 2 * SS + 2 * NTB + 2 * NBR + 1;
-  static constexpr int SMEM = 1024 + SO * OSTAGE + SP * PSTAGE + SS * SSTAGE + NBR * 2 * BR_BYTES + NBAR * 8 + 16;
-  static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
-};
+constexpr int kBN = 128;       // output columns per tile
+constexpr int kKS = 128;       // K per stage (128 codes: 64 packed bytes, 128 operand bytes per row)
+constexpr int kSG = 8;         // groups per scale slot
+constexpr int kNX = 2;         // expander warps
+constexpr int kThreads = 384;  // 12 warps
+constexpr int kLaunchRegs = 168;
+constexpr int kRegsCtl = 48;   // warpgroup 0 (producer, MMA, expanders)
+constexpr int kRegsEpi = 224;  // warpgroups 1-2 (epilogue)
+static_assert(128 * kRegsCtl + 256 * kRegsEpi <= kThreads * kLaunchRegs, "register split above the launch allocation");
+constexpr int SO = 4;  // operand stages
+constexpr int SP = 4;  // packed stages
+constexpr int SS = 2;  // scale slots
+constexpr int A_PK = kBM * 64;                // packed A rows (64 bytes each), then B rows
+constexpr int PSTAGE = (kBM + kBN) * 64;      // 16 KB
+constexpr int A_OP = kBM * 128;               // byte operands, 128-byte rows, 128-byte swizzle
+constexpr int OSTAGE = (kBM + kBN) * 128;     // 32 KB
+constexpr int SX_BYTES = kSG * kBM * 4;       // s_x [kSG][128]
+constexpr int SSLOT = kSG * (kBM + kBN) * 4;  // then sigma [kSG][128]
+constexpr int ONES_BYTES = 512;               // 128 floats of 1.0: the branch group's scales
+constexpr int NBAR = 2 * (SO + SP + SS + 4) + 1;
+constexpr int SMEM = 1024 + SO * OSTAGE + SP * PSTAGE + SS * SSLOT + ONES_BYTES + NBAR * 8 + 16;
+static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 
 typedef unsigned long long f2;  // two packed float32 (for the f32x2 instructions)
 
-__device__ __forceinline__ f2 pk(float lo, float hi) {
-  return static_cast<f2>(__float_as_uint(lo)) | (static_cast<f2>(__float_as_uint(hi)) << 32);
-}
-__device__ __forceinline__ f2 pku(uint32_t lo, uint32_t hi) {
-  return static_cast<f2>(lo) | (static_cast<f2>(hi) << 32);
-}
 __device__ __forceinline__ float lo_f(f2 v) { return __uint_as_float(static_cast<uint32_t>(v)); }
 __device__ __forceinline__ float hi_f(f2 v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
 __device__ __forceinline__ f2 fma2(f2 a, f2 b, f2 c) {
@@ -102,86 +88,179 @@ __device__ __forceinline__ f2 fma2(f2 a, f2 b, f2 c) {
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
   return d;
 }
+__device__ __forceinline__ f2 mul2(f2 a, f2 b) {
+  f2 d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
 __device__ __forceinline__ f2 add2(f2 a, f2 b) {
   f2 d;
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
+__device__ __forceinline__ f2 pk2u(uint32_t a, uint32_t b) {
+  f2 d;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "r"(a), "r"(b));
+  return d;
+}
+__device__ __forceinline__ f2 pk4(float a, float b) {
+  f2 d;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(a), "f"(b));
+  return d;
+}
 
-template <int RP>
+// SM4 word -> the E4M3 bytes of its eight codes (k order).
+__device__ __forceinline__ uint2 sm4_expand(uint32_t w) {
+  return make_uint2(w & 0x87878787u, __funnelshift_r(w, w, 4) & 0x87878787u);
+}
+
+// Everything one epilogue warp needs to process a group (see the epilogue in gemm_kernel).
+struct EpiCtx {
+  const uint8_t* sring;   // scale slots
+  const float* ones;      // 128 floats of 1.0 (the branch group's scales)
+  uint64_t* sfull;
+  uint64_t* sempty;
+  uint64_t* tfull;
+  uint64_t* tempty;
+  WaitCtl wc;
+  uint32_t tq;            // TMEM address of this warp's lane quadrant and column half
+  int quad, h, rq, cq;
+  int ngk, ngt, total;    // K groups per tile, groups per tile, groups of this CTA
+};
+
+// One group of the epilogue: g is the CTA's running group index (TMEM unit g % 4), gi its index in
+// the tile, sl the running index of the scale slot it reads.  Its TMEM loads sit in v[CUR] (issued
+// while the previous group was computed); the loads of group g + 1 go to v[CUR ^ 1] block by block.
+template <int CUR>
+__device__ __forceinline__ void epi_group(const EpiCtx& c, f2 (&acc)[32], uint32_t (&v)[2][4][16], int& g, int& gi,
+                                          int& sl, bool& ok) {
+  const bool more = g + 1 < c.total;
+  const bool kgroup = gi < c.ngk;
+  const int gi_n = gi + 1 == c.ngt ? 0 : gi + 1;
+  const bool slot_n = gi_n < c.ngk && (gi_n & (kSG - 1)) == 0;  // group g + 1 starts a scale slot
+  const int gl = gi & (kSG - 1);
+  // v[CUR][2b + rh][4j + 2rr + {0, 1}] = columns (32b + 8j + 2cq, +1) of row rq + 16 rh + 8 rr
+  tmem_ld_wait_dep4(v[CUR]);
+  tc_fence_before();
+  // Every load of the unit has landed: release it before waiting for the next group (whose stage
+  // the MMA issuer may only start once this unit is free).
+  warp_arrive(&c.tempty[g & 3]);
+  // The next group's phases, tested now and used after the first block: the test's latency
+  // overlaps the arithmetic.
+  const bool ready_n = !more || ((!slot_n || mbar_test_wait(&c.sfull[(sl + 1) & (SS - 1)], ((sl + 1) / SS) & 1)) &&
+                                 mbar_test_wait(&c.tfull[(g + 1) & 3], ((g + 1) >> 2) & 1));
+  const uint8_t* slot = c.sring + (sl & (SS - 1)) * SSLOT;
+  const float* sxb = kgroup ? reinterpret_cast<const float*>(slot) + gl * kBM : c.ones;
+  const float* sgb = kgroup ? reinterpret_cast<const float*>(slot + SX_BYTES) + gl * kBN : c.ones;
+  float sx[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) sx[k] = sxb[c.quad * 32 + c.rq + 8 * k];
+  const uint32_t tn = c.tq + static_cast<uint32_t>(((g + 1) & 3) * kBN);
+#pragma unroll
+  for (int b = 0; b < 2; ++b) {
+    const float4* sgp = reinterpret_cast<const float4*>(sgb + 64 * c.h + 32 * b + c.cq * 8);
+    const float4 s0 = sgp[0], s1 = sgp[1];
+    const f2 sg[4] = {pk4(s0.x, s0.y), pk4(s0.z, s0.w), pk4(s1.x, s1.y), pk4(s1.z, s1.w)};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const f2 sx2 = dup2(sx[k]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t* dv = &v[CUR][2 * b + (k >> 1)][4 * j + 2 * (k & 1)];
+        const f2 t = mul2(pk2u(dv[0], dv[1]), sx2);
+        acc[16 * b + 4 * k + j] = fma2(t, sg[j], acc[16 * b + 4 * k + j]);
+      }
+    }
+    if (b == 0) {
+      if (!ready_n && ok) {
+        if (slot_n) ok = mbar_wait_inline(&c.sfull[(sl + 1) & (SS - 1)], ((sl + 1) / SS) & 1, c.wc);
+        if (ok) ok = mbar_wait_inline(&c.tfull[(g + 1) & 3], ((g + 1) >> 2) & 1, c.wc);
+      }
+      tc_fence_after();
+    }
+    // Issued on every path (after the CTA's last group it reads a unit nobody uses any more), so
+    // that each wait's registers come from the loads just before it.
+    tmem_ld16x256_x4(tn + 32 * b, v[CUR ^ 1][2 * b]);
+    tmem_ld16x256_x4(tn + (16u << 16) + 32 * b, v[CUR ^ 1][2 * b + 1]);
+  }
+  if (kgroup && (gl == kSG - 1 || gi == c.ngk - 1)) {
+    fence_proxy_async_smem();  // reads of the TMA-written scales before the slot is refilled
+    warp_arrive(&c.sempty[sl & (SS - 1)]);
+  }
+  if (slot_n) ++sl;
+  ++g;
+  gi = gi_n;
+}
+
+template <int G>
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_kernel(const __grid_constant__ CUtensorMap qx_map, const __grid_constant__ CUtensorMap qw_map,
-                const __grid_constant__ CUtensorMap ab_map, const __grid_constant__ CUtensorMap sw_map, const __grid_constant__ CUtensorMap ph_map,
-                const __grid_constant__ CUtensorMap bh_map, const GemmArgs a) {
-  using Cfg = GemmCfg<RP>;
+    gemm_kernel(const __grid_constant__ CUtensorMap qa_map, const __grid_constant__ CUtensorMap qw_map,
+                const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap sw_map,
+                const __grid_constant__ CUtensorMap ph_map, const __grid_constant__ CUtensorMap bh_map,
+                const GemmArgs a) {
+  constexpr int GPS = kKS / G;  // groups per K stage
+  static_assert(kSG % GPS == 0, "a scale slot covers whole stages");
   extern __shared__ uint8_t smem_raw[];
   pdl_launch_dependents();
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* oring = smem;                           // SO x (A 16 KB | X 16 KB), 1024-aligned
-  uint8_t* pring = oring + SO * OSTAGE;            // SP x packed weights
-  uint8_t* sring = pring + SP * PSTAGE;            // SS x ((alpha, beta) | s_w)
-  uint8_t* br = sring + SS * SSTAGE;               // NBR x (p_hat | B_hat)
-  uint64_t* bars = reinterpret_cast<uint64_t*>(br + NBR * 2 * Cfg::BR_BYTES);
-  uint64_t* ofull = bars;
-  uint64_t* oempty = ofull + SO;
-  uint64_t* pfull = oempty + SO;
+  uint8_t* oring = smem;                 // SO x (A bytes | B bytes)
+  uint8_t* pring = oring + SO * OSTAGE;  // SP x (A packed | B packed)
+  uint8_t* sring = pring + SP * PSTAGE;  // SS x (s_x | sigma)
+  float* ones = reinterpret_cast<float*>(sring + SS * SSLOT);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sring + SS * SSLOT + ONES_BYTES);
+  uint64_t* pfull = bars;
   uint64_t* pempty = pfull + SP;
-  uint64_t* sfull = pempty + SP;
+  uint64_t* ofull = pempty + SP;
+  uint64_t* oempty = ofull + SO;
+  uint64_t* sfull = oempty + SO;
   uint64_t* sempty = sfull + SS;
   uint64_t* tfull = sempty + SS;
-  uint64_t* tempty = tfull + NTB;
-  uint64_t* bfull = tempty + NTB;
-  uint64_t* bempty = bfull + NBR;
-  uint64_t* drain = bempty + NBR;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + Cfg::NBAR);
+  uint64_t* tempty = tfull + 4;
+  uint64_t* drain = tempty + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NBAR);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const uint32_t wid = warp_id(), lane = lane_id();
-  const int G = a.G;
-  const int gps = kGemmKS / G;                    // groups per stage (2 or 4)
-  const int ngroups = a.K / G;
-  const int nst = (a.K + kGemmKS - 1) / kGemmKS;  // the last stage may be partly past K (zero-filled)
+  const int ngk = a.K / G;     // K groups per tile
+  const int nks = (a.K + kKS - 1) / kKS;  // K stages per tile (the last is half past K when K % 128 == 64:
+                                          // TMA zero-fills it and its missing groups are skipped)
+  const int nbs = a.nbs;       // branch stages per tile
+  const int nst = nks + nbs;
+  const int ngt = ngk + (nbs > 0 ? 1 : 0);  // groups per tile, the branch included
+  const int nsl = (ngk + kSG - 1) / kSG;    // scale slots per tile
   const int ntiles = a.m_tiles * a.n_tiles;
   const int my_tiles = ntiles > static_cast<int>(blockIdx.x)
                            ? (ntiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
                                  static_cast<int>(gridDim.x)
                            : 0;
-  auto tile_mn = [&](int i, int& m0, int& n0) {  // i-th tile of this CTA, m-major order
+  auto tile_mn = [&](int i, int& m0, int& n0) {
     const int t = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
     m0 = (t / a.n_tiles) * kBM;
-    n0 = (t % a.n_tiles) * kGemmBN;
+    n0 = (t % a.n_tiles) * kBN;
   };
-  auto groups_in = [&](int st) { return (st * gps + gps <= ngroups) ? gps : ngroups - st * gps; };
-  // A scale stage starts with every K stage whose first group is a multiple of kScaleGroups
-  // (gps divides kScaleGroups) and ends with the K stage that reaches the next one, or K.
-  auto scale_starts = [&](int st) { return (st * gps) % kScaleGroups == 0; };
-  auto scale_ends = [&](int st) { return ((st + 1) * gps) % kScaleGroups == 0 || st + 1 == nst; };
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < SO; ++i) {
-      mbar_init(&ofull[i], 1 + NXW);  // the producer's expect-tx arrival + one per expander warp
-      mbar_init(&oempty[i], 1);
-    }
     for (int i = 0; i < SP; ++i) {
       mbar_init(&pfull[i], 1);
-      mbar_init(&pempty[i], NXW);
+      mbar_init(&pempty[i], kNX);
+    }
+    for (int i = 0; i < SO; ++i) {
+      mbar_init(&ofull[i], kNX);
+      mbar_init(&oempty[i], 1);
     }
     for (int i = 0; i < SS; ++i) {
       mbar_init(&sfull[i], 1);
-      mbar_init(&sempty[i], NEPIW);
+      mbar_init(&sempty[i], 8);
     }
-    for (int i = 0; i < NTB; ++i) {
+    for (int i = 0; i < 4; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], NEPIW);
-    }
-    for (int i = 0; i < NBR; ++i) {
-      mbar_init(&bfull[i], 1);
-      mbar_init(&bempty[i], 1);
+      mbar_init(&tempty[i], 8);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
+  if (threadIdx.x < 128) ones[threadIdx.x] = 1.0f;
   if (wid == 1) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
@@ -196,132 +275,101 @@ __global__ void __launch_bounds__(kThreads, 1)
     setmaxnreg_dec<kRegsCtl>();
     if (wid == 0) {
       // ----------------------------------------------------------- TMA producer
-      // The whole warp walks the loop (so addresses, coordinates and barrier phases are
-      // warp-uniform and stay in uniform registers); one elected lane issues each copy.
+      // The whole warp walks the loop (warp-uniform state); one elected lane issues each copy.
       bool ok = true;
-      int s = 0, ss = 0;  // running K-stage and scale-stage counters (every role walks the same)
+      int s = 0, ss = 0;
       for (int ti = 0; ti < my_tiles && ok; ++ti) {
         int m0, n0;
         tile_mn(ti, m0, n0);
         for (int st = 0; st < nst && ok; ++st, ++s) {
-          if (scale_starts(st)) {
-            // (alpha, beta) and s_w of the next kScaleGroups groups (zero-filled past K)
+          if (st < nks && (st * GPS) % kSG == 0) {
+            // s_x and sigma of the next kSG groups (zero-filled past K)
             const int sb = ss % SS;
             if (ss >= SS) ok = mbar_wait_inline(&sempty[sb], ((ss / SS) & 1) ^ 1, wc);
             if (!ok) break;
-            uint8_t* q = sring + sb * SSTAGE;
+            uint8_t* q = sring + sb * SSLOT;
             if (elect_one()) {
-              mbar_arrive_expect_tx(&sfull[sb], SSTAGE);
-              tma_load_2d(q, &ab_map, &sfull[sb], 2 * m0, st * gps);
-              tma_load_2d(q + SAB_BYTES, &sw_map, &sfull[sb], n0, st * gps);
+              mbar_arrive_expect_tx(&sfull[sb], SSLOT);
+              tma_load_2d(q, &sx_map, &sfull[sb], m0, st * GPS);
+              tma_load_2d(q + SX_BYTES, &sw_map, &sfull[sb], n0, st * GPS);
             }
             __syncwarp();
             ++ss;
           }
-          // packed weights of this stage
           const int ps = s % SP;
           if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
           if (!ok) break;
           uint8_t* p = pring + ps * PSTAGE;
           if (elect_one()) {
-            mbar_arrive_expect_tx(&pfull[ps], PB_BYTES);
-            tma_load_2d(p, &qw_map, &pfull[ps], st * (kGemmKS / 2), n0);
-          }
-          __syncwarp();
-          // activation codes of this stage
-          const int os = s % SO;
-          if (s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
-          if (!ok) break;
-          if (elect_one()) {
-            mbar_arrive_expect_tx(&ofull[os], A_BYTES);
-            tma_load_2d(oring + os * OSTAGE, &qx_map, &ofull[os], st * kGemmKS, m0);
-          }
-          __syncwarp();
-        }
-        if constexpr (RP > 0) {
-          // the branch operands are needed only after the tile's last stage
-          const int bs = ti % NBR;
-          if (ok && ti >= NBR) ok = mbar_wait_inline(&bempty[bs], ((ti / NBR) & 1) ^ 1, wc);
-          if (!ok) break;
-          uint8_t* b = br + bs * 2 * Cfg::BR_BYTES;
-          if (elect_one()) {
-            mbar_arrive_expect_tx(&bfull[bs], 2 * Cfg::BR_BYTES);
-            for (int q = 0; q < RP / 8; ++q) {
-              tma_load_2d(b + q * 2048, &ph_map, &bfull[bs], q * 8, m0);
-              tma_load_2d(b + Cfg::BR_BYTES + q * 2048, &bh_map, &bfull[bs], q * 8, n0);
+            mbar_arrive_expect_tx(&pfull[ps], PSTAGE);
+            if (st < nks) {
+              tma_load_2d(p, &qa_map, &pfull[ps], st * (kKS / 2), m0);
+              tma_load_2d(p + A_PK, &qw_map, &pfull[ps], st * (kKS / 2), n0);
+            } else {
+              const int bs = st - nks;
+              tma_load_2d(p, &ph_map, &pfull[ps], bs * 32, m0);
+              tma_load_2d(p + A_PK, &bh_map, &pfull[ps], bs * 32, n0);
             }
           }
           __syncwarp();
         }
       }
-      // Let every issued load land before the CTA can exit (these phases complete in the
-      // normal course; after an abort the waits end at the deadline).
+      // Let every issued load land before the CTA can exit (these phases complete in the normal
+      // course; after an abort the waits end at the deadline).
       int never = 0;
       const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
       for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
       for (int j = (ss > SS ? ss - SS : 0); j < ss; ++j) mbar_wait_inline(&sfull[j % SS], (j / SS) & 1, dc);
-      // An operand stage also needs the expanders' arrivals: in the normal course they come;
-      // after an abort the wait ends at the deadline, long after the tile has landed.
-      for (int j = (s > SO ? s - SO : 0); j < s; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
-      if constexpr (RP > 0) {
-        for (int t = (my_tiles > NBR ? my_tiles - NBR : 0); t < my_tiles; ++t)
-          mbar_wait_inline(&bfull[t % NBR], (t / NBR) & 1, dc);
-      }
     } else if (wid == 1) {
       // ----------------------------------------------------------- MMA issuer
-      // The epilogue consumes accumulators in units of two groups (one TMEM buffer of 2 x 128
-      // columns); a unit never straddles a stage because a full stage holds an even number of
-      // groups.  The whole warp walks the loop and forms the descriptors (warp-uniform values);
-      // one elected lane (the same one throughout, as the commits track its MMAs) issues.
+      // The whole warp walks the loop and forms the descriptors; one elected lane (the same one
+      // throughout, as the commits track its MMAs) issues a stage's MMAs and commits together.
       bool ok = true;
-      constexpr uint32_t idesc = idesc_e4m3(kBM, kGemmBN);
-      int s = 0, u_all = 0;  // running stage and accumulator-unit counters
+      constexpr uint32_t idesc = idesc_e4m3(kBM, kBN);
+      constexpr uint32_t idesc_br = idesc_f16(kBM, kBN);
+      int s = 0, gr = 0;  // running stage and group counters
       for (int ti = 0; ti < my_tiles && ok; ++ti) {
         for (int st = 0; st < nst && ok; ++st, ++s) {
-          const int gn = groups_in(st);
           const int os = s % SO;
+          const bool kst = st < nks;
+          const int gn = kst ? min(GPS, ngk - st * GPS) : 1;  // groups this stage writes
           ok = mbar_wait_inline(&ofull[os], (s / SO) & 1, wc);
+          // the last TMEM unit this stage writes: its release (four groups back) implies the
+          // earlier ones (the epilogue releases units in order)
+          const int glast = gr + gn - 1;
+          if (ok && glast >= 4 && (kst || st == nks))
+            ok = mbar_wait_inline(&tempty[glast & 3], ((glast >> 2) & 1) ^ 1, wc);
           if (!ok) break;
-          const uint32_t aa = smem_u32(oring + os * OSTAGE), xa = aa + A_BYTES;
-          const uint64_t adesc0 = smem_desc(aa, 16, 1024, kSw128), xdesc0 = smem_desc(xa, 16, 1024, kSw128);
-          for (int g0 = 0; g0 < gn && ok; g0 += 2, ++u_all) {
-            const int ub = u_all % NTB;
-            if (u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
-            if (!ok) break;
-            tc_fence_after();
-            const int g1 = (g0 + 2 < gn) ? g0 + 2 : gn;
-            if (elect_one()) {
-              for (int gi = g0; gi < g1; ++gi)
-                for (int kk = 0; kk < G / 32; ++kk) {
-                  const uint64_t off = static_cast<uint64_t>((gi * (G / 32) + kk) * 32) >> 4;  // 16-byte units
-                  mma_f8f6f4(tmem + ub * 256 + (gi - g0) * 128, adesc0 + off, xdesc0 + off, idesc, kk != 0);
-                }
-              mma_commit(&tfull[ub]);
-            }
-            __syncwarp();
-          }
-          if (elect_one()) mma_commit(&oempty[os]);
-          __syncwarp();
-        }
-        if constexpr (RP > 0) {
-          const int bs = ti % NBR, ub = u_all % NTB;
-          if (ok) ok = mbar_wait_inline(&bfull[bs], (ti / NBR) & 1, wc);
-          if (ok && u_all >= NTB) ok = mbar_wait_inline(&tempty[ub], ((u_all / NTB) & 1) ^ 1, wc);
-          if (ok) {
-            tc_fence_after();
-            constexpr uint32_t idesc_br = idesc_f16(kBM, kGemmBN);
-            const uint32_t pa = smem_u32(br + bs * 2 * Cfg::BR_BYTES), pb = pa + Cfg::BR_BYTES;
-            const uint64_t pdesc0 = smem_desc(pa, 2048, 128, kSwNone), bdesc0 = smem_desc(pb, 2048, 128, kSwNone);
-            if (elect_one()) {
+          tc_fence_after();
+          const uint32_t aa = smem_u32(oring + os * OSTAGE);
+          const uint64_t adesc = smem_desc(aa, 16, 1024, kSw128), bdesc = smem_desc(aa + A_OP, 16, 1024, kSw128);
+          if (elect_one()) {
+            if (kst) {
 #pragma unroll
-              for (int kk = 0; kk < RP / 16; ++kk)
-                mma_f16(tmem + ub * 256, pdesc0 + kk * 256, bdesc0 + kk * 256, idesc_br, kk != 0);  // 4096 B
-              mma_commit(&tfull[ub]);
-              mma_commit(&bempty[bs]);
+              for (int gi = 0; gi < GPS; ++gi) {
+                if (gi >= gn) break;
+                const uint32_t d = tmem + static_cast<uint32_t>(((gr + gi) & 3) * kBN);
+#pragma unroll
+                for (int kk = 0; kk < G / 32; ++kk) {
+                  const uint64_t off = static_cast<uint64_t>((gi * G + kk * 32) >> 4);  // 16-byte units
+                  mma_f8f6f4(d, adesc + off, bdesc + off, idesc, kk != 0);
+                }
+                mma_commit(&tfull[(gr + gi) & 3]);
+              }
+            } else {
+              const int bs = st - nks;
+              const uint32_t d = tmem + static_cast<uint32_t>((gr & 3) * kBN);
+              mma_f16(d, adesc, bdesc, idesc_br, bs != 0);
+              mma_f16(d, adesc + 2, bdesc + 2, idesc_br, 1);
+              if (bs == nbs - 1) mma_commit(&tfull[gr & 3]);
             }
-            __syncwarp();
-            ++u_all;
+            mma_commit(&oempty[os]);
           }
+          __syncwarp();
+          if (kst)
+            gr += gn;
+          else if (st == nst - 1)
+            ++gr;
         }
       }
       if (elect_one()) mma_commit(drain);
@@ -330,14 +378,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
       mbar_wait_inline(drain, 0, dc);
     } else {
-      // ----------------------------------------------------------- weight expanders
-      // Thread e (0..63) owns the 16-byte chunk j = e % 8 of rows e/8 + 8 i (i = 0..15): its source
-      // and destination offsets only step by constants (512 and 1024 bytes).
+      // ----------------------------------------------------------- expanders
+      // Thread e (0..63) takes the 16-byte piece q = e % 4 of packed rows r0 + 16 i (r0 = e / 4,
+      // i = 0..15; rows 0..127 are A, 128..255 B): a K stage expands it to the operand chunks
+      // 2q, 2q + 1 of the row, a branch stage copies it to chunk q.  Operand rows are 128 bytes with
+      // the 128-byte swizzle (chunk c of row r at c ^ (r % 8)); r % 8 = r0 % 8 for all of this
+      // thread's rows, so every offset below is a constant.
       const int e = static_cast<int>(threadIdx.x) - 64;
-      const int r0 = e >> 3, j = e & 7;
-      const int src0 = r0 * 64 + j * 8;
-      const int dst0 = r0 * 128 + ((j ^ r0) << 4);
-      const uint32_t kX8 = 0x88888888u;
+      const int r0 = e >> 2, q = e & 3, sw = r0 & 7;
+      const int src0 = r0 * 64 + q * 16;
+      const int dlo = r0 * 128 + (((2 * q) ^ sw) << 4), dhi = r0 * 128 + (((2 * q + 1) ^ sw) << 4);
+      const int dcp = r0 * 128 + ((q ^ sw) << 4);
       bool ok = true;
       int s = 0;
       for (int ti = 0; ti < my_tiles && ok; ++ti) {
@@ -346,139 +397,122 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = mbar_wait_inline(&pfull[ps], (s / SP) & 1, wc);
           if (ok && s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
           if (!ok) break;
-          const uint8_t* p = pring + ps * PSTAGE;
-          uint8_t* xb = oring + os * OSTAGE + A_BYTES;
+          const uint8_t* src = pring + ps * PSTAGE + src0;
+          uint8_t* dst = oring + os * OSTAGE;
+          // Four loads, then four expansions and their stores: the stores may alias the loads as far
+          // as the compiler knows, so written in this order the loads are in flight together.
+          if (st < nks) {
+#pragma unroll 1
+            for (int i0 = 0; i0 < 16; i0 += 4) {
+              uint4 v[4];
 #pragma unroll
-          for (int h8 = 0; h8 < 16; h8 += 8) {
-            uint2 pkd[8];
+              for (int i = 0; i < 4; ++i) v[i] = *reinterpret_cast<const uint4*>(src + (i0 + i) * 1024);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) pkd[i] = *reinterpret_cast<const uint2*>(p + src0 + (h8 + i) * 512);
+              for (int i = 0; i < 4; ++i) {
+                const uint2 x = sm4_expand(v[i].x), y = sm4_expand(v[i].y), z = sm4_expand(v[i].z),
+                            w = sm4_expand(v[i].w);
+                *reinterpret_cast<uint4*>(dst + dlo + (i0 + i) * 2048) = make_uint4(x.x, x.y, y.x, y.y);
+                *reinterpret_cast<uint4*>(dst + dhi + (i0 + i) * 2048) = make_uint4(z.x, z.y, w.x, w.y);
+              }
+            }
+          } else {
+#pragma unroll 1
+            for (int i0 = 0; i0 < 16; i0 += 4) {
+              uint4 v[4];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              uint4 o;
-              o.x = (pkd[i].x ^ kX8) & 0x0F0F0F0Fu;
-              o.y = ((pkd[i].x >> 4) ^ kX8) & 0x0F0F0F0Fu;
-              o.z = (pkd[i].y ^ kX8) & 0x0F0F0F0Fu;
-              o.w = ((pkd[i].y >> 4) ^ kX8) & 0x0F0F0F0Fu;
-              *reinterpret_cast<uint4*>(xb + dst0 + (h8 + i) * 1024) = o;
+              for (int i = 0; i < 4; ++i) v[i] = *reinterpret_cast<const uint4*>(src + (i0 + i) * 1024);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) *reinterpret_cast<uint4*>(dst + dcp + (i0 + i) * 2048) = v[i];
             }
           }
-          // Orders the generic writes of the expanded weights before the MMA reads them, and the
+          // Orders the generic writes of the operand stage before the MMA reads them, and the
           // generic reads of the packed stage before TMA refills it.
           fence_proxy_async_smem();
           warp_arrive(&ofull[os]);
-          if (lane == 0) mbar_arrive(&pempty[ps]);
+          warp_arrive(&pempty[ps]);
         }
       }
     }
   } else {
     setmaxnreg_inc<kRegsEpi>();
     // ------------------------------------------------------------- epilogue
-    // Warp w reads TMEM lanes 32*(w%4).. (its quadrant of rows) and the 32 CBW output columns
-    // from 32 CBW ((w-4)/4).  Thread t holds rows rq + 8k (k = 0..3, rq = t/4 within the
-    // quadrant) and, in each 32-column block cb, columns 8j + 2 cq + {0, 1} (j = 0..3,
-    // cq = t % 4): acc[16 cb + 4k + j] is that pair.
-    const int quad = wid & 3;
-    const int col0 = 32 * CBW * ((static_cast<int>(wid) - 4) >> 2);
+    // Warp 4 + 4h + q reads TMEM lanes 32q.. (its quadrant of rows), columns 64h .. 64h + 63 of
+    // each unit.  With the 16x256b load shape, thread t holds rows rq + 8k (k = 0..3, rq = t / 4)
+    // and, in each 32-column block b, columns 8j + 2cq + {0, 1} (j = 0..3, cq = t % 4):
+    // acc[16b + 4k + j] is that pair.  Per group and output: t = D s_x, acc += t sigma.  Sigma is
+    // stored permuted within each 32-column block, so the thread's eight scales of a block are
+    // contiguous (two 16-byte loads).
+    const int quad = static_cast<int>(wid & 3), h = (static_cast<int>(wid) - 4) >> 2;
     const int rq = static_cast<int>(lane) >> 2, cq = static_cast<int>(lane) & 3;
-    const int rbase = quad * 32 + rq;
-    const uint32_t tq = tmem + (static_cast<uint32_t>(quad * 32) << 16) + col0;
+    EpiCtx c;
+    c.sring = sring;
+    c.ones = ones;
+    c.sfull = sfull;
+    c.sempty = sempty;
+    c.tfull = tfull;
+    c.tempty = tempty;
+    c.wc = wc;
+    c.tq = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(64 * h);
+    c.quad = quad;
+    c.h = h;
+    c.rq = rq;
+    c.cq = cq;
+    c.ngk = ngk;
+    c.ngt = ngt;
+    c.total = my_tiles * ngt;  // groups this CTA's epilogue walks (branch included)
     bool ok = true;
-    int u_all = 0, s = 0, ss = 0;  // accumulator-unit, K-stage and scale-stage counters
+    uint32_t v[2][4][16];  // TMEM loads of two groups: [buffer][block b * 2 + row half][16]
+    f2 acc[32];
+    if (c.total > 0) {
+      if (ok) ok = mbar_wait_inline(&sfull[0], 0, wc);
+      if (ok) ok = mbar_wait_inline(&tfull[0], 0, wc);
+      tc_fence_after();
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        tmem_ld16x256_x4(c.tq + 32 * b, v[0][2 * b]);
+        tmem_ld16x256_x4(c.tq + (16u << 16) + 32 * b, v[0][2 * b + 1]);
+      }
+    }
+    // Group g of the CTA lands in buffer g % 2.  A tile's groups run in pairs from a buffer parity
+    // fixed at compile time (one copy of the loop per parity, chosen by the tile's first group), so
+    // the accumulator is zeroed and stored outside the per-group code.  The branch group takes the
+    // same arithmetic with unit scales (D * 1 * 1 + acc = D + acc exactly).
+    int g = 0, sl = 0;
     for (int ti = 0; ti < my_tiles; ++ti) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) acc[i] = 0ull;
+      // (gi is advanced by epi_group and wraps to 0 after the tile's last group; the loops below
+      // count the tile's groups with their own index)
+      int gi = 0;
+      if ((g & 1) == 0) {
+        for (int j = 0; j + 2 <= ngt; j += 2) {
+          epi_group<0>(c, acc, v, g, gi, sl, ok);
+          epi_group<1>(c, acc, v, g, gi, sl, ok);
+        }
+        if (ngt & 1) epi_group<0>(c, acc, v, g, gi, sl, ok);
+      } else {
+        for (int j = 0; j + 2 <= ngt; j += 2) {
+          epi_group<1>(c, acc, v, g, gi, sl, ok);
+          epi_group<0>(c, acc, v, g, gi, sl, ok);
+        }
+        if (ngt & 1) epi_group<1>(c, acc, v, g, gi, sl, ok);
+      }
+      // the tile's output: Y (plus the bias)
       int m0, n0;
       tile_mn(ti, m0, n0);
-      f2 acc[16 * CBW];
-#pragma unroll
-      for (int i = 0; i < 16 * CBW; ++i) acc[i] = 0ull;
-      for (int st = 0; st < nst; ++st, ++s) {
-        const int gn = groups_in(st);
-        const int sb = ss % SS;
-        if (scale_starts(st) && ok) ok = mbar_wait_inline(&sfull[sb], (ss / SS) & 1, wc);
-        const int gl0 = (st * gps) % kScaleGroups;  // the stage's first group within the scale stage
-        const float2* pab = reinterpret_cast<const float2*>(sring + sb * SSTAGE) + gl0 * 128;
-        const float* psw = reinterpret_cast<const float*>(sring + sb * SSTAGE + SAB_BYTES) + gl0 * 128;
-        for (int g0 = 0; g0 < gn; g0 += 2, ++u_all) {
-          const int ub = u_all % NTB;
-          const int nmem = (g0 + 1 < gn) ? 2 : 1;
-          if (ok) ok = mbar_wait_inline(&tfull[ub], (u_all / NTB) & 1, wc);
-          tc_fence_after();
-          for (int mi = 0; mi < nmem; ++mi) {
-            const int gi = g0 + mi;
-            uint32_t v0[CBW][16], v1[CBW][16];
-#pragma unroll
-            for (int cb = 0; cb < CBW; ++cb) {
-              tmem_ld16x256_x4(tq + ub * 256 + mi * 128 + 32 * cb, v0[cb]);
-              tmem_ld16x256_x4(tq + (16u << 16) + ub * 256 + mi * 128 + 32 * cb, v1[cb]);
-            }
-            float2 abr[4];  // (alpha, beta) of rows rbase + 8k
-#pragma unroll
-            for (int k = 0; k < 4; ++k) abr[k] = pab[gi * 128 + rbase + 8 * k];
-            f2 sw2[4 * CBW];
-#pragma unroll
-            for (int j = 0; j < 4 * CBW; ++j)
-              sw2[j] = *reinterpret_cast<const f2*>(psw + gi * 128 + col0 + 8 * j + 2 * cq);
-            f2 d[CBW][16];  // d[cb][8h + 2j + rr] = columns (8j + 2cq, +1) of row rq + 16h + 8rr
-#pragma unroll
-            for (int cb = 0; cb < CBW; ++cb) tmem_ld_wait_pairs(v0[cb], v1[cb], d[cb]);
-            if (mi == nmem - 1) {
-              tc_fence_before();
-              warp_arrive(&tempty[ub]);  // every load of the unit has landed
-            }
-            // acc += (alpha D + beta) * s_w, alpha = 2^18 s_x, beta = -8 s_x S_a (from kernel (a))
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              const f2 al2 = dup2(abr[k].x), be2 = dup2(abr[k].y);
-#pragma unroll
-              for (int cb = 0; cb < CBW; ++cb)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                  const f2 t = fma2(d[cb][8 * (k >> 1) + 2 * j + (k & 1)], al2, be2);
-                  acc[16 * cb + 4 * k + j] = fma2(t, sw2[4 * cb + j], acc[16 * cb + 4 * k + j]);
-                }
-            }
-          }
-        }
-        if (scale_ends(st)) {
-          fence_proxy_async_smem();  // reads of the TMA-written scales before the slot is refilled
-          warp_arrive(&sempty[sb]);
-          ++ss;
-        }
-      }
-      if constexpr (RP > 0) {
-        const int ub = u_all % NTB;
-        if (ok) ok = mbar_wait_inline(&tfull[ub], (u_all / NTB) & 1, wc);
-        tc_fence_after();
-#pragma unroll
-        for (int cb = 0; cb < CBW; ++cb) {
-          uint32_t v0[16], v1[16];
-          tmem_ld16x256_x4(tq + ub * 256 + 32 * cb, v0);
-          tmem_ld16x256_x4(tq + (16u << 16) + ub * 256 + 32 * cb, v1);
-          f2 d[16];
-          tmem_ld_wait_pairs(v0, v1, d);
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              acc[16 * cb + 4 * k + j] = add2(acc[16 * cb + 4 * k + j], d[8 * (k >> 1) + 2 * j + (k & 1)]);
-        }
-        tc_fence_before();
-        warp_arrive(&tempty[ub]);
-        ++u_all;
-      }
       if (ok) {
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          const int m = m0 + rbase + 8 * k;
+          const int m = m0 + quad * 32 + rq + 8 * k;
           if (m >= a.M) continue;
 #pragma unroll
-          for (int cb = 0; cb < CBW; ++cb)
+          for (int b = 0; b < 2; ++b)
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-              const int n = n0 + col0 + 32 * cb + 8 * j + 2 * cq;  // even; N is a multiple of 8
+              const int n = n0 + 64 * h + 32 * b + 8 * j + 2 * cq;  // even; N is a multiple of 8
               if (n >= a.N) continue;
               const size_t off = static_cast<size_t>(m) * a.N + n;
-              const f2 y = acc[16 * cb + 4 * k + j];
+              const f2 y = acc[16 * b + 4 * k + j];
               float y0 = lo_f(y), y1 = hi_f(y);
               if (a.bias) {
                 const float2 bb = *reinterpret_cast<const float2*>(a.bias + n);
@@ -495,6 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    tmem_ld_wait();  // the loads issued after the last group land before TMEM is released
   }
 
   __syncthreads();
@@ -504,16 +539,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int RP>
-cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, cudaStream_t s) {
-  using Cfg = GemmCfg<RP>;
+template <int G>
+cudaError_t launch_g(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, cudaStream_t s) {
   GemmArgs a;
   a.M = M;
   a.N = h.N;
   a.K = h.K;
-  a.G = h.G;
+  a.nbs = (h.r_pad + 31) / 32;
   a.m_tiles = (M + kBM - 1) / kBM;
-  a.n_tiles = (h.N + kGemmBN - 1) / kGemmBN;
+  a.n_tiles = (h.N + kBN - 1) / kBN;
   a.Y = Y;
   a.y_f32 = y_f32 ? 1 : 0;
   a.bias = h.bias;
@@ -521,39 +555,33 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, 
   a.timeout_ns = deadline_budget_ns(h);
   static bool attr_done = false;
   if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
   const int ntiles = a.m_tiles * a.n_tiles;
   const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
-  const CUtensorMap& ph = (RP > 0) ? am.ph_map : am.qx_map;
-  const CUtensorMap& bh = (RP > 0) ? h.Bh_map : am.qx_map;
+  // Without a branch the p_hat / B_hat maps are never used; any valid map fills the slots.
+  const CUtensorMap& ph = (h.r_pad > 0) ? am.ph32_map : am.qa_map;
+  const CUtensorMap& bh = (h.r_pad > 0) ? h.bh32_map : am.qa_map;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.dynamicSmemBytes = SMEM;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, gemm_kernel<RP>, am.qx_map, h.qw_map, am.ab_map, h.sw32_map, ph, bh, a);
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<G>, am.qa_map, h.qw_map, am.sx_map, h.sw32_map, ph, bh, a);
 }
 
 }  // namespace
 
 cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s) {
   (void)ws;
-  switch (h.r_pad) {
-    case 0: return launch_rp<0>(h, am, M, Y, y_f32, s);
-    case 16: return launch_rp<16>(h, am, M, Y, y_f32, s);
-    case 32: return launch_rp<32>(h, am, M, Y, y_f32, s);
-    case 48: return launch_rp<48>(h, am, M, Y, y_f32, s);
-    case 64: return launch_rp<64>(h, am, M, Y, y_f32, s);
-    default: return cudaErrorInvalidValue;
-  }
+  return h.G == 32 ? launch_g<32>(h, am, M, Y, y_f32, s) : launch_g<64>(h, am, M, Y, y_f32, s);
 }
 
 }  // namespace qwam

@@ -16,8 +16,7 @@ constexpr int kBM = 128;        // token rows per CTA tile (one TMEM lane per ro
 constexpr int kChunk = 64;      // K columns per activation chunk (bf16: one 128-byte row)
 constexpr int kMaxRank = 64;    // largest protected rank of this build
 constexpr int kGemmBN = 128;    // output columns per GEMM CTA tile
-constexpr int kGemmKS = 128;    // K elements per GEMM pipeline stage
-constexpr int kScaleGroups = 8; // groups per GEMM scale stage (epilogue constants and s_w)
+constexpr int kScaleGroups = 8; // groups per INT4 GEMM scale slot (s_x and the weight scale)
 
 // NVFP4 variant (App. B.1): E2M1 codes, one E4M3 scale per 16 consecutive K, one float32 scale per
 // weight tensor.  Block scales are stored in 512-byte atoms, one per 128 rows x 64 K: the four
@@ -30,15 +29,33 @@ enum Format : int { kFmtInt4 = 0, kFmtNvfp4 = 1 };
 
 inline int round_up(int a, int b) { return (a + b - 1) / b * b; }
 
+// INT4 codes are stored packed at four bits in SM4 words (sign-magnitude): word j of a row holds
+// k = 8j .. 8j+7.  Byte i carries code 8j+i in its sign bit 7 and magnitude bits 0-2, the
+// magnitude of code 8j+4+i in bits 4-6, and in bit 3 the sign of code 8j+4+((i+3) mod 4).  From
+// lo and hi, the E4M3 bytes (sign | magnitude, the value c 2^-9) of codes 8j..8j+3 and
+// 8j+4..8j+7, the word is lo | rotl(hi, 4); back: lo = w & 0x87878787, hi = rotr(w, 4) & 0x87878787.
+__host__ __device__ inline uint32_t sm4_pack(uint32_t lo, uint32_t hi) { return lo | (hi << 4) | (hi >> 28); }
+// E4M3 byte (sign | magnitude) of an integer code in [-7, 7].
+__host__ __device__ inline uint32_t sm4_byte(int c) {
+  return static_cast<uint32_t>(c < 0 ? -c : c) | (c < 0 ? 0x80u : 0u);
+}
+// Position of weight-scale column n within its 32-column block in the GEMM's float32 copy: the
+// epilogue thread with q = (n % 8) / 2 reads columns 8j + 2q + {0, 1} (j = 0..3) as 8 floats.
+__host__ __device__ inline int sigma_pos(int n) {
+  const int t = n & 31;
+  return (n & ~31) + 8 * ((t & 7) >> 1) + 2 * (t >> 3) + (t & 1);
+}
+
 // Activation-side tensor maps for one (workspace, X, M) triple.
 struct ActMaps {
   const void* ws = nullptr;
   const void* x = nullptr;
   int M = -1;
   CUtensorMap x_map;    // X bf16 [M, K], box {64, 128}, 128-byte swizzle
-  CUtensorMap qx_map;   // code bytes [M, K], box {128, 128}, 128-byte swizzle
-  CUtensorMap ab_map;   // epilogue constants f32 [K/G, M_pad, 2] (dims {2M, K/G}), box {256, 8}
-  CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128}
+  CUtensorMap qa_map;   // INT4: packed SM4 codes [M, K/2] bytes, box {64, 128}
+  CUtensorMap sx_map;   // INT4: s_x f32 [K/G, M_pad], box {128, kScaleGroups}
+  CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128} (NVFP4 GEMM)
+  CUtensorMap ph32_map; // p_hat f16 [M, r_pad], box {32, 128} (INT4 GEMM)
   CUtensorMap qx4_map;  // NVFP4 codes [M, K/2] bytes, box {128, 128}, 128-byte swizzle
 };
 
@@ -48,17 +65,18 @@ struct Handle {
   int device = 0;
   int num_sms = 148;
   void* block = nullptr;             // one device allocation holding every buffer below
-  uint8_t* qw = nullptr;             // [N_pad, K/2]; word j of a row holds k = 8j..8j+3 in the low
-                                     // and 8j+4..8j+7 in the high nibbles of its bytes
+  uint8_t* qw = nullptr;             // INT4: [N_pad, K/2] SM4 words (word j of a row: k = 8j..8j+7,
+                                     // see sm4_pack); NVFP4: E2M1 codes, low nibble = even k
   __half* sw = nullptr;              // [K/G, N_pad]
-  float* sw32 = nullptr;             // [K/G, N_pad]: the same scales widened to float32 (GEMM epilogue)
+  float* sw32 = nullptr;             // [K/G, N_pad]: sigma = 2^18 s_w in float32 (GEMM epilogue), each
+                                     // 32-column block permuted: column 8j + 2q + b at 8q + 2j + b
   __half* Bh = nullptr;              // [N_pad, r_pad]
   __nv_bfloat16* ucat_t = nullptr;   // [2 r_pad, K]: rows 0..r_pad-1 = U_hi^T, then U_lo^T
   __nv_bfloat16* ucat3 = nullptr;    // [K, ku3]: row k = U_hi[k,:], U_lo[k,:], U_hi[k,:], zeros
   uint8_t* sfw = nullptr;            // NVFP4: E4M3 block scales of W_perp in atoms (N_pad rows)
   float sg = 0.0f;                   // NVFP4: float32 per-tensor weight scale
   int* err = nullptr;                // sticky device error word
-  // Smoothing and block Hadamard rotation in front of the layer (Sec. 2 Eq. (pair)): the packed
+  // Smoothing and block Hadamard rotation in front of the layer (Sec. 3 Eq. (pair)): the packed
   // weight is W~ = H diag(s) W, the activations are rotated at run time, x~ = H diag(s)^-1 x.
   // ucat_t then holds diag(s)^-1 H U (the projection x~ U = x (diag(s)^-1 H U)) and ucat3 holds
   // diag(s) H U (the remainder x - diag(s) H U p, which H diag(s)^-1 maps to x~ - U p).
@@ -70,12 +88,18 @@ struct Handle {
   float* ur32 = nullptr;             // [r_pad, K] float32 reconstruction basis (U, or diag(s) H U), transposed
   int small_m = 256;                 // token counts up to this take the small-M activation kernel
   double timeout_s = 2.0;
-  CUtensorMap qw_map, sw32_map, Bh_map, ucat_t_map, ucat3_map;
+  CUtensorMap qw_map;                // INT4 weight codes [N, K/2] bytes, box {64, 128}
+  CUtensorMap sw32_map;              // sigma [K/G, N], box {128, kScaleGroups}
+  CUtensorMap Bh_map;                // B_hat [N, r_pad] f16, box {8, 128} (NVFP4 GEMM)
+  CUtensorMap bh32_map;              // B_hat [N, r_pad] f16, box {32, 128} (INT4 GEMM)
+  CUtensorMap ucat_t_map, ucat3_map;
   CUtensorMap qw4_map;               // NVFP4 weight codes [N, K/2], box {128, 128}, 128-byte swizzle
   ActMaps act_cache[4];
   int act_next = 0;
 };
 
+// Workspace of M tokens.  INT4: packed SM4 codes [M, K/2], s_x f32 [K/G, M_pad], p_hat f16
+// [M, r_pad]; NVFP4: E2M1 codes [M, K/2], scale atoms, p_hat.  ab_off = phat_off (no region).
 struct ActLayout {
   size_t codes_off, scales_off, ab_off, phat_off, bytes;
   size_t resid_off;  // rotated handles with r > 0: float32 [M, K] remainder before the rotation
@@ -101,7 +125,7 @@ cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, voi
 cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
 cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s);
 cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
-                                        uint8_t* scales, float2* ab, int M_pad, cudaStream_t s);
+                                        uint8_t* scales, int M_pad, cudaStream_t s);
 cudaError_t launch_debug_quantize_rows(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
                                        void* scales, cudaStream_t s);
 // The offline choice of what to protect (subspace.cu).

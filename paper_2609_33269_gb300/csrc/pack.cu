@@ -1,5 +1,5 @@
-// pack.cu -- offline packing of one ASP layer (Sec. 3.2 Eq. (asp) and the derivation of the
-// deflated weight W_perp = (I - U U^T) W; Eq. (quant) of Sec. 2 applied to W_perp per output
+// pack.cu -- offline packing of one ASP layer (Sec. 4.2 Eq. (asp) and the derivation of the
+// deflated weight W_perp = (I - U U^T) W; Eq. (quant) of Sec. 3 applied to W_perp per output
 // channel and group, App. B.1; or, for the NVFP4 variant of App. B.1, E2M1 codes with an E4M3
 // scale per 16 K and one float32 scale per tensor).  float64 on the device, untimed.
 //
@@ -61,8 +61,8 @@ __device__ __forceinline__ int nearest_code_f64(double w, double s) {
 }
 
 // One thread per (output channel n, group g): s_w = RN_f16(absmax / 7), codes packed 4 bits
-// each into qw[n, :]: 32-bit word j holds k = 8j..8j+3 in the low nibbles and k = 8j+4..8j+7 in
-// the high nibbles of its four bytes (the GEMM expands a word to bytes with three logic ops).
+// each into qw[n, :] as SM4 words (sm4_pack: word j holds k = 8j..8j+7, sign-magnitude, so that
+// the GEMM expands a word to its eight E4M3 bytes with one funnel shift and two masks).
 template <typename WT>
 __global__ void quantize_weight_kernel(const WT* __restrict__ W, const float* __restrict__ U,
                                        const double* __restrict__ Bf, int K, int N, int r, int G, int N_pad,
@@ -76,21 +76,23 @@ __global__ void quantize_weight_kernel(const WT* __restrict__ W, const float* __
   __half sh = __double2half(__ddiv_rn(amax, 7.0));
   double s = static_cast<double>(__half2float(sh));
   sw[static_cast<size_t>(g) * N_pad + n] = sh;
-  sw32[static_cast<size_t>(g) * N_pad + n] = static_cast<float>(s);
+  // sigma = 2^18 s_w (exact), at the permuted position the GEMM epilogue reads
+  sw32[static_cast<size_t>(g) * N_pad + sigma_pos(n)] = static_cast<float>(s) * 262144.0f;
   bool ok_scale = isfinite(s);
   if (!ok_scale) atomicOr(err, kErrRange);
   uint32_t* row = reinterpret_cast<uint32_t*>(qw + static_cast<size_t>(n) * (K / 2));
   for (int k = g * G; k < (g + 1) * G; k += 8) {
-    uint32_t word = 0;
+    uint32_t lo = 0, hi = 0;
     for (int i = 0; i < 8; ++i) {
       int c = 0;
       if (s > 0.0 && ok_scale) c = nearest_code_f64(wperp(W, U, Bf, N, r, k + i, n), s);
       if (c < -7 || c > 7) atomicOr(err, kErrRange);
-      // k + i (i < 4) -> low nibble of byte i; k + 4 + i -> high nibble of byte i
-      const int shift = (i < 4) ? 8 * i : 8 * (i - 4) + 4;
-      word |= (static_cast<uint32_t>(c) & 0xFu) << shift;
+      if (i < 4)
+        lo |= sm4_byte(c) << (8 * i);
+      else
+        hi |= sm4_byte(c) << (8 * (i - 4));
     }
-    row[k / 8] = word;
+    row[k / 8] = sm4_pack(lo, hi);
   }
 }
 
@@ -211,7 +213,7 @@ __global__ void quantize_weight_nvfp4_kernel(const WT* __restrict__ W, const flo
   *reinterpret_cast<uint2*>(qw + static_cast<size_t>(n) * (K / 2) + b * (kFp4Block / 2)) = make_uint2(lo, hi);
 }
 
-// ---- smoothing and block Hadamard rotation (Sec. 2 Eq. (pair); App. B.1), float64
+// ---- smoothing and block Hadamard rotation (Sec. 3 Eq. (pair); App. B.1), float64
 
 // Columns n0 .. n0+15 of rows [kb, kb + B) of A [K, N] (bf16 or float32), each times scale[k]
 // when scale is given, through the block Walsh-Hadamard butterflies (a + b, a - b) at spans

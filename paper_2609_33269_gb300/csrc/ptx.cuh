@@ -67,6 +67,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test of a phase (never suspends): issued early, its result is consumed later, so
+// that its latency overlaps independent work.
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\n"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      "selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // Every wait in the kernels is bounded.  A kernel gives up when its deadline passes or when
 // another warp of the CTA has already given up (shared abort flag); it then records
 // kErrTimeout in the sticky error word and unwinds.
@@ -76,16 +90,29 @@ struct WaitCtl {
   uint64_t deadline_ns;      // %globaltimer value after which waits give up
 };
 
+// try_wait with a suspend-time hint: a thread whose phase is not complete sleeps until it
+// completes or `ns` nanoseconds pass, instead of polling and taking issue slots from the warps
+// that do the work.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\n"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+      "selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(ns)
+      : "memory");
+  return ok != 0;
+}
+
 __device__ __forceinline__ bool wait_loop(uint64_t* bar, uint32_t parity, const WaitCtl& c) {
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 127) == 0) {
-      if (*c.abort_flag) return false;
-      if (globaltimer_ns() > c.deadline_ns) {
-        *c.abort_flag = 1;
-        atomicOr(c.err, kErrTimeout);
-        return false;
-      }
+  for (;;) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (*c.abort_flag) return false;
+    if (globaltimer_ns() > c.deadline_ns) {
+      *c.abort_flag = 1;
+      atomicOr(c.err, kErrTimeout);
+      return false;
     }
   }
 }
@@ -355,6 +382,72 @@ __device__ __forceinline__ void tmem_ld_wait_pairs(const uint32_t (&a)[16], cons
       "mov.b64 %15, {%46, %47};\n"
       : "=l"(p[0]), "=l"(p[1]), "=l"(p[2]), "=l"(p[3]), "=l"(p[4]), "=l"(p[5]), "=l"(p[6]), "=l"(p[7]), "=l"(p[8]), "=l"(p[9]), "=l"(p[10]), "=l"(p[11]), "=l"(p[12]), "=l"(p[13]), "=l"(p[14]), "=l"(p[15])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(a[4]), "r"(a[5]), "r"(a[6]), "r"(a[7]), "r"(a[8]), "r"(a[9]), "r"(a[10]), "r"(a[11]), "r"(a[12]), "r"(a[13]), "r"(a[14]), "r"(a[15]), "r"(b[0]), "r"(b[1]), "r"(b[2]), "r"(b[3]), "r"(b[4]), "r"(b[5]), "r"(b[6]), "r"(b[7]), "r"(b[8]), "r"(b[9]), "r"(b[10]), "r"(b[11]), "r"(b[12]), "r"(b[13]), "r"(b[14]), "r"(b[15])
+      : "memory");
+}
+// Wait for outstanding tcgen05.ld and hand one 16-register result on as 8 packed pairs
+// p[i] = {r[2i], r[2i + 1]}.
+__device__ __forceinline__ void tmem_ld_wait_pairs8(const uint32_t (&a)[16], unsigned long long (&p)[8]) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;\n"
+      "mov.b64 %0, {%8, %9};\n"
+      "mov.b64 %1, {%10, %11};\n"
+      "mov.b64 %2, {%12, %13};\n"
+      "mov.b64 %3, {%14, %15};\n"
+      "mov.b64 %4, {%16, %17};\n"
+      "mov.b64 %5, {%18, %19};\n"
+      "mov.b64 %6, {%20, %21};\n"
+      "mov.b64 %7, {%22, %23};\n"
+      : "=l"(p[0]), "=l"(p[1]), "=l"(p[2]), "=l"(p[3]), "=l"(p[4]), "=l"(p[5]), "=l"(p[6]), "=l"(p[7])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(a[4]), "r"(a[5]), "r"(a[6]), "r"(a[7]), "r"(a[8]),
+        "r"(a[9]), "r"(a[10]), "r"(a[11]), "r"(a[12]), "r"(a[13]), "r"(a[14]), "r"(a[15])
+      : "memory");
+}
+// Wait for outstanding tcgen05.ld and hand four 16-register results on as packed pairs
+// p[i][j] = {r[i][2j], r[i][2j + 1]}.
+__device__ __forceinline__ void tmem_ld_wait_pairs8x4(const uint32_t (&a)[4][16], unsigned long long (&p)[4][8]) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;\n"
+      "mov.b64 %0, {%32, %33};\n mov.b64 %1, {%34, %35};\n mov.b64 %2, {%36, %37};\n mov.b64 %3, {%38, %39};\n"
+      "mov.b64 %4, {%40, %41};\n mov.b64 %5, {%42, %43};\n mov.b64 %6, {%44, %45};\n mov.b64 %7, {%46, %47};\n"
+      "mov.b64 %8, {%48, %49};\n mov.b64 %9, {%50, %51};\n mov.b64 %10, {%52, %53};\n mov.b64 %11, {%54, %55};\n"
+      "mov.b64 %12, {%56, %57};\n mov.b64 %13, {%58, %59};\n mov.b64 %14, {%60, %61};\n mov.b64 %15, {%62, %63};\n"
+      "mov.b64 %16, {%64, %65};\n mov.b64 %17, {%66, %67};\n mov.b64 %18, {%68, %69};\n mov.b64 %19, {%70, %71};\n"
+      "mov.b64 %20, {%72, %73};\n mov.b64 %21, {%74, %75};\n mov.b64 %22, {%76, %77};\n mov.b64 %23, {%78, %79};\n"
+      "mov.b64 %24, {%80, %81};\n mov.b64 %25, {%82, %83};\n mov.b64 %26, {%84, %85};\n mov.b64 %27, {%86, %87};\n"
+      "mov.b64 %28, {%88, %89};\n mov.b64 %29, {%90, %91};\n mov.b64 %30, {%92, %93};\n mov.b64 %31, {%94, %95};\n"
+      : "=l"(p[0][0]), "=l"(p[0][1]), "=l"(p[0][2]), "=l"(p[0][3]), "=l"(p[0][4]), "=l"(p[0][5]), "=l"(p[0][6]),
+        "=l"(p[0][7]), "=l"(p[1][0]), "=l"(p[1][1]), "=l"(p[1][2]), "=l"(p[1][3]), "=l"(p[1][4]), "=l"(p[1][5]),
+        "=l"(p[1][6]), "=l"(p[1][7]), "=l"(p[2][0]), "=l"(p[2][1]), "=l"(p[2][2]), "=l"(p[2][3]), "=l"(p[2][4]),
+        "=l"(p[2][5]), "=l"(p[2][6]), "=l"(p[2][7]), "=l"(p[3][0]), "=l"(p[3][1]), "=l"(p[3][2]), "=l"(p[3][3]),
+        "=l"(p[3][4]), "=l"(p[3][5]), "=l"(p[3][6]), "=l"(p[3][7])
+      : "r"(a[0][0]), "r"(a[0][1]), "r"(a[0][2]), "r"(a[0][3]), "r"(a[0][4]), "r"(a[0][5]), "r"(a[0][6]),
+        "r"(a[0][7]), "r"(a[0][8]), "r"(a[0][9]), "r"(a[0][10]), "r"(a[0][11]), "r"(a[0][12]), "r"(a[0][13]),
+        "r"(a[0][14]), "r"(a[0][15]), "r"(a[1][0]), "r"(a[1][1]), "r"(a[1][2]), "r"(a[1][3]), "r"(a[1][4]),
+        "r"(a[1][5]), "r"(a[1][6]), "r"(a[1][7]), "r"(a[1][8]), "r"(a[1][9]), "r"(a[1][10]), "r"(a[1][11]),
+        "r"(a[1][12]), "r"(a[1][13]), "r"(a[1][14]), "r"(a[1][15]), "r"(a[2][0]), "r"(a[2][1]), "r"(a[2][2]),
+        "r"(a[2][3]), "r"(a[2][4]), "r"(a[2][5]), "r"(a[2][6]), "r"(a[2][7]), "r"(a[2][8]), "r"(a[2][9]),
+        "r"(a[2][10]), "r"(a[2][11]), "r"(a[2][12]), "r"(a[2][13]), "r"(a[2][14]), "r"(a[2][15]), "r"(a[3][0]),
+        "r"(a[3][1]), "r"(a[3][2]), "r"(a[3][3]), "r"(a[3][4]), "r"(a[3][5]), "r"(a[3][6]), "r"(a[3][7]),
+        "r"(a[3][8]), "r"(a[3][9]), "r"(a[3][10]), "r"(a[3][11]), "r"(a[3][12]), "r"(a[3][13]), "r"(a[3][14]),
+        "r"(a[3][15])
+      : "memory");
+}
+// Wait for outstanding tcgen05.ld, naming four 16-register results as its operands (see
+// tmem_ld_wait_dep: no use of those registers moves above the wait).
+__device__ __forceinline__ void tmem_ld_wait_dep4(uint32_t (&a)[4][16]) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;"
+      : "+r"(a[0][0]), "+r"(a[0][1]), "+r"(a[0][2]), "+r"(a[0][3]), "+r"(a[0][4]), "+r"(a[0][5]), "+r"(a[0][6]),
+        "+r"(a[0][7]), "+r"(a[0][8]), "+r"(a[0][9]), "+r"(a[0][10]), "+r"(a[0][11]), "+r"(a[0][12]), "+r"(a[0][13]),
+        "+r"(a[0][14]), "+r"(a[0][15]), "+r"(a[1][0]), "+r"(a[1][1]), "+r"(a[1][2]), "+r"(a[1][3]), "+r"(a[1][4]),
+        "+r"(a[1][5]), "+r"(a[1][6]), "+r"(a[1][7]), "+r"(a[1][8]), "+r"(a[1][9]), "+r"(a[1][10]), "+r"(a[1][11]),
+        "+r"(a[1][12]), "+r"(a[1][13]), "+r"(a[1][14]), "+r"(a[1][15]), "+r"(a[2][0]), "+r"(a[2][1]), "+r"(a[2][2]),
+        "+r"(a[2][3]), "+r"(a[2][4]), "+r"(a[2][5]), "+r"(a[2][6]), "+r"(a[2][7]), "+r"(a[2][8]), "+r"(a[2][9]),
+        "+r"(a[2][10]), "+r"(a[2][11]), "+r"(a[2][12]), "+r"(a[2][13]), "+r"(a[2][14]), "+r"(a[2][15]), "+r"(a[3][0]),
+        "+r"(a[3][1]), "+r"(a[3][2]), "+r"(a[3][3]), "+r"(a[3][4]), "+r"(a[3][5]), "+r"(a[3][6]), "+r"(a[3][7]),
+        "+r"(a[3][8]), "+r"(a[3][9]), "+r"(a[3][10]), "+r"(a[3][11]), "+r"(a[3][12]), "+r"(a[3][13]), "+r"(a[3][14]),
+        "+r"(a[3][15])
+      :
       : "memory");
 }
 // {x, x} as a packed pair.

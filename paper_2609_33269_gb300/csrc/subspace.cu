@@ -1,9 +1,9 @@
-// subspace.cu -- the offline choice of what ASP protects (Q-WAM Sec. 3.2-3.3; App. A; App. B.1).
+// subspace.cu -- the offline choice of what ASP protects (Q-WAM Sec. 4.2-4.3; App. A; App. B.1).
 //
 //   smoothing factors   s_j = max|X_j|^alpha / max|W_j,:|^(1 - alpha)          (App. B.1)
-//   rotated AOG         G~  = H diag(gamma) G diag(gamma) H                      (Sec. 3.2)
-//   action subspace     V   = the eigenvectors of the r largest eigenvalues of G~ (Sec. 3.2; App. A)
-//   action mass         mu_E = sum of tr G~ over an expert's layers               (Sec. 3.3, Eq. (mass))
+//   rotated AOG         G~  = H diag(gamma) G diag(gamma) H                      (Sec. 4.2)
+//   action subspace     V   = the eigenvectors of the r largest eigenvalues of G~ (Sec. 4.2; App. A)
+//   action mass         mu_E = sum of tr G~ over an expert's layers               (Sec. 4.3, Eq. (mass))
 //
 // H is block diagonal with normalised Sylvester Hadamard blocks of size B, the largest power of
 // two dividing d (at most 1024).  G~ is formed with two passes of a block fast Walsh-Hadamard

@@ -3,7 +3,7 @@ benchmark.
 
 This module draws inputs only; it holds none of the layer's arithmetic.  The paper measures on
 trained World Action Models over RoboTwin 2.0, which are not available here; these generators
-stand in for its DiT / action-expert linear layers (shapes of Sec. 4 and App. B.1: rank r = 32,
+stand in for its DiT / action-expert linear layers (shapes of Sec. 5 and App. B.1: rank r = 32,
 group-wise 4-bit quantization).  Every array comes from NumPy's PCG64 seeded with
 ``[seed, layer_id, step]`` so that both sides of a comparison see the same bytes.
 

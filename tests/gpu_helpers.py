@@ -14,12 +14,21 @@ def to_dev_bf16(bits: np.ndarray) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).cuda().view(torch.bfloat16)
 
 
-def decode_code_bytes(b: np.ndarray) -> np.ndarray:
-    """Activation code bytes (E4M3 of c * 2^-9: sign bit | magnitude) -> int8 codes."""
-    b = np.ascontiguousarray(b, np.uint8)
-    assert not (b & 0x78).any(), "activation code byte outside the E4M3 subnormal code range"
+def decode_sm4(packed: np.ndarray) -> np.ndarray:
+    """INT4 codes packed as SM4 words, uint8 [R, K/2] -> int8 [R, K].
+
+    Word j of a row (little-endian 32 bits) holds k = 8j..8j+7: the E4M3 bytes (sign bit 7 |
+    magnitude bits 0-2) of k = 8j..8j+3 are word & 0x87878787 and those of k = 8j+4..8j+7 are
+    rotr(word, 4) & 0x87878787."""
+    p = np.ascontiguousarray(packed, np.uint8)
+    w = p.view("<u4").astype(np.uint64)
+    lo = (w & 0x87878787).astype(np.uint32)
+    hi = (((w >> 4) | (w << 28)) & 0x87878787).astype(np.uint32)
+    b = np.empty((p.shape[0], w.shape[1], 8), np.uint8)
+    b[:, :, :4] = lo[:, :, None].view(np.uint8).reshape(p.shape[0], -1, 4)
+    b[:, :, 4:] = hi[:, :, None].view(np.uint8).reshape(p.shape[0], -1, 4)
     mag = (b & 0x7).astype(np.int8)
-    return np.where(b & 0x80, -mag, mag).astype(np.int8)
+    return np.where(b & 0x80, -mag, mag).astype(np.int8).reshape(p.shape[0], -1)
 
 
 def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
@@ -79,19 +88,11 @@ class Case:
         return dict(qw=unpack_nibbles(e["qw"]), sw=e["sw"], Bh=e["Bh"][:, :self.r].T.copy(), Uhl=e["Uhl"])
 
     def gpu_act(self, rows=None):
-        codes, scales, ab, ph = self.layer.act_views(self.M)
+        codes, scales, ph = self.layer.act_views(self.M)
         torch.cuda.synchronize()
-        qx = decode_code_bytes(codes.cpu().numpy())
+        qx = decode_sm4(codes.cpu().numpy())
         sx = scales.cpu().numpy()[:, :self.M].T.copy()
-        abv = ab.cpu().numpy()[:, :self.M, :].transpose(1, 0, 2).copy()  # [M, K/G, 2]
         phv = ph.cpu().numpy().view(np.uint16)[:, :self.r].copy()
-        # the epilogue constants are (2^18 s_x, -8 s_x S_a) with S_a the exact sum of the group's
-        # codes, each rounded once in float32
-        sa = qx.reshape(self.M, -1, self.G).sum(axis=2).astype(np.float32)
-        alpha = (sx * np.float32(262144.0)).astype(np.float32)
-        beta = ((np.float32(-8.0) * sx).astype(np.float32) * sa).astype(np.float32)
-        for i, want in enumerate((alpha, beta)):
-            np.testing.assert_array_equal(abv[:, :, i].view(np.uint32), want.view(np.uint32))
         if rows is not None:
             qx, sx, phv = qx[rows], sx[rows], phv[rows]
         return dict(qx=qx, sx=sx, ph=phv)

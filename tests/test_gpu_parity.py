@@ -5,7 +5,7 @@ Bars (stated once here, used below):
     U, and every activation code and scale when r = 0 -- bit-exact;
   * with r > 0, the quantizer applied to the kernel's own float32 remainder is bit-exact; end to
     end against the float64 oracle, codes may differ only at near-ties of the float64 remainder
-    (Sec. 3.2 remainder formed in float32 on the GPU), at a rate below 1e-4;
+    (Sec. 4.2 remainder formed in float32 on the GPU), at a rate below 1e-4;
   * the layer output (float32 variant) within max |dY| <= 1e-3 * max |y| per row of the oracle;
     given the kernel's own codes and scales, within 1e-5 (float32 accumulation order only);
   * the bf16 output equals RN_bf16 of the float32 output bit for bit.

@@ -1,4 +1,4 @@
-"""GPU parity of the layer with smoothing and the block Hadamard rotation in front (Sec. 2
+"""GPU parity of the layer with smoothing and the block Hadamard rotation in front (Sec. 3
 Eq. (pair); App. B.1), through the C ABI, against the float64 oracle.
 
 Bars:

@@ -25,6 +25,8 @@ import torch
 import oracle
 from paper_2609_33269_gb300 import asp
 
+from gpu_helpers import decode_sm4
+
 pytestmark = pytest.mark.gpu
 
 E2M1_MIDPOINTS = (0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0)
@@ -155,21 +157,11 @@ def run_lanes(R, fmt, G):
         b = np.arange(K // 16)[None, :]
         sf = a[((r // 128) * (K // 64) + b // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + b % 4]
         return codes.cpu().numpy(), sf
-    codes = torch.zeros((M, K), dtype=torch.uint8, device="cuda")
+    codes = torch.zeros((M, K // 2), dtype=torch.uint8, device="cuda")
     scales = torch.zeros((K // G, M_pad), dtype=torch.float32, device="cuda")
-    ab = torch.zeros((K // G, M_pad, 2), dtype=torch.float32, device="cuda")
-    asp.qwam_asp_debug_quantize_lanes(Rd, M, K, fmt, G, codes, scales, ab)
+    asp.qwam_asp_debug_quantize_lanes(Rd, M, K, fmt, G, codes, scales)
     torch.cuda.synchronize()
-    c = codes.cpu().numpy()
-    sx = scales.cpu().numpy()[:, :M].T.copy()
-    # the epilogue constants: (2^18 s_x, -8 s_x S_a), S_a the group's code sum, each rounded once
-    q = (c & 0x7F).astype(np.int32) * np.where(c & 0x80, -1, 1)
-    sa = q.reshape(M, -1, G).sum(axis=2).astype(np.float32)
-    abv = ab.cpu().numpy()[:, :M, :].transpose(1, 0, 2)
-    np.testing.assert_array_equal(abv[:, :, 0].view(np.uint32), (sx * np.float32(262144.0)).view(np.uint32))
-    np.testing.assert_array_equal(abv[:, :, 1].view(np.uint32),
-                                  ((np.float32(-8.0) * sx).astype(np.float32) * sa).astype(np.float32).view(np.uint32))
-    return c, sx
+    return decode_sm4(codes.cpu().numpy()), scales.cpu().numpy()[:, :M].T.copy()
 
 
 IMPLS = {"thread_rows": None, "warp_lanes": run_lanes}
@@ -184,11 +176,12 @@ def run(R, fmt, G, impl="thread_rows"):
         codes = torch.zeros((M, K // 2), dtype=torch.uint8, device="cuda")
         scales = torch.zeros((M, K // 16), dtype=torch.uint8, device="cuda")
     else:
-        codes = torch.zeros((M, K), dtype=torch.uint8, device="cuda")
+        codes = torch.zeros((M, K // 2), dtype=torch.uint8, device="cuda")
         scales = torch.zeros((M, K // G), dtype=torch.float32, device="cuda")
     asp.qwam_asp_debug_quantize_rows(Rd, M, K, fmt, G, codes, scales)
     torch.cuda.synchronize()
-    return codes.cpu().numpy(), scales.cpu().numpy()
+    c = codes.cpu().numpy()
+    return (c if fmt == asp.QWAM_FMT_NVFP4 else decode_sm4(c)), scales.cpu().numpy()
 
 
 @pytest.mark.parametrize("impl", list(IMPLS))
@@ -196,8 +189,8 @@ def run(R, fmt, G, impl="thread_rows"):
 def test_int4_rounding_on_and_next_to_ties(G, impl):
     rng = np.random.default_rng(100 + G)
     R = as_rows(int4_groups(G, rng), G, 256)
-    b, s = run(R, asp.QWAM_FMT_INT4, G, impl)
-    q = (b & 0x7F).astype(np.int16) * np.where(b & 0x80, -1, 1)
+    q, s = run(R, asp.QWAM_FMT_INT4, G, impl)
+    q = q.astype(np.int16)
     oq, os_ = oracle.quantize_residual(R, G)
     np.testing.assert_array_equal(s.view(np.uint32), os_.view(np.uint32))
     np.testing.assert_array_equal(q, oq.astype(np.int16))

@@ -1,4 +1,4 @@
-"""GPU parity of the offline choice of what ASP protects (Sec. 3.2-3.3; App. A; App. B.1) against
+"""GPU parity of the offline choice of what ASP protects (Sec. 4.2-4.3; App. A; App. B.1) against
 the float64 oracle (oracle/subspace.py), through the C ABI: smoothing factors, the rotated AOG
 G~ = H diag(gamma) G diag(gamma) H, its trace, and its top-r eigenvectors; and a layer packed with
 the subspace the GPU chose.

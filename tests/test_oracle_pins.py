@@ -5,7 +5,7 @@ Each pin is independent of the oracle's own code:
   * brute-force argmin over the code grid for the quantizer (Eq. (quant)),
   * hand-derived closed-form group cases (tests/golden/quant_cases.txt),
   * library conversions (numpy float16) for the 16-bit format,
-  * invariants of Sec. 3.2: x = U(U^T x) + x_perp, U^T W_perp = 0, x_perp U = 0, Eq. (asp) with
+  * invariants of Sec. 4.2: x = U(U^T x) + x_perp, U^T W_perp = 0, x_perp U = 0, Eq. (asp) with
     Q = identity equals X W, r = 0 is plain per-group W4A4, r = K leaves a zero remainder,
   * storage of Table 3 (4.50 bits per weight at group 32) and the isotropy share r/K of App. C.
 """
@@ -226,7 +226,7 @@ def test_layer_matches_exact_rational_arithmetic(r, G):
     np.testing.assert_allclose(Y, Yex, rtol=1e-12, atol=1e-12 * np.abs(Yex).max())
 
 
-# ---------------------------------------------------------------- invariants of Sec. 3.2
+# ---------------------------------------------------------------- invariants of Sec. 4.2
 
 def _small_case(M=16, K=256, N=96, r=8, G=64, seed=1):
     Xb = wl.activations(M, K, seed=seed, layer_id=7, dist="outlier", n_outlier=4)
@@ -425,7 +425,7 @@ def test_rotation_with_full_rank_protection_is_the_plain_product():
 
 
 def test_rotation_spreads_an_outlier_channel():
-    """Sec. 2: the rotation spreads one large channel over its Hadamard block: every rotated entry
+    """Sec. 3: the rotation spreads one large channel over its Hadamard block: every rotated entry
     is at most ||x||_1 / sqrt(B) (each is a +-1/sqrt(B) combination of the block), and the norm is
     kept (H is orthogonal)."""
     K = 256

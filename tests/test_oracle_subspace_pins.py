@@ -1,4 +1,4 @@
-"""Pins of the oracle's offline subspace choice (oracle/subspace.py: Sec. 3.2-3.3, App. A, App. B.1)
+"""Pins of the oracle's offline subspace choice (oracle/subspace.py: Sec. 4.2-4.3, App. A, App. B.1)
 against definitions written out here: the Hadamard matrix from its bit formula and from the
 butterfly recursion, known spectra, the Ky Fan maximum principle checked against random frames,
 the trace and cost identities of the rotation, the smoothing factor's closed forms, and a

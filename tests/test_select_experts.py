@@ -1,4 +1,4 @@
-"""The expert choice of Sec. 3.3 (qwam_asp_select_experts, host-only, no GPU needed) against the
+"""The expert choice of Sec. 4.3 (qwam_asp_select_experts, host-only, no GPU needed) against the
 oracle: decreasing action mass per added 16-bit value while the additions fit the budget."""
 import numpy as np
 import pytest

@@ -49,7 +49,7 @@ def test_static_workspace_rejects_oversize_before_launch():
     W = _dev_bf16(wl.weight(K, N, seed=4, layer_id=0))
     layer = asp.AspLinear(W, None, 64)
     try:
-        M = asp.STATIC_WS_BYTES // K + 1  # the codes alone exceed the scratch
+        M = asp.STATIC_WS_BYTES // (K // 2) + 1  # the packed codes alone exceed the scratch
         assert asp.qwam_asp_act_workspace_bytes(layer.h, M) > asp.STATIC_WS_BYTES
         X = torch.zeros((M, K), dtype=torch.bfloat16, device="cuda")
         Y = torch.zeros((M, N), dtype=torch.float32, device="cuda")
