@@ -27,7 +27,7 @@
  *     returns QWAM_ERR_INVALID_ARG and launches nothing.  A failed CUDA call returns
  *     QWAM_ERR_CUDA.  Run-time entry points are asynchronous and allocate no device memory.
  *   - Device-side waits are bounded.  A wait that runs out records QWAM_ERR_TIMEOUT in the
- *     handle's sticky error word (read with qwam_asp_get_error) and the kernel returns.
+ *     handle's error word (read and cleared by qwam_asp_get_error) and the kernel returns.
  *   - Inputs must be finite.  A handle may be used from one host thread at a time.
  */
 #ifndef QWAM_ASP_H
@@ -127,8 +127,11 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
  * allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
  *
  *   - Size limit: the workspace qwam_asp_act_workspace_bytes(h, M) reports must fit in
- *     QWAM_STATIC_WS_BYTES (24 MiB: e.g. M = 4096 tokens at K = 3072, group 32 or 64, r <= 64).
- *     Larger requests return QWAM_ERR_TOO_LARGE before anything is launched.
+ *     QWAM_STATIC_WS_BYTES (24 MiB); larger requests return QWAM_ERR_TOO_LARGE before anything
+ *     is launched.  Per token the workspace holds about K/2 + 4K/G + 2 r_pad bytes (INT4) or
+ *     K/2 + K/16 + 2 r_pad bytes (NVFP4): at K = 3072, group 64, r = 32 about 1.8 KB, so up to
+ *     about 14,000 tokens fit.  A rotated handle with r > 0 also keeps its float32 remainder,
+ *     4K more bytes per token: at K = 3072 about 1,780 tokens fit, and M = 4096 is refused.
  *   - Nothing in the scratch needs to start at zero: kernel (a) writes every byte the GEMM
  *     then reads, on every call, so the scratch is never cleared.
  *   - One scratch per device: calls that may overlap in time on one device (different streams
@@ -136,7 +139,10 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
  *     results.  Order such calls, e.g. issue them on one stream.
  *   - The first call on each device looks the scratch's device address up (cudaGetSymbolAddress,
  *     with that device current) and keeps it; later calls reuse it.  Make that first call
- *     before any stream capture begins on the stream you pass.
+ *     before any stream capture begins on the stream you pass.  The kept address belongs to
+ *     the device context of that first call: after cudaDeviceReset (or any other reset of the
+ *     device's primary context) the library's device code is loaded anew and the kept address
+ *     is stale, so a process that resets a device must not call this function again on it.
  * Other arguments and errors are those of qwam_asp_linear; the handle's device must be current. */
 #define QWAM_STATIC_WS_BYTES (24u * 1024u * 1024u)
 qwam_status qwam_asp_linear_static(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
@@ -222,8 +228,14 @@ qwam_status qwam_asp_format(qwam_asp_handle h, int* format);
  * Returns QWAM_ERR_INVALID_ARG for an INT4 handle (and qwam_asp_export does for an NVFP4 one). */
 qwam_status qwam_asp_export_nvfp4(qwam_asp_handle h, void* qw, void* sfw, float* sg, void* Bh);
 
-/* Sticky device-side error of the handle (QWAM_OK, QWAM_ERR_TIMEOUT or QWAM_ERR_RANGE);
- * synchronizes the device.  The word is cleared by this call. */
+/* Read-and-clear: returns the handle's device-side error word (QWAM_OK, QWAM_ERR_TIMEOUT or
+ * QWAM_ERR_RANGE) and resets it to QWAM_OK.  The word keeps the first error of any launch of
+ * the handle until this call reads it.  The call waits for the handle's last launch made outside
+ * a stream capture (an event on that launch's stream), not for the whole device: other streams
+ * and other users of the GPU go on.  Launches captured into a CUDA graph are not tracked:
+ * synchronize the stream that replays the graph before calling.  A timeout in kernel (a) does not
+ * stop the GEMM that follows it on the stream from running on the half-written workspace: treat
+ * the outputs of every launch since the last QWAM_OK as invalid when this returns an error. */
 qwam_status qwam_asp_get_error(qwam_asp_handle h);
 
 /* Shape of a handle (any output pointer may be NULL); `group` is 16 for an NVFP4 handle. */

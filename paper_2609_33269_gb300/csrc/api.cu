@@ -154,6 +154,28 @@ using qwam::Handle;
 
 static qwam_status from_cuda_status(cudaError_t e) { return e == cudaSuccess ? QWAM_OK : QWAM_ERR_CUDA; }
 
+// Frees everything a handle owns (any member may still be unset).
+static void release_handle(qwam_asp_handle hs) {
+  Handle& h = hs->h;
+  if (h.block) cudaFree(h.block);
+  if (h.bias) cudaFree(h.bias);
+  if (h.done) cudaEventDestroy(h.done);
+  if (h.err_stream) cudaStreamDestroy(h.err_stream);
+  if (h.err_host) cudaFreeHost(h.err_host);
+  delete hs;
+}
+
+// After a launch of the handle's kernels on `s`: remember it for qwam_asp_get_error.  Launches
+// into a stream capture are not tracked (an event recorded there belongs to the graph).
+static cudaError_t note_launch(Handle& h, cudaStream_t s) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(s, &cs);
+  if (e != cudaSuccess || cs != cudaStreamCaptureStatusNone) return e;
+  e = cudaEventRecord(h.done, s);
+  if (e == cudaSuccess) h.done_valid = true;
+  return e;
+}
+
 extern "C" {
 
 const char* qwam_status_string(qwam_status s) {
@@ -266,8 +288,7 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
                           static_cast<uint64_t>(h.ku3) * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
   }
   if (!ok) {
-    cudaFree(h.block);
-    delete hs;
+    release_handle(hs);
     return QWAM_ERR_CUDA;
   }
   cudaError_t e = cudaMemsetAsync(h.block, 0, total, s);
@@ -279,10 +300,14 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
       e = nv ? qwam::launch_pack_nvfp4(h, W, r > 0 ? U : nullptr, s) : qwam::launch_pack(h, W, r > 0 ? U : nullptr, s);
   }
   int herr = 0;
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);  // `s` may be a non-blocking stream
   if (e == cudaSuccess) e = cudaMemcpy(&herr, h.err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h.done, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h.err_stream, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaMallocHost(&h.err_host, sizeof(int));
   if (e != cudaSuccess || herr != 0) {
-    cudaFree(h.block);
-    delete hs;
+    cudaGetLastError();
+    release_handle(hs);
     return e != cudaSuccess ? QWAM_ERR_CUDA : QWAM_ERR_RANGE;
   }
   *out = hs;
@@ -349,7 +374,10 @@ static qwam_status quantize_impl(const void* X, int M, qwam_asp_handle hs, void*
   Handle& h = hs->h;
   const qwam::ActMaps* am = qwam::get_act_maps(h, X, ws, M);
   if (!am) return QWAM_ERR_CUDA;
-  return from_cuda_status(qwam::launch_actquant(h, *am, ws, M, dump, reinterpret_cast<cudaStream_t>(stream)));
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = qwam::launch_actquant(h, *am, ws, M, dump, s);
+  if (e == cudaSuccess) e = note_launch(h, s);
+  return from_cuda_status(e);
 }
 
 qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws,
@@ -452,11 +480,11 @@ qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle hs, void* Y
   Handle& h = hs->h;
   const qwam::ActMaps* am = qwam::get_act_maps(h, nullptr, act_ws, M);
   if (!am) return QWAM_ERR_CUDA;
-  if (h.fmt == qwam::kFmtNvfp4)
-    return from_cuda_status(qwam::launch_gemm_nvfp4(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32,
-                                                    reinterpret_cast<cudaStream_t>(stream)));
-  return from_cuda_status(qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32,
-                                            reinterpret_cast<cudaStream_t>(stream)));
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = h.fmt == qwam::kFmtNvfp4 ? qwam::launch_gemm_nvfp4(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s)
+                                           : qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s);
+  if (e == cudaSuccess) e = note_launch(h, s);
+  return from_cuda_status(e);
 }
 
 qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype, void* act_ws,
@@ -470,10 +498,14 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
 
 qwam_status qwam_asp_get_error(qwam_asp_handle hs) {
   if (!hs) return QWAM_ERR_INVALID_ARG;
-  if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
-  int v = 0;
-  if (cudaMemcpy(&v, hs->h.err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return QWAM_ERR_CUDA;
-  if (cudaMemset(hs->h.err, 0, sizeof(int)) != cudaSuccess) return QWAM_ERR_CUDA;
+  Handle& h = hs->h;
+  // read and clear the word on the handle's own stream, after the handle's last tracked launch
+  cudaError_t e = h.done_valid ? cudaStreamWaitEvent(h.err_stream, h.done, 0) : cudaSuccess;
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h.err_host, h.err, sizeof(int), cudaMemcpyDeviceToHost, h.err_stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h.err, 0, sizeof(int), h.err_stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h.err_stream);
+  if (e != cudaSuccess) return QWAM_ERR_CUDA;
+  const int v = *h.err_host;
   if (v & qwam::kErrTimeout) return QWAM_ERR_TIMEOUT;
   if (v & qwam::kErrRange) return QWAM_ERR_RANGE;
   return QWAM_OK;
@@ -558,10 +590,8 @@ qwam_status qwam_asp_export_nvfp4(qwam_asp_handle hs, void* qw, void* sfw, float
 
 qwam_status qwam_asp_destroy(qwam_asp_handle hs) {
   if (!hs) return QWAM_ERR_INVALID_ARG;
-  cudaDeviceSynchronize();
-  cudaError_t e = cudaFree(hs->h.block);
-  if (hs->h.bias) cudaFree(hs->h.bias);
-  delete hs;
+  const cudaError_t e = cudaDeviceSynchronize();
+  release_handle(hs);
   return from_cuda_status(e);
 }
 
@@ -607,7 +637,10 @@ qwam_status qwam_asp_set_timeout(qwam_asp_handle hs, double seconds) {
 
 qwam_status qwam_asp_debug_wait_timeout(qwam_asp_handle hs, int timeout_us, struct CUstream_st* stream) {
   if (!hs || timeout_us <= 0 || timeout_us > 10000000) return QWAM_ERR_INVALID_ARG;
-  return from_cuda_status(qwam::launch_wait_probe(hs->h, timeout_us, reinterpret_cast<cudaStream_t>(stream)));
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = qwam::launch_wait_probe(hs->h, timeout_us, s);
+  if (e == cudaSuccess) e = note_launch(hs->h, s);
+  return from_cuda_status(e);
 }
 
 }  // extern "C"

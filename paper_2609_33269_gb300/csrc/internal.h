@@ -75,7 +75,13 @@ struct Handle {
   __nv_bfloat16* ucat3 = nullptr;    // [K, ku3]: row k = U_hi[k,:], U_lo[k,:], U_hi[k,:], zeros
   uint8_t* sfw = nullptr;            // NVFP4: E4M3 block scales of W_perp in atoms (N_pad rows)
   float sg = 0.0f;                   // NVFP4: float32 per-tensor weight scale
-  int* err = nullptr;                // sticky device error word
+  int* err = nullptr;                // device error word (first error kept until read)
+  // qwam_asp_get_error waits for the handle's last launch, not for the device: an event
+  // recorded after each launch outside a stream capture, read through a stream of its own
+  cudaEvent_t done = nullptr;
+  bool done_valid = false;
+  cudaStream_t err_stream = nullptr;
+  int* err_host = nullptr;           // pinned host copy of the word
   // Smoothing and block Hadamard rotation in front of the layer (Sec. 3 Eq. (pair)): the packed
   // weight is W~ = H diag(s) W, the activations are rotated at run time, x~ = H diag(s)^-1 x.
   // ucat_t then holds diag(s)^-1 H U (the projection x~ U = x (diag(s)^-1 H U)) and ucat3 holds

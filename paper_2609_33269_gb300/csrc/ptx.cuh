@@ -83,10 +83,10 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
 
 // Every wait in the kernels is bounded.  A kernel gives up when its deadline passes or when
 // another warp of the CTA has already given up (shared abort flag); it then records
-// kErrTimeout in the sticky error word and unwinds.
+// kErrTimeout in the error word and unwinds.
 struct WaitCtl {
   volatile int* abort_flag;  // shared memory, 0 = running
-  int* err;                  // global sticky error word
+  int* err;                  // global error word (first error kept until read)
   uint64_t deadline_ns;      // %globaltimer value after which waits give up
 };
 

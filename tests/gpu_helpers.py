@@ -144,3 +144,51 @@ def check_layer_output(Y, Yo, Yk, qx_gpu, qx_oracle):
     if flip.any():
         assert rowwise_rel_err(Y[flip], Yk[flip]).max() <= 1e-5
     assert flip.mean() <= 0.05, flip.mean()
+
+
+E2M1_MIDPOINTS = np.array([0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0])
+_E4M3_POSITIVE = None
+
+
+def e4m3_positive_values():
+    """Values of the E4M3 codes 0..126 (the non-negative finite ones), from the oracle."""
+    global _E4M3_POSITIVE
+    if _E4M3_POSITIVE is None:
+        _E4M3_POSITIVE = np.array([oracle.e4m3_value(b) for b in range(127)])
+    return _E4M3_POSITIVE
+
+
+def nvfp4_mismatches(qx_gpu, sfx_gpu, qx_ref, sfx_ref, Xperp, eps=1e-3):
+    """NVFP4 activation codes and block scales against the oracle's (reading N3: per block of 16,
+    s = RN_e4m3(amax / 6) and code = RN_e2m1(x / s)), with Xperp the oracle's float64 remainder.
+
+    A block scale may differ only where amax / 6 lies within eps (relative) of a midpoint between
+    two E4M3 values; a code in a block whose scale agrees may differ only where |x| / s lies within
+    eps of an E2M1 midpoint.  Codes in a block whose scale differs follow that scale and are not
+    counted again.  Returns (number of mismatches, whether each is such a near tie)."""
+    M, K = qx_ref.shape
+    nb = K // 16
+    tab = e4m3_positive_values()
+    mids = (tab[1:] + tab[:-1]) / 2
+    t = np.abs(np.asarray(Xperp, np.float64)).reshape(M, nb, 16).max(axis=2) / 6.0
+    near = []
+    sbad = np.argwhere(sfx_gpu != sfx_ref)
+    for m, b in sbad:
+        near.append(np.abs(mids - t[m, b]).min() <= eps * t[m, b])
+    cbad = np.argwhere((qx_gpu != qx_ref) & np.repeat(sfx_gpu == sfx_ref, 16, axis=1))
+    for m, k in cbad:
+        s = tab[int(sfx_ref[m, k // 16])]
+        near.append(s > 0 and np.abs(E2M1_MIDPOINTS - abs(float(Xperp[m, k])) / s).min() <= eps)
+    return len(sbad) + len(cbad), np.array(near, bool)
+
+
+def check_nvfp4_activations(ga, oa, Xperp, R, Xin):
+    """The NVFP4 activation bar at r > 0: every differing code or block scale is a near tie, at
+    most max(2, 1e-4 * codes) differ, and the kernel's float32 remainder R is within 2e-5 of the
+    float64 one per row (relative to the row's largest input value Xin)."""
+    err = np.abs(R - Xperp).max(axis=1) / np.maximum(np.abs(Xin).max(axis=1), 1e-30)
+    assert err.max() <= 2e-5, err.max()
+    n_bad, near = nvfp4_mismatches(ga["qx"], ga["sfx"], oa["qx"], oa["sfx"], Xperp)
+    assert near.all(), (n_bad, near)
+    assert n_bad <= max(2, 1e-4 * ga["qx"].size), n_bad
+    return n_bad
