@@ -47,7 +47,7 @@ typedef struct qwam_asp_handle_s* qwam_asp_handle;
 typedef enum {
   QWAM_OK = 0,
   QWAM_ERR_INVALID_ARG = -1,
-  QWAM_ERR_UNSUPPORTED = -2, /* valid request that this build does not implement (e.g. r > 64) */
+  QWAM_ERR_UNSUPPORTED = -2, /* valid request that this build does not implement (e.g. r > 64 when rotated) */
   QWAM_ERR_CUDA = -3,
   QWAM_ERR_OOM = -4,
   QWAM_ERR_TIMEOUT = -5,     /* a bounded device wait gave up */
@@ -61,7 +61,10 @@ enum { QWAM_Y_BF16 = 0, QWAM_Y_FP32 = 1 };
  *   W_bf16 : device, bf16 [K, N] row-major (the paper's W~ in its transformed coordinates)
  *   U      : device, float32 [K, r] row-major, orthonormal columns; may be NULL iff r == 0
  *   K      : input dimension, K % 64 == 0;   N : output dimension, N % 8 == 0
- *   r      : protected rank, 0 <= r <= min(K, 64) (larger r returns QWAM_ERR_UNSUPPORTED)
+ *   r      : protected rank, 0 <= r <= K.  Ranks up to 64 run kernel (a) on the tensor cores;
+ *            larger ones take a general-rank activation path on the CUDA cores (cost K r per
+ *            token, for correctness rather than speed), which needs K % 256 == 0 (otherwise
+ *            QWAM_ERR_UNSUPPORTED).  Rotated handles are limited to r <= 64.
  *   group  : quantization group along K, 32 or 64
  *   out    : receives the new handle
  * Computes, in float64 on the device: B_f = U^T W, W_perp = W - U B_f, per (output channel,
@@ -246,7 +249,8 @@ qwam_status qwam_asp_shape(qwam_asp_handle h, int* K, int* N, int* r, int* group
  *   sw  : uint16 (float16 bits) [K/group, N]
  *   Bh  : uint16 (float16 bits) [N, r_pad]   (B_hat transposed, zero beyond r)
  *   Uhl : uint16 (bf16 bits) [2, K, r_pad]   (hi and lo parts of the projection basis: U, or
- *         diag(s)^-1 H U for a rotated handle; zero beyond r) */
+ *         diag(s)^-1 H U for a rotated handle; zero beyond r; all zero for r > 64, whose
+ *         general-rank path keeps the basis in float32 only) */
 qwam_status qwam_asp_export(qwam_asp_handle h, void* qw, void* sw, void* Bh, void* Uhl);
 
 /* Free the handle and its device buffers (synchronizes the device). */

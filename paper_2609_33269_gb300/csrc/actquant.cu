@@ -1001,6 +1001,106 @@ cudaError_t launch_smallq(const Handle& h, const void* X, const void* ws, int M,
   }
 }
 
+// ---- the general-rank path (r_pad > kMaxRank, any rank up to K; K a multiple of 256) ---------
+// Eq. (xsplit) on the CUDA cores, one CTA of four warps per token row, for ranks whose projection
+// does not fit kernel (a)'s tensor-memory layout.  The row goes to shared memory in float32; warp
+// w forms p_j for j = w, w + 4, ... as one warp-wide dot product over K (lane l takes channels
+// 256 c + 8 l .. + 7), all four warps then form the remainder of their 256-channel chunks as
+// x - sum_j p_j U[k, j] (j ascending) and quantize it with the lane quantizers, bit for bit those
+// of the other paths.  It is the rank range's correctness path, not a tuned one: its cost grows
+// as K r per token.
+template <bool NV>
+__global__ void __launch_bounds__(128) generalq_kernel(const __nv_bfloat16* __restrict__ X, const SmallArgs a, int RP) {
+  extern __shared__ float gsm[];
+  float* xs = gsm;          // [K] the row in float32
+  float* ps = gsm + a.K;    // [RP] its projection
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = static_cast<int>(threadIdx.x & 31), w = static_cast<int>(threadIdx.x >> 5);
+  const int m = blockIdx.x;
+  const __nv_bfloat16* row = X + static_cast<size_t>(m) * a.K;
+  const int nc = a.K / 256;
+  for (int c = w; c < nc; c += 4) {
+    const int k = 256 * c + 8 * lane;
+    float x[8];
+    load8(row + k, x);
+    reinterpret_cast<float4*>(xs + k)[0] = make_float4(x[0], x[1], x[2], x[3]);
+    reinterpret_cast<float4*>(xs + k)[1] = make_float4(x[4], x[5], x[6], x[7]);
+  }
+  __syncthreads();
+  for (int j = w; j < RP; j += 4) {
+    float acc = 0.0f;
+    for (int c = 0; c < nc; ++c) {
+      const int k = 256 * c + 8 * lane;
+      float x[8], u[8];
+      load8(xs + k, x);
+      load8(a.up + static_cast<size_t>(j) * a.K + k, u);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc = fmaf(x[i], u[i], acc);
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, off);
+    if (lane == 0) {
+      ps[j] = acc;
+      a.phat[static_cast<size_t>(m) * RP + j] = __float2half_rn(acc);
+    }
+  }
+  __syncthreads();
+  for (int c = w; c < nc; c += 4) {
+    const int k = 256 * c + 8 * lane;
+    float x[8], acc[8] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+    load8(xs + k, x);
+    for (int j = 0; j < RP; ++j) {
+      float u[8];
+      load8(a.ur + static_cast<size_t>(j) * a.K + k, u);
+      const float pj = ps[j];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] = fmaf(pj, u[i], acc[i]);
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) x[i] -= acc[i];
+    if (a.dump) {
+      float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + k);
+      d[0] = make_float4(x[0], x[1], x[2], x[3]);
+      d[1] = make_float4(x[4], x[5], x[6], x[7]);
+    }
+    quantize8_lanes<NV>(x, lane, m, k, a.q);
+  }
+}
+
+template <bool NV>
+cudaError_t launch_general(const Handle& h, const void* X, const void* ws, int M, float* dump, cudaStream_t s) {
+  const ActLayout L = act_layout(h, M);
+  uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
+  SmallArgs a;
+  a.M = M;
+  a.K = h.K;
+  a.up = h.up32;
+  a.ur = h.ur32;
+  a.phat = reinterpret_cast<__half*>(base + L.phat_off);
+  a.dump = dump;
+  a.q = quant_out(h, L, base);
+  a.inv_s = nullptr;
+  a.hb = 0;
+  const size_t smem = sizeof(float) * (static_cast<size_t>(h.K) + h.r_pad);
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(generalq_kernel<NV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(M, 1, 1);
+  cfg.blockDim = dim3(128, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, generalq_kernel<NV>, static_cast<const __nv_bfloat16*>(X), a, h.r_pad);
+}
+
 // Test support: the lane quantizers (quantize8_lanes, as the small-M and rotation kernels run
 // them) applied to caller-given float32 rows, one warp per row and 256 values.
 template <bool NV>
@@ -1140,6 +1240,7 @@ cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4
 
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
   const bool nv = h.fmt == kFmtNvfp4;
+  if (h.r_pad > kMaxRank) return nv ? launch_general<true>(h, am.x, ws, M, dump, s) : launch_general<false>(h, am.x, ws, M, dump, s);
   // The small-M kernel for few tokens, and for unrotated r = 0 layers at any token count (with no
   // projection its warp-wide pass beats kernel (a)'s tile pipeline: 15.0 against 19.0 us INT4 and
   // 14.6 against 30.0 us NVFP4 at M = 4096, K = 3072); small_m = 0 always takes kernel (a).

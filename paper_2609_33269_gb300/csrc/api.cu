@@ -92,6 +92,11 @@ ActLayout act_layout(const Handle& h, int M) {
       L.resid_off = L.bytes;
       L.bytes += up256(static_cast<size_t>(M) * h.K * 4);
     }
+    L.ytmp_off = 0;
+    if (h.r_pad > kMaxRank) {  // the 4-bit part in float32, before the branch is added
+      L.ytmp_off = L.bytes;
+      L.bytes += up256(static_cast<size_t>(M) * h.N * 4);
+    }
     return L;
   }
   L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
@@ -103,6 +108,7 @@ ActLayout act_layout(const Handle& h, int M) {
     L.resid_off = L.bytes;
     L.bytes += up256(static_cast<size_t>(M) * h.K * 4);
   }
+  L.ytmp_off = 0;
   return L;
 }
 
@@ -202,7 +208,9 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
   if (fmt == qwam::kFmtInt4 && group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
   if (r < 0 || r > K) return QWAM_ERR_INVALID_ARG;
   if (r > 0 && (!U || !qwam::aligned16(U))) return QWAM_ERR_INVALID_ARG;
-  if (r > qwam::kMaxRank) return QWAM_ERR_UNSUPPORTED;
+  // Ranks above kMaxRank take the general-rank activation path (one warp per 256 channels of a
+  // row); the rotated layers keep the tensor-core path only.
+  if (r > qwam::kMaxRank && (rot || K % 256 != 0)) return QWAM_ERR_UNSUPPORTED;
   // the run-time rotation works on sub-blocks of 256 channels (one warp, eight per lane)
   if (rot && (K % 256 != 0 || (sm && !qwam::aligned16(sm)))) return QWAM_ERR_INVALID_ARG;
   if (!qwam::ensure_encoder()) return QWAM_ERR_CUDA;
@@ -233,8 +241,10 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
                          : qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
   const size_t b_s32 = nv ? 0 : qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 4);
   const size_t b_bh = qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2);
-  const size_t b_ut = qwam::up256(static_cast<size_t>(2 * h.r_pad) * K * 2);
-  const size_t b_u3 = qwam::up256(static_cast<size_t>(K) * h.ku3 * 2);
+  // the bf16 split bases feed kernel (a)'s tensor-core path only (r_pad <= kMaxRank)
+  const bool tc_bases = h.r_pad > 0 && h.r_pad <= qwam::kMaxRank;
+  const size_t b_ut = tc_bases ? qwam::up256(static_cast<size_t>(2 * h.r_pad) * K * 2) : 0;
+  const size_t b_u3 = tc_bases ? qwam::up256(static_cast<size_t>(K) * h.ku3 * 2) : 0;
   const size_t b_is = rot ? qwam::up256(static_cast<size_t>(K) * 4) : 0;
   const size_t b_u32 = qwam::up256(static_cast<size_t>(K) * h.r_pad * 4);
   const size_t total = b_qw + b_sw + b_s32 + b_bh + b_ut + b_u3 + b_is + 2 * b_u32 + 256;
@@ -253,8 +263,10 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
   }
   uint8_t* q = p + b_qw + b_sw + b_s32;
   h.Bh = reinterpret_cast<__half*>(q);
-  h.ucat_t = reinterpret_cast<__nv_bfloat16*>(q + b_bh);
-  h.ucat3 = reinterpret_cast<__nv_bfloat16*>(q + b_bh + b_ut);
+  if (tc_bases) {
+    h.ucat_t = reinterpret_cast<__nv_bfloat16*>(q + b_bh);
+    h.ucat3 = reinterpret_cast<__nv_bfloat16*>(q + b_bh + b_ut);
+  }
   if (rot) h.inv_s = reinterpret_cast<float*>(q + b_bh + b_ut + b_u3);
   if (h.r_pad > 0) {
     // without rotation both bases are U: one copy, so the small-M kernel's reconstruction reads
@@ -282,6 +294,8 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
                           static_cast<uint64_t>(h.r_pad) * 2, 8, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
     ok &= qwam::encode_2d(&h.bh32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,
                           static_cast<uint64_t>(h.r_pad) * 2, 32, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+  }
+  if (tc_bases) {
     ok &= qwam::encode_2d(&h.ucat_t_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h.ucat_t, K, 2 * h.r_pad,
                           static_cast<uint64_t>(K) * 2, qwam::kChunk, 2 * h.r_pad, CU_TENSOR_MAP_SWIZZLE_128B);
     ok &= qwam::encode_2d(&h.ucat3_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h.ucat3, h.ku3, K,
@@ -550,15 +564,21 @@ qwam_status qwam_asp_export(qwam_asp_handle hs, void* qw, void* sw, void* Bh, vo
   if (e == cudaSuccess && Bh && h.r_pad > 0)
     e = cudaMemcpy(Bh, h.Bh, static_cast<size_t>(h.N) * h.r_pad * 2, cudaMemcpyDeviceToHost);
   if (e == cudaSuccess && Uhl && h.r_pad > 0) {
-    std::vector<uint16_t> t(static_cast<size_t>(2 * h.r_pad) * h.K);
-    e = cudaMemcpy(t.data(), h.ucat_t, t.size() * 2, cudaMemcpyDeviceToHost);
     uint16_t* o = static_cast<uint16_t*>(Uhl);
-    for (int part = 0; part < 2 && e == cudaSuccess; ++part)
-      for (int k = 0; k < h.K; ++k)
-        for (int j = 0; j < h.r_pad; ++j)
-          o[(static_cast<size_t>(part) * h.K + k) * h.r_pad + j] =
-              t[static_cast<size_t>(part * h.r_pad + j) * h.K + k];
+    if (h.ucat_t) {
+      std::vector<uint16_t> t(static_cast<size_t>(2 * h.r_pad) * h.K);
+      e = cudaMemcpy(t.data(), h.ucat_t, t.size() * 2, cudaMemcpyDeviceToHost);
+      for (int part = 0; part < 2 && e == cudaSuccess; ++part)
+        for (int k = 0; k < h.K; ++k)
+          for (int j = 0; j < h.r_pad; ++j)
+            o[(static_cast<size_t>(part) * h.K + k) * h.r_pad + j] =
+                t[static_cast<size_t>(part * h.r_pad + j) * h.K + k];
+    } else {
+      // the general-rank path keeps no bf16 split: none to export
+      std::fill(o, o + static_cast<size_t>(2 * h.K) * h.r_pad, static_cast<uint16_t>(0));
+    }
   }
+  if (e != cudaSuccess) cudaGetLastError();  // leave no error behind for the next call
   return from_cuda_status(e);
 }
 

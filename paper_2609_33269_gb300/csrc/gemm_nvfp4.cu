@@ -317,8 +317,31 @@ __global__ void __launch_bounds__(kThreads4, 1)
   }
 }
 
+// Ranks above kMaxRank: the 16-bit branch added to the 4-bit part (float32, no bias) after the GEMM,
+// one thread per output, float32 sums over j ascending:  Y = Y4 + p_hat B_hat^T (+ bias).
+__global__ void __launch_bounds__(128) branch_finalize_kernel(const float* __restrict__ y4,
+                                                              const __half* __restrict__ ph,
+                                                              const __half* __restrict__ bh, const float* bias, int M,
+                                                              int N, int rp, void* Y, int y_f32) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int n = blockIdx.x * blockDim.x + threadIdx.x, m = blockIdx.y;
+  if (n >= N || m >= M) return;
+  float acc = 0.0f;
+  for (int j = 0; j < rp; ++j)
+    acc = fmaf(__half2float(ph[static_cast<size_t>(m) * rp + j]), __half2float(bh[static_cast<size_t>(n) * rp + j]), acc);
+  float y = y4[static_cast<size_t>(m) * N + n] + acc;
+  if (bias) y += bias[n];
+  const size_t off = static_cast<size_t>(m) * N + n;
+  if (y_f32)
+    static_cast<float*>(Y)[off] = y;
+  else
+    static_cast<__nv_bfloat16*>(Y)[off] = __float2bfloat16_rn(y);
+}
+
 template <int RP>
-cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s) {
+cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s,
+                      bool with_bias = true) {
   using Cfg = Gemm4Cfg<RP>;
   const ActLayout L = act_layout(h, M);
   Gemm4Args a;
@@ -332,7 +355,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, void*
   a.sg = h.sg;
   a.Y = Y;
   a.y_f32 = y_f32 ? 1 : 0;
-  a.bias = h.bias;
+  a.bias = with_bias ? h.bias : nullptr;
   a.err = h.err;
   a.timeout_ns = deadline_budget_ns(h);
   static bool attr_done = false;
@@ -367,8 +390,27 @@ cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int 
     case 32: return launch_rp<32>(h, am, ws, M, Y, y_f32, s);
     case 48: return launch_rp<48>(h, am, ws, M, Y, y_f32, s);
     case 64: return launch_rp<64>(h, am, ws, M, Y, y_f32, s);
-    default: return cudaErrorInvalidValue;
+    default: break;
   }
+  if (h.r_pad <= kMaxRank) return cudaErrorInvalidValue;
+  // larger ranks: the 4-bit part in float32 into the workspace, then the branch and the bias
+  const ActLayout L = act_layout(h, M);
+  uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
+  float* y4 = reinterpret_cast<float*>(base + L.ytmp_off);
+  cudaError_t e = launch_rp<0>(h, am, ws, M, y4, true, s, false);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((h.N + 127) / 128, M, 1);
+  cfg.blockDim = dim3(128, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, branch_finalize_kernel, static_cast<const float*>(y4),
+                            reinterpret_cast<const __half*>(base + L.phat_off), static_cast<const __half*>(h.Bh),
+                            static_cast<const float*>(h.bias), M, h.N, h.r_pad, Y, y_f32 ? 1 : 0);
 }
 
 }  // namespace qwam

@@ -14,7 +14,7 @@ namespace qwam {
 
 constexpr int kBM = 128;        // token rows per CTA tile (one TMEM lane per row)
 constexpr int kChunk = 64;      // K columns per activation chunk (bf16: one 128-byte row)
-constexpr int kMaxRank = 64;    // largest protected rank of this build
+constexpr int kMaxRank = 64;    // largest rank of kernel (a)'s tensor-core path (above: the general-rank path)
 constexpr int kGemmBN = 128;    // output columns per GEMM CTA tile
 constexpr int kScaleGroups = 8; // groups per INT4 GEMM scale slot (s_x and the weight scale)
 
@@ -109,6 +109,7 @@ struct Handle {
 struct ActLayout {
   size_t codes_off, scales_off, ab_off, phat_off, bytes;
   size_t resid_off;  // rotated handles with r > 0: float32 [M, K] remainder before the rotation
+  size_t ytmp_off;   // NVFP4 with r_pad > kMaxRank: float32 [M, N] 4-bit part before the branch
   int M_pad;
 };
 ActLayout act_layout(const Handle& h, int M);

@@ -296,7 +296,8 @@ cudaError_t pack_nvfp4(Handle& h, const WT* W, const float* U, const float* Up, 
                                                                           sg_dev);
     if (r > 0) {
       branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
-      split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+      if (h.ucat_t)  // kernel (a)'s tensor-core bases (r_pad <= kMaxRank)
+        split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
       basis32_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.up32, h.ur32);
     }
     e = cudaGetLastError();
@@ -324,7 +325,8 @@ cudaError_t pack_int4(Handle& h, const WT* W, const float* U, const float* Up, c
                                                                      h.err);
   if (r > 0) {
     branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
-    split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
+    if (h.ucat_t)  // kernel (a)'s tensor-core bases (r_pad <= kMaxRank)
+      split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
     basis32_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.up32, h.ur32);
   }
   e = cudaGetLastError();

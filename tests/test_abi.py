@@ -53,8 +53,11 @@ def test_host_validation_rejects_bad_arguments_without_a_launch(lib):
     # misaligned W
     assert lib.qwam_asp_pack_weights(V((1 << 20) + 2), None, 64, 64, 0, 64, None,
                                      ctypes.byref(h)) == asp.QWAM_ERR_INVALID_ARG
-    # rank above this build's maximum (valid per the paper) is reported as unsupported
-    assert lib.qwam_asp_pack_weights(fake, fake, 256, 64, 65, 64, None, ctypes.byref(h)) == asp.QWAM_ERR_UNSUPPORTED
+    # a rank above 64 is valid per the paper; this build supports it when K % 256 == 0 and the
+    # handle is not rotated, and reports the other cases as unsupported
+    assert lib.qwam_asp_pack_weights(fake, fake, 320, 64, 65, 64, None, ctypes.byref(h)) == asp.QWAM_ERR_UNSUPPORTED
+    assert lib.qwam_asp_pack_weights_rotated(fake, None, fake, 256, 64, 65, 64, None,
+                                             ctypes.byref(h)) == asp.QWAM_ERR_UNSUPPORTED
     size = ctypes.c_size_t()
     assert lib.qwam_asp_act_workspace_bytes(None, 4, ctypes.byref(size)) == asp.QWAM_ERR_INVALID_ARG
     assert lib.qwam_asp_linear(None, 4, None, None, 0, None, None) == asp.QWAM_ERR_INVALID_ARG

@@ -21,7 +21,7 @@ import oracle
 from paper_2609_33269_gb300 import asp
 from paper_2609_33269_gb300 import workloads as wl
 
-from gpu_helpers import check_nvfp4_activations, rowwise_rel_err, to_dev_bf16
+from gpu_helpers import NvCase, atoms_to_rows, check_nvfp4_activations, rowwise_rel_err, to_dev_bf16, unpack_e2m1
 
 pytestmark = pytest.mark.gpu
 
@@ -31,68 +31,6 @@ def built():
     from paper_2609_33269_gb300 import build
     build.build()
     asp.load()
-
-
-def unpack_e2m1(packed):
-    """uint8 [R, K/2] -> E2M1 codes uint8 [R, K], low nibble = even k."""
-    p = np.ascontiguousarray(packed)
-    out = np.empty((p.shape[0], p.shape[1] * 2), np.uint8)
-    out[:, 0::2] = p & 0xF
-    out[:, 1::2] = p >> 4
-    return out
-
-
-def atoms_to_rows(atoms, rows, K):
-    """Scale atoms (512 bytes per 128 rows x 64 K; row r's four scales at (r % 32) * 16 +
-    (r % 128 // 32) * 4) -> row-major uint8 [rows, K/16]."""
-    a = np.asarray(atoms, np.uint8)
-    r = np.arange(rows)[:, None]
-    b = np.arange(K // 16)[None, :]
-    idx = ((r // 128) * (K // 64) + b // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + b % 4
-    return a[idx]
-
-
-class NvCase:
-    def __init__(self, M, K, N, r, seed=0, layer_id=0, dist="outlier"):
-        self.M, self.K, self.N, self.r = M, K, N, r
-        self.Xb = wl.activations(M, K, seed=seed, layer_id=layer_id, dist=dist)
-        self.Wb = wl.weight(K, N, seed=seed, layer_id=layer_id)
-        self.U = wl.basis(K, r, seed=seed, layer_id=layer_id)
-        self.X = to_dev_bf16(self.Xb)
-        W = to_dev_bf16(self.Wb)
-        Ud = torch.from_numpy(self.U).cuda() if r > 0 else None
-        self.layer = asp.AspLinear(W, Ud, fmt=asp.QWAM_FMT_NVFP4)
-        self._ow = None
-
-    def oracle_weights(self):
-        if self._ow is None:
-            self._ow = oracle.pack_nvfp4(self.Wb, self.U)
-        return self._ow
-
-    def gpu_weights(self):
-        e = asp.qwam_asp_export_nvfp4(self.layer.h)
-        return dict(qw=unpack_e2m1(e["qw"]), sfw=e["sfw"], sg=e["sg"], Bh=e["Bh"][:, :self.r].T.copy())
-
-    def gpu_act(self):
-        codes, atoms, ph = self.layer.act_views_nvfp4(self.M)
-        torch.cuda.synchronize()
-        return dict(qx=unpack_e2m1(codes.cpu().numpy()),
-                    sfx=atoms_to_rows(atoms.cpu().numpy(), self.M, self.K),
-                    ph=ph.cpu().numpy().view(np.uint16)[:, :self.r].copy())
-
-    def residual(self):
-        R = torch.empty((self.M, self.K), dtype=torch.float32, device="cuda")
-        asp.qwam_asp_debug_residual(self.X, self.M, self.layer.h, self.layer.workspace(self.M), R)
-        torch.cuda.synchronize()
-        return R.cpu().numpy()
-
-    def run(self, fp32=True):
-        Y = self.layer(self.X, fp32=fp32)
-        torch.cuda.synchronize()
-        return Y
-
-    def close(self):
-        self.layer.close()
 
 
 PACK_SHAPES = [(512, 512, 16), (256, 136, 0), (1024, 384, 48), (256, 64, 64), (768, 264, 32)]

@@ -21,7 +21,8 @@ import oracle
 from paper_2609_33269_gb300 import asp
 from paper_2609_33269_gb300 import workloads as wl
 
-from gpu_helpers import Case, check_layer_output, check_nvfp4_activations, near_tie_mismatches, rowwise_rel_err, to_dev_bf16
+from gpu_helpers import (Case, atoms_to_rows, check_layer_output, check_nvfp4_activations, near_tie_mismatches,
+                         rowwise_rel_err, to_dev_bf16, unpack_e2m1)
 
 pytestmark = pytest.mark.gpu
 
@@ -170,22 +171,6 @@ def test_rotated_full_size_sampled_rows():
 
 
 # ---- NVFP4 variant with the rotation ------------------------------------------------------------
-
-def unpack_e2m1(packed):
-    p = np.ascontiguousarray(packed)
-    out = np.empty((p.shape[0], p.shape[1] * 2), np.uint8)
-    out[:, 0::2] = p & 0xF
-    out[:, 1::2] = p >> 4
-    return out
-
-
-def atoms_to_rows(atoms, rows, K):
-    a = np.asarray(atoms, np.uint8)
-    rr = np.arange(rows)[:, None]
-    b = np.arange(K // 16)[None, :]
-    idx = ((rr // 128) * (K // 64) + b // 4) * 512 + (rr % 32) * 16 + ((rr % 128) // 32) * 4 + b % 4
-    return a[idx]
-
 
 @PATHS
 @pytest.mark.parametrize("shape", [(200, 512, 256, 16), (65, 1536, 136, 0), (130, 3072, 128, 32)],
