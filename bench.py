@@ -245,9 +245,11 @@ def run_reference(args):
     return 0
 
 
-def cpu_baseline(rows_req: int, nvfp4: bool = False, rotate: bool = False):
+def cpu_baseline(rows_req: int, nvfp4: bool = False, rotate: bool = False, gpu=None):
     """The oracle as it stands on the host cores: whole passes over a sample of the workload's
-    rows, repeated until about ten seconds of CPU work (packing excluded, as on the GPU)."""
+    rows, repeated until about ten seconds of CPU work (packing excluded, as on the GPU).  With
+    `gpu` (the GPU's codes, scales and float32 output for the workload's first rows), the sample's
+    oracle result is also compared with them, after the timing (see parity_sample)."""
     K, N = WORKLOAD["K"], WORKLOAD["N"]
     rows = rows_req or WORKLOAD["M"]
     Xb, U, wts, layer = oracle_sample(rows, nvfp4, rotate)
@@ -258,9 +260,58 @@ def cpu_baseline(rows_req: int, nvfp4: bool = False, rotate: bool = False):
         dt = time.perf_counter() - t0
         if dt >= 10.0 or reps >= 50:
             break
-    return {"value": 2.0 * rows * N * K * reps / dt / 1e12, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-            "sample": f"{reps} pass(es) over {rows} of {WORKLOAD['M']} token rows (activation quantization + "
-                      f"output, {dt:.1f} s); weight packing offline"}
+    out = {"value": 2.0 * rows * N * K * reps / dt / 1e12, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+           "sample": f"{reps} pass(es) over {rows} of {WORKLOAD['M']} token rows (activation quantization + "
+                     f"output, {dt:.1f} s); weight packing offline"}
+    if gpu is not None and not rotate:
+        n = min(rows, len(gpu["Y"]))
+        out["parity_sample"] = parity_sample(Xb[:n], U, wts, layer.G, nvfp4, {k: v[:n] for k, v in gpu.items()})
+    return out
+
+
+def parity_sample(Xb, U, wts, G, nvfp4, gpu):
+    """Flip and row-error counts of the timed configuration's GPU result against the oracle on the
+    same rows.  At r > 0 the kernel's float32 remainder differs from the oracle's float64 one in
+    the last bits, so a code (or an NVFP4 block scale) can round the other way where the float64
+    quotient sits next to a rounding midpoint: every such flip is counted and checked to be within
+    1e-3 of a midpoint; the output is compared per row (max |dY| / max |Y|), separately for rows
+    with and without a flip."""
+    import oracle
+    oa = oracle.quantize_act(Xb, U, 32 if nvfp4 else G, want_float64=True)
+    Xp = oa["Xperp"]
+    if nvfp4:
+        oa = oracle.quantize_act_nvfp4(Xb, U)
+        Yo = oracle.linear_nvfp4(oa, wts)
+        tab = np.array([oracle.e4m3_value(b) for b in range(127)])
+        mids = (tab[1:] + tab[:-1]) / 2
+        M, K = oa["qx"].shape
+        t = np.abs(Xp).reshape(M, K // 16, 16).max(axis=2) / 6.0
+        sbad = np.argwhere(gpu["sfx"] != oa["sfx"])
+        near = [np.abs(mids - t[m, b]).min() <= 1e-3 * t[m, b] for m, b in sbad]
+        cbad = np.argwhere((gpu["qx"] != oa["qx"]) & np.repeat(gpu["sfx"] == oa["sfx"], 16, axis=1))
+        e2m1_mids = np.array([0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0])
+        for m, k in cbad:
+            s = tab[int(oa["sfx"][m, k // 16])]
+            near.append(s > 0 and np.abs(e2m1_mids - abs(Xp[m, k]) / s).min() <= 1e-3)
+        flips, scale_flips = len(sbad) + len(cbad), len(sbad)
+        flip_rows = np.any(gpu["qx"] != oa["qx"], axis=1) | np.any(gpu["sfx"] != oa["sfx"], axis=1)
+    else:
+        Yo = oracle.linear(oa, wts, G)
+        bad = np.argwhere(gpu["qx"] != oa["qx"])
+        near = []
+        for m, k in bad:
+            s = float(oa["sx"][m, k // G])
+            q = abs(float(Xp[m, k])) / s if s > 0 else 0.0
+            near.append(abs(q - np.floor(q) - 0.5) <= 1e-3)
+        flips, scale_flips = len(bad), int(np.sum(gpu["sx"].view(np.uint32) != oa["sx"].view(np.uint32)))
+        flip_rows = np.any(gpu["qx"] != oa["qx"], axis=1)
+    err = np.abs(gpu["Y"] - Yo).max(axis=1) / np.maximum(np.abs(Yo).max(axis=1), 1e-30)
+    return {"rows": int(len(Yo)), "codes": int(gpu["qx"].size), "code_or_block_scale_flips": int(flips),
+            "all_flips_near_ties": bool(all(near)), "scales_not_bit_equal": int(scale_flips),
+            "rows_with_a_flip": int(flip_rows.sum()),
+            "max_row_err_rows_without_flip": float(err[~flip_rows].max()) if (~flip_rows).any() else None,
+            "max_row_err_rows_with_flip": float(err[flip_rows].max()) if flip_rows.any() else None,
+            "note": "bit-exact codes and scales only given the kernel's own float32 remainder at r > 0"}
 
 
 def kernel_traffic(kernel: str):
@@ -334,18 +385,23 @@ def small_m_latencies(asp, wl, dev, stream, dev_bf16):
             "layers": out}
 
 
-def denoise_sweep(asp, wl, dev, stream, fmt, steps):
+def denoise_sweep(asp, wl, dev, stream, fmt, steps, hbm_peak, mma_peak, peak_source):
     """The denoising-step layer sweep: 30 DiT blocks x {qkv 3072->9216, o 3072->3072, up
     3072->12288, down 12288->3072} at M = 4096 tokens, ASP (r = 32) on the workload's seeded third of
-    the blocks and r = 0 elsewhere, over `steps` denoising steps with a fresh activation set each
-    step.  Weights and activations are drawn on the device (seeded torch generator) with the
-    recipe's distributions, so that the 120 layers pack in seconds (the bases are the workload's
-    own); every layer is packed once.
-    Two activation sets per input width alternate, so a layer's input may still be in L2 from an
-    earlier layer, as the previous layer's output would be in a model.  Returns aggregate effective
-    TOPS over all layer calls and a breakdown by layer kind and rank."""
+    the blocks and r = 0 elsewhere, over `steps` denoising steps.  Weights and activations are drawn
+    on the device (seeded torch generator) with the recipe's distributions, so that the 120 layers
+    pack in seconds (the bases are the workload's own); every layer is packed once.
+    Headline (`value`): every step gets fresh activations, drawn in the untimed gap before it,
+    and L2 is flushed (a 256 MB write) before it; each step is timed on its own and the steps'
+    times are summed.  Within a step two activation sets per input width alternate, so a layer's
+    input may still be in L2 from an earlier layer of the step, as the previous layer's output
+    would be in a model.  `l2_warm` times the same steps back to back on one activation draw.
+    Also: a roofline object (the aggregate against the MMA kind's peak) and the layers' roofline
+    fraction (sum over calls of max(algorithmic bytes / HBM, flops / MMA peak) over the measured
+    time), and a breakdown by layer kind and rank."""
     import torch
     W = wl.denoise_sweep(steps=steps)
+    nv = fmt == asp.QWAM_FMT_NVFP4
     g = torch.Generator(device=dev)
     g.manual_seed(0)
     lins = []
@@ -354,8 +410,8 @@ def denoise_sweep(asp, wl, dev, stream, fmt, steps):
         U = torch.from_numpy(L.u()).to(dev) if L.r else None  # the workload's seeded basis (host QR)
         lins.append(asp.AspLinear(Wt, U, L.G, fmt=fmt))
         del Wt
-    # activation sets: two per input width and step parity, 1 % outlier channels x U(10, 30), and
-    # Student-t (nu = 4) for the down projections' input
+    # activation sets: two per input width, 1 % outlier channels x U(10, 30), and Student-t
+    # (nu = 4) for the down projections' input
     def draw(K, student):
         if student:  # t(4) = N(0, 1) / sqrt(chi2(4) / 4)
             z = torch.randn((5, 4096, K), generator=g, device=dev)
@@ -366,9 +422,14 @@ def denoise_sweep(asp, wl, dev, stream, fmt, steps):
             ch = torch.randperm(K, generator=g, device=dev)[: K // 100]
             x[:, ch] *= torch.empty(K // 100, device=dev).uniform_(10.0, 30.0, generator=g)
         return x.to(torch.bfloat16).contiguous()
-    xs = {(K, st, i): draw(K, st) for K, st in ((3072, False), (12288, True)) for i in range(2)}
+
+    def draw_all():
+        return {(K, st, i): draw(K, st) for K, st in ((3072, False), (12288, True)) for i in range(2)}
+
+    xs = draw_all()
     outs = {N: torch.empty((4096, N), dtype=torch.bfloat16, device=dev) for N in (3072, 9216, 12288)}
     ws = torch.empty(max(asp.qwam_asp_act_workspace_bytes(l.h, 4096) for l in lins), dtype=torch.uint8, device=dev)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)  # 256 MB > L2
 
     def one_step(i, ev=None):
         for j, (L, lin) in enumerate(zip(W.layers, lins)):
@@ -384,15 +445,38 @@ def denoise_sweep(asp, wl, dev, stream, fmt, steps):
     for lin in lins:
         if asp.qwam_asp_get_error(lin.h) != asp.QWAM_OK:
             raise RuntimeError("device error in the sweep warm-up")
+    # fresh activations and a cold L2 before every step; each step timed alone
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * len(lins))] for _ in range(steps)]
+    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for i in range(steps):
+        xs = draw_all()
+        flush.zero_()
+        torch.cuda.synchronize()
+        step_ev[i][0].record(stream)
+        one_step(i, evs[i])
+        step_ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    total_ms = sum(a.elapsed_time(b) for a, b in step_ev)
+    # the same steps back to back on one draw (inputs partly L2-resident across steps)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(steps):
-        one_step(i, evs[i])
+        one_step(i)
     e1.record(stream)
     torch.cuda.synchronize()
-    total_ms = e0.elapsed_time(e1)
+    warm_ms = e0.elapsed_time(e1)
+    for lin in lins:
+        if asp.qwam_asp_get_error(lin.h) != asp.QWAM_OK:
+            raise RuntimeError("device error in the sweep")
     flops = sum(2.0 * L.M * L.N * L.K for L in W.layers) * steps
+    # per call: the slower of the algorithmic bytes over HBM (X, packed W and its scales, U, B_hat,
+    # the bf16 Y) and the flops over the MMA kind's peak
+    t_roof = 0.0
+    for L, lin in zip(W.layers, lins):
+        w_bytes = L.N * L.K // 2 + (L.N * L.K // 16 if nv else 2 * L.N * L.K // L.G)
+        by = 2 * L.M * L.K + w_bytes + 2 * L.K * lin.r_pad + 2 * L.N * lin.r_pad + 2 * L.M * L.N
+        t_roof += max(by / (hbm_peak * 1e9), 2.0 * L.M * L.N * L.K / (mma_peak * 1e12))
+    t_roof *= steps
     kinds = {}
     for j, L in enumerate(W.layers):
         key = "%s_r%d" % (L.name.split("_", 1)[1], L.r)
@@ -403,8 +487,15 @@ def denoise_sweep(asp, wl, dev, stream, fmt, steps):
         k[2] += steps
     for lin in lins:
         lin.close()
-    return {"value": flops / (total_ms * 1e-3) / 1e12, "unit": UNIT, "steps": steps,
+    value = flops / (total_ms * 1e-3) / 1e12
+    return {"value": value, "unit": UNIT, "steps": steps,
             "ms_per_denoising_step": total_ms / steps, "layers_per_step": len(W.layers),
+            "inputs": "fresh activations drawn before every step, L2 flushed before every step, steps timed alone",
+            "l2_warm": {"value": flops / (warm_ms * 1e-3) / 1e12, "ms_per_denoising_step": warm_ms / steps,
+                        "inputs": "one activation draw, steps back to back"},
+            "roofline": {"bound": "tensor", "achieved": value, "peak": mma_peak, "unit": "TFLOP/s",
+                         "frac": value / mma_peak, "traffic": None, "peak_source": peak_source},
+            "layer_roofline_frac": t_roof * 1e3 / total_ms,
             "asp_blocks": W.note, "what": "30 DiT blocks x {qkv, o, up, down} at M = 4096, r = 32 on a third "
             "of the blocks, r = 0 elsewhere; one qwam_asp_linear per layer; device-drawn synthetic data",
             "by_layer": {k: {"us_per_call": round(v[0] / v[2] * 1e3, 1), "tops": round(v[1] / (v[0] * 1e-3) / 1e12, 1)}
@@ -520,6 +611,11 @@ def run_ours(args):
                     "achieved_tflops": flops / (t_b * 1e-3) / 1e12, f"peak_tflops_{pname}": peak},
         }
         kern["actquant"]["frac"] = kern["actquant"]["achieved_gbs"] / hbm_peak
+        # what kernel (a) moves: the algorithmic bytes (4-bit codes written packed, as counted),
+        # plus, with r > 0, its second pass over X (re-read from L2 after the projection)
+        moved = a_bytes + (2 * M * K if r_pad > 0 else 0)
+        kern["actquant"].update(moved_bytes=moved, achieved_gbs_of_moved_bytes=moved / (t_a * 1e-3) / 1e9,
+                                moved_note="second pass over X served from L2" if r_pad > 0 else "one pass")
         kern[gname]["frac"] = kern[gname]["achieved_tflops"] / peak
         if t_b >= t_a:
             roof = {"kernel": gname, "bound": "tensor", "achieved": kern[gname]["achieved_tflops"],
@@ -548,6 +644,10 @@ def run_ours(args):
     sets, total_ms, t_a, t_b = main_run["sets"], main_run["total_ms"], main_run["t_a"], main_run["t_b"]
     value = main_run["value"]
     working_mb = main_run["mb"]
+    # the first rows' codes, scales and output, for the oracle comparison in the CPU baseline
+    gpu_par = None
+    if not args.no_cpu_baseline and world == 1 and not args.rotate:
+        gpu_par = gpu_sample(sets[0][0], sets[0][1], M, 512, fmt == asp.QWAM_FMT_NVFP4)
 
     # End to end through the public API, as a serving loop would run it: every step copies its
     # activations from pinned host memory to the device, runs the layer (qwam_asp_linear) and
@@ -614,8 +714,10 @@ def run_ours(args):
         for s_ in vr["sets"]:
             s_[0].close()
         variants["small_m"] = small_m_latencies(asp, wl, dev, stream, dev_bf16)
-        variants["sweep_int4"] = denoise_sweep(asp, wl, dev, stream, asp.QWAM_FMT_INT4, 10)
-        variants["sweep_nvfp4"] = denoise_sweep(asp, wl, dev, stream, asp.QWAM_FMT_NVFP4, 10)
+        variants["sweep_int4"] = denoise_sweep(asp, wl, dev, stream, asp.QWAM_FMT_INT4, 10, hbm_peak, fp8_peak,
+                                               "measured bf16 burst x 2 (nominal fp8/bf16 dense ratio), of measured")
+        variants["sweep_nvfp4"] = denoise_sweep(asp, wl, dev, stream, asp.QWAM_FMT_NVFP4, 10, hbm_peak, fp4_peak,
+                                                "measured bf16 burst x 6 (nominal fp4/bf16 dense ratio), of measured")
         # Smoothing and the block Hadamard rotation (B = 1024) in front of the same layer: kernel (a)
         # writes the float32 remainder, the rotation kernel rotates and quantizes it (two launches
         # in qwam_asp_quantize_act).
@@ -653,11 +755,45 @@ def run_ours(args):
         "clocks": clocks.summary(),
     }
     if not args.no_cpu_baseline and world == 1:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_rows, fmt == asp.QWAM_FMT_NVFP4, args.rotate)
+        line["cpu_baseline"] = cpu_baseline(args.cpu_rows, fmt == asp.QWAM_FMT_NVFP4, args.rotate, gpu_par)
     print(json.dumps(line))
     for s_ in sets:
         s_[0].close()
     return 0
+
+
+def gpu_sample(lin, X, M, rows, nvfp4):
+    """The GPU's codes, scales and float32 output for the first `rows` token rows of X (one
+    untimed call), decoded to the oracle's layouts: INT4 codes from SM4 words (word j holds
+    k = 8j..8j+7: bytes sign | magnitude, the upper four codes rotated by four bits), NVFP4 E2M1
+    codes two per byte (low nibble first) and block scales from the 512-byte atoms."""
+    import torch
+    Y = lin(X, fp32=True)
+    torch.cuda.synchronize()
+    out = {"Y": Y[:rows].cpu().numpy().astype(np.float64)}
+    if nvfp4:
+        codes, atoms, _ = lin.act_views_nvfp4(M)
+        p = codes[:rows].cpu().numpy()
+        q = np.empty((rows, p.shape[1] * 2), np.uint8)
+        q[:, 0::2], q[:, 1::2] = p & 0xF, p >> 4
+        a = atoms.cpu().numpy()
+        K = q.shape[1]
+        rr = np.arange(rows)[:, None]
+        b = np.arange(K // 16)[None, :]
+        out["qx"] = q
+        out["sfx"] = a[((rr // 128) * (K // 64) + b // 4) * 512 + (rr % 32) * 16 + ((rr % 128) // 32) * 4 + b % 4]
+    else:
+        codes, scales, _ = lin.act_views(M)
+        w = np.ascontiguousarray(codes[:rows].cpu().numpy()).view("<u4").astype(np.uint64)
+        lo = (w & 0x87878787).astype(np.uint32)
+        hi = (((w >> 4) | (w << 28)) & 0x87878787).astype(np.uint32)
+        by = np.empty((rows, w.shape[1], 8), np.uint8)
+        by[:, :, :4] = lo[:, :, None].view(np.uint8).reshape(rows, -1, 4)
+        by[:, :, 4:] = hi[:, :, None].view(np.uint8).reshape(rows, -1, 4)
+        mag = (by & 7).astype(np.int8)
+        out["qx"] = np.where(by & 0x80, -mag, mag).astype(np.int8).reshape(rows, -1)
+        out["sx"] = scales.cpu().numpy()[:, :rows].T.copy()
+    return out
 
 
 def lin_ws_bytes(lin, M):
