@@ -17,7 +17,8 @@ points run the pack and the activation path on those float64 values, and ``forwa
 
 Every function returns semantic arrays in the paper's row-major notation:
 X [M,K] tokens, W [K,N], U [K,r] (the paper's V), codes as int8 in [-7, 7], activation scales
-float32 [M, K/G], weight scales float16 [K/G, N], branch factors float16.
+[M, K/G] (bfloat16 values held in float32), weight scales bfloat16 bits [K/G, N], branch factors
+float16.
 """
 from __future__ import annotations
 
@@ -68,6 +69,8 @@ def _load():
             lib.qo_f16_value.restype = ctypes.c_double
             lib.qo_nearest_code.argtypes = [ctypes.c_double, ctypes.c_double]
             lib.qo_nearest_code.restype = ctypes.c_int
+            lib.qo_bf16_bits_div7_rn.argtypes = [ctypes.c_double]
+            lib.qo_bf16_bits_div7_rn.restype = ctypes.c_uint16
             lib.qo_pack_nvfp4.argtypes = [P, P, I, I, I, P, P, P, P]
             lib.qo_quantize_act_nvfp4.argtypes = [P, P, I, I, I, P, P, P]
             lib.qo_pack_nvfp4_f64.argtypes = [P, P, I, I, I, P, P, P, P]
@@ -110,7 +113,7 @@ def pack(W_bf16_bits, U, G, want_float64=False):
     """Offline packing (Sec. 4.2 Eq. (asp) and the W_perp derivation; Eq. (quant) on weights).
 
     W_bf16_bits: uint16 [K,N]; U: float32 [K,r] (r may be 0).
-    Returns dict(qw int8 [N,K], sw uint16 fp16-bits [K/G,N], Bh uint16 fp16-bits [r,N],
+    Returns dict(qw int8 [N,K], sw uint16 bf16-bits [K/G,N], Bh uint16 fp16-bits [r,N],
     and Bf / Wperp float64 when want_float64)."""
     W = _c(W_bf16_bits, np.uint16)
     K, N = W.shape
@@ -132,7 +135,7 @@ def pack(W_bf16_bits, U, G, want_float64=False):
 def quantize_act(X_bf16_bits, U, G, want_float64=False):
     """Run-time activation path (Eq. (xsplit), then Eq. (quant) per token and group).
 
-    Returns dict(qx int8 [M,K], sx float32 [M,K/G], ph uint16 fp16-bits [M,r],
+    Returns dict(qx int8 [M,K], sx float32 [M,K/G] (bfloat16 values), ph uint16 fp16-bits [M,r],
     and p / Xperp float64 when want_float64)."""
     X = _c(X_bf16_bits, np.uint16)
     M, K = X.shape
@@ -286,6 +289,11 @@ def f16_value(h: int) -> float:
 
 def nearest_code(x: float, s: float) -> int:
     return int(_load().qo_nearest_code(float(x), float(s)))
+
+
+def bf16_bits_div7(a: float) -> int:
+    """bfloat16 bits of RN_bf16(a / 7) for the exact quotient (readings R3, R4), a >= 0."""
+    return int(_load().qo_bf16_bits_div7_rn(float(a)))
 
 
 # ---- NVFP4 variant (App. B.1) ----------------------------------------------------------------

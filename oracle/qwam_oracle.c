@@ -31,12 +31,14 @@
  * Readings of points the paper leaves open (each is one line of the design notes):
  *   R1  format: INT4 codes in [-7, 7] (absmax/7 never produces -8), group G along K.
  *   R2  round to nearest = nearest integer to the EXACT quotient x/s, ties to even.
- *   R3  activation scale: float32, s_x = RN_f32(amax / 7) of the group's absmax.
- *   R4  weight scale: float16, s_w = RN_f16(amax / 7) computed from the float64 absmax.
+ *   R3  activation scale: bfloat16, s_x = RN_bf16(amax / 7) of the group's absmax, one rounding
+ *       of the exact quotient (ties to even).
+ *   R4  weight scale: bfloat16 (the 16-bit scale of Table 3), s_w = RN_bf16(amax / 7) of the
+ *       float64 absmax, one rounding of the exact quotient.
  *   R5  codes are taken against the stored (rounded) scale; a zero scale gives zero codes.
  *   R6  the "16-bit" branch is float16: p_hat = RN_f16(x U), B_hat = RN_f16(U^T W).
  *   R7  the branch uses float64 B_f = U^T W for the deflation, B_hat only for the output.
- *   R11 on float64 activations (the rotated x~) the scale is RN_f32(RN_f64(amax / 7)).
+ *   R11 on float64 activations (the rotated x~) the scale follows R3 on the float64 absmax.
  */
 #include <math.h>
 #include <stdint.h>
@@ -92,11 +94,46 @@ static uint16_t f16_bits_rn(double x) {
   return sign | (uint16_t)(((E + 15) << 10) | ((int)q - 1024));
 }
 
+/* bfloat16 bits of RN_bf16(a / 7) for the exact quotient of a finite a >= 0, ties to even
+ * (readings R3 and R4).  q = fl64(a / 7) lies within half a float64 unit of a / 7, so when q is
+ * itself a bfloat16 value it is the answer; otherwise the two bfloat16 values around q are
+ * n u and (n + 1) u, u the quantum of q's binade (8 significant bits; the subnormal binade of
+ * bfloat16 below 2^-126 has u = 2^-133), and comparing a with 7 (n + 1/2) u -- a product of at
+ * most 12 significant bits, exact in float64 -- decides between them. */
+static uint16_t bf16_bits_div7_rn(double a) {
+  if (!(a > 0.0)) return 0;
+  const double q = a / 7.0;
+  int e2;
+  frexp(q, &e2);
+  int E = e2 - 1; /* q in [2^E, 2^(E+1)) */
+  if (E < -126) E = -126;
+  const double u = ldexp(1.0, E - 7);
+  const double n = floor(q / u); /* q / u is a power-of-two scaling: exact */
+  double v;
+  if (n * u == q) {
+    v = q;
+  } else {
+    const double t = 7.0 * ((n + 0.5) * u);
+    if (a > t)
+      v = (n + 1.0) * u;
+    else if (a < t)
+      v = n * u;
+    else
+      v = (fmod(n, 2.0) == 0.0) ? n * u : (n + 1.0) * u;
+  }
+  if (v > 3.3895313892515355e38) return 0x7f80; /* above the largest bfloat16: infinity */
+  /* v lies on the bfloat16 grid, hence on the float32 grid: the upper half of its float32 bits */
+  const float f = (float)v;
+  uint32_t b;
+  memcpy(&b, &f, sizeof b);
+  return (uint16_t)(b >> 16);
+}
+
 /* ---- the quantizer of Eq. (quant) ------------------------------------------------------ */
 
 /* Nearest integer to the exact quotient x/s, ties to even (reading R2); s > 0.
  * c = nearbyint(fl(x/s)) is within one of the answer.  For the operand formats used here
- * (x in float32 or float64, s in float32 or float16, |x| <= ~7.5 s) both c*s and x - c*s are
+ * (x in float32 or float64, s in bfloat16, float32 or float16, |x| <= ~7.5 s) both c*s and x - c*s are
  * exact in float64, so the remainder e decides the rounding exactly. */
 static int nearest_code(double x, double s) {
   double c = nearbyint(x / s);
@@ -112,7 +149,7 @@ static int nearest_code(double x, double s) {
 /* ---- offline packing: Eq. (asp), W_perp derivation, Eq. (quant) on weights ------------- */
 
 /* W_bf16 [K,N] bf16 bits; U [K,r] float32 (orthonormal columns; ignored when r == 0).
- * Outputs: qw [N,K] int8 codes, sw [K/G,N] float16 bits, Bh [r,N] float16 bits,
+ * Outputs: qw [N,K] int8 codes, sw [K/G,N] bfloat16 bits, Bh [r,N] float16 bits,
  *          Bf [r,N] float64 (optional), Wperp [K,N] float64 (optional). */
 static int pack_core(const double* W, const float* U, int K, int N, int r, int G, int8_t* qw, uint16_t* sw,
                      uint16_t* Bh, double* Bf_out, double* Wperp_out) {
@@ -141,7 +178,7 @@ static int pack_core(const double* W, const float* U, int K, int N, int r, int G
       for (int j = 0; j < r; ++j) acc += (double)U[(size_t)k * r + j] * Bf[(size_t)j * N + n];
       Wp[(size_t)k * N + n] = W[(size_t)k * N + n] - acc;
     }
-  /* Per output channel n and group g of G consecutive inputs: s_w = RN_f16(amax/7), codes. */
+  /* Per output channel n and group g of G consecutive inputs: s_w = RN_bf16(amax/7), codes. */
   int ng = K / G;
 #pragma omp parallel for schedule(static) reduction(min : status)
   for (int n = 0; n < N; ++n)
@@ -151,8 +188,8 @@ static int pack_core(const double* W, const float* U, int K, int N, int r, int G
         double a = fabs(Wp[(size_t)k * N + n]);
         if (a > amax) amax = a;
       }
-      uint16_t sbits = f16_bits_rn(amax / 7.0);
-      double s = f16_value(sbits);
+      uint16_t sbits = bf16_bits_div7_rn(amax);
+      double s = bf16_value(sbits);
       if (isinf(s)) status = QO_ERANGE;
       sw[(size_t)g * N + n] = sbits;
       for (int k = g * G; k < (g + 1) * G; ++k) {
@@ -192,7 +229,8 @@ int qo_pack_f64(const double* W, const float* U, int K, int N, int r, int G, int
 /* ---- run-time activation path: Eq. (xsplit), then Eq. (quant) per token and group ------- */
 
 /* X_bf16 [M,K] bf16 bits; U [K,r] float32.
- * Outputs: qx [M,K] int8 codes, sx [M,K/G] float32 scales, ph [M,r] float16 bits,
+ * Outputs: qx [M,K] int8 codes, sx [M,K/G] scales (bfloat16 values, held in float32),
+ *          ph [M,r] float16 bits,
  *          p [M,r] float64 (optional), Xperp [M,K] float64 (optional). */
 static int quantize_act_core(const uint16_t* X_bf16, const double* X_f64, const float* U, int M, int K, int r,
                              int G, int8_t* qx, float* sx, uint16_t* ph, double* p_out, double* Xperp_out) {
@@ -228,10 +266,11 @@ static int quantize_act_core(const uint16_t* X_bf16, const double* X_f64, const 
         double amax = 0.0;
         for (int k = g * G; k < (g + 1) * G; ++k)
           if (fabs(x[k]) > amax) amax = fabs(x[k]);
-        float s = (float)(amax / 7.0);
+        float s = (float)bf16_value(bf16_bits_div7_rn(amax));
+        if (isinf(s)) status = QO_ERANGE;
         sx[(size_t)m * ng + g] = s;
         for (int k = g * G; k < (g + 1) * G; ++k) {
-          int c = (s > 0.0f) ? nearest_code(x[k], (double)s) : 0;
+          int c = (s > 0.0f && !isinf(s)) ? nearest_code(x[k], (double)s) : 0;
           if (c < -7 || c > 7) status = QO_ERANGE;
           qx[(size_t)m * K + k] = (int8_t)c;
         }
@@ -288,9 +327,8 @@ int qo_block_fwht(double* data, int count, int n, long vstride, long estride, co
   return QO_OK;
 }
 
-/* The quantizer alone, applied to a given float32 remainder R [M,K] (reading R3 with an exact
- * float32 input: RN_f32(amax/7) through float64 is exact rounding of the true quotient because
- * 53 >= 2*24 + 2).  Outputs q [M,K] int8 and s [M,K/G] float32. */
+/* The quantizer alone, applied to a given float32 remainder R [M,K] (reading R3 on the float32
+ * absmax).  Outputs q [M,K] int8 and s [M,K/G] (bfloat16 values, held in float32). */
 int qo_quantize_residual_f32(const float* R, int M, int K, int G, int8_t* q, float* s_out) {
   if (M < 0 || K <= 0 || G <= 0 || K % G) return QO_EINVAL;
   int status = QO_OK;
@@ -303,10 +341,11 @@ int qo_quantize_residual_f32(const float* R, int M, int K, int G, int8_t* q, flo
         float a = fabsf(R[(size_t)m * K + k]);
         if (a > amax) amax = a;
       }
-      float s = (float)((double)amax / 7.0);
+      float s = (float)bf16_value(bf16_bits_div7_rn((double)amax));
+      if (isinf(s)) status = QO_ERANGE;
       s_out[(size_t)m * ng + g] = s;
       for (int k = g * G; k < (g + 1) * G; ++k) {
-        int c = (s > 0.0f) ? nearest_code((double)R[(size_t)m * K + k], (double)s) : 0;
+        int c = (s > 0.0f && !isinf(s)) ? nearest_code((double)R[(size_t)m * K + k], (double)s) : 0;
         if (c < -7 || c > 7) status = QO_ERANGE;
         q[(size_t)m * K + k] = (int8_t)c;
       }
@@ -318,7 +357,7 @@ int qo_quantize_residual_f32(const float* R, int M, int K, int G, int8_t* q, flo
 
 /* Y[m,n] = sum_g s_x[m,g] s_w[g,n] P_g[m,n]  +  sum_j p_hat[m,j] B_hat[j,n],
  * P_g[m,n] = sum_{k in group g} qx[m,k] qw[n,k]  (exact int64).
- * Each group term s_x * s_w * P_g has at most 24 + 11 + 13 significant bits, so it is exact in
+ * Each group term s_x * s_w * P_g has at most 8 + 8 + 13 significant bits, so it is exact in
  * float64; only the sum over groups and branch terms rounds. */
 int qo_linear(const int8_t* qx, const float* sx, const uint16_t* ph, const int8_t* qw,
               const uint16_t* sw, const uint16_t* Bh, int M, int K, int N, int r, int G, double* Y) {
@@ -331,7 +370,7 @@ int qo_linear(const int8_t* qx, const float* sx, const uint16_t* ph, const int8_
     free(bhv);
     return QO_EINVAL;
   }
-  for (size_t i = 0; i < (size_t)ng * N; ++i) swv[i] = f16_value(sw[i]);
+  for (size_t i = 0; i < (size_t)ng * N; ++i) swv[i] = bf16_value(sw[i]);
   for (size_t i = 0; i < (size_t)r * N; ++i) bhv[i] = f16_value(Bh[i]);
 #pragma omp parallel for schedule(dynamic, 4)
   for (int m = 0; m < M; ++m)
@@ -372,6 +411,7 @@ int qo_linear_split_exact(const double* p, const double* Xperp, const double* Bf
 uint16_t qo_f16_bits_rn(double x) { return f16_bits_rn(x); }
 double qo_f16_value(uint16_t h) { return f16_value(h); }
 int qo_nearest_code(double x, double s) { return nearest_code(x, s); }
+uint16_t qo_bf16_bits_div7_rn(double a) { return bf16_bits_div7_rn(a); }
 
 /* ==== NVFP4 variant (App. B.1: on Blackwell GPUs the paper stores E2M1 values with an E4M3
  * scale per group of 16 elements, for weights and activations, and one extra float32 scale per

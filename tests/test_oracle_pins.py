@@ -4,7 +4,8 @@ Each pin is independent of the oracle's own code:
   * exact rational arithmetic (fractions.Fraction) of the whole layer on tiny shapes,
   * brute-force argmin over the code grid for the quantizer (Eq. (quant)),
   * hand-derived closed-form group cases (tests/golden/quant_cases.txt),
-  * library conversions (numpy float16) for the 16-bit format,
+  * library conversions (numpy float16) for the float16 format and exact rational rounding for
+    the bfloat16 scales,
   * invariants of Sec. 4.2: x = U(U^T x) + x_perp, U^T W_perp = 0, x_perp U = 0, Eq. (asp) with
     Q = identity equals X W, r = 0 is plain per-group W4A4, r = K leaves a zero remainder,
   * storage of Table 3 (4.50 bits per weight at group 32) and the isotropy share r/K of App. C.
@@ -54,12 +55,12 @@ def rn_binary(fr: Fraction, mant: int, emin: int) -> Fraction:
     return sgn * n * quantum
 
 
-def rn_f32(fr):
-    return rn_binary(fr, 24, -126)
-
-
 def rn_f16(fr):
     return rn_binary(fr, 11, -14)
+
+
+def rn_bf16(fr):
+    return rn_binary(fr, 8, -126)
 
 
 def brute_code(x: Fraction, s: Fraction) -> int:
@@ -101,6 +102,30 @@ def test_f16_rounding_matches_numpy():
         assert oracle.f16_value(h) == float(np.array([h], np.uint16).view(np.float16)[0])
 
 
+def test_bf16_scale_rounding_is_exact_rounding_of_the_quotient():
+    """Readings R3 and R4: s = RN_bf16(a / 7), one rounding of the exact quotient, against exact
+    rational rounding -- including float32 subnormal absmaxes, where rounding the quotient to
+    float32 first can land on a bfloat16 midpoint that the exact quotient is not on."""
+    g = np.random.default_rng(17)
+    vals = list(np.abs(g.standard_normal(4000) * 10.0 ** g.integers(-30, 30, 4000)).astype(np.float32))
+    vals += list((g.integers(1, 2 ** 23, 2000) * 2.0 ** -149).astype(np.float32))  # float32 subnormals
+    # 7 times every bfloat16 midpoint of a few binades, and its float32 neighbours
+    for e in (-133, -130, -10, 0, 5, 100):
+        for n in range(0, 256, 7):
+            t = np.float32(7 * (2 * n + 1) * 2.0 ** (e - 1))
+            vals += [t, np.nextafter(t, np.float32(0)), np.nextafter(t, np.float32(np.inf))]
+    vals += [np.float32(1146881 * 2.0 ** -149), np.float32(7.0), np.float32(1.0), np.float32(0.0)]
+    for a in vals:
+        a = float(a)
+        want = rn_bf16(Fraction(a) / 7)
+        got = bf16_frac(oracle.bf16_bits_div7(a))
+        assert got == want, a
+    # the float32-first double rounding differs on this subnormal absmax (the golden file has it)
+    a = 1146881 * 2.0 ** -149
+    assert float(np.float32(a / 7)) == 5 * 2.0 ** -134   # RN_f32 lands on a bfloat16 midpoint
+    assert oracle.bf16_bits_div7(a) == 0x0003            # the exact quotient is above it
+
+
 # ---------------------------------------------------------------- quantizer (Eq. (quant))
 
 def _golden_cases():
@@ -110,7 +135,8 @@ def _golden_cases():
         if not line or line.startswith("#"):
             continue
         kind, vals, sbits, codes = [t.strip() for t in line.split("|")]
-        cases.append((kind, [float(v) for v in vals.split(",")], int(sbits, 16),
+        num = [float.fromhex(v) if "p" in v else float(v) for v in vals.split(",")]
+        cases.append((kind, num, int(sbits, 16),
                       [int(c) for c in codes.split(",")]))
     return cases
 
@@ -120,8 +146,11 @@ def test_golden_group_cases(case):
     kind, vals, sbits, codes = case
     G = len(vals)
     if kind == "act":
-        q, s = oracle.quantize_residual(np.array([vals], np.float32), G)
-        assert f32_bits(float(s[0, 0])) == sbits
+        R = np.array([vals], np.float32)
+        assert R[0].tolist() == vals  # every value is exact in float32
+        q, s = oracle.quantize_residual(R, G)
+        b = f32_bits(float(s[0, 0]))
+        assert b & 0xFFFF == 0 and b >> 16 == sbits  # a bfloat16 value
         assert q[0].tolist() == codes
     else:
         # weight path: one output channel, K = G, r = 0, W holds the values exactly in bf16
@@ -159,7 +188,7 @@ def test_quantize_residual_bruteforce_and_error_bound():
             for gi in range(128 // G):
                 grp = [Fraction(float(v)) for v in R[m, gi * G:(gi + 1) * G]]
                 amax = max(abs(v) for v in grp)
-                s_exact = rn_f32(amax / 7)
+                s_exact = rn_bf16(amax / 7)
                 assert Fraction(float(s[m, gi])) == s_exact
                 for k, v in enumerate(grp):
                     c = brute_code(v, s_exact)
@@ -188,14 +217,14 @@ def _exact_layer_values(X, W, U, G):
     Bf = [[sum(Uf[k][j] * W[k][n] for k in range(K)) for n in range(N)] for j in range(r)]
     Wp = [[W[k][n] - sum(Uf[k][j] * Bf[j][n] for j in range(r)) for n in range(N)] for k in range(K)]
     ng = K // G
-    sw = [[rn_f16(max(abs(Wp[k][n]) for k in range(g * G, (g + 1) * G)) / 7) for n in range(N)]
+    sw = [[rn_bf16(max(abs(Wp[k][n]) for k in range(g * G, (g + 1) * G)) / 7) for n in range(N)]
           for g in range(ng)]
     qw = [[brute_code(Wp[k][n], sw[k // G][n]) for k in range(K)] for n in range(N)]
     Bh = [[rn_f16(Bf[j][n]) for n in range(N)] for j in range(r)]
     # activations
     p = [[sum(X[m][k] * Uf[k][j] for k in range(K)) for j in range(r)] for m in range(M)]
     Xp = [[X[m][k] - sum(p[m][j] * Uf[k][j] for j in range(r)) for k in range(K)] for m in range(M)]
-    sx = [[rn_f32(max(abs(Xp[m][k]) for k in range(g * G, (g + 1) * G)) / 7) for g in range(ng)]
+    sx = [[rn_bf16(max(abs(Xp[m][k]) for k in range(g * G, (g + 1) * G)) / 7) for g in range(ng)]
           for m in range(M)]
     qx = [[brute_code(Xp[m][k], sx[m][k // G]) for k in range(K)] for m in range(M)]
     ph = [[rn_f16(p[m][j]) for j in range(r)] for m in range(M)]
@@ -217,7 +246,7 @@ def test_layer_matches_exact_rational_arithmetic(r, G):
     a = oracle.quantize_act(Xb, U, G)
     Y = oracle.linear(a, w, G)
     assert w["qw"].tolist() == ex["qw"]
-    assert [[f16_frac(b) for b in row] for row in w["sw"]] == ex["sw"]
+    assert [[bf16_frac(b) for b in row] for row in w["sw"]] == ex["sw"]
     assert [[f16_frac(b) for b in row] for row in w["Bh"]] == ex["Bh"]
     assert a["qx"].tolist() == ex["qx"]
     assert [[Fraction(float(v)) for v in row] for row in a["sx"]] == ex["sx"]
@@ -272,16 +301,15 @@ def test_r0_is_plain_per_group_w4a4():
     # independent numpy statement of per-group W4A4 (Eq. (quant) on both operands)
     X = wl.bf16_bits_to_f32(Xb).reshape(M, K // G, G)
     amax = np.abs(X).max(axis=2)
-    sx = (amax.astype(np.float64) / 7.0).astype(np.float32)   # exact rounding: 53 >= 2*24+2
+    sx = np.array([[float(rn_bf16(Fraction(float(a)) / 7)) for a in row] for row in amax], np.float32)
     with np.errstate(invalid="ignore", divide="ignore"):
         qx = np.where(sx[..., None] > 0, np.rint(X / sx[..., None].astype(np.float64)), 0).astype(np.int64)
     np.testing.assert_array_equal(a["sx"], sx)
     np.testing.assert_array_equal(a["qx"], qx.reshape(M, K))
     Wt = wl.bf16_bits_to_f32(Wb).astype(np.float64).T.reshape(N, K // G, G)
-    swv = np.abs(Wt).max(axis=2) / 7.0
-    sw_bits = swv.astype(np.float16).view(np.uint16)
+    swf = np.array([[float(rn_bf16(Fraction(float(a)) / 7)) for a in row] for row in np.abs(Wt).max(axis=2)])
+    sw_bits = (swf.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
     np.testing.assert_array_equal(w["sw"], sw_bits.T)
-    swf = sw_bits.view(np.float16).astype(np.float64)
     with np.errstate(invalid="ignore", divide="ignore"):
         qw = np.where(swf[..., None] > 0, np.rint(Wt / swf[..., None]), 0).astype(np.int64)
     np.testing.assert_array_equal(w["qw"], qw.reshape(N, K))
@@ -401,7 +429,7 @@ def test_rotated_layer_matches_exact_rational_arithmetic(r):
     ex = _exact_layer_values([[Fraction(float(v)) for v in row] for row in Xt],
                              [[Fraction(float(v)) for v in row] for row in Wt], U, G)
     assert w["qw"].tolist() == ex["qw"]
-    assert [[f16_frac(b) for b in row] for row in w["sw"]] == ex["sw"]
+    assert [[bf16_frac(b) for b in row] for row in w["sw"]] == ex["sw"]
     assert [[f16_frac(b) for b in row] for row in w["Bh"]] == ex["Bh"]
     assert a["qx"].tolist() == ex["qx"]
     assert [[Fraction(float(v)) for v in row] for row in a["sx"]] == ex["sx"]
