@@ -35,7 +35,10 @@
  *       of the exact quotient (ties to even).
  *   R4  weight scale: bfloat16 (the 16-bit scale of Table 3), s_w = RN_bf16(amax / 7) of the
  *       float64 absmax, one rounding of the exact quotient.
- *   R5  codes are taken against the stored (rounded) scale; a zero scale gives zero codes.
+ *   R5  codes are taken against the stored (rounded) scale; a zero scale gives zero codes; the
+ *       code is the nearest one in [-7, 7] (it saturates), which differs from the nearest
+ *       integer only for bfloat16-subnormal scales (below 2^-126), where rounding amax / 7 to
+ *       few significant bits can leave amax / s above 7.5.
  *   R6  the "16-bit" branch is float16: p_hat = RN_f16(x U), B_hat = RN_f16(U^T W).
  *   R7  the branch uses float64 B_f = U^T W for the deflation, B_hat only for the output.
  *   R11 on float64 activations (the rotated x~) the scale follows R3 on the float64 absmax.
@@ -131,7 +134,7 @@ static uint16_t bf16_bits_div7_rn(double a) {
 
 /* ---- the quantizer of Eq. (quant) ------------------------------------------------------ */
 
-/* Nearest integer to the exact quotient x/s, ties to even (reading R2); s > 0.
+/* Nearest code in [-7, 7] to the exact quotient x/s, ties to even (readings R2, R5); s > 0.
  * c = nearbyint(fl(x/s)) is within one of the answer.  For the operand formats used here
  * (x in float32 or float64, s in bfloat16, float32 or float16, |x| <= ~7.5 s) both c*s and x - c*s are
  * exact in float64, so the remainder e decides the rounding exactly. */
@@ -143,6 +146,8 @@ static int nearest_code(double x, double s) {
     c += (e > 0.0) ? 1.0 : -1.0;
   else if (t == s && fmod(c, 2.0) != 0.0)
     c += (e > 0.0) ? 1.0 : -1.0;
+  if (c > 7.0) c = 7.0;
+  if (c < -7.0) c = -7.0;
   return (int)c;
 }
 
