@@ -13,9 +13,10 @@
  * with B_hat = RN_f16(U^T W), p_hat = RN_f16(p), and Q4 the symmetric group quantizer of
  * Eq. (quant) (Sec. 3) with b = 4: scale s = absmax / 7 per group of `group` consecutive input
  * channels (App. B.1), codes = nearest integer to x / s (exact quotient, ties to even), so codes
- * lie in [-7, 7].  Activation scales are float32, weight scales float16 (Table 3: 4.50 bits per
- * weight at group 32 implies a 16-bit weight scale).  r = 0 gives plain per-group W4A4 (experts
- * that ASP does not select, Sec. 4.3).
+ * lie in [-7, 7].  Both scales are bfloat16, s = RN_bf16(absmax / 7) rounded once from the exact
+ * quotient (Table 3: 4.50 bits per weight at group 32 implies a 16-bit weight scale; the paper
+ * leaves the activation scale's format open).  r = 0 gives plain per-group W4A4 (experts that
+ * ASP does not select, Sec. 4.3).
  *
  * Conventions for every entry point:
  *   - Pointers marked "device" are CUDA device pointers on the current device; "host" pointers
@@ -68,9 +69,10 @@ enum { QWAM_Y_BF16 = 0, QWAM_Y_FP32 = 1 };
  *   group  : quantization group along K, 32 or 64
  *   out    : receives the new handle
  * Computes, in float64 on the device: B_f = U^T W, W_perp = W - U B_f, per (output channel,
- * group) s_w = RN_f16(absmax / 7) and the codes of W_perp / s_w, B_hat = RN_f16(B_f), and the
- * bf16 hi/lo split of U used by the activation kernel.  Synchronizes `stream` before returning.
- * Returns QWAM_ERR_RANGE if a weight scale or a branch value overflows float16. */
+ * group) s_w = RN_bf16(absmax / 7) and the codes of W_perp / s_w, B_hat = RN_f16(B_f), the
+ * bf16 hi/lo split of U used by the activation kernel, and the GEMM's float16 copies of s_w and
+ * B_hat scaled by a power of two per output column.  Synchronizes `stream` before returning.
+ * Returns QWAM_ERR_RANGE if a weight scale or a branch value overflows its 16-bit format. */
 qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int N, int r, int group,
                                   struct CUstream_st* stream, qwam_asp_handle* out);
 
@@ -78,14 +80,12 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
 qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes);
 
 /* Layout of the activation workspace for M tokens (byte offsets from its start):
- *   codes  : uint8 [M, K/2], the activation codes c in [-7, 7] packed at four bits as SM4 words:
- *            the little-endian 32-bit word j of a row holds k = 8j .. 8j+7.  Byte i of the word
- *            carries code 8j+i in its sign bit 7 and magnitude bits 0-2, the magnitude of code
- *            8j+4+i in bits 4-6, and in bit 3 the sign of code 8j+4+((i+3) mod 4).  With lo and
- *            hi the words of E4M3 bytes (c < 0 ? 0x80 : 0) | |c| of k = 8j..8j+3 and 8j+4..8j+7,
- *            word = lo | rotl(hi, 4), and back lo = word & 0x87878787, hi = rotr(word, 4) &
- *            0x87878787 (the GEMM expands the words this way, with one funnel shift and two masks)
- *   scales : float32 [K/group, M_pad] (M_pad = M rounded up to 128), s_x of token m, group g
+ *   codes  : uint8 [M, K/2], the activation codes c in [-7, 7] packed at four bits as OB4 words:
+ *            the little-endian 32-bit word j of a row holds k = 8j .. 8j+7 as offset-binary
+ *            nibbles c + 8, code 8j + 2p in bits 4p .. 4p+3 and code 8j + 2p + 1 in bits
+ *            16 + 4p .. 16 + 4p + 3 (p = 0..3).  (The GEMM turns pair p into two float16 values
+ *            with one shift, one and-or under the float16 pattern of 1024 and one subtraction.)
+ *   scales : bfloat16 [K/group, M_pad] (M_pad = M rounded up to 128), s_x of token m, group g
  *            at [g * M_pad + m]
  *   ab     : no region (ab_off == phat_off); kept in the call for the layout's stability
  *   p_hat  : float16 [M, r_pad] (r_pad = r rounded up to 16; columns >= r are zero)
@@ -97,7 +97,7 @@ qwam_status qwam_asp_act_layout(qwam_asp_handle h, int M, size_t* codes_off, siz
 /* Kernel (a): Eq. (xsplit) and the run-time half of Eq. (quant), one launch, asynchronous.
  *   X_bf16 : device, bf16 [M, K] row-major;  act_ws : device workspace (see above), written
  * Reads X once from HBM, forms p = X U on tensor cores (bf16 hi/lo split of U, float32
- * accumulation), X_perp = X - p U^T in float32, and writes the packed codes, float32 scales and
+ * accumulation), X_perp = X - p U^T in float32, and writes the packed codes, bfloat16 scales and
  * p_hat. */
 qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws,
                                   struct CUstream_st* stream);
@@ -105,12 +105,13 @@ qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, 
 /* Kernel (b): the 4-bit GEMM with the low-rank branch in its epilogue, asynchronous.
  *   act_ws : device workspace filled by qwam_asp_quantize_act for the same M
  *   Y      : device [M, N] row-major, bf16 (y_dtype QWAM_Y_BF16) or float32 (QWAM_Y_FP32)
- * Both operands stay packed at four bits in HBM and are expanded to E4M3 bytes of c * 2^-9 in
- * shared memory.  Per group g the tensor cores form the exact integer partial sums
- * D = 2^-18 P_g, P_g = sum_k qx qw (E4M3 holds the codes exactly; float32 accumulation of these
- * integer multiples of 2^-18 below 2^-5 is exact), and the epilogue adds (D s_x[m,g]) sigma[g,n]
- * in float32, sigma = 2^18 s_w (= s_w[g,n] s_x[m,g] P_g with two roundings), and, last, the
- * branch p_hat B_hat (float16 operands, float32 accumulation; any r_pad). */
+ * Both operands stay packed at four bits in HBM.  With bfloat16 scales every dequantized value
+ * s c has at most 11 significant bits, so the kernel forms s_x c and s_w c in float16 (exactly,
+ * after a power-of-two scaling per token row and per output column that keeps them in float16's
+ * range and is undone in the epilogue) and the tensor cores contract [s_x q_x | p_hat] with
+ * [s_w q_w | B_hat] over K + r_pad in one float32 accumulator (tcgen05.mma kind::f16): the
+ * group scales and the 16-bit branch need no separate pass.  The result differs from the exact
+ * sum of Eq. (asp) only by the float32 accumulation. */
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle h, void* Y, int y_dtype,
                           struct CUstream_st* stream);
 
@@ -131,8 +132,8 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
  *
  *   - Size limit: the workspace qwam_asp_act_workspace_bytes(h, M) reports must fit in
  *     QWAM_STATIC_WS_BYTES (24 MiB); larger requests return QWAM_ERR_TOO_LARGE before anything
- *     is launched.  Per token the workspace holds about K/2 + 4K/G + 2 r_pad bytes (INT4) or
- *     K/2 + K/16 + 2 r_pad bytes (NVFP4): at K = 3072, group 64, r = 32 about 1.8 KB, so up to
+ *     is launched.  Per token the workspace holds about K/2 + 2K/G + 2 r_pad bytes (INT4) or
+ *     K/2 + K/16 + 2 r_pad bytes (NVFP4): at K = 3072, group 64, r = 32 about 1.7 KB, so up to
  *     about 14,000 tokens fit.  A rotated handle with r > 0 also keeps its float32 remainder,
  *     4K more bytes per token: at K = 3072 about 1,780 tokens fit, and M = 4096 is refused.
  *   - Nothing in the scratch needs to start at zero: kernel (a) writes every byte the GEMM
@@ -246,7 +247,7 @@ qwam_status qwam_asp_shape(qwam_asp_handle h, int* K, int* N, int* r, int* group
 
 /* Copy the packed weights to HOST buffers (any may be NULL), synchronously:
  *   qw  : uint8 [N, K/2] codes of W_perp, low nibble = even k (two's complement)
- *   sw  : uint16 (float16 bits) [K/group, N]
+ *   sw  : uint16 (bfloat16 bits) [K/group, N]
  *   Bh  : uint16 (float16 bits) [N, r_pad]   (B_hat transposed, zero beyond r)
  *   Uhl : uint16 (bf16 bits) [2, K, r_pad]   (hi and lo parts of the projection basis: U, or
  *         diag(s)^-1 H U for a rotated handle; zero beyond r; all zero for r > 64, whose
@@ -280,9 +281,9 @@ qwam_status qwam_asp_debug_residual(const void* X_bf16, int M, qwam_asp_handle h
  *   R      : device float32 [M, K], row-major, 16-byte aligned; K % 64 == 0
  *   fmt    : QWAM_FMT_INT4 or QWAM_FMT_NVFP4
  *   group  : 32 or 64 for INT4 (ignored for NVFP4, whose block is 16)
- *   codes  : device, 16-byte aligned.  INT4: uint8 [M, K/2], SM4 words as in the activation
+ *   codes  : device, 16-byte aligned.  INT4: uint8 [M, K/2], OB4 words as in the activation
  *            workspace.  NVFP4: uint8 [M, K/2], two E2M1 codes per byte, low nibble = even k.
- *   scales : device.  INT4: float32 [M, K/group] row-major (4-byte aligned).  NVFP4: uint8 E4M3
+ *   scales : device.  INT4: bfloat16 [M, K/group] row-major (2-byte aligned).  NVFP4: uint8 E4M3
  *            bit patterns [M, K/16] row-major.
  * Asynchronous on `stream`; QWAM_ERR_INVALID_ARG for bad sizes, formats or alignment. */
 qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, int group, void* codes,
@@ -292,7 +293,7 @@ qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, 
  * per lane, a group over neighbouring lanes) on caller-given float32 rows, with the same rounding
  * rules as qwam_asp_debug_quantize_rows; K % 256 == 0.  Outputs are written in the activation
  * workspace's layouts with M_pad = ceil(M / 128) * 128 rows:
- *   INT4:  codes uint8 [M, K/2] (SM4 words, described at qwam_asp_act_layout), scales float32
+ *   INT4:  codes uint8 [M, K/2] (OB4 words, described at qwam_asp_act_layout), scales bfloat16
  *          [K/group, M_pad];
  *   NVFP4: codes uint8 [M, K/2] (two per byte, low nibble = even k), scales uint8 E4M3 in the
  *          512-byte atoms described above (M_pad * K/16 bytes).

@@ -224,7 +224,7 @@ def qwam_asp_shape(h: int) -> dict:
 
 
 def qwam_asp_export(h: int):
-    """Packed weights on the host: qw uint8 [N, K/2], sw float16-bits [K/G, N],
+    """Packed weights on the host: qw uint8 [N, K/2], sw bfloat16-bits [K/G, N],
     Bh float16-bits [N, r_pad], Uhl bf16-bits [2, K, r_pad] (numpy arrays)."""
     import numpy as np
     sh = qwam_asp_shape(h)
@@ -362,8 +362,8 @@ class AspLinear:
         return self._ws
 
     def act_views(self, M: int, ws: torch.Tensor | None = None):
-        """Views of the workspace for M tokens: packed codes uint8 [M, K/2] (SM4 words: word j of a
-        row holds k = 8j..8j+7, see qwam_asp_act_layout), scales f32 [K/G, M_pad], p_hat f16
+        """Views of the workspace for M tokens: packed codes uint8 [M, K/2] (OB4 words: word j of a
+        row holds k = 8j..8j+7, see qwam_asp_act_layout), scales bf16 [K/G, M_pad], p_hat f16
         [M, r_pad]."""
         ws = self.workspace(M) if ws is None else ws
         L = qwam_asp_act_layout(self.h, M)
@@ -371,7 +371,7 @@ class AspLinear:
             return self.act_views_nvfp4(M, ws)
         codes = ws[L["codes_off"]:L["codes_off"] + M * (self.K // 2)].view(M, self.K // 2)
         ns = self.K // self.group
-        scales = ws[L["scales_off"]:L["scales_off"] + ns * L["M_pad"] * 4].view(torch.float32).view(ns, L["M_pad"])
+        scales = ws[L["scales_off"]:L["scales_off"] + ns * L["M_pad"] * 2].view(torch.bfloat16).view(ns, L["M_pad"])
         ph = ws[L["phat_off"]:L["phat_off"] + M * self.r_pad * 2].view(torch.float16).view(M, self.r_pad)
         return codes, scales, ph
 

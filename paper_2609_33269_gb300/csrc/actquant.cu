@@ -2,7 +2,7 @@
 //
 //   p      = X U                (Sec. 4.2 Eq. (xsplit): the protected coordinates V^T x)
 //   X_perp = X - p U^T          (the remainder (I - V V^T) x)
-//   s_x    = RN_f32(absmax(X_perp over a group) / 7),  codes = nearest(X_perp / s_x)
+//   s_x    = RN_bf16(absmax(X_perp over a group) / 7),  codes = nearest(X_perp / s_x)
 //                               (Eq. (quant) with b = 4; App. B.1: per token, per group)
 //   p_hat  = RN_f16(p)          (the 16-bit branch input of Eq. (asp))
 //
@@ -16,9 +16,9 @@
 // X_perp = X - R in float32 and quantize it.  With r = 0 the kernel is one streaming pass.
 //
 // Outputs per token row m and group g (the activation workspace):
-//   codes[m, :]   packed at four bits, SM4 words (sm4_pack: word j holds k = 8j..8j+7,
-//                 sign-magnitude), which the GEMM expands to E4M3 bytes of c * 2^-9;
-//   s_x[g, m]     float32 scale;
+//   codes[m, :]   packed at four bits, OB4 words (ob4_word: word j holds k = 8j..8j+7 as
+//                 offset-binary nibbles), which the GEMM expands to float16 values s_x c;
+//   s_x[g, m]     bfloat16 scale;
 //   p_hat[m, :]   float16.
 // NVFP4 variant (App. B.1, the same kernel with one template flag): per block of 16 K an E4M3
 // scale (in the 512-byte atoms the GEMM copies to tensor memory) and E2M1 codes, two per byte.
@@ -44,9 +44,9 @@ namespace {
 
 struct ActArgs {
   int M, K, G, C, Kc, M_pad;
-  uint8_t* codes;   // [M, K/2]: SM4 words (NVFP4: E2M1 codes, two per byte, low nibble = even k)
+  uint8_t* codes;   // [M, K/2]: OB4 words (NVFP4: E2M1 codes, two per byte, low nibble = even k)
   uint8_t* sf;      // NVFP4: E4M3 block scales in 512-byte atoms
-  float* scales;    // [K/G, M_pad]
+  __nv_bfloat16* scales;  // [K/G, M_pad]
   __half* phat;     // [M, RP]
   float* dump;      // optional [M, K]
   int resid_only;   // rotated layer: write the remainder to dump and stop (the rotation kernel quantizes)
@@ -76,11 +76,12 @@ struct ActCfg {
 constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23: adding it rounds to an integer (ties to even)
 constexpr int kMagicBits = 0x4B400000;
 
-// Nearest integer to the exact quotient x / s, ties to even (s > 0, |x| <= ~7.5 s).
-// c = rint(x * (1/s)) is the answer or its neighbour; the remainder e = x - c s is exact in
-// float32 (c and the true answer differ by at most one), and |e| < s/2 exactly when c is right
+// Nearest code in [-7, 7] to the exact quotient x / s, ties to even (s > 0, |x| <= amax).
+// c = rint(x * (1/s)) is the nearest integer or its neighbour; the remainder e = x - c s is exact
+// in float32 (c and the true answer differ by at most one), and |e| < s/2 exactly when c is right
 // and not a tie.  The correction is taken with selects rather than a branch: a branch per value
-// keeps the compiler from overlapping the 64 independent roundings of a group.
+// keeps the compiler from overlapping the 64 independent roundings of a group.  The result
+// saturates at -+7, which only a bfloat16-subnormal scale (few significant bits) can need.
 __device__ __forceinline__ int nearest_code(float x, float s, float inv, float hs) {
   const float t = fmaf(x, inv, kMagic);
   const float c = t - kMagic;
@@ -89,7 +90,7 @@ __device__ __forceinline__ int nearest_code(float x, float s, float inv, float h
   const float ae = fabsf(e);
   // |e| > s/2: the neighbour on e's side; |e| == s/2 (a tie): the even one of the two
   const int adj = static_cast<int>(ae > hs) | (static_cast<int>(ae == hs) & ci & 1);
-  return ci + (e > 0.0f ? adj : -adj);
+  return min(7, max(-7, ci + (e > 0.0f ? adj : -adj)));
 }
 // Approximate reciprocal (the hardware's single-instruction estimate).  It only seeds the
 // rounding in nearest_code, whose exact remainder test corrects a seed that is off by one.
@@ -99,10 +100,21 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return r;
 }
 
-// One group of GS remainder values -> scale and GS/8 SM4 words of codes.  The absmax is formed
+// s_x = RN_bf16(amax / 7) of the exact quotient, ties to even: the quotient rounded toward zero to
+// float32 with its last bit set when the division is inexact (round to odd; the remainder
+// amax - 7 q is exact), then rounded to the nearest bfloat16.  Rounding to odd first and to nearest
+// after is exact rounding because 24 >= 8 + 2.
+__device__ __forceinline__ float bf16_scale_div7(float amax) {
+  const float q = __fdiv_rz(amax, 7.0f);
+  const float rem = fmaf(-q, 7.0f, amax);
+  const float qo = __uint_as_float(__float_as_uint(q) | (rem != 0.0f ? 1u : 0u));
+  return __bfloat162float(__float2bfloat16_rn(qo));
+}
+
+// One group of GS remainder values -> scale and GS/8 OB4 words of codes.  The absmax is formed
 // as a tree (max is exact, so the order does not matter), which keeps the dependency chain short.
 template <int GS>
-__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words, float* scale_out) {
+__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words, __nv_bfloat16* scale_out) {
   float mx[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) mx[j] = fabsf(xp[j]);
@@ -113,7 +125,7 @@ __device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words,
 #pragma unroll
     for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
   const float amax = mx[0];
-  const float sc = __fdiv_rn(amax, 7.0f);
+  const float sc = bf16_scale_div7(amax);
   // Codes are invariant under a common power-of-two scaling of the values and the scale (exact
   // in float32), which keeps 1/s finite for the rare group whose scale is tiny.
   const float k = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100
@@ -122,14 +134,12 @@ __device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words,
   const float hs = 0.5f * scs;
 #pragma unroll
   for (int w = 0; w < GS / 8; ++w) {
-    uint32_t b[8];
+    int c[8];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) b[u] = sm4_byte(nearest_code(xp[8 * w + u] * k, scs, inv, hs));
-    const uint32_t lo = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
-    const uint32_t hi = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
-    words[w] = sm4_pack(lo, hi);
+    for (int u = 0; u < 8; ++u) c[u] = nearest_code(xp[8 * w + u] * k, scs, inv, hs);
+    words[w] = ob4_word(c);
   }
-  *scale_out = sc;
+  *scale_out = __float2bfloat16_rn(sc);  // exact: sc is a bfloat16 value
 }
 
 // ---- NVFP4 variant (App. B.1): one block of 16 remainder values -> E4M3 scale and E2M1 codes.
@@ -590,7 +600,7 @@ __global__ void __launch_bounds__(128) debug_quantize_kernel(const float* R, int
     dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
   } else {
     uint32_t words[8];
-    float* sc = static_cast<float*>(scales) + static_cast<size_t>(m) * (K / G) + c * (kChunk / G);
+    __nv_bfloat16* sc = static_cast<__nv_bfloat16*>(scales) + static_cast<size_t>(m) * (K / G) + c * (kChunk / G);
     if (G == 64) {
       quantize_group<64>(xp, words, sc);
     } else {
@@ -618,7 +628,7 @@ struct QuantOut {
   int K, G, M_pad;
   uint8_t* codes;
   uint8_t* sf;
-  float* scales;
+  __nv_bfloat16* scales;
 };
 
 struct RotArgs {
@@ -668,7 +678,7 @@ __device__ __forceinline__ uint32_t codes8_nvfp4(const float* x, float sc, float
 // The quantizers of kernel (a) on a warp-wide layout: each lane holds 8 consecutive remainder
 // values x (channels k .. k+7 of token row m, k a multiple of 8) and the lanes of one quantization
 // group (INT4: G/8 lanes; NVFP4: 2 lanes per block of 16) are neighbours.  Writes the codes (INT4:
-// the lane's SM4 word) and, from the group's first lane, its scale.  The scale and the codes are
+// the lane's OB4 word) and, from the group's first lane, its scale.  The scale and the codes are
 // those of quantize_group / quantize_block_nvfp4, bit for bit.
 template <bool NV>
 __device__ __forceinline__ void quantize8_lanes(const float* x, int lane, int m, int k, const QuantOut& o) {
@@ -691,18 +701,16 @@ __device__ __forceinline__ void quantize8_lanes(const float* x, int lane, int m,
     am = fmaxf(am, __shfl_xor_sync(kAll, am, 1));
     am = fmaxf(am, __shfl_xor_sync(kAll, am, 2));
     if (o.G == 64) am = fmaxf(am, __shfl_xor_sync(kAll, am, 4));
-    const float sc = __fdiv_rn(am, 7.0f);
+    const float sc = bf16_scale_div7(am);
     const float ks = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100 (see quantize_group)
     const float scs = sc * ks;
     const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
     const float hs = 0.5f * scs;
-    uint32_t b[8];
+    int c[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) b[i] = sm4_byte(nearest_code(x[i] * ks, scs, inv, hs));
-    const uint32_t lo = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
-    const uint32_t hi = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
-    *reinterpret_cast<uint32_t*>(o.codes + static_cast<size_t>(m) * (o.K / 2) + k / 2) = sm4_pack(lo, hi);
-    if ((lane & (o.G / 8 - 1)) == 0) o.scales[static_cast<size_t>(k / o.G) * o.M_pad + m] = sc;
+    for (int i = 0; i < 8; ++i) c[i] = nearest_code(x[i] * ks, scs, inv, hs);
+    *reinterpret_cast<uint32_t*>(o.codes + static_cast<size_t>(m) * (o.K / 2) + k / 2) = ob4_word(c);
+    if ((lane & (o.G / 8 - 1)) == 0) o.scales[static_cast<size_t>(k / o.G) * o.M_pad + m] = __float2bfloat16_rn(sc);
   }
 }
 
@@ -782,7 +790,7 @@ QuantOut quant_out(const Handle& h, const ActLayout& L, uint8_t* base) {
   q.M_pad = L.M_pad;
   q.codes = base + L.codes_off;
   q.sf = base + L.scales_off;
-  q.scales = reinterpret_cast<float*>(base + L.scales_off);
+  q.scales = reinterpret_cast<__nv_bfloat16*>(base + L.scales_off);
   return q;
 }
 
@@ -1141,7 +1149,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
   a.codes = base + L.codes_off;
   a.sf = base + L.scales_off;
-  a.scales = reinterpret_cast<float*>(base + L.scales_off);
+  a.scales = reinterpret_cast<__nv_bfloat16*>(base + L.scales_off);
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
   a.dump = dump;
   a.resid_only = resid_only ? 1 : 0;
@@ -1228,7 +1236,7 @@ cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4
   q.M_pad = M_pad;
   q.codes = codes;
   q.sf = scales;
-  q.scales = reinterpret_cast<float*>(scales);
+  q.scales = reinterpret_cast<__nv_bfloat16*>(scales);
   const long long warps = static_cast<long long>(M) * (K / 256);
   const int grid = static_cast<int>((warps + 7) / 8);
   if (nvfp4)

@@ -100,7 +100,7 @@ ActLayout act_layout(const Handle& h, int M) {
     return L;
   }
   L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
-  L.ab_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 4);
+  L.ab_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 2);
   L.phat_off = L.ab_off;
   L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
   L.resid_off = 0;
@@ -131,16 +131,16 @@ const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
     ok &= encode_2d(&c.qx4_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, kFp4KS / 2,
                     kBM, CU_TENSOR_MAP_SWIZZLE_128B);
   } else {
-    ok &= encode_2d(&c.qa_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, 64, kBM,
+    ok &= encode_2d(&c.qa_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, base + L.codes_off, h.K / 2, M, h.K / 2, 32, kBM,
                     CU_TENSOR_MAP_SWIZZLE_NONE);
-    ok &= encode_2d(&c.sx_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base + L.scales_off, M, h.K / h.G,
-                    static_cast<uint64_t>(L.M_pad) * 4, kBM, kScaleGroups, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= encode_2d(&c.sx_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base + L.scales_off, M, h.K / h.G,
+                    static_cast<uint64_t>(L.M_pad) * 2, kBM, 64 / h.G, CU_TENSOR_MAP_SWIZZLE_NONE);
   }
   if (h.r_pad > 0) {
     ok &= encode_2d(&c.ph_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
                     static_cast<uint64_t>(h.r_pad) * 2, 8, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
-    ok &= encode_2d(&c.ph32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
-                    static_cast<uint64_t>(h.r_pad) * 2, 32, kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= encode_2d(&c.ph64_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
+                    static_cast<uint64_t>(h.r_pad) * 2, 64, kBM, CU_TENSOR_MAP_SWIZZLE_128B);
   }
   if (!ok) return nullptr;
   c.ws = ws;
@@ -224,7 +224,7 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
   h.r = r;
   h.G = group;
   h.r_pad = r == 0 ? 0 : qwam::round_up(r, 16);
-  h.N_pad = qwam::round_up(N, qwam::kGemmBN);
+  h.N_pad = qwam::round_up(N, fmt == qwam::kFmtNvfp4 ? qwam::kGemmBN : qwam::kGemm16BN);
   h.ku3 = h.r_pad == 0 ? 0 : qwam::round_up(3 * h.r_pad, 64);
   h.rot = rot;
   if (rot) {
@@ -236,10 +236,14 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
 
   const bool nv = fmt == qwam::kFmtNvfp4;
   const size_t b_qw = qwam::up256(static_cast<size_t>(h.N_pad) * (K / 2));
-  // INT4: float16 scales and their float32 copy; NVFP4: E4M3 scale atoms (N_pad rows)
+  // INT4: bfloat16 scales, then the GEMM's float16 copies (scaled per column) and column factors;
+  // NVFP4: E4M3 scale atoms (N_pad rows)
   const size_t b_sw = nv ? qwam::up256(static_cast<size_t>(h.N_pad) * (K / qwam::kFp4Block))
                          : qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
-  const size_t b_s32 = nv ? 0 : qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 4);
+  const size_t b_s32 = nv ? 0
+                          : qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2) +
+                                qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2) +
+                                qwam::up256(static_cast<size_t>(h.N_pad) * 4);
   const size_t b_bh = qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2);
   // the bf16 split bases feed kernel (a)'s tensor-core path only (r_pad <= kMaxRank)
   const bool tc_bases = h.r_pad > 0 && h.r_pad <= qwam::kMaxRank;
@@ -258,8 +262,13 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
   if (nv) {
     h.sfw = p + b_qw;
   } else {
-    h.sw = reinterpret_cast<__half*>(p + b_qw);
-    h.sw32 = reinterpret_cast<float*>(p + b_qw + b_sw);
+    h.sw = reinterpret_cast<__nv_bfloat16*>(p + b_qw);
+    uint8_t* c = p + b_qw + b_sw;
+    h.swh = reinterpret_cast<__half*>(c);
+    c += qwam::up256(static_cast<size_t>(K / group) * h.N_pad * 2);
+    h.Bhs = reinterpret_cast<__half*>(c);
+    c += qwam::up256(static_cast<size_t>(h.N_pad) * h.r_pad * 2);
+    h.fcol = reinterpret_cast<float*>(c);
   }
   uint8_t* q = p + b_qw + b_sw + b_s32;
   h.Bh = reinterpret_cast<__half*>(q);
@@ -282,18 +291,18 @@ static qwam_status pack_impl(int fmt, const void* W_bf16, const float* U, const 
     ok &= qwam::encode_2d(&h.qw4_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, qwam::kFp4KS / 2,
                           qwam::kGemmBN, CU_TENSOR_MAP_SWIZZLE_128B);
   } else {
-    ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, N, K / 2, 64, qwam::kBM,
+    ok &= qwam::encode_2d(&h.qw_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, h.qw, K / 2, h.N_pad, K / 2, 32,
+                          qwam::kGemm16BN, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok &= qwam::encode_2d(&h.swh_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.swh, h.N_pad, K / group,
+                          static_cast<uint64_t>(h.N_pad) * 2, qwam::kGemm16BN, 64 / group,
                           CU_TENSOR_MAP_SWIZZLE_NONE);
-    // sigma is permuted within 32-column blocks, so the map spans every column of N_pad
-    ok &= qwam::encode_2d(&h.sw32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, h.sw32, h.N_pad, K / group,
-                          static_cast<uint64_t>(h.N_pad) * 4, qwam::kBM, qwam::kScaleGroups,
-                          CU_TENSOR_MAP_SWIZZLE_NONE);
+    if (h.r_pad > 0)
+      ok &= qwam::encode_2d(&h.bhs_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bhs, h.r_pad, h.N_pad,
+                            static_cast<uint64_t>(h.r_pad) * 2, 64, qwam::kGemm16BN, CU_TENSOR_MAP_SWIZZLE_128B);
   }
   if (h.r_pad > 0) {
     ok &= qwam::encode_2d(&h.Bh_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,
                           static_cast<uint64_t>(h.r_pad) * 2, 8, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
-    ok &= qwam::encode_2d(&h.bh32_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h.Bh, h.r_pad, N,
-                          static_cast<uint64_t>(h.r_pad) * 2, 32, qwam::kBM, CU_TENSOR_MAP_SWIZZLE_NONE);
   }
   if (tc_bases) {
     ok &= qwam::encode_2d(&h.ucat_t_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h.ucat_t, K, 2 * h.r_pad,
@@ -412,7 +421,7 @@ qwam_status qwam_asp_debug_quantize_rows(const float* R, int M, int K, int fmt, 
   if (fmt == QWAM_FMT_INT4 && group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
   if (M == 0) return QWAM_OK;
   if (!R || !codes || !scales || !qwam::aligned16(R) || !qwam::aligned16(codes)) return QWAM_ERR_INVALID_ARG;
-  if (fmt == QWAM_FMT_INT4 && reinterpret_cast<uintptr_t>(scales) % 4 != 0) return QWAM_ERR_INVALID_ARG;
+  if (fmt == QWAM_FMT_INT4 && reinterpret_cast<uintptr_t>(scales) % 2 != 0) return QWAM_ERR_INVALID_ARG;
   return from_cuda_status(qwam::launch_debug_quantize_rows(R, M, K, fmt == QWAM_FMT_NVFP4, group,
                                                            static_cast<uint8_t*>(codes), scales,
                                                            reinterpret_cast<cudaStream_t>(stream)));
@@ -425,7 +434,7 @@ qwam_status qwam_asp_debug_quantize_lanes(const float* R, int M, int K, int fmt,
   if (fmt == QWAM_FMT_INT4 && group != 32 && group != 64) return QWAM_ERR_INVALID_ARG;
   if (M == 0) return QWAM_OK;
   if (!R || !codes || !scales || !qwam::aligned16(R) || !qwam::aligned16(codes)) return QWAM_ERR_INVALID_ARG;
-  if (fmt == QWAM_FMT_INT4 && reinterpret_cast<uintptr_t>(scales) % 4 != 0) return QWAM_ERR_INVALID_ARG;
+  if (fmt == QWAM_FMT_INT4 && reinterpret_cast<uintptr_t>(scales) % 2 != 0) return QWAM_ERR_INVALID_ARG;
   const int M_pad = qwam::round_up(M, qwam::kBM);
   return from_cuda_status(qwam::launch_debug_quantize_lanes(
       R, M, K, fmt == QWAM_FMT_NVFP4, fmt == QWAM_FMT_NVFP4 ? qwam::kFp4Block : group, static_cast<uint8_t*>(codes),
@@ -542,21 +551,15 @@ qwam_status qwam_asp_export(qwam_asp_handle hs, void* qw, void* sw, void* Bh, vo
   if (cudaDeviceSynchronize() != cudaSuccess) return QWAM_ERR_CUDA;
   cudaError_t e = cudaSuccess;
   if (qw) {
-    // device rows are SM4 words (word j: k = 8j..8j+7, sign-magnitude); export two's-complement
-    // nibbles, low nibble = even k
+    // device rows are OB4 words (word j: k = 8j..8j+7, offset binary, see ob4_word); export
+    // two's-complement nibbles, low nibble = even k
     std::vector<uint32_t> t(static_cast<size_t>(h.N) * (h.K / 8));
     e = cudaMemcpy(t.data(), h.qw, t.size() * 4, cudaMemcpyDeviceToHost);
     uint8_t* o = static_cast<uint8_t*>(qw);
-    for (size_t wd = 0; e == cudaSuccess && wd < t.size(); ++wd) {
-      const uint32_t lo = t[wd] & 0x87878787u, hi = ((t[wd] >> 4) | (t[wd] << 28)) & 0x87878787u;
-      uint8_t c[8];
-      for (int i = 0; i < 8; ++i) {
-        const uint32_t b = ((i < 4 ? lo : hi) >> (8 * (i & 3))) & 0xFFu;
-        const int v = (b & 0x80u) ? -static_cast<int>(b & 7u) : static_cast<int>(b & 7u);
-        c[i] = static_cast<uint8_t>(v & 0xF);
-      }
-      for (int q = 0; q < 4; ++q) o[4 * wd + q] = static_cast<uint8_t>(c[2 * q] | (c[2 * q + 1] << 4));
-    }
+    for (size_t wd = 0; e == cudaSuccess && wd < t.size(); ++wd)
+      for (int q = 0; q < 4; ++q)
+        o[4 * wd + q] = static_cast<uint8_t>((qwam::ob4_code(t[wd], 2 * q) & 0xF) |
+                                             ((qwam::ob4_code(t[wd], 2 * q + 1) & 0xF) << 4));
   }
   if (e == cudaSuccess && sw)
     e = cudaMemcpy2D(sw, static_cast<size_t>(h.N) * 2, h.sw, static_cast<size_t>(h.N_pad) * 2,

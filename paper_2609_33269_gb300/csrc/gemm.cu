@@ -3,42 +3,55 @@
 // packed at 4 bits and adds the protected branch in its epilogue).
 //
 //   Y[m, n] = sum_g s_x[m, g] s_w[g, n] P_g[m, n]  +  sum_j p_hat[m, j] B_hat[n, j]
-//   P_g[m, n] = sum_{k in group g} q_x[m, k] q_w[n, k]          (exact integers)
+//   P_g[m, n] = sum_{k in group g} q_x[m, k] q_w[n, k]
 //
-// sm_103a has no integer tensor-core MMA, so both operands go to tcgen05.mma.kind::f8f6f4 as
-// E4M3 bytes of c * 2^-9 (sign | |c|: E4M3 subnormals, which the tensor core keeps exactly).  One
-// group's float32 accumulator then holds D = 2^-18 P_g exactly (every partial sum is an integer
-// below 2^13 times 2^-18).  The epilogue accumulates s_x s_w P_g as (D s_x) sigma, where
-// sigma = 2^18 s_w is the handle's float32 copy of the weight scale: two float32 roundings per
-// output and group, the float32 running sum a third.
+// Both scales are bfloat16 (8 significant bits) and the codes lie in [-7, 7] (3 bits), so every
+// dequantized operand s q has at most 11 significant bits: it is exact in float16.  The layer is
+// then one contraction over K + r_pad columns,
 //
-// Both operands stay packed at 4 bits in HBM (SM4 words, see sm4_pack) and are expanded to bytes
-// in shared memory: lo = w & 0x87878787 (k = 8j..8j+3), hi = rotr(w, 4) & 0x87878787 (k = 8j+4..).
+//   Y = [s_x q_x | p_hat] [s_w q_w | B_hat]^T,
 //
-// Persistent CTAs (one per SM) walk output tiles of 128 x 128 with a static stride (row-block
-// major, so the CTAs working at one time share the activation rows in L2).  Every ring runs
-// continuously across tiles.  384 threads:
-//   warp 0        TMA producer: packed codes of both operands per stage, scale slots;
-//   warp 1        MMA issuer and TMEM owner;
-//   warps 2, 3    expanders: packed stage -> byte operand stage (128-byte swizzle);
-//   warps 4..11   epilogue: warp 4 + 4h + q reads TMEM lane quadrant q, columns 64h .. 64h + 63.
-// Stages cover 128 K (two groups of 64 or four of 32).  After a tile's K stages come r_pad / 32
-// branch stages: the producer brings 32 columns of p_hat and B_hat (float16) through the same
-// packed ring, the expanders copy them into the operand layout, and the MMA issuer runs two
-// kind::f16 MMAs (K = 16 each); the branch accumulates in its own TMEM unit, which the epilogue
-// adds with scale 1.  Any r_pad works.
-// TMEM holds four units of 128 columns, one group each (unit g mod 4), so the MMA issuer runs up
-// to four groups ahead of the epilogue.  An mbarrier wait costs on the order of a hundred cycles
-// even when its phase has completed, so each role waits as little as possible: the MMA issuer
-// once per stage for its operands and once for the last TMEM unit the stage writes (the epilogue
-// releases units in order); each epilogue warp once per group, for the unit after the one it is
-// about to compute (its TMEM loads are double-buffered across groups, so a group's load latency
-// overlaps the arithmetic of the previous one).
-// Rings (every wait is bounded):
-//   P  packed stage (A and B codes, or p_hat / B_hat)   TMA -> expanders          SP slots
-//   O  operand stage (A and B bytes)                    expanders -> MMA          SO slots
-//   S  scale slot: s_x and sigma of kSG groups           TMA -> epilogue           SS slots
-//   T  TMEM units                                       MMA -> epilogue           4 units
+// which this kernel runs on tcgen05.mma.kind::f16 (float16 operands, float32 accumulation in TMEM)
+// with the operands dequantized from the packed 4-bit codes on the fly.  No per-group rescale is
+// left for the epilogue: the tensor cores apply both scales, and the branch is r_pad more K
+// columns of the same accumulator.
+//
+// Range.  float16 holds s q exactly while it stays in [2^-14, 2^16) (and down to 2^-24 when its
+// low bits allow).  Row m of the activation operand is therefore scaled by 2^e_m and column n of
+// the weight operand by 2^e_n, powers of two chosen so that the largest dequantized value of the
+// row (7 max_g s_x, or max |p_hat|) and of the column (7 max_g s_w, or max |B_hat|) lies in
+// [2^10, 2^11) (so that 24 s, a constant of the dequantization below, stays finite); the
+// epilogue multiplies by 2^-e_n and then 2^-e_m, which is exact unless the result is a float32
+// subnormal.  Only values below 2^-24 of their row's or column's largest can lose bits, which is
+// at the float32 accumulator's own resolution.  The weight side is done
+// once, at pack time (the handle's swh, Bhs, fcol); the row factors are formed here from s_x and
+// p_hat by the row-scale warp.
+//
+// Tiles are 128 tokens x 256 outputs (one tcgen05 MMA of M = 128, N = 256, K = 16 per 16 columns),
+// K stages of 64.  The activation operand lives in TMEM (tcgen05.mma with A from tensor memory:
+// lane m holds row m, column c the float16 pair k = 2c, 2c + 1), written by tcgen05.st from the
+// expanders' registers; the weight operand lives in shared memory in the 128-byte swizzled K-major
+// layout.  (An A operand in TMEM takes the shared-memory bandwidth of the MMA down by a third.)
+// Persistent CTAs, one per SM, walk the tiles with a static stride.  896 threads:
+//   warp 0        TMA producer: per K stage the packed codes of both operands and their scales
+//   warp 1        MMA issuer and TMEM owner
+//   warp 2        row scales: 2^e_m and 2^-e_m of the tile's 128 rows, one slot per tile
+//   warp 3        idle
+//   warps 4..19   expanders, two groups of eight that take alternate stages (group x the stages
+//                 whose running index is x mod 2), so that each warp has two stage times for its
+//                 work.  Warp e of a group takes the activation codes k = 32h .. 32h + 31
+//                 (h = e / 4) of the 32 token rows in TMEM lane quadrant q = e % 4 (16 columns
+//                 stored with tcgen05.st) and weight rows 32e .. 32e + 31 of the stage's 256
+//                 (float16 into the shared-memory operand)
+//   warps 20..27  epilogue: warp 20 + 4h + q reads lanes 32q.., columns 128h..128h+127
+// Branch stages (after the K stages, r_pad / 64 rounded up): the expanders load p_hat by TMA (one
+// buffer per group) and scale it by 2^e_m into TMEM, and B_hat 2^e_n comes by TMA straight into the
+// operand stage.  Every wait is bounded.
+// Rings:
+//   P  packed stage: A and B codes, s_x and s_w 2^e_n of its groups   TMA -> expanders   SP slots
+//   O  operand stage: A (TMEM, 32 columns) and B (shared memory)  expanders -> MMA   SO slots
+//   R  row-scale slot                          row-scale warp -> expanders, epilogue   2 slots
+//   the accumulator (TMEM columns 0..255)     MMA -> epilogue             1
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -46,188 +59,154 @@ namespace qwam {
 namespace {
 
 struct GemmArgs {
-  int M, N, K;
-  int nbs;  // branch stages per tile (r_pad / 32, rounded up)
+  int M, N, K, r_pad, M_pad;
+  int nbs;  // branch stages per tile
   int m_tiles, n_tiles;
+  const __nv_bfloat16* sx;  // workspace s_x [K/G, M_pad] (row-scale warp)
+  const __half* phat;       // workspace p_hat [M, r_pad] (row-scale warp; null when r_pad == 0)
+  const float* fcol;        // handle: 2^-e_n [N_pad]
   void* Y;
   int y_f32;
-  const float* bias;  // optional [N], added to the float32 result before it is stored
+  const float* bias;        // optional [N], added to the float32 result before it is stored
   int* err;
   uint64_t timeout_ns;
 };
 
-constexpr int kBN = 128;       // output columns per tile
-constexpr int kKS = 128;       // K per stage (128 codes: 64 packed bytes, 128 operand bytes per row)
-constexpr int kSG = 8;         // groups per scale slot
-constexpr int kNX = 2;         // expander warps
-constexpr int kThreads = 384;  // 12 warps
-constexpr int kLaunchRegs = 168;
-constexpr int kRegsCtl = 48;   // warpgroup 0 (producer, MMA, expanders)
-constexpr int kRegsEpi = 224;  // warpgroups 1-2 (epilogue)
-static_assert(128 * kRegsCtl + 256 * kRegsEpi <= kThreads * kLaunchRegs, "register split above the launch allocation");
-constexpr int SO = 4;  // operand stages
-constexpr int SP = 4;  // packed stages
-constexpr int SS = 2;  // scale slots
-constexpr int A_PK = kBM * 64;                // packed A rows (64 bytes each), then B rows
-constexpr int PSTAGE = (kBM + kBN) * 64;      // 16 KB
-constexpr int A_OP = kBM * 128;               // byte operands, 128-byte rows, 128-byte swizzle
-constexpr int OSTAGE = (kBM + kBN) * 128;     // 32 KB
-constexpr int SX_BYTES = kSG * kBM * 4;       // s_x [kSG][128]
-constexpr int SSLOT = kSG * (kBM + kBN) * 4;  // then sigma [kSG][128]
-constexpr int ONES_BYTES = 512;               // 128 floats of 1.0: the branch group's scales
-constexpr int NBAR = 2 * (SO + SP + SS + 4) + 1;
-constexpr int SMEM = 1024 + SO * OSTAGE + SP * PSTAGE + SS * SSLOT + ONES_BYTES + NBAR * 8 + 16;
+constexpr int BM = kBM;        // 128 token rows
+constexpr int BN = kGemm16BN;  // 256 output columns
+constexpr int KS = 64;         // K per stage
+constexpr int kThreads = 896;
+constexpr int SP = 4, SO = 4;
+constexpr int PA = BM * KS / 2;          // packed A bytes per stage (4 KB)
+constexpr int PB = BN * KS / 2;          // packed B bytes per stage (8 KB)
+constexpr int PSX = 2 * BM * 2;          // s_x [GPS][128] bf16 (room for two groups)
+constexpr int PSTAGE = PA + PB + PSX + 2 * BN * 2;  // then s_w 2^e_n [GPS][256] f16
+constexpr int BSTAGE = BN * KS * 2;      // float16 weight operand, 128-byte rows (32 KB)
+constexpr int PHB = BM * KS * 2;         // p_hat stage [128][64] f16, 128-byte swizzle (one per group)
+constexpr int RSB = BM * 8;              // {2^e_m, 2^-e_m} per row
+constexpr int NBAR = 2 * SP + 2 * SO + 2 + 2 * 2 + 2 * 2 + 1;
+constexpr int OFF_B = 0;
+constexpr int OFF_PH = OFF_B + SO * BSTAGE;
+constexpr int OFF_P = OFF_PH + 2 * PHB;
+constexpr int OFF_R = OFF_P + SP * PSTAGE;
+constexpr int OFF_BAR = OFF_R + 2 * RSB;
+constexpr int SMEM = 1024 + OFF_BAR + NBAR * 8 + 16;
 static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
+constexpr uint32_t TMEM_COLS = 512;  // accumulator 0..255, A ring 256 + 32 i
+constexpr uint32_t TMEM_A = 256;
 
-typedef unsigned long long f2;  // two packed float32 (for the f32x2 instructions)
-
-__device__ __forceinline__ float lo_f(f2 v) { return __uint_as_float(static_cast<uint32_t>(v)); }
-__device__ __forceinline__ float hi_f(f2 v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
-__device__ __forceinline__ f2 fma2(f2 a, f2 b, f2 c) {
-  f2 d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ f2 mul2(f2 a, f2 b) {
-  f2 d;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ f2 add2(f2 a, f2 b) {
-  f2 d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ f2 pk2u(uint32_t a, uint32_t b) {
-  f2 d;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "r"(a), "r"(b));
-  return d;
-}
-__device__ __forceinline__ f2 pk4(float a, float b) {
-  f2 d;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(a), "f"(b));
-  return d;
+__device__ __forceinline__ void mma_f16_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
 }
 
-// SM4 word -> the E4M3 bytes of its eight codes (k order).
-__device__ __forceinline__ uint2 sm4_expand(uint32_t w) {
-  return make_uint2(w & 0x87878787u, __funnelshift_r(w, w, 4) & 0x87878787u);
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// Packed float16 pairs live in 32-bit registers throughout (low half = the even k).
+__device__ __forceinline__ uint32_t mul_f16x2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+__device__ __forceinline__ uint32_t f32x2_to_f16x2(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+__device__ __forceinline__ uint32_t f32x2_to_bf16x2(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+__device__ __forceinline__ float f16_lo(uint32_t u) { return __half2float(__ushort_as_half(static_cast<unsigned short>(u))); }
+__device__ __forceinline__ float f16_hi(uint32_t u) { return __half2float(__ushort_as_half(static_cast<unsigned short>(u >> 16))); }
+
+__device__ __forceinline__ uint32_t sub_f16x2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
 }
 
-// Everything one epilogue warp needs to process a group (see the epilogue in gemm_kernel).
-struct EpiCtx {
-  const uint8_t* sring;   // scale slots
-  const float* ones;      // 128 floats of 1.0 (the branch group's scales)
-  uint64_t* sfull;
-  uint64_t* sempty;
-  uint64_t* tfull;
-  uint64_t* tempty;
-  WaitCtl wc;
-  uint32_t tq;            // TMEM address of this warp's lane quadrant and column half
-  int quad, h, rq, cq;
-  int ngk, ngt, total;    // K groups per tile, groups per tile, groups of this CTA
+// The dequantization constants of one scale s (float16, 8 significant bits): the pairs (s, s) and
+// (s/16, s/16), both exact.
+struct DqScale {
+  uint32_t s1, s16;
 };
+__device__ __forceinline__ DqScale dq_scale(float s) {
+  return DqScale{f32x2_to_f16x2(s, s), f32x2_to_f16x2(0.0625f * s, 0.0625f * s)};
+}
 
-// One group of the epilogue: g is the CTA's running group index (TMEM unit g % 4), gi its index in
-// the tile, sl the running index of the scale slot it reads.  Its TMEM loads sit in v[CUR] (issued
-// while the previous group was computed); the loads of group g + 1 go to v[CUR ^ 1] block by block.
-template <int CUR>
-__device__ __forceinline__ void epi_group(const EpiCtx& c, f2 (&acc)[32], uint32_t (&v)[2][4][16], int& g, int& gi,
-                                          int& sl, bool& ok) {
-  const bool more = g + 1 < c.total;
-  const bool kgroup = gi < c.ngk;
-  const int gi_n = gi + 1 == c.ngt ? 0 : gi + 1;
-  const bool slot_n = gi_n < c.ngk && (gi_n & (kSG - 1)) == 0;  // group g + 1 starts a scale slot
-  const int gl = gi & (kSG - 1);
-  // v[CUR][2b + rh][4j + 2rr + {0, 1}] = columns (32b + 8j + 2cq, +1) of row rq + 16 rh + 8 rr
-  tmem_ld_wait_dep4(v[CUR]);
-  tc_fence_before();
-  // Every load of the unit has landed: release it before waiting for the next group (whose stage
-  // the MMA issuer may only start once this unit is free).
-  warp_arrive(&c.tempty[g & 3]);
-  // The next group's phases, tested now and used after the first block: the test's latency
-  // overlaps the arithmetic.
-  const bool ready_n = !more || ((!slot_n || mbar_test_wait(&c.sfull[(sl + 1) & (SS - 1)], ((sl + 1) / SS) & 1)) &&
-                                 mbar_test_wait(&c.tfull[(g + 1) & 3], ((g + 1) >> 2) & 1));
-  const uint8_t* slot = c.sring + (sl & (SS - 1)) * SSLOT;
-  const float* sxb = kgroup ? reinterpret_cast<const float*>(slot) + gl * kBM : c.ones;
-  const float* sgb = kgroup ? reinterpret_cast<const float*>(slot + SX_BYTES) + gl * kBN : c.ones;
-  float sx[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) sx[k] = sxb[c.quad * 32 + c.rq + 8 * k];
-  const uint32_t tn = c.tq + static_cast<uint32_t>(((g + 1) & 3) * kBN);
-#pragma unroll
-  for (int b = 0; b < 2; ++b) {
-    const float4* sgp = reinterpret_cast<const float4*>(sgb + 64 * c.h + 32 * b + c.cq * 8);
-    const float4 s0 = sgp[0], s1 = sgp[1];
-    const f2 sg[4] = {pk4(s0.x, s0.y), pk4(s0.z, s0.w), pk4(s1.x, s1.y), pk4(s1.z, s1.w)};
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const f2 sx2 = dup2(sx[k]);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t* dv = &v[CUR][2 * b + (k >> 1)][4 * j + 2 * (k & 1)];
-        const f2 t = mul2(pk2u(dv[0], dv[1]), sx2);
-        acc[16 * b + 4 * k + j] = fma2(t, sg[j], acc[16 * b + 4 * k + j]);
-      }
-    }
-    if (b == 0) {
-      if (!ready_n && ok) {
-        if (slot_n) ok = mbar_wait_inline(&c.sfull[(sl + 1) & (SS - 1)], ((sl + 1) / SS) & 1, c.wc);
-        if (ok) ok = mbar_wait_inline(&c.tfull[(g + 1) & 3], ((g + 1) >> 2) & 1, c.wc);
-      }
-      tc_fence_after();
-    }
-    // Issued on every path (after the CTA's last group it reads a unit nobody uses any more), so
-    // that each wait's registers come from the loads just before it.
-    tmem_ld16x256_x4(tn + 32 * b, v[CUR ^ 1][2 * b]);
-    tmem_ld16x256_x4(tn + (16u << 16) + 32 * b, v[CUR ^ 1][2 * b + 1]);
-  }
-  if (kgroup && (gl == kSG - 1 || gi == c.ngk - 1)) {
-    fence_proxy_async_smem();  // reads of the TMA-written scales before the slot is refilled
-    warp_arrive(&c.sempty[sl & (SS - 1)]);
-  }
-  if (slot_n) ++sl;
-  ++g;
-  gi = gi_n;
+// One OB4 word (codes k = 8j..8j+7, nibbles n = c + 8) times the scale -> four float16 pairs in k
+// order.  Under the float16 pattern of 1024 (0x6400, whose unit in the last place is 1) the nibbles
+// of bits 0..3 read as 1024 + n and those of bits 4..7 as 1024 + 16 n; subtracting 1032 or 1152
+// leaves c or 16 c exactly, and multiplying by s or s/16 gives c s exactly (at most 11 significant
+// bits).  Pairs 2 and 3 take the same steps on the word shifted down by 8.  Five integer and eight
+// float16 operations per 8 codes.
+__device__ __forceinline__ void dequant_word(uint32_t w, const DqScale& d, uint32_t* out) {
+  constexpr uint32_t k1032 = 0x64086408u, k1152 = 0x64806480u, kMag = 0x64006400u;
+  const uint32_t w2 = w >> 8;
+  out[0] = mul_f16x2(sub_f16x2((w & 0x000F000Fu) | kMag, k1032), d.s1);
+  out[1] = mul_f16x2(sub_f16x2((w & 0x00F000F0u) | kMag, k1152), d.s16);
+  out[2] = mul_f16x2(sub_f16x2((w2 & 0x000F000Fu) | kMag, k1032), d.s1);
+  out[3] = mul_f16x2(sub_f16x2((w2 & 0x00F000F0u) | kMag, k1152), d.s16);
+}
+
+// s (bfloat16) times 2^e, rounded to float16 (exact while in range), as dequantization constants.
+__device__ __forceinline__ DqScale scale_consts(__nv_bfloat16 s, float mul) {
+  return dq_scale(__half2float(__float2half_rn(__bfloat162float(s) * mul)));
+}
+
+// 32 TMEM lanes x 16 consecutive 32-bit columns from registers.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+// Transaction bytes expected on a barrier, without an arrival.
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
 }
 
 template <int G>
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_kernel(const __grid_constant__ CUtensorMap qa_map, const __grid_constant__ CUtensorMap qw_map,
-                const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap sw_map,
-                const __grid_constant__ CUtensorMap ph_map, const __grid_constant__ CUtensorMap bh_map,
-                const GemmArgs a) {
-  constexpr int GPS = kKS / G;  // groups per K stage
-  static_assert(kSG % GPS == 0, "a scale slot covers whole stages");
+    gemm16_kernel(const __grid_constant__ CUtensorMap qa_map, const __grid_constant__ CUtensorMap qw_map,
+                  const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap sw_map,
+                  const __grid_constant__ CUtensorMap ph_map, const __grid_constant__ CUtensorMap bh_map,
+                  const GemmArgs a) {
+  constexpr int GPS = KS / G;   // groups per K stage (1 or 2)
   extern __shared__ uint8_t smem_raw[];
   pdl_launch_dependents();
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* oring = smem;                 // SO x (A bytes | B bytes)
-  uint8_t* pring = oring + SO * OSTAGE;  // SP x (A packed | B packed)
-  uint8_t* sring = pring + SP * PSTAGE;  // SS x (s_x | sigma)
-  float* ones = reinterpret_cast<float*>(sring + SS * SSLOT);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sring + SS * SSLOT + ONES_BYTES);
+  uint8_t* bring = smem + OFF_B;
+  uint8_t* phbuf = smem + OFF_PH;
+  uint8_t* pring = smem + OFF_P;
+  float2* rslot = reinterpret_cast<float2*>(smem + OFF_R);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* pfull = bars;
   uint64_t* pempty = pfull + SP;
   uint64_t* ofull = pempty + SP;
   uint64_t* oempty = ofull + SO;
-  uint64_t* sfull = oempty + SO;
-  uint64_t* sempty = sfull + SS;
-  uint64_t* tfull = sempty + SS;
-  uint64_t* tempty = tfull + 4;
-  uint64_t* drain = tempty + 4;
+  uint64_t* accfull = oempty + SO;
+  uint64_t* accempty = accfull + 1;
+  uint64_t* rfull = accempty + 1;
+  uint64_t* rempty = rfull + 2;
+  uint64_t* phfull = rempty + 2;   // one per expander group
+  uint64_t* phempty = phfull + 2;
+  uint64_t* drain = phempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NBAR);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const uint32_t wid = warp_id(), lane = lane_id();
-  const int ngk = a.K / G;     // K groups per tile
-  const int nks = (a.K + kKS - 1) / kKS;  // K stages per tile (the last is half past K when K % 128 == 64:
-                                          // TMA zero-fills it and its missing groups are skipped)
-  const int nbs = a.nbs;       // branch stages per tile
-  const int nst = nks + nbs;
-  const int ngt = ngk + (nbs > 0 ? 1 : 0);  // groups per tile, the branch included
-  const int nsl = (ngk + kSG - 1) / kSG;    // scale slots per tile
+  const int nks = a.K / KS;
+  const int nst = nks + a.nbs;
   const int ntiles = a.m_tiles * a.n_tiles;
   const int my_tiles = ntiles > static_cast<int>(blockIdx.x)
                            ? (ntiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
@@ -235,34 +214,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                            : 0;
   auto tile_mn = [&](int i, int& m0, int& n0) {
     const int t = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
-    m0 = (t / a.n_tiles) * kBM;
-    n0 = (t % a.n_tiles) * kBN;
+    m0 = (t / a.n_tiles) * BM;
+    n0 = (t % a.n_tiles) * BN;
   };
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < SP; ++i) {
       mbar_init(&pfull[i], 1);
-      mbar_init(&pempty[i], kNX);
+      mbar_init(&pempty[i], 8);
     }
     for (int i = 0; i < SO; ++i) {
-      mbar_init(&ofull[i], kNX);
+      mbar_init(&ofull[i], 8);
       mbar_init(&oempty[i], 1);
     }
-    for (int i = 0; i < SS; ++i) {
-      mbar_init(&sfull[i], 1);
-      mbar_init(&sempty[i], 8);
-    }
-    for (int i = 0; i < 4; ++i) {
-      mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], 8);
+    mbar_init(accfull, 1);
+    mbar_init(accempty, 8);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&rfull[i], 1);
+      mbar_init(&rempty[i], 24);
+      mbar_init(&phfull[i], 1);
+      mbar_init(&phempty[i], 8);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (threadIdx.x < 128) ones[threadIdx.x] = 1.0f;
   if (wid == 1) {
-    tmem_alloc(tmem_slot, 512);
+    tmem_alloc(tmem_slot, TMEM_COLS);
     tmem_relinquish();
   }
   __syncthreads();
@@ -271,283 +249,318 @@ __global__ void __launch_bounds__(kThreads, 1)
   const WaitCtl wc{abort_flag, a.err, globaltimer_ns() + a.timeout_ns};
   pdl_wait();  // every global access of this kernel comes after the previous kernel's
 
-  if (wid < 4) {
-    setmaxnreg_dec<kRegsCtl>();
-    if (wid == 0) {
-      // ----------------------------------------------------------- TMA producer
-      // The whole warp walks the loop (warp-uniform state); one elected lane issues each copy.
-      bool ok = true;
-      int s = 0, ss = 0;
-      for (int ti = 0; ti < my_tiles && ok; ++ti) {
-        int m0, n0;
-        tile_mn(ti, m0, n0);
-        for (int st = 0; st < nst && ok; ++st, ++s) {
-          if (st < nks && (st * GPS) % kSG == 0) {
-            // s_x and sigma of the next kSG groups (zero-filled past K)
-            const int sb = ss % SS;
-            if (ss >= SS) ok = mbar_wait_inline(&sempty[sb], ((ss / SS) & 1) ^ 1, wc);
-            if (!ok) break;
-            uint8_t* q = sring + sb * SSLOT;
-            if (elect_one()) {
-              mbar_arrive_expect_tx(&sfull[sb], SSLOT);
-              tma_load_2d(q, &sx_map, &sfull[sb], m0, st * GPS);
-              tma_load_2d(q + SX_BYTES, &sw_map, &sfull[sb], n0, st * GPS);
-            }
-            __syncwarp();
-            ++ss;
-          }
-          const int ps = s % SP;
-          if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
-          if (!ok) break;
-          uint8_t* p = pring + ps * PSTAGE;
-          if (elect_one()) {
-            mbar_arrive_expect_tx(&pfull[ps], PSTAGE);
-            if (st < nks) {
-              tma_load_2d(p, &qa_map, &pfull[ps], st * (kKS / 2), m0);
-              tma_load_2d(p + A_PK, &qw_map, &pfull[ps], st * (kKS / 2), n0);
-            } else {
-              const int bs = st - nks;
-              tma_load_2d(p, &ph_map, &pfull[ps], bs * 32, m0);
-              tma_load_2d(p + A_PK, &bh_map, &pfull[ps], bs * 32, n0);
-            }
-          }
-          __syncwarp();
-        }
-      }
-      // Let every issued load land before the CTA can exit (these phases complete in the normal
-      // course; after an abort the waits end at the deadline).
-      int never = 0;
-      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-      for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
-      for (int j = (ss > SS ? ss - SS : 0); j < ss; ++j) mbar_wait_inline(&sfull[j % SS], (j / SS) & 1, dc);
-    } else if (wid == 1) {
-      // ----------------------------------------------------------- MMA issuer
-      // The whole warp walks the loop and forms the descriptors; one elected lane (the same one
-      // throughout, as the commits track its MMAs) issues a stage's MMAs and commits together.
-      bool ok = true;
-      constexpr uint32_t idesc = idesc_e4m3(kBM, kBN);
-      constexpr uint32_t idesc_br = idesc_f16(kBM, kBN);
-      int s = 0, gr = 0;  // running stage and group counters
-      for (int ti = 0; ti < my_tiles && ok; ++ti) {
-        for (int st = 0; st < nst && ok; ++st, ++s) {
-          const int os = s % SO;
-          const bool kst = st < nks;
-          const int gn = kst ? min(GPS, ngk - st * GPS) : 1;  // groups this stage writes
-          ok = mbar_wait_inline(&ofull[os], (s / SO) & 1, wc);
-          // the last TMEM unit this stage writes: its release (four groups back) implies the
-          // earlier ones (the epilogue releases units in order)
-          const int glast = gr + gn - 1;
-          if (ok && glast >= 4 && (kst || st == nks))
-            ok = mbar_wait_inline(&tempty[glast & 3], ((glast >> 2) & 1) ^ 1, wc);
-          if (!ok) break;
-          tc_fence_after();
-          const uint32_t aa = smem_u32(oring + os * OSTAGE);
-          const uint64_t adesc = smem_desc(aa, 16, 1024, kSw128), bdesc = smem_desc(aa + A_OP, 16, 1024, kSw128);
-          if (elect_one()) {
-            if (kst) {
-#pragma unroll
-              for (int gi = 0; gi < GPS; ++gi) {
-                if (gi >= gn) break;
-                const uint32_t d = tmem + static_cast<uint32_t>(((gr + gi) & 3) * kBN);
-#pragma unroll
-                for (int kk = 0; kk < G / 32; ++kk) {
-                  const uint64_t off = static_cast<uint64_t>((gi * G + kk * 32) >> 4);  // 16-byte units
-                  mma_f8f6f4(d, adesc + off, bdesc + off, idesc, kk != 0);
-                }
-                mma_commit(&tfull[(gr + gi) & 3]);
-              }
-            } else {
-              const int bs = st - nks;
-              const uint32_t d = tmem + static_cast<uint32_t>((gr & 3) * kBN);
-              mma_f16(d, adesc, bdesc, idesc_br, bs != 0);
-              mma_f16(d, adesc + 2, bdesc + 2, idesc_br, 1);
-              if (bs == nbs - 1) mma_commit(&tfull[gr & 3]);
-            }
-            mma_commit(&oempty[os]);
-          }
-          __syncwarp();
-          if (kst)
-            gr += gn;
-          else if (st == nst - 1)
-            ++gr;
-        }
-      }
-      if (elect_one()) mma_commit(drain);
-      __syncwarp();
-      int never = 0;
-      const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-      mbar_wait_inline(drain, 0, dc);
-    } else {
-      // ----------------------------------------------------------- expanders
-      // Thread e (0..63) takes the 16-byte piece q = e % 4 of packed rows r0 + 16 i (r0 = e / 4,
-      // i = 0..15; rows 0..127 are A, 128..255 B): a K stage expands it to the operand chunks
-      // 2q, 2q + 1 of the row, a branch stage copies it to chunk q.  Operand rows are 128 bytes with
-      // the 128-byte swizzle (chunk c of row r at c ^ (r % 8)); r % 8 = r0 % 8 for all of this
-      // thread's rows, so every offset below is a constant.
-      const int e = static_cast<int>(threadIdx.x) - 64;
-      const int r0 = e >> 2, q = e & 3, sw = r0 & 7;
-      const int src0 = r0 * 64 + q * 16;
-      const int dlo = r0 * 128 + (((2 * q) ^ sw) << 4), dhi = r0 * 128 + (((2 * q + 1) ^ sw) << 4);
-      const int dcp = r0 * 128 + ((q ^ sw) << 4);
-      bool ok = true;
-      int s = 0;
-      for (int ti = 0; ti < my_tiles && ok; ++ti) {
-        for (int st = 0; st < nst && ok; ++st, ++s) {
-          const int ps = s % SP, os = s % SO;
-          ok = mbar_wait_inline(&pfull[ps], (s / SP) & 1, wc);
-          if (ok && s >= SO) ok = mbar_wait_inline(&oempty[os], ((s / SO) & 1) ^ 1, wc);
-          if (!ok) break;
-          const uint8_t* src = pring + ps * PSTAGE + src0;
-          uint8_t* dst = oring + os * OSTAGE;
-          // Four loads, then four expansions and their stores: the stores may alias the loads as far
-          // as the compiler knows, so written in this order the loads are in flight together.
-          if (st < nks) {
-#pragma unroll 1
-            for (int i0 = 0; i0 < 16; i0 += 4) {
-              uint4 v[4];
-#pragma unroll
-              for (int i = 0; i < 4; ++i) v[i] = *reinterpret_cast<const uint4*>(src + (i0 + i) * 1024);
-#pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                const uint2 x = sm4_expand(v[i].x), y = sm4_expand(v[i].y), z = sm4_expand(v[i].z),
-                            w = sm4_expand(v[i].w);
-                *reinterpret_cast<uint4*>(dst + dlo + (i0 + i) * 2048) = make_uint4(x.x, x.y, y.x, y.y);
-                *reinterpret_cast<uint4*>(dst + dhi + (i0 + i) * 2048) = make_uint4(z.x, z.y, w.x, w.y);
-              }
-            }
-          } else {
-#pragma unroll 1
-            for (int i0 = 0; i0 < 16; i0 += 4) {
-              uint4 v[4];
-#pragma unroll
-              for (int i = 0; i < 4; ++i) v[i] = *reinterpret_cast<const uint4*>(src + (i0 + i) * 1024);
-#pragma unroll
-              for (int i = 0; i < 4; ++i) *reinterpret_cast<uint4*>(dst + dcp + (i0 + i) * 2048) = v[i];
-            }
-          }
-          // Orders the generic writes of the operand stage before the MMA reads them, and the
-          // generic reads of the packed stage before TMA refills it.
-          fence_proxy_async_smem();
-          warp_arrive(&ofull[os]);
-          warp_arrive(&pempty[ps]);
-        }
-      }
-    }
-  } else {
-    setmaxnreg_inc<kRegsEpi>();
-    // ------------------------------------------------------------- epilogue
-    // Warp 4 + 4h + q reads TMEM lanes 32q.. (its quadrant of rows), columns 64h .. 64h + 63 of
-    // each unit.  With the 16x256b load shape, thread t holds rows rq + 8k (k = 0..3, rq = t / 4)
-    // and, in each 32-column block b, columns 8j + 2cq + {0, 1} (j = 0..3, cq = t % 4):
-    // acc[16b + 4k + j] is that pair.  Per group and output: t = D s_x, acc += t sigma.  Sigma is
-    // stored permuted within each 32-column block, so the thread's eight scales of a block are
-    // contiguous (two 16-byte loads).
-    const int quad = static_cast<int>(wid & 3), h = (static_cast<int>(wid) - 4) >> 2;
-    const int rq = static_cast<int>(lane) >> 2, cq = static_cast<int>(lane) & 3;
-    EpiCtx c;
-    c.sring = sring;
-    c.ones = ones;
-    c.sfull = sfull;
-    c.sempty = sempty;
-    c.tfull = tfull;
-    c.tempty = tempty;
-    c.wc = wc;
-    c.tq = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(64 * h);
-    c.quad = quad;
-    c.h = h;
-    c.rq = rq;
-    c.cq = cq;
-    c.ngk = ngk;
-    c.ngt = ngt;
-    c.total = my_tiles * ngt;  // groups this CTA's epilogue walks (branch included)
+  if (wid == 0) {
+    // ------------------------------------------------------------- TMA producer
     bool ok = true;
-    uint32_t v[2][4][16];  // TMEM loads of two groups: [buffer][block b * 2 + row half][16]
-    f2 acc[32];
-    if (c.total > 0) {
-      if (ok) ok = mbar_wait_inline(&sfull[0], 0, wc);
-      if (ok) ok = mbar_wait_inline(&tfull[0], 0, wc);
-      tc_fence_after();
-#pragma unroll
-      for (int b = 0; b < 2; ++b) {
-        tmem_ld16x256_x4(c.tq + 32 * b, v[0][2 * b]);
-        tmem_ld16x256_x4(c.tq + (16u << 16) + 32 * b, v[0][2 * b + 1]);
-      }
-    }
-    // Group g of the CTA lands in buffer g % 2.  A tile's groups run in pairs from a buffer parity
-    // fixed at compile time (one copy of the loop per parity, chosen by the tile's first group), so
-    // the accumulator is zeroed and stored outside the per-group code.  The branch group takes the
-    // same arithmetic with unit scales (D * 1 * 1 + acc = D + acc exactly).
-    int g = 0, sl = 0;
-    for (int ti = 0; ti < my_tiles; ++ti) {
-#pragma unroll
-      for (int i = 0; i < 32; ++i) acc[i] = 0ull;
-      // (gi is advanced by epi_group and wraps to 0 after the tile's last group; the loops below
-      // count the tile's groups with their own index)
-      int gi = 0;
-      if ((g & 1) == 0) {
-        for (int j = 0; j + 2 <= ngt; j += 2) {
-          epi_group<0>(c, acc, v, g, gi, sl, ok);
-          epi_group<1>(c, acc, v, g, gi, sl, ok);
-        }
-        if (ngt & 1) epi_group<0>(c, acc, v, g, gi, sl, ok);
-      } else {
-        for (int j = 0; j + 2 <= ngt; j += 2) {
-          epi_group<1>(c, acc, v, g, gi, sl, ok);
-          epi_group<0>(c, acc, v, g, gi, sl, ok);
-        }
-        if (ngt & 1) epi_group<1>(c, acc, v, g, gi, sl, ok);
-      }
-      // the tile's output: Y (plus the bias)
+    int s = 0;
+    for (int ti = 0; ti < my_tiles && ok; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
-      if (ok) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int m = m0 + quad * 32 + rq + 8 * k;
-          if (m >= a.M) continue;
-#pragma unroll
-          for (int b = 0; b < 2; ++b)
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const int n = n0 + 64 * h + 32 * b + 8 * j + 2 * cq;  // even; N is a multiple of 8
-              if (n >= a.N) continue;
-              const size_t off = static_cast<size_t>(m) * a.N + n;
-              const f2 y = acc[16 * b + 4 * k + j];
-              float y0 = lo_f(y), y1 = hi_f(y);
-              if (a.bias) {
-                const float2 bb = *reinterpret_cast<const float2*>(a.bias + n);
-                y0 += bb.x;
-                y1 += bb.y;
-              }
-              if (a.y_f32) {
-                *reinterpret_cast<float2*>(static_cast<float*>(a.Y) + off) = make_float2(y0, y1);
-              } else {
-                *reinterpret_cast<__nv_bfloat162*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
-                    __floats2bfloat162_rn(y0, y1);
-              }
-            }
+      for (int st = 0; st < nks && ok; ++st, ++s) {
+        const int ps = s % SP;
+        if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
+        if (!ok) break;
+        uint8_t* p = pring + ps * PSTAGE;
+        if (elect_one()) {
+          mbar_arrive_expect_tx(&pfull[ps], PA + PB + GPS * (BM + BN) * 2);
+          tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
+          tma_load_2d(p + PA, &qw_map, &pfull[ps], st * (KS / 2), n0);
+          tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
+          tma_load_2d(p + PA + PB + PSX, &sw_map, &pfull[ps], n0, st * GPS);
         }
+        __syncwarp();
       }
     }
-    tmem_ld_wait();  // the loads issued after the last group land before TMEM is released
+    // every issued load lands before the CTA can exit
+    int never = 0;
+    const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+    for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
+  } else if (wid == 1) {
+    // ------------------------------------------------------------- MMA issuer
+    constexpr uint32_t idesc = idesc_f16(BM, BN);
+    bool ok = true;
+    int so = 0;
+    for (int ti = 0; ti < my_tiles && ok; ++ti) {
+      if (ti > 0) ok = mbar_wait_inline(accempty, (ti - 1) & 1, wc);  // the epilogue has read the last tile
+      for (int st = 0; st < nst && ok; ++st, ++so) {
+        const int os = so % SO;
+        ok = mbar_wait_inline(&ofull[os], (so / SO) & 1, wc);
+        if (!ok) break;
+        tc_fence_after();
+        const uint64_t bdesc = smem_desc(smem_u32(bring + os * BSTAGE), 16, 1024, kSw128);
+        const uint32_t at = tmem + TMEM_A + static_cast<uint32_t>(os * 32);
+        if (elect_one()) {
+#pragma unroll
+          for (int kk = 0; kk < KS / 16; ++kk)
+            mma_f16_tmem_a(tmem, at + 8 * kk, bdesc + 2 * kk, idesc, (st | kk) != 0 ? 1u : 0u);
+          mma_commit(&oempty[os]);
+          if (st == nst - 1) mma_commit(accfull);
+        }
+        __syncwarp();
+      }
+    }
+    if (elect_one()) mma_commit(drain);
+    __syncwarp();
+    int never = 0;
+    const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+    mbar_wait_inline(drain, 0, dc);
+  } else if (wid == 2) {
+    // ------------------------------------------------------------- row scales
+    // Lane l takes rows m0 + 4l .. m0 + 4l + 3: the largest dequantized value of the row,
+    // a_m = max(7 max_g s_x[m, g], max_j |p_hat[m, j]|), gives e_m = 10 - floor(log2 a_m).
+    bool ok = true;
+    const int ng = a.K / G;
+    for (int ti = 0; ti < my_tiles && ok; ++ti) {
+      int m0, n0;
+      tile_mn(ti, m0, n0);
+      const int sl = ti & 1;
+      if (ti >= 2) ok = mbar_wait_inline(&rempty[sl], ((ti >> 1) & 1) ^ 1, wc);
+      if (!ok) break;
+      const int mr = m0 + 4 * static_cast<int>(lane);  // < M_pad (a multiple of 128)
+      float smax[4] = {0.f, 0.f, 0.f, 0.f};
+      const __nv_bfloat16* sp = a.sx + mr;
+#pragma unroll 4
+      for (int g = 0; g < ng; ++g) {
+        const uint2 v = *reinterpret_cast<const uint2*>(sp + static_cast<size_t>(g) * a.M_pad);
+        smax[0] = fmaxf(smax[0], __uint_as_float(v.x << 16));
+        smax[1] = fmaxf(smax[1], __uint_as_float(v.x & 0xFFFF0000u));
+        smax[2] = fmaxf(smax[2], __uint_as_float(v.y << 16));
+        smax[3] = fmaxf(smax[3], __uint_as_float(v.y & 0xFFFF0000u));
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float am = 7.0f * smax[i];  // exact: 8 + 3 significant bits
+        const int m = mr + i;
+        if (a.r_pad > 0 && m < a.M) {
+          const uint4* pr = reinterpret_cast<const uint4*>(a.phat + static_cast<size_t>(m) * a.r_pad);
+          for (int j = 0; j < a.r_pad / 8; ++j) {
+            const uint4 u = pr[j];
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) am = fmaxf(am, fmaxf(fabsf(f16_lo(w4[t])), fabsf(f16_hi(w4[t]))));
+          }
+        }
+        int e = 0;
+        if (am > 0.0f) {
+          int ex;
+          frexpf(am, &ex);  // am in [2^(ex-1), 2^ex)
+          e = min(126, max(-126, 11 - ex));
+        }
+        rslot[sl * BM + 4 * lane + i] = make_float2(ldexpf(1.0f, e), ldexpf(1.0f, -e));
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&rfull[sl]);
+      __syncwarp();
+    }
+  } else if (wid >= 4 && wid < 20) {
+    // ------------------------------------------------------------- expanders
+    // Activation part: row r = 32q + lane (TMEM lane), codes k = 32h .. 32h + 31 of the stage
+    // (packed words 4h .. 4h+3), to TMEM columns 16h .. 16h + 15 of the stage's slot.
+    // Weight part: rows R = 32e + 16i + lane/2 (i = 0, 1), half hh = lane % 2 of the row (words
+    // 4hh .. 4hh+3, codes 32hh ..), written as the 16-byte chunks 4hh + jj of row R at their
+    // swizzled places (chunk c of row R at c ^ (R % 8); R % 8 = (lane / 2) % 8 for every i).
+    const int gx = (static_cast<int>(wid) - 4) >> 3;  // expander group
+    const int e = (static_cast<int>(wid) - 4) & 7;
+    const int q = e & 3, h = e >> 2;
+    const int r = 32 * q + static_cast<int>(lane);
+    const int hh = static_cast<int>(lane) & 1;
+    const int Rb = 32 * e + (static_cast<int>(lane) >> 1);
+    const uint32_t tlane = tmem + (static_cast<uint32_t>(32 * q) << 16) + TMEM_A + static_cast<uint32_t>(16 * h);
+    uint8_t* phb = phbuf + gx * PHB;
+    uint32_t xo[4];  // swizzled chunk offsets of this thread's weight chunks within a row
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) xo[jj] = static_cast<uint32_t>(((4 * hh + jj) ^ (Rb & 7)) << 4);
+    bool ok = true;
+    int s = 0, so = 0, ph = 0;
+    for (int ti = 0; ti < my_tiles && ok; ++ti) {
+      int m0, n0;
+      tile_mn(ti, m0, n0);
+      ok = mbar_wait_inline(&rfull[ti & 1], (ti >> 1) & 1, wc);
+      if (!ok) break;
+      const float mul = rslot[(ti & 1) * BM + r].x;
+      for (int st = 0; st < nst && ok; ++st, ++so) {
+        const bool kst = st < nks;
+        const int ps = s % SP;
+        const int pphase = (s / SP) & 1;
+        if (kst) ++s;
+        if ((so & 1) != gx) continue;  // the other group's stage
+        const int os = so % SO;
+        if (so >= SO) ok = mbar_wait_inline(&oempty[os], ((so / SO) & 1) ^ 1, wc);
+        if (!ok) break;
+        tc_fence_after();
+        uint8_t* dst = bring + os * BSTAGE;
+        uint32_t v[16];
+        if (kst) {
+          ok = mbar_wait_inline(&pfull[ps], pphase, wc);
+          if (!ok) break;
+          const uint8_t* pk = pring + ps * PSTAGE;
+          // every load of the stage first (the operand stores may alias them as far as the
+          // compiler knows), then the conversions and stores
+          const uint4 wa = *reinterpret_cast<const uint4*>(pk + r * (KS / 2) + 16 * h);
+          const __nv_bfloat16 sxa = reinterpret_cast<const __nv_bfloat16*>(pk + PA + PB)[(GPS == 2 ? h : 0) * BM + r];
+          uint4 wb[2];
+          __half swb[2];
+#pragma unroll
+          for (int i = 0; i < 2; ++i) {
+            const int R = Rb + 16 * i;
+            wb[i] = *reinterpret_cast<const uint4*>(pk + PA + R * (KS / 2) + 16 * hh);
+            swb[i] = reinterpret_cast<const __half*>(pk + PA + PB + PSX)[(GPS == 2 ? hh : 0) * BN + R];
+          }
+          const DqScale da = scale_consts(sxa, mul);
+          dequant_word(wa.x, da, v + 0);
+          dequant_word(wa.y, da, v + 4);
+          dequant_word(wa.z, da, v + 8);
+          dequant_word(wa.w, da, v + 12);
+#pragma unroll
+          for (int i = 0; i < 2; ++i) {
+            const DqScale db = dq_scale(__half2float(swb[i]));
+            uint8_t* row = dst + (Rb + 16 * i) * 128;
+            const uint32_t wv[4] = {wb[i].x, wb[i].y, wb[i].z, wb[i].w};
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+              uint32_t o[4];
+              dequant_word(wv[jj], db, o);
+              *reinterpret_cast<uint4*>(row + xo[jj]) = make_uint4(o[0], o[1], o[2], o[3]);
+            }
+          }
+          // orders the operand writes before the MMA reads them, and the packed reads before TMA
+          // refills the stage
+          fence_proxy_async_smem();
+          warp_arrive(&pempty[ps]);
+        } else {
+          // branch stage: p_hat 2^e_m into TMEM (exact unless p_hat itself is zero: then 0), and
+          // B_hat 2^e_n by TMA straight into the operand stage (its bytes complete the stage's
+          // barrier together with the eight arrivals)
+          if (ph > 0) ok = mbar_wait_inline(&phempty[gx], (ph - 1) & 1, wc);  // the group's last p_hat was read
+          if (!ok) break;
+          if (e == 0) {
+            if (elect_one()) {
+              mbar_expect_tx(&ofull[os], BSTAGE);
+              tma_load_2d(dst, &bh_map, &ofull[os], (st - nks) * KS, n0);
+              mbar_arrive_expect_tx(&phfull[gx], PHB);
+              tma_load_2d(phb, &ph_map, &phfull[gx], (st - nks) * KS, m0);
+            }
+            __syncwarp();
+          }
+          ok = mbar_wait_inline(&phfull[gx], ph & 1, wc);
+          ++ph;
+          if (!ok) break;
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const uint4 u = *reinterpret_cast<const uint4*>(phb + r * 128 + (((4 * h + c) ^ (r & 7)) << 4));
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) v[4 * c + t] = f32x2_to_f16x2(f16_lo(w4[t]) * mul, f16_hi(w4[t]) * mul);
+          }
+          fence_proxy_async_smem();
+          warp_arrive(&phempty[gx]);
+        }
+        tmem_st16(tlane + static_cast<uint32_t>(os * 32), v);
+        tmem_st_wait();
+        tc_fence_before();
+        warp_arrive(&ofull[os]);
+      }
+      warp_arrive(&rempty[ti & 1]);
+    }
+    // the last TMA loads this warp issued have landed (they have, unless the kernel aborted first)
+    int never = 0;
+    const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+    if (ph > 0) mbar_wait_inline(&phfull[gx], (ph - 1) & 1, dc);
+    if (e == 0 && a.nbs > 0) {
+      // this group's last branch stage: its B_hat load completed the stage's barrier
+      int lb = -1;
+      for (int j = so - 1; j >= 0 && j >= so - a.nbs; --j)
+        if ((j & 1) == gx) {
+          lb = j;
+          break;
+        }
+      if (lb >= 0) mbar_wait_inline(&ofull[lb % SO], (lb / SO) & 1, dc);
+    }
+  } else if (wid >= 20) {
+    // ------------------------------------------------------------- epilogue
+    const int ew = static_cast<int>(wid) - 20;
+    const int q = ew & 3, hf = ew >> 2;
+    const int r = 32 * q + static_cast<int>(lane);
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * hf);
+    bool ok = true;
+    for (int ti = 0; ti < my_tiles && ok; ++ti) {
+      int m0, n0;
+      tile_mn(ti, m0, n0);
+      ok = mbar_wait_inline(&rfull[ti & 1], (ti >> 1) & 1, wc);
+      if (ok) ok = mbar_wait_inline(accfull, ti & 1, wc);
+      if (!ok) break;
+      tc_fence_after();
+      const float fm = rslot[(ti & 1) * BM + r].y;
+      const int m = m0 + r;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        uint32_t acc[32];
+        tmem_ld32(tbase + 32 * c, acc);
+        tmem_ld_wait_dep(acc);
+        if (c == 3) {
+          // the tile's accumulator has been read: the MMA may start the next tile
+          tc_fence_before();
+          warp_arrive(accempty);
+        }
+        const int nb = n0 + 128 * hf + 32 * c;
+        if (m < a.M) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int n = nb + 8 * j;
+            if (n >= a.N) continue;
+            const float4 f0 = *reinterpret_cast<const float4*>(a.fcol + n);
+            const float4 f1 = *reinterpret_cast<const float4*>(a.fcol + n + 4);
+            const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+            float y[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(acc[8 * j + t]) * fn[t]) * fm;
+            if (a.bias) {
+              const float4 b0 = *reinterpret_cast<const float4*>(a.bias + n);
+              const float4 b1 = *reinterpret_cast<const float4*>(a.bias + n + 4);
+              y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
+              y[4] += b1.x; y[5] += b1.y; y[6] += b1.z; y[7] += b1.w;
+            }
+            const size_t off = static_cast<size_t>(m) * a.N + n;
+            if (a.y_f32) {
+              float4* yp = reinterpret_cast<float4*>(static_cast<float*>(a.Y) + off);
+              yp[0] = make_float4(y[0], y[1], y[2], y[3]);
+              yp[1] = make_float4(y[4], y[5], y[6], y[7]);
+            } else {
+              *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
+                  make_uint4(f32x2_to_bf16x2(y[0], y[1]), f32x2_to_bf16x2(y[2], y[3]), f32x2_to_bf16x2(y[4], y[5]),
+                             f32x2_to_bf16x2(y[6], y[7]));
+            }
+          }
+        }
+      }
+      warp_arrive(&rempty[ti & 1]);
+    }
+    tmem_ld_wait();
   }
 
   __syncthreads();
   if (wid == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 512);
+    tmem_dealloc(tmem, TMEM_COLS);
   }
 }
 
 template <int G>
-cudaError_t launch_g(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, cudaStream_t s) {
+cudaError_t launch_g(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s) {
+  const ActLayout L = act_layout(h, M);
+  const uint8_t* base = static_cast<const uint8_t*>(ws);
   GemmArgs a;
   a.M = M;
   a.N = h.N;
   a.K = h.K;
-  a.nbs = (h.r_pad + 31) / 32;
-  a.m_tiles = (M + kBM - 1) / kBM;
-  a.n_tiles = (h.N + kBN - 1) / kBN;
+  a.r_pad = h.r_pad;
+  a.M_pad = L.M_pad;
+  a.nbs = (h.r_pad + KS - 1) / KS;
+  a.m_tiles = (M + BM - 1) / BM;
+  a.n_tiles = (h.N + BN - 1) / BN;
+  a.sx = reinterpret_cast<const __nv_bfloat16*>(base + L.scales_off);
+  a.phat = h.r_pad > 0 ? reinterpret_cast<const __half*>(base + L.phat_off) : nullptr;
+  a.fcol = h.fcol;
   a.Y = Y;
   a.y_f32 = y_f32 ? 1 : 0;
   a.bias = h.bias;
@@ -555,15 +568,15 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, c
   a.timeout_ns = deadline_budget_ns(h);
   static bool attr_done = false;
   if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+    cudaError_t e = cudaFuncSetAttribute(gemm16_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
   const int ntiles = a.m_tiles * a.n_tiles;
   const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
   // Without a branch the p_hat / B_hat maps are never used; any valid map fills the slots.
-  const CUtensorMap& ph = (h.r_pad > 0) ? am.ph32_map : am.qa_map;
-  const CUtensorMap& bh = (h.r_pad > 0) ? h.bh32_map : am.qa_map;
+  const CUtensorMap& ph = (h.r_pad > 0) ? am.ph64_map : am.qa_map;
+  const CUtensorMap& bh = (h.r_pad > 0) ? h.bhs_map : am.qa_map;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
@@ -574,14 +587,13 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, int M, void* Y, bool y_f32, c
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, gemm_kernel<G>, am.qa_map, h.qw_map, am.sx_map, h.sw32_map, ph, bh, a);
+  return cudaLaunchKernelEx(&cfg, gemm16_kernel<G>, am.qa_map, h.qw_map, am.sx_map, h.swh_map, ph, bh, a);
 }
 
 }  // namespace
 
 cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s) {
-  (void)ws;
-  return h.G == 32 ? launch_g<32>(h, am, M, Y, y_f32, s) : launch_g<64>(h, am, M, Y, y_f32, s);
+  return h.G == 32 ? launch_g<32>(h, am, ws, M, Y, y_f32, s) : launch_g<64>(h, am, ws, M, Y, y_f32, s);
 }
 
 }  // namespace qwam

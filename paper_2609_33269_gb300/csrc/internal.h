@@ -15,8 +15,8 @@ namespace qwam {
 constexpr int kBM = 128;        // token rows per CTA tile (one TMEM lane per row)
 constexpr int kChunk = 64;      // K columns per activation chunk (bf16: one 128-byte row)
 constexpr int kMaxRank = 64;    // largest rank of kernel (a)'s tensor-core path (above: the general-rank path)
-constexpr int kGemmBN = 128;    // output columns per GEMM CTA tile
-constexpr int kScaleGroups = 8; // groups per INT4 GEMM scale slot (s_x and the weight scale)
+constexpr int kGemmBN = 128;    // output columns per NVFP4 GEMM CTA tile
+constexpr int kGemm16BN = 256;  // output columns per INT4 GEMM CTA tile (float16 tensor-core kernel)
 
 // NVFP4 variant (App. B.1): E2M1 codes, one E4M3 scale per 16 consecutive K, one float32 scale per
 // weight tensor.  Block scales are stored in 512-byte atoms, one per 128 rows x 64 K: the four
@@ -29,21 +29,21 @@ enum Format : int { kFmtInt4 = 0, kFmtNvfp4 = 1 };
 
 inline int round_up(int a, int b) { return (a + b - 1) / b * b; }
 
-// INT4 codes are stored packed at four bits in SM4 words (sign-magnitude): word j of a row holds
-// k = 8j .. 8j+7.  Byte i carries code 8j+i in its sign bit 7 and magnitude bits 0-2, the
-// magnitude of code 8j+4+i in bits 4-6, and in bit 3 the sign of code 8j+4+((i+3) mod 4).  From
-// lo and hi, the E4M3 bytes (sign | magnitude, the value c 2^-9) of codes 8j..8j+3 and
-// 8j+4..8j+7, the word is lo | rotl(hi, 4); back: lo = w & 0x87878787, hi = rotr(w, 4) & 0x87878787.
-__host__ __device__ inline uint32_t sm4_pack(uint32_t lo, uint32_t hi) { return lo | (hi << 4) | (hi >> 28); }
-// E4M3 byte (sign | magnitude) of an integer code in [-7, 7].
-__host__ __device__ inline uint32_t sm4_byte(int c) {
-  return static_cast<uint32_t>(c < 0 ? -c : c) | (c < 0 ? 0x80u : 0u);
+// INT4 codes are stored packed at four bits in OB4 words (offset binary): word j of a row holds
+// k = 8j .. 8j+7 as nibbles c + 8 in [1, 15], k = 8j + 2p in bits 4p .. 4p+3 and k = 8j + 2p + 1
+// in bits 16 + 4p .. 16 + 4p + 3 (p = 0..3).  Pair p then becomes the float16 pair
+// (c_{8j+2p}, c_{8j+2p+1}) in one 32-bit register with one shift, one and-or with
+// 0x000F000F / 0x64006400 (0x6400 | n is the float16 value 1024 + n) and one float16 subtraction of
+// 1032.  A zero word (TMA fill outside the tensor) decodes to -8 everywhere, and its scale to 0.
+__host__ __device__ inline uint32_t ob4_word(const int (&c)[8]) {
+  uint32_t w = 0;
+  for (int p = 0; p < 4; ++p)
+    w |= (static_cast<uint32_t>(c[2 * p] + 8) << (4 * p)) | (static_cast<uint32_t>(c[2 * p + 1] + 8) << (16 + 4 * p));
+  return w;
 }
-// Position of weight-scale column n within its 32-column block in the GEMM's float32 copy: the
-// epilogue thread with q = (n % 8) / 2 reads columns 8j + 2q + {0, 1} (j = 0..3) as 8 floats.
-__host__ __device__ inline int sigma_pos(int n) {
-  const int t = n & 31;
-  return (n & ~31) + 8 * ((t & 7) >> 1) + 2 * (t >> 3) + (t & 1);
+// Code k (0..7) of an OB4 word.
+__host__ __device__ inline int ob4_code(uint32_t w, int k) {
+  return static_cast<int>((w >> ((k & 1) * 16 + (k >> 1) * 4)) & 0xFu) - 8;
 }
 
 // Activation-side tensor maps for one (workspace, X, M) triple.
@@ -52,10 +52,10 @@ struct ActMaps {
   const void* x = nullptr;
   int M = -1;
   CUtensorMap x_map;    // X bf16 [M, K], box {64, 128}, 128-byte swizzle
-  CUtensorMap qa_map;   // INT4: packed SM4 codes [M, K/2] bytes, box {64, 128}
-  CUtensorMap sx_map;   // INT4: s_x f32 [K/G, M_pad], box {128, kScaleGroups}
+  CUtensorMap qa_map;   // INT4: packed OB4 codes [M, K/2] bytes, box {32, 128}
+  CUtensorMap sx_map;   // INT4: s_x bf16 [K/G, M] (row pitch M_pad), box {128, 64/G}: one GEMM stage's groups
   CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128} (NVFP4 GEMM)
-  CUtensorMap ph32_map; // p_hat f16 [M, r_pad], box {32, 128} (INT4 GEMM)
+  CUtensorMap ph64_map; // p_hat f16 [M, r_pad], box {64, 128}, 128-byte swizzle (INT4 GEMM)
   CUtensorMap qx4_map;  // NVFP4 codes [M, K/2] bytes, box {128, 128}, 128-byte swizzle
 };
 
@@ -65,11 +65,15 @@ struct Handle {
   int device = 0;
   int num_sms = 148;
   void* block = nullptr;             // one device allocation holding every buffer below
-  uint8_t* qw = nullptr;             // INT4: [N_pad, K/2] SM4 words (word j of a row: k = 8j..8j+7,
-                                     // see sm4_pack); NVFP4: E2M1 codes, low nibble = even k
-  __half* sw = nullptr;              // [K/G, N_pad]
-  float* sw32 = nullptr;             // [K/G, N_pad]: sigma = 2^18 s_w in float32 (GEMM epilogue), each
-                                     // 32-column block permuted: column 8j + 2q + b at 8q + 2j + b
+  uint8_t* qw = nullptr;             // INT4: [N_pad, K/2] OB4 words (word j of a row: k = 8j..8j+7,
+                                     // see ob4_word); NVFP4: E2M1 codes, low nibble = even k
+  __nv_bfloat16* sw = nullptr;       // INT4: s_w [K/G, N_pad], bfloat16
+  // The INT4 GEMM's copies, scaled per output column n by 2^e_n (e_n chosen so that the column's
+  // largest dequantized value 7 s_w, or its largest |B_hat|, lies in [2^10, 2^11)): float16
+  // s_w 2^e_n [K/G, N_pad] and B_hat 2^e_n [N_pad, r_pad], and the float32 factor 2^-e_n [N_pad].
+  __half* swh = nullptr;
+  __half* Bhs = nullptr;
+  float* fcol = nullptr;
   __half* Bh = nullptr;              // [N_pad, r_pad]
   __nv_bfloat16* ucat_t = nullptr;   // [2 r_pad, K]: rows 0..r_pad-1 = U_hi^T, then U_lo^T
   __nv_bfloat16* ucat3 = nullptr;    // [K, ku3]: row k = U_hi[k,:], U_lo[k,:], U_hi[k,:], zeros
@@ -94,17 +98,17 @@ struct Handle {
   float* ur32 = nullptr;             // [r_pad, K] float32 reconstruction basis (U, or diag(s) H U), transposed
   int small_m = 256;                 // token counts up to this take the small-M activation kernel
   double timeout_s = 2.0;
-  CUtensorMap qw_map;                // INT4 weight codes [N, K/2] bytes, box {64, 128}
-  CUtensorMap sw32_map;              // sigma [K/G, N], box {128, kScaleGroups}
+  CUtensorMap qw_map;                // INT4 weight codes [N_pad, K/2] bytes, box {32, 256}
+  CUtensorMap swh_map;               // s_w 2^e_n f16 [K/G, N_pad], box {256, 64/G}: one GEMM stage's groups
   CUtensorMap Bh_map;                // B_hat [N, r_pad] f16, box {8, 128} (NVFP4 GEMM)
-  CUtensorMap bh32_map;              // B_hat [N, r_pad] f16, box {32, 128} (INT4 GEMM)
+  CUtensorMap bhs_map;               // B_hat 2^e_n [N_pad, r_pad] f16, box {64, 256}, 128-byte swizzle
   CUtensorMap ucat_t_map, ucat3_map;
   CUtensorMap qw4_map;               // NVFP4 weight codes [N, K/2], box {128, 128}, 128-byte swizzle
   ActMaps act_cache[4];
   int act_next = 0;
 };
 
-// Workspace of M tokens.  INT4: packed SM4 codes [M, K/2], s_x f32 [K/G, M_pad], p_hat f16
+// Workspace of M tokens.  INT4: packed OB4 codes [M, K/2], s_x bf16 [K/G, M_pad], p_hat f16
 // [M, r_pad]; NVFP4: E2M1 codes [M, K/2], scale atoms, p_hat.  ab_off = phat_off (no region).
 struct ActLayout {
   size_t codes_off, scales_off, ab_off, phat_off, bytes;

@@ -48,51 +48,94 @@ __device__ __forceinline__ double wperp(const WT* __restrict__ W, const float* _
   return __dsub_rn(wval(W, static_cast<size_t>(k) * N + n), acc);
 }
 
-// Nearest integer to the exact quotient w / s, ties to even.  s is a float16 value and w a
-// float64 with |w| <= ~7.5 s, so c * s and w - c * s are exact in float64 and the remainder
-// decides the rounding.
+// Nearest code in [-7, 7] to the exact quotient w / s, ties to even (saturating, which only a
+// bfloat16-subnormal scale can need).  s is a bfloat16 value and w a float64 with |w| <= ~9 s,
+// so c * s and w - c * s are exact in float64 and the remainder decides the rounding.
 __device__ __forceinline__ int nearest_code_f64(double w, double s) {
   double c = rint(__ddiv_rn(w, s));
   double e = __dsub_rn(w, __dmul_rn(c, s));
   double t = 2.0 * fabs(e);
   bool odd = (static_cast<long long>(c) & 1LL) != 0;
   if (t > s || (t == s && odd)) c = __dadd_rn(c, e > 0.0 ? 1.0 : -1.0);
-  return static_cast<int>(c);
+  return min(7, max(-7, static_cast<int>(c)));
 }
 
-// One thread per (output channel n, group g): s_w = RN_f16(absmax / 7), codes packed 4 bits
-// each into qw[n, :] as SM4 words (sm4_pack: word j holds k = 8j..8j+7, sign-magnitude, so that
-// the GEMM expands a word to its eight E4M3 bytes with one funnel shift and two masks).
+// s_w = RN_bf16(a / 7) of the exact quotient (a >= 0, float64), ties to even.  The float64
+// quotient q is within half a float64 unit of a / 7; if q is on the bfloat16 grid it is the
+// answer, else the grid points n u < q < (n + 1) u (u = 2^(E - 7) for q in [2^E, 2^(E+1)), and
+// 2^-133 below 2^-126) are decided by comparing a with 7 (n + 1/2) u, exact in float64.  Returns
+// the bfloat16; infinity above the largest finite bfloat16.
+__device__ __forceinline__ __nv_bfloat16 bf16_div7_f64(double a) {
+  if (!(a > 0.0)) return __float2bfloat16_rn(0.0f);
+  const double q = __ddiv_rn(a, 7.0);
+  int E = ilogb(q);
+  if (E < -126) E = -126;
+  const double u = ldexp(1.0, E - 7);
+  const double n = floor(__dmul_rn(q, ldexp(1.0, 7 - E)));
+  double v = __dmul_rn(n, u);
+  if (v != q) {
+    const double t = __dmul_rn(7.0, __dmul_rn(__dadd_rn(n, 0.5), u));
+    const bool up = a > t || (a == t && fmod(n, 2.0) != 0.0);
+    if (up) v = __dmul_rn(__dadd_rn(n, 1.0), u);
+  }
+  if (v > 3.3895313892515355e38) return __ushort_as_bfloat16(static_cast<unsigned short>(0x7f80));
+  return __float2bfloat16_rn(static_cast<float>(v));  // exact: v lies on the bfloat16 grid
+}
+
+// One thread per (output channel n, group g): s_w = RN_bf16(absmax / 7), codes packed 4 bits
+// each into qw[n, :] as OB4 words (ob4_word: word j holds k = 8j..8j+7 as offset-binary nibbles,
+// the form the GEMM turns into float16 pairs).
 template <typename WT>
 __global__ void quantize_weight_kernel(const WT* __restrict__ W, const float* __restrict__ U,
                                        const double* __restrict__ Bf, int K, int N, int r, int G, int N_pad,
-                                       uint8_t* __restrict__ qw, __half* __restrict__ sw, float* __restrict__ sw32,
-                                       int* err) {
+                                       uint8_t* __restrict__ qw, __nv_bfloat16* __restrict__ sw, int* err) {
   int n = blockIdx.x * blockDim.x + threadIdx.x;
   int g = blockIdx.y;
   if (n >= N) return;
   double amax = 0.0;
   for (int k = g * G; k < (g + 1) * G; ++k) amax = fmax(amax, fabs(wperp(W, U, Bf, N, r, k, n)));
-  __half sh = __double2half(__ddiv_rn(amax, 7.0));
-  double s = static_cast<double>(__half2float(sh));
-  sw[static_cast<size_t>(g) * N_pad + n] = sh;
-  // sigma = 2^18 s_w (exact), at the permuted position the GEMM epilogue reads
-  sw32[static_cast<size_t>(g) * N_pad + sigma_pos(n)] = static_cast<float>(s) * 262144.0f;
+  const __nv_bfloat16 sb = bf16_div7_f64(amax);
+  const double s = static_cast<double>(__bfloat162float(sb));
+  sw[static_cast<size_t>(g) * N_pad + n] = sb;
   bool ok_scale = isfinite(s);
   if (!ok_scale) atomicOr(err, kErrRange);
   uint32_t* row = reinterpret_cast<uint32_t*>(qw + static_cast<size_t>(n) * (K / 2));
   for (int k = g * G; k < (g + 1) * G; k += 8) {
-    uint32_t lo = 0, hi = 0;
+    int c[8];
     for (int i = 0; i < 8; ++i) {
-      int c = 0;
-      if (s > 0.0 && ok_scale) c = nearest_code_f64(wperp(W, U, Bf, N, r, k + i, n), s);
-      if (c < -7 || c > 7) atomicOr(err, kErrRange);
-      if (i < 4)
-        lo |= sm4_byte(c) << (8 * i);
-      else
-        hi |= sm4_byte(c) << (8 * (i - 4));
+      c[i] = 0;
+      if (s > 0.0 && ok_scale) c[i] = nearest_code_f64(wperp(W, U, Bf, N, r, k + i, n), s);
     }
-    row[k / 8] = sm4_pack(lo, hi);
+    row[k / 8] = ob4_word(c);
+  }
+}
+
+// The INT4 GEMM's per-column copies (one thread per column n < N_pad): with
+// b_n = max(7 max_g s_w[g, n], max_j |B_hat[n, j]|), e_n = 10 - floor(log2 b_n) clamped to
+// [-126, 126] (0 for an all-zero column), s_w 2^e_n and B_hat 2^e_n rounded to float16 (exact
+// while they stay above 2^-21 and 2^-24 of the column's largest value, which lies in
+// [2^10, 2^11)) and the float32 factor 2^-e_n that the epilogue applies.
+__global__ void column_shift_kernel(const __nv_bfloat16* __restrict__ sw, const __half* __restrict__ Bh, int ng,
+                                    int N_pad, int r_pad, __half* __restrict__ swh, __half* __restrict__ Bhs,
+                                    float* __restrict__ fcol) {
+  const int n = blockIdx.x * blockDim.x + threadIdx.x;
+  if (n >= N_pad) return;
+  double b = 0.0;
+  for (int g = 0; g < ng; ++g)
+    b = fmax(b, __dmul_rn(7.0, static_cast<double>(__bfloat162float(sw[static_cast<size_t>(g) * N_pad + n]))));
+  for (int j = 0; j < r_pad; ++j)
+    b = fmax(b, fabs(static_cast<double>(__half2float(Bh[static_cast<size_t>(n) * r_pad + j]))));
+  int e = 0;
+  if (b > 0.0) e = min(126, max(-126, 10 - ilogb(b)));
+  fcol[n] = static_cast<float>(ldexp(1.0, -e));
+  const double f = ldexp(1.0, e);
+  for (int g = 0; g < ng; ++g) {
+    const size_t i = static_cast<size_t>(g) * N_pad + n;
+    swh[i] = __double2half(__dmul_rn(static_cast<double>(__bfloat162float(sw[i])), f));
+  }
+  for (int j = 0; j < r_pad; ++j) {
+    const size_t i = static_cast<size_t>(n) * r_pad + j;
+    Bhs[i] = __double2half(__dmul_rn(static_cast<double>(__half2float(Bh[i])), f));
   }
 }
 
@@ -321,7 +364,7 @@ cudaError_t pack_int4(Handle& h, const WT* W, const float* U, const float* Up, c
   if (r > 0) {
     branch_weight_kernel<<<dim3((N + T - 1) / T, r), T, 0, s>>>(W, U, K, N, r, Bf);
   }
-  quantize_weight_kernel<<<dim3((N + T - 1) / T, K / h.G), T, 0, s>>>(W, U, Bf, K, N, r, h.G, h.N_pad, h.qw, h.sw, h.sw32,
+  quantize_weight_kernel<<<dim3((N + T - 1) / T, K / h.G), T, 0, s>>>(W, U, Bf, K, N, r, h.G, h.N_pad, h.qw, h.sw,
                                                                      h.err);
   if (r > 0) {
     branch_half_kernel<<<(N + T - 1) / T, T, 0, s>>>(Bf, N, r, h.r_pad, h.Bh, h.err);
@@ -329,6 +372,7 @@ cudaError_t pack_int4(Handle& h, const WT* W, const float* U, const float* Up, c
       split_basis_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.ku3, h.ucat_t, h.ucat3);
     basis32_kernel<<<(K + T - 1) / T, T, 0, s>>>(Up, Ur, K, r, h.r_pad, h.up32, h.ur32);
   }
+  column_shift_kernel<<<(h.N_pad + T - 1) / T, T, 0, s>>>(h.sw, h.Bh, K / h.G, h.N_pad, h.r_pad, h.swh, h.Bhs, h.fcol);
   e = cudaGetLastError();
   cudaError_t e2 = cudaStreamSynchronize(s);
   cudaFree(Bf);

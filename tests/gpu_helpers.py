@@ -2,6 +2,8 @@
 nibble unpacking and the comparison rules."""
 from __future__ import annotations
 
+import math
+
 import numpy as np
 import torch
 
@@ -14,21 +16,18 @@ def to_dev_bf16(bits: np.ndarray) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).cuda().view(torch.bfloat16)
 
 
-def decode_sm4(packed: np.ndarray) -> np.ndarray:
-    """INT4 codes packed as SM4 words, uint8 [R, K/2] -> int8 [R, K].
+def decode_ob4(packed: np.ndarray) -> np.ndarray:
+    """INT4 codes packed as OB4 words, uint8 [R, K/2] -> int8 [R, K].
 
-    Word j of a row (little-endian 32 bits) holds k = 8j..8j+7: the E4M3 bytes (sign bit 7 |
-    magnitude bits 0-2) of k = 8j..8j+3 are word & 0x87878787 and those of k = 8j+4..8j+7 are
-    rotr(word, 4) & 0x87878787."""
+    Word j of a row (little-endian 32 bits) holds k = 8j..8j+7 as offset-binary nibbles c + 8:
+    code 8j + 2p in bits 4p..4p+3 and code 8j + 2p + 1 in bits 16 + 4p..16 + 4p + 3."""
     p = np.ascontiguousarray(packed, np.uint8)
-    w = p.view("<u4").astype(np.uint64)
-    lo = (w & 0x87878787).astype(np.uint32)
-    hi = (((w >> 4) | (w << 28)) & 0x87878787).astype(np.uint32)
-    b = np.empty((p.shape[0], w.shape[1], 8), np.uint8)
-    b[:, :, :4] = lo[:, :, None].view(np.uint8).reshape(p.shape[0], -1, 4)
-    b[:, :, 4:] = hi[:, :, None].view(np.uint8).reshape(p.shape[0], -1, 4)
-    mag = (b & 0x7).astype(np.int8)
-    return np.where(b & 0x80, -mag, mag).astype(np.int8).reshape(p.shape[0], -1)
+    w = p.view("<u4")
+    out = np.empty((p.shape[0], w.shape[1], 8), np.int8)
+    for q in range(4):
+        out[:, :, 2 * q] = ((w >> (4 * q)) & 0xF).astype(np.int16) - 8
+        out[:, :, 2 * q + 1] = ((w >> (16 + 4 * q)) & 0xF).astype(np.int16) - 8
+    return out.reshape(p.shape[0], -1)
 
 
 def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
@@ -90,8 +89,8 @@ class Case:
     def gpu_act(self, rows=None):
         codes, scales, ph = self.layer.act_views(self.M)
         torch.cuda.synchronize()
-        qx = decode_sm4(codes.cpu().numpy())
-        sx = scales.cpu().numpy()[:, :self.M].T.copy()
+        qx = decode_ob4(codes.cpu().numpy())
+        sx = scales.float().cpu().numpy()[:, :self.M].T.copy()
         phv = ph.cpu().numpy().view(np.uint16)[:, :self.r].copy()
         if rows is not None:
             qx, sx, phv = qx[rows], sx[rows], phv[rows]
@@ -120,6 +119,15 @@ def rowwise_rel_err(Y, ref):
     return d / np.maximum(n, 1e-30)
 
 
+def gemm_tol(K, r_pad=0):
+    """Bound on max |Y - Yk| / max |Yk| per row, Yk the oracle's output on the kernel's own codes,
+    scales and branch inputs.  The kernel forms every product exactly (float16 x float16) and adds
+    the K + r_pad of them into one float32 accumulator, 16 per MMA step; a rounding of 2^-24 of the
+    running sum per step grows like sqrt((K + r_pad) / 16) 2^-24 times the sum's scale, and
+    4e-7 sqrt(K + r_pad) is about four times the largest error measured (K = 12288)."""
+    return max(1e-5, 4e-7 * math.sqrt(K + r_pad))
+
+
 def near_tie_mismatches(q_gpu, q_ref, x_ref, s_ref, G, eps_rel):
     """Indices where the codes differ, and whether each lies within eps (relative to the scale)
     of a rounding boundary of the reference remainder x_ref / s_ref."""
@@ -132,17 +140,55 @@ def near_tie_mismatches(q_gpu, q_ref, x_ref, s_ref, G, eps_rel):
     return bad, np.array(ok, bool)
 
 
-def check_layer_output(Y, Yo, Yk, qx_gpu, qx_oracle):
-    """Rows whose activation codes all equal the oracle's meet max |dY| <= 1e-3 |y|inf against
-    the oracle.  A row holding a near-tie flip (checked separately) differs from the oracle by
-    that flip's weight column times s_x s_w, which can exceed 1e-3 in an outlier group; such a
-    row must equal the oracle evaluated on the kernel's own codes (1e-5)."""
-    flip = np.any(qx_gpu != qx_oracle, axis=1)
+def _bf16_bits(v):
+    return int(np.float32(v).view(np.uint32)) >> 16
+
+
+def check_int4_act(ga, oa, G):
+    """INT4 activation codes and scales at r > 0 against the oracle's (readings R2, R3, R5), with
+    oa the oracle's float64 path (Xperp and p).  The kernel's float32 remainder is within
+    2e-5 max|x| of the oracle's (asserted by the residual tests), and max|x| <= max|Xperp| + |p|.
+
+    * A scale may differ only by one bfloat16 step, and only where the oracle's amax / 7 lies
+      within that remainder error (over 7) of the midpoint between the two values.
+    * A code in a group whose scale agrees may differ only within 1e-3 (relative to the scale) of
+      a rounding boundary of the oracle's quotient; codes of a group whose scale differs follow
+      that scale (the quantizer on the kernel's own remainder is checked bit for bit elsewhere).
+    * At most max(2, 1e-2 groups) scales and max(2, 1e-4 codes) codes differ.
+    Returns a bool per row: any code or scale of the row differs."""
+    Xp = np.asarray(oa["Xperp"], np.float64)
+    M, K = Xp.shape
+    pn = np.linalg.norm(oa["p"], axis=1) if oa["p"].size else np.zeros(M)
+    delta = 2e-5 * (np.abs(Xp).max(axis=1) + pn)
+    amax = np.abs(Xp).reshape(M, K // G, G).max(axis=2)
+    sg, so = np.asarray(ga["sx"], np.float32), np.asarray(oa["sx"], np.float32)
+    sdiff = sg != so
+    sbad = np.argwhere(sdiff)
+    for m, g in sbad:
+        bg, bo = _bf16_bits(sg[m, g]), _bf16_bits(so[m, g])
+        assert abs(int(bg) - int(bo)) == 1, (m, g, sg[m, g], so[m, g])
+        mid = (float(sg[m, g]) + float(so[m, g])) / 2
+        assert abs(amax[m, g] / 7 - mid) <= delta[m] / 7, (m, g, amax[m, g] / 7, mid, delta[m])
+    assert len(sbad) <= max(2, 1e-2 * sg.size), len(sbad)
+    same = np.repeat(~sdiff, G, axis=1)
+    qbad, qnear = near_tie_mismatches(np.where(same, ga["qx"], 0), np.where(same, oa["qx"], 0), Xp,
+                                      oa["sx"], G, 1e-3)
+    assert qnear.all(), qbad[~qnear][:5]
+    assert len(qbad) <= max(2, 1e-4 * ga["qx"].size), len(qbad)
+    return np.any(ga["qx"] != oa["qx"], axis=1) | np.any(sdiff, axis=1)
+
+
+def check_layer_output(Y, Yo, Yk, flip, tol_k=1e-5):
+    """Rows whose activation codes and scales all equal the oracle's meet max |dY| <= 1e-3 |y|inf
+    against the oracle.  A row holding a near-tie flip (checked separately) differs from the
+    oracle by that flip's weight column times s_x s_w, which can exceed 1e-3 in an outlier group;
+    such a row must equal the oracle evaluated on the kernel's own codes (tol_k, see gemm_tol)."""
+    flip = np.asarray(flip, bool)
     e = rowwise_rel_err(Y, Yo)
     if (~flip).any():
         assert e[~flip].max() <= 1e-3, e[~flip].max()
     if flip.any():
-        assert rowwise_rel_err(Y[flip], Yk[flip]).max() <= 1e-5
+        assert rowwise_rel_err(Y[flip], Yk[flip]).max() <= tol_k
     assert flip.mean() <= 0.05, flip.mean()
 
 

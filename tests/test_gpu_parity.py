@@ -18,7 +18,8 @@ import oracle
 from paper_2609_33269_gb300 import asp
 from paper_2609_33269_gb300 import workloads as wl
 
-from gpu_helpers import Case, check_layer_output, near_tie_mismatches, rowwise_rel_err, to_dev_bf16, unpack_nibbles
+from gpu_helpers import (Case, check_int4_act, check_layer_output, gemm_tol, rowwise_rel_err, to_dev_bf16,
+                         unpack_nibbles)
 
 pytestmark = pytest.mark.gpu
 
@@ -111,17 +112,16 @@ def test_end_to_end_codes_and_output(shape):
         if r == 0:
             np.testing.assert_array_equal(ga["qx"], oa["qx"])
             np.testing.assert_array_equal(ga["sx"], oa["sx"])
+            flip = np.zeros(M, bool)
         else:
-            np.testing.assert_allclose(ga["sx"], oa["sx"], rtol=1e-4, atol=0)
-            bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], G, 1e-3)
-            assert len(bad) <= max(1, 1e-4 * ga["qx"].size), len(bad)
-            assert near.all()
+            flip = check_int4_act(ga, oa, G)
+        tol = gemm_tol(K, -(-r // 16) * 16)
         # the GEMM alone: oracle output from the kernel's own codes, scales and branch input
         Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), G)
-        assert rowwise_rel_err(Y, Yk).max() <= 1e-5
+        assert rowwise_rel_err(Y, Yk).max() <= tol
         # the whole layer against the oracle
         Yo = oracle.linear(oa, ow, G)
-        check_layer_output(Y, Yo, Yk, ga["qx"], oa["qx"])
+        check_layer_output(Y, Yo, Yk, flip, tol)
         # bf16 output is the float32 output rounded once
         Yb = c.run(fp32=False)
         ref = torch.from_numpy(Y).cuda().to(torch.bfloat16)
@@ -200,14 +200,16 @@ def test_full_size_sampled_rows(cfg):
         np.testing.assert_array_equal(gw["qw"], ow["qw"])
         np.testing.assert_array_equal(gw["sw"], ow["sw"])
         oa = c.oracle_act(rows)
+        tol = gemm_tol(K, -(-r // 16) * 16)
         Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), G)
-        assert rowwise_rel_err(Y[rows], Yk).max() <= 1e-5
+        assert rowwise_rel_err(Y[rows], Yk).max() <= tol
         Yo = oracle.linear(oa, ow, G)
-        check_layer_output(Y[rows], Yo, Yk, ga["qx"], oa["qx"])
         if r == 0:
             np.testing.assert_array_equal(ga["qx"], oa["qx"])
+            np.testing.assert_array_equal(ga["sx"], oa["sx"])
+            flip = np.zeros(len(rows), bool)
         else:
-            bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], G, 1e-3)
-            assert len(bad) <= max(2, 1e-4 * ga["qx"].size) and near.all()
+            flip = check_int4_act(ga, oa, G)
+        check_layer_output(Y[rows], Yo, Yk, flip, tol)
     finally:
         c.close()

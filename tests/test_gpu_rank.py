@@ -20,7 +20,7 @@ import oracle
 from paper_2609_33269_gb300 import asp
 from paper_2609_33269_gb300 import workloads as wl
 
-from gpu_helpers import Case, NvCase, check_layer_output, check_nvfp4_activations, near_tie_mismatches, rowwise_rel_err
+from gpu_helpers import Case, NvCase, check_int4_act, check_layer_output, check_nvfp4_activations, gemm_tol, rowwise_rel_err
 
 pytestmark = pytest.mark.gpu
 
@@ -78,12 +78,11 @@ def test_int4_end_to_end(shape):
         oa, ow = c.oracle_act(), c.oracle_weights()
         np.testing.assert_array_equal(gw["qw"], ow["qw"])
         np.testing.assert_array_equal(gw["Bh"], ow["Bh"])
-        bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], G, 1e-3)
-        assert len(bad) <= max(1, 1e-4 * ga["qx"].size), len(bad)
-        assert near.all()
+        flip = check_int4_act(ga, oa, G)
+        tol = gemm_tol(K, -(-r // 16) * 16)
         Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), G)
-        assert rowwise_rel_err(Y, Yk).max() <= 1e-5
-        check_layer_output(Y, oracle.linear(oa, ow, G), Yk, ga["qx"], oa["qx"])
+        assert rowwise_rel_err(Y, Yk).max() <= tol
+        check_layer_output(Y, oracle.linear(oa, ow, G), Yk, flip, tol)
         Yb = c.run(fp32=False)
         assert torch.equal(Yb.view(torch.int16), torch.from_numpy(Y).cuda().to(torch.bfloat16).view(torch.int16))
         assert asp.qwam_asp_get_error(c.layer.h) == asp.QWAM_OK
@@ -103,7 +102,10 @@ def test_int4_r_equals_K_gives_the_16_bit_gemm(K, G):
         W = wl.bf16_bits_to_f32(c.Wb).astype(np.float64)
         assert np.abs(R).max() <= 1e-4 * np.abs(X).max()
         gw = c.gpu_weights()
-        assert not gw["qw"].any() and not gw["sw"].any()  # W_perp = 0: the 4-bit part vanishes
+        # W_perp is float64 roundoff of the float32 basis: the 4-bit part is negligible (its
+        # bfloat16 scales are tiny, not zero: bfloat16 has float32's exponent range)
+        sw = wl.bf16_bits_to_f32(gw["sw"]).astype(np.float64)
+        assert 7 * sw.max() <= 2e-5 * np.abs(W).max()
         Yo = oracle.linear(c.oracle_act(), c.oracle_weights(), G)
         assert rowwise_rel_err(Y, Yo).max() <= 1e-3
         assert rowwise_rel_err(Y, X @ W).max() <= 5e-3

@@ -21,7 +21,7 @@ import oracle
 from paper_2609_33269_gb300 import asp
 from paper_2609_33269_gb300 import workloads as wl
 
-from gpu_helpers import (Case, atoms_to_rows, check_layer_output, check_nvfp4_activations, near_tie_mismatches,
+from gpu_helpers import (Case, atoms_to_rows, check_int4_act, check_layer_output, check_nvfp4_activations, gemm_tol,
                          rowwise_rel_err, to_dev_bf16, unpack_e2m1)
 
 pytestmark = pytest.mark.gpu
@@ -123,13 +123,13 @@ def test_rotated_end_to_end(shape, small):
         Y = c.run(fp32=True).cpu().numpy()
         ga, gw = c.gpu_act(), c.gpu_weights()
         oa, ow = c.oracle_act(), c.oracle_weights()
-        bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], G, 1e-3)
-        assert len(bad) <= max(1, 1e-4 * ga["qx"].size), len(bad)
-        assert near.all()
+        # the rotated remainder is a float64 value on the oracle's side even at r = 0
+        flip = check_int4_act(ga, oa, G)
+        tol = gemm_tol(K, -(-r // 16) * 16)
         Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), G)
-        assert rowwise_rel_err(Y, Yk).max() <= 1e-5
+        assert rowwise_rel_err(Y, Yk).max() <= tol
         Yo = oracle.linear(oa, ow, G)
-        check_layer_output(Y, Yo, Yk, ga["qx"], oa["qx"])
+        check_layer_output(Y, Yo, Yk, flip, tol)
         Yb = c.run(fp32=False)
         assert torch.equal(Yb.view(torch.int16), torch.from_numpy(Y).cuda().to(torch.bfloat16).view(torch.int16))
     finally:
@@ -161,11 +161,11 @@ def test_rotated_full_size_sampled_rows():
         np.testing.assert_array_equal(gw["sw"], ow["sw"])
         np.testing.assert_array_equal(gw["Bh"], ow["Bh"])
         oa = c.oracle_act(rows)
+        tol = gemm_tol(K, 32)
         Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), G)
-        assert rowwise_rel_err(Y[rows], Yk).max() <= 1e-5
-        check_layer_output(Y[rows], oracle.linear(oa, ow, G), Yk, ga["qx"], oa["qx"])
-        bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], G, 1e-3)
-        assert len(bad) <= max(2, 1e-4 * ga["qx"].size) and near.all()
+        assert rowwise_rel_err(Y[rows], Yk).max() <= tol
+        flip = check_int4_act(ga, oa, G)
+        check_layer_output(Y[rows], oracle.linear(oa, ow, G), Yk, flip, tol)
     finally:
         c.close()
 

@@ -8,10 +8,11 @@ where they hand over to exact decisions, so the values here are placed on and ne
 boundaries themselves:
 
 * INT4 (Eq. (quant), readings R2/R3/R5): code = nearest integer to x / s, ties to even, with
-  s = RN_f32(amax / 7).  Values sit at (c + 1/2) s exactly (scales with few significant bits make
-  these products exact, so they are true ties) and one to three float32 steps either side of the
-  rounded product for scales with many significant bits; groups of zeros and groups small enough
-  to take the power-of-two rescaling path are included.
+  s = RN_bf16(amax / 7) of the exact quotient.  Values sit at (c + 1/2) s exactly (a bfloat16 s
+  makes these products exact, so they are true ties) and one to three float32 steps either side,
+  for scales from absmaxes of few and of many significant bits; groups of zeros, groups small
+  enough to take the power-of-two rescaling path, and a float32 subnormal absmax whose quotient
+  rounded to float32 would sit on a bfloat16 midpoint are included.
 * NVFP4 (App. B.1, readings N1-N3): code = RN_e2m1(RN_f32(x / s)), s = RN_e4m3(RN_f32(amax / 6)).
   Values sit on every E2M1 midpoint m (m s is exact for an E4M3 s), one to four float32 steps
   from it (where the float32 quotient can round onto the midpoint and become a tie), at relative
@@ -25,7 +26,7 @@ import torch
 import oracle
 from paper_2609_33269_gb300 import asp
 
-from gpu_helpers import decode_sm4
+from gpu_helpers import decode_ob4
 
 pytestmark = pytest.mark.gpu
 
@@ -64,20 +65,25 @@ def fill(vals, size, amax, rng):
     return out
 
 
+def bf16_scale(A):
+    """The oracle's scale RN_bf16(A / 7) as a float32 value."""
+    return np.array([oracle.bf16_bits_div7(float(f32(A))) << 16], np.uint32).view(np.float32)[0]
+
+
 def int4_groups(G, rng):
     groups = []
     # exact ties: scales with few significant bits, amax = 7 s exactly
     for s_t in (0.375, 1.0, 0.0625, 3.0, 5.0 * 2.0 ** -20, 0.8125):
         s = f32(s_t)
         A = f32(7 * s)
-        assert f32(np.float64(A) / 7) == s
+        assert bf16_scale(A) == s
         vals = [(c + 0.5) * s for c in range(-7, 7)] + [-(c + 0.5) * s for c in range(0, 7)]
         vals += [c * s for c in range(-7, 8)]
         groups.append(fill(vals, G, A, rng))
         groups.append(fill([-v for v in vals], G, -A, rng))
-    # near ties: many-bit scales; the float32 product and its neighbours
+    # near ties: absmaxes of many significant bits; the ties (c + 1/2) s and their neighbours
     for A in (1.0, 2.9, 0.123456, 17.77, 3.3e-5, 1234.5678):
-        s = f32(np.float64(f32(A)) / 7)
+        s = bf16_scale(A)
         vals = []
         for c in range(-7, 7):
             t = f32((c + 0.5) * np.float64(s))
@@ -85,9 +91,10 @@ def int4_groups(G, rng):
         for i in range(0, len(vals), G - 1):
             groups.append(fill(vals[i:i + G - 1], G, A, rng))
     groups.append(np.zeros(G, np.float32))
-    # tiny groups: the scale is below 2^-100 and the codes are formed on rescaled values
-    for A in (3e-33, 7.5e-36):
-        s = f32(np.float64(f32(A)) / 7)
+    # tiny groups: the scale is below 2^-100 and the codes are formed on rescaled values; the
+    # last absmax is a float32 subnormal whose exact quotient lies just above a bfloat16 midpoint
+    for A in (3e-33, 7.5e-36, 1146881 * 2.0 ** -149):
+        s = bf16_scale(A)
         vals = []
         for c in range(-7, 7):
             t = f32((c + 0.5) * np.float64(s))
@@ -158,10 +165,10 @@ def run_lanes(R, fmt, G):
         sf = a[((r // 128) * (K // 64) + b // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + b % 4]
         return codes.cpu().numpy(), sf
     codes = torch.zeros((M, K // 2), dtype=torch.uint8, device="cuda")
-    scales = torch.zeros((K // G, M_pad), dtype=torch.float32, device="cuda")
+    scales = torch.zeros((K // G, M_pad), dtype=torch.bfloat16, device="cuda")
     asp.qwam_asp_debug_quantize_lanes(Rd, M, K, fmt, G, codes, scales)
     torch.cuda.synchronize()
-    return decode_sm4(codes.cpu().numpy()), scales.cpu().numpy()[:, :M].T.copy()
+    return decode_ob4(codes.cpu().numpy()), scales.float().cpu().numpy()[:, :M].T.copy()
 
 
 IMPLS = {"thread_rows": None, "warp_lanes": run_lanes}
@@ -177,11 +184,13 @@ def run(R, fmt, G, impl="thread_rows"):
         scales = torch.zeros((M, K // 16), dtype=torch.uint8, device="cuda")
     else:
         codes = torch.zeros((M, K // 2), dtype=torch.uint8, device="cuda")
-        scales = torch.zeros((M, K // G), dtype=torch.float32, device="cuda")
+        scales = torch.zeros((M, K // G), dtype=torch.bfloat16, device="cuda")
     asp.qwam_asp_debug_quantize_rows(Rd, M, K, fmt, G, codes, scales)
     torch.cuda.synchronize()
     c = codes.cpu().numpy()
-    return (c if fmt == asp.QWAM_FMT_NVFP4 else decode_sm4(c)), scales.cpu().numpy()
+    if fmt == asp.QWAM_FMT_NVFP4:
+        return c, scales.cpu().numpy()
+    return decode_ob4(c), scales.float().cpu().numpy()
 
 
 @pytest.mark.parametrize("impl", list(IMPLS))

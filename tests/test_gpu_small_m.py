@@ -16,7 +16,7 @@ import oracle
 from paper_2609_33269_gb300 import asp
 from paper_2609_33269_gb300 import workloads as wl
 
-from gpu_helpers import Case, check_layer_output, near_tie_mismatches, rowwise_rel_err, to_dev_bf16
+from gpu_helpers import Case, check_int4_act, check_layer_output, gemm_tol, rowwise_rel_err, to_dev_bf16
 
 pytestmark = pytest.mark.gpu
 
@@ -59,19 +59,20 @@ def test_activation_paths_against_the_oracle(shape, small):
         if r == 0:
             np.testing.assert_array_equal(ga["qx"], oa["qx"])
             np.testing.assert_array_equal(ga["sx"], oa["sx"])
+            flip = np.zeros(M, bool)
         else:
             gp = ga["ph"].view(np.float16).astype(np.float64)
             op = oa["ph"].view(np.float16).astype(np.float64)
             ulp = np.spacing(np.maximum(np.abs(gp), np.abs(op)).astype(np.float16)).astype(np.float64)
             tol = ulp + 2e-5 * np.abs(oa["p"]).max(axis=1, keepdims=True)
             assert (np.abs(gp - op) <= tol).all(), np.abs(gp - op).max()
-            bad, near = near_tie_mismatches(ga["qx"], oa["qx"], oa["Xperp"], oa["sx"], G, 1e-3)
-            assert len(bad) <= max(1, 1e-4 * ga["qx"].size) and near.all()
+            flip = check_int4_act(ga, oa, G)
         Y = c.run(fp32=True).cpu().numpy()
         gw = c.gpu_weights()
+        tol = gemm_tol(K, -(-r // 16) * 16)
         Yk = oracle.linear(ga, dict(qw=gw["qw"], sw=gw["sw"], Bh=gw["Bh"]), G)
-        assert rowwise_rel_err(Y, Yk).max() <= 1e-5
-        check_layer_output(Y, oracle.linear(oa, ow, G), Yk, ga["qx"], oa["qx"])
+        assert rowwise_rel_err(Y, Yk).max() <= tol
+        check_layer_output(Y, oracle.linear(oa, ow, G), Yk, flip, tol)
     finally:
         c.close()
 
