@@ -20,12 +20,12 @@
 // low bits allow).  Row m of the activation operand is therefore scaled by 2^e_m and column n of
 // the weight operand by 2^e_n, powers of two chosen so that the largest dequantized value of the
 // row (7 max_g s_x, or max |p_hat|) and of the column (7 max_g s_w, or max |B_hat|) lies in
-// [2^10, 2^11) (so that 24 s, a constant of the dequantization below, stays finite); the
+// [2^10, 2^11) (so that 16 s and the dequantization's other constants stay finite); the
 // epilogue multiplies by 2^-e_n and then 2^-e_m, which is exact unless the result is a float32
 // subnormal.  Only values below 2^-24 of their row's or column's largest can lose bits, which is
 // at the float32 accumulator's own resolution.  The weight side is done
 // once, at pack time (the handle's swh, Bhs, fcol); the row factors are formed here from s_x and
-// p_hat by the row-scale warp.
+// p_hat by the epilogue warps.
 //
 // Tiles are 128 tokens x 256 outputs (one tcgen05 MMA of M = 128, N = 256, K = 16 per 16 columns),
 // K stages of 64.  The activation operand lives in TMEM (tcgen05.mma with A from tensor memory:
@@ -35,22 +35,23 @@
 // Persistent CTAs, one per SM, walk the tiles with a static stride.  896 threads:
 //   warp 0        TMA producer: per K stage the packed codes of both operands and their scales
 //   warp 1        MMA issuer and TMEM owner
-//   warp 2        row scales: 2^e_m and 2^-e_m of the tile's 128 rows, one slot per tile
-//   warp 3        idle
+//   warps 2, 3    idle
 //   warps 4..19   expanders, two groups of eight that take alternate stages (group x the stages
 //                 whose running index is x mod 2), so that each warp has two stage times for its
 //                 work.  Warp e of a group takes the activation codes k = 32h .. 32h + 31
 //                 (h = e / 4) of the 32 token rows in TMEM lane quadrant q = e % 4 (16 columns
 //                 stored with tcgen05.st) and weight rows 32e .. 32e + 31 of the stage's 256
 //                 (float16 into the shared-memory operand)
-//   warps 20..27  epilogue: warp 20 + 4h + q reads lanes 32q.., columns 128h..128h+127
+//   warps 20..27  epilogue: warp 20 + 4h + q reads lanes 32q.., columns 128h..128h+127; between
+//                 tiles the same warps form the row scales 2^e_m, 2^-e_m of the tile after next
+//                 (two threads per row) and stage their columns' 2^-e_n and bias in shared memory
 // Branch stages (after the K stages, r_pad / 64 rounded up): the expanders load p_hat by TMA (one
 // buffer per group) and scale it by 2^e_m into TMEM, and B_hat 2^e_n comes by TMA straight into the
 // operand stage.  Every wait is bounded.
 // Rings:
 //   P  packed stage: A and B codes, s_x and s_w 2^e_n of its groups   TMA -> expanders   SP slots
 //   O  operand stage: A (TMEM, 32 columns) and B (shared memory)  expanders -> MMA   SO slots
-//   R  row-scale slot                          row-scale warp -> expanders, epilogue   2 slots
+//   R  row-scale slot                          epilogue warps -> expanders, epilogue   2 slots
 //   the accumulator (TMEM columns 0..255)     MMA -> epilogue             1
 #include "internal.h"
 #include "ptx.cuh"
@@ -84,12 +85,14 @@ constexpr int PSTAGE = PA + PB + PSX + 2 * BN * 2;  // then s_w 2^e_n [GPS][256]
 constexpr int BSTAGE = BN * KS * 2;      // float16 weight operand, 128-byte rows (32 KB)
 constexpr int PHB = BM * KS * 2;         // p_hat stage [128][64] f16, 128-byte swizzle (one per group)
 constexpr int RSB = BM * 8;              // {2^e_m, 2^-e_m} per row
+constexpr int EFB = 2 * 128 * 4;         // per epilogue warp: 2^-e_n and bias of its 128 columns
 constexpr int NBAR = 2 * SP + 2 * SO + 2 + 2 * 2 + 2 * 2 + 1;
 constexpr int OFF_B = 0;
 constexpr int OFF_PH = OFF_B + SO * BSTAGE;
 constexpr int OFF_P = OFF_PH + 2 * PHB;
 constexpr int OFF_R = OFF_P + SP * PSTAGE;
-constexpr int OFF_BAR = OFF_R + 2 * RSB;
+constexpr int OFF_E = OFF_R + 2 * RSB;
+constexpr int OFF_BAR = OFF_E + 8 * EFB;
 constexpr int SMEM = 1024 + OFF_BAR + NBAR * 8 + 16;
 static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 constexpr uint32_t TMEM_COLS = 512;  // accumulator 0..255, A ring 256 + 32 i
@@ -121,6 +124,21 @@ __device__ __forceinline__ uint32_t f32x2_to_bf16x2(float lo, float hi) {
   uint32_t d;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
   return d;
+}
+// Global stores and read-only loads named as such: a generic store could alias the shared-memory
+// reads around it as far as the compiler knows, which would serialize the epilogue.
+__device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.global.v4.b32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(a), "r"(b), "r"(c), "r"(d));
+}
+__device__ __forceinline__ uint32_t ld_nc_u16(const void* p) {
+  unsigned short v;
+  asm volatile("ld.global.nc.u16 %0, [%1];" : "=h"(v) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint4 ld_nc_v4(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
 }
 __device__ __forceinline__ float f16_lo(uint32_t u) { return __half2float(__ushort_as_half(static_cast<unsigned short>(u))); }
 __device__ __forceinline__ float f16_hi(uint32_t u) { return __half2float(__ushort_as_half(static_cast<unsigned short>(u >> 16))); }
@@ -189,6 +207,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* phbuf = smem + OFF_PH;
   uint8_t* pring = smem + OFF_P;
   float2* rslot = reinterpret_cast<float2*>(smem + OFF_R);
+  float* efb = reinterpret_cast<float*>(smem + OFF_E);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* pfull = bars;
   uint64_t* pempty = pfull + SP;
@@ -230,7 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(accfull, 1);
     mbar_init(accempty, 8);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&rfull[i], 1);
+      mbar_init(&rfull[i], 8);
       mbar_init(&rempty[i], 24);
       mbar_init(&phfull[i], 1);
       mbar_init(&phempty[i], 8);
@@ -304,54 +323,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     int never = 0;
     const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
     mbar_wait_inline(drain, 0, dc);
-  } else if (wid == 2) {
-    // ------------------------------------------------------------- row scales
-    // Lane l takes rows m0 + 4l .. m0 + 4l + 3: the largest dequantized value of the row,
-    // a_m = max(7 max_g s_x[m, g], max_j |p_hat[m, j]|), gives e_m = 10 - floor(log2 a_m).
-    bool ok = true;
-    const int ng = a.K / G;
-    for (int ti = 0; ti < my_tiles && ok; ++ti) {
-      int m0, n0;
-      tile_mn(ti, m0, n0);
-      const int sl = ti & 1;
-      if (ti >= 2) ok = mbar_wait_inline(&rempty[sl], ((ti >> 1) & 1) ^ 1, wc);
-      if (!ok) break;
-      const int mr = m0 + 4 * static_cast<int>(lane);  // < M_pad (a multiple of 128)
-      float smax[4] = {0.f, 0.f, 0.f, 0.f};
-      const __nv_bfloat16* sp = a.sx + mr;
-#pragma unroll 4
-      for (int g = 0; g < ng; ++g) {
-        const uint2 v = *reinterpret_cast<const uint2*>(sp + static_cast<size_t>(g) * a.M_pad);
-        smax[0] = fmaxf(smax[0], __uint_as_float(v.x << 16));
-        smax[1] = fmaxf(smax[1], __uint_as_float(v.x & 0xFFFF0000u));
-        smax[2] = fmaxf(smax[2], __uint_as_float(v.y << 16));
-        smax[3] = fmaxf(smax[3], __uint_as_float(v.y & 0xFFFF0000u));
-      }
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        float am = 7.0f * smax[i];  // exact: 8 + 3 significant bits
-        const int m = mr + i;
-        if (a.r_pad > 0 && m < a.M) {
-          const uint4* pr = reinterpret_cast<const uint4*>(a.phat + static_cast<size_t>(m) * a.r_pad);
-          for (int j = 0; j < a.r_pad / 8; ++j) {
-            const uint4 u = pr[j];
-            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-            for (int t = 0; t < 4; ++t) am = fmaxf(am, fmaxf(fabsf(f16_lo(w4[t])), fabsf(f16_hi(w4[t]))));
-          }
-        }
-        int e = 0;
-        if (am > 0.0f) {
-          int ex;
-          frexpf(am, &ex);  // am in [2^(ex-1), 2^ex)
-          e = min(126, max(-126, 11 - ex));
-        }
-        rslot[sl * BM + 4 * lane + i] = make_float2(ldexpf(1.0f, e), ldexpf(1.0f, -e));
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&rfull[sl]);
-      __syncwarp();
-    }
   } else if (wid >= 4 && wid < 20) {
     // ------------------------------------------------------------- expanders
     // Activation part: row r = 32q + lane (TMEM lane), codes k = 32h .. 32h + 31 of the stage
@@ -477,20 +448,79 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lb >= 0) mbar_wait_inline(&ofull[lb % SO], (lb / SO) & 1, dc);
     }
   } else if (wid >= 20) {
-    // ------------------------------------------------------------- epilogue
+    // ------------------------------------------------------------- epilogue and row scales
     const int ew = static_cast<int>(wid) - 20;
     const int q = ew & 3, hf = ew >> 2;
     const int r = 32 * q + static_cast<int>(lane);
     const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(128 * hf);
+    float* fcb = efb + ew * (EFB / 4);  // [0, 128): 2^-e_n, [128, 256): bias of columns n0 + 128 hf ..
+    // Row scales of tile tt into slot tt % 2: thread u takes row u / 2 and every other group from
+    // u % 2 (and that half of p_hat); the pair combines by a shuffle.  a_m = max(7 max_g s_x[m, g],
+    // max_j |p_hat[m, j]|) gives e_m = 10 - floor(log2 a_m).
+    const int u = 32 * ew + static_cast<int>(lane);
+    const int rr = u >> 1, hs = u & 1;
+    const int ng = a.K / G;
+    auto rowscale = [&](int tt) -> bool {
+      int m0t, n0t;
+      tile_mn(tt, m0t, n0t);
+      const int sl = tt & 1;
+      if (tt >= 2 && !mbar_wait_inline(&rempty[sl], ((tt >> 1) & 1) ^ 1, wc)) return false;
+      const int m = m0t + rr;  // < M_pad (a multiple of 128)
+      const __nv_bfloat16* sp = a.sx + m;
+      // (the workspace was written by the previous kernel of the stream, complete before pdl_wait)
+      auto sx_at = [&](int g) { return __uint_as_float(ld_nc_u16(sp + static_cast<size_t>(g) * a.M_pad) << 16); };
+      float s0 = 0.0f, s1 = 0.0f, s2 = 0.0f, s3 = 0.0f;
+      int g = hs;
+#pragma unroll 4
+      for (; g + 6 < ng; g += 8) {  // up to 16 independent loads in flight
+        s0 = fmaxf(s0, sx_at(g));
+        s1 = fmaxf(s1, sx_at(g + 2));
+        s2 = fmaxf(s2, sx_at(g + 4));
+        s3 = fmaxf(s3, sx_at(g + 6));
+      }
+      for (; g < ng; g += 2) s0 = fmaxf(s0, sx_at(g));
+      float am = 7.0f * fmaxf(fmaxf(s0, s1), fmaxf(s2, s3));  // exact: 8 + 3 significant bits
+      if (a.r_pad > 0 && m < a.M) {
+        const uint4* pr = reinterpret_cast<const uint4*>(a.phat + static_cast<size_t>(m) * a.r_pad) + hs * (a.r_pad / 16);
+#pragma unroll 4
+        for (int j = 0; j < a.r_pad / 16; ++j) {
+          const uint4 u4 = ld_nc_v4(pr + j);
+          const uint32_t w4[4] = {u4.x, u4.y, u4.z, u4.w};
+#pragma unroll
+          for (int t = 0; t < 4; ++t) am = fmaxf(am, fmaxf(fabsf(f16_lo(w4[t])), fabsf(f16_hi(w4[t]))));
+        }
+      }
+      am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
+      int e = 0;
+      if (am > 0.0f) {
+        int ex;
+        frexpf(am, &ex);  // am in [2^(ex-1), 2^ex)
+        e = min(126, max(-126, 11 - ex));
+      }
+      if (hs == 0) rslot[sl * BM + rr] = make_float2(ldexpf(1.0f, e), ldexpf(1.0f, -e));
+      warp_arrive(&rfull[sl]);
+      return true;
+    };
     bool ok = true;
+    if (my_tiles > 0) ok = rowscale(0);
+    if (ok && my_tiles > 1) ok = rowscale(1);
     for (int ti = 0; ti < my_tiles && ok; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
+      {  // this warp's columns' 2^-e_n and bias, staged while the tile's MMAs run
+        const int n = n0 + 128 * hf + 4 * static_cast<int>(lane);  // < N_pad
+        reinterpret_cast<float4*>(fcb)[lane] = *reinterpret_cast<const float4*>(a.fcol + n);
+        float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (a.bias && n < a.N) b = *reinterpret_cast<const float4*>(a.bias + n);
+        reinterpret_cast<float4*>(fcb + 128)[lane] = b;
+        __syncwarp();
+      }
       ok = mbar_wait_inline(&rfull[ti & 1], (ti >> 1) & 1, wc);
       if (ok) ok = mbar_wait_inline(accfull, ti & 1, wc);
       if (!ok) break;
       tc_fence_after();
       const float fm = rslot[(ti & 1) * BM + r].y;
+      warp_arrive(&rempty[ti & 1]);
       const int m = m0 + r;
 #pragma unroll 1
       for (int c = 0; c < 4; ++c) {
@@ -508,32 +538,33 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = 0; j < 4; ++j) {
             const int n = nb + 8 * j;
             if (n >= a.N) continue;
-            const float4 f0 = *reinterpret_cast<const float4*>(a.fcol + n);
-            const float4 f1 = *reinterpret_cast<const float4*>(a.fcol + n + 4);
+            const float4 f0 = reinterpret_cast<const float4*>(fcb)[8 * c + 2 * j];
+            const float4 f1 = reinterpret_cast<const float4*>(fcb)[8 * c + 2 * j + 1];
+            const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[8 * c + 2 * j];
+            const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[8 * c + 2 * j + 1];
             const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+            const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
             float y[8];
 #pragma unroll
-            for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(acc[8 * j + t]) * fn[t]) * fm;
-            if (a.bias) {
-              const float4 b0 = *reinterpret_cast<const float4*>(a.bias + n);
-              const float4 b1 = *reinterpret_cast<const float4*>(a.bias + n + 4);
-              y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
-              y[4] += b1.x; y[5] += b1.y; y[6] += b1.z; y[7] += b1.w;
+            for (int t = 0; t < 8; ++t) {
+              y[t] = (__uint_as_float(acc[8 * j + t]) * fn[t]) * fm;
+              if (a.bias) y[t] += bb[t];
             }
             const size_t off = static_cast<size_t>(m) * a.N + n;
             if (a.y_f32) {
-              float4* yp = reinterpret_cast<float4*>(static_cast<float*>(a.Y) + off);
-              yp[0] = make_float4(y[0], y[1], y[2], y[3]);
-              yp[1] = make_float4(y[4], y[5], y[6], y[7]);
+              float* yp = static_cast<float*>(a.Y) + off;
+              st_global_v4(yp, __float_as_uint(y[0]), __float_as_uint(y[1]), __float_as_uint(y[2]), __float_as_uint(y[3]));
+              st_global_v4(yp + 4, __float_as_uint(y[4]), __float_as_uint(y[5]), __float_as_uint(y[6]),
+                           __float_as_uint(y[7]));
             } else {
-              *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
-                  make_uint4(f32x2_to_bf16x2(y[0], y[1]), f32x2_to_bf16x2(y[2], y[3]), f32x2_to_bf16x2(y[4], y[5]),
-                             f32x2_to_bf16x2(y[6], y[7]));
+              st_global_v4(static_cast<__nv_bfloat16*>(a.Y) + off, f32x2_to_bf16x2(y[0], y[1]), f32x2_to_bf16x2(y[2], y[3]),
+                           f32x2_to_bf16x2(y[4], y[5]), f32x2_to_bf16x2(y[6], y[7]));
             }
           }
         }
       }
-      warp_arrive(&rempty[ti & 1]);
+      __syncwarp();  // every lane's reads of the staged columns are done before the next tile's
+      if (ti + 2 < my_tiles) ok = rowscale(ti + 2);
     }
     tmem_ld_wait();
   }
