@@ -76,7 +76,10 @@ enum { QWAM_Y_BF16 = 0, QWAM_Y_FP32 = 1 };
 qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int N, int r, int group,
                                   struct CUstream_st* stream, qwam_asp_handle* out);
 
-/* Bytes of the caller-owned activation workspace needed for M tokens. */
+/* Bytes of the caller-owned activation workspace needed for M tokens.  For INT4 layers of 512 or
+ * more tokens it includes a float16 copy of the layer's weights, N_pad (K + r_pad) 2 bytes (N_pad =
+ * N rounded up to 256), which qwam_asp_gemm fills once per call and reads from L2 for every row
+ * tile. */
 qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes);
 
 /* Layout of the activation workspace for M tokens (byte offsets from its start):
@@ -130,9 +133,11 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
  * (QWAM_STATIC_WS_BYTES per device, set aside when the library's device code is loaded).  It
  * allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
  *
- *   - Size limit: the workspace qwam_asp_act_workspace_bytes(h, M) reports must fit in
- *     QWAM_STATIC_WS_BYTES (24 MiB); larger requests return QWAM_ERR_TOO_LARGE before anything
- *     is launched.  Per token the workspace holds about K/2 + 2K/G + 2 r_pad bytes (INT4) or
+ *   - Size limit: the workspace must fit in QWAM_STATIC_WS_BYTES (24 MiB); larger requests return
+ *     QWAM_ERR_TOO_LARGE before anything is launched.  This call uses the workspace without the
+ *     per-call float16 copy of the weights that qwam_asp_act_workspace_bytes counts for INT4
+ *     layers of 512 or more tokens (its GEMM converts the weights tile by tile instead), so it
+ *     needs less than qwam_asp_act_workspace_bytes reports for such layers.  Per token the workspace holds about K/2 + 2K/G + 2 r_pad bytes (INT4) or
  *     K/2 + K/16 + 2 r_pad bytes (NVFP4): at K = 3072, group 64, r = 32 about 1.7 KB, so up to
  *     about 14,000 tokens fit.  A rotated handle with r > 0 also keeps its float32 remainder,
  *     4K more bytes per token: at K = 3072 about 1,780 tokens fit, and M = 4096 is refused.

@@ -78,7 +78,7 @@ bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const
   return r == CUDA_SUCCESS;
 }
 
-ActLayout act_layout(const Handle& h, int M) {
+ActLayout act_layout(const Handle& h, int M, bool lean) {
   ActLayout L;
   L.M_pad = round_up(M > 0 ? M : 1, kBM);
   L.codes_off = 0;
@@ -97,6 +97,7 @@ ActLayout act_layout(const Handle& h, int M) {
       L.ytmp_off = L.bytes;
       L.bytes += up256(static_cast<size_t>(M) * h.N * 4);
     }
+    L.w16_off = 0;
     return L;
   }
   L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
@@ -109,18 +110,23 @@ ActLayout act_layout(const Handle& h, int M) {
     L.bytes += up256(static_cast<size_t>(M) * h.K * 4);
   }
   L.ytmp_off = 0;
+  L.w16_off = 0;
+  if (!lean && L.M_pad / kBM >= kPreExpandMinTiles) {
+    L.w16_off = L.bytes;
+    L.bytes += up256(static_cast<size_t>(h.N_pad) * (h.K + h.r_pad) * 2);
+  }
   return L;
 }
 
 uint64_t deadline_budget_ns(const Handle& h) { return static_cast<uint64_t>(h.timeout_s * 1e9); }
 
-const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
+const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M, bool lean) {
   for (auto& c : h.act_cache)
-    if (c.ws == ws && c.M == M && (x == nullptr || c.x == x)) return &c;
+    if (c.ws == ws && c.M == M && c.lean == lean && (x == nullptr || c.x == x)) return &c;
   ActMaps& c = h.act_cache[h.act_next];
   h.act_next = (h.act_next + 1) % 4;
   c.ws = nullptr;
-  const ActLayout L = act_layout(h, M);
+  const ActLayout L = act_layout(h, M, lean);
   const uint8_t* base = static_cast<const uint8_t*>(ws);
   bool ok = true;
   if (x) {
@@ -142,10 +148,14 @@ const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M) {
     ok &= encode_2d(&c.ph64_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.phat_off, h.r_pad, M,
                     static_cast<uint64_t>(h.r_pad) * 2, 64, kBM, CU_TENSOR_MAP_SWIZZLE_128B);
   }
+  if (L.w16_off)
+    ok &= encode_2d(&c.w16_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base + L.w16_off, h.K + h.r_pad, h.N_pad,
+                    static_cast<uint64_t>(h.K + h.r_pad) * 2, 64, kGemm16BN, CU_TENSOR_MAP_SWIZZLE_128B);
   if (!ok) return nullptr;
   c.ws = ws;
   c.x = x;
   c.M = M;
+  c.lean = lean;
   return &c;
 }
 
@@ -181,6 +191,35 @@ static cudaError_t note_launch(Handle& h, cudaStream_t s) {
   if (e == cudaSuccess) h.done_valid = true;
   return e;
 }
+
+static qwam_status gemm_impl(const void* act_ws, int M, qwam_asp_handle hs, void* Y, int y_dtype,
+                             struct CUstream_st* stream, bool lean) {
+  if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
+  if (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32) return QWAM_ERR_INVALID_ARG;
+  if (M == 0) return QWAM_OK;
+  if (!act_ws || !Y || !qwam::aligned16(act_ws) || !qwam::aligned16(Y)) return QWAM_ERR_INVALID_ARG;
+  Handle& h = hs->h;
+  const qwam::ActMaps* am = qwam::get_act_maps(h, nullptr, act_ws, M, lean);
+  if (!am) return QWAM_ERR_CUDA;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = h.fmt == qwam::kFmtNvfp4 ? qwam::launch_gemm_nvfp4(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s)
+                                           : qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s, lean);
+  if (e == cudaSuccess) e = note_launch(h, s);
+  return from_cuda_status(e);
+}
+
+namespace qwam {
+// The layer on a workspace of act_layout(h, M, lean): qwam_asp_linear (lean = false) and the
+// static-scratch entry (lean = true, no expanded-weight region).
+qwam_status linear_impl(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype, void* act_ws,
+                        struct CUstream_st* stream, bool lean) {
+  if (!h || M < 0 || (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32)) return QWAM_ERR_INVALID_ARG;
+  if (M > 0 && (!Y || !qwam::aligned16(Y))) return QWAM_ERR_INVALID_ARG;
+  qwam_status st = qwam_asp_quantize_act(X_bf16, M, h, act_ws, stream);
+  if (st != QWAM_OK) return st;
+  return gemm_impl(act_ws, M, h, Y, y_dtype, stream, lean);
+}
+}  // namespace qwam
 
 extern "C" {
 
@@ -496,27 +535,12 @@ qwam_status qwam_asp_select_experts(const double* mass, const double* cost, int 
 
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle hs, void* Y, int y_dtype,
                           struct CUstream_st* stream) {
-  if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
-  if (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32) return QWAM_ERR_INVALID_ARG;
-  if (M == 0) return QWAM_OK;
-  if (!act_ws || !Y || !qwam::aligned16(act_ws) || !qwam::aligned16(Y)) return QWAM_ERR_INVALID_ARG;
-  Handle& h = hs->h;
-  const qwam::ActMaps* am = qwam::get_act_maps(h, nullptr, act_ws, M);
-  if (!am) return QWAM_ERR_CUDA;
-  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = h.fmt == qwam::kFmtNvfp4 ? qwam::launch_gemm_nvfp4(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s)
-                                           : qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s);
-  if (e == cudaSuccess) e = note_launch(h, s);
-  return from_cuda_status(e);
+  return gemm_impl(act_ws, M, hs, Y, y_dtype, stream, false);
 }
 
 qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype, void* act_ws,
                             struct CUstream_st* stream) {
-  if (!h || M < 0 || (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32)) return QWAM_ERR_INVALID_ARG;
-  if (M > 0 && (!Y || !qwam::aligned16(Y))) return QWAM_ERR_INVALID_ARG;
-  qwam_status st = qwam_asp_quantize_act(X_bf16, M, h, act_ws, stream);
-  if (st != QWAM_OK) return st;
-  return qwam_asp_gemm(act_ws, M, h, Y, y_dtype, stream);
+  return qwam::linear_impl(X_bf16, M, h, Y, y_dtype, act_ws, stream, false);
 }
 
 qwam_status qwam_asp_get_error(qwam_asp_handle hs) {

@@ -48,6 +48,10 @@
 // Branch stages (after the K stages, r_pad / 64 rounded up): the expanders load p_hat by TMA (one
 // buffer per group) and scale it by 2^e_m into TMEM, and B_hat 2^e_n comes by TMA straight into the
 // operand stage.  Every wait is bounded.
+// Layers with several 128-row tiles (kPreExpandMinTiles) would convert every weight stage once per
+// row tile; for them `dequant_weights_kernel` writes the float16 weights [s_w 2^e_n c | B_hat 2^e_n]
+// once per call into the workspace (the PREB instantiation), the producer loads each weight stage
+// by TMA straight into the operand ring, and the expanders convert the activations only.
 // Rings:
 //   P  packed stage: A and B codes, s_x and s_w 2^e_n of its groups   TMA -> expanders   SP slots
 //   O  operand stage: A (TMEM, 32 columns) and B (shared memory)  expanders -> MMA   SO slots
@@ -193,7 +197,36 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.expect_tx.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
 }
 
+// The weights of one call in float16, [N_pad, K + r_pad] row-major: W16[n, k] = s_w[g, n] 2^e_n c[n, k]
+// for k < K (g = k / G; exact, as in the GEMM's own conversion) and B_hat[n, k - K] 2^e_n after.  One
+// thread per 8 consecutive k of a row.
 template <int G>
+__global__ void __launch_bounds__(256) dequant_weights_kernel(const uint32_t* __restrict__ qw,
+                                                              const __half* __restrict__ swh,
+                                                              const __half* __restrict__ bhs, int K, int r_pad,
+                                                              int N_pad, __half* __restrict__ w16) {
+  pdl_launch_dependents();
+  pdl_wait();  // the workspace may still be read by the stream's previous GEMM until then
+  const int wpr = (K + r_pad) / 8;  // 8-wide pieces per row
+  const long long total = static_cast<long long>(N_pad) * wpr;
+  for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int n = static_cast<int>(i / wpr), j = static_cast<int>(i % wpr);
+    uint4 o;
+    if (8 * j < K) {
+      const uint32_t w = qw[static_cast<size_t>(n) * (K / 8) + j];
+      const DqScale d = dq_scale(__half2float(swh[static_cast<size_t>(8 * j / G) * N_pad + n]));
+      uint32_t v[4];
+      dequant_word(w, d, v);
+      o = make_uint4(v[0], v[1], v[2], v[3]);
+    } else {
+      o = *reinterpret_cast<const uint4*>(bhs + static_cast<size_t>(n) * r_pad + (8 * j - K));
+    }
+    *reinterpret_cast<uint4*>(w16 + static_cast<size_t>(n) * (K + r_pad) + 8 * j) = o;
+  }
+}
+
+template <int G, bool PREB>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm16_kernel(const __grid_constant__ CUtensorMap qa_map, const __grid_constant__ CUtensorMap qw_map,
                   const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap sw_map,
@@ -243,7 +276,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&pempty[i], 8);
     }
     for (int i = 0; i < SO; ++i) {
-      mbar_init(&ofull[i], 8);
+      mbar_init(&ofull[i], PREB ? 9 : 8);  // the group's eight expanders (and, with PREB, the producer)
       mbar_init(&oempty[i], 1);
     }
     mbar_init(accfull, 1);
@@ -271,29 +304,51 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (wid == 0) {
     // ------------------------------------------------------------- TMA producer
     bool ok = true;
-    int s = 0;
+    int s = 0, so = 0;
     for (int ti = 0; ti < my_tiles && ok; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
-      for (int st = 0; st < nks && ok; ++st, ++s) {
-        const int ps = s % SP;
-        if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
-        if (!ok) break;
-        uint8_t* p = pring + ps * PSTAGE;
-        if (elect_one()) {
-          mbar_arrive_expect_tx(&pfull[ps], PA + PB + GPS * (BM + BN) * 2);
-          tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
-          tma_load_2d(p + PA, &qw_map, &pfull[ps], st * (KS / 2), n0);
-          tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
-          tma_load_2d(p + PA + PB + PSX, &sw_map, &pfull[ps], n0, st * GPS);
+      for (int st = 0; st < (PREB ? nst : nks) && ok; ++st, ++so) {
+        if (st < nks) {
+          const int ps = s % SP;
+          if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
+          if (!ok) break;
+          uint8_t* p = pring + ps * PSTAGE;
+          if (elect_one()) {
+            if (PREB) {
+              mbar_arrive_expect_tx(&pfull[ps], PA + GPS * BM * 2);
+              tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
+              tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
+            } else {
+              mbar_arrive_expect_tx(&pfull[ps], PA + PB + GPS * (BM + BN) * 2);
+              tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
+              tma_load_2d(p + PA, &qw_map, &pfull[ps], st * (KS / 2), n0);
+              tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
+              tma_load_2d(p + PA + PB + PSX, &sw_map, &pfull[ps], n0, st * GPS);
+            }
+          }
+          __syncwarp();
+          ++s;
         }
-        __syncwarp();
+        if (PREB) {
+          // the stage's float16 weights (W_perp, or B_hat in a branch stage) into the operand ring
+          const int os = so % SO;
+          if (so >= SO) ok = mbar_wait_inline(&oempty[os], ((so / SO) & 1) ^ 1, wc);
+          if (!ok) break;
+          if (elect_one()) {
+            mbar_arrive_expect_tx(&ofull[os], BSTAGE);
+            tma_load_2d(bring + os * BSTAGE, &bh_map, &ofull[os], st * KS, n0);
+          }
+          __syncwarp();
+        }
       }
     }
     // every issued load lands before the CTA can exit
     int never = 0;
     const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
     for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
+    if (PREB)
+      for (int j = (so > SO ? so - SO : 0); j < so; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
     constexpr uint32_t idesc = idesc_f16(BM, BN);
@@ -371,11 +426,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           const __nv_bfloat16 sxa = reinterpret_cast<const __nv_bfloat16*>(pk + PA + PB)[(GPS == 2 ? h : 0) * BM + r];
           uint4 wb[2];
           __half swb[2];
+          if (!PREB) {
 #pragma unroll
-          for (int i = 0; i < 2; ++i) {
-            const int R = Rb + 16 * i;
-            wb[i] = *reinterpret_cast<const uint4*>(pk + PA + R * (KS / 2) + 16 * hh);
-            swb[i] = reinterpret_cast<const __half*>(pk + PA + PB + PSX)[(GPS == 2 ? hh : 0) * BN + R];
+            for (int i = 0; i < 2; ++i) {
+              const int R = Rb + 16 * i;
+              wb[i] = *reinterpret_cast<const uint4*>(pk + PA + R * (KS / 2) + 16 * hh);
+              swb[i] = reinterpret_cast<const __half*>(pk + PA + PB + PSX)[(GPS == 2 ? hh : 0) * BN + R];
+            }
           }
           const DqScale da = scale_consts(sxa, mul);
           dequant_word(wa.x, da, v + 0);
@@ -383,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           dequant_word(wa.z, da, v + 8);
           dequant_word(wa.w, da, v + 12);
 #pragma unroll
-          for (int i = 0; i < 2; ++i) {
+          for (int i = 0; i < (PREB ? 0 : 2); ++i) {
             const DqScale db = dq_scale(__half2float(swb[i]));
             uint8_t* row = dst + (Rb + 16 * i) * 128;
             const uint32_t wv[4] = {wb[i].x, wb[i].y, wb[i].z, wb[i].w};
@@ -406,8 +463,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
           if (e == 0) {
             if (elect_one()) {
-              mbar_expect_tx(&ofull[os], BSTAGE);
-              tma_load_2d(dst, &bh_map, &ofull[os], (st - nks) * KS, n0);
+              if (!PREB) {  // (with PREB the producer brings B_hat with the other weight stages)
+                mbar_expect_tx(&ofull[os], BSTAGE);
+                tma_load_2d(dst, &bh_map, &ofull[os], (st - nks) * KS, n0);
+              }
               mbar_arrive_expect_tx(&phfull[gx], PHB);
               tma_load_2d(phb, &ph_map, &phfull[gx], (st - nks) * KS, m0);
             }
@@ -437,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int never = 0;
     const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
     if (ph > 0) mbar_wait_inline(&phfull[gx], (ph - 1) & 1, dc);
-    if (e == 0 && a.nbs > 0) {
+    if (!PREB && e == 0 && a.nbs > 0) {
       // this group's last branch stage: its B_hat load completed the stage's barrier
       int lb = -1;
       for (int j = so - 1; j >= 0 && j >= so - a.nbs; --j)
@@ -576,9 +635,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int G>
-cudaError_t launch_g(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s) {
-  const ActLayout L = act_layout(h, M);
+template <int G, bool PREB>
+cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const void* ws, int M, void* Y, bool y_f32,
+                     cudaStream_t s) {
   const uint8_t* base = static_cast<const uint8_t*>(ws);
   GemmArgs a;
   a.M = M;
@@ -599,32 +658,49 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const void* ws, int M, void* 
   a.timeout_ns = deadline_budget_ns(h);
   static bool attr_done = false;
   if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(gemm16_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+    cudaError_t e = cudaFuncSetAttribute(gemm16_kernel<G, PREB>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  const int ntiles = a.m_tiles * a.n_tiles;
-  const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
-  // Without a branch the p_hat / B_hat maps are never used; any valid map fills the slots.
-  const CUtensorMap& ph = (h.r_pad > 0) ? am.ph64_map : am.qa_map;
-  const CUtensorMap& bh = (h.r_pad > 0) ? h.bhs_map : am.qa_map;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid, 1, 1);
-  cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = SMEM;
-  cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.stream = s;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, gemm16_kernel<G>, am.qa_map, h.qw_map, am.sx_map, h.swh_map, ph, bh, a);
+  if (PREB) {
+    __half* w16 = reinterpret_cast<__half*>(const_cast<uint8_t*>(base) + L.w16_off);
+    const long long pieces = static_cast<long long>(h.N_pad) * ((h.K + h.r_pad) / 8);
+    const long long blocks = (pieces + 255) / 256;
+    cfg.gridDim = dim3(static_cast<unsigned>(blocks < 8 * h.num_sms ? blocks : 8 * h.num_sms), 1, 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.dynamicSmemBytes = 0;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, dequant_weights_kernel<G>, reinterpret_cast<const uint32_t*>(h.qw),
+                                       static_cast<const __half*>(h.swh), static_cast<const __half*>(h.Bhs), h.K,
+                                       h.r_pad, h.N_pad, w16);
+    if (e != cudaSuccess) return e;
+  }
+  const int ntiles = a.m_tiles * a.n_tiles;
+  const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
+  // With PREB every weight stage comes through the expanded-weight map; without a branch the
+  // p_hat / B_hat maps are never used and any valid map fills the slots.
+  const CUtensorMap& ph = (h.r_pad > 0) ? am.ph64_map : am.qa_map;
+  const CUtensorMap& bh = PREB ? am.w16_map : ((h.r_pad > 0) ? h.bhs_map : am.qa_map);
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = SMEM;
+  return cudaLaunchKernelEx(&cfg, gemm16_kernel<G, PREB>, am.qa_map, h.qw_map, am.sx_map, h.swh_map, ph, bh, a);
 }
 
 }  // namespace
 
-cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s) {
-  return h.G == 32 ? launch_g<32>(h, am, ws, M, Y, y_f32, s) : launch_g<64>(h, am, ws, M, Y, y_f32, s);
+cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s,
+                        bool lean) {
+  const ActLayout L = act_layout(h, M, lean);
+  if (L.w16_off)
+    return h.G == 32 ? launch_g<32, true>(h, am, L, ws, M, Y, y_f32, s) : launch_g<64, true>(h, am, L, ws, M, Y, y_f32, s);
+  return h.G == 32 ? launch_g<32, false>(h, am, L, ws, M, Y, y_f32, s) : launch_g<64, false>(h, am, L, ws, M, Y, y_f32, s);
 }
 
 }  // namespace qwam

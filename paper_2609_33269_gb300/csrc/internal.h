@@ -17,6 +17,9 @@ constexpr int kChunk = 64;      // K columns per activation chunk (bf16: one 128
 constexpr int kMaxRank = 64;    // largest rank of kernel (a)'s tensor-core path (above: the general-rank path)
 constexpr int kGemmBN = 128;    // output columns per NVFP4 GEMM CTA tile
 constexpr int kGemm16BN = 256;  // output columns per INT4 GEMM CTA tile (float16 tensor-core kernel)
+// INT4 layers with at least this many 128-row tiles have their weights expanded to float16 once per
+// call (into the workspace) instead of once per tile inside the GEMM.
+constexpr int kPreExpandMinTiles = 4;
 
 // NVFP4 variant (App. B.1): E2M1 codes, one E4M3 scale per 16 consecutive K, one float32 scale per
 // weight tensor.  Block scales are stored in 512-byte atoms, one per 128 rows x 64 K: the four
@@ -57,6 +60,8 @@ struct ActMaps {
   CUtensorMap ph_map;   // p_hat f16 [M, r_pad], box {8, 128} (NVFP4 GEMM)
   CUtensorMap ph64_map; // p_hat f16 [M, r_pad], box {64, 128}, 128-byte swizzle (INT4 GEMM)
   CUtensorMap qx4_map;  // NVFP4 codes [M, K/2] bytes, box {128, 128}, 128-byte swizzle
+  CUtensorMap w16_map;  // INT4, large M: float16 weights [N_pad, K + r_pad], box {64, 256}, 128-byte swizzle
+  bool lean = false;    // the layout without the expanded-weight region
 };
 
 struct Handle {
@@ -114,25 +119,33 @@ struct ActLayout {
   size_t codes_off, scales_off, ab_off, phat_off, bytes;
   size_t resid_off;  // rotated handles with r > 0: float32 [M, K] remainder before the rotation
   size_t ytmp_off;   // NVFP4 with r_pad > kMaxRank: float32 [M, N] 4-bit part before the branch
+  size_t w16_off;    // INT4 with >= kPreExpandMinTiles row tiles: float16 [N_pad, K + r_pad], the
+                     // dequantized W_perp (s_w 2^e_n c) and B_hat 2^e_n of the call (0: none)
   int M_pad;
 };
-ActLayout act_layout(const Handle& h, int M);
+// `lean`: without the expanded-weight region (the GEMM then expands the weights tile by tile).
+ActLayout act_layout(const Handle& h, int M, bool lean = false);
 
 // Tensor-map encoder (driver entry point fetched through the runtime).
 bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint64_t inner, uint64_t outer,
                uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle sw);
 bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const uint64_t dims[3],
                const uint64_t strides_bytes[2], const uint32_t box[3]);
-const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M);
+const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M, bool lean = false);
 
 uint64_t deadline_budget_ns(const Handle& h);
+
+// The layer on a workspace of act_layout(h, M, lean) (api.cu).
+qwam_status linear_impl(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype, void* act_ws,
+                        struct CUstream_st* stream, bool lean);
 
 // Launchers (return cudaSuccess or the launch error).
 cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
 cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
 cudaError_t launch_pack_rotated(Handle& h, const __nv_bfloat16* W, const float* s, const float* U, cudaStream_t st);
 cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s);
-cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
+cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s,
+                        bool lean = false);
 cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
 cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s);
 cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,

@@ -45,12 +45,11 @@ qwam_status static_ws_address(void** out) {
 qwam_status qwam_asp_linear_static(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
                                    struct CUstream_st* stream) {
   if (!h || M < 0) return QWAM_ERR_INVALID_ARG;
-  size_t need = 0;
-  const qwam_status st = qwam_asp_act_workspace_bytes(h, M, &need);
-  if (st != QWAM_OK) return st;
+  // the layout without the per-call float16 weights: the GEMM expands them tile by tile
+  const size_t need = qwam::act_layout(h->h, M, true).bytes;
   if (need > kStaticWsBytes) return QWAM_ERR_TOO_LARGE;
   void* ws = nullptr;
   const qwam_status sa = static_ws_address(&ws);
   if (sa != QWAM_OK) return sa;
-  return qwam_asp_linear(X_bf16, M, h, Y, y_dtype, ws, stream);
+  return qwam::linear_impl(X_bf16, M, h, Y, y_dtype, ws, stream, true);
 }
