@@ -35,7 +35,8 @@
 // Persistent CTAs, one per SM, walk the tiles with a static stride.  896 threads:
 //   warp 0        TMA producer: per K stage the packed codes of both operands and their scales
 //   warp 1        MMA issuer and TMEM owner
-//   warps 2, 3    idle
+//   warp 2        idle
+//   warp 3        with PREB (below): TMA producer of the float16 weight stages; else idle
 //   warps 4..19   expanders, two groups of eight that take alternate stages (group x the stages
 //                 whose running index is x mod 2), so that each warp has two stage times for its
 //                 work.  Warp e of a group takes the activation codes k = 32h .. 32h + 31
@@ -133,6 +134,10 @@ __device__ __forceinline__ uint32_t f32x2_to_bf16x2(float lo, float hi) {
 // reads around it as far as the compiler knows, which would serialize the epilogue.
 __device__ __forceinline__ void st_global_v4(void* p, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.global.v4.b32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(a), "r"(b), "r"(c), "r"(d));
+}
+__device__ __forceinline__ void st_global_v8(void* p, const uint32_t* v) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(v[0]), "r"(v[1]), "r"(v[2]),
+               "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]));
 }
 __device__ __forceinline__ uint32_t ld_nc_u16(const void* p) {
   unsigned short v;
@@ -302,53 +307,61 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();  // every global access of this kernel comes after the previous kernel's
 
   if (wid == 0) {
-    // ------------------------------------------------------------- TMA producer
+    // ------------------------------------------------------------- TMA producer (activations)
+    // Per K stage: the packed codes of both operands and their scales (with PREB: the activation
+    // codes and s_x; warp 3 brings the float16 weights).
     bool ok = true;
-    int s = 0, so = 0;
+    int s = 0;
     for (int ti = 0; ti < my_tiles && ok; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
-      for (int st = 0; st < (PREB ? nst : nks) && ok; ++st, ++so) {
-        if (st < nks) {
-          const int ps = s % SP;
-          if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
-          if (!ok) break;
-          uint8_t* p = pring + ps * PSTAGE;
-          if (elect_one()) {
-            if (PREB) {
-              mbar_arrive_expect_tx(&pfull[ps], PA + GPS * BM * 2);
-              tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
-              tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
-            } else {
-              mbar_arrive_expect_tx(&pfull[ps], PA + PB + GPS * (BM + BN) * 2);
-              tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
-              tma_load_2d(p + PA, &qw_map, &pfull[ps], st * (KS / 2), n0);
-              tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
-              tma_load_2d(p + PA + PB + PSX, &sw_map, &pfull[ps], n0, st * GPS);
-            }
+      for (int st = 0; st < nks && ok; ++st, ++s) {
+        const int ps = s % SP;
+        if (s >= SP) ok = mbar_wait_inline(&pempty[ps], ((s / SP) & 1) ^ 1, wc);
+        if (!ok) break;
+        uint8_t* p = pring + ps * PSTAGE;
+        if (elect_one()) {
+          if (PREB) {
+            mbar_arrive_expect_tx(&pfull[ps], PA + GPS * BM * 2);
+            tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
+            tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
+          } else {
+            mbar_arrive_expect_tx(&pfull[ps], PA + PB + GPS * (BM + BN) * 2);
+            tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
+            tma_load_2d(p + PA, &qw_map, &pfull[ps], st * (KS / 2), n0);
+            tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
+            tma_load_2d(p + PA + PB + PSX, &sw_map, &pfull[ps], n0, st * GPS);
           }
-          __syncwarp();
-          ++s;
         }
-        if (PREB) {
-          // the stage's float16 weights (W_perp, or B_hat in a branch stage) into the operand ring
-          const int os = so % SO;
-          if (so >= SO) ok = mbar_wait_inline(&oempty[os], ((so / SO) & 1) ^ 1, wc);
-          if (!ok) break;
-          if (elect_one()) {
-            mbar_arrive_expect_tx(&ofull[os], BSTAGE);
-            tma_load_2d(bring + os * BSTAGE, &bh_map, &ofull[os], st * KS, n0);
-          }
-          __syncwarp();
-        }
+        __syncwarp();
       }
     }
     // every issued load lands before the CTA can exit
     int never = 0;
     const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
     for (int j = (s > SP ? s - SP : 0); j < s; ++j) mbar_wait_inline(&pfull[j % SP], (j / SP) & 1, dc);
-    if (PREB)
-      for (int j = (so > SO ? so - SO : 0); j < so; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
+  } else if (wid == 3 && PREB) {
+    // ------------------------------------------------------------- TMA producer (weights, PREB)
+    // Every stage's float16 weights (W_perp, or B_hat in a branch stage) into the operand ring.
+    bool ok = true;
+    int so = 0;
+    for (int ti = 0; ti < my_tiles && ok; ++ti) {
+      int m0, n0;
+      tile_mn(ti, m0, n0);
+      for (int st = 0; st < nst && ok; ++st, ++so) {
+        const int os = so % SO;
+        if (so >= SO) ok = mbar_wait_inline(&oempty[os], ((so / SO) & 1) ^ 1, wc);
+        if (!ok) break;
+        if (elect_one()) {
+          mbar_arrive_expect_tx(&ofull[os], BSTAGE);
+          tma_load_2d(bring + os * BSTAGE, &bh_map, &ofull[os], st * KS, n0);
+        }
+        __syncwarp();
+      }
+    }
+    int never = 0;
+    const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
+    for (int j = (so > SO ? so - SO : 0); j < so; ++j) mbar_wait_inline(&ofull[j % SO], (j / SO) & 1, dc);
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
     constexpr uint32_t idesc = idesc_f16(BM, BN);
@@ -594,30 +607,64 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nb = n0 + 128 * hf + 32 * c;
         if (m < a.M) {
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int n = nb + 8 * j;
+          for (int j2 = 0; j2 < 2; ++j2) {  // 16 columns at a time: one 32-byte store per row (bf16)
+            const int n = nb + 16 * j2;
             if (n >= a.N) continue;
-            const float4 f0 = reinterpret_cast<const float4*>(fcb)[8 * c + 2 * j];
-            const float4 f1 = reinterpret_cast<const float4*>(fcb)[8 * c + 2 * j + 1];
-            const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[8 * c + 2 * j];
-            const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[8 * c + 2 * j + 1];
-            const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
-            const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-            float y[8];
+            // results of columns n + 8 h8 .. + 7: (acc 2^-e_n) 2^-e_m (+ bias)
+            auto cols8 = [&](int h8, float (&y)[8]) {
+              const int cb = 32 * c + 16 * j2 + 8 * h8;  // column within the warp's 128
+              const float4 f0 = reinterpret_cast<const float4*>(fcb)[cb / 4];
+              const float4 f1 = reinterpret_cast<const float4*>(fcb)[cb / 4 + 1];
+              const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
 #pragma unroll
-            for (int t = 0; t < 8; ++t) {
-              y[t] = (__uint_as_float(acc[8 * j + t]) * fn[t]) * fm;
-              if (a.bias) y[t] += bb[t];
-            }
+              for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(acc[16 * j2 + 8 * h8 + t]) * fn[t]) * fm;
+              if (a.bias) {
+                const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4];
+                const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4 + 1];
+                y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
+                y[4] += b1.x; y[5] += b1.y; y[6] += b1.z; y[7] += b1.w;
+              }
+            };
             const size_t off = static_cast<size_t>(m) * a.N + n;
+            const bool two = n + 16 <= a.N;  // N is a multiple of 8: the second 8 may lie past it
             if (a.y_f32) {
               float* yp = static_cast<float*>(a.Y) + off;
-              st_global_v4(yp, __float_as_uint(y[0]), __float_as_uint(y[1]), __float_as_uint(y[2]), __float_as_uint(y[3]));
-              st_global_v4(yp + 4, __float_as_uint(y[4]), __float_as_uint(y[5]), __float_as_uint(y[6]),
-                           __float_as_uint(y[7]));
+#pragma unroll
+              for (int h8 = 0; h8 < 2; ++h8) {
+                if (h8 == 1 && !two) break;
+                float y[8];
+                cols8(h8, y);
+                uint32_t u[8];
+#pragma unroll
+                for (int t = 0; t < 8; ++t) u[t] = __float_as_uint(y[t]);
+                if ((off & 7) == 0) {
+                  st_global_v8(yp + 8 * h8, u);
+                } else {
+                  st_global_v4(yp + 8 * h8, u[0], u[1], u[2], u[3]);
+                  st_global_v4(yp + 8 * h8 + 4, u[4], u[5], u[6], u[7]);
+                }
+              }
             } else {
-              st_global_v4(static_cast<__nv_bfloat16*>(a.Y) + off, f32x2_to_bf16x2(y[0], y[1]), f32x2_to_bf16x2(y[2], y[3]),
-                           f32x2_to_bf16x2(y[4], y[5]), f32x2_to_bf16x2(y[6], y[7]));
+              __nv_bfloat16* yp = static_cast<__nv_bfloat16*>(a.Y) + off;
+              uint32_t u[8];
+              {
+                float y[8];
+                cols8(0, y);
+#pragma unroll
+                for (int t = 0; t < 4; ++t) u[t] = f32x2_to_bf16x2(y[2 * t], y[2 * t + 1]);
+              }
+              if (two) {
+                float y[8];
+                cols8(1, y);
+#pragma unroll
+                for (int t = 0; t < 4; ++t) u[4 + t] = f32x2_to_bf16x2(y[2 * t], y[2 * t + 1]);
+              }
+              if (two && (off & 15) == 0) {
+                st_global_v8(yp, u);
+              } else {
+                st_global_v4(yp, u[0], u[1], u[2], u[3]);
+                if (two) st_global_v4(yp + 8, u[4], u[5], u[6], u[7]);
+              }
             }
           }
         }
