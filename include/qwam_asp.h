@@ -79,7 +79,8 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
 /* Bytes of the caller-owned activation workspace needed for M tokens.  For INT4 layers of 512 or
  * more tokens it includes a float16 copy of the layer's weights, N_pad (K + r_pad) 2 bytes (N_pad =
  * N rounded up to 256), which qwam_asp_gemm fills once per call and reads from L2 for every row
- * tile. */
+ * tile.  For 0 < r_pad <= 64 it also includes kernel (a)'s scratch for the partial projections of
+ * the C CTAs that share a row tile's K (float32, C M_pad r_pad 4 bytes, C <= 8). */
 qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes);
 
 /* Layout of the activation workspace for M tokens (byte offsets from its start):
@@ -138,9 +139,11 @@ qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* 
  *     per-call float16 copy of the weights that qwam_asp_act_workspace_bytes counts for INT4
  *     layers of 512 or more tokens (its GEMM converts the weights tile by tile instead), so it
  *     needs less than qwam_asp_act_workspace_bytes reports for such layers.  Per token the workspace holds about K/2 + 2K/G + 2 r_pad bytes (INT4) or
- *     K/2 + K/16 + 2 r_pad bytes (NVFP4): at K = 3072, group 64, r = 32 about 1.7 KB, so up to
- *     about 14,000 tokens fit.  A rotated handle with r > 0 also keeps its float32 remainder,
- *     4K more bytes per token: at K = 3072 about 1,780 tokens fit, and M = 4096 is refused.
+ *     K/2 + K/16 + 2 r_pad bytes (NVFP4), plus 4 C r_pad bytes for kernel (a)'s exchange of
+ *     partial projections (C = 2, 4 or 8 CTAs per row tile, fewer for more tokens): at K = 3072,
+ *     group 64, r = 32 about 2.2 KB, so up to about 12,800 tokens fit.  A rotated handle with
+ *     r > 0 also keeps its float32 remainder, 4K more bytes per token: at K = 3072 about 1,660
+ *     tokens fit, and M = 4096 is refused.
  *   - Nothing in the scratch needs to start at zero: kernel (a) writes every byte the GEMM
  *     then reads, on every call, so the scratch is never cleared.
  *   - One scratch per device: calls that may overlap in time on one device (different streams

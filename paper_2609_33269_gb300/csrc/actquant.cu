@@ -9,8 +9,9 @@
 // One CTA owns 128 token rows (one TMEM lane per row) and a slice of K; the C CTAs of a
 // thread-block cluster cover the whole of K for the same rows.  Each CTA streams its X slice
 // through a TMA ring twice: pass 1 feeds p_part = X_slice [U_hi | U_lo] into TMEM (bf16
-// tensor-core MMA, float32 accumulation); the partial projections are summed across the
-// cluster through distributed shared memory (fixed order, so every CTA sees the same p);
+// tensor-core MMA, float32 accumulation); the CTAs' partial projections meet in a float32
+// scratch in the workspace (through L2, one cluster barrier) and each CTA sums them in rank
+// order, so every CTA sees the same p;
 // pass 2 re-reads the slice (L2-resident by then) while the tensor cores form
 // R = [p_hi | p_hi | p_lo] [U_hi | U_lo | U_hi]^T chunk by chunk, and the epilogue warps form
 // X_perp = X - R in float32 and quantize it.  With r = 0 the kernel is one streaming pass.
@@ -23,9 +24,12 @@
 // NVFP4 variant (App. B.1, the same kernel with one template flag): per block of 16 K an E4M3
 // scale (in the 512-byte atoms the GEMM copies to tensor memory) and E2M1 codes, two per byte.
 //
-// Warp roles (320 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2..9
-// epilogue: warps 2..5 and 6..9 each cover the four 32-row TMEM quadrants and take the even
-// and the odd K chunks respectively.
+// Warp roles (576 threads): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2..17
+// epilogue: in groups of four they cover the four 32-row TMEM quadrants, and the groups take
+// (even chunks, columns 0..31), (odd, 0..31), (even, 32..63), (odd, 32..63) of each 64-column
+// chunk, one thread per row.  A group of 64 columns has its absmax formed from the two halves'
+// partial maxima, swapped through shared memory.  The quantizer's codes come from a fast
+// rounding that an exact remainder test confirms (codes8_fast).
 //
 // Also in this file, sharing kernel (a)'s quantizers (the same rounding, bit for bit):
 //   rotquant_kernel  smoothing and block Hadamard rotation of the remainder (Sec. 3 Eq. (pair)),
@@ -48,6 +52,7 @@ struct ActArgs {
   uint8_t* sf;      // NVFP4: E4M3 block scales in 512-byte atoms
   __nv_bfloat16* scales;  // [K/G, M_pad]
   __half* phat;     // [M, RP]
+  float* part;      // [C, M_pad, RP] float32: the CTAs' partial projections, exchanged through L2
   float* dump;      // optional [M, K]
   int resid_only;   // rotated layer: write the remainder to dump and stop (the rotation kernel quantizes)
   int* err;
@@ -55,6 +60,7 @@ struct ActArgs {
 };
 
 constexpr int kNumRec = 4;  // TMEM reconstruction buffers (64 columns each)
+constexpr int kActThreads = 576;  // warp 0 TMA, warp 1 MMA, warps 2..17 epilogue
 
 template <int RP>
 struct ActCfg {
@@ -66,9 +72,9 @@ struct ActCfg {
   static constexpr int STAGE = X_BYTES + U_BYTES;
   static constexpr int S = RP == 0 ? 8 : (RP <= 32 ? 4 : (RP <= 48 ? 3 : 2));
   static constexpr int AREC_BYTES = kBM * KU3 * 2;
-  static constexpr int PP_BYTES = kBM * RP * 4;
-  static constexpr int NBAR = 2 * S + 3 + 2 * kNumRec;
-  static constexpr int SMEM = 1024 + S * STAGE + AREC_BYTES + 2 * PP_BYTES + NBAR * 8 + 16;
+  static constexpr int XAM_BYTES = 2 * 2 * 2 * kBM * 4;  // partial absmax: [use & 1][parity][half][row]
+  static constexpr int NBAR = 2 * S + 3 + 2 * kNumRec + 8;
+  static constexpr int SMEM = 1024 + S * STAGE + AREC_BYTES + XAM_BYTES + NBAR * 8 + 16;
   static constexpr uint32_t TMEM_COLS = 512;  // proj at col 0 (2*RP <= 128), rec buffers at 128 + 64 b
   static_assert(SMEM <= 232448, "kernel (a) shared memory above the 227 KB per-CTA limit");
 };
@@ -111,21 +117,65 @@ __device__ __forceinline__ float bf16_scale_div7(float amax) {
   return __bfloat162float(__float2bfloat16_rn(qo));
 }
 
-// One group of GS remainder values -> scale and GS/8 OB4 words of codes.  The absmax is formed
-// as a tree (max is exact, so the order does not matter), which keeps the dependency chain short.
+// ---- packed float32 pairs: two IEEE round-to-nearest operations per instruction, each rounded
+// exactly as its scalar form.
+__device__ __forceinline__ uint64_t f2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_split(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma_f32x2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t sub_f32x2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// Eight values -> a candidate OB4 word, and the largest |x - c s| over them folded into emax.
+// t = RN(x * inv + (1.5 * 2^23 + 8)) is an integer-valued float whose low four bits are c + 8 for
+// the candidate code c = t - (1.5 * 2^23 + 8) (|c| <= 8), so the nibbles come straight from t's
+// bits.  The candidate is the nearest code exactly when |x - c s| < s/2: a wrong neighbour and a
+// tie both give |x - c s| >= s/2 (a rounded remainder keeps that order, s/2 being a float), which
+// is the caller's test for the whole group.
+constexpr float kMagic8 = 12582920.0f;
+__device__ __forceinline__ uint32_t codes8_fast(const float* x, uint64_t inv2, uint64_t nsc2, float& emax) {
+  const uint64_t m2 = f2(kMagic8, kMagic8), nm2 = f2(-kMagic8, -kMagic8);
+  uint32_t t[8];
+#pragma unroll
+  for (int u = 0; u < 8; u += 2) {
+    const uint64_t x2 = f2(x[u], x[u + 1]);
+    const uint64_t t2 = fma_f32x2(x2, inv2, m2);
+    const uint64_t e2 = fma_f32x2(add_f32x2(t2, nm2), nsc2, x2);
+    float tl, th, el, eh;
+    f2_split(t2, tl, th);
+    f2_split(e2, el, eh);
+    t[u] = __float_as_uint(tl);
+    t[u + 1] = __float_as_uint(th);
+    emax = fmaxf(emax, fmaxf(fabsf(el), fabsf(eh)));
+  }
+  // OB4: the code of k = 2p in bits 4p.., the code of k = 2p + 1 in bits 16 + 4p..
+  uint32_t q[4];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) q[p] = __byte_perm(t[2 * p], t[2 * p + 1], 0x5410) & 0x000F000Fu;
+  return q[0] | (q[1] << 4) | (q[2] << 8) | (q[3] << 12);
+}
+
+// The codes of a group with the exact test per value (nearest_code): the path for a group whose
+// fast candidates failed the remainder test, and for a zero or tiny scale.
 template <int GS>
-__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words, __nv_bfloat16* scale_out) {
-  float mx[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) mx[j] = fabsf(xp[j]);
-#pragma unroll
-  for (int i = 8; i < GS; ++i) mx[i & 7] = fmaxf(mx[i & 7], fabsf(xp[i]));
-#pragma unroll
-  for (int w = 4; w >= 1; w >>= 1)
-#pragma unroll
-    for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
-  const float amax = mx[0];
-  const float sc = bf16_scale_div7(amax);
+__device__ __forceinline__ void codes_exact(const float* xp, uint32_t* words, float sc) {
   // Codes are invariant under a common power-of-two scaling of the values and the scale (exact
   // in float32), which keeps 1/s finite for the rare group whose scale is tiny.
   const float k = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100
@@ -139,6 +189,46 @@ __device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words,
     for (int u = 0; u < 8; ++u) c[u] = nearest_code(xp[8 * w + u] * k, scs, inv, hs);
     words[w] = ob4_word(c);
   }
+}
+
+// The largest |x| of GS values, formed as a tree (max is exact, so the order does not matter),
+// which keeps the dependency chain short.
+template <int GS>
+__device__ __forceinline__ float absmax(const float* xp) {
+  float mx[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) mx[j] = fabsf(xp[j]);
+#pragma unroll
+  for (int i = 8; i < GS; ++i) mx[i & 7] = fmaxf(mx[i & 7], fabsf(xp[i]));
+#pragma unroll
+  for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+    for (int j = 0; j < w; ++j) mx[j] = fmaxf(mx[j], mx[j + w]);
+  return mx[0];
+}
+
+// GS values -> GS/8 OB4 words of their nearest codes under the scale sc.  The codes take the fast
+// candidates of codes8_fast; values whose candidates fail the remainder test (a near-tie, rare),
+// and a zero or tiny scale, are redone by the exact per-value test.
+template <int GS>
+__device__ __forceinline__ void codes_for_scale(const float* xp, uint32_t* words, float sc) {
+  bool exact = !(sc >= 7.8886091e-31f);  // zero or tiny scale
+  if (!exact) {
+    const float inv = rcp_approx(sc);
+    const uint64_t inv2 = f2(inv, inv), nsc2 = f2(-sc, -sc);
+    float em[2] = {0.0f, 0.0f};
+#pragma unroll
+    for (int w = 0; w < GS / 8; ++w) words[w] = codes8_fast(xp + 8 * w, inv2, nsc2, em[w & 1]);
+    exact = fmaxf(em[0], em[1]) >= 0.5f * sc;
+  }
+  if (exact) codes_exact<GS>(xp, words, sc);
+}
+
+// One group of GS remainder values -> scale and GS/8 OB4 words of codes.
+template <int GS>
+__device__ __forceinline__ void quantize_group(const float* xp, uint32_t* words, __nv_bfloat16* scale_out) {
+  const float sc = bf16_scale_div7(absmax<GS>(xp));
+  codes_for_scale<GS>(xp, words, sc);
   *scale_out = __float2bfloat16_rn(sc);  // exact: sc is a bfloat16 value
 }
 
@@ -217,7 +307,7 @@ __device__ __forceinline__ uint32_t quantize_block_nvfp4(const float* x, uint32_
 }
 
 template <int RP, bool NV>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(kActThreads, 1)
     actquant_kernel(const __grid_constant__ CUtensorMap x_map, const __grid_constant__ CUtensorMap ut_map,
                     const __grid_constant__ CUtensorMap u3_map, const ActArgs a) {
   using Cfg = ActCfg<RP>;
@@ -227,9 +317,8 @@ __global__ void __launch_bounds__(320, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* stages = smem;
   uint8_t* arec = stages + S * Cfg::STAGE;
-  float* ppart = reinterpret_cast<float*>(arec + Cfg::AREC_BYTES);
-  float* pred = ppart + kBM * RP;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(pred) + Cfg::PP_BYTES);
+  float* xam = reinterpret_cast<float*>(arec + Cfg::AREC_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(arec + Cfg::AREC_BYTES + Cfg::XAM_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + S;
   uint64_t* proj_done = bars + 2 * S;
@@ -237,6 +326,7 @@ __global__ void __launch_bounds__(320, 1)
   uint64_t* drain = proj_done + 2;
   uint64_t* tfull = proj_done + 3;
   uint64_t* tempty = tfull + kNumRec;
+  uint64_t* xch = tempty + kNumRec;  // [parity * 4 + quadrant]: the two halves' partial absmax are in
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + Cfg::NBAR);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
@@ -252,15 +342,16 @@ __global__ void __launch_bounds__(320, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 4);  // pass 2: the four warps of one chunk parity; pass 1: the MMA commit + 3
+      mbar_init(&empty[i], 8);  // pass 2: the eight warps of one chunk parity; pass 1: the MMA commit + 7
     }
     mbar_init(proj_done, 1);
     mbar_init(arec_ready, 8);   // epilogue warps
     mbar_init(drain, 1);
     for (int i = 0; i < kNumRec; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], 4);   // the four warps of one chunk parity
+      mbar_init(&tempty[i], 8);   // the eight warps of one chunk parity
     }
+    for (int i = 0; i < 8; ++i) mbar_init(&xch[i], 2);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -283,7 +374,7 @@ __global__ void __launch_bounds__(320, 1)
     bool ok = true;
     auto produce = [&](bool first_pass, int c) {
       const int s = it % S;
-      if (ok && it >= S) ok = mbar_wait(&empty[s], ((it / S) & 1) ^ 1, wc);
+      if (ok && it >= S) ok = mbar_wait_inline(&empty[s], ((it / S) & 1) ^ 1, wc);
       if (ok && elect_one()) {
         const uint32_t bytes = Cfg::X_BYTES + (first_pass ? Cfg::U1_BYTES : (RP > 0 ? Cfg::U2_BYTES : 0));
         mbar_arrive_expect_tx(&full[s], bytes);
@@ -303,16 +394,12 @@ __global__ void __launch_bounds__(320, 1)
     __syncwarp();
     for (int c = 0; c < pass1; ++c) produce(true, c);
     for (; issued2 < nch && issued2 < S; ++issued2) produce(false, issued2);
-    if (RP > 0) {
-      cluster_sync();
-      cluster_sync();
-      cluster_sync();
-    }
+    if (RP > 0) cluster_sync();
     for (; issued2 < nch; ++issued2) produce(false, issued2);
     // Let every load issued into the ring land before the CTA can exit.
     int never = 0;
     const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-    for (int j = (it > S ? it - S : 0); j < it; ++j) mbar_wait(&full[j % S], (j / S) & 1, dc);
+    for (int j = (it > S ? it - S : 0); j < it; ++j) mbar_wait_inline(&full[j % S], (j / S) & 1, dc);
   } else if (wid == 1) {
     // ------------------------------------------------------------- MMA issuer
     if constexpr (RP > 0) {
@@ -322,7 +409,7 @@ __global__ void __launch_bounds__(320, 1)
         constexpr uint32_t idesc_proj = idesc_bf16(kBM, 2 * RP);
         for (int c = 0; c < nch && ok; ++c) {
           const int s = c % S;
-          ok = mbar_wait(&full[s], (c / S) & 1, wc);
+          ok = mbar_wait_inline(&full[s], (c / S) & 1, wc);
           if (!ok) break;
           tc_fence_after();
           const uint32_t xa = smem_u32(stage_x(s)), ua = smem_u32(stage_u(s));
@@ -331,10 +418,9 @@ __global__ void __launch_bounds__(320, 1)
             for (int kk = 0; kk < 4; ++kk)
               mma_f16(tmem, smem_desc(xa + kk * 32, 16, 1024, kSw128), smem_desc(ua + kk * 32, 16, 1024, kSw128),
                       idesc_proj, (c | kk) != 0);
-            // the stage frees when these MMAs complete (the commit is the last of four arrivals)
-            mbar_arrive(&empty[s]);
-            mbar_arrive(&empty[s]);
-            mbar_arrive(&empty[s]);
+            // the stage frees when these MMAs complete (the commit is the last of eight arrivals)
+#pragma unroll
+            for (int i = 0; i < 7; ++i) mbar_arrive(&empty[s]);
             mma_commit(&empty[s]);
           }
           __syncwarp();
@@ -343,17 +429,15 @@ __global__ void __launch_bounds__(320, 1)
       }
       __syncwarp();
       cluster_sync();
-      cluster_sync();
-      cluster_sync();
       {
-        if (ok) ok = mbar_wait(arec_ready, 0, wc);
+        if (ok) ok = mbar_wait_inline(arec_ready, 0, wc);
         tc_fence_after();
         constexpr uint32_t idesc_rec = idesc_bf16(kBM, kChunk);
         const uint32_t ar = smem_u32(arec);
         for (int c = 0; c < nch && ok; ++c) {
           const int it = pass1 + c, s = it % S, b = c % kNumRec;
-          ok = mbar_wait(&full[s], (it / S) & 1, wc);
-          if (ok && c >= kNumRec) ok = mbar_wait(&tempty[b], ((c / kNumRec) & 1) ^ 1, wc);
+          ok = mbar_wait_inline(&full[s], (it / S) & 1, wc);
+          if (ok && c >= kNumRec) ok = mbar_wait_inline(&tempty[b], ((c / kNumRec) & 1) ^ 1, wc);
           if (!ok) break;
           tc_fence_after();
           const uint32_t ua = smem_u32(stage_u(s));
@@ -373,25 +457,30 @@ __global__ void __launch_bounds__(320, 1)
         __syncwarp();
         int never = 0;
         const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
-        mbar_wait(drain, 0, dc);
+        mbar_wait_inline(drain, 0, dc);
       }
       __syncwarp();
     }
   } else {
     // ------------------------------------------------------------- epilogue (thread = row)
+    // Warp 2 + e (e = 0..15): TMEM quadrant wid & 3, chunk parity (e >> 2) & 1, and half e >> 3 of
+    // each chunk's 64 columns in pass 2; the eight warps of half 0 also form p (pass 1's epilogue).
     const int quad = wid & 3;
-    const int par = (static_cast<int>(wid) - 2) >> 2;  // 0: even chunks, 1: odd chunks
+    const int par = ((static_cast<int>(wid) - 2) >> 2) & 1;  // 0: even chunks, 1: odd chunks
+    const int half = (static_cast<int>(wid) - 2) >> 3;
     const int row = quad * 32 + static_cast<int>(lane);
     const int m = m0 + row;
-    const int et = static_cast<int>(wid - 2) * 32 + static_cast<int>(lane);  // 0..255
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     bool ok = true;
 
     if constexpr (RP > 0) {
+     if (half == 1) {
+      cluster_sync();  // the exchange barrier of the projection below
+     } else {
       constexpr int HR = RP / 2;  // projection columns handled by this thread (half of them)
       const int j0 = par * HR;
       // -- partial projection of this CTA's K slice: hi part + lo part, columns [j0, j0 + HR)
-      ok = mbar_wait(proj_done, 0, wc);
+      ok = mbar_wait_inline(proj_done, 0, wc);
       tc_fence_after();
       float pp[HR];
 #pragma unroll
@@ -411,50 +500,57 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
         for (int i = 0; i < 8; ++i) pp[q * 8 + i] = __uint_as_float(vh[i]) + __uint_as_float(vl[i]);
       }
-      float4* prow = reinterpret_cast<float4*>(ppart + row * RP + j0);
+      // -- the partial goes to the float32 scratch (slice `rank`, row m0 + row, columns
+      //    [j0, j0 + HR)); the cluster barrier's release / acquire orders it before the reads below
+      {
+        float4* dst = reinterpret_cast<float4*>(a.part + (static_cast<size_t>(rank) * a.M_pad + m0 + row) * RP + j0);
 #pragma unroll
-      for (int j = 0; j < HR / 4; ++j) prow[j] = make_float4(pp[4 * j], pp[4 * j + 1], pp[4 * j + 2], pp[4 * j + 3]);
-      cluster_sync();  // A: every CTA's partial is in its shared memory
-      // -- reduce-scatter: this CTA sums rows [rank*Rc, (rank+1)*Rc) over the cluster, in rank order
-      const int Rc = kBM / C;
-      const int n4 = Rc * RP / 4;
-      const uint32_t pp_base = smem_u32(ppart);
-      for (int i = et; i < n4; i += 256) {
-        const uint32_t off = static_cast<uint32_t>((static_cast<int>(rank) * Rc * RP + 4 * i) * 4);
-        float4 acc = ld_dsmem_f4(mapa_smem(pp_base + off, 0));
-        for (int q = 1; q < C; ++q) {
-          const float4 v = ld_dsmem_f4(mapa_smem(pp_base + off, static_cast<uint32_t>(q)));
-          acc.x += v.x;
-          acc.y += v.y;
-          acc.z += v.z;
-          acc.w += v.w;
-        }
-        reinterpret_cast<float4*>(pred)[i] = acc;
-        const int lr = (4 * i) / RP, col = (4 * i) % RP;
-        const int gm = m0 + static_cast<int>(rank) * Rc + lr;
-        if (gm < a.M) {
-          __half2 h01 = __floats2half2_rn(acc.x, acc.y), h23 = __floats2half2_rn(acc.z, acc.w);
-          uint2 hv;
-          hv.x = *reinterpret_cast<uint32_t*>(&h01);
-          hv.y = *reinterpret_cast<uint32_t*>(&h23);
-          *reinterpret_cast<uint2*>(a.phat + static_cast<size_t>(gm) * RP + col) = hv;
-        }
+        for (int j = 0; j < HR / 4; ++j) dst[j] = make_float4(pp[4 * j], pp[4 * j + 1], pp[4 * j + 2], pp[4 * j + 3]);
       }
-      cluster_sync();  // B: the reduced rows are in their owners' shared memory
-      // -- gather this thread's half row of p from its owner
-      const int owner = row / Rc, lr = row % Rc;
-      const uint32_t pr_base = smem_u32(pred);
+      cluster_sync();  // every partial of the cluster is in the scratch
+      // -- p for this thread's row and columns: the C partials summed in rank order (every CTA of
+      //    the cluster forms the same p), the loads of QL slices in flight at a time
       float p[HR];
+      {
+        constexpr int QL = HR <= 16 ? 64 / HR : 2;  // at most 16 float4 loads per round
+        const float* src = a.part + static_cast<size_t>(m0 + row) * RP + j0;
+        const size_t slice = static_cast<size_t>(a.M_pad) * RP;
 #pragma unroll
-      for (int j = 0; j < HR / 4; ++j) {
-        const float4 v = ld_dsmem_f4(mapa_smem(pr_base + static_cast<uint32_t>((lr * RP + j0 + 4 * j) * 4),
-                                               static_cast<uint32_t>(owner)));
-        p[4 * j] = v.x;
-        p[4 * j + 1] = v.y;
-        p[4 * j + 2] = v.z;
-        p[4 * j + 3] = v.w;
+        for (int j = 0; j < HR; ++j) p[j] = 0.0f;
+        for (int q0 = 0; q0 < C; q0 += QL) {
+          float4 v[QL][HR / 4];
+#pragma unroll
+          for (int i = 0; i < QL; ++i)
+#pragma unroll
+            for (int j = 0; j < HR / 4; ++j)
+              v[i][j] = q0 + i < C ? reinterpret_cast<const float4*>(src + (q0 + i) * slice)[j] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int i = 0; i < QL; ++i) {
+            if (q0 + i >= C) break;
+#pragma unroll
+            for (int j = 0; j < HR / 4; ++j) {
+              // rank 0's slice starts the sum exactly (0 + x == x), then the others in order
+              p[4 * j] += v[i][j].x;
+              p[4 * j + 1] += v[i][j].y;
+              p[4 * j + 2] += v[i][j].z;
+              p[4 * j + 3] += v[i][j].w;
+            }
+          }
+        }
       }
-      cluster_sync();  // C: no CTA reads a peer's shared memory after this point
+      // -- p_hat = RN_f16(p): each row written once, by the CTA whose rank owns its slice of rows
+      if (row / (kBM / C) == static_cast<int>(rank) && m < a.M) {
+#pragma unroll
+        for (int j = 0; j < HR / 8; ++j) {
+          uint32_t w[4];
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const __half2 h2 = __floats2half2_rn(p[8 * j + 2 * t], p[8 * j + 2 * t + 1]);
+            w[t] = *reinterpret_cast<const uint32_t*>(&h2);
+          }
+          reinterpret_cast<uint4*>(a.phat + static_cast<size_t>(m) * RP + j0)[j] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+      }
       // -- A operand of the reconstruction: [p_hi | p_hi | p_lo | 0], 128-byte swizzle.
       //    This thread writes its columns j0..j0+HR-1 of each segment (8 bf16 = one 16-byte chunk).
       __nv_bfloat16 hi[HR], lo[HR];
@@ -485,82 +581,88 @@ __global__ void __launch_bounds__(320, 1)
       }
       fence_proxy_async_smem();
       warp_arrive(arec_ready);
+     }
     }
 
-    // -- pass 2: remainder and quantization; this warp takes the chunks of its parity
-    for (int c = par; c < nch; c += 2) {
+    // -- pass 2: remainder and quantization; this warp takes, of each chunk of its parity, the 32
+    //    columns of its half for the 32 rows of its quadrant
+    for (int c = par, use = 0; c < nch; c += 2, ++use) {
       const int it = pass1 + c, s = it % S;
-      float xp[kChunk];
+      float xp[32];
       if constexpr (RP > 0) {
         const int b = c % kNumRec;
-        if (ok) ok = mbar_wait(&tfull[b], (c / kNumRec) & 1, wc);
+        if (ok) ok = mbar_wait_inline(&tfull[b], (c / kNumRec) & 1, wc);
         tc_fence_after();
-        uint32_t r0[32], r1[32];
-        tmem_ld32(tlane + 128 + 64 * b, r0);
-        tmem_ld32(tlane + 128 + 64 * b + 32, r1);
+        uint32_t r0[32];
+        tmem_ld32(tlane + 128 + 64 * b + 32 * half, r0);
         tmem_ld_wait();
         tc_fence_before();
         warp_arrive(&tempty[b]);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          xp[i] = __uint_as_float(r0[i]);
-          xp[32 + i] = __uint_as_float(r1[i]);
-        }
-      } else {
-#pragma unroll
-        for (int i = 0; i < kChunk; ++i) xp[i] = 0.0f;
+        for (int i = 0; i < 32; ++i) xp[i] = __uint_as_float(r0[i]);
       }
-      if (ok) ok = mbar_wait(&full[s], (it / S) & 1, wc);
+      if (ok) ok = mbar_wait_inline(&full[s], (it / S) & 1, wc);
       const uint8_t* xs = stage_x(s) + row * 128;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const uint4 v = *reinterpret_cast<const uint4*>(xs + ((j ^ (row & 7)) << 4));
+      for (int j = 0; j < 4; ++j) {
+        const uint4 v = *reinterpret_cast<const uint4*>(xs + (((4 * half + j) ^ (row & 7)) << 4));
         const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const float lo_f = __uint_as_float(wv[t] << 16);
           const float hi_f = __uint_as_float(wv[t] & 0xFFFF0000u);
-          xp[8 * j + 2 * t] = lo_f - xp[8 * j + 2 * t];
-          xp[8 * j + 2 * t + 1] = hi_f - xp[8 * j + 2 * t + 1];
+          if constexpr (RP > 0) {
+            const uint64_t d = sub_f32x2(f2(lo_f, hi_f), f2(xp[8 * j + 2 * t], xp[8 * j + 2 * t + 1]));
+            f2_split(d, xp[8 * j + 2 * t], xp[8 * j + 2 * t + 1]);
+          } else {
+            xp[8 * j + 2 * t] = lo_f;
+            xp[8 * j + 2 * t + 1] = hi_f;
+          }
         }
       }
       // The stage goes back to the TMA producer: order these generic-proxy reads before the
-      // async-proxy write that will refill it; each of the four warps that read it releases it.
+      // async-proxy write that will refill it; each of the eight warps that read it releases it.
       fence_proxy_async_smem();
       warp_arrive(&empty[s]);
-      if (!ok || m >= a.M) continue;
-
-      const int kc = k0 + c * kChunk;
+      const bool live = ok && m < a.M;
+      const int kc = k0 + c * kChunk + 32 * half;  // this half's first column
       if (a.dump) {
-        float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + kc);
+        if (live) {
+          float4* d = reinterpret_cast<float4*>(a.dump + static_cast<size_t>(m) * a.K + kc);
 #pragma unroll
-        for (int i = 0; i < kChunk / 4; ++i) d[i] = make_float4(xp[4 * i], xp[4 * i + 1], xp[4 * i + 2], xp[4 * i + 3]);
+          for (int i = 0; i < 8; ++i) d[i] = make_float4(xp[4 * i], xp[4 * i + 1], xp[4 * i + 2], xp[4 * i + 3]);
+        }
         if (a.resid_only) continue;
       }
+      uint8_t* crow = a.codes + static_cast<size_t>(m) * (a.K / 2) + kc / 2;
       if constexpr (NV) {
-        uint32_t w[8];
-        uint32_t sf4 = 0;
-#pragma unroll
-        for (int b = 0; b < 4; ++b) sf4 |= quantize_block_nvfp4(xp + 16 * b, w + 2 * b) << (8 * b);
-        uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * (a.K / 2) + kc / 2);
-        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
-        dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+        if (!live) continue;
+        uint32_t w[4];
+        const uint32_t sf2 = quantize_block_nvfp4(xp, w) | (quantize_block_nvfp4(xp + 16, w + 2) << 8);
+        *reinterpret_cast<uint4*>(crow) = make_uint4(w[0], w[1], w[2], w[3]);
         const int mr = m % kBM;
-        *reinterpret_cast<uint32_t*>(a.sf + (static_cast<size_t>(m / kBM) * (a.K / 64) + kc / 64) * kSfAtom +
-                                     (mr % 32) * 16 + (mr / 32) * 4) = sf4;
+        *reinterpret_cast<uint16_t*>(a.sf + (static_cast<size_t>(m / kBM) * (a.K / 64) + (kc - 32 * half) / 64) * kSfAtom +
+                                     (mr % 32) * 16 + (mr / 32) * 4 + 2 * half) = static_cast<uint16_t>(sf2);
         continue;
       }
-      uint32_t words[8];
+      uint32_t words[4];
       if (a.G == 64) {
-        quantize_group<64>(xp, words, a.scales + static_cast<size_t>(kc / 64) * a.M_pad + m);
+        // The group spans both halves: the two warps of this quadrant and parity swap their
+        // partial absmax through shared memory (double-buffered by use, one pairwise barrier).
+        float* slot = xam + ((use & 1) * 4 + par * 2) * kBM;
+        const float am = absmax<32>(xp);
+        slot[half * kBM + row] = am;
+        warp_arrive(&xch[par * 4 + quad]);
+        if (!mbar_wait_inline(&xch[par * 4 + quad], use & 1, wc)) ok = false;
+        const float sc = bf16_scale_div7(fmaxf(am, slot[(half ^ 1) * kBM + row]));
+        codes_for_scale<32>(xp, words, sc);
+        if (half == 0 && live) a.scales[static_cast<size_t>((kc - 32 * half) / 64) * a.M_pad + m] = __float2bfloat16_rn(sc);
       } else {
-        const size_t gi = static_cast<size_t>(kc / 32) * a.M_pad + m;
-        quantize_group<32>(xp, words, a.scales + gi);
-        quantize_group<32>(xp + 32, words + 4, a.scales + gi + a.M_pad);
+        const float sc = bf16_scale_div7(absmax<32>(xp));
+        codes_for_scale<32>(xp, words, sc);
+        if (live) a.scales[static_cast<size_t>(kc / 32) * a.M_pad + m] = __float2bfloat16_rn(sc);
       }
-      uint4* dst = reinterpret_cast<uint4*>(a.codes + static_cast<size_t>(m) * (a.K / 2) + kc / 2);
-      dst[0] = make_uint4(words[0], words[1], words[2], words[3]);
-      dst[1] = make_uint4(words[4], words[5], words[6], words[7]);
+      if (live) *reinterpret_cast<uint4*>(crow) = make_uint4(words[0], words[1], words[2], words[3]);
     }
   }
 
@@ -702,14 +804,16 @@ __device__ __forceinline__ void quantize8_lanes(const float* x, int lane, int m,
     am = fmaxf(am, __shfl_xor_sync(kAll, am, 2));
     if (o.G == 64) am = fmaxf(am, __shfl_xor_sync(kAll, am, 4));
     const float sc = bf16_scale_div7(am);
-    const float ks = (sc < 7.8886091e-31f) ? 1.2676506e30f : 1.0f;  // 2^-100, 2^100 (see quantize_group)
-    const float scs = sc * ks;
-    const float inv = sc > 0.0f ? rcp_approx(scs) : 0.0f;
-    const float hs = 0.5f * scs;
-    int c[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) c[i] = nearest_code(x[i] * ks, scs, inv, hs);
-    *reinterpret_cast<uint32_t*>(o.codes + static_cast<size_t>(m) * (o.K / 2) + k / 2) = ob4_word(c);
+    uint32_t word = 0u;
+    bool exact = !(sc >= 7.8886091e-31f);  // zero or tiny scale
+    if (!exact) {
+      const float inv = rcp_approx(sc);
+      float em = 0.0f;
+      word = codes8_fast(x, f2(inv, inv), f2(-sc, -sc), em);
+      exact = em >= 0.5f * sc;
+    }
+    if (exact) codes_exact<8>(x, &word, sc);
+    *reinterpret_cast<uint32_t*>(o.codes + static_cast<size_t>(m) * (o.K / 2) + k / 2) = word;
     if ((lane & (o.G / 8 - 1)) == 0) o.scales[static_cast<size_t>(k / o.G) * o.M_pad + m] = __float2bfloat16_rn(sc);
   }
 }
@@ -1124,13 +1228,6 @@ __global__ void __launch_bounds__(256) debug_lanes_kernel(const float* __restric
 }
 
 // Cluster size (CTAs along K per 128-row tile): as many as fit one wave of the GPU.
-int choose_split(int K, int tiles, int sms) {
-  const int chunks = K / kChunk;
-  int C = 1;
-  while (C < 8 && chunks % (2 * C) == 0 && tiles * 2 * C <= sms) C *= 2;
-  if (C == 1 && chunks % 2 == 0 && tiles < sms) C = 2;
-  return C;
-}
 
 template <int RP, bool NV>
 cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, bool resid_only,
@@ -1142,7 +1239,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   a.K = h.K;
   a.G = h.G;
   const int tiles = (M + kBM - 1) / kBM;
-  const int C = choose_split(h.K, tiles, h.num_sms);
+  const int C = act_split(h.K, tiles, h.num_sms);
   a.C = C;
   a.Kc = h.K / C;
   a.M_pad = L.M_pad;
@@ -1151,6 +1248,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   a.sf = base + L.scales_off;
   a.scales = reinterpret_cast<__nv_bfloat16*>(base + L.scales_off);
   a.phat = reinterpret_cast<__half*>(base + L.phat_off);
+  a.part = reinterpret_cast<float*>(base + L.part_off);
   a.dump = dump;
   a.resid_only = resid_only ? 1 : 0;
   a.err = h.err;
@@ -1164,7 +1262,7 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(C, tiles, 1);
-  cfg.blockDim = dim3(320, 1, 1);
+  cfg.blockDim = dim3(kActThreads, 1, 1);
   cfg.dynamicSmemBytes = Cfg::SMEM;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];

@@ -78,15 +78,40 @@ bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const
   return r == CUDA_SUCCESS;
 }
 
+const CUtensorMap* get_y_map(Handle& h, const void* Y, int M, bool y_f32) {
+  for (auto& c : h.y_cache)
+    if (c.y == Y && c.M == M && c.f32 == y_f32) return &c.map;
+  Handle::YMap& c = h.y_cache[h.y_next];
+  c.y = nullptr;
+  const uint32_t es = y_f32 ? 4u : 2u;
+  if (!encode_2d(&c.map, y_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, Y, h.N, M,
+                 static_cast<uint64_t>(h.N) * es, 128 / es, 32, CU_TENSOR_MAP_SWIZZLE_128B))
+    return nullptr;
+  c.y = Y;
+  c.M = M;
+  c.f32 = y_f32;
+  h.y_next = (h.y_next + 1) % 4;
+  return &c.map;
+}
+
 ActLayout act_layout(const Handle& h, int M, bool lean) {
   ActLayout L;
   L.M_pad = round_up(M > 0 ? M : 1, kBM);
   L.codes_off = 0;
+  // kernel (a)'s exchange of partial projections (handles whose rank it takes on the tensor cores)
+  auto add_part = [&](ActLayout& l) {
+    l.part_off = 0;
+    if (h.r_pad == 0 || h.r_pad > kMaxRank) return;
+    l.part_off = l.bytes;
+    const int C = act_split(h.K, l.M_pad / kBM, h.num_sms);
+    l.bytes += up256(static_cast<size_t>(C) * l.M_pad * h.r_pad * 4);
+  };
   if (h.fmt == kFmtNvfp4) {  // packed codes [M, K/2], scale atoms (M_pad rows), no epilogue constants
     L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
     L.ab_off = L.scales_off + up256(static_cast<size_t>(L.M_pad) * (h.K / kFp4Block));
     L.phat_off = L.ab_off;
     L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
+    add_part(L);
     L.resid_off = 0;
     if (h.rot && h.r > 0) {
       L.resid_off = L.bytes;
@@ -104,6 +129,7 @@ ActLayout act_layout(const Handle& h, int M, bool lean) {
   L.ab_off = L.scales_off + up256(static_cast<size_t>(h.K / h.G) * L.M_pad * 2);
   L.phat_off = L.ab_off;
   L.bytes = L.phat_off + up256(static_cast<size_t>(M) * h.r_pad * 2 + 16);
+  add_part(L);
   L.resid_off = 0;
   if (h.rot && h.r > 0) {
     L.resid_off = L.bytes;

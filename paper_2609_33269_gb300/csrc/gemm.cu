@@ -86,7 +86,7 @@ constexpr int SP = 4, SO = 4;
 constexpr int PA = BM * KS / 2;          // packed A bytes per stage (4 KB)
 constexpr int PB = BN * KS / 2;          // packed B bytes per stage (8 KB)
 constexpr int PSX = 2 * BM * 2;          // s_x [GPS][128] bf16 (room for two groups)
-constexpr int PSTAGE = PA + PB + PSX + 2 * BN * 2;  // then s_w 2^e_n [GPS][256] f16
+constexpr int PSTAGE = PA + PSX + 2 * BN * 2;  // packed A, s_x, then s_w 2^e_n [GPS][256] f16
 constexpr int BSTAGE = BN * KS * 2;      // float16 weight operand, 128-byte rows (32 KB)
 constexpr int PHB = BM * KS * 2;         // p_hat stage [128][64] f16, 128-byte swizzle (one per group)
 constexpr int RSB = BM * 8;              // {2^e_m, 2^-e_m} per row
@@ -94,11 +94,17 @@ constexpr int EFB = 2 * 128 * 4;         // per epilogue warp: 2^-e_n and bias o
 constexpr int NBAR = 2 * SP + 2 * SO + 2 + 2 * 2 + 2 * 2 + 1;
 constexpr int OFF_B = 0;
 constexpr int OFF_PH = OFF_B + SO * BSTAGE;
-constexpr int OFF_P = OFF_PH + 2 * PHB;
+constexpr int OFF_PB = OFF_PH + 2 * PHB;  // packed B of each stage [SP][PB]; PREB: the output staging
+constexpr int OFF_P = OFF_PB + SP * PB;
 constexpr int OFF_R = OFF_P + SP * PSTAGE;
 constexpr int OFF_E = OFF_R + 2 * RSB;
 constexpr int OFF_BAR = OFF_E + 8 * EFB;
 constexpr int SMEM = 1024 + OFF_BAR + NBAR * 8 + 16;
+static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
+// PREB: each epilogue warp stages 32 rows x 128 bytes of output (128-byte swizzle, 1024-byte
+// aligned) in the packed-B slots, which that mode does not use, and stores them by TMA.
+constexpr int YSTG = 4096;
+static_assert(8 * YSTG <= SP * PB && OFF_PB % 1024 == 0 && PB % 1024 == 0, "output staging");
 static_assert(SMEM <= 232448, "kernel (b) shared memory above the 227 KB per-CTA limit");
 constexpr uint32_t TMEM_COLS = 512;  // accumulator 0..255, A ring 256 + 32 i
 constexpr uint32_t TMEM_A = 256;
@@ -236,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     gemm16_kernel(const __grid_constant__ CUtensorMap qa_map, const __grid_constant__ CUtensorMap qw_map,
                   const __grid_constant__ CUtensorMap sx_map, const __grid_constant__ CUtensorMap sw_map,
                   const __grid_constant__ CUtensorMap ph_map, const __grid_constant__ CUtensorMap bh_map,
-                  const GemmArgs a) {
+                  const __grid_constant__ CUtensorMap y_map, const GemmArgs a) {
   constexpr int GPS = KS / G;   // groups per K stage (1 or 2)
   extern __shared__ uint8_t smem_raw[];
   pdl_launch_dependents();
@@ -244,6 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* bring = smem + OFF_B;
   uint8_t* phbuf = smem + OFF_PH;
   uint8_t* pring = smem + OFF_P;
+  uint8_t* pbring = smem + OFF_PB;
   float2* rslot = reinterpret_cast<float2*>(smem + OFF_R);
   float* efb = reinterpret_cast<float*>(smem + OFF_E);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
@@ -324,13 +331,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (PREB) {
             mbar_arrive_expect_tx(&pfull[ps], PA + GPS * BM * 2);
             tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
-            tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
+            tma_load_2d(p + PA, &sx_map, &pfull[ps], m0, st * GPS);
           } else {
             mbar_arrive_expect_tx(&pfull[ps], PA + PB + GPS * (BM + BN) * 2);
             tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
-            tma_load_2d(p + PA, &qw_map, &pfull[ps], st * (KS / 2), n0);
-            tma_load_2d(p + PA + PB, &sx_map, &pfull[ps], m0, st * GPS);
-            tma_load_2d(p + PA + PB + PSX, &sw_map, &pfull[ps], n0, st * GPS);
+            tma_load_2d(pbring + ps * PB, &qw_map, &pfull[ps], st * (KS / 2), n0);
+            tma_load_2d(p + PA, &sx_map, &pfull[ps], m0, st * GPS);
+            tma_load_2d(p + PA + PSX, &sw_map, &pfull[ps], n0, st * GPS);
           }
         }
         __syncwarp();
@@ -436,15 +443,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           // every load of the stage first (the operand stores may alias them as far as the
           // compiler knows), then the conversions and stores
           const uint4 wa = *reinterpret_cast<const uint4*>(pk + r * (KS / 2) + 16 * h);
-          const __nv_bfloat16 sxa = reinterpret_cast<const __nv_bfloat16*>(pk + PA + PB)[(GPS == 2 ? h : 0) * BM + r];
+          const __nv_bfloat16 sxa = reinterpret_cast<const __nv_bfloat16*>(pk + PA)[(GPS == 2 ? h : 0) * BM + r];
           uint4 wb[2];
           __half swb[2];
           if (!PREB) {
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
               const int R = Rb + 16 * i;
-              wb[i] = *reinterpret_cast<const uint4*>(pk + PA + R * (KS / 2) + 16 * hh);
-              swb[i] = reinterpret_cast<const __half*>(pk + PA + PB + PSX)[(GPS == 2 ? hh : 0) * BN + R];
+              wb[i] = *reinterpret_cast<const uint4*>(pbring + ps * PB + R * (KS / 2) + 16 * hh);
+              swb[i] = reinterpret_cast<const __half*>(pk + PA + PSX)[(GPS == 2 ? hh : 0) * BN + R];
             }
           }
           const DqScale da = scale_consts(sxa, mul);
@@ -594,76 +601,134 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float fm = rslot[(ti & 1) * BM + r].y;
       warp_arrive(&rempty[ti & 1]);
       const int m = m0 + r;
+      if constexpr (PREB) {
+        // Output through the staging buffer: this warp's 32 rows x 32 columns of a chunk (fp32), or
+        // of two chunks (bf16), 128 bytes per row in the 128-byte swizzle, then one TMA store of
+        // the box (rows >= M and columns >= N are not written).
+        uint8_t* stg = pbring + (ew >> 1) * PB + (ew & 1) * YSTG;
+        uint8_t* srow = stg + lane * 128;
+        const uint32_t sw = lane & 7u;
+        auto cols8p = [&](int cb, const uint32_t* av, float (&y)[8]) {  // cb: column within the warp's 128
+          const float4 f0 = reinterpret_cast<const float4*>(fcb)[cb / 4];
+          const float4 f1 = reinterpret_cast<const float4*>(fcb)[cb / 4 + 1];
+          const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+#pragma unroll
+          for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(av[t]) * fn[t]) * fm;
+          if (a.bias) {
+            const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4];
+            const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4 + 1];
+            y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
+            y[4] += b1.x; y[5] += b1.y; y[6] += b1.z; y[7] += b1.w;
+          }
+        };
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
-        uint32_t acc[32];
-        tmem_ld32(tbase + 32 * c, acc);
-        tmem_ld_wait_dep(acc);
-        if (c == 3) {
-          // the tile's accumulator has been read: the MMA may start the next tile
-          tc_fence_before();
-          warp_arrive(accempty);
-        }
-        const int nb = n0 + 128 * hf + 32 * c;
-        if (m < a.M) {
+        for (int c = 0; c < 4; ++c) {
+          uint32_t acc[32];
+          tmem_ld32(tbase + 32 * c, acc);
+          tmem_ld_wait_dep(acc);
+          if (c == 3) {
+            // the tile's accumulator has been read: the MMA may start the next tile
+            tc_fence_before();
+            warp_arrive(accempty);
+          }
+          if (a.y_f32 || (c & 1) == 0) {  // the buffer is free once the last store has read it
+            if (lane == 0) bulk_wait_read();
+            __syncwarp();
+          }
 #pragma unroll
-          for (int j2 = 0; j2 < 2; ++j2) {  // 16 columns at a time: one 32-byte store per row (bf16)
-            const int n = nb + 16 * j2;
-            if (n >= a.N) continue;
-            // results of columns n + 8 h8 .. + 7: (acc 2^-e_n) 2^-e_m (+ bias)
-            auto cols8 = [&](int h8, float (&y)[8]) {
-              const int cb = 32 * c + 16 * j2 + 8 * h8;  // column within the warp's 128
-              const float4 f0 = reinterpret_cast<const float4*>(fcb)[cb / 4];
-              const float4 f1 = reinterpret_cast<const float4*>(fcb)[cb / 4 + 1];
-              const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
-#pragma unroll
-              for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(acc[16 * j2 + 8 * h8 + t]) * fn[t]) * fm;
-              if (a.bias) {
-                const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4];
-                const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4 + 1];
-                y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
-                y[4] += b1.x; y[5] += b1.y; y[6] += b1.z; y[7] += b1.w;
-              }
-            };
-            const size_t off = static_cast<size_t>(m) * a.N + n;
-            const bool two = n + 16 <= a.N;  // N is a multiple of 8: the second 8 may lie past it
+          for (int j = 0; j < 4; ++j) {
+            float y[8];
+            cols8p(32 * c + 8 * j, acc + 8 * j, y);
             if (a.y_f32) {
-              float* yp = static_cast<float*>(a.Y) + off;
-#pragma unroll
-              for (int h8 = 0; h8 < 2; ++h8) {
-                if (h8 == 1 && !two) break;
-                float y[8];
-                cols8(h8, y);
-                uint32_t u[8];
-#pragma unroll
-                for (int t = 0; t < 8; ++t) u[t] = __float_as_uint(y[t]);
-                if ((off & 7) == 0) {
-                  st_global_v8(yp + 8 * h8, u);
-                } else {
-                  st_global_v4(yp + 8 * h8, u[0], u[1], u[2], u[3]);
-                  st_global_v4(yp + 8 * h8 + 4, u[4], u[5], u[6], u[7]);
-                }
-              }
+              *reinterpret_cast<float4*>(srow + (((2u * j) ^ sw) << 4)) = make_float4(y[0], y[1], y[2], y[3]);
+              *reinterpret_cast<float4*>(srow + (((2u * j + 1u) ^ sw) << 4)) = make_float4(y[4], y[5], y[6], y[7]);
             } else {
-              __nv_bfloat16* yp = static_cast<__nv_bfloat16*>(a.Y) + off;
-              uint32_t u[8];
-              {
-                float y[8];
-                cols8(0, y);
-#pragma unroll
-                for (int t = 0; t < 4; ++t) u[t] = f32x2_to_bf16x2(y[2 * t], y[2 * t + 1]);
-              }
-              if (two) {
-                float y[8];
-                cols8(1, y);
-#pragma unroll
-                for (int t = 0; t < 4; ++t) u[4 + t] = f32x2_to_bf16x2(y[2 * t], y[2 * t + 1]);
-              }
-              if (two && (off & 15) == 0) {
-                st_global_v8(yp, u);
+              *reinterpret_cast<uint4*>(srow + ((static_cast<uint32_t>(4 * (c & 1) + j) ^ sw) << 4)) =
+                  make_uint4(f32x2_to_bf16x2(y[0], y[1]), f32x2_to_bf16x2(y[2], y[3]), f32x2_to_bf16x2(y[4], y[5]),
+                             f32x2_to_bf16x2(y[6], y[7]));
+            }
+          }
+          if (a.y_f32 || (c & 1) == 1) {
+            fence_proxy_async_smem();  // the staged rows, before the async proxy reads them
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&y_map, stg, n0 + 128 * hf + (a.y_f32 ? 32 * c : 64 * (c >> 1)), m0 + 32 * q);
+              bulk_commit();
+            }
+          }
+        }
+      } else {
+  #pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t acc[32];
+          tmem_ld32(tbase + 32 * c, acc);
+          tmem_ld_wait_dep(acc);
+          if (c == 3) {
+            // the tile's accumulator has been read: the MMA may start the next tile
+            tc_fence_before();
+            warp_arrive(accempty);
+          }
+          const int nb = n0 + 128 * hf + 32 * c;
+          if (m < a.M) {
+  #pragma unroll
+            for (int j2 = 0; j2 < 2; ++j2) {  // 16 columns at a time: one 32-byte store per row (bf16)
+              const int n = nb + 16 * j2;
+              if (n >= a.N) continue;
+              // results of columns n + 8 h8 .. + 7: (acc 2^-e_n) 2^-e_m (+ bias)
+              auto cols8 = [&](int h8, float (&y)[8]) {
+                const int cb = 32 * c + 16 * j2 + 8 * h8;  // column within the warp's 128
+                const float4 f0 = reinterpret_cast<const float4*>(fcb)[cb / 4];
+                const float4 f1 = reinterpret_cast<const float4*>(fcb)[cb / 4 + 1];
+                const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+  #pragma unroll
+                for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(acc[16 * j2 + 8 * h8 + t]) * fn[t]) * fm;
+                if (a.bias) {
+                  const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4];
+                  const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4 + 1];
+                  y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
+                  y[4] += b1.x; y[5] += b1.y; y[6] += b1.z; y[7] += b1.w;
+                }
+              };
+              const size_t off = static_cast<size_t>(m) * a.N + n;
+              const bool two = n + 16 <= a.N;  // N is a multiple of 8: the second 8 may lie past it
+              if (a.y_f32) {
+                float* yp = static_cast<float*>(a.Y) + off;
+  #pragma unroll
+                for (int h8 = 0; h8 < 2; ++h8) {
+                  if (h8 == 1 && !two) break;
+                  float y[8];
+                  cols8(h8, y);
+                  uint32_t u[8];
+  #pragma unroll
+                  for (int t = 0; t < 8; ++t) u[t] = __float_as_uint(y[t]);
+                  if ((off & 7) == 0) {
+                    st_global_v8(yp + 8 * h8, u);
+                  } else {
+                    st_global_v4(yp + 8 * h8, u[0], u[1], u[2], u[3]);
+                    st_global_v4(yp + 8 * h8 + 4, u[4], u[5], u[6], u[7]);
+                  }
+                }
               } else {
-                st_global_v4(yp, u[0], u[1], u[2], u[3]);
-                if (two) st_global_v4(yp + 8, u[4], u[5], u[6], u[7]);
+                __nv_bfloat16* yp = static_cast<__nv_bfloat16*>(a.Y) + off;
+                uint32_t u[8];
+                {
+                  float y[8];
+                  cols8(0, y);
+  #pragma unroll
+                  for (int t = 0; t < 4; ++t) u[t] = f32x2_to_bf16x2(y[2 * t], y[2 * t + 1]);
+                }
+                if (two) {
+                  float y[8];
+                  cols8(1, y);
+  #pragma unroll
+                  for (int t = 0; t < 4; ++t) u[4 + t] = f32x2_to_bf16x2(y[2 * t], y[2 * t + 1]);
+                }
+                if (two && (off & 15) == 0) {
+                  st_global_v8(yp, u);
+                } else {
+                  st_global_v4(yp, u[0], u[1], u[2], u[3]);
+                  if (two) st_global_v4(yp + 8, u[4], u[5], u[6], u[7]);
+                }
               }
             }
           }
@@ -671,6 +736,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();  // every lane's reads of the staged columns are done before the next tile's
       if (ti + 2 < my_tiles) ok = rowscale(ti + 2);
+    }
+    if (PREB) {  // every output store is complete before the CTA exits
+      if (lane == 0) bulk_wait_all();
+      __syncwarp();
     }
     tmem_ld_wait();
   }
@@ -734,10 +803,13 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
   // p_hat / B_hat maps are never used and any valid map fills the slots.
   const CUtensorMap& ph = (h.r_pad > 0) ? am.ph64_map : am.qa_map;
   const CUtensorMap& bh = PREB ? am.w16_map : ((h.r_pad > 0) ? h.bhs_map : am.qa_map);
+  // PREB stores the output by TMA (the map of Y); otherwise any valid map fills the slot.
+  const CUtensorMap* ym = PREB ? get_y_map(h, Y, M, y_f32) : &am.qa_map;
+  if (!ym) return cudaErrorInvalidValue;
   cfg.gridDim = dim3(grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = SMEM;
-  return cudaLaunchKernelEx(&cfg, gemm16_kernel<G, PREB>, am.qa_map, h.qw_map, am.sx_map, h.swh_map, ph, bh, a);
+  return cudaLaunchKernelEx(&cfg, gemm16_kernel<G, PREB>, am.qa_map, h.qw_map, am.sx_map, h.swh_map, ph, bh, *ym, a);
 }
 
 }  // namespace

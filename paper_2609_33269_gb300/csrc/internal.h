@@ -111,12 +111,34 @@ struct Handle {
   CUtensorMap qw4_map;               // NVFP4 weight codes [N, K/2], box {128, 128}, 128-byte swizzle
   ActMaps act_cache[4];
   int act_next = 0;
+  // Output maps of the INT4 GEMM's TMA-store epilogue: Y [M, N] (bf16 or float32), box 128 bytes
+  // x 32 rows, 128-byte swizzle; the last few (Y, M, dtype) triples.
+  struct YMap {
+    const void* y = nullptr;
+    int M = -1;
+    bool f32 = false;
+    CUtensorMap map;
+  };
+  YMap y_cache[4];
+  int y_next = 0;
 };
 
 // Workspace of M tokens.  INT4: packed OB4 codes [M, K/2], s_x bf16 [K/G, M_pad], p_hat f16
 // [M, r_pad]; NVFP4: E2M1 codes [M, K/2], scale atoms, p_hat.  ab_off = phat_off (no region).
+// Kernel (a)'s split of K over the CTAs of a cluster (C = 1, 2, 4 or 8) for `tiles` row tiles:
+// as many CTAs as the SMs allow, each with an even number of 64-wide chunks.
+inline int act_split(int K, int tiles, int sms) {
+  const int chunks = K / kChunk;
+  int C = 1;
+  while (C < 8 && chunks % (2 * C) == 0 && tiles * 2 * C <= sms) C *= 2;
+  if (C == 1 && chunks % 2 == 0 && tiles < sms) C = 2;
+  return C;
+}
+
 struct ActLayout {
   size_t codes_off, scales_off, ab_off, phat_off, bytes;
+  size_t part_off;   // r_pad <= kMaxRank: float32 [C, M_pad, r_pad], kernel (a)'s partial projections
+                     // of its C CTAs per row tile (C = act_split), exchanged through L2 (0: none)
   size_t resid_off;  // rotated handles with r > 0: float32 [M, K] remainder before the rotation
   size_t ytmp_off;   // NVFP4 with r_pad > kMaxRank: float32 [M, N] 4-bit part before the branch
   size_t w16_off;    // INT4 with >= kPreExpandMinTiles row tiles: float16 [N_pad, K + r_pad], the
@@ -129,6 +151,8 @@ ActLayout act_layout(const Handle& h, int M, bool lean = false);
 // Tensor-map encoder (driver entry point fetched through the runtime).
 bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint64_t inner, uint64_t outer,
                uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle sw);
+// The output map of Y [M, N] for the INT4 GEMM's TMA-store epilogue (cached per handle).
+const CUtensorMap* get_y_map(Handle& h, const void* Y, int M, bool y_f32);
 bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const uint64_t dims[3],
                const uint64_t strides_bytes[2], const uint32_t box[3]);
 const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M, bool lean = false);

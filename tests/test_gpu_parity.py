@@ -37,6 +37,8 @@ SHAPES = [  # M, K, N, r, G
     (1, 256, 136, 0, 64),       # single token, r = 0
     (200, 1024, 384, 48, 64),
     (130, 640, 264, 64, 32),
+    (600, 512, 200, 16, 64),    # >= 512 tokens: float16 weight copy, TMA-store epilogue; M, N ragged
+    (520, 384, 72, 0, 32),      # the same with r = 0, group 32, a single partial column tile
     (128, 64, 64, 64, 64),      # r = K
 ]
 
@@ -101,7 +103,7 @@ def test_quantizer_bit_exact_on_kernel_remainder(shape):
         c.close()
 
 
-@pytest.mark.parametrize("shape", SHAPES[:5], ids=lambda s: "M%d_K%d_N%d_r%d_g%d" % s)
+@pytest.mark.parametrize("shape", [s for s in SHAPES if s[3] < s[1]], ids=lambda s: "M%d_K%d_N%d_r%d_g%d" % s)
 def test_end_to_end_codes_and_output(shape):
     M, K, N, r, G = shape
     c = Case(M, K, N, r, G, seed=6, layer_id=K + r)
