@@ -123,6 +123,7 @@ ActLayout act_layout(const Handle& h, int M, bool lean) {
       L.bytes += up256(static_cast<size_t>(M) * h.N * 4);
     }
     L.w16_off = 0;
+    L.gsplit_off = 0;
     return L;
   }
   L.scales_off = up256(static_cast<size_t>(M) * (h.K / 2));
@@ -137,9 +138,16 @@ ActLayout act_layout(const Handle& h, int M, bool lean) {
   }
   L.ytmp_off = 0;
   L.w16_off = 0;
+  L.gsplit_off = 0;
   if (!lean && L.M_pad / kBM >= kPreExpandMinTiles) {
     L.w16_off = L.bytes;
     L.bytes += up256(static_cast<size_t>(h.N_pad) * (h.K + h.r_pad) * 2);
+  } else if (M > 0) {
+    const int S = gemm_split(M, h.N, h.K, h.num_sms);
+    if (S > 1) {
+      L.gsplit_off = L.bytes;
+      L.bytes += up256(static_cast<size_t>(S) * M * h.N * 4);
+    }
   }
   return L;
 }

@@ -74,6 +74,8 @@ struct GemmArgs {
   void* Y;
   int y_f32;
   const float* bias;        // optional [N], added to the float32 result before it is stored
+  int splits;               // > 1: split-K over a cluster of `splits` CTAs per tile (below)
+  float* part;              // splits > 1: float32 [splits, M, N] partial results (workspace)
   int* err;
   uint64_t timeout_ns;
 };
@@ -269,18 +271,33 @@ __global__ void __launch_bounds__(kThreads, 1)
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const uint32_t wid = warp_id(), lane = lane_id();
-  const int nks = a.K / KS;
-  const int nst = nks + a.nbs;
+  // Split-K (few tiles, many idle SMs): the `splits` CTAs of a cluster share one tile, CTA `rank`
+  // taking K stages [kb, kb + nks) and, the last one, the branch stages; each writes its float32
+  // partial tile (without the bias) to the workspace, and after one cluster barrier each sums a
+  // 1/splits slice of the tile's columns over the partials in rank order and stores the output.
+  const bool split = !PREB && a.splits > 1;  // (the float16-weight GEMM never splits)
+  const int rank = split ? static_cast<int>(cluster_ctarank()) : 0;
+  const int nks_all = a.K / KS;
+  const int kb = rank * nks_all / a.splits;
+  const int nks = (rank + 1) * nks_all / a.splits - kb;
+  const int nbs = rank == a.splits - 1 ? a.nbs : 0;
+  const int nst = nks + nbs;
   const int ntiles = a.m_tiles * a.n_tiles;
-  const int my_tiles = ntiles > static_cast<int>(blockIdx.x)
+  const int my_tiles = split ? 1
+                       : ntiles > static_cast<int>(blockIdx.x)
                            ? (ntiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
                                  static_cast<int>(gridDim.x)
                            : 0;
   auto tile_mn = [&](int i, int& m0, int& n0) {
-    const int t = static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
+    const int t = split ? static_cast<int>(blockIdx.x) / a.splits
+                        : static_cast<int>(blockIdx.x) + i * static_cast<int>(gridDim.x);
     m0 = (t / a.n_tiles) * BM;
     n0 = (t % a.n_tiles) * BN;
   };
+  // where the epilogue writes: the output, or (split-K) this CTA's partial slice, float32, no bias
+  void* const yout = split ? static_cast<void*>(a.part + static_cast<size_t>(rank) * a.M * a.N) : a.Y;
+  const int yf32 = split ? 1 : a.y_f32;
+  const float* const ybias = split ? nullptr : a.bias;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < SP; ++i) {
@@ -311,7 +328,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const WaitCtl wc{abort_flag, a.err, globaltimer_ns() + a.timeout_ns};
-  pdl_wait();  // every global access of this kernel comes after the previous kernel's
+  // Every global access of this kernel that reads what the previous kernel of the stream wrote
+  // comes after this wait (the producer's first weight stages, which it did not write, go before).
+  if (wid != 0 || PREB) pdl_wait();
 
   if (wid == 0) {
     // ------------------------------------------------------------- TMA producer (activations)
@@ -319,6 +338,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     // codes and s_x; warp 3 brings the float16 weights).
     bool ok = true;
     int s = 0;
+    int pre = 0;  // stages of the first tile whose weight part was requested before the wait
+    if (!PREB) {
+      if (my_tiles > 0) {
+        int m0, n0;
+        tile_mn(0, m0, n0);
+        pre = nks < SP ? nks : SP;
+        if (elect_one())
+          for (int st = 0; st < pre; ++st) {
+            uint8_t* p = pring + st * PSTAGE;
+            mbar_arrive_expect_tx(&pfull[st], PA + PB + GPS * (BM + BN) * 2);
+            tma_load_2d(pbring + st * PB, &qw_map, &pfull[st], (kb + st) * (KS / 2), n0);
+            tma_load_2d(p + PA + PSX, &sw_map, &pfull[st], n0, (kb + st) * GPS);
+          }
+        __syncwarp();
+      }
+      pdl_wait();
+    }
     for (int ti = 0; ti < my_tiles && ok; ++ti) {
       int m0, n0;
       tile_mn(ti, m0, n0);
@@ -330,14 +366,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (elect_one()) {
           if (PREB) {
             mbar_arrive_expect_tx(&pfull[ps], PA + GPS * BM * 2);
-            tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
-            tma_load_2d(p + PA, &sx_map, &pfull[ps], m0, st * GPS);
+            tma_load_2d(p, &qa_map, &pfull[ps], (kb + st) * (KS / 2), m0);
+            tma_load_2d(p + PA, &sx_map, &pfull[ps], m0, (kb + st) * GPS);
+          } else if (s < pre) {  // the weight part is on its way
+            tma_load_2d(p, &qa_map, &pfull[ps], (kb + st) * (KS / 2), m0);
+            tma_load_2d(p + PA, &sx_map, &pfull[ps], m0, (kb + st) * GPS);
           } else {
             mbar_arrive_expect_tx(&pfull[ps], PA + PB + GPS * (BM + BN) * 2);
-            tma_load_2d(p, &qa_map, &pfull[ps], st * (KS / 2), m0);
-            tma_load_2d(pbring + ps * PB, &qw_map, &pfull[ps], st * (KS / 2), n0);
-            tma_load_2d(p + PA, &sx_map, &pfull[ps], m0, st * GPS);
-            tma_load_2d(p + PA + PSX, &sw_map, &pfull[ps], n0, st * GPS);
+            tma_load_2d(p, &qa_map, &pfull[ps], (kb + st) * (KS / 2), m0);
+            tma_load_2d(pbring + ps * PB, &qw_map, &pfull[ps], (kb + st) * (KS / 2), n0);
+            tma_load_2d(p + PA, &sx_map, &pfull[ps], m0, (kb + st) * GPS);
+            tma_load_2d(p + PA + PSX, &sw_map, &pfull[ps], n0, (kb + st) * GPS);
           }
         }
         __syncwarp();
@@ -516,10 +555,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     int never = 0;
     const WaitCtl dc{&never, a.err, globaltimer_ns() + a.timeout_ns};
     if (ph > 0) mbar_wait_inline(&phfull[gx], (ph - 1) & 1, dc);
-    if (!PREB && e == 0 && a.nbs > 0) {
+    if (!PREB && e == 0 && nbs > 0) {
       // this group's last branch stage: its B_hat load completed the stage's barrier
       int lb = -1;
-      for (int j = so - 1; j >= 0 && j >= so - a.nbs; --j)
+      for (int j = so - 1; j >= 0 && j >= so - nbs; --j)
         if ((j & 1) == gx) {
           lb = j;
           break;
@@ -548,6 +587,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       const __nv_bfloat16* sp = a.sx + m;
       // (the workspace was written by the previous kernel of the stream, complete before pdl_wait)
       auto sx_at = [&](int g) { return __uint_as_float(ld_nc_u16(sp + static_cast<size_t>(g) * a.M_pad) << 16); };
+      // the first p_hat pieces are loaded ahead of the scales, so that both are in flight together
+      const bool has_ph = a.r_pad > 0 && m < a.M;
+      const uint4* pr = has_ph ? reinterpret_cast<const uint4*>(a.phat + static_cast<size_t>(m) * a.r_pad) + hs * (a.r_pad / 16)
+                               : nullptr;
+      const int nph = has_ph ? a.r_pad / 16 : 0;  // 16-byte pieces of this thread's half row
+      uint4 ph4[2];
+#pragma unroll
+      for (int j = 0; j < 2; ++j) ph4[j] = j < nph ? ld_nc_v4(pr + j) : make_uint4(0u, 0u, 0u, 0u);
       float s0 = 0.0f, s1 = 0.0f, s2 = 0.0f, s3 = 0.0f;
       int g = hs;
 #pragma unroll 4
@@ -559,16 +606,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       for (; g < ng; g += 2) s0 = fmaxf(s0, sx_at(g));
       float am = 7.0f * fmaxf(fmaxf(s0, s1), fmaxf(s2, s3));  // exact: 8 + 3 significant bits
-      if (a.r_pad > 0 && m < a.M) {
-        const uint4* pr = reinterpret_cast<const uint4*>(a.phat + static_cast<size_t>(m) * a.r_pad) + hs * (a.r_pad / 16);
-#pragma unroll 4
-        for (int j = 0; j < a.r_pad / 16; ++j) {
-          const uint4 u4 = ld_nc_v4(pr + j);
-          const uint32_t w4[4] = {u4.x, u4.y, u4.z, u4.w};
+      auto ph_max = [&](const uint4& u4) {
+        const uint32_t w4[4] = {u4.x, u4.y, u4.z, u4.w};
 #pragma unroll
-          for (int t = 0; t < 4; ++t) am = fmaxf(am, fmaxf(fabsf(f16_lo(w4[t])), fabsf(f16_hi(w4[t]))));
-        }
-      }
+        for (int t = 0; t < 4; ++t) am = fmaxf(am, fmaxf(fabsf(f16_lo(w4[t])), fabsf(f16_hi(w4[t]))));
+      };
+#pragma unroll
+      for (int j = 0; j < 2; ++j) ph_max(ph4[j]);  // (zero pieces past nph leave am as it is)
+#pragma unroll 4
+      for (int j = 2; j < nph; ++j) ph_max(ld_nc_v4(pr + j));
       am = fmaxf(am, __shfl_xor_sync(0xFFFFFFFFu, am, 1));
       int e = 0;
       if (am > 0.0f) {
@@ -590,7 +636,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int n = n0 + 128 * hf + 4 * static_cast<int>(lane);  // < N_pad
         reinterpret_cast<float4*>(fcb)[lane] = *reinterpret_cast<const float4*>(a.fcol + n);
         float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (a.bias && n < a.N) b = *reinterpret_cast<const float4*>(a.bias + n);
+        if (ybias && n < a.N) b = *reinterpret_cast<const float4*>(ybias + n);
         reinterpret_cast<float4*>(fcb + 128)[lane] = b;
         __syncwarp();
       }
@@ -614,7 +660,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
 #pragma unroll
           for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(av[t]) * fn[t]) * fm;
-          if (a.bias) {
+          if (ybias) {
             const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4];
             const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4 + 1];
             y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
@@ -631,7 +677,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             warp_arrive(accempty);
           }
-          if (a.y_f32 || (c & 1) == 0) {  // the buffer is free once the last store has read it
+          if (yf32 || (c & 1) == 0) {  // the buffer is free once the last store has read it
             if (lane == 0) bulk_wait_read();
             __syncwarp();
           }
@@ -639,7 +685,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = 0; j < 4; ++j) {
             float y[8];
             cols8p(32 * c + 8 * j, acc + 8 * j, y);
-            if (a.y_f32) {
+            if (yf32) {
               *reinterpret_cast<float4*>(srow + (((2u * j) ^ sw) << 4)) = make_float4(y[0], y[1], y[2], y[3]);
               *reinterpret_cast<float4*>(srow + (((2u * j + 1u) ^ sw) << 4)) = make_float4(y[4], y[5], y[6], y[7]);
             } else {
@@ -648,11 +694,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                              f32x2_to_bf16x2(y[6], y[7]));
             }
           }
-          if (a.y_f32 || (c & 1) == 1) {
+          if (yf32 || (c & 1) == 1) {
             fence_proxy_async_smem();  // the staged rows, before the async proxy reads them
             __syncwarp();
             if (lane == 0) {
-              tma_store_2d(&y_map, stg, n0 + 128 * hf + (a.y_f32 ? 32 * c : 64 * (c >> 1)), m0 + 32 * q);
+              tma_store_2d(&y_map, stg, n0 + 128 * hf + (yf32 ? 32 * c : 64 * (c >> 1)), m0 + 32 * q);
               bulk_commit();
             }
           }
@@ -682,7 +728,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float fn[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
   #pragma unroll
                 for (int t = 0; t < 8; ++t) y[t] = (__uint_as_float(acc[16 * j2 + 8 * h8 + t]) * fn[t]) * fm;
-                if (a.bias) {
+                if (ybias) {
                   const float4 b0 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4];
                   const float4 b1 = reinterpret_cast<const float4*>(fcb + 128)[cb / 4 + 1];
                   y[0] += b0.x; y[1] += b0.y; y[2] += b0.z; y[3] += b0.w;
@@ -691,8 +737,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               };
               const size_t off = static_cast<size_t>(m) * a.N + n;
               const bool two = n + 16 <= a.N;  // N is a multiple of 8: the second 8 may lie past it
-              if (a.y_f32) {
-                float* yp = static_cast<float*>(a.Y) + off;
+              if (yf32) {
+                float* yp = static_cast<float*>(yout) + off;
   #pragma unroll
                 for (int h8 = 0; h8 < 2; ++h8) {
                   if (h8 == 1 && !two) break;
@@ -709,7 +755,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   }
                 }
               } else {
-                __nv_bfloat16* yp = static_cast<__nv_bfloat16*>(a.Y) + off;
+                __nv_bfloat16* yp = static_cast<__nv_bfloat16*>(yout) + off;
                 uint32_t u[8];
                 {
                   float y[8];
@@ -744,6 +790,51 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_ld_wait();
   }
 
+  if (!PREB && split) {
+    // Every thread of the cluster arrives here once its role is done; the barrier's release /
+    // acquire orders the partial tiles written above before the reads below.
+    cluster_sync();
+    int m0, n0;
+    tile_mn(0, m0, n0);
+    const int W = BN / a.splits;  // this CTA's columns of the tile
+    const int c0 = n0 + rank * W;
+    const int rows = min(BM, a.M - m0);
+    const int w4 = W / 4;
+    const size_t slice = static_cast<size_t>(a.M) * a.N;
+    for (int i = static_cast<int>(threadIdx.x); i < rows * w4; i += kThreads) {
+      const int m = m0 + i / w4, n = c0 + 4 * (i % w4);
+      if (n >= a.N) continue;  // N is a multiple of 8, so n < N covers n .. n + 3
+      const float* pp = a.part + static_cast<size_t>(m) * a.N + n;
+      float4 v[8];  // every split's partial in flight at once (splits <= 8), summed in rank order
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        v[q] = q < a.splits ? *reinterpret_cast<const float4*>(pp + q * slice) : make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 y = v[0];
+#pragma unroll
+      for (int q = 1; q < 8; ++q) {
+        if (q >= a.splits) break;
+        y.x += v[q].x;
+        y.y += v[q].y;
+        y.z += v[q].z;
+        y.w += v[q].w;
+      }
+      if (a.bias) {
+        const float4 b = *reinterpret_cast<const float4*>(a.bias + n);
+        y.x += b.x;
+        y.y += b.y;
+        y.z += b.z;
+        y.w += b.w;
+      }
+      const size_t off = static_cast<size_t>(m) * a.N + n;
+      if (a.y_f32) {
+        *reinterpret_cast<float4*>(static_cast<float*>(a.Y) + off) = y;
+      } else {
+        *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(a.Y) + off) =
+            make_uint2(f32x2_to_bf16x2(y.x, y.y), f32x2_to_bf16x2(y.z, y.w));
+      }
+    }
+  }
+
   __syncthreads();
   if (wid == 1) {
     tc_fence_after();
@@ -770,6 +861,8 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
   a.Y = Y;
   a.y_f32 = y_f32 ? 1 : 0;
   a.bias = h.bias;
+  a.splits = L.gsplit_off ? gemm_split(M, h.N, h.K, h.num_sms) : 1;
+  a.part = L.gsplit_off ? reinterpret_cast<float*>(const_cast<uint8_t*>(base) + L.gsplit_off) : nullptr;
   a.err = h.err;
   a.timeout_ns = deadline_budget_ns(h);
   static bool attr_done = false;
@@ -778,9 +871,13 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;  // split-K: the splits of a tile form a cluster
+  attr[1].val.clusterDim.x = a.splits;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cudaLaunchConfig_t cfg = {};
   cfg.stream = s;
   cfg.attrs = attr;
@@ -798,7 +895,8 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
     if (e != cudaSuccess) return e;
   }
   const int ntiles = a.m_tiles * a.n_tiles;
-  const int grid = ntiles < h.num_sms ? ntiles : h.num_sms;
+  const int grid = a.splits > 1 ? ntiles * a.splits : (ntiles < h.num_sms ? ntiles : h.num_sms);
+  cfg.numAttrs = a.splits > 1 ? 2 : 1;
   // With PREB every weight stage comes through the expanded-weight map; without a branch the
   // p_hat / B_hat maps are never used and any valid map fills the slots.
   const CUtensorMap& ph = (h.r_pad > 0) ? am.ph64_map : am.qa_map;

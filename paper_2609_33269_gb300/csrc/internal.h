@@ -135,8 +135,26 @@ inline int act_split(int K, int tiles, int sms) {
   return C;
 }
 
+// The INT4 GEMM's split of K over a cluster of CTAs per output tile (1, 2, 4 or 8) for layers
+// whose 128 x kGemm16BN tiles would leave most SMs idle: CTAs on at most half the SMs (the
+// clusters are then placed at once, beside the activation kernel's), each with at least two
+// 64-wide K stages, and float32 partials of at most 8 MiB.
+inline int gemm_split(int M, int N, int K, int sms) {
+  // (layers of kPreExpandMinTiles row tiles or more take the float16-weight GEMM, unsplit, so that
+  // the workspace-free call, which converts the weights tile by tile, gives the same sums)
+  if ((M + kBM - 1) / kBM >= kPreExpandMinTiles) return 1;
+  const int tiles = ((M + kBM - 1) / kBM) * ((N + kGemm16BN - 1) / kGemm16BN);
+  const int nks = K / kChunk;
+  int S = 1;
+  while (S < 8 && tiles * 4 * S <= sms && nks >= 4 * S &&
+         static_cast<size_t>(2 * S) * M * N * 4 <= (size_t{8} << 20))
+    S *= 2;
+  return S;
+}
+
 struct ActLayout {
   size_t codes_off, scales_off, ab_off, phat_off, bytes;
+  size_t gsplit_off;  // INT4 with a split-K GEMM: float32 [S, M, N] partial outputs (0: none)
   size_t part_off;   // r_pad <= kMaxRank: float32 [C, M_pad, r_pad], kernel (a)'s partial projections
                      // of its C CTAs per row tile (C = act_split), exchanged through L2 (0: none)
   size_t resid_off;  // rotated handles with r > 0: float32 [M, K] remainder before the rotation
