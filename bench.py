@@ -6,7 +6,10 @@ batch of the DiT attention-projection workload: X bf16 [M=4096, K=3072], W [3072
 r = 32, group 64, seeded synthetic data (1% outlier channels x10..30).
 
 Output: one JSON line.  `value` is the effective TOPS (2*M*N*K per step over the device time of
-the timed steps, max over ranks, summed over ranks' work); `e2e` repeats the measurement through
+the timed steps of qwam_asp_linear, max over ranks, summed over ranks' work; for INT4 at 512 or
+more tokens a step is three launches: kernel (a), the float16 weight expansion and the GEMM); the
+per-kernel split comes from a second pass with the two calls timed apart; `e2e`
+repeats the measurement through
 the C ABI with the activations copied from pinned host memory and the output copied back inside
 the timed region; `roofline` describes the dominant kernel; `cpu_baseline` times the CPU oracle
 on a bounded sample of rows.  `--impl reference` times the CPU oracle alone (the reference arm).
@@ -17,7 +20,7 @@ the layer shards by rows with no collective); weak scaling.
 The NVFP4 variant (App. B.1: E2M1 with an E4M3 scale per 16 K, block scales applied by the
 tensor cores) is timed on the same workload and reported under `variants`; `--format nvfp4` makes
 it the headline.  So is the layer with smoothing and the block Hadamard rotation in front (Sec. 3
-Eq. (pair)); `--rotate` makes that the headline (three launches per step with r > 0).  The
+Eq. (pair)); `--rotate` makes that the headline (one more launch per step with r > 0).  The
 denoising-step layer sweep (30 DiT blocks, ASP on a third of them) is reported per format under
 `variants.sweep_int4` / `variants.sweep_nvfp4`.
 """
@@ -541,9 +544,11 @@ def run_ours(args):
     flops = 2.0 * M * N * K
 
     def timed(fmt, nsteps, warmup, clocks=None, smooth=None):
-        """Per-kernel CUDA-event times of `nsteps` steps over rotating sets (weights packed per
-        set, activations, workspaces, outputs), after `warmup` untimed steps.  `smooth`: pack
-        rotated layers (Eq. (pair)) with these smoothing factors."""
+        """The layer through qwam_asp_linear (the public call) for `nsteps` timed steps over
+        rotating sets (weights packed per set, activations, workspaces, outputs), after `warmup`
+        untimed steps; then, outside the timed region, the split of a step into its two calls
+        (qwam_asp_quantize_act, qwam_asp_gemm) from CUDA events around each, over up to 200
+        steps.  `smooth`: pack rotated layers (Eq. (pair)) with these smoothing factors."""
         sets = []
         for i in range(ROTATE_SETS):
             if smooth is None:
@@ -553,16 +558,18 @@ def run_ours(args):
             X = X0 if i == 0 else X0.clone()
             sets.append((lin, X, lin.workspace(M), torch.empty((M, N), dtype=torch.bfloat16, device=dev)))
         mb = ROTATE_SETS * (2 * M * K + 2 * M * N + lin_ws_bytes(sets[0][0], M) + N * K // 2) / 1e6
+
+        def check(where):
+            for lin_, *_ in sets:
+                st = asp.qwam_asp_get_error(lin_.h)
+                if st != asp.QWAM_OK:
+                    raise RuntimeError(f"device error {where}: {asp.status_string(st)}")
+
         for i in range(warmup):
             lin, X, ws, Y = sets[i % ROTATE_SETS]
-            asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
-            asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
+            asp.qwam_asp_linear(X, M, lin.h, Y, asp.QWAM_Y_BF16, ws, stream)
         torch.cuda.synchronize()
-        for lin, *_ in sets:
-            st = asp.qwam_asp_get_error(lin.h)
-            if st != asp.QWAM_OK:
-                raise RuntimeError(f"device error after warm-up: {asp.status_string(st)}")
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * nsteps)]
+        check("after warm-up")
         if clocks is not None:
             clocks.start()
             time.sleep(0.3)
@@ -575,11 +582,7 @@ def run_ours(args):
         start.record(stream)
         for i in range(nsteps):
             lin, X, ws, Y = sets[i % ROTATE_SETS]
-            ev[3 * i].record(stream)
-            asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
-            ev[3 * i + 1].record(stream)
-            asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
-            ev[3 * i + 2].record(stream)
+            asp.qwam_asp_linear(X, M, lin.h, Y, asp.QWAM_Y_BF16, ws, stream)
         end.record(stream)
         torch.cuda.synchronize()
         if clocks is not None:
@@ -588,13 +591,29 @@ def run_ours(args):
         if clocks is not None:
             clocks.stop()
         total_ms = start.elapsed_time(end)
-        t_a = sum(ev[3 * i].elapsed_time(ev[3 * i + 1]) for i in range(nsteps)) / nsteps
-        t_b = sum(ev[3 * i + 1].elapsed_time(ev[3 * i + 2]) for i in range(nsteps)) / nsteps
-        for lin, *_ in sets:
-            st = asp.qwam_asp_get_error(lin.h)
-            if st != asp.QWAM_OK:
-                raise RuntimeError(f"device error in the timed region: {asp.status_string(st)}")
+        check("in the timed region")
         total_ms = max_over_ranks(total_ms, world, dev)
+        # the split of a step into its two calls (the GEMM call includes the float16 weight
+        # expansion); CUDA events between the calls keep the two from overlapping, so this pass
+        # is slightly slower than the timed region
+        nsplit = min(nsteps, 200)
+        for i in range(3):
+            lin, X, ws, Y = sets[i % ROTATE_SETS]
+            asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
+            asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * nsplit)]
+        torch.cuda.synchronize()
+        for i in range(nsplit):
+            lin, X, ws, Y = sets[i % ROTATE_SETS]
+            ev[3 * i].record(stream)
+            asp.qwam_asp_quantize_act(X, M, lin.h, ws, stream)
+            ev[3 * i + 1].record(stream)
+            asp.qwam_asp_gemm(ws, M, lin.h, Y, asp.QWAM_Y_BF16, stream)
+            ev[3 * i + 2].record(stream)
+        torch.cuda.synchronize()
+        t_a = sum(ev[3 * i].elapsed_time(ev[3 * i + 1]) for i in range(nsplit)) / nsplit
+        t_b = sum(ev[3 * i + 1].elapsed_time(ev[3 * i + 2]) for i in range(nsplit)) / nsplit
+        check("in the split pass")
         return dict(sets=sets, total_ms=total_ms, t_a=t_a, t_b=t_b, mb=mb,
                     value=aggregate_value(flops, nsteps, world, total_ms))
 
@@ -734,7 +753,7 @@ def run_ours(args):
             "act_path_ms": rr["t_a"], "gemm_ms": rr["t_b"],
             "act_path_gbs_of_fused_bytes": a_fused / (rr["t_a"] * 1e-3) / 1e9,
             "act_path_gbs_of_moved_bytes": a_split / (rr["t_a"] * 1e-3) / 1e9, "peak_gbs": hbm_peak,
-            "launches_per_step": 3}
+            "launches_per_step": 4}
         for s_ in rr["sets"]:
             s_[0].close()
 
@@ -751,7 +770,10 @@ def run_ours(args):
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 2 * M * K, "d2h_bytes_per_step": 2 * M * N,
                 "steps": e2e_steps,
                 "pipeline": "copies on their own streams, overlapping the layer of the neighbouring steps"},
-        "gpu_launches": (3 if args.rotate and r > 0 else 2) * nsteps,
+        # per qwam_asp_linear call: kernel (a) and the GEMM, the rotation kernel of a rotated layer
+        # with r > 0, and the float16 weight expansion of an INT4 layer of 512 or more tokens
+        "gpu_launches": (2 + (1 if args.rotate and r > 0 else 0)
+                         + (1 if fmt == asp.QWAM_FMT_INT4 and M >= 512 else 0)) * nsteps,
         "roofline": roof,
         "layer_roofline_frac": layer_frac,
         "kernels": kern,

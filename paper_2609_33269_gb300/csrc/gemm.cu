@@ -211,31 +211,55 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
 }
 
 // The weights of one call in float16, [N_pad, K + r_pad] row-major: W16[n, k] = s_w[g, n] 2^e_n c[n, k]
-// for k < K (g = k / G; exact, as in the GEMM's own conversion) and B_hat[n, k - K] 2^e_n after.  One
-// thread per 8 consecutive k of a row.
+// for k < K (g = k / G; exact, as in the GEMM's own conversion) and B_hat[n, k - K] 2^e_n after.  A
+// piece is 8 consecutive k of a row; each thread takes 8 pieces a grid stride apart per round,
+// with all their loads issued before the first conversion (bytes in flight without a large grid).
 template <int G>
 __global__ void __launch_bounds__(256) dequant_weights_kernel(const uint32_t* __restrict__ qw,
-                                                              const __half* __restrict__ swh,
-                                                              const __half* __restrict__ bhs, int K, int r_pad,
-                                                              int N_pad, __half* __restrict__ w16) {
+                                                                 const __half* __restrict__ swh,
+                                                                 const __half* __restrict__ bhs, int K, int r_pad,
+                                                                 int N_pad, __half* __restrict__ w16) {
   pdl_launch_dependents();
   pdl_wait();  // the workspace may still be read by the stream's previous GEMM until then
-  const int wpr = (K + r_pad) / 8;  // 8-wide pieces per row
-  const long long total = static_cast<long long>(N_pad) * wpr;
-  for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
-       i += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const int n = static_cast<int>(i / wpr), j = static_cast<int>(i % wpr);
-    uint4 o;
-    if (8 * j < K) {
-      const uint32_t w = qw[static_cast<size_t>(n) * (K / 8) + j];
-      const DqScale d = dq_scale(__half2float(swh[static_cast<size_t>(8 * j / G) * N_pad + n]));
-      uint32_t v[4];
-      dequant_word(w, d, v);
-      o = make_uint4(v[0], v[1], v[2], v[3]);
-    } else {
-      o = *reinterpret_cast<const uint4*>(bhs + static_cast<size_t>(n) * r_pad + (8 * j - K));
+  constexpr int P = 8;
+  const int kp = K / 8;  // pieces of the K part per row
+  const int ld = K + r_pad;
+  // (N_pad (K + r_pad) / 8 < 2^31 for every layer the pack accepts: 32-bit piece indices)
+  const int stride = static_cast<int>(gridDim.x * blockDim.x);
+  const int first = static_cast<int>(blockIdx.x * blockDim.x + threadIdx.x);
+  const int total = N_pad * kp;
+  for (int i0 = first; i0 < total; i0 += P * stride) {
+    uint32_t w[P];
+    unsigned short sc[P];
+#pragma unroll
+    for (int u = 0; u < P; ++u) {
+      const int i = i0 + u * stride;
+      w[u] = 0u;
+      sc[u] = 0;
+      if (i < total) {
+        const int n = i / kp, j = i - n * kp;
+        w[u] = qw[i];  // row n, word j: qw is [N_pad, K/8] words
+        sc[u] = __half_as_ushort(swh[static_cast<size_t>(8 * j / G) * N_pad + n]);
+      }
     }
-    *reinterpret_cast<uint4*>(w16 + static_cast<size_t>(n) * (K + r_pad) + 8 * j) = o;
+#pragma unroll
+    for (int u = 0; u < P; ++u) {
+      const int i = i0 + u * stride;
+      if (i < total) {
+        const int n = i / kp, j = i - n * kp;
+        uint32_t v[4];
+        dequant_word(w[u], dq_scale(__half2float(__ushort_as_half(sc[u]))), v);
+        *reinterpret_cast<uint4*>(w16 + static_cast<size_t>(n) * ld + 8 * j) = make_uint4(v[0], v[1], v[2], v[3]);
+      }
+    }
+  }
+  // the branch columns: B_hat 2^e_n copied after the K part of each row
+  const int bp = r_pad / 8;
+  const int total_b = N_pad * bp;
+  for (int i = first; i < total_b; i += stride) {
+    const int n = i / bp, j = i - n * bp;
+    *reinterpret_cast<uint4*>(w16 + static_cast<size_t>(n) * ld + K + 8 * j) =
+        *reinterpret_cast<const uint4*>(bhs + static_cast<size_t>(n) * r_pad + 8 * j);
   }
 }
 
@@ -885,7 +909,7 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
   if (PREB) {
     __half* w16 = reinterpret_cast<__half*>(const_cast<uint8_t*>(base) + L.w16_off);
     const long long pieces = static_cast<long long>(h.N_pad) * ((h.K + h.r_pad) / 8);
-    const long long blocks = (pieces + 255) / 256;
+    const long long blocks = (pieces + 8 * 256 - 1) / (8 * 256);  // eight pieces a thread
     cfg.gridDim = dim3(static_cast<unsigned>(blocks < 8 * h.num_sms ? blocks : 8 * h.num_sms), 1, 1);
     cfg.blockDim = dim3(256, 1, 1);
     cfg.dynamicSmemBytes = 0;
