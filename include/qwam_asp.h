@@ -80,7 +80,9 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
  * more tokens it includes a float16 copy of the layer's weights, N_pad (K + r_pad) 2 bytes (N_pad =
  * N rounded up to 256), which qwam_asp_gemm fills once per call and reads from L2 for every row
  * tile.  For 0 < r_pad <= 64 it also includes kernel (a)'s scratch for the partial projections of
- * the C CTAs that share a row tile's K (float32, C M_pad r_pad 4 bytes, C <= 8). */
+ * the C CTAs that share a row tile's K (float32, C M_pad r_pad 4 bytes, C <= 8).  Layers of fewer
+ * tokens whose 128 x 256 output tiles leave most SMs idle add the split-K GEMM's float32 partial
+ * outputs (S M N 4 bytes, S <= 8, at most 8 MiB). */
 qwam_status qwam_asp_act_workspace_bytes(qwam_asp_handle h, int M, size_t* bytes);
 
 /* Layout of the activation workspace for M tokens (byte offsets from its start):
