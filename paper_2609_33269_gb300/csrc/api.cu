@@ -67,20 +67,38 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint6
 }
 
 bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const uint64_t dims[3],
-               const uint64_t strides_bytes[2], const uint32_t box[3]) {
+               const uint64_t strides_bytes[2], const uint32_t box[3], CUtensorMapSwizzle sw) {
   if (!ensure_encoder()) return false;
   cuuint64_t d[3] = {dims[0], dims[1], dims[2]};
   cuuint64_t st[2] = {strides_bytes[0], strides_bytes[1]};
   cuuint32_t b[3] = {box[0], box[1], box[2]};
   cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = g_encode(map, dt, 3, const_cast<void*>(base), d, st, b, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = g_encode(map, dt, 3, const_cast<void*>(base), d, st, b, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+const CUtensorMap* get_part_map(Handle& h, const void* part, int M, int S) {
+  for (auto& c : h.y_cache)
+    if (c.y == part && c.M == M && c.S == S) return &c.map;
+  Handle::YMap& c = h.y_cache[h.y_next];
+  c.y = nullptr;
+  const uint64_t dims[3] = {static_cast<uint64_t>(h.N), static_cast<uint64_t>(M), static_cast<uint64_t>(S)};
+  const uint64_t strides[2] = {static_cast<uint64_t>(h.N) * 4, static_cast<uint64_t>(M) * h.N * 4};
+  const uint32_t box[3] = {32, 32, 1};
+  if (!encode_3d(&c.map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, part, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+    return nullptr;
+  c.y = part;
+  c.M = M;
+  c.f32 = true;
+  c.S = S;
+  h.y_next = (h.y_next + 1) % 4;
+  return &c.map;
 }
 
 const CUtensorMap* get_y_map(Handle& h, const void* Y, int M, bool y_f32) {
   for (auto& c : h.y_cache)
-    if (c.y == Y && c.M == M && c.f32 == y_f32) return &c.map;
+    if (c.y == Y && c.M == M && c.f32 == y_f32 && c.S == 0) return &c.map;
   Handle::YMap& c = h.y_cache[h.y_next];
   c.y = nullptr;
   const uint32_t es = y_f32 ? 4u : 2u;
@@ -90,6 +108,7 @@ const CUtensorMap* get_y_map(Handle& h, const void* Y, int M, bool y_f32) {
   c.y = Y;
   c.M = M;
   c.f32 = y_f32;
+  c.S = 0;
   h.y_next = (h.y_next + 1) % 4;
   return &c.map;
 }

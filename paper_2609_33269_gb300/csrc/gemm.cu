@@ -727,6 +727,54 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
+      } else if (split && m0 + 32 * q >= a.M) {
+        // Split-K, a lane quadrant with no row of the layer: nothing to write
+        tc_fence_before();
+        warp_arrive(accempty);
+      } else if (split && a.M - m0 > 32) {
+        // Split-K: this warp's scaled partial (no bias), 32 rows x 32 columns a chunk, through a
+        // staging buffer in the operand ring (idle once the item's MMAs have completed) and a TMA
+        // store into the CTA's slice of the workspace (rows >= M and columns >= N not written).
+        // (With one quadrant of rows the direct stores below finish sooner: the store's
+        // completion is waited for before the cluster barrier.)
+        uint8_t* stg = bring + ew * YSTG;
+        uint8_t* srow = stg + lane * 128;
+        const uint32_t sw = lane & 7u;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t acc[32];
+          tmem_ld32(tbase + 32 * c, acc);
+          tmem_ld_wait_dep(acc);
+          if (c == 3) {
+            tc_fence_before();
+            warp_arrive(accempty);
+          }
+          if (lane == 0) bulk_wait_read();  // the buffer's last store has read it
+          __syncwarp();
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int cb = 32 * c + 8 * j;  // column within the warp's 128
+            const float4 f0 = reinterpret_cast<const float4*>(fcb)[cb / 4];
+            const float4 f1 = reinterpret_cast<const float4*>(fcb)[cb / 4 + 1];
+            *reinterpret_cast<float4*>(srow + (((2u * j) ^ sw) << 4)) =
+                make_float4((__uint_as_float(acc[8 * j]) * f0.x) * fm, (__uint_as_float(acc[8 * j + 1]) * f0.y) * fm,
+                            (__uint_as_float(acc[8 * j + 2]) * f0.z) * fm, (__uint_as_float(acc[8 * j + 3]) * f0.w) * fm);
+            *reinterpret_cast<float4*>(srow + (((2u * j + 1u) ^ sw) << 4)) =
+                make_float4((__uint_as_float(acc[8 * j + 4]) * f1.x) * fm, (__uint_as_float(acc[8 * j + 5]) * f1.y) * fm,
+                            (__uint_as_float(acc[8 * j + 6]) * f1.z) * fm, (__uint_as_float(acc[8 * j + 7]) * f1.w) * fm);
+          }
+          fence_proxy_async_smem();  // the staged rows, before the async proxy reads them
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_3d(&y_map, stg, n0 + 128 * hf + 32 * c, m0 + 32 * q, rank);
+            bulk_commit();
+          }
+        }
+        if (lane == 0) {  // the partial is written before this CTA reaches the cluster barrier
+          bulk_wait_all();
+          fence_proxy_async_all();
+        }
+        __syncwarp();
       } else {
   #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
@@ -925,8 +973,10 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
   // p_hat / B_hat maps are never used and any valid map fills the slots.
   const CUtensorMap& ph = (h.r_pad > 0) ? am.ph64_map : am.qa_map;
   const CUtensorMap& bh = PREB ? am.w16_map : ((h.r_pad > 0) ? h.bhs_map : am.qa_map);
-  // PREB stores the output by TMA (the map of Y); otherwise any valid map fills the slot.
-  const CUtensorMap* ym = PREB ? get_y_map(h, Y, M, y_f32) : &am.qa_map;
+  // PREB stores the output by TMA (the map of Y), the split-K GEMM its partials (their map);
+  // otherwise any valid map fills the slot.
+  const CUtensorMap* ym = PREB ? get_y_map(h, Y, M, y_f32)
+                               : (a.splits > 1 ? get_part_map(h, a.part, M, a.splits) : &am.qa_map);
   if (!ym) return cudaErrorInvalidValue;
   cfg.gridDim = dim3(grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);

@@ -117,6 +117,7 @@ struct Handle {
     const void* y = nullptr;
     int M = -1;
     bool f32 = false;
+    int S = 0;  // > 0: the split-K GEMM's partial outputs [S, M, N] (float32, box 32 x 32 x 1)
     CUtensorMap map;
   };
   YMap y_cache[4];
@@ -171,8 +172,11 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint6
                uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle sw);
 // The output map of Y [M, N] for the INT4 GEMM's TMA-store epilogue (cached per handle).
 const CUtensorMap* get_y_map(Handle& h, const void* Y, int M, bool y_f32);
+// The map of the split-K GEMM's float32 partial outputs [S, M, N], box 32 x 32 x 1, 128-byte swizzle.
+const CUtensorMap* get_part_map(Handle& h, const void* part, int M, int S);
 bool encode_3d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, const uint64_t dims[3],
-               const uint64_t strides_bytes[2], const uint32_t box[3]);
+               const uint64_t strides_bytes[2], const uint32_t box[3],
+               CUtensorMapSwizzle sw = CU_TENSOR_MAP_SWIZZLE_NONE);
 const ActMaps* get_act_maps(Handle& h, const void* x, const void* ws, int M, bool lean = false);
 
 uint64_t deadline_budget_ns(const Handle& h);

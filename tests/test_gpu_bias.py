@@ -33,7 +33,8 @@ def run(layer, X, fp32=True):
 
 @pytest.mark.parametrize("fmt,rotate", [(asp.QWAM_FMT_INT4, False), (asp.QWAM_FMT_NVFP4, False),
                                         (asp.QWAM_FMT_INT4, True)], ids=["int4", "nvfp4", "int4_rotated"])
-@pytest.mark.parametrize("shape", [(200, 512, 264, 16), (33, 1024, 136, 0)], ids=lambda s: "M%d_K%d_N%d_r%d" % s)
+@pytest.mark.parametrize("shape", [(200, 512, 264, 16), (33, 1024, 136, 0), (600, 512, 264, 16)],
+                         ids=lambda s: "M%d_K%d_N%d_r%d" % s)
 def test_bias_is_one_float32_addition(fmt, rotate, shape):
     M, K, N, r = shape
     Xb = wl.activations(M, K, seed=13, layer_id=K, dist="outlier")
