@@ -6,9 +6,10 @@ batch of the DiT attention-projection workload: X bf16 [M=4096, K=3072], W [3072
 r = 32, group 64, seeded synthetic data (1% outlier channels x10..30).
 
 Output: one JSON line.  `value` is the effective TOPS (2*M*N*K per step over the device time of
-the timed steps of qwam_asp_linear, max over ranks, summed over ranks' work; for INT4 at 512 or
-more tokens a step is three launches: kernel (a), the float16 weight expansion and the GEMM); the
-per-kernel split comes from a second pass with the two calls timed apart; `e2e`
+the timed steps of qwam_asp_linear, max over ranks, summed over ranks' work; a step is two
+launches, kernel (a) (which for INT4 at 512 or more tokens also writes the float16 weights) and the
+GEMM); the per-kernel split comes from a second pass with the two public calls timed apart (there
+the GEMM call runs the weight expansion as a launch of its own); `e2e`
 repeats the measurement through
 the C ABI with the activations copied from pinned host memory and the output copied back inside
 the timed region; `roofline` describes the dominant kernel; `cpu_baseline` times the CPU oracle
@@ -753,7 +754,7 @@ def run_ours(args):
             "act_path_ms": rr["t_a"], "gemm_ms": rr["t_b"],
             "act_path_gbs_of_fused_bytes": a_fused / (rr["t_a"] * 1e-3) / 1e9,
             "act_path_gbs_of_moved_bytes": a_split / (rr["t_a"] * 1e-3) / 1e9, "peak_gbs": hbm_peak,
-            "launches_per_step": 4}
+            "launches_per_step": 3}
         for s_ in rr["sets"]:
             s_[0].close()
 
@@ -771,9 +772,10 @@ def run_ours(args):
                 "steps": e2e_steps,
                 "pipeline": "copies on their own streams, overlapping the layer of the neighbouring steps"},
         # per qwam_asp_linear call: kernel (a) and the GEMM, the rotation kernel of a rotated layer
-        # with r > 0, and the float16 weight expansion of an INT4 layer of 512 or more tokens
+        # with r > 0, and the float16 weight expansion of an INT4 layer of 512 or more tokens as a
+        # launch of its own when r = 0 (with r > 0 kernel (a) does it)
         "gpu_launches": (2 + (1 if args.rotate and r > 0 else 0)
-                         + (1 if fmt == asp.QWAM_FMT_INT4 and M >= 512 else 0)) * nsteps,
+                         + (1 if fmt == asp.QWAM_FMT_INT4 and M >= 512 and r == 0 else 0)) * nsteps,
         "roofline": roof,
         "layer_roofline_frac": layer_frac,
         "kernels": kern,

@@ -78,8 +78,8 @@ qwam_status qwam_asp_pack_weights(const void* W_bf16, const float* U, int K, int
 
 /* Bytes of the caller-owned activation workspace needed for M tokens.  For INT4 layers of 512 or
  * more tokens it includes a float16 copy of the layer's weights, N_pad (K + r_pad) 2 bytes (N_pad =
- * N rounded up to 256), which qwam_asp_gemm fills once per call and reads from L2 for every row
- * tile.  For 0 < r_pad <= 64 it also includes kernel (a)'s scratch for the partial projections of
+ * N rounded up to 256), which is filled once per call and read from L2 for every row tile: by
+ * kernel (a) inside qwam_asp_linear when r > 0, otherwise by qwam_asp_gemm before its GEMM.  For 0 < r_pad <= 64 it also includes kernel (a)'s scratch for the partial projections of
  * the C CTAs that share a row tile's K (float32, C M_pad r_pad 4 bytes, C <= 8).  Layers of fewer
  * tokens whose 128 x 256 output tiles leave most SMs idle add the split-K GEMM's float32 partial
  * outputs (S M N 4 bytes, S <= 8, at most 8 MiB). */
@@ -121,7 +121,10 @@ qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, 
 qwam_status qwam_asp_gemm(const void* act_ws, int M, qwam_asp_handle h, void* Y, int y_dtype,
                           struct CUstream_st* stream);
 
-/* The whole layer: qwam_asp_quantize_act followed by qwam_asp_gemm on `stream`. */
+/* The whole layer: qwam_asp_quantize_act followed by qwam_asp_gemm on `stream`.  For an INT4 layer
+ * of 512 or more tokens with r > 0, kernel (a) also writes the float16 copy of the weights into
+ * act_ws (while its first pass waits on HBM) and the GEMM uses it, instead of the separate
+ * expansion that qwam_asp_gemm runs when called on its own: the same results, one launch fewer. */
 qwam_status qwam_asp_linear(const void* X_bf16, int M, qwam_asp_handle h, void* Y, int y_dtype,
                             void* act_ws, struct CUstream_st* stream);
 

@@ -55,6 +55,7 @@ struct ActArgs {
   float* part;      // [C, M_pad, RP] float32: the CTAs' partial projections, exchanged through L2
   float* dump;      // optional [M, K]
   int resid_only;   // rotated layer: write the remainder to dump and stop (the rotation kernel quantizes)
+  W16Args w;        // INT4 with r > 0: the call's float16 weights for the GEMM (w.w16 == nullptr: none)
   int* err;
   uint64_t timeout_ns;
 };
@@ -472,6 +473,17 @@ __global__ void __launch_bounds__(kActThreads, 1)
     const int m = m0 + row;
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     bool ok = true;
+
+    if constexpr (!NV && RP > 0) {
+      // The GEMM's float16 weights (expand_w16), a grid-stride share per epilogue thread, while
+      // pass 1 waits on HBM.  The stream's previous GEMM, which read the region, has completed
+      // (the wait at the top), and the GEMM of this call reads it only after this kernel completes.
+      if (a.w.w16 != nullptr) {
+        constexpr int kEpi = kActThreads - 64;
+        expand_w16<8>(a.w, static_cast<int>(blockIdx.y * gridDim.x + blockIdx.x) * kEpi + static_cast<int>(threadIdx.x) - 64,
+                      static_cast<int>(gridDim.x * gridDim.y) * kEpi);
+      }
+    }
 
     if constexpr (RP > 0) {
      if (half == 1) {
@@ -1231,7 +1243,7 @@ __global__ void __launch_bounds__(256) debug_lanes_kernel(const float* __restric
 
 template <int RP, bool NV>
 cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, bool resid_only,
-                      cudaStream_t s) {
+                      cudaStream_t s, bool expand_w16) {
   using Cfg = ActCfg<RP>;
   const ActLayout L = act_layout(h, M);
   ActArgs a;
@@ -1251,6 +1263,8 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
   a.part = reinterpret_cast<float*>(base + L.part_off);
   a.dump = dump;
   a.resid_only = resid_only ? 1 : 0;
+  a.w = w16_args(h, L, ws);
+  if (!expand_w16) a.w.w16 = nullptr;
   a.err = h.err;
   a.timeout_ns = deadline_budget_ns(h);
 
@@ -1281,13 +1295,13 @@ cudaError_t launch_rp(Handle& h, const ActMaps& am, const void* ws, int M, float
 
 template <bool NV>
 cudaError_t launch_fmt(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, bool resid_only,
-                       cudaStream_t s) {
+                       cudaStream_t s, bool expand_w16 = false) {
   switch (h.r_pad) {
-    case 0: return launch_rp<0, NV>(h, am, ws, M, dump, resid_only, s);
-    case 16: return launch_rp<16, NV>(h, am, ws, M, dump, resid_only, s);
-    case 32: return launch_rp<32, NV>(h, am, ws, M, dump, resid_only, s);
-    case 48: return launch_rp<48, NV>(h, am, ws, M, dump, resid_only, s);
-    case 64: return launch_rp<64, NV>(h, am, ws, M, dump, resid_only, s);
+    case 0: return launch_rp<0, NV>(h, am, ws, M, dump, resid_only, s, false);
+    case 16: return launch_rp<16, NV>(h, am, ws, M, dump, resid_only, s, expand_w16);
+    case 32: return launch_rp<32, NV>(h, am, ws, M, dump, resid_only, s, expand_w16);
+    case 48: return launch_rp<48, NV>(h, am, ws, M, dump, resid_only, s, expand_w16);
+    case 64: return launch_rp<64, NV>(h, am, ws, M, dump, resid_only, s, expand_w16);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -1297,7 +1311,7 @@ cudaError_t launch_fmt(Handle& h, const ActMaps& am, const void* ws, int M, floa
 // kernel reads X itself.  `dump` (optional) receives x~_perp.
 template <bool NV>
 cudaError_t launch_rotated(Handle& h, const ActMaps& am, const void* X, const void* ws, int M, float* dump,
-                           cudaStream_t s) {
+                           cudaStream_t s, bool expand_w16) {
   const ActLayout L = act_layout(h, M);
   uint8_t* base = static_cast<uint8_t*>(const_cast<void*>(ws));
   RotArgs a;
@@ -1308,7 +1322,7 @@ cudaError_t launch_rotated(Handle& h, const ActMaps& am, const void* X, const vo
   a.q = quant_out(h, L, base);
   if (h.r == 0) return launch_rotquant_t<__nv_bfloat16, NV>(h, static_cast<const __nv_bfloat16*>(X), a, s);
   float* resid = reinterpret_cast<float*>(base + L.resid_off);
-  cudaError_t e = launch_fmt<NV>(h, am, ws, M, resid, true, s);
+  cudaError_t e = launch_fmt<NV>(h, am, ws, M, resid, true, s, expand_w16);
   if (e != cudaSuccess) return e;
   return launch_rotquant_t<float, NV>(h, resid, a, s);
 }
@@ -1344,16 +1358,25 @@ cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4
   return cudaGetLastError();
 }
 
-cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s) {
+cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s,
+                            bool expand_w16, bool* expanded) {
   const bool nv = h.fmt == kFmtNvfp4;
+  if (expanded) *expanded = false;
   if (h.r_pad > kMaxRank) return nv ? launch_general<true>(h, am.x, ws, M, dump, s) : launch_general<false>(h, am.x, ws, M, dump, s);
   // The small-M kernel for few tokens, and for unrotated r = 0 layers at any token count (with no
   // projection its warp-wide pass beats kernel (a)'s tile pipeline: 15.0 against 19.0 us INT4 and
   // 14.6 against 30.0 us NVFP4 at M = 4096, K = 3072); small_m = 0 always takes kernel (a).
   if (h.K % 256 == 0 && h.small_m > 0 && (M <= h.small_m || (h.r == 0 && !h.rot)))
     return nv ? launch_smallq<true>(h, am.x, ws, M, dump, s) : launch_smallq<false>(h, am.x, ws, M, dump, s);
-  if (h.rot) return nv ? launch_rotated<true>(h, am, am.x, ws, M, dump, s) : launch_rotated<false>(h, am, am.x, ws, M, dump, s);
-  return nv ? launch_fmt<true>(h, am, ws, M, dump, false, s) : launch_fmt<false>(h, am, ws, M, dump, false, s);
+  // kernel (a) with a projection (r > 0), INT4: it can also write the GEMM's float16 weights
+  const bool ex = expand_w16 && !nv && h.r_pad > 0 && act_layout(h, M).w16_off != 0;
+  cudaError_t e;
+  if (h.rot)
+    e = nv ? launch_rotated<true>(h, am, am.x, ws, M, dump, s, false) : launch_rotated<false>(h, am, am.x, ws, M, dump, s, ex);
+  else
+    e = nv ? launch_fmt<true>(h, am, ws, M, dump, false, s) : launch_fmt<false>(h, am, ws, M, dump, false, s, ex);
+  if (e == cudaSuccess && expanded) *expanded = ex;
+  return e;
 }
 
 }  // namespace qwam

@@ -245,8 +245,24 @@ static cudaError_t note_launch(Handle& h, cudaStream_t s) {
   return e;
 }
 
+// expand_w16 / expanded: see launch_actquant.
+static qwam_status quantize_impl(const void* X, int M, qwam_asp_handle hs, void* ws, float* dump,
+                                 struct CUstream_st* stream, bool expand_w16 = false, bool* expanded = nullptr) {
+  if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
+  if (M == 0) return QWAM_OK;
+  if (!X || !ws || !qwam::aligned16(X) || !qwam::aligned16(ws)) return QWAM_ERR_INVALID_ARG;
+  if (dump && !qwam::aligned16(dump)) return QWAM_ERR_INVALID_ARG;
+  Handle& h = hs->h;
+  const qwam::ActMaps* am = qwam::get_act_maps(h, X, ws, M);
+  if (!am) return QWAM_ERR_CUDA;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = qwam::launch_actquant(h, *am, ws, M, dump, s, expand_w16, expanded);
+  if (e == cudaSuccess) e = note_launch(h, s);
+  return from_cuda_status(e);
+}
+
 static qwam_status gemm_impl(const void* act_ws, int M, qwam_asp_handle hs, void* Y, int y_dtype,
-                             struct CUstream_st* stream, bool lean) {
+                             struct CUstream_st* stream, bool lean, bool w16_ready = false) {
   if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
   if (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32) return QWAM_ERR_INVALID_ARG;
   if (M == 0) return QWAM_OK;
@@ -256,7 +272,8 @@ static qwam_status gemm_impl(const void* act_ws, int M, qwam_asp_handle hs, void
   if (!am) return QWAM_ERR_CUDA;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = h.fmt == qwam::kFmtNvfp4 ? qwam::launch_gemm_nvfp4(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s)
-                                           : qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s, lean);
+                                           : qwam::launch_gemm(h, *am, act_ws, M, Y, y_dtype == QWAM_Y_FP32, s, lean,
+                                                               w16_ready);
   if (e == cudaSuccess) e = note_launch(h, s);
   return from_cuda_status(e);
 }
@@ -268,9 +285,12 @@ qwam_status linear_impl(const void* X_bf16, int M, qwam_asp_handle h, void* Y, i
                         struct CUstream_st* stream, bool lean) {
   if (!h || M < 0 || (y_dtype != QWAM_Y_BF16 && y_dtype != QWAM_Y_FP32)) return QWAM_ERR_INVALID_ARG;
   if (M > 0 && (!Y || !qwam::aligned16(Y))) return QWAM_ERR_INVALID_ARG;
-  qwam_status st = qwam_asp_quantize_act(X_bf16, M, h, act_ws, stream);
+  // Through this entry the activation kernel may also write the GEMM's float16 weights (the lean
+  // layout has no region for them), which the GEMM then need not expand itself.
+  bool expanded = false;
+  qwam_status st = quantize_impl(X_bf16, M, h, act_ws, nullptr, stream, !lean, &expanded);
   if (st != QWAM_OK) return st;
-  return gemm_impl(act_ws, M, h, Y, y_dtype, stream, lean);
+  return gemm_impl(act_ws, M, h, Y, y_dtype, stream, lean, expanded);
 }
 }  // namespace qwam
 
@@ -478,21 +498,6 @@ qwam_status qwam_asp_act_layout(qwam_asp_handle hs, int M, size_t* codes_off, si
   if (M_pad) *M_pad = L.M_pad;
   if (r_pad) *r_pad = hs->h.r_pad;
   return QWAM_OK;
-}
-
-static qwam_status quantize_impl(const void* X, int M, qwam_asp_handle hs, void* ws, float* dump,
-                                 struct CUstream_st* stream) {
-  if (!hs || M < 0) return QWAM_ERR_INVALID_ARG;
-  if (M == 0) return QWAM_OK;
-  if (!X || !ws || !qwam::aligned16(X) || !qwam::aligned16(ws)) return QWAM_ERR_INVALID_ARG;
-  if (dump && !qwam::aligned16(dump)) return QWAM_ERR_INVALID_ARG;
-  Handle& h = hs->h;
-  const qwam::ActMaps* am = qwam::get_act_maps(h, X, ws, M);
-  if (!am) return QWAM_ERR_CUDA;
-  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = qwam::launch_actquant(h, *am, ws, M, dump, s);
-  if (e == cudaSuccess) e = note_launch(h, s);
-  return from_cuda_status(e);
 }
 
 qwam_status qwam_asp_quantize_act(const void* X_bf16, int M, qwam_asp_handle h, void* act_ws,

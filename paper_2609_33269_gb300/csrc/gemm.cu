@@ -58,6 +58,7 @@
 //   O  operand stage: A (TMEM, 32 columns) and B (shared memory)  expanders -> MMA   SO slots
 //   R  row-scale slot                          epilogue warps -> expanders, epilogue   2 slots
 //   the accumulator (TMEM columns 0..255)     MMA -> epilogue             1
+#include "dequant.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -122,17 +123,6 @@ __device__ __forceinline__ void mma_f16_tmem_a(uint32_t d_tmem, uint32_t a_tmem,
 
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
-// Packed float16 pairs live in 32-bit registers throughout (low half = the even k).
-__device__ __forceinline__ uint32_t mul_f16x2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-__device__ __forceinline__ uint32_t f32x2_to_f16x2(float lo, float hi) {
-  uint32_t d;
-  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
-  return d;
-}
 __device__ __forceinline__ uint32_t f32x2_to_bf16x2(float lo, float hi) {
   uint32_t d;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
@@ -160,35 +150,6 @@ __device__ __forceinline__ uint4 ld_nc_v4(const void* p) {
 __device__ __forceinline__ float f16_lo(uint32_t u) { return __half2float(__ushort_as_half(static_cast<unsigned short>(u))); }
 __device__ __forceinline__ float f16_hi(uint32_t u) { return __half2float(__ushort_as_half(static_cast<unsigned short>(u >> 16))); }
 
-__device__ __forceinline__ uint32_t sub_f16x2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-
-// The dequantization constants of one scale s (float16, 8 significant bits): the pairs (s, s) and
-// (s/16, s/16), both exact.
-struct DqScale {
-  uint32_t s1, s16;
-};
-__device__ __forceinline__ DqScale dq_scale(float s) {
-  return DqScale{f32x2_to_f16x2(s, s), f32x2_to_f16x2(0.0625f * s, 0.0625f * s)};
-}
-
-// One OB4 word (codes k = 8j..8j+7, nibbles n = c + 8) times the scale -> four float16 pairs in k
-// order.  Under the float16 pattern of 1024 (0x6400, whose unit in the last place is 1) the nibbles
-// of bits 0..3 read as 1024 + n and those of bits 4..7 as 1024 + 16 n; subtracting 1032 or 1152
-// leaves c or 16 c exactly, and multiplying by s or s/16 gives c s exactly (at most 11 significant
-// bits).  Pairs 2 and 3 take the same steps on the word shifted down by 8.  Five integer and eight
-// float16 operations per 8 codes.
-__device__ __forceinline__ void dequant_word(uint32_t w, const DqScale& d, uint32_t* out) {
-  constexpr uint32_t k1032 = 0x64086408u, k1152 = 0x64806480u, kMag = 0x64006400u;
-  const uint32_t w2 = w >> 8;
-  out[0] = mul_f16x2(sub_f16x2((w & 0x000F000Fu) | kMag, k1032), d.s1);
-  out[1] = mul_f16x2(sub_f16x2((w & 0x00F000F0u) | kMag, k1152), d.s16);
-  out[2] = mul_f16x2(sub_f16x2((w2 & 0x000F000Fu) | kMag, k1032), d.s1);
-  out[3] = mul_f16x2(sub_f16x2((w2 & 0x00F000F0u) | kMag, k1152), d.s16);
-}
 
 // s (bfloat16) times 2^e, rounded to float16 (exact while in range), as dequantization constants.
 __device__ __forceinline__ DqScale scale_consts(__nv_bfloat16 s, float mul) {
@@ -210,57 +171,12 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.expect_tx.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
 }
 
-// The weights of one call in float16, [N_pad, K + r_pad] row-major: W16[n, k] = s_w[g, n] 2^e_n c[n, k]
-// for k < K (g = k / G; exact, as in the GEMM's own conversion) and B_hat[n, k - K] 2^e_n after.  A
-// piece is 8 consecutive k of a row; each thread takes 8 pieces a grid stride apart per round,
-// with all their loads issued before the first conversion (bytes in flight without a large grid).
-template <int G>
-__global__ void __launch_bounds__(256) dequant_weights_kernel(const uint32_t* __restrict__ qw,
-                                                                 const __half* __restrict__ swh,
-                                                                 const __half* __restrict__ bhs, int K, int r_pad,
-                                                                 int N_pad, __half* __restrict__ w16) {
+// The weights of one call in float16 (expand_w16), for layers with several row tiles.  Each thread
+// takes eight pieces a grid stride apart per round.
+__global__ void __launch_bounds__(256) dequant_weights_kernel(const W16Args w) {
   pdl_launch_dependents();
   pdl_wait();  // the workspace may still be read by the stream's previous GEMM until then
-  constexpr int P = 8;
-  const int kp = K / 8;  // pieces of the K part per row
-  const int ld = K + r_pad;
-  // (N_pad (K + r_pad) / 8 < 2^31 for every layer the pack accepts: 32-bit piece indices)
-  const int stride = static_cast<int>(gridDim.x * blockDim.x);
-  const int first = static_cast<int>(blockIdx.x * blockDim.x + threadIdx.x);
-  const int total = N_pad * kp;
-  for (int i0 = first; i0 < total; i0 += P * stride) {
-    uint32_t w[P];
-    unsigned short sc[P];
-#pragma unroll
-    for (int u = 0; u < P; ++u) {
-      const int i = i0 + u * stride;
-      w[u] = 0u;
-      sc[u] = 0;
-      if (i < total) {
-        const int n = i / kp, j = i - n * kp;
-        w[u] = qw[i];  // row n, word j: qw is [N_pad, K/8] words
-        sc[u] = __half_as_ushort(swh[static_cast<size_t>(8 * j / G) * N_pad + n]);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < P; ++u) {
-      const int i = i0 + u * stride;
-      if (i < total) {
-        const int n = i / kp, j = i - n * kp;
-        uint32_t v[4];
-        dequant_word(w[u], dq_scale(__half2float(__ushort_as_half(sc[u]))), v);
-        *reinterpret_cast<uint4*>(w16 + static_cast<size_t>(n) * ld + 8 * j) = make_uint4(v[0], v[1], v[2], v[3]);
-      }
-    }
-  }
-  // the branch columns: B_hat 2^e_n copied after the K part of each row
-  const int bp = r_pad / 8;
-  const int total_b = N_pad * bp;
-  for (int i = first; i < total_b; i += stride) {
-    const int n = i / bp, j = i - n * bp;
-    *reinterpret_cast<uint4*>(w16 + static_cast<size_t>(n) * ld + K + 8 * j) =
-        *reinterpret_cast<const uint4*>(bhs + static_cast<size_t>(n) * r_pad + 8 * j);
-  }
+  expand_w16<8>(w, static_cast<int>(blockIdx.x * blockDim.x + threadIdx.x), static_cast<int>(gridDim.x * blockDim.x));
 }
 
 template <int G, bool PREB>
@@ -916,7 +832,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int G, bool PREB>
 cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const void* ws, int M, void* Y, bool y_f32,
-                     cudaStream_t s) {
+                     cudaStream_t s, bool w16_ready) {
   const uint8_t* base = static_cast<const uint8_t*>(ws);
   GemmArgs a;
   a.M = M;
@@ -954,16 +870,13 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
   cfg.stream = s;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (PREB) {
-    __half* w16 = reinterpret_cast<__half*>(const_cast<uint8_t*>(base) + L.w16_off);
+  if (PREB && !w16_ready) {
     const long long pieces = static_cast<long long>(h.N_pad) * ((h.K + h.r_pad) / 8);
     const long long blocks = (pieces + 8 * 256 - 1) / (8 * 256);  // eight pieces a thread
     cfg.gridDim = dim3(static_cast<unsigned>(blocks < 8 * h.num_sms ? blocks : 8 * h.num_sms), 1, 1);
     cfg.blockDim = dim3(256, 1, 1);
     cfg.dynamicSmemBytes = 0;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, dequant_weights_kernel<G>, reinterpret_cast<const uint32_t*>(h.qw),
-                                       static_cast<const __half*>(h.swh), static_cast<const __half*>(h.Bhs), h.K,
-                                       h.r_pad, h.N_pad, w16);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, dequant_weights_kernel, w16_args(h, L, base));
     if (e != cudaSuccess) return e;
   }
   const int ntiles = a.m_tiles * a.n_tiles;
@@ -986,12 +899,27 @@ cudaError_t launch_g(Handle& h, const ActMaps& am, const ActLayout& L, const voi
 
 }  // namespace
 
+W16Args w16_args(const Handle& h, const ActLayout& L, const void* ws) {
+  W16Args w;
+  w.qw = reinterpret_cast<const uint32_t*>(h.qw);
+  w.swh = h.swh;
+  w.bhs = h.Bhs;
+  w.w16 = L.w16_off ? reinterpret_cast<__half*>(static_cast<uint8_t*>(const_cast<void*>(ws)) + L.w16_off) : nullptr;
+  w.K = h.K;
+  w.r_pad = h.r_pad;
+  w.N_pad = h.N_pad;
+  w.gshift = h.G == 32 ? 2 : 3;
+  return w;
+}
+
 cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s,
-                        bool lean) {
+                        bool lean, bool w16_ready) {
   const ActLayout L = act_layout(h, M, lean);
   if (L.w16_off)
-    return h.G == 32 ? launch_g<32, true>(h, am, L, ws, M, Y, y_f32, s) : launch_g<64, true>(h, am, L, ws, M, Y, y_f32, s);
-  return h.G == 32 ? launch_g<32, false>(h, am, L, ws, M, Y, y_f32, s) : launch_g<64, false>(h, am, L, ws, M, Y, y_f32, s);
+    return h.G == 32 ? launch_g<32, true>(h, am, L, ws, M, Y, y_f32, s, w16_ready)
+                     : launch_g<64, true>(h, am, L, ws, M, Y, y_f32, s, w16_ready);
+  return h.G == 32 ? launch_g<32, false>(h, am, L, ws, M, Y, y_f32, s, false)
+                   : launch_g<64, false>(h, am, L, ws, M, Y, y_f32, s, false);
 }
 
 }  // namespace qwam

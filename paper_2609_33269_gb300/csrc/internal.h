@@ -9,6 +9,7 @@
 #include <stdint.h>
 
 #include "../../include/qwam_asp.h"
+#include "dequant.cuh"
 
 namespace qwam {
 
@@ -189,9 +190,16 @@ qwam_status linear_impl(const void* X_bf16, int M, qwam_asp_handle h, void* Y, i
 cudaError_t launch_pack(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
 cudaError_t launch_pack_nvfp4(Handle& h, const __nv_bfloat16* W, const float* U, cudaStream_t s);
 cudaError_t launch_pack_rotated(Handle& h, const __nv_bfloat16* W, const float* s, const float* U, cudaStream_t st);
-cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s);
+// expand_w16: kernel (a) also writes the call's float16 weights into the workspace's expanded-weight
+// region when it is the activation kernel of an INT4 layer whose GEMM takes them (act_layout(h, M)
+// has the region); *expanded tells whether it did, and the GEMM launch then skips its own expansion
+// (w16_ready).
+cudaError_t launch_actquant(Handle& h, const ActMaps& am, const void* ws, int M, float* dump, cudaStream_t s,
+                            bool expand_w16 = false, bool* expanded = nullptr);
 cudaError_t launch_gemm(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s,
-                        bool lean = false);
+                        bool lean = false, bool w16_ready = false);
+// The arguments of expand_w16 for the handle's weights and the expanded-weight region of layout L.
+W16Args w16_args(const Handle& h, const ActLayout& L, const void* ws);
 cudaError_t launch_gemm_nvfp4(Handle& h, const ActMaps& am, const void* ws, int M, void* Y, bool y_f32, cudaStream_t s);
 cudaError_t launch_wait_probe(Handle& h, int timeout_us, cudaStream_t s);
 cudaError_t launch_debug_quantize_lanes(const float* R, int M, int K, bool nvfp4, int G, uint8_t* codes,
