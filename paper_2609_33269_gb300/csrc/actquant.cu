@@ -29,7 +29,9 @@
 // (even chunks, columns 0..31), (odd, 0..31), (even, 32..63), (odd, 32..63) of each 64-column
 // chunk, one thread per row.  A group of 64 columns has its absmax formed from the two halves'
 // partial maxima, swapped through shared memory.  The quantizer's codes come from a fast
-// rounding that an exact remainder test confirms (codes8_fast).
+// rounding that an exact remainder test confirms (codes8_fast).  For an INT4 layer whose GEMM
+// takes float16 weights, the epilogue warps first write those weights (expand_w16) while pass 1
+// waits on HBM, when the launch asks for it (qwam_asp_linear).
 //
 // Also in this file, sharing kernel (a)'s quantizers (the same rounding, bit for bit):
 //   rotquant_kernel  smoothing and block Hadamard rotation of the remainder (Sec. 3 Eq. (pair)),

@@ -50,9 +50,10 @@
 // buffer per group) and scale it by 2^e_m into TMEM, and B_hat 2^e_n comes by TMA straight into the
 // operand stage.  Every wait is bounded.
 // Layers with several 128-row tiles (kPreExpandMinTiles) would convert every weight stage once per
-// row tile; for them `dequant_weights_kernel` writes the float16 weights [s_w 2^e_n c | B_hat 2^e_n]
-// once per call into the workspace (the PREB instantiation), the producer loads each weight stage
-// by TMA straight into the operand ring, and the expanders convert the activations only.
+// row tile; for them the float16 weights [s_w 2^e_n c | B_hat 2^e_n] are written once per call into
+// the workspace (the PREB instantiation): by kernel (a) inside qwam_asp_linear when r > 0, else by
+// `dequant_weights_kernel` just before this kernel.  The producer loads each weight stage by TMA
+// straight into the operand ring, and the expanders convert the activations only.
 // Rings:
 //   P  packed stage: A and B codes, s_x and s_w 2^e_n of its groups   TMA -> expanders   SP slots
 //   O  operand stage: A (TMEM, 32 columns) and B (shared memory)  expanders -> MMA   SO slots
